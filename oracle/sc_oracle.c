@@ -1,0 +1,460 @@
+/*
+ * TEST INFRASTRUCTURE -- fp64 CPU oracle for the verification step of
+ * speculative cascades (Narasimhan et al., "Faster Cascades via Speculative
+ * Decoding").  Only the tests, the smoke check and the benchmark's CPU
+ * baseline leg load this library; the product path never calls it.  It shares
+ * no code, header or constant with the CUDA library.
+ *
+ * What it computes, step by step in the paper's order:
+ *
+ *   GenSpecSample (Algorithm 4) with the SpecCascade target (Algorithm 5):
+ *     for every drafted position j < gamma of sequence b
+ *       q_j = softmax(z^q_j / T), p_j = softmax(z^p_j / T)     (temperature sampling, Sec. 6)
+ *       delta_j = deferral rule of Table 1:
+ *          Chow: max q < 1 - alpha                              (Eq. 2)
+ *          Diff: max q < max p - alpha                          (Eq. 5)
+ *          OPT : max q < max p - alpha * D_TV(p, q)             (Eq. 10)
+ *          with D_TV(p, q) = sum_v max(0, p(v) - q(v))          (Lemma 3)
+ *       pi_j = (1 - delta_j) q_j + delta_j p_j                  (Eq. 6)
+ *       a_j  = [u_{b,j} < min(1, pi_j(x_j) / q_j(x_j))]         (Algorithm 4, Bernoulli draw)
+ *     a_gamma = 0;  j* = min{ j : a_j = 0 }
+ *     next token ~ norm(max(0, pi_{j*} - q_{j*}))  if j* < gamma
+ *                ~ pi_gamma                         otherwise
+ *
+ * Readings where the paper leaves a choice open:
+ *   - the bonus position has no draft row, so pi_gamma := p_gamma (as in
+ *     SpecDecode, Algorithm 1);
+ *   - the Bernoulli draw of position j is "u_{b,j} < rho" with the supplied
+ *     uniform u in [0, 1); a draft whose q(x) <= pi(x) is always accepted, and
+ *     so is a draft with q(x) = 0;
+ *   - the single uniform u_{b,gamma} drives the residual or bonus sample, by
+ *     inverse CDF in ascending vocabulary order: the smallest k whose cumulative
+ *     weight C_k exceeds u * R, R the total weight;
+ *   - the deferral inequalities are strict, as printed in Table 1.
+ *
+ * Decision margins: for every decision that depends on a floating-point
+ * comparison, the oracle records how far it was from flipping (deferral:
+ * |lhs - rhs|; acceptance: |u - pi(x)/q(x)|; sample: distance of u*R to the
+ * nearest cumulative boundary, relative to R).  A sequence whose smallest
+ * margin over positions 0..j* is below 1e-6 is "flagged": an fp32 computation
+ * may legitimately decide it the other way.
+ *
+ * Everything is fp64 with Neumaier-compensated sums; bf16 logits are widened
+ * exactly.  One sequence per OpenMP iteration.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+#define OR_F32 0
+#define OR_BF16 1
+
+#define OR_CHOW 0
+#define OR_DIFF 1
+#define OR_OPT 2
+#define OR_ALWAYS 3 /* delta = 1: standard speculative sampling (Algorithm 1) */
+#define OR_NEVER 4  /* delta = 0: pi = q */
+
+/* per-row record layout, [B][gamma][OR_ROW_FIELDS] */
+#define OR_ROW_MAXQ 0
+#define OR_ROW_MAXP 1
+#define OR_ROW_TV 2
+#define OR_ROW_DELTA 3
+#define OR_ROW_ACCEPT 4
+#define OR_ROW_QX 5
+#define OR_ROW_PIX 6
+#define OR_ROW_MARGIN_DELTA 7
+#define OR_ROW_MARGIN_ACCEPT 8
+#define OR_ROW_FIELDS 9
+
+/* per-sequence record layout, [B][OR_SEQ_FIELDS] */
+#define OR_SEQ_MIN_MARGIN 0
+#define OR_SEQ_SAMPLE_MARGIN 1
+#define OR_SEQ_STATUS 2
+#define OR_SEQ_BONUS_MAXP 3
+#define OR_SEQ_FIELDS 4
+
+/* status bits of a sequence with invalid input */
+#define OR_BAD_TOKEN 1
+#define OR_BAD_LOGIT 2
+#define OR_BAD_UNIFORM 4
+
+/* ------------------------------------------------------------ helpers */
+
+static double logit_at(const void *base, int dtype, size_t i)
+{
+    if (dtype == OR_BF16) {
+        uint32_t w = (uint32_t)((const uint16_t *)base)[i] << 16;
+        float f;
+        memcpy(&f, &w, sizeof f);
+        return (double)f;
+    }
+    return (double)((const float *)base)[i];
+}
+
+/* Neumaier's compensated summation. */
+typedef struct {
+    double s, c;
+} csum;
+
+static void csum_add(csum *k, double x)
+{
+    double t = k->s + x;
+    if (fabs(k->s) >= fabs(x))
+        k->c += (k->s - t) + x;
+    else
+        k->c += (x - t) + k->s;
+    k->s = t;
+}
+
+static double csum_value(const csum *k) { return k->s + k->c; }
+
+/*
+ * Tempered softmax of one row: probs[v] = exp(z_v/T - M) / S, with
+ * M = max_v z_v/T and S = sum_v exp(z_v/T - M).  Returns 0, or -1 when the row
+ * is not a distribution (a NaN or +inf logit, or every logit -inf).
+ */
+static int tempered_softmax(const void *z, int dtype, size_t off, int V, double T,
+                            double *probs)
+{
+    double M = -INFINITY;
+    for (int v = 0; v < V; ++v) {
+        double y = logit_at(z, dtype, off + (size_t)v);
+        if (isnan(y) || y == INFINITY)
+            return -1;
+        y = y / T;
+        probs[v] = y;
+        if (y > M)
+            M = y;
+    }
+    if (!isfinite(M))
+        return -1;
+    csum S = {0.0, 0.0};
+    for (int v = 0; v < V; ++v) {
+        double e = exp(probs[v] - M);
+        probs[v] = e;
+        csum_add(&S, e);
+    }
+    double s = csum_value(&S);
+    for (int v = 0; v < V; ++v)
+        probs[v] /= s;
+    return 0;
+}
+
+static double max_of(const double *x, int V)
+{
+    double m = x[0];
+    for (int v = 1; v < V; ++v)
+        if (x[v] > m)
+            m = x[v];
+    return m;
+}
+
+/* D_TV(p, q) = sum_v max(0, p(v) - q(v))  (Lemma 3; equals 0.5 * ||p - q||_1). */
+static double tv_distance(const double *p, const double *q, int V)
+{
+    csum t = {0.0, 0.0};
+    for (int v = 0; v < V; ++v) {
+        double d = p[v] - q[v];
+        if (d > 0.0)
+            csum_add(&t, d);
+    }
+    return csum_value(&t);
+}
+
+/*
+ * Deferral decision delta(q, p) of Table 1 from the three row scalars.
+ * *margin receives |lhs - rhs| of the strict inequality (infinity for the two
+ * constant rules).
+ */
+static int deferral(int rule, double alpha, double maxq, double maxp, double tv, double *margin)
+{
+    double lhs = maxq, rhs;
+    switch (rule) {
+    case OR_CHOW: rhs = 1.0 - alpha; break;        /* Eq. 2  */
+    case OR_DIFF: rhs = maxp - alpha; break;       /* Eq. 5  */
+    case OR_OPT: rhs = maxp - alpha * tv; break;   /* Eq. 10 */
+    case OR_ALWAYS: *margin = INFINITY; return 1;
+    default: *margin = INFINITY; return 0;
+    }
+    *margin = fabs(lhs - rhs);
+    return lhs < rhs ? 1 : 0;
+}
+
+/*
+ * Inverse-CDF draw from the unnormalised weights w[0..V-1] >= 0 with the
+ * uniform u: the smallest k with C_k = sum_{v<=k} w_v > u * R, R = sum_v w_v.
+ * If rounding leaves u*R at or above the last cumulative value, the largest k
+ * with w_k > 0 is taken.  *margin = min(u R - C_{k-1}, C_k - u R) / R.
+ * Returns -1 when R == 0.
+ */
+static int inverse_cdf(const double *w, int V, double u, double *margin)
+{
+    csum R = {0.0, 0.0};
+    for (int v = 0; v < V; ++v)
+        csum_add(&R, w[v]);
+    double r = csum_value(&R);
+    if (!(r > 0.0)) {
+        *margin = 0.0;
+        return -1;
+    }
+    double t = u * r;
+    csum C = {0.0, 0.0};
+    double prev = 0.0;
+    for (int k = 0; k < V; ++k) {
+        csum_add(&C, w[k]);
+        double c = csum_value(&C);
+        if (c > t) {
+            double m1 = t - prev, m2 = c - t;
+            *margin = (m1 < m2 ? m1 : m2) / r;
+            return k;
+        }
+        prev = c;
+    }
+    *margin = 0.0;
+    for (int k = V - 1; k >= 0; --k)
+        if (w[k] > 0.0)
+            return k;
+    return -1;
+}
+
+/* ------------------------------------------------------------ one sequence */
+
+static void verify_sequence(const void *draft, const void *target, int dtype,
+                            const int32_t *tokens, const float *uniforms, int b, int gamma,
+                            int V, int rule, double alpha, double T, int32_t *num_accepted,
+                            int32_t *next_token, double *row_info, double *seq_info,
+                            double *q, double *p, double *w)
+{
+    const size_t dbase = (size_t)b * gamma * V;
+    const size_t tbase = (size_t)b * (gamma + 1) * V;
+    const int32_t *x = tokens + (size_t)b * gamma;
+    const float *u = uniforms + (size_t)b * (gamma + 1);
+    int status = 0;
+    for (int j = 0; j < gamma; ++j)
+        if (x[j] < 0 || x[j] >= V)
+            status |= OR_BAD_TOKEN;
+    for (int j = 0; j <= gamma; ++j)
+        if (!(u[j] >= 0.0f && u[j] < 1.0f))
+            status |= OR_BAD_UNIFORM;
+
+    int jstar = gamma;          /* a_gamma = 0 */
+    double min_margin = INFINITY;
+    int delta_star = 0;         /* delta at j* */
+    for (int j = 0; j < gamma; ++j) {
+        int okq = tempered_softmax(draft, dtype, dbase + (size_t)j * V, V, T, q);
+        int okp = tempered_softmax(target, dtype, tbase + (size_t)j * V, V, T, p);
+        if (okq || okp) {
+            status |= OR_BAD_LOGIT;
+            continue;
+        }
+        double maxq = max_of(q, V), maxp = max_of(p, V), tv = tv_distance(p, q, V);
+        double m_delta, m_acc = INFINITY;
+        int delta = deferral(rule, alpha, maxq, maxp, tv, &m_delta);
+        int accept = 1;
+        double qx = 0.0, pix = 0.0;
+        if (!(status & OR_BAD_TOKEN)) {
+            qx = q[x[j]];
+            pix = delta ? p[x[j]] : qx; /* pi(x) = (1 - delta) q(x) + delta p(x) */
+            if (delta && qx > pix) {     /* q(x) <= pi(x) (or q(x) = 0) always accepts */
+                double ratio = pix / qx;
+                accept = (double)u[j] < ratio;
+                m_acc = fabs((double)u[j] - ratio);
+            }
+        }
+        if (row_info) {
+            double *r = row_info + ((size_t)b * gamma + j) * OR_ROW_FIELDS;
+            r[OR_ROW_MAXQ] = maxq;
+            r[OR_ROW_MAXP] = maxp;
+            r[OR_ROW_TV] = tv;
+            r[OR_ROW_DELTA] = delta;
+            r[OR_ROW_ACCEPT] = accept;
+            r[OR_ROW_QX] = qx;
+            r[OR_ROW_PIX] = pix;
+            r[OR_ROW_MARGIN_DELTA] = m_delta;
+            r[OR_ROW_MARGIN_ACCEPT] = m_acc;
+        }
+        if (j <= jstar) {
+            if (m_delta < min_margin) min_margin = m_delta;
+            if (m_acc < min_margin) min_margin = m_acc;
+        }
+        if (!accept && j < jstar) {
+            jstar = j;
+            delta_star = delta;
+        }
+    }
+
+    /* The bonus row is always checked, so that its max p is reported. */
+    double bonus_maxp = NAN;
+    if (tempered_softmax(target, dtype, tbase + (size_t)gamma * V, V, T, p) == 0)
+        bonus_maxp = max_of(p, V);
+    else
+        status |= OR_BAD_LOGIT;
+
+    int tok = -1;
+    double m_sample = 0.0;
+    if (status == 0) {
+        if (jstar < gamma) {
+            /* residual norm(max(0, pi - q)) of row j*; pi = p there since a
+               rejection implies delta = 1 */
+            tempered_softmax(draft, dtype, dbase + (size_t)jstar * V, V, T, q);
+            tempered_softmax(target, dtype, tbase + (size_t)jstar * V, V, T, p);
+            for (int v = 0; v < V; ++v) {
+                double pi = delta_star ? p[v] : q[v];
+                double d = pi - q[v];
+                w[v] = d > 0.0 ? d : 0.0;
+            }
+            tok = inverse_cdf(w, V, (double)u[gamma], &m_sample);
+        } else {
+            /* bonus position: sample from pi_gamma = p_gamma (p still holds it) */
+            tok = inverse_cdf(p, V, (double)u[gamma], &m_sample);
+        }
+        if (m_sample < min_margin)
+            min_margin = m_sample;
+        num_accepted[b] = jstar;
+        next_token[b] = tok;
+    } else {
+        num_accepted[b] = 0;
+        next_token[b] = -1;
+        min_margin = 0.0;
+    }
+    if (seq_info) {
+        double *s = seq_info + (size_t)b * OR_SEQ_FIELDS;
+        s[OR_SEQ_MIN_MARGIN] = min_margin;
+        s[OR_SEQ_SAMPLE_MARGIN] = m_sample;
+        s[OR_SEQ_STATUS] = status;
+        s[OR_SEQ_BONUS_MAXP] = bonus_maxp;
+    }
+}
+
+/* ------------------------------------------------------------ exported API */
+
+int oracle_row_fields(void) { return OR_ROW_FIELDS; }
+int oracle_seq_fields(void) { return OR_SEQ_FIELDS; }
+
+int oracle_num_threads(int nthreads)
+{
+#ifdef _OPENMP
+    return nthreads > 0 ? nthreads : omp_get_max_threads();
+#else
+    (void)nthreads;
+    return 1;
+#endif
+}
+
+/*
+ * The whole verification step for B sequences.
+ *   draft    [B][gamma][V]   f32 or bf16 bits (dtype)
+ *   target   [B][gamma+1][V]
+ *   tokens   [B][gamma] int32,   uniforms [B][gamma+1] float32
+ *   num_accepted, next_token   [B] outputs (0 and -1 for an invalid sequence)
+ *   row_info [B][gamma][OR_ROW_FIELDS] or NULL;  seq_info [B][OR_SEQ_FIELDS] or NULL
+ * Returns 0, or -1 on bad arguments.
+ */
+int oracle_verify(const void *draft, const void *target, int dtype, const int32_t *tokens,
+                  const float *uniforms, int B, int gamma, int V, int rule, double alpha,
+                  double T, int32_t *num_accepted, int32_t *next_token, double *row_info,
+                  double *seq_info, int nthreads)
+{
+    if (!draft || !target || !tokens || !uniforms || !num_accepted || !next_token)
+        return -1;
+    if (B < 0 || gamma < 1 || V < 1 || !(T > 0.0) || rule < 0 || rule > 4)
+        return -1;
+    int failed = 0;
+#ifdef _OPENMP
+#pragma omp parallel num_threads(oracle_num_threads(nthreads)) reduction(| : failed)
+#endif
+    {
+        double *q = malloc(sizeof(double) * (size_t)V);
+        double *p = malloc(sizeof(double) * (size_t)V);
+        double *w = malloc(sizeof(double) * (size_t)V);
+        if (!q || !p || !w) {
+            failed = 1;
+        } else {
+#ifdef _OPENMP
+#pragma omp for schedule(dynamic, 1)
+#endif
+            for (int b = 0; b < B; ++b)
+                verify_sequence(draft, target, dtype, tokens, uniforms, b, gamma, V, rule, alpha,
+                                T, num_accepted, next_token, row_info, seq_info, q, p, w);
+        }
+        free(q);
+        free(p);
+        free(w);
+    }
+    return failed ? -1 : 0;
+}
+
+/*
+ * Per-pair statistics (max q, max p, D_TV) for every (b, j < gamma):
+ * outputs [B*gamma].  Returns 0, or -1 (bad arguments or an invalid row).
+ */
+int oracle_row_stats(const void *draft, const void *target, int dtype, int B, int gamma, int V,
+                     double T, double *maxq, double *maxp, double *tv, int nthreads)
+{
+    if (!draft || !target || !maxq || !maxp || !tv || B < 0 || gamma < 1 || V < 1 || !(T > 0.0))
+        return -1;
+    int bad = 0;
+#ifdef _OPENMP
+#pragma omp parallel num_threads(oracle_num_threads(nthreads)) reduction(| : bad)
+#endif
+    {
+        double *q = malloc(sizeof(double) * (size_t)V);
+        double *p = malloc(sizeof(double) * (size_t)V);
+        if (!q || !p) {
+            bad = 1;
+        } else {
+#ifdef _OPENMP
+#pragma omp for schedule(dynamic, 1)
+#endif
+            for (int r = 0; r < B * gamma; ++r) {
+                int b = r / gamma, j = r % gamma;
+                int e1 = tempered_softmax(draft, dtype, (size_t)r * V, V, T, q);
+                int e2 = tempered_softmax(target, dtype, ((size_t)b * (gamma + 1) + j) * V, V, T, p);
+                if (e1 || e2) {
+                    bad = 1;
+                    maxq[r] = maxp[r] = tv[r] = NAN;
+                    continue;
+                }
+                maxq[r] = max_of(q, V);
+                maxp[r] = max_of(p, V);
+                tv[r] = tv_distance(p, q, V);
+            }
+        }
+        free(q);
+        free(p);
+    }
+    return bad ? -1 : 0;
+}
+
+/* Exported building blocks, for pinning each step on its own. */
+int oracle_softmax(const void *z, int dtype, int V, double T, double *probs)
+{
+    if (!z || !probs || V < 1 || !(T > 0.0))
+        return -1;
+    return tempered_softmax(z, dtype, 0, V, T, probs);
+}
+
+double oracle_tv(const double *p, const double *q, int V) { return tv_distance(p, q, V); }
+
+int oracle_deferral(int rule, double alpha, double maxq, double maxp, double tv, double *margin)
+{
+    double m;
+    int d = deferral(rule, alpha, maxq, maxp, tv, &m);
+    if (margin)
+        *margin = m;
+    return d;
+}
+
+int oracle_inverse_cdf(const double *w, int V, double u, double *margin)
+{
+    double m;
+    int k = inverse_cdf(w, V, u, &m);
+    if (margin)
+        *margin = m;
+    return k;
+}

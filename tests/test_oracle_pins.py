@@ -1,0 +1,341 @@
+"""Pins of the fp64 oracle to what the paper and the mathematics fix.
+
+Nothing here compares the oracle with itself: each check is against a library
+routine (scipy softmax, numpy norms), a hand-worked example of the paper's
+definitions (tests/golden/), a closed form (Lemma 3's rejection rate), or the
+correctness property of speculative sampling (the emitted token at every
+reached position is pi-distributed), established by exact enumeration over
+draft tokens and over the 2^24 float32 uniform grid.
+"""
+import itertools
+
+import numpy as np
+import pytest
+
+import oracle
+from helpers import load_golden, np_softmax, rows_workload
+from paper_2405_19261_gb300.workloads import (bf16_bits_to_f32, f32_to_bf16_bits, logits_as_f64,
+                                              synthetic)
+
+RNG = np.random.default_rng(12345)
+
+
+# ----------------------------------------------------------------- step pins
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("T", [1.0, 0.7, 0.1, 2.5])
+@pytest.mark.parametrize("V", [1, 2, 7, 1000, 32128])
+def test_softmax_matches_scipy(dtype, T, V):
+    z = (RNG.standard_normal(V) * 3).astype(np.float32)
+    if dtype == "bf16":
+        z = f32_to_bf16_bits(z)
+    got = oracle.softmax(z, dtype, T)
+    want = np_softmax(logits_as_f64(z, dtype), T)
+    np.testing.assert_allclose(got, want, rtol=1e-12, atol=1e-300)
+    assert abs(got.sum() - 1.0) < 1e-13
+
+
+def test_softmax_extreme_logits():
+    # +-large logits must neither overflow nor lose the head; -inf means probability 0.
+    z = np.array([1e4, -1e4, 9990.0, -np.inf, 0.0], np.float32)
+    got = oracle.softmax(z, "f32", 1.0)
+    want = np_softmax(np.where(np.isinf(z), -1e300, z), 1.0)
+    np.testing.assert_allclose(got, want, rtol=1e-12, atol=1e-300)
+    assert got[3] == 0.0
+    for bad in (np.nan, np.inf):
+        with pytest.raises(ValueError):
+            oracle.softmax(np.array([0.0, bad], np.float32), "f32", 1.0)
+    with pytest.raises(ValueError):
+        oracle.softmax(np.array([-np.inf, -np.inf], np.float32), "f32", 1.0)
+
+
+def test_bf16_decoding_is_exact():
+    vals = np.array([1.0, -2.0, 0.15625, 3.0e38, -1.0e-30, 0.0], np.float32)
+    bits = np.array([0x3F80, 0xC000, 0x3E20], np.uint16)
+    np.testing.assert_array_equal(bf16_bits_to_f32(bits), [1.0, -2.0, 0.15625])
+    rt = bf16_bits_to_f32(f32_to_bf16_bits(vals))
+    assert np.all(np.abs(rt - vals) <= np.abs(vals) * 2.0 ** -8)
+    # the oracle widens the same bits to the same doubles: a one-hot check
+    z = np.array([0x3F80, 0xFF80], np.uint16)  # 1.0, -inf
+    np.testing.assert_array_equal(oracle.softmax(z, "bf16", 1.0), [1.0, 0.0])
+
+
+@pytest.mark.parametrize("V", [1, 3, 50, 32128])
+def test_tv_is_half_l1(V):
+    p = RNG.dirichlet(np.ones(V))
+    q = RNG.dirichlet(np.ones(V) * 0.3)
+    assert abs(oracle.tv(p, q) - 0.5 * np.abs(p - q).sum()) < 1e-13
+    assert oracle.tv(p, p) == 0.0
+    # disjoint supports: TV = 1
+    if V >= 2:
+        a = np.zeros(V); a[0] = 1
+        b = np.zeros(V); b[1] = 1
+        assert oracle.tv(a, b) == 1.0
+
+
+def test_row_stats_match_library_routines():
+    w = synthetic(3, 4, 997, dtype="bf16", kind="zipf", sigma=0.7, seed=3, temperature=0.7)
+    mq, mp, tv = oracle.row_stats(w.draft, w.target, w.dtype, w.B, w.gamma, w.V, w.temperature)
+    d = logits_as_f64(w.draft, "bf16")
+    t = logits_as_f64(w.target, "bf16")[:, :w.gamma]
+    q = np_softmax(d, w.temperature).reshape(-1, w.V)
+    p = np_softmax(t, w.temperature).reshape(-1, w.V)
+    np.testing.assert_allclose(mq, q.max(1), rtol=1e-12)
+    np.testing.assert_allclose(mp, p.max(1), rtol=1e-12)
+    np.testing.assert_allclose(tv, 0.5 * np.abs(p - q).sum(1), rtol=1e-11, atol=1e-15)
+
+
+def test_deferral_table1_golden():
+    g = load_golden("table1_deferral.json")
+    for c in g["cases"]:
+        d, m = oracle.deferral(c["rule"], c["alpha"], c["maxq"], c["maxp"], c["tv"])
+        assert d == c["delta"], c
+
+
+def test_inverse_cdf_brackets_u_times_total():
+    for V in (1, 2, 5, 1000):
+        w = RNG.exponential(size=V)
+        w[RNG.random(V) < 0.3] = 0.0
+        if w.sum() == 0:
+            w[-1] = 1.0
+        c = np.cumsum(w)
+        R = c[-1]
+        for u in np.concatenate([RNG.random(300), [0.0, 1 - 2 ** -24]]):
+            k, margin = oracle.inverse_cdf(w, u)
+            assert 0 <= k < V and w[k] > 0
+            lo = c[k - 1] if k > 0 else 0.0
+            if margin > 1e-12:
+                assert lo <= u * R < c[k], (V, u, k)
+    assert oracle.inverse_cdf(np.zeros(4), 0.5)[0] == -1
+
+
+# ----------------------------------------------------------------- worked examples
+
+def test_worked_examples_golden():
+    g = load_golden("worked_examples.json")
+    for ex in g["examples"]:
+        for c in ex["cases"]:
+            w = rows_workload(ex["q"], ex["p"], ex["tokens"], c["u"], c["rule"], c["alpha"])
+            r = oracle.verify_workload(w)
+            assert (r.num_accepted[0], r.next_token[0]) == (c["num_accepted"], c["next_token"]), \
+                (ex["name"], c)
+            assert not r.flagged[0]
+
+
+# ----------------------------------------------------------------- closed forms
+
+def _random_workload(V, gamma, seed, rule, alpha, T=1.0, B=64):
+    w = synthetic(B, gamma, V, dtype="f32", kind="gauss", sigma=1.5, rule=rule, alpha=alpha,
+                  temperature=T, seed=seed)
+    return w
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_never_defer_accepts_every_draft(seed):
+    w = _random_workload(50, 5, seed, "never", 0.0)
+    r = oracle.verify_workload(w)
+    assert np.all(r.num_accepted == w.gamma)
+    # Chow with alpha = 1 can never defer either (max q < 0 is impossible)
+    r = oracle.verify_workload(w, rule="chow", alpha=1.0)
+    assert np.all(r.num_accepted == w.gamma)
+    assert np.all(r.row("delta") == 0)
+
+
+def test_opt_and_diff_coincide_at_alpha_zero():
+    w = _random_workload(40, 4, 9, "opt", 0.0, B=128)
+    a = oracle.verify_workload(w)
+    b = oracle.verify_workload(w, rule="diff", alpha=0.0)
+    np.testing.assert_array_equal(a.num_accepted, b.num_accepted)
+    np.testing.assert_array_equal(a.next_token, b.next_token)
+
+
+def test_always_defer_is_speculative_decoding():
+    # delta = 1 for every row: pi(x) = p(x) everywhere, acceptance min(1, p/q)
+    w = _random_workload(30, 3, 5, "always", 0.0, B=256)
+    r = oracle.verify_workload(w)
+    assert np.all(r.row("delta") == 1)
+    np.testing.assert_allclose(r.row("pix"), np.take_along_axis(
+        np_softmax(logits_as_f64(w.target, "f32")[:, :w.gamma], 1.0), w.tokens[..., None], -1)[..., 0],
+        rtol=1e-12)
+
+
+def test_forced_rejection_is_rejected():
+    w = synthetic(24, 7, 4096, dtype="bf16", kind="zipf", sigma=(0.2, 1.5), rule="diff", alpha=0.1,
+                  temperature=0.7, seed=11, force_reject_frac=1.0)
+    r = oracle.verify_workload(w)
+    j0 = w.forced
+    assert np.all(j0 >= 0)
+    assert np.all(r.num_accepted <= j0)
+    b = np.arange(w.B)
+    assert np.all(r.row("delta")[b, j0] == 1)
+    assert np.all(r.row("accept")[b, j0] == 0)
+
+
+def test_invalid_inputs_give_defined_outputs():
+    w = _random_workload(20, 3, 1, "opt", 0.2, B=5)
+    w.tokens[1, 2] = 20            # out of range
+    w.draft[2, 1, 4] = np.nan      # NaN logit
+    w.target[3, 3, 0] = np.inf     # +inf in the bonus row
+    w.uniforms[4, 0] = 1.0         # uniform outside [0, 1)
+    r = oracle.verify_workload(w)
+    assert list(r.status) == [0, 1, 2, 2, 4]
+    assert np.all(r.num_accepted[1:] == 0) and np.all(r.next_token[1:] == -1)
+    assert r.next_token[0] >= 0
+
+
+# ----------------------------------------------------------------- exact enumeration
+
+GRID = 1 << 24  # uniforms are k * 2^-24
+
+
+def _batched(w, X, K):
+    """Oracle outputs for sequences that share w's rows, with draft tokens X
+    [N, gamma] and uniform grid indices K [N, gamma+1]."""
+    N = X.shape[0]
+    draft = np.broadcast_to(w.draft[:1], (N,) + w.draft.shape[1:]).copy()
+    target = np.broadcast_to(w.target[:1], (N,) + w.target.shape[1:]).copy()
+    u = (K.astype(np.float64) / GRID).astype(np.float32)
+    r = oracle.verify(draft, target, w.dtype, X.astype(np.int32), u, N, w.gamma, w.V, w.rule,
+                      w.alpha, w.temperature, nthreads=1)
+    return r
+
+
+def _first_true(pred, N):
+    """Smallest k in [0, GRID] with pred(k) true, for monotone predicates (batched)."""
+    lo = np.zeros(N, np.int64)
+    hi = np.full(N, GRID, np.int64)
+    while np.any(lo < hi):
+        mid = (lo + hi) // 2
+        t = pred(np.minimum(mid, GRID - 1)) | (mid >= GRID)
+        hi = np.where(t, mid, hi)
+        lo = np.where(t, lo, mid + 1)
+    return lo
+
+
+def exact_output_law(w):
+    """Exact law of the oracle's output over draft tokens x ~ prod_j q_j and the
+    float32 uniform grid.  Returns per position j: P(reach j), the law of the
+    token emitted at j given reach, and P(reject at j | reach j)."""
+    g, V = w.gamma, w.V
+    X = np.array(list(itertools.product(range(V), repeat=g)), np.int64)
+    N = len(X)
+    q = np_softmax(logits_as_f64(w.draft[0], w.dtype), w.temperature)
+    wx = np.prod(q[np.arange(g)[None, :], X], axis=1)
+
+    # acceptance measure a_j(x): earlier positions accept (u = 0), later ones are irrelevant
+    acc = np.zeros((N, g))
+    for j in range(g):
+        def rejects(k, j=j):
+            K = np.zeros((N, g + 1), np.int64)
+            K[:, j] = k
+            return _batched(w, X, K).num_accepted == j
+        acc[:, j] = _first_true(rejects, N) / GRID
+
+    def token_law(j_reject):
+        # law of the sampled token as a function of u_gamma, given the acceptance pattern
+        NV = N * (V + 1)
+        Xr = np.repeat(X, V + 1, axis=0)
+        vv = np.tile(np.arange(V + 1), N)
+        base = np.zeros((NV, g + 1), np.int64)
+        if j_reject < g:
+            base[:, j_reject] = GRID - 1
+
+        def at_least(k):
+            K = base.copy()
+            K[:, g] = k
+            return _batched(w, Xr, K).next_token >= vv
+        first = _first_true(at_least, NV).reshape(N, V + 1)
+        first[:, V] = GRID
+        first[:, 0] = 0
+        return np.diff(first, axis=1) / GRID  # [N, V]
+
+    laws, reach, reject = [], [], []
+    pre = np.ones(N)
+    for j in range(g + 1):
+        pr = float(np.sum(wx * pre))
+        if j < g:
+            res = token_law(j)
+            emit = acc[:, j:j + 1] * (np.arange(V)[None, :] == X[:, j:j + 1]) + (1 - acc[:, j:j + 1]) * res
+            rj = float(np.sum(wx * pre * (1 - acc[:, j]))) / pr
+        else:
+            emit = token_law(g)
+            rj = 1.0
+        laws.append(np.sum((wx * pre)[:, None] * emit, axis=0) / pr)
+        reach.append(pr)
+        reject.append(rj)
+        if j < g:
+            pre = pre * acc[:, j]
+    return reach, laws, reject
+
+
+ENUM_CASES = [
+    # (V, gamma, rule, alpha, T, seed)
+    (2, 1, "always", 0.0, 1.0, 0),
+    (3, 2, "always", 0.0, 1.0, 1),
+    (4, 3, "always", 0.0, 0.7, 2),
+    (8, 2, "always", 0.0, 1.0, 3),
+    (5, 2, "never", 0.0, 1.0, 4),
+    (4, 3, "chow", 0.45, 1.0, 5),
+    (6, 2, "diff", 0.05, 1.0, 6),
+    (4, 3, "opt", 0.3, 1.0, 7),
+    (7, 2, "opt", 0.8, 0.5, 8),
+    (3, 3, "diff", 0.0, 2.0, 9),
+]
+
+
+@pytest.mark.parametrize("V,gamma,rule,alpha,T,seed", ENUM_CASES)
+def test_enumeration_emitted_token_is_pi_distributed(V, gamma, rule, alpha, T, seed):
+    """Speculative sampling with a general target (Algorithm 4): conditional on
+    reaching position j, the emitted token is pi_j-distributed, with
+    pi_j = (1 - delta_j) q_j + delta_j p_j (Eq. 6) and pi_gamma = p_gamma; the
+    rejection probability at j is delta_j * D_TV(p_j, q_j) (Lemma 3)."""
+    rng = np.random.default_rng(seed)
+    q_log = (rng.standard_normal((gamma, V)) * 1.5).astype(np.float32)
+    p_log = (q_log[np.r_[0:gamma, gamma - 1]] + rng.standard_normal((gamma + 1, V)) * 1.2).astype(np.float32)
+    w = rows_workload(np.exp(q_log), np.exp(p_log), np.zeros(gamma), np.zeros(gamma + 1), rule,
+                      alpha, temperature=T)
+    # rows_workload multiplies the log-probabilities by T, so softmax(z/T) = the rows above
+    info = oracle.verify_workload(w)
+    q = np_softmax(logits_as_f64(w.draft[0], "f32"), T)
+    p = np_softmax(logits_as_f64(w.target[0], "f32"), T)
+    delta = info.row("delta")[0]
+    np.testing.assert_allclose(info.row("maxq")[0], q.max(1), rtol=1e-12)
+    np.testing.assert_allclose(info.row("maxp")[0], p[:gamma].max(1), rtol=1e-12)
+    tv = 0.5 * np.abs(p[:gamma] - q).sum(1)
+    np.testing.assert_allclose(info.row("tv")[0], tv, rtol=1e-11, atol=1e-15)
+    for j in range(gamma):
+        assert delta[j] == oracle.deferral(rule, alpha, q[j].max(), p[j].max(), tv[j])[0]
+    if rule == "always":
+        assert np.all(delta == 1)
+    if rule == "never":
+        assert np.all(delta == 0)
+
+    reach, laws, reject = exact_output_law(w)
+    tol = 4.0 * V / GRID + 1e-9
+    for j in range(gamma):
+        pi = (1 - delta[j]) * q[j] + delta[j] * p[j]
+        np.testing.assert_allclose(laws[j], pi, atol=tol, err_msg=f"position {j}")
+        assert abs(reject[j] - delta[j] * tv[j]) < tol, (j, reject[j], delta[j] * tv[j])
+    np.testing.assert_allclose(laws[gamma], p[gamma], atol=tol, err_msg="bonus position")
+    # P(reach j + 1) = P(reach j) (1 - delta_j TV_j)
+    for j in range(gamma):
+        assert abs(reach[j + 1] - reach[j] * (1 - delta[j] * tv[j])) < tol
+
+
+def test_enumeration_agrees_with_fine_grid_bruteforce():
+    """V = 2, gamma = 1: tally the oracle over an explicit grid of uniforms and
+    draft tokens, independent of the bisection machinery above."""
+    w = rows_workload([[0.7, 0.3]], [[0.2, 0.8], [0.6, 0.4]], [0], [0, 0], "always", 0.0)
+    n = 512
+    grid = (np.arange(n) + 0.5) / n
+    q = np.array([0.7, 0.3])
+    emit0 = np.zeros(2)
+    for x in (0, 1):
+        U = np.array(list(itertools.product(grid, grid)), np.float32)
+        X = np.full((len(U), 1), x, np.int64)
+        draft = np.broadcast_to(w.draft[:1], (len(U), 1, 2)).copy()
+        target = np.broadcast_to(w.target[:1], (len(U), 2, 2)).copy()
+        r = oracle.verify(draft, target, "f32", X.astype(np.int32), U, len(U), 1, 2, "always", 0.0, 1.0)
+        tok0 = np.where(r.num_accepted >= 1, x, r.next_token)
+        emit0 += q[x] * np.bincount(tok0, minlength=2) / len(U)
+    np.testing.assert_allclose(emit0, [0.2, 0.8], atol=2.0 / n)
