@@ -1,0 +1,379 @@
+#!/usr/bin/env python3
+"""Benchmark of the speculative-cascade verification step on GB300.
+
+Default: one GPU, workload cfg3 (B=128, gamma=7, V=256000 bf16 Zipf logits,
+T=0.7, Diff rule alpha=0.1, half the sequences with a planted early
+rejection): 983 MB of logits per step, more than the 129 MB L2, so steps run
+back to back without an L2 flush.  A step is one sc_verify call (one kernel
+launch) over the whole batch.
+
+Prints ONE JSON line (rank 0).  Keys beyond the base contract:
+  roofline      achieved HBM GB/s of the verification kernel (algorithmic bytes
+                / CUDA-event time) against the measured copy bandwidth
+  cpu_baseline  the fp64 oracle timed on this machine's host cores on a bounded
+                sample of the same workload
+  e2e           the same metric through the public API with host buffers, the
+                host->device copy of the inputs and the device->host read of
+                the outputs inside the timed region
+  clocks        nvidia-smi SM clock samples taken while the kernel ran
+
+--impl reference times the oracle (the only other implementation of this
+method here) on the host cores, on bounded samples of the same workload.
+--gpus N under torchrun: every rank verifies its own full batch (weak scaling,
+no collective on the data path); value = all ranks' positions / max time.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "verified positions/s"
+UNIT = "positions/s"
+KERNEL_SRC = os.path.join(ROOT, "paper_2405_19261_gb300", "csrc", "sc_verify.cu")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
+NOMINAL_HBM_GBS = 8000.0
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", type=int, default=3)
+    ap.add_argument("--B", type=int, default=None)
+    ap.add_argument("--gamma", type=int, default=None)
+    ap.add_argument("--rule", default=None)
+    ap.add_argument("--alpha", type=float, default=None)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--min-warmup-s", type=float, default=0.5,
+                    help="keep warming up (untimed) until this long has passed, for clock samples")
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def kernel_sha():
+    with open(KERNEL_SRC, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def stored_traffic(workload_name):
+    """ncu DRAM bytes per launch, if recorded for this exact kernel source."""
+    if not os.path.exists(TRAFFIC_FILE):
+        return None
+    with open(TRAFFIC_FILE) as f:
+        d = json.load(f)
+    e = d.get(workload_name)
+    if not e or e.get("kernel_sha") != kernel_sha():
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+# ------------------------------------------------------------------ clocks
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str, interval_ms: int = 50):
+        self.gpu_id = gpu_id
+        self.interval_ms = interval_ms
+        self.proc = None
+        self.samples = []
+        self.t0 = None
+
+    def start(self):
+        self.tmp = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", self.gpu_id, f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", f"-lms={self.interval_ms}"],
+                stdout=self.tmp, stderr=subprocess.DEVNULL)
+        except (OSError, ValueError):
+            self.proc = None
+        self.t0 = time.time()
+
+    def stop(self):
+        if self.proc is None:
+            return
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.tmp.flush()
+        self.tmp.seek(0)
+        for line in self.tmp.read().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                self.samples.append(dict(sm=float(parts[1]), smax=float(parts[2]),
+                                         active=parts[4], hw=parts[5], hwt=parts[6],
+                                         swt=parts[7], pcap=parts[8]))
+            except ValueError:
+                continue
+        os.unlink(self.tmp.name)
+
+    def summary(self):
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+        reasons = set()
+        for s in self.samples:
+            for key, name in (("hw", "hw_slowdown"), ("hwt", "hw_thermal_slowdown"),
+                              ("swt", "sw_thermal_slowdown"), ("pcap", "sw_power_cap")):
+                if s[key].lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(s["sm"] for s in self.samples),
+                "sm_max_mhz": max(s["smax"] for s in self.samples),
+                "reasons": sorted(reasons), "samples": len(self.samples)}
+
+
+# ------------------------------------------------------------------ oracle timing
+
+def oracle_throughput(w, max_seqs=64, target_s=15.0):
+    """Time the fp64 oracle (all host cores) on a bounded sample of sequences."""
+    import oracle
+    cores = oracle.num_threads(0)
+    n = min(w.B, max(1, min(max_seqs, cores * 4)))
+    sub = w.subset(list(range(n)))
+    t0 = time.perf_counter()
+    oracle.verify_workload(sub, nthreads=cores)
+    dt = time.perf_counter() - t0
+    return dict(value=n * w.gamma / dt, unit=UNIT, cores=cores, kind="oracle",
+                sample=f"first {n} of {w.B} sequences ({n * (2 * w.gamma + 1)} rows of V={w.V}), "
+                       f"{dt:.2f} s wall on {cores} threads"), dt, n
+
+
+# ------------------------------------------------------------------ main
+
+def workload_from(args):
+    from paper_2405_19261_gb300.workloads import CONFIG_TEXT, config
+    kw = {}
+    if args.rule is not None:
+        kw["rule"] = args.rule
+    if args.alpha is not None:
+        kw["alpha"] = args.alpha
+    if args.config == 4:
+        kw["B"] = args.B or 64
+        kw["gamma"] = args.gamma or 4
+    w = config(args.config, **kw)
+    desc = CONFIG_TEXT[args.config]
+    if args.config == 4:
+        desc = f"B={w.B} gamma={w.gamma} V=256000 bf16, zipf sigma=0.7, T=1, {w.rule} a={w.alpha}"
+    return w, f"cfg{args.config}: {desc}"
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    w, desc = workload_from(args)
+    for _ in range(max(0, args.warmup)):
+        pass  # the oracle has no warm state worth warming beyond its first call
+    times, info = [], None
+    for _ in range(args.steps):
+        info, dt, n_seq = oracle_throughput(w, max_seqs=16)
+        times.append(dt)
+    ms = 1e3 * sum(times) / len(times)
+    value = n_seq * w.gamma / (ms / 1e3)
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "config": {"workload": desc, "B": w.B, "gamma": w.gamma, "V": w.V, "rule": w.rule,
+                       "alpha": w.alpha, "temperature": w.temperature,
+                       "note": "each step runs the oracle on a bounded sample of the workload's sequences"},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": info["cores"], "kind": "oracle",
+                             "sample": info["sample"]},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    rank, world, local = dist_env()
+    if world > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local if world > 1 else 0)
+    from paper_2405_19261_gb300 import binding
+
+    w, desc = workload_from(args)
+    d, t, x, u = binding.to_device(w, dev)
+    B, g = w.B, w.gamma
+    ws = binding.new_workspace(B, g, dev)
+    na = torch.empty(B, dtype=torch.int32, device=dev)
+    nt = torch.empty(B, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        binding.sc_verify(d, t, x, u, w.rule, w.alpha, w.temperature, num_accepted=na,
+                          next_token=nt, workspace=ws, stream=stream)
+
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    flush = w.logit_bytes < 3 * l2
+    flush_buf = torch.empty(int(2 * l2), dtype=torch.uint8, device=dev) if flush else None
+
+    props = torch.cuda.get_device_properties(dev)
+    gpu_id = str(getattr(props, "uuid", "")) or str(local)
+    if gpu_id and not gpu_id.startswith("GPU-") and len(gpu_id) > 8:
+        gpu_id = "GPU-" + gpu_id
+    sampler = ClockSampler(gpu_id)
+    sampler.start()
+
+    # warm-up: at least W steps and at least --min-warmup-s seconds
+    t_w = time.perf_counter()
+    nwarm = 0
+    while nwarm < max(3, args.warmup) or time.perf_counter() - t_w < args.min_warmup_s:
+        step()
+        nwarm += 1
+        if nwarm % 50 == 0:
+            torch.cuda.synchronize(dev)
+    torch.cuda.synchronize(dev)
+
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    if flush:
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(args.steps)]
+        for e0, e1 in evs:
+            flush_buf.fill_(1)
+            e0.record(stream)
+            step()
+            e1.record(stream)
+        torch.cuda.synchronize(dev)
+        ms_total = sum(e0.elapsed_time(e1) for e0, e1 in evs)
+    else:
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            step()
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        ms_total = e0.elapsed_time(e1)
+    if world > 1:
+        dist.barrier()
+    sampler.stop()
+    clocks = sampler.summary()
+
+    ms_step = ms_total / args.steps
+    if world > 1:
+        tt = torch.tensor([ms_step], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms_step = float(tt.item())
+    positions = B * g * world
+    value = positions / (ms_step / 1e3)
+
+    # roofline of the verification kernel (the only kernel in a step)
+    peak, peak_kind = measured_peaks()
+    alg = w.algorithmic_bytes()
+    achieved = alg / (ms_step / 1e3) / 1e9
+    traffic = stored_traffic(desc)
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": achieved / peak, "traffic": traffic,
+                "peak_kind": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
+                "frac_of_nominal_8TBs": achieved / NOMINAL_HBM_GBS,
+                "algorithmic_bytes_per_launch": alg}
+
+    # end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        hd = d.cpu().pin_memory()
+        ht = t.cpu().pin_memory()
+        hx = x.cpu().pin_memory()
+        hu = u.cpu().pin_memory()
+        hna = torch.empty(B, dtype=torch.int32).pin_memory()
+        hnt = torch.empty(B, dtype=torch.int32).pin_memory()
+
+        def e2e_step():
+            d.copy_(hd, non_blocking=True)
+            t.copy_(ht, non_blocking=True)
+            x.copy_(hx, non_blocking=True)
+            u.copy_(hu, non_blocking=True)
+            step()
+            hna.copy_(na, non_blocking=True)
+            hnt.copy_(nt, non_blocking=True)
+
+        for _ in range(max(3, args.warmup)):
+            e2e_step()
+        torch.cuda.synchronize(dev)
+        if world > 1:
+            dist.barrier()
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        for _ in range(args.steps):
+            e2e_step()
+        a1.record(stream)
+        torch.cuda.synchronize(dev)
+        e2e_ms = a0.elapsed_time(a1) / args.steps
+        if world > 1:
+            tt = torch.tensor([e2e_ms], device=dev)
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            e2e_ms = float(tt.item())
+        h2d = sum(tn.numel() * tn.element_size() for tn in (hd, ht, hx, hu))
+        e2e = {"value": positions / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": 8 * B, "ms_per_step": e2e_ms}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu, _, _ = oracle_throughput(w)
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+                "config": {"workload": desc, "B": B, "gamma": g, "V": w.V, "logits": w.dtype,
+                           "rule": w.rule, "alpha": w.alpha, "temperature": w.temperature,
+                           "rows_per_s": w.rows * world / (ms_step / 1e3),
+                           "l2": ("L2 flushed (2x L2 write) before every timed step" if flush else
+                                  f"inputs {w.logit_bytes / 1e6:.0f} MB > L2 {l2 / 1e6:.0f} MB, back to back"),
+                           "parallelism": f"{world} independent replica(s), no collective"},
+                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+                "gpu_launches": args.steps, "clocks": clocks}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,143 @@
+/*
+ * sc.h -- C ABI of the GB300 (sm_103a) verification step of speculative
+ * cascades (Narasimhan et al., "Faster Cascades via Speculative Decoding").
+ *
+ * The library implements one call of GenSpecSample's verification phase
+ * (Algorithm 4) with the SpecCascade target of Algorithm 5,
+ *
+ *     pi_j = (1 - delta_j) q_j + delta_j p_j                          (Eq. 6)
+ *
+ * where q_j = softmax(draft_logits[b, j] / T), p_j = softmax(target_logits[b, j] / T)
+ * and delta_j is a deferral rule of Table 1.  Per sequence b it accepts draft
+ * token x_j when u[b, j] < min(1, pi_j(x_j) / q_j(x_j)), finds the first
+ * rejection j*, and draws one new token from norm(max(0, pi_{j*} - q_{j*})),
+ * or from pi_gamma when all gamma drafts are accepted.
+ *
+ * Conventions of every entry point:
+ *  - All array pointers are CUDA device pointers owned by the caller.  The
+ *    library allocates no device memory per call and never synchronises: work
+ *    is queued on `stream` and results are valid once the stream reaches them.
+ *  - Logits are row-major, contiguous, float32 or bf16 (raw 16-bit patterns).
+ *  - Synchronous argument errors return a negative sc_status and queue no work.
+ *    Data errors found on the device never trap: they set bits in the optional
+ *    `device_status` word (see SC_DEV_*) and the affected sequence receives the
+ *    defined outputs num_accepted = 0, next_token = -1.
+ *  - Limits: B, gamma, V >= 1; gamma <= SC_MAX_GAMMA; V <= sc_max_vocab(dtype);
+ *    0 < T < inf; 0 <= alpha <= 1 (the paper sweeps alpha over [0, 1]).
+ */
+#ifndef SC_H_
+#define SC_H_
+
+#include <stddef.h>
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum { SC_F32 = 0, SC_BF16 = 1 } sc_dtype;
+
+/* Deferral rules delta(q, p) of Table 1 (strict inequalities as printed). */
+typedef enum {
+  SC_RULE_CHOW = 0,         /* max_v q(v) < 1 - alpha                           (Eq. 2)  */
+  SC_RULE_DIFF = 1,         /* max_v q(v) < max_v p(v) - alpha                  (Eq. 5)  */
+  SC_RULE_OPT = 2,          /* max_v q(v) < max_v p(v) - alpha * D_TV(p, q)     (Eq. 10) */
+  SC_RULE_ALWAYS_DEFER = 3, /* delta = 1: standard speculative sampling, pi = p (Algorithm 1) */
+  SC_RULE_NEVER_DEFER = 4   /* delta = 0: pi = q, every draft is accepted */
+} sc_rule;
+
+typedef enum {
+  SC_OK = 0,
+  SC_ERR_INVALID_ARG = -1, /* a size, rule, alpha, T or pointer is out of its domain */
+  SC_ERR_CUDA = -2,        /* the launch failed; cudaGetLastError() has the cause */
+  SC_ERR_WORKSPACE = -3,   /* workspace missing or smaller than sc_workspace_bytes() */
+  SC_ERR_UNSUPPORTED = -4  /* V too large for one thread-block cluster per row */
+} sc_status;
+
+/* Bits of the optional device status word (OR-ed in, never cleared). */
+#define SC_DEV_BAD_TOKEN 1u   /* a draft token outside [0, V) */
+#define SC_DEV_BAD_LOGIT 2u   /* a NaN or +inf logit, or a row whose logits are all -inf */
+#define SC_DEV_BAD_UNIFORM 4u /* a uniform outside [0, 1) */
+#define SC_DEV_TIMEOUT 8u     /* an on-chip copy did not complete within the wait limit */
+
+#define SC_MAX_GAMMA 255
+
+/* Per-position diagnostics written by sc_verify_rows, [B][gamma+1][SC_ROW_FIELDS]
+ * float32.  Position gamma (the bonus position) fills only MAXP and CAND. */
+#define SC_ROW_MAXQ 0   /* max_v q_j(v) */
+#define SC_ROW_MAXP 1   /* max_v p_j(v) */
+#define SC_ROW_TV 2     /* D_TV(p_j, q_j) = sum_v max(0, p_j(v) - q_j(v)) (Lemma 3), or -1
+                           when the rule did not need it */
+#define SC_ROW_DELTA 3  /* delta_j in {0, 1} */
+#define SC_ROW_ACCEPT 4 /* a_j in {0, 1} (a_gamma = 0) */
+#define SC_ROW_QX 5     /* q_j(x_j) */
+#define SC_ROW_PIX 6    /* pi_j(x_j) */
+#define SC_ROW_CAND 7   /* token this position would emit if it were j* (-1 if none) */
+#define SC_ROW_FIELDS 8
+
+/* Device workspace needed by sc_verify for B sequences of gamma drafts
+ * (independent of V).  Before its first use the workspace must be zeroed
+ * (sc_workspace_init or a memset); every completed call leaves it zeroed again.
+ * Calls that share one workspace must be ordered on one stream. */
+size_t sc_workspace_bytes(int B, int gamma, int V);
+
+/* Zero a workspace on `stream` (a cudaMemsetAsync). */
+int sc_workspace_init(void *workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/* Largest supported vocabulary for a logit type. */
+int sc_max_vocab(sc_dtype dtype);
+
+/*
+ * sc_verify -- one verification step (Algorithm 4 with Algorithm 5's target).
+ *   draft_logits   [B][gamma][V]     q logits for the gamma drafted positions
+ *   target_logits  [B][gamma+1][V]   p logits for positions 0..gamma
+ *   draft_tokens   [B][gamma] int32  x_j, sampled by the drafter from q_j
+ *   uniforms       [B][gamma+1] f32  u[b][j < gamma] is the Bernoulli draw of
+ *                                    position j; u[b][gamma] is the single draw
+ *                                    for the residual or bonus sample
+ *   rule, alpha    deferral rule of Table 1 and its cost parameter
+ *   temperature    T > 0; both q and p are softmax(logits / T)
+ *   num_accepted   [B] int32 out: j* in [0, gamma]
+ *   next_token     [B] int32 out: the token emitted at position j*.  The
+ *                  emitted tokens of sequence b are draft_tokens[b][0 .. j*-1]
+ *                  followed by next_token[b].
+ *   workspace      sc_workspace_bytes(B, gamma, V) bytes, zeroed before first use
+ *   device_status  optional int32 word receiving SC_DEV_* bits (may be NULL)
+ * The residual and bonus draws are inverse-CDF samples in ascending vocabulary
+ * order; the bonus position samples pi_gamma := p_gamma (no draft row exists there).
+ */
+int sc_verify(const void *draft_logits, const void *target_logits, sc_dtype dtype,
+              const int32_t *draft_tokens, const float *uniforms, int B, int gamma, int V,
+              sc_rule rule, float alpha, float temperature, int32_t *num_accepted,
+              int32_t *next_token, void *workspace, size_t workspace_bytes,
+              int32_t *device_status, cudaStream_t stream);
+
+/* sc_verify that also writes the per-position diagnostics row_info
+ * [B][gamma+1][SC_ROW_FIELDS] (row_info may be NULL, which equals sc_verify). */
+int sc_verify_rows(const void *draft_logits, const void *target_logits, sc_dtype dtype,
+                   const int32_t *draft_tokens, const float *uniforms, int B, int gamma, int V,
+                   sc_rule rule, float alpha, float temperature, int32_t *num_accepted,
+                   int32_t *next_token, void *workspace, size_t workspace_bytes,
+                   int32_t *device_status, float *row_info, cudaStream_t stream);
+
+/*
+ * sc_row_stats -- the per-position quantities the deferral rules of Table 1
+ * read: max_v q_j(v), max_v p_j(v) and D_TV(p_j, q_j) (Lemma 3), for every pair
+ * (b, j < gamma).  Outputs are [B*gamma] float32 each, index b*gamma + j.  A
+ * row that is not a distribution (NaN / +inf logit, or all -inf) yields NaN.
+ * target_logits has the same [B][gamma+1][V] layout as for sc_verify (the
+ * bonus row is not read).
+ */
+int sc_row_stats(const void *draft_logits, const void *target_logits, sc_dtype dtype, int B,
+                 int gamma, int V, float temperature, float *max_q, float *max_p, float *tv,
+                 cudaStream_t stream);
+
+/* Static description of an sc_status code. */
+const char *sc_status_string(int code);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SC_H_ */

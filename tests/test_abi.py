@@ -1,0 +1,58 @@
+"""The C-ABI library loads and exports every entry point include/sc.h declares,
+and its host-only entry points behave (no GPU needed)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "sc.h")
+
+
+@pytest.fixture(scope="module")
+def so():
+    import __graft_entry__ as g
+    if not os.path.exists(g.LIB) or os.path.getmtime(g.LIB) < os.path.getmtime(g.CSRC):
+        g.build_library()
+    return ctypes.CDLL(g.LIB)
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    names = re.findall(r"\b(sc_[a-z_]+)\s*\(", text)
+    return sorted(set(names))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for n in ("sc_verify", "sc_row_stats", "sc_workspace_bytes", "sc_status_string"):
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(so):
+    for n in declared_functions():
+        assert hasattr(so, n), n
+
+
+def test_host_only_entry_points(so):
+    so.sc_workspace_bytes.restype = ctypes.c_size_t
+    so.sc_workspace_bytes.argtypes = [ctypes.c_int] * 3
+    assert so.sc_workspace_bytes(0, 5, 10) == 0
+    assert so.sc_workspace_bytes(8, 5, 256000) >= 8 * 4 + 2 * 8 * 6 * 4
+    so.sc_status_string.restype = ctypes.c_char_p
+    assert so.sc_status_string(0) == b"ok"
+    assert so.sc_status_string(-1) == b"invalid argument"
+    so.sc_max_vocab.argtypes = [ctypes.c_int]
+    assert so.sc_max_vocab(1) >= 256000   # bf16 Gemma vocabulary
+    assert so.sc_max_vocab(0) >= 256000   # f32 too
+
+
+def test_null_pointers_are_rejected_without_a_gpu(so):
+    P, I, F, S = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_size_t
+    so.sc_verify.argtypes = [P, P, I, P, P, I, I, I, I, F, F, P, P, P, S, P, P]
+    rc = so.sc_verify(None, None, 1, None, None, 1, 1, 8, 0, 0.5, 1.0, None, None, None, 0, None, None)
+    assert rc == -1
+    rc = so.sc_verify(None, None, 1, None, None, 0, 1, 8, 0, 0.5, 1.0, None, None, None, 0, None, None)
+    assert rc == -1

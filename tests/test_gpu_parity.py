@@ -1,0 +1,242 @@
+"""Parity of the CUDA verification step with the fp64 oracle (GPU only).
+
+Bar: num_accepted and next_token bit-exact on every sequence the oracle does
+not flag (a decision closer than 1e-6 to flipping); max q, max p, TV, q(x) and
+pi(x) within 1e-5 absolute; deferral and acceptance decisions equal wherever
+their own margin is at least 1e-6.
+"""
+import numpy as np
+import pytest
+
+import oracle
+from helpers import load_golden, rows_workload
+from paper_2405_19261_gb300.workloads import config, synthetic
+
+pytestmark = pytest.mark.gpu
+
+TOL = 1e-5
+
+
+@pytest.fixture(scope="module")
+def sc():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2405_19261_gb300 import binding
+    binding.lib()
+    return binding
+
+
+def run_gpu(sc, w, rows=True, rule=None, alpha=None):
+    import torch
+    d, t, x, u = sc.to_device(w)
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    ri = torch.full((w.B, w.gamma + 1, sc.ROW_FIELDS), -7.0, dtype=torch.float32, device="cuda") if rows else None
+    na, nt = sc.sc_verify(d, t, x, u, w.rule if rule is None else rule,
+                          w.alpha if alpha is None else alpha, w.temperature,
+                          status=status, row_info=ri)
+    torch.cuda.synchronize()
+    return (na.cpu().numpy(), nt.cpu().numpy(), None if ri is None else ri.cpu().numpy(),
+            int(status.item()))
+
+
+def assert_parity(w, gpu, ref, check_rows=True):
+    na, nt, ri, status = gpu
+    assert status == 0
+    ok = ~ref.flagged
+    bad = np.nonzero(ok & ((na != ref.num_accepted) | (nt != ref.next_token)))[0]
+    assert len(bad) == 0, (f"{w.name}: {len(bad)} unflagged mismatches, first b={bad[:5]}, "
+                           f"gpu={na[bad[:5]]},{nt[bad[:5]]} oracle={ref.num_accepted[bad[:5]]},{ref.next_token[bad[:5]]}")
+    if ri is None or not check_rows:
+        return
+    g = w.gamma
+    R = ri[:, :g]
+    np.testing.assert_allclose(R[..., 0], ref.row("maxq"), atol=TOL)
+    np.testing.assert_allclose(R[..., 1], ref.row("maxp"), atol=TOL)
+    np.testing.assert_allclose(ri[:, g, 1], ref.seqs[:, oracle.SEQ["bonus_maxp"]], atol=TOL)
+    tv = R[..., 2]
+    have = tv >= 0
+    np.testing.assert_allclose(tv[have], ref.row("tv")[have], atol=TOL)
+    sure_d = ref.row("margin_delta") >= oracle.FLAG_MARGIN
+    np.testing.assert_array_equal(R[..., 3][sure_d], ref.row("delta")[sure_d])
+    same_d = R[..., 3] == ref.row("delta")
+    sure_a = sure_d & (ref.row("margin_accept") >= oracle.FLAG_MARGIN)
+    np.testing.assert_array_equal(R[..., 4][sure_a], ref.row("accept")[sure_a])
+    np.testing.assert_allclose(R[..., 5], ref.row("qx"), atol=TOL)
+    np.testing.assert_allclose(R[..., 6][same_d], ref.row("pix")[same_d], atol=TOL)
+
+
+# ----------------------------------------------------------------- hand-worked goldens
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_worked_examples(sc, dtype):
+    g = load_golden("worked_examples.json")
+    for ex in g["examples"]:
+        for c in ex["cases"]:
+            w = rows_workload(ex["q"], ex["p"], ex["tokens"], c["u"], c["rule"], c["alpha"], dtype=dtype)
+            na, nt, _, status = run_gpu(sc, w)
+            assert status == 0
+            assert (na[0], nt[0]) == (c["num_accepted"], c["next_token"]), (ex["name"], c)
+
+
+# ----------------------------------------------------------------- named configs
+
+def test_cfg0(sc):
+    w = config(0)
+    assert_parity(w, run_gpu(sc, w), oracle.verify_workload(w))
+
+
+@pytest.mark.parametrize("rule", ["chow", "diff", "opt"])
+@pytest.mark.parametrize("alpha", [0.0, 0.1, 0.3, 0.5, 1.0])
+def test_cfg1(sc, rule, alpha):
+    w = config(1, rule=rule, alpha=alpha)
+    assert_parity(w, run_gpu(sc, w), oracle.verify_workload(w))
+
+
+@pytest.mark.parametrize("seed", range(6))
+@pytest.mark.parametrize("rule", ["always", "opt", "diff"])
+def test_many_seeds_t5_shape(sc, seed, rule):
+    w = synthetic(16, 5, 32128, dtype="bf16", kind="zipf", sigma=0.7, rule=rule,
+                  alpha={"always": 0.0, "opt": 0.3, "diff": 0.05}[rule], temperature=1.0,
+                  seed=1000 + seed)
+    assert_parity(w, run_gpu(sc, w), oracle.verify_workload(w))
+
+
+def _sampled_parity(sc, w, nseq=12, seed=0):
+    gpu = run_gpu(sc, w)
+    pick = np.sort(np.random.default_rng(seed).choice(w.B, size=min(nseq, w.B), replace=False))
+    ref = oracle.verify_workload(w.subset(pick))
+    na, nt, ri, status = gpu
+    assert_parity(w.subset(pick), (na[pick], nt[pick], ri[pick], status), ref)
+    return gpu
+
+
+@pytest.mark.slow
+def test_cfg2_full_size_sampled(sc):
+    _sampled_parity(sc, config(2), nseq=12)
+
+
+@pytest.mark.slow
+def test_cfg3_full_size_sampled(sc):
+    w = config(3)
+    na, nt, ri, status = _sampled_parity(sc, w, nseq=12)
+    # planted rejections: every forced sequence stops at or before its forced position
+    f = w.forced >= 0
+    assert np.all(na[f] <= w.forced[f])
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("rule", ["chow", "diff", "opt"])
+def test_cfg4_smallest_point_sampled(sc, rule):
+    _sampled_parity(sc, config(4, B=64, gamma=4, rule=rule), nseq=6)
+
+
+# ----------------------------------------------------------------- row statistics
+
+@pytest.mark.parametrize("case", ["cfg1", "zipf-256k", "f32-odd"])
+def test_row_stats(sc, case):
+    import torch
+    if case == "cfg1":
+        w = config(1)
+    elif case == "zipf-256k":
+        w = synthetic(3, 4, 256000, dtype="bf16", kind="zipf", sigma=0.7, seed=5, temperature=0.7)
+    else:
+        w = synthetic(4, 3, 10007, dtype="f32", kind="gauss", sigma=1.0, seed=6, temperature=1.3)
+    d, t, _, _ = sc.to_device(w)
+    mq, mp, tv = sc.sc_row_stats(d, t, w.temperature)
+    torch.cuda.synchronize()
+    rq, rp, rt = oracle.row_stats(w.draft, w.target, w.dtype, w.B, w.gamma, w.V, w.temperature)
+    np.testing.assert_allclose(mq.cpu().numpy(), rq, atol=TOL)
+    np.testing.assert_allclose(mp.cpu().numpy(), rp, atol=TOL)
+    np.testing.assert_allclose(tv.cpu().numpy(), rt, atol=TOL)
+
+
+# ----------------------------------------------------------------- edge cases
+
+@pytest.mark.parametrize("V", [1, 2, 3, 7, 8, 9, 31, 4095, 4096, 4097, 8193, 32127])
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_ragged_vocab(sc, V, dtype):
+    w = synthetic(5, 3, V, dtype=dtype, kind="gauss", sigma=1.0, rule="always", alpha=0.0,
+                  seed=V, temperature=0.9)
+    assert_parity(w, run_gpu(sc, w), oracle.verify_workload(w))
+    w2 = w.with_rule("opt", 0.25)
+    assert_parity(w2, run_gpu(sc, w2), oracle.verify_workload(w2))
+
+
+@pytest.mark.parametrize("gamma", [1, 2, 8, 31, 40])
+def test_gamma_range(sc, gamma):
+    w = synthetic(3, gamma, 1000, dtype="bf16", kind="zipf", sigma=1.0, rule="always", alpha=0.0, seed=gamma)
+    assert_parity(w, run_gpu(sc, w), oracle.verify_workload(w))
+
+
+def test_degenerate_rows(sc):
+    B, g, V = 6, 3, 777
+    w = synthetic(B, g, V, dtype="f32", kind="gauss", sigma=1.0, rule="always", alpha=0.0, seed=77)
+    w.draft[0] = 0.0                 # all-equal logits: q uniform
+    w.target[0] = 0.0
+    w.draft[1, :, 5] = 80.0          # one huge logit: q one-hot-like
+    w.target[1, :, 9] = 80.0
+    w.draft[2] *= 1e4                # +-large logits, no overflow
+    w.target[2] *= 1e4
+    w.draft[3, :, :100] = -np.inf    # masked tokens have probability 0
+    w.target[3, :, 50:150] = -np.inf
+    w.tokens[3] = 200
+    w.draft[4, 0, w.tokens[4, 0]] = -200.0   # the draft token's q underflows
+    w.draft[5] = w.target[5, :g]     # identical rows: TV = 0, always accepted
+    w.uniforms[5] = 0.999
+    ref = oracle.verify_workload(w)
+    gpu = run_gpu(sc, w)
+    assert_parity(w, gpu, ref)
+    assert gpu[0][5] == g
+
+
+def test_invalid_inputs_flagged_on_device(sc):
+    w = synthetic(5, 3, 300, dtype="f32", kind="gauss", sigma=1.0, rule="opt", alpha=0.2, seed=8)
+    w.tokens[1, 2] = 300
+    w.draft[2, 1, 4] = np.nan
+    w.target[3, 3, 0] = np.inf
+    w.uniforms[4, 0] = 1.0
+    na, nt, _, status = run_gpu(sc, w)
+    assert status == 1 | 2 | 4
+    assert np.all(na[1:] == 0) and np.all(nt[1:] == -1)
+    ref = oracle.verify_workload(w)
+    assert (na[0], nt[0]) == (ref.num_accepted[0], ref.next_token[0]) or ref.flagged[0]
+
+
+def test_host_argument_errors(sc):
+    import torch
+    w = synthetic(2, 2, 64, dtype="f32", kind="gauss", seed=1)
+    d, t, x, u = sc.to_device(w)
+    with pytest.raises(sc.SCError):
+        sc.sc_verify(d, t, x, u, "opt", 1.5, 1.0)       # alpha outside [0, 1]
+    with pytest.raises(sc.SCError):
+        sc.sc_verify(d, t, x, u, "opt", 0.2, 0.0)       # T = 0
+    with pytest.raises(sc.SCError):
+        sc.sc_verify(d, t, x, u, 9, 0.2, 1.0)           # unknown rule
+    with pytest.raises(sc.SCError):
+        sc.sc_verify(d, t, x, u, "opt", 0.2, 1.0, workspace=torch.zeros(4, dtype=torch.uint8, device="cuda"))
+    with pytest.raises(TypeError):
+        sc.sc_verify(d.cpu(), t, x, u, "opt", 0.2, 1.0)
+    with pytest.raises(ValueError):
+        sc.sc_verify(d, t[:, :2], x, u, "opt", 0.2, 1.0)
+
+
+def test_repeatable_and_workspace_reuse(sc):
+    import torch
+    w1 = config(1, rule="opt", alpha=0.3)
+    w2 = synthetic(8, 5, 32128, dtype="bf16", kind="gauss", sigma=0.5, rule="opt", alpha=0.3, seed=99)
+    ws = sc.new_workspace(8, 5)
+    outs = []
+    for w in (w1, w2, w1):
+        d, t, x, u = sc.to_device(w)
+        ri = torch.zeros((w.B, w.gamma + 1, 8), device="cuda")
+        na, nt = sc.sc_verify(d, t, x, u, w.rule, w.alpha, w.temperature, workspace=ws, row_info=ri)
+        torch.cuda.synchronize()
+        outs.append((na.cpu().numpy(), nt.cpu().numpy(), ri.cpu().numpy()))
+    for a, b in zip(outs[0], outs[2]):
+        np.testing.assert_array_equal(a, b)   # bitwise identical on a re-run
+    assert torch.count_nonzero(ws[:4 * 8]).item() == 0   # tickets are left zeroed
+    ref2 = oracle.verify_workload(w2)
+    ok = ~ref2.flagged
+    np.testing.assert_array_equal(outs[1][0][ok], ref2.num_accepted[ok])
+    np.testing.assert_array_equal(outs[1][1][ok], ref2.next_token[ok])
