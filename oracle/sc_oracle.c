@@ -118,8 +118,8 @@ static double csum_value(const csum *k) { return k->s + k->c; }
  * M = max_v z_v/T and S = sum_v exp(z_v/T - M).  Returns 0, or -1 when the row
  * is not a distribution (a NaN or +inf logit, or every logit -inf).
  */
-static int tempered_softmax(const void *z, int dtype, size_t off, int V, double T,
-                            double *probs)
+static int tempered_softmax_ln(const void *z, int dtype, size_t off, int V, double T,
+                               double *probs, double *M_out, double *lnS_out)
 {
     double M = -INFINITY;
     for (int v = 0; v < V; ++v) {
@@ -142,7 +142,24 @@ static int tempered_softmax(const void *z, int dtype, size_t off, int V, double 
     double s = csum_value(&S);
     for (int v = 0; v < V; ++v)
         probs[v] /= s;
+    if (M_out)
+        *M_out = M;
+    if (lnS_out)
+        *lnS_out = log(s);
     return 0;
+}
+
+static int tempered_softmax(const void *z, int dtype, size_t off, int V, double T,
+                            double *probs)
+{
+    return tempered_softmax_ln(z, dtype, off, V, T, probs, NULL, NULL);
+}
+
+/* ln of the tempered probability of token x: z_x/T - M - ln S (no underflow). */
+static double log_prob(const void *z, int dtype, size_t off, int x, double T, double M,
+                       double lnS)
+{
+    return logit_at(z, dtype, off + (size_t)x) / T - M - lnS;
 }
 
 static double max_of(const double *x, int V)
@@ -246,8 +263,9 @@ static void verify_sequence(const void *draft, const void *target, int dtype,
     double min_margin = INFINITY;
     int delta_star = 0;         /* delta at j* */
     for (int j = 0; j < gamma; ++j) {
-        int okq = tempered_softmax(draft, dtype, dbase + (size_t)j * V, V, T, q);
-        int okp = tempered_softmax(target, dtype, tbase + (size_t)j * V, V, T, p);
+        double Mq, lnSq, Mp, lnSp;
+        int okq = tempered_softmax_ln(draft, dtype, dbase + (size_t)j * V, V, T, q, &Mq, &lnSq);
+        int okp = tempered_softmax_ln(target, dtype, tbase + (size_t)j * V, V, T, p, &Mp, &lnSp);
         if (okq || okp) {
             status |= OR_BAD_LOGIT;
             continue;
@@ -260,10 +278,17 @@ static void verify_sequence(const void *draft, const void *target, int dtype,
         if (!(status & OR_BAD_TOKEN)) {
             qx = q[x[j]];
             pix = delta ? p[x[j]] : qx; /* pi(x) = (1 - delta) q(x) + delta p(x) */
-            if (delta && qx > pix) {     /* q(x) <= pi(x) (or q(x) = 0) always accepts */
-                double ratio = pix / qx;
-                accept = (double)u[j] < ratio;
-                m_acc = fabs((double)u[j] - ratio);
+            if (delta) {
+                /* pi(x)/q(x) = p(x)/q(x), formed from log-probabilities so that it
+                   stays exact when both underflow; q(x) <= pi(x) always accepts
+                   (q(x) = 0 only for a -inf logit) */
+                double lq = log_prob(draft, dtype, dbase + (size_t)j * V, x[j], T, Mq, lnSq);
+                double lp = log_prob(target, dtype, tbase + (size_t)j * V, x[j], T, Mp, lnSp);
+                if (lq > lp) {
+                    double ratio = exp(lp - lq);
+                    accept = (double)u[j] < ratio;
+                    m_acc = fabs((double)u[j] - ratio);
+                }
             }
         }
         if (row_info) {
