@@ -66,6 +66,7 @@ struct Params {
   float alpha;
   float temperature;
   float k;        // log2(e) / T
+  double inv_t;   // 1 / T
   int L;          // slice length per CTA (multiple of 8 elements)
   int cluster;    // CTAs per unit
   int bulk;       // 1: TMA bulk copies, 0: per-thread loads (unaligned rows)
@@ -173,7 +174,7 @@ struct Elt<float> {
 struct __align__(16) Shared {
   uint64_t bar[kMaxChunks];
   float4 part_ms;        // this CTA's (m_q, s_q, m_p, s_p), read by the cluster
-  float part_tv;         // this CTA's sum of min(p, q)
+  float part_tv;         // this CTA's sum of 2^min(a, b + c)
   float part_r;          // this CTA's total sampling weight
   int cand;              // sampled token (written remotely into rank 0)
   int timeout;
@@ -181,12 +182,12 @@ struct __align__(16) Shared {
   float wtot[kNW + 1];
   // row statistics, identical in every CTA of the cluster
   float Mq, Sq, Mp, Sp;
-  float lq, lp;          // log2 S
+  float c;               // log2(S_q / S_p)
   float tv;
   int err, delta, need_tv, need_sample, accept;
   float qx, pix;
-  float rprefix;         // cluster prefix of the sampling weights before this CTA
-  double t_local;        // u * R - rprefix
+  double t_local;        // u * R minus the weight of the CTAs before the crossing one
+  float ug;              // u[b][gamma], the residual / bonus draw
   int sample_here;       // 1: crossing inside this CTA, 2: take its last positive weight
 };
 
@@ -226,30 +227,38 @@ __device__ __forceinline__ void online_chunk(const E *row, int vbeg, int vend, f
   s = acc;
 }
 
-// Sampling weight of one element: residual max(0, p - q) of a pair, or the
-// unnormalised p of the bonus row.
+// Row scalars in registers for the shared-memory passes.  With
+// a_v = (y^q_v - M_q) k and b_v = (y^p_v - M_p) k (k = log2(e)/T):
+//   q_v = 2^{a_v} / S_q,   p_v = 2^{b_v} / S_p = 2^{b_v + c} / S_q,   c = log2(S_q / S_p).
+struct RowScalars {
+  float Mq, Mp, k, c;
+};
+
+// Sampling weight of one element, up to the common factor 1/S_q:
+// residual max(0, p - q) of a pair, or p of the bonus row.
 template <bool kPair>
-__device__ __forceinline__ float weight(float yq, float yp, const Shared &sh, float k,
-                                        float inv_sq, float inv_sp) {
-  const float ep = ex2((yp - sh.Mp) * k);
+__device__ __forceinline__ float weight(float yq, float yp, const RowScalars &r) {
   if constexpr (kPair) {
-    const float eq = ex2((yq - sh.Mq) * k);
-    return fmaxf(0.0f, ep * inv_sp - eq * inv_sq);
+    const float a = (yq - r.Mq) * r.k;
+    const float b = fmaf(yp - r.Mp, r.k, r.c);
+    return fmaxf(0.0f, ex2(b) - ex2(a));
   } else {
-    return ep;
+    return ex2((yp - r.Mp) * r.k);
   }
 }
 
-// Inverse-CDF draw over the cluster's slices (see the file comment).  Every
-// thread of every CTA calls it; returns nothing, the chosen token lands in
-// rank 0's Shared::cand.
+// f32 a, f64 t: (a > t) == (a > round_down_to_f32(t)).
+__device__ __forceinline__ float f32_floor(double t) { return __double2float_rd(t); }
+
+// Inverse-CDF draw over the cluster's slices.  Every thread of every CTA calls
+// it; the chosen token is written into rank 0's Shared::cand, visible there
+// after the caller's next cluster barrier.
 template <typename E, bool kPair>
-__device__ void sample_unit(const E *sq, const E *sp, int nv, int v0, Shared &sh, float k,
-                            double u, cg::cluster_group &cluster, int rank, int C) {
+__device__ void sample_unit(const E *sq, const E *sp, int nv, int v0, Shared &sh,
+                            const RowScalars &rs, float u, cg::cluster_group &cluster, int rank,
+                            int C) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const float inv_sq = kPair ? 1.0f / sh.Sq : 0.0f;
-  const float inv_sp = kPair ? 1.0f / sh.Sp : 0.0f;
-  // contiguous ownership, odd stride: conflict-free 16-byte shared loads
+  // contiguous ownership with an odd stride: conflict-free 16-byte shared loads
   const int G = ((nv + kNT - 1) / kNT) | 1;
   const int vb = tid * G, ve = min(nv, vb + G);
   float gt = 0.0f;
@@ -258,7 +267,7 @@ __device__ void sample_unit(const E *sq, const E *sp, int nv, int v0, Shared &sh
     if constexpr (kPair) Elt<E>::load8(sq + 8 * v, yq);
     Elt<E>::load8(sp + 8 * v, yp);
 #pragma unroll
-    for (int e = 0; e < 8; ++e) gt += weight<kPair>(kPair ? yq[e] : 0.0f, yp[e], sh, k, inv_sq, inv_sp);
+    for (int e = 0; e < 8; ++e) gt += weight<kPair>(kPair ? yq[e] : 0.0f, yp[e], rs);
   }
   // block scan of the thread totals: warp inclusive scan, then warp offsets
   float incl = gt;
@@ -267,7 +276,7 @@ __device__ void sample_unit(const E *sq, const E *sp, int nv, int v0, Shared &sh
     const float t = __shfl_up_sync(0xFFFFFFFFu, incl, o);
     if (lane >= o) incl += t;
   }
-  float prev = __shfl_up_sync(0xFFFFFFFFu, incl, 1);
+  const float prev = __shfl_up_sync(0xFFFFFFFFu, incl, 1);
   if (lane == 31) sh.wtot[warp] = incl;
   __syncthreads();
   if (tid == 0) {
@@ -282,36 +291,41 @@ __device__ void sample_unit(const E *sq, const E *sp, int nv, int v0, Shared &sh
   }
   __syncthreads();
   const float woff = sh.wtot[warp];
-  const float excl = lane == 0 ? woff : woff + prev;
+  const float excl = lane == 0 ? woff : woff + prev;  // == previous thread's inclusive prefix
   const float inc = woff + incl;
   cluster.sync();  // totals of every CTA are published
 
   if (warp == 0) {
     float tot = 0.0f;
     if (lane < C) tot = *cluster.map_shared_rank(&sh.part_r, lane);
-    // sequential prefix over ranks, done by lane 0 for a fixed order
-    float totals[kMaxCluster];
+    // inclusive prefix over ranks in rank order (lane r: ranks 0..r)
+    float pre = tot;
 #pragma unroll
-    for (int r = 0; r < kMaxCluster; ++r) totals[r] = __shfl_sync(0xFFFFFFFFu, tot, r);
+    for (int o = 1; o < 32; o <<= 1) {
+      const float t = __shfl_up_sync(0xFFFFFFFFu, pre, o);
+      if (lane >= o) pre += t;
+    }
+    const float R = __shfl_sync(0xFFFFFFFFu, pre, C - 1);
+    float before = __shfl_up_sync(0xFFFFFFFFu, pre, 1);  // previous rank's inclusive prefix
+    if (lane == 0) before = 0.0f;
+    const double t = static_cast<double>(u) * static_cast<double>(R);
+    const bool cross = lane < C && tot > 0.0f && t >= static_cast<double>(before) &&
+                       t < static_cast<double>(pre);
+    const unsigned cm = __ballot_sync(0xFFFFFFFFu, cross);
+    const unsigned pm = __ballot_sync(0xFFFFFFFFu, lane < C && tot > 0.0f);
+    const int cr = cm ? __ffs(cm) - 1 : -1;
+    const float bcr = __shfl_sync(0xFFFFFFFFu, before, cr >= 0 ? cr : 0);
     if (lane == 0) {
-      float pre[kMaxCluster + 1];
-      pre[0] = 0.0f;
-      for (int r = 0; r < C; ++r) pre[r + 1] = pre[r] + totals[r];
-      const double R = pre[C];
       int here = 0;
       double tl = 0.0;
-      if (R > 0.0) {
-        const double t = u * R;
-        int cr = -1;
-        for (int r = 0; r < C; ++r)
-          if (t >= static_cast<double>(pre[r]) && t < static_cast<double>(pre[r + 1])) { cr = r; break; }
+      if (R > 0.0f) {
         if (cr >= 0) {
-          if (cr == rank) { here = 1; tl = t - static_cast<double>(pre[rank]); }
-        } else {
-          int last = -1;
-          for (int r = 0; r < C; ++r)
-            if (totals[r] > 0.0f) last = r;
-          if (last == rank) here = 2;
+          if (cr == rank) {
+            here = 1;
+            tl = t - static_cast<double>(bcr);
+          }
+        } else if (pm && 31 - __clz(pm) == rank) {
+          here = 2;  // rounding left u R at the top: take the last positive weight
         }
       }
       sh.sample_here = here;
@@ -323,30 +337,28 @@ __device__ void sample_unit(const E *sq, const E *sp, int nv, int v0, Shared &sh
     const double tl = sh.t_local;
     const int mine = (tl >= static_cast<double>(excl) && tl < static_cast<double>(inc)) ? 1 : 0;
     const int any = __syncthreads_or(mine);
-    int who = mine;
-    if (!any) who = 0;  // rounding gap: fall back to the last positive weight below
-    int token = -1;
-    if (who) {
+    if (mine) {
+      const float tf = f32_floor(tl - static_cast<double>(excl));
       float acc = 0.0f;
-      int lastpos = -1;
+      int token = -1, lastpos = -1;
       for (int v = vb; v < ve && token < 0; ++v) {
         float yq[8], yp[8];
         if constexpr (kPair) Elt<E>::load8(sq + 8 * v, yq);
         Elt<E>::load8(sp + 8 * v, yp);
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
-          const float w = weight<kPair>(kPair ? yq[e] : 0.0f, yp[e], sh, k, inv_sq, inv_sp);
+          const float w = weight<kPair>(kPair ? yq[e] : 0.0f, yp[e], rs);
           acc += w;
           if (w > 0.0f) lastpos = 8 * v + e;
-          if (token < 0 && tl < static_cast<double>(excl) + static_cast<double>(acc)) token = 8 * v + e;
+          if (token < 0 && acc > tf) token = 8 * v + e;
         }
       }
       if (token < 0) token = lastpos;
       if (token >= 0) *cluster.map_shared_rank(&sh.cand, 0) = v0 + token;
     }
-    if (!any) sh.sample_here = 2;
+    if (!any && tid == 0) sh.sample_here = 2;  // rounding gap between the two scan levels
+    __syncthreads();
   }
-  __syncthreads();
   if (sh.sample_here == 2) {
     // last positive weight of this CTA: the highest thread with gt > 0 scans
     const int mine = gt > 0.0f ? tid : -1;
@@ -365,18 +377,46 @@ __device__ void sample_unit(const E *sq, const E *sp, int nv, int v0, Shared &sh
         Elt<E>::load8(sp + 8 * v, yp);
 #pragma unroll
         for (int e = 0; e < 8; ++e)
-          if (weight<kPair>(kPair ? yq[e] : 0.0f, yp[e], sh, k, inv_sq, inv_sp) > 0.0f) lastpos = 8 * v + e;
+          if (weight<kPair>(kPair ? yq[e] : 0.0f, yp[e], rs) > 0.0f) lastpos = 8 * v + e;
       }
       if (lastpos >= 0) *cluster.map_shared_rank(&sh.cand, 0) = v0 + lastpos;
     }
   }
-  cluster.sync();  // the candidate is in rank 0
+}
+
+// exp(a) for an f64 argument, to f32 accuracy without f64 transcendentals:
+// a = hi + lo with hi = f32(a), exp(a) ~= expf(hi) (1 + lo).
+__device__ __forceinline__ float exp_split(double a) {
+  const float hi = static_cast<float>(a);
+  const float lo = static_cast<float>(a - static_cast<double>(hi));
+  return expf(hi) * (1.0f + lo);
+}
+
+// Acceptance of draft x (Algorithm 4): a = 1 when delta = 0 or q(x) <= pi(x),
+// else a = [u < pi(x)/q(x)].  ln p(x) - ln q(x) is formed in f64 from exact
+// logit differences, so the ratio carries only the f32 error of S_q / S_p.
+__device__ __forceinline__ void accept_test(Shared &sh, float yqx, float ypx, float u,
+                                            double invT) {
+  const double dq = static_cast<double>(yqx) - static_cast<double>(sh.Mq);
+  const double dp = static_cast<double>(ypx) - static_cast<double>(sh.Mp);
+  const double lq = static_cast<double>(logf(sh.Sq)), lp = static_cast<double>(logf(sh.Sp));
+  const float qx = exp_split(dq * invT - lq);
+  const float px = exp_split(dp * invT - lp);
+  int accept = 1;
+  if (sh.delta) {
+    const double L = (dp - dq) * invT + static_cast<double>(logf(sh.Sq / sh.Sp));
+    if (L < 0.0) accept = u < exp_split(L);
+  }
+  sh.accept = accept;
+  sh.qx = qx;
+  sh.pix = sh.delta ? px : qx;
+  sh.need_sample = !accept;
 }
 
 // ------------------------------------------------------------------ the kernel
 
 template <typename E>
-__global__ void __launch_bounds__(kNT, 2) sc_unit_kernel(const Params P) {
+__global__ void __launch_bounds__(kNT, 3) sc_unit_kernel(const Params P) {
   extern __shared__ __align__(128) unsigned char smem_raw[];
   cg::cluster_group cluster = cg::this_cluster();
   const int C = P.cluster;
@@ -396,8 +436,10 @@ __global__ void __launch_bounds__(kNT, 2) sc_unit_kernel(const Params P) {
     j = unit % P.gamma;
     pair = true;
   }
-  const E *gq = static_cast<const E *>(P.draft) + (static_cast<size_t>(b) * P.gamma + j) * P.V;
-  const E *gp = static_cast<const E *>(P.target) + (static_cast<size_t>(b) * G1 + j) * P.V;
+  const size_t qoff = (static_cast<size_t>(b) * P.gamma + j) * P.V;
+  const size_t poff = (static_cast<size_t>(b) * G1 + j) * P.V;
+  const E *gq = static_cast<const E *>(P.draft) + qoff;
+  const E *gp = static_cast<const E *>(P.target) + poff;
   const int v0 = rank * P.L;
   const int len = max(0, min(P.L, P.V - v0));
   const int lenp = (len + 7) & ~7;
@@ -406,9 +448,12 @@ __global__ void __launch_bounds__(kNT, 2) sc_unit_kernel(const Params P) {
 
   E *sq = reinterpret_cast<E *>(smem_raw);
   E *sp = sq + P.L;
-  Shared &sh = *reinterpret_cast<Shared *>(smem_raw + ((2 * static_cast<size_t>(P.L) * sizeof(E) + 15) & ~size_t(15)));
+  Shared &sh = *reinterpret_cast<Shared *>(
+      smem_raw + ((2 * static_cast<size_t>(P.L) * sizeof(E) + 15) & ~size_t(15)));
 
-  // ---- stage the slices
+  // ---- stage the slices; thread 0 then prefetches the row's scalars
+  float uj = 0.0f, ug = 0.0f, yqx = 0.0f, ypx = 0.0f;
+  int x = 0;
   if (tid == 0) {
     sh.cand = -1;
     sh.timeout = 0;
@@ -424,6 +469,17 @@ __global__ void __launch_bounds__(kNT, 2) sc_unit_kernel(const Params P) {
         bulk_g2s(sp + e0, gp + v0 + e0, bytes, &sh.bar[c]);
       }
     }
+    if (P.mode == kVerify) {
+      uj = P.uniforms[static_cast<size_t>(b) * G1 + j];
+      ug = P.uniforms[static_cast<size_t>(b) * G1 + P.gamma];
+      if (pair) {
+        x = P.tokens[static_cast<size_t>(b) * P.gamma + j];
+        if (x >= 0 && x < P.V) {
+          yqx = Elt<E>::at(P.draft, qoff + x);
+          ypx = Elt<E>::at(P.target, poff + x);
+        }
+      }
+    }
   }
   if (!P.bulk) {
     for (int i = tid; i < len; i += kNT) {
@@ -437,7 +493,7 @@ __global__ void __launch_bounds__(kNT, 2) sc_unit_kernel(const Params P) {
   }
   __syncthreads();
 
-  // ---- pass 1: online max and sum of exponentials
+  // ---- pass 1: online max and sum of exponentials while the chunks land
   const float k = P.k;
   float mq = -FLT_MAX, s_q = 0.0f, mp = -FLT_MAX, s_p = 0.0f;
   int tmo = 0;
@@ -449,7 +505,6 @@ __global__ void __launch_bounds__(kNT, 2) sc_unit_kernel(const Params P) {
     online_chunk<E>(sp, vbeg, vend, k, mp, s_p);
   }
   tmo = __syncthreads_or(tmo);
-  // warp then CTA reduction (fixed order: lane 0 of the shfl_down tree)
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     const float m2q = __shfl_down_sync(0xFFFFFFFFu, mq, o), s2q = __shfl_down_sync(0xFFFFFFFFu, s_q, o);
@@ -489,23 +544,15 @@ __global__ void __launch_bounds__(kNT, 2) sc_unit_kernel(const Params P) {
       ms_combine(a, as, a2, as2, k);
       ms_combine(c, cs, c2, cs2, k);
     }
-    if (lane == 0) {
+    if (lane == 0) {  // thread 0: it holds the prefetched scalars
       sh.Mq = a; sh.Sq = as; sh.Mp = c; sh.Sp = cs;
-      // ---- row validity, deferral (Table 1) and, where possible, acceptance
       int err = 0;
       const bool okq = !pair || (isfinite(a) && isfinite(as) && as > 0.0f);
       const bool okp = isfinite(c) && isfinite(cs) && cs > 0.0f;
       if (!(okq && okp)) err |= SC_DEV_BAD_LOGIT;
-      double u = 0.0;
-      int x = 0;
       if (P.mode == kVerify) {
-        const float uf = P.uniforms[static_cast<size_t>(b) * G1 + j];
-        if (!(uf >= 0.0f && uf < 1.0f)) err |= SC_DEV_BAD_UNIFORM;
-        u = uf;
-        if (pair) {
-          x = P.tokens[static_cast<size_t>(b) * P.gamma + j];
-          if (x < 0 || x >= P.V) err |= SC_DEV_BAD_TOKEN;
-        }
+        if (!(uj >= 0.0f && uj < 1.0f)) err |= SC_DEV_BAD_UNIFORM;
+        if (pair && (x < 0 || x >= P.V)) err |= SC_DEV_BAD_TOKEN;
       }
       if (err && P.status) atomicOr(P.status, err);
       sh.err = err;
@@ -516,17 +563,20 @@ __global__ void __launch_bounds__(kNT, 2) sc_unit_kernel(const Params P) {
       sh.tv = -1.0f;
       sh.qx = 0.0f;
       sh.pix = 0.0f;
-      if (!err && pair) {
-        sh.lq = static_cast<float>(log2(static_cast<double>(as)));
-        sh.lp = static_cast<float>(log2(static_cast<double>(cs)));
-        const double maxq = 1.0 / as, maxp = 1.0 / cs, al = P.alpha;
-        if (P.mode == kStats) {
+      sh.c = pair && !err ? log2f(as / cs) : 0.0f;
+      sh.ug = ug;
+      if (!err) {
+        if (!pair) {
+          sh.need_sample = P.mode == kVerify;  // bonus row: drawn speculatively
+        } else if (P.mode == kStats) {
           sh.need_tv = 1;
         } else {
+          // deferral rule (Table 1); max q = 1/S_q, max p = 1/S_p
+          const float maxq = 1.0f / as, maxp = 1.0f / cs, al = P.alpha;
           switch (P.rule) {
-            case SC_RULE_CHOW: sh.delta = maxq < 1.0 - al; break;
-            case SC_RULE_DIFF: sh.delta = maxq < maxp - al; break;
-            case SC_RULE_OPT:
+            case SC_RULE_CHOW: sh.delta = maxq < 1.0f - al; break;  // Eq. 2
+            case SC_RULE_DIFF: sh.delta = maxq < maxp - al; break;  // Eq. 5
+            case SC_RULE_OPT:                                       // Eq. 10
               // alpha * TV lies in [0, alpha]: the TV term decides only inside that band
               if (!(maxq < maxp)) sh.delta = 0;
               else if (maxq < maxp - al) sh.delta = 1;
@@ -535,15 +585,16 @@ __global__ void __launch_bounds__(kNT, 2) sc_unit_kernel(const Params P) {
             case SC_RULE_ALWAYS_DEFER: sh.delta = 1; break;
             default: sh.delta = 0; break;
           }
+          if (!sh.need_tv) accept_test(sh, yqx, ypx, uj, P.inv_t);
         }
       }
     }
   }
   __syncthreads();
+  const RowScalars rs = {sh.Mq, sh.Mp, k, sh.c};
 
-  // ---- TV pass (shared memory only)
+  // ---- TV pass (shared memory only): sum_v min(p_v, q_v) = (1/S_q) sum_v 2^min(a_v, b_v + c)
   if (sh.need_tv) {
-    const float Mq = sh.Mq, Mp = sh.Mp, lq = sh.lq, lp = sh.lp;
     float acc = 0.0f;
     for (int v = tid; v < nv; v += kNT) {
       float yq[8], yp[8];
@@ -551,7 +602,7 @@ __global__ void __launch_bounds__(kNT, 2) sc_unit_kernel(const Params P) {
       Elt<E>::load8(sp + 8 * v, yp);
 #pragma unroll
       for (int e = 0; e < 8; ++e)
-        acc += ex2(fminf(fmaf(yq[e] - Mq, k, -lq), fmaf(yp[e] - Mp, k, -lp)));
+        acc += ex2(fminf((yq[e] - rs.Mq) * k, fmaf(yp[e] - rs.Mp, k, rs.c)));
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) acc += __shfl_down_sync(0xFFFFFFFFu, acc, o);
@@ -569,47 +620,27 @@ __global__ void __launch_bounds__(kNT, 2) sc_unit_kernel(const Params P) {
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) t += __shfl_down_sync(0xFFFFFFFFu, t, o);
       if (lane == 0) {
-        const float tv = fminf(1.0f, fmaxf(0.0f, 1.0f - t));
+        const float tv = fminf(1.0f, fmaxf(0.0f, 1.0f - t / sh.Sq));  // Lemma 3
         sh.tv = tv;
         if (P.mode == kVerify) {
-          const double maxq = 1.0 / sh.Sq, maxp = 1.0 / sh.Sp;
-          sh.delta = maxq < maxp - static_cast<double>(P.alpha) * tv;  // Eq. 10
+          sh.delta = 1.0f / sh.Sq < 1.0f / sh.Sp - P.alpha * tv;  // Eq. 10
+          accept_test(sh, yqx, ypx, uj, P.inv_t);
         }
       }
     }
     __syncthreads();
   }
 
-  // ---- acceptance (Algorithm 4: a_j ~ Ber(min(1, pi(x)/q(x))))
-  if (P.mode == kVerify && tid == 0) {
-    if (!sh.err) {
-      if (pair) {
-        const int x = P.tokens[static_cast<size_t>(b) * P.gamma + j];
-        const double invT = 1.0 / static_cast<double>(P.temperature);
-        const double yqx = Elt<E>::at(P.draft, (static_cast<size_t>(b) * P.gamma + j) * P.V + x);
-        const double ypx = Elt<E>::at(P.target, (static_cast<size_t>(b) * G1 + j) * P.V + x);
-        const double qx = exp((yqx - sh.Mq) * invT) / sh.Sq;
-        const double px = exp((ypx - sh.Mp) * invT) / sh.Sp;
-        const double pix = sh.delta ? px : qx;
-        const double u = P.uniforms[static_cast<size_t>(b) * G1 + j];
-        int accept = 1;
-        if (sh.delta && qx > pix) accept = u < pix / qx;
-        sh.accept = accept;
-        sh.qx = static_cast<float>(qx);
-        sh.pix = static_cast<float>(pix);
-        sh.need_sample = !accept;
-      } else {
-        sh.need_sample = 1;  // bonus row: drawn speculatively, used when j* = gamma
-      }
-    }
-  }
-  __syncthreads();
-
   if (sh.need_sample) {
-    const double u = P.uniforms[static_cast<size_t>(b) * G1 + P.gamma];
-    if (pair) sample_unit<E, true>(sq, sp, nv, v0, sh, k, u, cluster, rank, C);
-    else sample_unit<E, false>(sq, sp, nv, v0, sh, k, u, cluster, rank, C);
+    const float u = sh.ug;  // thread 0 prefetched it
+    if (pair) sample_unit<E, true>(sq, sp, nv, v0, sh, rs, u, cluster, rank, C);
+    else sample_unit<E, false>(sq, sp, nv, v0, sh, rs, u, cluster, rank, C);
   }
+  if (sh.timeout && tid == 0 && P.bulk) {
+    // let copies still in flight land before this CTA's shared memory is released
+    for (int c = 0; c < nchunks; ++c) mbar_wait(&sh.bar[c], 0);
+  }
+  cluster.sync();  // candidate visible in rank 0; no peer reads this CTA's shared memory after
 
   // ---- publish this unit; the last unit of the sequence finishes it
   if (rank == 0 && tid == 0) {
@@ -635,10 +666,12 @@ __global__ void __launch_bounds__(kNT, 2) sc_unit_kernel(const Params P) {
       }
       P.unit_flags[r] = (sh.accept ? 1 : 0) | (sh.err ? 2 : 0);
       P.unit_cand[r] = cand;
-      __threadfence();
-      const uint32_t ticket = atomicAdd(&P.tickets[b], 1u);
+      uint32_t ticket;
+      asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;"
+                   : "=r"(ticket)
+                   : "l"(P.tickets + b)
+                   : "memory");
       if (ticket == static_cast<uint32_t>(P.gamma)) {
-        __threadfence();
         int jstar = P.gamma, bad = 0;
         const size_t base = static_cast<size_t>(b) * G1;
         for (int jj = 0; jj <= P.gamma; ++jj) {
@@ -653,11 +686,6 @@ __global__ void __launch_bounds__(kNT, 2) sc_unit_kernel(const Params P) {
       }
     }
   }
-  if (sh.timeout && tid == 0 && P.bulk) {
-    // let copies still in flight land before this CTA's shared memory is released
-    for (int c = 0; c < nchunks; ++c) mbar_wait(&sh.bar[c], 0);
-  }
-  cluster.sync();  // no CTA leaves while a peer may still read its shared memory
 }
 
 // ------------------------------------------------------------------ host side
@@ -832,6 +860,7 @@ int sc_verify_rows(const void *draft_logits, const void *target_logits, sc_dtype
   P.alpha = alpha;
   P.temperature = temperature;
   P.k = static_cast<float>(1.4426950408889634 / static_cast<double>(temperature));
+  P.inv_t = 1.0 / static_cast<double>(temperature);
   P.mode = kVerify;
   P.num_accepted = num_accepted;
   P.next_token = next_token;
@@ -871,6 +900,7 @@ int sc_row_stats(const void *draft_logits, const void *target_logits, sc_dtype d
   P.V = V;
   P.temperature = temperature;
   P.k = static_cast<float>(1.4426950408889634 / static_cast<double>(temperature));
+  P.inv_t = 1.0 / static_cast<double>(temperature);
   P.mode = kStats;
   P.max_q = max_q;
   P.max_p = max_p;
