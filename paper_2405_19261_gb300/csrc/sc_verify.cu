@@ -5,39 +5,40 @@
 // for B sequences of gamma drafted positions over a V-token vocabulary, in ONE
 // kernel launch:
 //
-//   unit  = one (b, j < gamma) row pair (draft row q_j, target row p_j), or the
-//           bonus target row (b, gamma);
-//   grid  = one thread-block cluster of C CTAs per unit; CTA r of the cluster
-//           owns the vocabulary slice [r L, (r+1) L) of both rows;
-//   HBM   = each logit is read once, by TMA bulk copies (cp.async.bulk) into the
-//           owning CTA's shared memory, in chunks that each have an mbarrier;
-//   pass1 = online max / sum-of-exp per thread while the chunks land, reduced
-//           over warps, then over the cluster through distributed shared memory;
-//   TV    = only when needed (sc_row_stats, or the OPT rule when the TV term can
-//           change the decision): sum_v min(p_v, q_v) from shared memory,
-//           D_TV = 1 - sum_v min(p_v, q_v) (Lemma 3);
-//   accept= delta (Table 1) and the Bernoulli test u < pi(x)/q(x) on two
-//           scalars, in fp64;
-//   sample= a rejecting pair (residual max(0, p - q)) or the bonus row (p)
-//           draws its token by inverse CDF: per-thread contiguous partial sums,
-//           a block scan, a cluster scan of CTA totals, then one thread finds
-//           the crossing element;
-//   scan  = the last unit of a sequence to finish (atomic ticket, no waiting)
-//           finds j* = min{j : a_j = 0} and writes the outputs.
+//   unit   one (b, j < gamma) row pair (draft row q_j, target row p_j), or the
+//          bonus target row (b, gamma);
+//   grid   one thread-block cluster of C CTAs per unit; CTA r of the cluster
+//          owns the vocabulary slice [r L, (r+1) L) of both rows;
+//   pass 1 the slice streams from HBM through a two-stage shared-memory ring
+//          filled by TMA bulk copies (cp.async.bulk + mbarrier), 2048 logits
+//          per row per stage; each thread keeps an online (max, sum of exp);
+//          the CTA partials are merged over the cluster through distributed
+//          shared memory, giving M and S of both rows, max q = 1/S_q and
+//          max p = 1/S_p, and the deferral decision of Table 1;
+//   pass 2 only when the unit needs it (a rejected draft, the bonus row, the
+//          OPT rule inside the band where its TV term decides, sc_row_stats):
+//          the slice is streamed again -- it is still in L2 -- and every
+//          element gets its residual weight max(0, p - q) (p for the bonus
+//          row).  Their total over the cluster is D_TV(p, q) * S_q (Lemma 3),
+//          and the per-(chunk, round, warp) totals drive the inverse-CDF search;
+//   search the CTA whose slice holds u * R finds the segment, one warp reloads
+//          it and scans it, and that CTA publishes the unit;
+//   scan   the last unit of a sequence to finish (atomic ticket, no waiting)
+//          finds j* = min{j : a_j = 0} and writes the outputs.
 //
-// Exponentials use ex2.approx on (y - M) * log2(e)/T; (y - M) is exact for bf16
-// logits.  Nothing in the kernel waits on another cluster; mbarrier waits are
-// bounded and report SC_DEV_TIMEOUT instead of hanging.
+// Exponentials are ex2.approx of fma(y, log2(e)/T, -R), R = fl(M log2(e)/T):
+// one rounding per logit.  No thread waits on another cluster; every mbarrier wait is bounded
+// and reports SC_DEV_TIMEOUT instead of hanging.
 
 #include "sc.h"
 
 #include <cooperative_groups.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cfloat>
 #include <cmath>
 #include <cstdint>
-#include <algorithm>
 #include <cstdlib>
 #include <mutex>
 
@@ -45,14 +46,17 @@ namespace cg = cooperative_groups;
 
 namespace {
 
-constexpr int kNT = 256;                      // threads per CTA
-constexpr int kNW = kNT / 32;                 // warps per CTA
-constexpr int kVPT = 2;                       // 8-element vectors per thread per chunk
-constexpr int kVecPerChunk = kNT * kVPT;      // 512 vectors = 4096 elements per chunk
-constexpr int kChunkElems = kVecPerChunk * 8;
-constexpr int kMaxChunks = 32;
+constexpr int kNT = 128;                   // threads per CTA
+constexpr int kNW = kNT / 32;              // warps per CTA
+constexpr int kCH = 2048;                  // logits per row per ring stage
+constexpr int kVPC = kCH / 8;              // 8-element vectors per chunk
+constexpr int kRounds = kVPC / kNT;        // vectors per thread per chunk
+constexpr int kStages = 2;                 // ring depth
+constexpr int kMaxChunks = 32;             // slice <= 65536 logits per row
 constexpr int kMaxCluster = 16;
-constexpr uint32_t kWaitLimit = 1u << 22;     // bounded mbarrier waits (~seconds)
+constexpr int kEntries = kMaxChunks * kRounds * kNW;  // (chunk, round, warp) segments
+constexpr uint32_t kWaitLimit = 1u << 22;  // bounded mbarrier waits (~seconds)
+constexpr int kMinBlocksPerSM = 8;
 
 enum Mode : int { kVerify = 0, kStats = 1 };
 
@@ -66,10 +70,10 @@ struct Params {
   float alpha;
   float temperature;
   float k;        // log2(e) / T
-  double inv_t;   // 1 / T
-  int L;          // slice length per CTA (multiple of 8 elements)
+  double kd;      // log2(e) / T in f64, for the decision scalars
+  int L;          // slice length per CTA (multiple of 8 logits)
   int cluster;    // CTAs per unit
-  int bulk;       // 1: TMA bulk copies, 0: per-thread loads (unaligned rows)
+  int bulk;       // 1: TMA bulk copies, 0: per-thread loads (rows not 16-byte aligned)
   int mode;
   int32_t *num_accepted;
   int32_t *next_token;
@@ -106,7 +110,7 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t *bar, uint32_t bytes) {
                : "memory");
 }
 
-// Bounded wait for phase `parity` of an mbarrier; false on timeout.
+// Bounded wait for the phase of parity `parity` of an mbarrier; false on timeout.
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity) {
   const uint32_t a = smem_u32(bar);
   for (uint32_t i = 0; i < kWaitLimit; ++i) {
@@ -133,6 +137,13 @@ __device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t by
       : "memory");
 }
 
+__device__ __forceinline__ void cluster_arrive() {
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
 // ------------------------------------------------------------------ logit types
 
 template <typename E>
@@ -140,9 +151,7 @@ struct Elt;
 
 template <>
 struct Elt<uint16_t> {  // bf16 bit patterns
-  static constexpr uint16_t kNegInf = 0xFF80u;
-  __device__ __forceinline__ static void load8(const uint16_t *s, float (&y)[8]) {
-    const uint4 v = *reinterpret_cast<const uint4 *>(s);
+  __device__ __forceinline__ static void unpack(const uint4 v, float (&y)[8]) {
     const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
@@ -150,273 +159,292 @@ struct Elt<uint16_t> {  // bf16 bit patterns
       y[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
     }
   }
-  __device__ __forceinline__ static float at(const void *g, size_t i) {
-    return __uint_as_float(static_cast<uint32_t>(static_cast<const uint16_t *>(g)[i]) << 16);
+  __device__ __forceinline__ static void load8(const uint16_t *s, float (&y)[8]) {
+    unpack(*reinterpret_cast<const uint4 *>(s), y);
+  }
+  __device__ __forceinline__ static void load8_global(const uint16_t *g, float (&y)[8]) {
+    unpack(__ldcs(reinterpret_cast<const uint4 *>(g)), y);
+  }
+  __device__ __forceinline__ static float at(const uint16_t *g, size_t i) {
+    return __uint_as_float(static_cast<uint32_t>(g[i]) << 16);
   }
 };
 
 template <>
 struct Elt<float> {
-  static constexpr float kNegInf = -INFINITY;
   __device__ __forceinline__ static void load8(const float *s, float (&y)[8]) {
     const float4 a = *reinterpret_cast<const float4 *>(s);
     const float4 b = *reinterpret_cast<const float4 *>(s + 4);
     y[0] = a.x; y[1] = a.y; y[2] = a.z; y[3] = a.w;
     y[4] = b.x; y[5] = b.y; y[6] = b.z; y[7] = b.w;
   }
-  __device__ __forceinline__ static float at(const void *g, size_t i) {
-    return static_cast<const float *>(g)[i];
+  __device__ __forceinline__ static void load8_global(const float *g, float (&y)[8]) {
+    const float4 a = __ldcs(reinterpret_cast<const float4 *>(g));
+    const float4 b = __ldcs(reinterpret_cast<const float4 *>(g + 4));
+    y[0] = a.x; y[1] = a.y; y[2] = a.z; y[3] = a.w;
+    y[4] = b.x; y[5] = b.y; y[6] = b.z; y[7] = b.w;
   }
+  __device__ __forceinline__ static float at(const float *g, size_t i) { return g[i]; }
 };
+
+// Eight logits starting at element e of a row slice of n valid logits; the
+// ones at or past n read as -inf (probability 0).
+template <typename E>
+__device__ __forceinline__ void load8_smem(const E *s, int e, int n, float (&y)[8]) {
+  if (e + 8 <= n) {
+    Elt<E>::load8(s + e, y);
+  } else {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) y[i] = e + i < n ? Elt<E>::at(s, e + i) : -INFINITY;
+  }
+}
+
+template <typename E>
+__device__ __forceinline__ void load8_gmem(const E *g, int e, int n, bool vec, float (&y)[8]) {
+  if (vec && e + 8 <= n) {
+    Elt<E>::load8_global(g + e, y);
+  } else {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) y[i] = e + i < n ? Elt<E>::at(g, e + i) : -INFINITY;
+  }
+}
 
 // ------------------------------------------------------------------ shared state
 
 struct __align__(16) Shared {
-  uint64_t bar[kMaxChunks];
-  float4 part_ms;        // this CTA's (m_q, s_q, m_p, s_p), read by the cluster
-  float part_tv;         // this CTA's sum of 2^min(a, b + c)
-  float part_r;          // this CTA's total sampling weight
-  int cand;              // sampled token (written remotely into rank 0)
+  uint64_t full[kStages];
+  // exchange 1: (m_q, s_q, m_p, s_p) of this CTA, raw logits at the draft token
+  float4 part_ms;
+  float2 part_x;
+  // exchange 2: this CTA's total residual weight
+  float part_r;
   int timeout;
   float red[kNW][4];
-  float wtot[kNW + 1];
-  // row statistics, identical in every CTA of the cluster
-  float Mq, Sq, Mp, Sp;
-  float c;               // log2(S_q / S_p)
-  float tv;
-  int err, delta, need_tv, need_sample, accept;
-  float qx, pix;
-  double t_local;        // u * R minus the weight of the CTAs before the crossing one
-  float ug;              // u[b][gamma], the residual / bonus draw
-  int sample_here;       // 1: crossing inside this CTA, 2: take its last positive weight
+  float seg[kEntries + 1];  // per-(chunk, round, warp) weights, then exclusive prefixes
+  float xq, xp;             // raw logits at the draft token, when in this slice
+  // row state, identical in every CTA of the cluster
+  float Mq, Sq, Mp, Sp, Rq, Rp, maxq, maxp, c, tv, qx, pix, ug;
+  int err, delta, accept, need_p2, sample;
+  int publisher;            // rank that publishes the unit
+  int cross_seg;            // segment holding u*R in the publishing CTA (-1: last positive)
+  float t_seg;              // u*R minus the weight before that segment
 };
 
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
+// Exponent reference of a running maximum m: r = fl(m k), floored at -1e30 so
+// that a slice of -inf logits keeps finite arithmetic.  Every exponential of
+// pass 1 is 2^{fma(y, k, -r)}: one rounding, no systematic error (the max
+// logit's own term is 2^{fma(M, k, -R)}, not exactly 1, and is treated so).
+__device__ __forceinline__ float refk(float m, float k) { return fmaxf(__fmul_rn(m, k), -1e30f); }
+
+// Merge two (max, sum) partials; each sum is relative to refk of its max.
 __device__ __forceinline__ void ms_combine(float &m, float &s, float m2, float s2, float k) {
   const float mn = fmaxf(m, m2);
-  s = s * ex2((m - mn) * k) + s2 * ex2((m2 - mn) * k);
+  const float rn = refk(mn, k);
+  s = s * ex2(refk(m, k) - rn) + s2 * ex2(refk(m2, k) - rn);
   m = mn;
 }
 
-// Per-thread online max / sum of exp2((y - m) k) over this thread's vectors of
-// one chunk (vectors vbeg + tid + i * kNT).
-template <typename E>
-__device__ __forceinline__ void online_chunk(const E *row, int vbeg, int vend, float k, float &m,
-                                             float &s) {
-  float y[kVPT][8];
-  bool act[kVPT];
-  float vmax = -FLT_MAX;
+// Pass 1 on one row of one chunk: this thread's kRounds vectors, online
+// (max m, sum s of 2^{y k - refk(m)}).  kFull: the chunk holds kCH logits.
+template <typename E, bool kFull>
+__device__ __forceinline__ void online_row(const E *src, int n, float k, float &m, float &s) {
+  float y[kRounds][8];
 #pragma unroll
-  for (int i = 0; i < kVPT; ++i) {
-    const int v = vbeg + static_cast<int>(threadIdx.x) + i * kNT;
-    act[i] = v < vend;
-    if (act[i]) {
-      Elt<E>::load8(row + 8 * v, y[i]);
-#pragma unroll
-      for (int e = 0; e < 8; ++e) vmax = fmaxf(vmax, y[i][e]);
+  for (int r = 0; r < kRounds; ++r) {
+    const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
+    if constexpr (kFull) {
+      Elt<E>::load8(src + e, y[r]);
+    } else {
+      load8_smem(src, e, n, y[r]);
     }
   }
-  const float mn = fmaxf(m, vmax);
-  float acc = s * ex2((m - mn) * k);
+  float mn = m;
 #pragma unroll
-  for (int i = 0; i < kVPT; ++i)
-    if (act[i]) {
+  for (int r = 0; r < kRounds; ++r)
 #pragma unroll
-      for (int e = 0; e < 8; ++e) acc += ex2((y[i][e] - mn) * k);
+    for (int i = 0; i < 8; i += 2) mn = max3(mn, y[r][i], y[r][i + 1]);
+  const float rn = refk(mn, k);
+  float s0 = s * ex2(refk(m, k) - rn), s1 = 0.0f;
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r)
+#pragma unroll
+    for (int i = 0; i < 8; i += 2) {
+      s0 += ex2(fmaf(y[r][i], k, -rn));
+      s1 += ex2(fmaf(y[r][i + 1], k, -rn));
     }
   m = mn;
-  s = acc;
+  s = s0 + s1;
 }
 
-// Row scalars in registers for the shared-memory passes.  With
-// a_v = (y^q_v - M_q) k and b_v = (y^p_v - M_p) k (k = log2(e)/T):
-//   q_v = 2^{a_v} / S_q,   p_v = 2^{b_v} / S_p = 2^{b_v + c} / S_q,   c = log2(S_q / S_p).
+// Row scalars of the weight formula.  With a_v = y^q_v k - R_q, b_v = y^p_v k - R_p
+// (R = refk(M)) and c = log2(S_q / S_p):
+//   q_v = 2^{a_v} / S_q,   p_v = 2^{b_v} / S_p = 2^{b_v + c} / S_q,
+// so max(0, p_v - q_v) = max(0, 2^{b_v + c} - 2^{a_v}) / S_q.
 struct RowScalars {
-  float Mq, Mp, k, c;
+  float Rq, Rp, k, c;
 };
 
-// Sampling weight of one element, up to the common factor 1/S_q:
-// residual max(0, p - q) of a pair, or p of the bonus row.
+// Sampling weight of one logit, up to the common factor 1/S_q: the residual
+// max(0, p - q) of a pair, or the unnormalised p of the bonus row.  Rounded
+// intrinsics keep every evaluation of the same logit bit-identical.
 template <bool kPair>
 __device__ __forceinline__ float weight(float yq, float yp, const RowScalars &r) {
   if constexpr (kPair) {
-    const float a = (yq - r.Mq) * r.k;
-    const float b = fmaf(yp - r.Mp, r.k, r.c);
-    return fmaxf(0.0f, ex2(b) - ex2(a));
+    const float a = __fmaf_rn(yq, r.k, -r.Rq);
+    const float b = __fadd_rn(__fmaf_rn(yp, r.k, -r.Rp), r.c);
+    return fmaxf(0.0f, __fsub_rn(ex2(b), ex2(a)));
   } else {
-    return ex2((yp - r.Mp) * r.k);
+    return ex2(__fmaf_rn(yp, r.k, -r.Rp));
   }
 }
 
-// f32 a, f64 t: (a > t) == (a > round_down_to_f32(t)).
-__device__ __forceinline__ float f32_floor(double t) { return __double2float_rd(t); }
-
-// Inverse-CDF draw over the cluster's slices.  Every thread of every CTA calls
-// it; the chosen token is written into rank 0's Shared::cand, visible there
-// after the caller's next cluster barrier.
-template <typename E, bool kPair>
-__device__ void sample_unit(const E *sq, const E *sp, int nv, int v0, Shared &sh,
-                            const RowScalars &rs, float u, cg::cluster_group &cluster, int rank,
-                            int C) {
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  // contiguous ownership with an odd stride: conflict-free 16-byte shared loads
-  const int G = ((nv + kNT - 1) / kNT) | 1;
-  const int vb = tid * G, ve = min(nv, vb + G);
-  float gt = 0.0f;
-  for (int v = vb; v < ve; ++v) {
-    float yq[8], yp[8];
-    if constexpr (kPair) Elt<E>::load8(sq + 8 * v, yq);
-    Elt<E>::load8(sp + 8 * v, yp);
+// Eight weights and their sum in index order.  Used identically by pass 2 and
+// by the search.
+template <bool kPair>
+__device__ __forceinline__ float vec_weights(const float (&yq)[8], const float (&yp)[8],
+                                             const RowScalars &r, float (&w)[8]) {
+  float s = 0.0f;
 #pragma unroll
-    for (int e = 0; e < 8; ++e) gt += weight<kPair>(kPair ? yq[e] : 0.0f, yp[e], rs);
+  for (int e = 0; e < 8; ++e) {
+    w[e] = weight<kPair>(kPair ? yq[e] : 0.0f, yp[e], r);
+    s = __fadd_rn(s, w[e]);
   }
-  // block scan of the thread totals: warp inclusive scan, then warp offsets
-  float incl = gt;
+  return s;
+}
+
+__device__ __forceinline__ float warp_incl_scan(float v, int lane) {
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
-    const float t = __shfl_up_sync(0xFFFFFFFFu, incl, o);
-    if (lane >= o) incl += t;
+    const float t = __shfl_up_sync(0xFFFFFFFFu, v, o);
+    if (lane >= o) v = __fadd_rn(v, t);
   }
-  const float prev = __shfl_up_sync(0xFFFFFFFFu, incl, 1);
-  if (lane == 31) sh.wtot[warp] = incl;
-  __syncthreads();
-  if (tid == 0) {
-    float acc = 0.0f;
-    for (int w = 0; w < kNW; ++w) {
-      const float t = sh.wtot[w];
-      sh.wtot[w] = acc;  // becomes the warp offset
-      acc = acc + t;
-    }
-    sh.wtot[kNW] = acc;
-    sh.part_r = acc;
-  }
-  __syncthreads();
-  const float woff = sh.wtot[warp];
-  const float excl = lane == 0 ? woff : woff + prev;  // == previous thread's inclusive prefix
-  const float inc = woff + incl;
-  cluster.sync();  // totals of every CTA are published
+  return v;
+}
 
-  if (warp == 0) {
-    float tot = 0.0f;
-    if (lane < C) tot = *cluster.map_shared_rank(&sh.part_r, lane);
-    // inclusive prefix over ranks in rank order (lane r: ranks 0..r)
-    float pre = tot;
+// Pass 2 on one chunk: per round, the warp's total weight (lane 31 of an
+// inclusive scan) lands in seg[(c, round, warp)].
+template <typename E, bool kPair, bool kFull>
+__device__ __forceinline__ void weights_chunk(const E *sq, const E *sp, int n, int c,
+                                              const RowScalars &rs, Shared &sh, int lane,
+                                              int warp) {
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const float t = __shfl_up_sync(0xFFFFFFFFu, pre, o);
-      if (lane >= o) pre += t;
+  for (int r = 0; r < kRounds; ++r) {
+    const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
+    float yq[8], yp[8], w[8];
+    if constexpr (kFull) {
+      if constexpr (kPair) Elt<E>::load8(sq + e, yq);
+      Elt<E>::load8(sp + e, yp);
+    } else {
+      if constexpr (kPair) load8_smem(sq, e, n, yq);
+      load8_smem(sp, e, n, yp);
     }
-    const float R = __shfl_sync(0xFFFFFFFFu, pre, C - 1);
-    float before = __shfl_up_sync(0xFFFFFFFFu, pre, 1);  // previous rank's inclusive prefix
-    if (lane == 0) before = 0.0f;
-    const double t = static_cast<double>(u) * static_cast<double>(R);
-    const bool cross = lane < C && tot > 0.0f && t >= static_cast<double>(before) &&
-                       t < static_cast<double>(pre);
-    const unsigned cm = __ballot_sync(0xFFFFFFFFu, cross);
-    const unsigned pm = __ballot_sync(0xFFFFFFFFu, lane < C && tot > 0.0f);
-    const int cr = cm ? __ffs(cm) - 1 : -1;
-    const float bcr = __shfl_sync(0xFFFFFFFFu, before, cr >= 0 ? cr : 0);
-    if (lane == 0) {
-      int here = 0;
-      double tl = 0.0;
-      if (R > 0.0f) {
-        if (cr >= 0) {
-          if (cr == rank) {
-            here = 1;
-            tl = t - static_cast<double>(bcr);
-          }
-        } else if (pm && 31 - __clz(pm) == rank) {
-          here = 2;  // rounding left u R at the top: take the last positive weight
-        }
-      }
-      sh.sample_here = here;
-      sh.t_local = tl;
-    }
-  }
-  __syncthreads();
-  if (sh.sample_here == 1) {
-    const double tl = sh.t_local;
-    const int mine = (tl >= static_cast<double>(excl) && tl < static_cast<double>(inc)) ? 1 : 0;
-    const int any = __syncthreads_or(mine);
-    if (mine) {
-      const float tf = f32_floor(tl - static_cast<double>(excl));
-      float acc = 0.0f;
-      int token = -1, lastpos = -1;
-      for (int v = vb; v < ve && token < 0; ++v) {
-        float yq[8], yp[8];
-        if constexpr (kPair) Elt<E>::load8(sq + 8 * v, yq);
-        Elt<E>::load8(sp + 8 * v, yp);
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const float w = weight<kPair>(kPair ? yq[e] : 0.0f, yp[e], rs);
-          acc += w;
-          if (w > 0.0f) lastpos = 8 * v + e;
-          if (token < 0 && acc > tf) token = 8 * v + e;
-        }
-      }
-      if (token < 0) token = lastpos;
-      if (token >= 0) *cluster.map_shared_rank(&sh.cand, 0) = v0 + token;
-    }
-    if (!any && tid == 0) sh.sample_here = 2;  // rounding gap between the two scan levels
-    __syncthreads();
-  }
-  if (sh.sample_here == 2) {
-    // last positive weight of this CTA: the highest thread with gt > 0 scans
-    const int mine = gt > 0.0f ? tid : -1;
-    int best = mine;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) best = max(best, __shfl_xor_sync(0xFFFFFFFFu, best, o));
-    if (lane == 0) sh.red[warp][0] = __int_as_float(best);
-    __syncthreads();
-    int top = -1;
-    for (int w = 0; w < kNW; ++w) top = max(top, __float_as_int(sh.red[w][0]));
-    if (tid == top) {
-      int lastpos = -1;
-      for (int v = vb; v < ve; ++v) {
-        float yq[8], yp[8];
-        if constexpr (kPair) Elt<E>::load8(sq + 8 * v, yq);
-        Elt<E>::load8(sp + 8 * v, yp);
-#pragma unroll
-        for (int e = 0; e < 8; ++e)
-          if (weight<kPair>(kPair ? yq[e] : 0.0f, yp[e], rs) > 0.0f) lastpos = 8 * v + e;
-      }
-      if (lastpos >= 0) *cluster.map_shared_rank(&sh.cand, 0) = v0 + lastpos;
-    }
+    const float vs = vec_weights<kPair>(yq, yp, rs, w);
+    const float incl = warp_incl_scan(vs, lane);
+    if (lane == 31) sh.seg[(c * kRounds + r) * kNW + warp] = incl;
   }
 }
 
-// exp(a) for an f64 argument, to f32 accuracy without f64 transcendentals:
-// a = hi + lo with hi = f32(a), exp(a) ~= expf(hi) (1 + lo).
-__device__ __forceinline__ float exp_split(double a) {
+// exp2(a) for an f64 argument to f32 accuracy without f64 transcendentals:
+// a = hi + lo with hi = f32(a), 2^a ~= exp2f(hi) (1 + lo ln 2).
+__device__ __forceinline__ float exp2_split(double a) {
   const float hi = static_cast<float>(a);
   const float lo = static_cast<float>(a - static_cast<double>(hi));
-  return expf(hi) * (1.0f + lo);
+  return exp2f(hi) * fmaf(lo, 0.69314718f, 1.0f);
 }
 
-// Acceptance of draft x (Algorithm 4): a = 1 when delta = 0 or q(x) <= pi(x),
-// else a = [u < pi(x)/q(x)].  ln p(x) - ln q(x) is formed in f64 from exact
-// logit differences, so the ratio carries only the f32 error of S_q / S_p.
-__device__ __forceinline__ void accept_test(Shared &sh, float yqx, float ypx, float u,
-                                            double invT) {
-  const double dq = static_cast<double>(yqx) - static_cast<double>(sh.Mq);
-  const double dp = static_cast<double>(ypx) - static_cast<double>(sh.Mp);
-  const double lq = static_cast<double>(logf(sh.Sq)), lp = static_cast<double>(logf(sh.Sp));
-  const float qx = exp_split(dq * invT - lq);
-  const float px = exp_split(dp * invT - lp);
+// Acceptance of the draft token x (Algorithm 4): a = 1 when delta = 0 or
+// q(x) <= pi(x), else a = [u < pi(x)/q(x)].  log2 p(x) - log2 q(x) is formed in
+// f64 from the logits, so the ratio carries only the f32 error of S_q / S_p.
+// q(x) and pi(x) themselves are evaluated only for the diagnostics output.
+__device__ __forceinline__ void accept_test(Shared &sh, float yqx, float ypx, float u, double kd,
+                                            bool want_probs) {
+  const double lq = static_cast<double>(yqx) * kd - static_cast<double>(sh.Rq);  // log2 q(x) + log2 S_q
+  const double lp = static_cast<double>(ypx) * kd - static_cast<double>(sh.Rp);
   int accept = 1;
   if (sh.delta) {
-    const double L = (dp - dq) * invT + static_cast<double>(logf(sh.Sq / sh.Sp));
-    if (L < 0.0) accept = u < exp_split(L);
+    const double L = lp - lq + static_cast<double>(log2f(sh.Sq / sh.Sp));
+    if (L < 0.0) accept = u < exp2_split(L);
   }
   sh.accept = accept;
-  sh.qx = qx;
-  sh.pix = sh.delta ? px : qx;
-  sh.need_sample = !accept;
+  if (want_probs) {
+    const float qx = exp2_split(lq - static_cast<double>(log2f(sh.Sq)));
+    const float px = exp2_split(lp - static_cast<double>(log2f(sh.Sp)));
+    sh.qx = qx;
+    sh.pix = sh.delta ? px : qx;
+  }
+}
+
+// ------------------------------------------------------------------ chunk ring
+
+template <typename E>
+struct Ring {
+  E *base;        // kStages stages of [2][kCH] logits (q then p)
+  const E *gq;    // slice start in global memory
+  const E *gp;
+  int len;        // valid logits in the slice
+  int nch;        // chunks in the slice
+  bool pair;
+  bool bulk;
+  __device__ E *q(int s) const { return base + static_cast<size_t>(s) * 2 * kCH; }
+  __device__ E *p(int s) const { return q(s) + kCH; }
+  __device__ int chunk_len(int c) const { return min(kCH, len - c * kCH); }
+  // thread 0, bulk mode: start the copies of chunk c into stage s
+  __device__ void issue(Shared &sh, int c, int s) const {
+    const uint32_t bytes = static_cast<uint32_t>(chunk_len(c)) * sizeof(E);
+    mbar_expect_tx(&sh.full[s], pair ? 2 * bytes : bytes);
+    if (pair) bulk_g2s(q(s), gq + static_cast<size_t>(c) * kCH, bytes, &sh.full[s]);
+    bulk_g2s(p(s), gp + static_cast<size_t>(c) * kCH, bytes, &sh.full[s]);
+  }
+  // all threads, per-thread mode: copy chunk c into stage s
+  __device__ void load_sync(int c, int s) const {
+    const int n = chunk_len(c);
+    const size_t o = static_cast<size_t>(c) * kCH;
+    for (int i = threadIdx.x; i < n; i += kNT) {
+      if (pair) q(s)[i] = gq[o + i];
+      p(s)[i] = gp[o + i];
+    }
+  }
+};
+
+// Stream every chunk of the slice through the ring and call body(c, stage) on
+// each.  `fills` counts stage fills since the kernel started (it fixes each
+// stage's mbarrier phase); the first kStages fills of this pass must already
+// be issued when bulk (see prime()).
+template <typename E, typename Body>
+__device__ __forceinline__ int stream(const Ring<E> &R, Shared &sh, int &fills, Body &&body) {
+  int tmo = 0;
+  for (int c = 0; c < R.nch; ++c) {
+    const int f = fills + c, s = f % kStages;
+    if (R.bulk) {
+      if (!mbar_wait(&sh.full[s], (f / kStages) & 1)) tmo = 1;
+    } else {
+      R.load_sync(c, s);
+      __syncthreads();
+    }
+    body(c, s);
+    __syncthreads();  // every thread is done with stage s
+    if (R.bulk && threadIdx.x == 0 && c + kStages < R.nch) R.issue(sh, c + kStages, s);
+  }
+  fills += R.nch;
+  return tmo;
+}
+
+template <typename E>
+__device__ __forceinline__ void prime(const Ring<E> &R, Shared &sh, int fills) {
+  if (R.bulk && threadIdx.x == 0)
+    for (int c = 0; c < min(kStages, R.nch); ++c) R.issue(sh, c, (fills + c) % kStages);
 }
 
 // ------------------------------------------------------------------ the kernel
 
 template <typename E>
-__global__ void __launch_bounds__(kNT, 3) sc_unit_kernel(const Params P) {
+__global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Params P) {
   extern __shared__ __align__(128) unsigned char smem_raw[];
   cg::cluster_group cluster = cg::this_cluster();
   const int C = P.cluster;
@@ -424,10 +452,11 @@ __global__ void __launch_bounds__(kNT, 3) sc_unit_kernel(const Params P) {
   const int unit = static_cast<int>(blockIdx.x) / C;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int G1 = P.gamma + 1;
+  const bool verify = P.mode == kVerify;
 
   int b, j;
   bool pair;
-  if (P.mode == kVerify) {
+  if (verify) {
     b = unit / G1;
     j = unit % G1;
     pair = j < P.gamma;
@@ -438,72 +467,59 @@ __global__ void __launch_bounds__(kNT, 3) sc_unit_kernel(const Params P) {
   }
   const size_t qoff = (static_cast<size_t>(b) * P.gamma + j) * P.V;
   const size_t poff = (static_cast<size_t>(b) * G1 + j) * P.V;
-  const E *gq = static_cast<const E *>(P.draft) + qoff;
-  const E *gp = static_cast<const E *>(P.target) + poff;
   const int v0 = rank * P.L;
   const int len = max(0, min(P.L, P.V - v0));
-  const int lenp = (len + 7) & ~7;
-  const int nv = lenp >> 3;
-  const int nchunks = (len + kChunkElems - 1) / kChunkElems;
 
-  E *sq = reinterpret_cast<E *>(smem_raw);
-  E *sp = sq + P.L;
-  Shared &sh = *reinterpret_cast<Shared *>(
-      smem_raw + ((2 * static_cast<size_t>(P.L) * sizeof(E) + 15) & ~size_t(15)));
+  Ring<E> R;
+  R.base = reinterpret_cast<E *>(smem_raw);
+  R.gq = static_cast<const E *>(P.draft) + qoff + v0;
+  R.gp = static_cast<const E *>(P.target) + poff + v0;
+  R.len = len;
+  R.nch = (len + kCH - 1) / kCH;
+  R.pair = pair;
+  R.bulk = P.bulk != 0;
+  Shared &sh = *reinterpret_cast<Shared *>(smem_raw + static_cast<size_t>(kStages) * 2 * kCH * sizeof(E));
 
-  // ---- stage the slices; thread 0 then prefetches the row's scalars
-  float uj = 0.0f, ug = 0.0f, yqx = 0.0f, ypx = 0.0f;
-  int x = 0;
+  // ---- start the stream; prefetch the row's scalars
   if (tid == 0) {
-    sh.cand = -1;
     sh.timeout = 0;
-    if (P.bulk) {
-      for (int c = 0; c < nchunks; ++c) mbar_init(&sh.bar[c], 1);
+    sh.xq = NAN;
+    sh.xp = NAN;
+    if (R.bulk) {
+      for (int s = 0; s < kStages; ++s) mbar_init(&sh.full[s], 1);
       asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      for (int c = 0; c < nchunks; ++c) {
-        const int e0 = c * kChunkElems, e1 = min(len, e0 + kChunkElems);
-        const uint32_t bytes = static_cast<uint32_t>(e1 - e0) * sizeof(E);
-        mbar_expect_tx(&sh.bar[c], pair ? 2 * bytes : bytes);
-        if (pair) bulk_g2s(sq + e0, gq + v0 + e0, bytes, &sh.bar[c]);
-        bulk_g2s(sp + e0, gp + v0 + e0, bytes, &sh.bar[c]);
-      }
-    }
-    if (P.mode == kVerify) {
-      uj = P.uniforms[static_cast<size_t>(b) * G1 + j];
-      ug = P.uniforms[static_cast<size_t>(b) * G1 + P.gamma];
-      if (pair) {
-        x = P.tokens[static_cast<size_t>(b) * P.gamma + j];
-        if (x >= 0 && x < P.V) {
-          yqx = Elt<E>::at(P.draft, qoff + x);
-          ypx = Elt<E>::at(P.target, poff + x);
-        }
-      }
     }
   }
-  if (!P.bulk) {
-    for (int i = tid; i < len; i += kNT) {
-      if (pair) sq[i] = gq[v0 + i];
-      sp[i] = gp[v0 + i];
-    }
-  }
-  for (int i = len + tid; i < lenp; i += kNT) {  // -inf padding: weight 0 everywhere
-    sq[i] = Elt<E>::kNegInf;
-    sp[i] = Elt<E>::kNegInf;
+  int fills = 0;
+  prime(R, sh, fills);
+  float uj = 0.0f, ug = 0.0f;
+  int x = -1;
+  if (verify && tid == 0) {
+    uj = P.uniforms[static_cast<size_t>(b) * G1 + j];
+    ug = P.uniforms[static_cast<size_t>(b) * G1 + P.gamma];
+    if (pair) x = P.tokens[static_cast<size_t>(b) * P.gamma + j];
   }
   __syncthreads();
 
-  // ---- pass 1: online max and sum of exponentials while the chunks land
+  // ---- pass 1: online max and sum of exponentials
   const float k = P.k;
   float mq = -FLT_MAX, s_q = 0.0f, mp = -FLT_MAX, s_p = 0.0f;
-  int tmo = 0;
-  const int nchunk_loop = P.bulk ? nchunks : (nv + kVecPerChunk - 1) / kVecPerChunk;
-  for (int c = 0; c < nchunk_loop; ++c) {
-    if (P.bulk && !mbar_wait(&sh.bar[c], 0)) tmo = 1;
-    const int vbeg = c * kVecPerChunk, vend = min(nv, vbeg + kVecPerChunk);
-    if (pair) online_chunk<E>(sq, vbeg, vend, k, mq, s_q);
-    online_chunk<E>(sp, vbeg, vend, k, mp, s_p);
-  }
+  const int lx = x - v0;  // draft token's offset in this slice (thread 0 only)
+  int tmo = stream(R, sh, fills, [&](int c, int s) {
+    const int n = R.chunk_len(c);
+    if (n == kCH) {
+      if (pair) online_row<E, true>(R.q(s), n, k, mq, s_q);
+      online_row<E, true>(R.p(s), n, k, mp, s_p);
+    } else {
+      if (pair) online_row<E, false>(R.q(s), n, k, mq, s_q);
+      online_row<E, false>(R.p(s), n, k, mp, s_p);
+    }
+    if (tid == 0 && static_cast<unsigned>(lx - c * kCH) < static_cast<unsigned>(n)) {
+      sh.xq = Elt<E>::at(R.q(s), lx - c * kCH);
+      sh.xp = Elt<E>::at(R.p(s), lx - c * kCH);
+    }
+  });
   tmo = __syncthreads_or(tmo);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
@@ -530,12 +546,17 @@ __global__ void __launch_bounds__(kNT, 3) sc_unit_kernel(const Params P) {
       if (P.status) atomicOr(P.status, static_cast<int32_t>(SC_DEV_TIMEOUT));
     }
     sh.part_ms = make_float4(a, as, c, cs);
+    sh.part_x = make_float2(sh.xq, sh.xp);
   }
-  cluster.sync();  // #1: partials published
+  cluster.sync();  // exchange 1
 
   if (warp == 0) {
     float4 v = make_float4(-FLT_MAX, 0.0f, -FLT_MAX, 0.0f);
-    if (lane < C) v = *cluster.map_shared_rank(&sh.part_ms, lane);
+    float2 xv = make_float2(NAN, NAN);
+    if (lane < C) {
+      v = *cluster.map_shared_rank(&sh.part_ms, lane);
+      xv = *cluster.map_shared_rank(&sh.part_x, lane);
+    }
     float a = v.x, as = v.y, c = v.z, cs = v.w;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
@@ -544,119 +565,242 @@ __global__ void __launch_bounds__(kNT, 3) sc_unit_kernel(const Params P) {
       ms_combine(a, as, a2, as2, k);
       ms_combine(c, cs, c2, cs2, k);
     }
-    if (lane == 0) {  // thread 0: it holds the prefetched scalars
+    const int xl = __shfl_sync(0xFFFFFFFFu, x, 0);
+    const int xr = (xl >= 0 && xl < P.V) ? xl / P.L : 0;
+    const float yqx = __shfl_sync(0xFFFFFFFFu, xv.x, xr);
+    const float ypx = __shfl_sync(0xFFFFFFFFu, xv.y, xr);
+    if (lane == 0) {  // thread 0: holds the prefetched scalars
+      // S = sum_v 2^{y_v k - R} with R = fl(M k); the max logit's own term is
+      // 2^{fma(M, k, -R)}, so max_v q(v) = 2^{fma(M, k, -R)} / S.
+      const float Rq = refk(a, k), Rp = refk(c, k);
       sh.Mq = a; sh.Sq = as; sh.Mp = c; sh.Sp = cs;
+      sh.Rq = Rq;
+      sh.Rp = Rp;
+      sh.maxq = ex2(fmaf(a, k, -Rq)) / as;
+      sh.maxp = ex2(fmaf(c, k, -Rp)) / cs;
       int err = 0;
       const bool okq = !pair || (isfinite(a) && isfinite(as) && as > 0.0f);
       const bool okp = isfinite(c) && isfinite(cs) && cs > 0.0f;
       if (!(okq && okp)) err |= SC_DEV_BAD_LOGIT;
-      if (P.mode == kVerify) {
+      if (verify) {
         if (!(uj >= 0.0f && uj < 1.0f)) err |= SC_DEV_BAD_UNIFORM;
         if (pair && (x < 0 || x >= P.V)) err |= SC_DEV_BAD_TOKEN;
       }
-      if (err && P.status) atomicOr(P.status, err);
+      if (err && P.status && rank == 0) atomicOr(P.status, err);
       sh.err = err;
       sh.delta = 0;
-      sh.need_tv = 0;
-      sh.need_sample = 0;
+      sh.need_p2 = 0;
+      sh.sample = 0;
       sh.accept = 0;
       sh.tv = -1.0f;
       sh.qx = 0.0f;
       sh.pix = 0.0f;
-      sh.c = pair && !err ? log2f(as / cs) : 0.0f;
       sh.ug = ug;
+      sh.c = pair && !err ? log2f(as / cs) : 0.0f;
       if (!err) {
         if (!pair) {
-          sh.need_sample = P.mode == kVerify;  // bonus row: drawn speculatively
-        } else if (P.mode == kStats) {
-          sh.need_tv = 1;
+          sh.need_p2 = verify;  // bonus row: drawn speculatively, used when j* = gamma
+          sh.sample = verify;
+        } else if (!verify) {
+          sh.need_p2 = 1;       // sc_row_stats: TV of every pair
         } else {
-          // deferral rule (Table 1); max q = 1/S_q, max p = 1/S_p
-          const float maxq = 1.0f / as, maxp = 1.0f / cs, al = P.alpha;
+          // deferral rule (Table 1)
+          const float maxq = sh.maxq, maxp = sh.maxp, al = P.alpha;
+          bool pending = false;
           switch (P.rule) {
             case SC_RULE_CHOW: sh.delta = maxq < 1.0f - al; break;  // Eq. 2
             case SC_RULE_DIFF: sh.delta = maxq < maxp - al; break;  // Eq. 5
             case SC_RULE_OPT:                                       // Eq. 10
-              // alpha * TV lies in [0, alpha]: the TV term decides only inside that band
+              // alpha * TV lies in [0, alpha]: TV decides only inside that band
               if (!(maxq < maxp)) sh.delta = 0;
               else if (maxq < maxp - al) sh.delta = 1;
-              else sh.need_tv = 1;
+              else pending = true;
               break;
             case SC_RULE_ALWAYS_DEFER: sh.delta = 1; break;
             default: sh.delta = 0; break;
           }
-          if (!sh.need_tv) accept_test(sh, yqx, ypx, uj, P.inv_t);
+          if (pending) {
+            sh.need_p2 = 1;
+          } else {
+            accept_test(sh, yqx, ypx, uj, P.kd, P.row_info != nullptr);
+            sh.need_p2 = !sh.accept;
+            sh.sample = !sh.accept;
+          }
         }
       }
+      // keep the draft-token logits for a decision after pass 2
+      sh.xq = yqx;
+      sh.xp = ypx;
+      sh.publisher = 0;
+      sh.cross_seg = -2;
     }
   }
   __syncthreads();
-  const RowScalars rs = {sh.Mq, sh.Mp, k, sh.c};
+  const RowScalars rs = {sh.Rq, sh.Rp, k, sh.c};
+  if (sh.need_p2) {
+    prime(R, sh, fills);  // the ring is free: restart the stream (L2-resident by now)
+  } else {
+    cluster_arrive();  // no further reads of peer shared memory
+  }
 
-  // ---- TV pass (shared memory only): sum_v min(p_v, q_v) = (1/S_q) sum_v 2^min(a_v, b_v + c)
-  if (sh.need_tv) {
-    float acc = 0.0f;
-    for (int v = tid; v < nv; v += kNT) {
-      float yq[8], yp[8];
-      Elt<E>::load8(sq + 8 * v, yq);
-      Elt<E>::load8(sp + 8 * v, yp);
-#pragma unroll
-      for (int e = 0; e < 8; ++e)
-        acc += ex2(fminf((yq[e] - rs.Mq) * k, fmaf(yp[e] - rs.Mp, k, rs.c)));
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) acc += __shfl_down_sync(0xFFFFFFFFu, acc, o);
-    if (lane == 0) sh.red[warp][0] = acc;
-    __syncthreads();
+  // ---- pass 2: residual weights and their per-segment totals
+  if (sh.need_p2) {
+    const int nseg = R.nch * kRounds * kNW;
+    tmo = stream(R, sh, fills, [&](int c, int s) {
+      const int n = R.chunk_len(c);
+      if (pair) {
+        if (n == kCH) weights_chunk<E, true, true>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
+        else weights_chunk<E, true, false>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
+      } else {
+        if (n == kCH) weights_chunk<E, false, true>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
+        else weights_chunk<E, false, false>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
+      }
+    });
+    tmo = __syncthreads_or(tmo);
     if (tid == 0) {
-      float t = 0.0f;
-      for (int w = 0; w < kNW; ++w) t += sh.red[w][0];
-      sh.part_tv = t;
+      float acc = 0.0f;  // exclusive prefixes in vocabulary order (chunk, round, warp)
+      for (int i = 0; i < nseg; ++i) {
+        const float t = sh.seg[i];
+        sh.seg[i] = acc;
+        acc = __fadd_rn(acc, t);
+      }
+      sh.seg[nseg] = acc;
+      if (tmo) {
+        acc = NAN;
+        sh.timeout = 1;
+        if (P.status) atomicOr(P.status, static_cast<int32_t>(SC_DEV_TIMEOUT));
+      }
+      sh.part_r = acc;
     }
-    cluster.sync();  // #2
+    cluster.sync();  // exchange 2
+
     if (warp == 0) {
-      float t = 0.0f;
-      if (lane < C) t = *cluster.map_shared_rank(&sh.part_tv, lane);
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) t += __shfl_down_sync(0xFFFFFFFFu, t, o);
+      float tot = 0.0f;
+      if (lane < C) tot = *cluster.map_shared_rank(&sh.part_r, lane);
+      const float pre = warp_incl_scan(tot, lane);  // through rank `lane`
+      const float Rtot = __shfl_sync(0xFFFFFFFFu, pre, C - 1);
+      float before = __shfl_up_sync(0xFFFFFFFFu, pre, 1);
+      if (lane == 0) before = 0.0f;
       if (lane == 0) {
-        const float tv = fminf(1.0f, fmaxf(0.0f, 1.0f - t / sh.Sq));  // Lemma 3
-        sh.tv = tv;
-        if (P.mode == kVerify) {
-          sh.delta = 1.0f / sh.Sq < 1.0f / sh.Sp - P.alpha * tv;  // Eq. 10
-          accept_test(sh, yqx, ypx, uj, P.inv_t);
+        if (!isfinite(Rtot)) {
+          sh.err |= SC_DEV_TIMEOUT;
+          sh.sample = 0;
+        } else if (pair) {
+          sh.tv = fminf(1.0f, fmaxf(0.0f, Rtot / sh.Sq));  // Lemma 3: R = S_q D_TV(p, q)
+        }
+        if (isfinite(Rtot) && pair && !sh.sample) {
+          // TV was needed to decide: sc_row_stats, or the OPT band
+          if (verify) {
+            sh.delta = sh.maxq < sh.maxp - P.alpha * sh.tv;  // Eq. 10
+            accept_test(sh, sh.xq, sh.xp, uj, P.kd, P.row_info != nullptr);
+            sh.sample = !sh.accept;
+          }
+        }
+      }
+      const int sample = __shfl_sync(0xFFFFFFFFu, sh.sample, 0);
+      if (sample && Rtot > 0.0f) {
+        const double t = static_cast<double>(sh.ug) * static_cast<double>(Rtot);
+        const bool cross = lane < C && tot > 0.0f && t >= static_cast<double>(before) &&
+                           t < static_cast<double>(pre);
+        const unsigned cm = __ballot_sync(0xFFFFFFFFu, cross);
+        const unsigned pm = __ballot_sync(0xFFFFFFFFu, lane < C && tot > 0.0f);
+        const int cr = cm ? __ffs(cm) - 1 : 31 - __clz(pm);
+        const float bcr = __shfl_sync(0xFFFFFFFFu, before, cr);
+        if (lane == 0) {
+          sh.publisher = cr;
+          if (cr == rank) {
+            // the segment of this CTA that holds t (or, past a rounding gap, none)
+            const double tl = cm ? t - static_cast<double>(bcr) : -1.0;
+            int sgi = -1;
+            if (cm)
+              for (int i = 0; i < nseg; ++i)
+                if (tl >= static_cast<double>(sh.seg[i]) && tl < static_cast<double>(sh.seg[i + 1]) &&
+                    sh.seg[i + 1] > sh.seg[i]) {
+                  sgi = i;
+                  break;
+                }
+            sh.cross_seg = sgi;
+            sh.t_seg = sgi >= 0 ? __double2float_rd(tl - static_cast<double>(sh.seg[sgi])) : 0.0f;
+          }
         }
       }
     }
+    cluster_arrive();  // no further reads of peer shared memory
     __syncthreads();
-  }
 
-  if (sh.need_sample) {
-    const float u = sh.ug;  // thread 0 prefetched it
-    if (pair) sample_unit<E, true>(sq, sp, nv, v0, sh, rs, u, cluster, rank, C);
-    else sample_unit<E, false>(sq, sp, nv, v0, sh, rs, u, cluster, rank, C);
+    // ---- search (only in the publishing CTA)
+    if (sh.sample && sh.publisher == rank && sh.cross_seg != -2) {
+      int sgi = sh.cross_seg;
+      if (sgi < 0) {
+        // rounding left u R past the last boundary: take the last segment with weight
+        for (int i = nseg - 1; i >= 0; --i)
+          if (sh.seg[i + 1] > sh.seg[i]) { sgi = i; break; }
+      }
+      const int sw = sgi >= 0 ? sgi % kNW : -1;
+      if (warp == sw) {
+        const int r = (sgi / kNW) % kRounds, c = sgi / (kNW * kRounds);
+        const int n = R.chunk_len(c);
+        const int e = 8 * (r * kNT + tid);
+        float yq[8], yp[8], w[8];
+        const E *gq = R.gq + static_cast<size_t>(c) * kCH;
+        const E *gp = R.gp + static_cast<size_t>(c) * kCH;
+        if (pair) load8_gmem(gq, e, n, R.bulk, yq);
+        load8_gmem(gp, e, n, R.bulk, yp);
+        const float vs = pair ? vec_weights<true>(yq, yp, rs, w) : vec_weights<false>(yq, yp, rs, w);
+        const float incl = warp_incl_scan(vs, lane);
+        float excl = __shfl_up_sync(0xFFFFFFFFu, incl, 1);
+        if (lane == 0) excl = 0.0f;
+        const float t = sh.cross_seg >= 0 ? sh.t_seg : FLT_MAX;
+        int tok = -1;
+        const bool mine = t >= excl && t < incl && vs > 0.0f;
+        const unsigned mm = __ballot_sync(0xFFFFFFFFu, mine);
+        if (mm) {
+          if (lane == __ffs(mm) - 1) {
+            const float tt = __fsub_rn(t, excl);
+            float acc = 0.0f;
+            int last = -1;
+            for (int i = 0; i < 8; ++i) {
+              acc = __fadd_rn(acc, w[i]);
+              if (w[i] > 0.0f) last = i;
+              if (tok < 0 && acc > tt) tok = i;
+            }
+            if (tok < 0) tok = last;
+            tok = v0 + c * kCH + e + tok;
+          }
+          tok = __shfl_sync(0xFFFFFFFFu, tok, __ffs(mm) - 1);
+        } else {
+          // last positive weight of the segment
+          int last = -1;
+          for (int i = 0; i < 8; ++i)
+            if (w[i] > 0.0f) last = i;
+          const unsigned lm = __ballot_sync(0xFFFFFFFFu, last >= 0);
+          if (lm) {
+            const int ln = 31 - __clz(lm);
+            const int li = __shfl_sync(0xFFFFFFFFu, last, ln);
+            tok = v0 + c * kCH + 8 * (r * kNT + warp * 32 + ln) + li;
+          }
+        }
+        if (lane == 0) sh.cross_seg = tok;  // reused: the sampled token
+      }
+      __syncthreads();
+    }
   }
-  if (sh.timeout && tid == 0 && P.bulk) {
-    // let copies still in flight land before this CTA's shared memory is released
-    for (int c = 0; c < nchunks; ++c) mbar_wait(&sh.bar[c], 0);
-  }
-  cluster.sync();  // candidate visible in rank 0; no peer reads this CTA's shared memory after
 
   // ---- publish this unit; the last unit of the sequence finishes it
-  if (rank == 0 && tid == 0) {
-    if (P.mode == kStats) {
+  if (tid == 0 && rank == sh.publisher) {
+    if (!verify) {
       const size_t r = static_cast<size_t>(b) * P.gamma + j;
       const bool bad = sh.err != 0;
-      P.max_q[r] = bad ? NAN : 1.0f / sh.Sq;
-      P.max_p[r] = bad ? NAN : 1.0f / sh.Sp;
+      P.max_q[r] = bad ? NAN : sh.maxq;
+      P.max_p[r] = bad ? NAN : sh.maxp;
       P.tv[r] = bad ? NAN : sh.tv;
     } else {
       const size_t r = static_cast<size_t>(b) * G1 + j;
-      const int cand = sh.need_sample ? sh.cand : -1;
+      const int cand = sh.sample && sh.need_p2 && sh.cross_seg >= 0 ? sh.cross_seg : -1;
       if (P.row_info) {
         float *ri = P.row_info + r * SC_ROW_FIELDS;
-        ri[SC_ROW_MAXQ] = pair && !sh.err ? 1.0f / sh.Sq : NAN;
-        ri[SC_ROW_MAXP] = !sh.err ? 1.0f / sh.Sp : NAN;
+        ri[SC_ROW_MAXQ] = pair && !sh.err ? sh.maxq : NAN;
+        ri[SC_ROW_MAXP] = !sh.err ? sh.maxp : NAN;
         ri[SC_ROW_TV] = sh.tv;
         ri[SC_ROW_DELTA] = static_cast<float>(sh.delta);
         ri[SC_ROW_ACCEPT] = static_cast<float>(sh.accept);
@@ -686,6 +830,11 @@ __global__ void __launch_bounds__(kNT, 3) sc_unit_kernel(const Params P) {
       }
     }
   }
+  if (sh.timeout && tid == 0 && R.bulk) {
+    // let copies still in flight land before this CTA's shared memory is released
+    for (int s = 0; s < kStages; ++s) mbar_wait(&sh.full[s], 0), mbar_wait(&sh.full[s], 1);
+  }
+  cluster_wait();  // peers are done reading this CTA's shared memory
 }
 
 // ------------------------------------------------------------------ host side
@@ -701,27 +850,27 @@ std::mutex g_mu;
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 template <typename E>
-size_t smem_bytes(int L) {
-  return align_up(2 * static_cast<size_t>(L) * sizeof(E), 16) + sizeof(Shared);
+size_t smem_bytes() {
+  return static_cast<size_t>(kStages) * 2 * kCH * sizeof(E) + sizeof(Shared);
 }
 
-// Slice length L (multiple of 8) and cluster size C for a row of V elements.
-template <typename E>
-int pick_layout(int V, int smem_optin, int *C_out, int *L_out) {
-  const size_t row_bytes = static_cast<size_t>(V) * sizeof(E);
-  size_t target = 32768;  // bytes per row per CTA: 64 KB of staging per CTA for a pair
-  if (const char *s = getenv("SC_SLICE_BYTES")) {
+// Cluster size C and slice length L (multiple of 8) for a row of V logits.
+int pick_layout(int V, int *C_out, int *L_out) {
+  long target = 16384;  // logits per row per CTA
+  if (const char *s = getenv("SC_SLICE")) {
     const long t = atol(s);
-    if (t >= 1024) target = static_cast<size_t>(t);
+    if (t >= 64) target = t;
   }
-  int C = static_cast<int>((row_bytes + target - 1) / target);
-  C = C < 1 ? 1 : C;
+  int C = static_cast<int>((V + target - 1) / target);
+  if (const char *s = getenv("SC_CLUSTER")) {
+    const int c = atoi(s);
+    if (c >= 1 && c <= kMaxCluster) C = c;
+  }
+  C = std::max(1, std::min(C, kMaxCluster));
   for (; C <= kMaxCluster; ++C) {
-    int L = static_cast<int>(align_up((static_cast<size_t>(V) + C - 1) / C, 8));
-    const int Ceff = (V + L - 1) / L;
-    if ((L + kChunkElems - 1) / kChunkElems > kMaxChunks) continue;
-    if (smem_bytes<E>(L) > static_cast<size_t>(smem_optin)) continue;
-    *C_out = Ceff;
+    const int L = static_cast<int>(align_up((static_cast<size_t>(V) + C - 1) / C, 8));
+    if ((L + kCH - 1) / kCH > kMaxChunks) continue;
+    *C_out = (V + L - 1) / L;
     *L_out = L;
     return 0;
   }
@@ -751,7 +900,7 @@ int launch(Params P, cudaStream_t stream, int units) {
       return SC_ERR_CUDA;
     if (!di.configured[ti]) {
       if (cudaFuncSetAttribute(sc_unit_kernel<E>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               di.smem_optin) != cudaSuccess ||
+                               static_cast<int>(smem_bytes<E>())) != cudaSuccess ||
           cudaFuncSetAttribute(sc_unit_kernel<E>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
               cudaSuccess)
         return SC_ERR_CUDA;
@@ -759,18 +908,7 @@ int launch(Params P, cudaStream_t stream, int units) {
     }
   }
   int C = 1, L = 8;
-  if (pick_layout<E>(P.V, di.smem_optin, &C, &L) != 0) return SC_ERR_UNSUPPORTED;
-  if (const char *s = getenv("SC_CLUSTER")) {  // tuning override (must still fit)
-    const int c = atoi(s);
-    if (c >= 1 && c <= kMaxCluster) {
-      const int Lc = static_cast<int>(align_up((static_cast<size_t>(P.V) + c - 1) / c, 8));
-      if (smem_bytes<E>(Lc) <= static_cast<size_t>(di.smem_optin) &&
-          (Lc + kChunkElems - 1) / kChunkElems <= kMaxChunks) {
-        L = Lc;
-        C = (P.V + L - 1) / L;
-      }
-    }
-  }
+  if (pick_layout(P.V, &C, &L) != 0) return SC_ERR_UNSUPPORTED;
   P.L = L;
   P.cluster = C;
   const size_t row_bytes = static_cast<size_t>(P.V) * sizeof(E);
@@ -781,7 +919,7 @@ int launch(Params P, cudaStream_t stream, int units) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(units) * static_cast<unsigned>(C), 1, 1);
   cfg.blockDim = dim3(kNT, 1, 1);
-  cfg.dynamicSmemBytes = smem_bytes<E>(L);
+  cfg.dynamicSmemBytes = smem_bytes<E>();
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -824,11 +962,8 @@ int sc_workspace_init(void *workspace, size_t workspace_bytes, cudaStream_t stre
 }
 
 int sc_max_vocab(sc_dtype dtype) {
-  // one cluster of kMaxCluster CTAs, each staging both rows of its slice
-  const size_t budget = 227 * 1024 - sizeof(Shared) - 64;
-  const size_t elt = dtype == SC_F32 ? 4 : 2;
-  const size_t per_cta = std::min(budget / (2 * elt), static_cast<size_t>(kMaxChunks) * kChunkElems) & ~size_t(7);
-  return static_cast<int>(per_cta * kMaxCluster);
+  (void)dtype;  // the ring does not depend on V: one cluster covers kMaxCluster slices
+  return kMaxCluster * kMaxChunks * kCH;
 }
 
 int sc_verify_rows(const void *draft_logits, const void *target_logits, sc_dtype dtype,
@@ -860,7 +995,7 @@ int sc_verify_rows(const void *draft_logits, const void *target_logits, sc_dtype
   P.alpha = alpha;
   P.temperature = temperature;
   P.k = static_cast<float>(1.4426950408889634 / static_cast<double>(temperature));
-  P.inv_t = 1.0 / static_cast<double>(temperature);
+  P.kd = 1.4426950408889634 / static_cast<double>(temperature);
   P.mode = kVerify;
   P.num_accepted = num_accepted;
   P.next_token = next_token;
@@ -868,9 +1003,10 @@ int sc_verify_rows(const void *draft_logits, const void *target_logits, sc_dtype
   P.status = device_status;
   unsigned char *ws = static_cast<unsigned char *>(workspace);
   const size_t n = static_cast<size_t>(B) * (gamma + 1);
+  const size_t off1 = align_up(4 * static_cast<size_t>(B), 256);
   P.tickets = reinterpret_cast<uint32_t *>(ws);
-  P.unit_flags = reinterpret_cast<int32_t *>(ws + align_up(4 * static_cast<size_t>(B), 256));
-  P.unit_cand = reinterpret_cast<int32_t *>(ws + align_up(4 * static_cast<size_t>(B), 256) + align_up(4 * n, 256));
+  P.unit_flags = reinterpret_cast<int32_t *>(ws + off1);
+  P.unit_cand = reinterpret_cast<int32_t *>(ws + off1 + align_up(4 * n, 256));
   const int units = B * (gamma + 1);
   return dtype == SC_BF16 ? launch<uint16_t>(P, stream, units) : launch<float>(P, stream, units);
 }
@@ -900,7 +1036,7 @@ int sc_row_stats(const void *draft_logits, const void *target_logits, sc_dtype d
   P.V = V;
   P.temperature = temperature;
   P.k = static_cast<float>(1.4426950408889634 / static_cast<double>(temperature));
-  P.inv_t = 1.0 / static_cast<double>(temperature);
+  P.kd = 1.4426950408889634 / static_cast<double>(temperature);
   P.mode = kStats;
   P.max_q = max_q;
   P.max_p = max_p;
