@@ -841,6 +841,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
 
 struct DeviceInfo {
   int smem_optin = 0;
+  int sms = 0;
   bool configured[2] = {false, false};
 };
 
@@ -855,8 +856,11 @@ size_t smem_bytes() {
 }
 
 // Cluster size C and slice length L (multiple of 8) for a row of V logits.
-int pick_layout(int V, int *C_out, int *L_out) {
-  long target = 16384;  // logits per row per CTA
+// Long slices amortise each unit's two cluster exchanges over more streamed
+// bytes; short ones give small batches enough CTAs to cover the GPU.
+int pick_layout(int V, int units, int sms, int *C_out, int *L_out) {
+  long target = 32768;  // logits per row per CTA
+  if (static_cast<long>(units) * ((V + target - 1) / target) < 4L * sms) target = 8192;
   if (const char *s = getenv("SC_SLICE")) {
     const long t = atol(s);
     if (t >= 64) target = t;
@@ -896,7 +900,8 @@ int launch(Params P, cudaStream_t stream, int units) {
   {
     std::lock_guard<std::mutex> lock(g_mu);
     if (!di.smem_optin &&
-        cudaDeviceGetAttribute(&di.smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+        (cudaDeviceGetAttribute(&di.smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
+         cudaDeviceGetAttribute(&di.sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess))
       return SC_ERR_CUDA;
     if (!di.configured[ti]) {
       if (cudaFuncSetAttribute(sc_unit_kernel<E>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -908,7 +913,7 @@ int launch(Params P, cudaStream_t stream, int units) {
     }
   }
   int C = 1, L = 8;
-  if (pick_layout(P.V, &C, &L) != 0) return SC_ERR_UNSUPPORTED;
+  if (pick_layout(P.V, units, di.sms, &C, &L) != 0) return SC_ERR_UNSUPPORTED;
   P.L = L;
   P.cluster = C;
   const size_t row_bytes = static_cast<size_t>(P.V) * sizeof(E);
