@@ -52,7 +52,8 @@ typedef enum {
   SC_ERR_INVALID_ARG = -1, /* a size, rule, alpha, T or pointer is out of its domain */
   SC_ERR_CUDA = -2,        /* the launch failed; cudaGetLastError() has the cause */
   SC_ERR_WORKSPACE = -3,   /* workspace missing or smaller than sc_workspace_bytes() */
-  SC_ERR_UNSUPPORTED = -4  /* V too large for one thread-block cluster per row */
+  SC_ERR_UNSUPPORTED = -4, /* V too large for one thread-block cluster per row */
+  SC_ERR_SCRATCH_LIMIT = -5 /* batch larger than sc_verify_static's built-in scratch */
 } sc_status;
 
 /* Bits of the optional device status word (OR-ed in, never cleared). */
@@ -135,6 +136,36 @@ int sc_row_stats(const void *draft_logits, const void *target_logits, sc_dtype d
 
 /* Static description of an sc_status code. */
 const char *sc_status_string(int code);
+
+/*
+ * sc_verify_static -- sc_verify for callers that cannot allocate device memory.
+ *
+ * The paper has no counterpart: this entry point exists for code that must not
+ * call cudaMalloc, e.g. an inference server whose device memory is carved up by
+ * its own allocator before the first request, or a caller running where a
+ * synchronising allocation would stall other streams.  Such callers still pass
+ * their inputs and outputs, but need no workspace: the sequence tickets, per-
+ * position flags and candidates live in a fixed array compiled into the library,
+ * one copy per device, held by every GPU that loads the library until exit.
+ *
+ * Limits: B <= SC_STATIC_MAX_B and B * (gamma + 1) <= SC_STATIC_MAX_UNITS
+ * (48 KiB of scratch); larger batches return SC_ERR_SCRATCH_LIMIT and queue no
+ * work.  Other arguments are those of sc_verify and are checked the same way.
+ *
+ * The first call on a device looks up the array's device address (the library's
+ * module is loaded then); make that first call before any stream capture.  Every
+ * call clears the tickets it uses on `stream` before launching.  All calls on a
+ * device share the one array and it keeps the last call's contents, so calls that
+ * may overlap on the GPU (different streams without ordering between them) race
+ * and must not be issued; order them on one stream or serialise them.  Nothing is
+ * allocated or freed by this call.
+ */
+#define SC_STATIC_MAX_B 4096
+#define SC_STATIC_MAX_UNITS 4096
+int sc_verify_static(const void *draft_logits, const void *target_logits, sc_dtype dtype,
+                     const int32_t *draft_tokens, const float *uniforms, int B, int gamma, int V,
+                     sc_rule rule, float alpha, float temperature, int32_t *num_accepted,
+                     int32_t *next_token, int32_t *device_status, cudaStream_t stream);
 
 #ifdef __cplusplus
 }

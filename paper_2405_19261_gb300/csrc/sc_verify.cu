@@ -948,6 +948,37 @@ int common_checks(const void *draft, const void *target, int dtype, int B, int g
   return SC_OK;
 }
 
+// ------------------------------------------------------------------ fixed scratch
+
+// Workspace of sc_verify_static: tickets [SC_STATIC_MAX_B] then unit flags and
+// candidates [SC_STATIC_MAX_UNITS] each, in sc_workspace_bytes' layout for the
+// largest accepted batch.  One copy per device, zeroed when the module loads.
+constexpr size_t kStaticScratchBytes =
+    ((4 * static_cast<size_t>(SC_STATIC_MAX_B) + 255) / 256) * 256 +
+    2 * (((4 * static_cast<size_t>(SC_STATIC_MAX_UNITS) + 255) / 256) * 256);
+static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
+
+void *g_static_ptr[64];
+std::mutex g_static_mu;
+
+// Device address of g_static_scratch on the current device, looked up once per
+// device.  The host-side name is only a stand-in and must never reach a kernel.
+int static_scratch(void **out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return SC_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  if (!g_static_ptr[dev]) {
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || !p) {
+      cudaGetLastError();
+      return SC_ERR_CUDA;
+    }
+    g_static_ptr[dev] = p;
+  }
+  *out = g_static_ptr[dev];
+  return SC_OK;
+}
+
 }  // namespace
 
 // ------------------------------------------------------------------ C ABI
@@ -1057,8 +1088,31 @@ const char *sc_status_string(int code) {
     case SC_ERR_CUDA: return "CUDA launch error";
     case SC_ERR_WORKSPACE: return "workspace missing or too small";
     case SC_ERR_UNSUPPORTED: return "vocabulary too large for one cluster per row";
+    case SC_ERR_SCRATCH_LIMIT: return "batch exceeds the fixed scratch of sc_verify_static";
     default: return "unknown status";
   }
+}
+
+// Same verification kernel, with its workspace in g_static_scratch instead of
+// caller memory.  No allocation: the tickets are cleared with a memset on the
+// caller's stream and sc_verify_rows runs on the fixed array.
+int sc_verify_static(const void *draft_logits, const void *target_logits, sc_dtype dtype,
+                     const int32_t *draft_tokens, const float *uniforms, int B, int gamma, int V,
+                     sc_rule rule, float alpha, float temperature, int32_t *num_accepted,
+                     int32_t *next_token, int32_t *device_status, cudaStream_t stream) {
+  if (B < 1 || gamma < 1) return SC_ERR_INVALID_ARG;
+  if (B > SC_STATIC_MAX_B || static_cast<long>(B) * (gamma + 1) > SC_STATIC_MAX_UNITS)
+    return SC_ERR_SCRATCH_LIMIT;
+  const size_t need = sc_workspace_bytes(B, gamma, V);
+  if (need > kStaticScratchBytes) return SC_ERR_SCRATCH_LIMIT;
+  void *ws = nullptr;
+  int rc = static_scratch(&ws);
+  if (rc != SC_OK) return rc;
+  // the previous call left the tickets at zero unless it was cut short: clear them
+  if (cudaMemsetAsync(ws, 0, 4 * static_cast<size_t>(B), stream) != cudaSuccess) return SC_ERR_CUDA;
+  return sc_verify_rows(draft_logits, target_logits, dtype, draft_tokens, uniforms, B, gamma, V,
+                        rule, alpha, temperature, num_accepted, next_token, ws, need,
+                        device_status, nullptr, stream);
 }
 
 }  // extern "C"
