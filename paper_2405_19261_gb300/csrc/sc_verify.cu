@@ -10,7 +10,7 @@
 //   grid   one thread-block cluster of C CTAs per unit; CTA r of the cluster
 //          owns the vocabulary slice [r L, (r+1) L) of both rows;
 //   pass 1 the slice streams from HBM through a two-stage shared-memory ring
-//          filled by TMA bulk copies (cp.async.bulk + mbarrier), 2048 logits
+//          filled by TMA bulk copies (cp.async.bulk + mbarrier), 4096 logits
 //          per row per stage; each thread keeps an online (max, sum of exp);
 //          the CTA partials are merged over the cluster through distributed
 //          shared memory, giving M and S of both rows, max q = 1/S_q and
@@ -33,6 +33,7 @@
 #include "sc.h"
 
 #include <cooperative_groups.h>
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -46,17 +47,28 @@ namespace cg = cooperative_groups;
 
 namespace {
 
+#ifndef SC_RING_STAGES
+#define SC_RING_STAGES 2
+#endif
+#ifndef SC_CHUNK
+#define SC_CHUNK 4096
+#endif
+#ifndef SC_MIN_BLOCKS
+#define SC_MIN_BLOCKS 6
+#endif
+
 constexpr int kNT = 128;                   // threads per CTA
 constexpr int kNW = kNT / 32;              // warps per CTA
-constexpr int kCH = 2048;                  // logits per row per ring stage
+constexpr int kCH = SC_CHUNK;              // logits per row per ring stage
 constexpr int kVPC = kCH / 8;              // 8-element vectors per chunk
 constexpr int kRounds = kVPC / kNT;        // vectors per thread per chunk
-constexpr int kStages = 2;                 // ring depth
-constexpr int kMaxChunks = 32;             // slice <= 65536 logits per row
+constexpr int kStages = SC_RING_STAGES;    // ring depth
+constexpr int kMaxChunks = 65536 / kCH;    // slice <= 65536 logits per row
 constexpr int kMaxCluster = 16;
 constexpr int kEntries = kMaxChunks * kRounds * kNW;  // (chunk, round, warp) segments
-constexpr uint32_t kWaitLimit = 1u << 22;  // bounded mbarrier waits (~seconds)
-constexpr int kMinBlocksPerSM = 8;
+constexpr uint32_t kWaitLimit = 1u << 21;  // bounded mbarrier waits (~seconds)
+constexpr uint32_t kSuspendNs = 1000;      // try_wait suspend hint
+constexpr int kMinBlocksPerSM = SC_MIN_BLOCKS;
 
 enum Mode : int { kVerify = 0, kStats = 1 };
 
@@ -111,16 +123,19 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t *bar, uint32_t bytes) {
 }
 
 // Bounded wait for the phase of parity `parity` of an mbarrier; false on timeout.
+// Each try_wait suspends the thread for up to kSuspendNs (it resumes as soon as
+// the phase completes), so a waiting warp issues a few instructions per
+// microsecond instead of spinning.
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity) {
   const uint32_t a = smem_u32(bar);
   for (uint32_t i = 0; i < kWaitLimit; ++i) {
     uint32_t done;
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
         "selp.u32 %0, 1, 0, p;\n\t}"
         : "=r"(done)
-        : "r"(a), "r"(parity)
+        : "r"(a), "r"(parity), "n"(kSuspendNs)
         : "memory");
     if (done) return true;
   }
@@ -251,9 +266,10 @@ __device__ __forceinline__ void ms_combine(float &m, float &s, float m2, float s
 }
 
 // Pass 1 on one row of one chunk: this thread's kRounds vectors, online
-// (max m, sum s of 2^{y k - refk(m)}).  kFull: the chunk holds kCH logits.
+// (max m, sum s of 2^{y k - refk(m)}), s kept as two partial sums.
+// kFull: the chunk holds kCH logits.
 template <typename E, bool kFull>
-__device__ __forceinline__ void online_row(const E *src, int n, float k, float &m, float &s) {
+__device__ __forceinline__ void online_row(const E *src, int n, float k, float &m, float2 &s) {
   float y[kRounds][8];
 #pragma unroll
   for (int r = 0; r < kRounds; ++r) {
@@ -270,7 +286,8 @@ __device__ __forceinline__ void online_row(const E *src, int n, float k, float &
 #pragma unroll
     for (int i = 0; i < 8; i += 2) mn = max3(mn, y[r][i], y[r][i + 1]);
   const float rn = refk(mn, k);
-  float s0 = s * ex2(refk(m, k) - rn), s1 = 0.0f;
+  const float sc = ex2(refk(m, k) - rn);
+  float s0 = s.x * sc, s1 = s.y * sc;
 #pragma unroll
   for (int r = 0; r < kRounds; ++r)
 #pragma unroll
@@ -279,7 +296,42 @@ __device__ __forceinline__ void online_row(const E *src, int n, float k, float &
       s1 += ex2(fmaf(y[r][i + 1], k, -rn));
     }
   m = mn;
-  s = s0 + s1;
+  s = make_float2(s0, s1);
+}
+
+__device__ __forceinline__ __nv_bfloat162 as_bf162(uint32_t w) {
+  return *reinterpret_cast<__nv_bfloat162 *>(&w);
+}
+
+// bf16 full chunk: the exact maximum from a packed bf16x2 max tree over the raw
+// words, then one packed f32x2 FMA per two logits for the exponent arguments
+// and packed f32x2 adds for the two partial sums.
+template <>
+__device__ __forceinline__ void online_row<uint16_t, true>(const uint16_t *src, int n, float k,
+                                                           float &m, float2 &s) {
+  (void)n;
+  uint32_t w[kRounds * 4];
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r) {
+    const uint4 v = *reinterpret_cast<const uint4 *>(src + 8 * (r * kNT + static_cast<int>(threadIdx.x)));
+    w[4 * r] = v.x; w[4 * r + 1] = v.y; w[4 * r + 2] = v.z; w[4 * r + 3] = v.w;
+  }
+  __nv_bfloat162 mx = as_bf162(w[0]);
+#pragma unroll
+  for (int i = 1; i < kRounds * 4; ++i) mx = __hmax2(mx, as_bf162(w[i]));
+  const float mn = fmaxf(m, fmaxf(__low2float(mx), __high2float(mx)));
+  const float rn = refk(mn, k);
+  const float sc = ex2(refk(m, k) - rn);
+  float2 acc = __fmul2_rn(s, make_float2(sc, sc));
+  const float2 kk = make_float2(k, k), nr = make_float2(-rn, -rn);
+#pragma unroll
+  for (int i = 0; i < kRounds * 4; ++i) {
+    const float2 y = make_float2(__uint_as_float(w[i] << 16), __uint_as_float(w[i] & 0xFFFF0000u));
+    const float2 t = __ffma2_rn(y, kk, nr);
+    acc = __fadd2_rn(acc, make_float2(ex2(t.x), ex2(t.y)));
+  }
+  m = mn;
+  s = acc;
 }
 
 // Row scalars of the weight formula.  With a_v = y^q_v k - R_q, b_v = y^p_v k - R_p
@@ -290,31 +342,34 @@ struct RowScalars {
   float Rq, Rp, k, c;
 };
 
-// Sampling weight of one logit, up to the common factor 1/S_q: the residual
-// max(0, p - q) of a pair, or the unnormalised p of the bonus row.  Rounded
-// intrinsics keep every evaluation of the same logit bit-identical.
-template <bool kPair>
-__device__ __forceinline__ float weight(float yq, float yp, const RowScalars &r) {
-  if constexpr (kPair) {
-    const float a = __fmaf_rn(yq, r.k, -r.Rq);
-    const float b = __fadd_rn(__fmaf_rn(yp, r.k, -r.Rp), r.c);
-    return fmaxf(0.0f, __fsub_rn(ex2(b), ex2(a)));
-  } else {
-    return ex2(__fmaf_rn(yp, r.k, -r.Rp));
-  }
-}
-
-// Eight weights and their sum in index order.  Used identically by pass 2 and
-// by the search.
+// Sampling weights of eight logits, up to the common factor 1/S_q: the
+// residual max(0, p - q) of a pair, or the unnormalised p of the bonus row,
+// computed two at a time in packed f32x2; returns their sum in index order.
+// Pass 2 and the search call exactly this, so the same logit always gets the
+// same weight and the same prefix sums.
 template <bool kPair>
 __device__ __forceinline__ float vec_weights(const float (&yq)[8], const float (&yp)[8],
                                              const RowScalars &r, float (&w)[8]) {
+  const float2 kk = make_float2(r.k, r.k);
+  const float2 nrp = make_float2(-r.Rp, -r.Rp);
+#pragma unroll
+  for (int e = 0; e < 8; e += 2) {
+    const float2 b = __ffma2_rn(make_float2(yp[e], yp[e + 1]), kk, nrp);
+    if constexpr (kPair) {
+      const float2 a = __ffma2_rn(make_float2(yq[e], yq[e + 1]), kk, make_float2(-r.Rq, -r.Rq));
+      const float2 bc = __fadd2_rn(b, make_float2(r.c, r.c));
+      const float2 d = __ffma2_rn(make_float2(ex2(a.x), ex2(a.y)), make_float2(-1.0f, -1.0f),
+                                  make_float2(ex2(bc.x), ex2(bc.y)));
+      w[e] = fmaxf(0.0f, d.x);
+      w[e + 1] = fmaxf(0.0f, d.y);
+    } else {
+      w[e] = ex2(b.x);
+      w[e + 1] = ex2(b.y);
+    }
+  }
   float s = 0.0f;
 #pragma unroll
-  for (int e = 0; e < 8; ++e) {
-    w[e] = weight<kPair>(kPair ? yq[e] : 0.0f, yp[e], r);
-    s = __fadd_rn(s, w[e]);
-  }
+  for (int e = 0; e < 8; ++e) s = __fadd_rn(s, w[e]);
   return s;
 }
 
@@ -441,6 +496,40 @@ __device__ __forceinline__ void prime(const Ring<E> &R, Shared &sh, int fills) {
     for (int c = 0; c < min(kStages, R.nch); ++c) R.issue(sh, c, (fills + c) % kStages);
 }
 
+// Pass 2 stream: the last min(kStages, nch) chunks of pass 1 are still in the
+// ring, so they are processed first with no copy; every stage they free is
+// refilled with the next chunk from the start of the slice (L2-resident), so
+// the first refill's latency overlaps work.  Chunk c still goes to body(c, s).
+template <typename E, typename Body>
+__device__ __forceinline__ int stream_again(const Ring<E> &R, Shared &sh, Body &&body) {
+  const int nch = R.nch;
+  const int nres = min(kStages, nch);
+  int tmo = 0;
+  for (int it = 0; it < nch; ++it) {
+    const int s = (nch - nres + it % nres) % kStages;
+    int c;
+    if (it < nres) {
+      c = nch - nres + it;
+    } else {
+      c = it - nres;
+      // fills of stage s so far: its pass-1 fills, then one refill per nres iterations
+      const int p1 = nch > s ? (nch - 1 - s) / kStages + 1 : 0;
+      const int fill = p1 + (it - nres) / nres;
+      if (R.bulk) {
+        if (!mbar_wait(&sh.full[s], fill & 1)) tmo = 1;
+      } else {
+        R.load_sync(c, s);
+        __syncthreads();
+      }
+    }
+    body(c, s);
+    __syncthreads();  // every thread is done with stage s
+    const int next = it;  // chunk to refill this stage with
+    if (R.bulk && threadIdx.x == 0 && next < nch - nres) R.issue(sh, next, s);
+  }
+  return tmo;
+}
+
 // ------------------------------------------------------------------ the kernel
 
 template <typename E>
@@ -504,22 +593,24 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
 
   // ---- pass 1: online max and sum of exponentials
   const float k = P.k;
-  float mq = -FLT_MAX, s_q = 0.0f, mp = -FLT_MAX, s_p = 0.0f;
+  float mq = -FLT_MAX, mp = -FLT_MAX;
+  float2 s2q = make_float2(0.0f, 0.0f), s2p = make_float2(0.0f, 0.0f);
   const int lx = x - v0;  // draft token's offset in this slice (thread 0 only)
   int tmo = stream(R, sh, fills, [&](int c, int s) {
     const int n = R.chunk_len(c);
     if (n == kCH) {
-      if (pair) online_row<E, true>(R.q(s), n, k, mq, s_q);
-      online_row<E, true>(R.p(s), n, k, mp, s_p);
+      if (pair) online_row<E, true>(R.q(s), n, k, mq, s2q);
+      online_row<E, true>(R.p(s), n, k, mp, s2p);
     } else {
-      if (pair) online_row<E, false>(R.q(s), n, k, mq, s_q);
-      online_row<E, false>(R.p(s), n, k, mp, s_p);
+      if (pair) online_row<E, false>(R.q(s), n, k, mq, s2q);
+      online_row<E, false>(R.p(s), n, k, mp, s2p);
     }
     if (tid == 0 && static_cast<unsigned>(lx - c * kCH) < static_cast<unsigned>(n)) {
       sh.xq = Elt<E>::at(R.q(s), lx - c * kCH);
       sh.xp = Elt<E>::at(R.p(s), lx - c * kCH);
     }
   });
+  float s_q = s2q.x + s2q.y, s_p = s2p.x + s2p.y;
   tmo = __syncthreads_or(tmo);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
@@ -637,16 +728,12 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   }
   __syncthreads();
   const RowScalars rs = {sh.Rq, sh.Rp, k, sh.c};
-  if (sh.need_p2) {
-    prime(R, sh, fills);  // the ring is free: restart the stream (L2-resident by now)
-  } else {
-    cluster_arrive();  // no further reads of peer shared memory
-  }
+  if (!sh.need_p2) cluster_arrive();  // no further reads of peer shared memory
 
   // ---- pass 2: residual weights and their per-segment totals
   if (sh.need_p2) {
     const int nseg = R.nch * kRounds * kNW;
-    tmo = stream(R, sh, fills, [&](int c, int s) {
+    tmo = stream_again(R, sh, [&](int c, int s) {
       const int n = R.chunk_len(c);
       if (pair) {
         if (n == kCH) weights_chunk<E, true, true>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
