@@ -74,7 +74,7 @@ typedef enum {
 #define SC_ROW_ACCEPT 4 /* a_j in {0, 1} (a_gamma = 0) */
 #define SC_ROW_QX 5     /* q_j(x_j) */
 #define SC_ROW_PIX 6    /* pi_j(x_j) */
-#define SC_ROW_CAND 7   /* token this position would emit if it were j* (-1 if none) */
+#define SC_ROW_CAND 7   /* next_token at position j*, -1 at every other position */
 #define SC_ROW_FIELDS 8
 
 /* Device workspace needed by sc_verify for B sequences of gamma drafts
@@ -144,12 +144,13 @@ const char *sc_status_string(int code);
  * call cudaMalloc, e.g. an inference server whose device memory is carved up by
  * its own allocator before the first request, or a caller running where a
  * synchronising allocation would stall other streams.  Such callers still pass
- * their inputs and outputs, but need no workspace: the sequence tickets, per-
- * position flags and candidates live in a fixed array compiled into the library,
- * one copy per device, held by every GPU that loads the library until exit.
+ * their inputs and outputs, but need no workspace: the tickets, per-position
+ * decision records and per-slice totals live in a fixed array compiled into the
+ * library, one copy per device, held by every GPU that loads the library until
+ * exit.
  *
  * Limits: B <= SC_STATIC_MAX_B and B * (gamma + 1) <= SC_STATIC_MAX_UNITS
- * (48 KiB of scratch); larger batches return SC_ERR_SCRATCH_LIMIT and queue no
+ * (about 1.5 MiB of scratch); larger batches return SC_ERR_SCRATCH_LIMIT and queue no
  * work.  Other arguments are those of sc_verify and are checked the same way.
  *
  * The first call on a device looks up the array's device address (the library's

@@ -5,30 +5,35 @@
 // for B sequences of gamma drafted positions over a V-token vocabulary, in ONE
 // kernel launch:
 //
-//   unit   one (b, j < gamma) row pair (draft row q_j, target row p_j), or the
-//          bonus target row (b, gamma);
-//   grid   one thread-block cluster of C CTAs per unit; CTA r of the cluster
-//          owns the vocabulary slice [r L, (r+1) L) of both rows;
-//   pass 1 the slice streams from HBM through a two-stage shared-memory ring
-//          filled by TMA bulk copies (cp.async.bulk + mbarrier), 4096 logits
-//          per row per stage; each thread keeps an online (max, sum of exp);
-//          the CTA partials are merged over the cluster through distributed
-//          shared memory, giving M and S of both rows, max q = 1/S_q and
-//          max p = 1/S_p, and the deferral decision of Table 1;
-//   pass 2 only when the unit needs it (a rejected draft, the bonus row, the
-//          OPT rule inside the band where its TV term decides, sc_row_stats):
-//          the slice is streamed again -- it is still in L2 -- and every
-//          element gets its residual weight max(0, p - q) (p for the bonus
-//          row).  Their total over the cluster is D_TV(p, q) * S_q (Lemma 3),
-//          and the per-(chunk, round, warp) totals drive the inverse-CDF search;
-//   search the CTA whose slice holds u * R finds the segment, one warp reloads
-//          it and scans it, and that CTA publishes the unit;
-//   scan   the last unit of a sequence to finish (atomic ticket, no waiting)
-//          finds j* = min{j : a_j = 0} and writes the outputs.
+//   unit    one (b, j < gamma) row pair (draft row q_j, target row p_j), or the
+//           bonus target row (b, gamma);
+//   grid    one thread-block cluster of C CTAs per unit; CTA r of the cluster
+//           owns the vocabulary slice [r L, (r+1) L) of both rows;
+//   pass 1  the slice streams from HBM through a two-stage shared-memory ring
+//           filled by TMA bulk copies (cp.async.bulk + mbarrier), 4096 logits
+//           per row per stage; each thread keeps an online (max, sum of exp);
+//           the CTA partials are merged over the cluster through distributed
+//           shared memory, giving M and S of both rows, max q = 1/S_q and
+//           max p = 1/S_p, the deferral decision of Table 1 and the acceptance
+//           test of the draft token;
+//   TV      only for the OPT rule inside the band where its TV term decides, and
+//           for sc_row_stats: the slice is streamed again (from L2) and the
+//           residual weights max(0, p - q) are summed over the cluster; their
+//           total is D_TV(p, q) S_q (Lemma 3);
+//   finish  every CTA writes its unit's decision record and takes a ticket of
+//           its slice rank r in the sequence.  The last CTA of rank r (all
+//           gamma + 1 decisions are in) knows j* = min{j : a_j = 0}, streams its
+//           slice of row j* -- the rejected pair, whose residual max(0, p - q)
+//           is sampled, or the bonus row p_gamma when all drafts were accepted --
+//           and stores the slice's total weight.  The last of those C slice
+//           passes does the inverse-CDF draw: it finds the slice and the
+//           (chunk, round, warp) segment holding u R, and one warp scans the
+//           segment's 256 logits.  Only the sampled row of each sequence gets a
+//           second pass, and no CTA ever waits on another cluster.
 //
 // Exponentials are ex2.approx of fma(y, log2(e)/T, -R), R = fl(M log2(e)/T):
-// one rounding per logit.  No thread waits on another cluster; every mbarrier wait is bounded
-// and reports SC_DEV_TIMEOUT instead of hanging.
+// one rounding per logit.  Every mbarrier wait is bounded and reports
+// SC_DEV_TIMEOUT instead of hanging.
 
 #include "sc.h"
 
@@ -63,7 +68,10 @@ constexpr int kCH = SC_CHUNK;              // logits per row per ring stage
 constexpr int kVPC = kCH / 8;              // 8-element vectors per chunk
 constexpr int kRounds = kVPC / kNT;        // vectors per thread per chunk
 constexpr int kStages = SC_RING_STAGES;    // ring depth
-constexpr int kMaxChunks = 65536 / kCH;    // slice <= 65536 logits per row
+#ifndef SC_MAX_SLICE
+#define SC_MAX_SLICE 131072
+#endif
+constexpr int kMaxChunks = SC_MAX_SLICE / kCH;  // slice <= SC_MAX_SLICE logits per row
 constexpr int kMaxCluster = 16;
 constexpr int kEntries = kMaxChunks * kRounds * kNW;  // (chunk, round, warp) segments
 constexpr uint32_t kWaitLimit = 1u << 21;  // bounded mbarrier waits (~seconds)
@@ -93,9 +101,12 @@ struct Params {
   float *max_q;
   float *max_p;
   float *tv;
-  uint32_t *tickets;
-  int32_t *unit_flags;
-  int32_t *unit_cand;
+  // workspace (verification only)
+  uint32_t *rank_tickets;  // [B][kMaxCluster] arrivals of the CTAs of slice rank r; zero at rest
+  uint32_t *seq_tickets;   // [B] finished slice passes of the sampled row; zero at rest
+  float4 *records;         // [B][kMaxCluster][gamma+1] (R_q, R_p, c, flags) as seen by rank r
+  float *slice_totals;     // [B][kMaxCluster] total weight of slice r of the sampled row
+  float *chunk_pre;        // [B][kMaxCluster][kMaxChunks + 1] its exclusive prefix at each chunk start
   int32_t *status;
 };
 
@@ -231,18 +242,28 @@ struct __align__(16) Shared {
   // exchange 1: (m_q, s_q, m_p, s_p) of this CTA, raw logits at the draft token
   float4 part_ms;
   float2 part_x;
-  // exchange 2: this CTA's total residual weight
+  // exchange 2 (TV pass): this CTA's total residual weight
   float part_r;
   int timeout;
   float red[kNW][4];
   float seg[kEntries + 1];  // per-(chunk, round, warp) weights, then exclusive prefixes
   float xq, xp;             // raw logits at the draft token, when in this slice
   // row state, identical in every CTA of the cluster
-  float Mq, Sq, Mp, Sp, Rq, Rp, maxq, maxp, c, tv, qx, pix, ug;
-  int err, delta, accept, need_p2, sample;
-  int publisher;            // rank that publishes the unit
-  int cross_seg;            // segment holding u*R in the publishing CTA (-1: last positive)
-  float t_seg;              // u*R minus the weight before that segment
+  float Mq, Sq, Mp, Sp, Rq, Rp, maxq, maxp, c, tv, qx, pix;
+  int err, delta, accept, need_p2;
+  // sequence finish
+  int rank_last;            // last CTA of this slice rank in the sequence: runs the sample pass
+  int seq_last;             // last sample pass of the sequence: draws the token
+  int jstar, bad, sample_ok;
+  float4 rj;                // (R_q, R_p, c, flags) of row j*
+  int cross_rank;           // slice holding u * R_tot
+  int cross_chunk;          // chunk of that slice holding it (else its last chunk with weight)
+  int have_t;               // u * R_tot lies inside that chunk (not past a rounding gap)
+  float chunk_lo;           // exclusive prefix of the slice at the start of that chunk
+  int cross_seg;            // segment of that chunk holding it (-1: none)
+  int token;                // the drawn token
+  double t_slice;           // u * R_tot minus the weight before the crossing slice
+  float t_seg;              // ... minus the weight before the crossing segment
 };
 
 __device__ __forceinline__ float max3(float a, float b, float c) {
@@ -467,17 +488,48 @@ struct Ring {
   }
 };
 
-// Stream every chunk of the slice through the ring and call body(c, stage) on
-// each.  `fills` counts stage fills since the kernel started (it fixes each
-// stage's mbarrier phase); the first kStages fills of this pass must already
-// be issued when bulk (see prime()).
+// A ring over slice `rank` of row pair (b, j) -- only the target row when j is
+// the bonus position gamma.
+template <typename E>
+__device__ __forceinline__ Ring<E> make_ring(const Params &P, unsigned char *smem, int b, int j,
+                                             int rank) {
+  const int v0 = rank * P.L;
+  Ring<E> R;
+  R.base = reinterpret_cast<E *>(smem);
+  R.pair = j < P.gamma;
+  R.gq = static_cast<const E *>(P.draft) +
+         (static_cast<size_t>(b) * P.gamma + (R.pair ? j : 0)) * P.V + v0;
+  R.gp = static_cast<const E *>(P.target) + (static_cast<size_t>(b) * (P.gamma + 1) + j) * P.V + v0;
+  R.len = max(0, min(P.L, P.V - v0));
+  R.nch = (R.len + kCH - 1) / kCH;
+  R.bulk = P.bulk != 0;
+  return R;
+}
+
+// Every pass starts with all stages free and puts chunk c in stage c % kStages.
+// Bit s of `ph` is the parity of the next completion of stage s's mbarrier;
+// all threads keep identical copies.
+template <typename E>
+__device__ __forceinline__ void prime(const Ring<E> &R, Shared &sh) {
+  if (R.bulk && threadIdx.x == 0)
+    for (int c = 0; c < min(kStages, R.nch); ++c) R.issue(sh, c, c);
+}
+
+__device__ __forceinline__ int wait_stage(Shared &sh, int s, uint32_t &ph) {
+  const bool ok = mbar_wait(&sh.full[s], (ph >> s) & 1u);
+  ph ^= 1u << s;
+  return ok ? 0 : 1;
+}
+
+// Stream every chunk of the slice through the ring (primed by prime()) and call
+// body(c, stage) on each.  Returns 1 if a copy did not land within the wait limit.
 template <typename E, typename Body>
-__device__ __forceinline__ int stream(const Ring<E> &R, Shared &sh, int &fills, Body &&body) {
+__device__ __forceinline__ int stream(const Ring<E> &R, Shared &sh, uint32_t &ph, Body &&body) {
   int tmo = 0;
   for (int c = 0; c < R.nch; ++c) {
-    const int f = fills + c, s = f % kStages;
+    const int s = c % kStages;
     if (R.bulk) {
-      if (!mbar_wait(&sh.full[s], (f / kStages) & 1)) tmo = 1;
+      tmo |= wait_stage(sh, s, ph);
     } else {
       R.load_sync(c, s);
       __syncthreads();
@@ -486,37 +538,24 @@ __device__ __forceinline__ int stream(const Ring<E> &R, Shared &sh, int &fills, 
     __syncthreads();  // every thread is done with stage s
     if (R.bulk && threadIdx.x == 0 && c + kStages < R.nch) R.issue(sh, c + kStages, s);
   }
-  fills += R.nch;
   return tmo;
 }
 
-template <typename E>
-__device__ __forceinline__ void prime(const Ring<E> &R, Shared &sh, int fills) {
-  if (R.bulk && threadIdx.x == 0)
-    for (int c = 0; c < min(kStages, R.nch); ++c) R.issue(sh, c, (fills + c) % kStages);
-}
-
-// Pass 2 stream: the last min(kStages, nch) chunks of pass 1 are still in the
-// ring, so they are processed first with no copy; every stage they free is
-// refilled with the next chunk from the start of the slice (L2-resident), so
-// the first refill's latency overlaps work.  Chunk c still goes to body(c, s).
+// Second pass over the slice just streamed: its last min(kStages, nch) chunks
+// are still in the ring, so they are processed first with no copy; every stage
+// they free is refilled with the next chunk from the start of the slice
+// (L2-resident), so the first refill's latency overlaps work.
 template <typename E, typename Body>
-__device__ __forceinline__ int stream_again(const Ring<E> &R, Shared &sh, Body &&body) {
+__device__ __forceinline__ int stream_again(const Ring<E> &R, Shared &sh, uint32_t &ph, Body &&body) {
   const int nch = R.nch;
   const int nres = min(kStages, nch);
   int tmo = 0;
   for (int it = 0; it < nch; ++it) {
     const int s = (nch - nres + it % nres) % kStages;
-    int c;
-    if (it < nres) {
-      c = nch - nres + it;
-    } else {
-      c = it - nres;
-      // fills of stage s so far: its pass-1 fills, then one refill per nres iterations
-      const int p1 = nch > s ? (nch - 1 - s) / kStages + 1 : 0;
-      const int fill = p1 + (it - nres) / nres;
+    const int c = it < nres ? nch - nres + it : it - nres;
+    if (it >= nres) {
       if (R.bulk) {
-        if (!mbar_wait(&sh.full[s], fill & 1)) tmo = 1;
+        tmo |= wait_stage(sh, s, ph);
       } else {
         R.load_sync(c, s);
         __syncthreads();
@@ -524,13 +563,126 @@ __device__ __forceinline__ int stream_again(const Ring<E> &R, Shared &sh, Body &
     }
     body(c, s);
     __syncthreads();  // every thread is done with stage s
-    const int next = it;  // chunk to refill this stage with
-    if (R.bulk && threadIdx.x == 0 && next < nch - nres) R.issue(sh, next, s);
+    if (R.bulk && threadIdx.x == 0 && it < nch - nres) R.issue(sh, it, s);
   }
   return tmo;
 }
 
+// Residual weights of one slice: per-(chunk, round, warp) totals in sh.seg.
+template <typename E>
+__device__ __forceinline__ int slice_weights(const Ring<E> &R, Shared &sh, uint32_t &ph,
+                                             const RowScalars &rs, bool again, int lane, int warp) {
+  auto body = [&](int c, int s) {
+    const int n = R.chunk_len(c);
+    if (R.pair) {
+      if (n == kCH) weights_chunk<E, true, true>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
+      else weights_chunk<E, true, false>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
+    } else {
+      if (n == kCH) weights_chunk<E, false, true>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
+      else weights_chunk<E, false, false>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
+    }
+  };
+  return again ? stream_again(R, sh, ph, body) : stream(R, sh, ph, body);
+}
+
+// Thread 0: turn sh.seg[0, nseg) into exclusive prefixes in vocabulary order
+// (chunk, round, warp); returns the slice total, also left in sh.seg[nseg].
+__device__ __forceinline__ float seg_prefix(Shared &sh, int nseg) {
+  float acc = 0.0f;
+  for (int i = 0; i < nseg; ++i) {
+    const float t = sh.seg[i];
+    sh.seg[i] = acc;
+    acc = __fadd_rn(acc, t);
+  }
+  sh.seg[nseg] = acc;
+  return acc;
+}
+
+// Segment totals of one chunk straight from global memory (L2): the same
+// vec_weights and warp scans as weights_chunk, so the same values; the totals
+// land in sh.seg[round * kNW + warp].
+template <typename E>
+__device__ __forceinline__ void chunk_segments(const Ring<E> &R, int c, const RowScalars &rs,
+                                               Shared &sh, int lane, int warp) {
+  const int n = R.chunk_len(c);
+  const E *gq = R.gq + static_cast<size_t>(c) * kCH;
+  const E *gp = R.gp + static_cast<size_t>(c) * kCH;
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r) {
+    const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
+    float yq[8], yp[8], w[8];
+    if (R.pair) load8_gmem(gq, e, n, R.bulk, yq);
+    load8_gmem(gp, e, n, R.bulk, yp);
+    const float vs = R.pair ? vec_weights<true>(yq, yp, rs, w) : vec_weights<false>(yq, yp, rs, w);
+    const float incl = warp_incl_scan(vs, lane);
+    if (lane == 31) sh.seg[r * kNW + warp] = incl;
+  }
+}
+
+__device__ __forceinline__ void flag_timeout(Shared &sh, const Params &P) {
+  sh.timeout = 1;
+  if (P.status) atomicOr(P.status, static_cast<int32_t>(SC_DEV_TIMEOUT));
+}
+
 // ------------------------------------------------------------------ the kernel
+
+__device__ __forceinline__ uint32_t atom_add_acq_rel(uint32_t *p, uint32_t v) {
+  uint32_t old;
+  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
+
+// The token inside segment sgi (chunk, round, warp) of a slice: the segment's
+// warp reloads its 8 x 32 logits from global memory (L2), recomputes their
+// weights with vec_weights -- the same values the slice pass summed -- and
+// takes the smallest k whose running sum passes t.  Without t (u R fell past
+// the last boundary by rounding), the segment's last positive weight.
+template <typename E>
+__device__ __forceinline__ int search_segment(const Ring<E> &R, const RowScalars &rs, int v0,
+                                              int sgi, bool have_t, float t, int lane, int warp) {
+  const int r = (sgi / kNW) % kRounds, c = sgi / (kNW * kRounds);
+  const int n = R.chunk_len(c);
+  const int e = 8 * (r * kNT + warp * 32 + lane);
+  float yq[8], yp[8], w[8];
+  const E *gq = R.gq + static_cast<size_t>(c) * kCH;
+  const E *gp = R.gp + static_cast<size_t>(c) * kCH;
+  if (R.pair) load8_gmem(gq, e, n, R.bulk, yq);
+  load8_gmem(gp, e, n, R.bulk, yp);
+  const float vs = R.pair ? vec_weights<true>(yq, yp, rs, w) : vec_weights<false>(yq, yp, rs, w);
+  const float incl = warp_incl_scan(vs, lane);
+  float excl = __shfl_up_sync(0xFFFFFFFFu, incl, 1);
+  if (lane == 0) excl = 0.0f;
+  const float tt0 = have_t ? t : FLT_MAX;
+  int tok = -1;
+  const unsigned mm = __ballot_sync(0xFFFFFFFFu, tt0 >= excl && tt0 < incl && vs > 0.0f);
+  if (mm) {
+    const int src = __ffs(mm) - 1;
+    if (lane == src) {
+      const float tt = __fsub_rn(tt0, excl);
+      float acc = 0.0f;
+      int last = -1;
+      for (int i = 0; i < 8; ++i) {
+        acc = __fadd_rn(acc, w[i]);
+        if (w[i] > 0.0f) last = i;
+        if (tok < 0 && acc > tt) tok = i;
+      }
+      if (tok < 0) tok = last;
+      tok = v0 + c * kCH + e + tok;
+    }
+    tok = __shfl_sync(0xFFFFFFFFu, tok, src);
+  } else {
+    int last = -1;
+    for (int i = 0; i < 8; ++i)
+      if (w[i] > 0.0f) last = i;
+    const unsigned lm = __ballot_sync(0xFFFFFFFFu, last >= 0);
+    if (lm) {
+      const int ln = 31 - __clz(lm);
+      const int li = __shfl_sync(0xFFFFFFFFu, last, ln);
+      tok = v0 + c * kCH + 8 * (r * kNT + warp * 32 + ln) + li;
+    }
+  }
+  return tok;
+}
 
 template <typename E>
 __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Params P) {
@@ -544,29 +696,16 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   const bool verify = P.mode == kVerify;
 
   int b, j;
-  bool pair;
   if (verify) {
     b = unit / G1;
     j = unit % G1;
-    pair = j < P.gamma;
   } else {
     b = unit / P.gamma;
     j = unit % P.gamma;
-    pair = true;
   }
-  const size_t qoff = (static_cast<size_t>(b) * P.gamma + j) * P.V;
-  const size_t poff = (static_cast<size_t>(b) * G1 + j) * P.V;
   const int v0 = rank * P.L;
-  const int len = max(0, min(P.L, P.V - v0));
-
-  Ring<E> R;
-  R.base = reinterpret_cast<E *>(smem_raw);
-  R.gq = static_cast<const E *>(P.draft) + qoff + v0;
-  R.gp = static_cast<const E *>(P.target) + poff + v0;
-  R.len = len;
-  R.nch = (len + kCH - 1) / kCH;
-  R.pair = pair;
-  R.bulk = P.bulk != 0;
+  const Ring<E> R = make_ring<E>(P, smem_raw, b, j, rank);
+  const bool pair = R.pair;
   Shared &sh = *reinterpret_cast<Shared *>(smem_raw + static_cast<size_t>(kStages) * 2 * kCH * sizeof(E));
 
   // ---- start the stream; prefetch the row's scalars
@@ -580,8 +719,8 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
   }
-  int fills = 0;
-  prime(R, sh, fills);
+  uint32_t ph = 0;
+  prime(R, sh);
   float uj = 0.0f, ug = 0.0f;
   int x = -1;
   if (verify && tid == 0) {
@@ -596,7 +735,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   float mq = -FLT_MAX, mp = -FLT_MAX;
   float2 s2q = make_float2(0.0f, 0.0f), s2p = make_float2(0.0f, 0.0f);
   const int lx = x - v0;  // draft token's offset in this slice (thread 0 only)
-  int tmo = stream(R, sh, fills, [&](int c, int s) {
+  int tmo = stream(R, sh, ph, [&](int c, int s) {
     const int n = R.chunk_len(c);
     if (n == kCH) {
       if (pair) online_row<E, true>(R.q(s), n, k, mq, s2q);
@@ -633,8 +772,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     if (tmo) {
       as = NAN;
       cs = NAN;
-      sh.timeout = 1;
-      if (P.status) atomicOr(P.status, static_cast<int32_t>(SC_DEV_TIMEOUT));
+      flag_timeout(sh, P);
     }
     sh.part_ms = make_float4(a, as, c, cs);
     sh.part_x = make_float2(sh.xq, sh.xp);
@@ -681,19 +819,14 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       sh.err = err;
       sh.delta = 0;
       sh.need_p2 = 0;
-      sh.sample = 0;
       sh.accept = 0;
       sh.tv = -1.0f;
       sh.qx = 0.0f;
       sh.pix = 0.0f;
-      sh.ug = ug;
       sh.c = pair && !err ? log2f(as / cs) : 0.0f;
-      if (!err) {
-        if (!pair) {
-          sh.need_p2 = verify;  // bonus row: drawn speculatively, used when j* = gamma
-          sh.sample = verify;
-        } else if (!verify) {
-          sh.need_p2 = 1;       // sc_row_stats: TV of every pair
+      if (!err && pair) {
+        if (!verify) {
+          sh.need_p2 = 1;  // sc_row_stats: TV of every pair
         } else {
           // deferral rule (Table 1)
           const float maxq = sh.maxq, maxp = sh.maxp, al = P.alpha;
@@ -710,182 +843,68 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
             case SC_RULE_ALWAYS_DEFER: sh.delta = 1; break;
             default: sh.delta = 0; break;
           }
-          if (pending) {
-            sh.need_p2 = 1;
-          } else {
-            accept_test(sh, yqx, ypx, uj, P.kd, P.row_info != nullptr);
-            sh.need_p2 = !sh.accept;
-            sh.sample = !sh.accept;
-          }
+          if (pending) sh.need_p2 = 1;
+          else accept_test(sh, yqx, ypx, uj, P.kd, P.row_info != nullptr);
         }
       }
-      // keep the draft-token logits for a decision after pass 2
+      // keep the draft-token logits for a decision after the TV pass
       sh.xq = yqx;
       sh.xp = ypx;
-      sh.publisher = 0;
-      sh.cross_seg = -2;
     }
   }
   __syncthreads();
-  const RowScalars rs = {sh.Rq, sh.Rp, k, sh.c};
   if (!sh.need_p2) cluster_arrive();  // no further reads of peer shared memory
 
-  // ---- pass 2: residual weights and their per-segment totals
+  // ---- TV pass (sc_row_stats, or the OPT band): residual weights of this row
   if (sh.need_p2) {
-    const int nseg = R.nch * kRounds * kNW;
-    tmo = stream_again(R, sh, [&](int c, int s) {
-      const int n = R.chunk_len(c);
-      if (pair) {
-        if (n == kCH) weights_chunk<E, true, true>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
-        else weights_chunk<E, true, false>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
-      } else {
-        if (n == kCH) weights_chunk<E, false, true>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
-        else weights_chunk<E, false, false>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
-      }
-    });
+    const RowScalars rs = {sh.Rq, sh.Rp, k, sh.c};
+    tmo = slice_weights(R, sh, ph, rs, true, lane, warp);
     tmo = __syncthreads_or(tmo);
     if (tid == 0) {
-      float acc = 0.0f;  // exclusive prefixes in vocabulary order (chunk, round, warp)
-      for (int i = 0; i < nseg; ++i) {
-        const float t = sh.seg[i];
-        sh.seg[i] = acc;
-        acc = __fadd_rn(acc, t);
-      }
-      sh.seg[nseg] = acc;
+      float acc = seg_prefix(sh, R.nch * kRounds * kNW);
       if (tmo) {
         acc = NAN;
-        sh.timeout = 1;
-        if (P.status) atomicOr(P.status, static_cast<int32_t>(SC_DEV_TIMEOUT));
+        flag_timeout(sh, P);
       }
       sh.part_r = acc;
     }
     cluster.sync();  // exchange 2
-
     if (warp == 0) {
       float tot = 0.0f;
       if (lane < C) tot = *cluster.map_shared_rank(&sh.part_r, lane);
-      const float pre = warp_incl_scan(tot, lane);  // through rank `lane`
-      const float Rtot = __shfl_sync(0xFFFFFFFFu, pre, C - 1);
-      float before = __shfl_up_sync(0xFFFFFFFFu, pre, 1);
-      if (lane == 0) before = 0.0f;
+      const float Rtot = __shfl_sync(0xFFFFFFFFu, warp_incl_scan(tot, lane), C - 1);
       if (lane == 0) {
         if (!isfinite(Rtot)) {
           sh.err |= SC_DEV_TIMEOUT;
-          sh.sample = 0;
-        } else if (pair) {
+        } else {
           sh.tv = fminf(1.0f, fmaxf(0.0f, Rtot / sh.Sq));  // Lemma 3: R = S_q D_TV(p, q)
-        }
-        if (isfinite(Rtot) && pair && !sh.sample) {
-          // TV was needed to decide: sc_row_stats, or the OPT band
           if (verify) {
             sh.delta = sh.maxq < sh.maxp - P.alpha * sh.tv;  // Eq. 10
             accept_test(sh, sh.xq, sh.xp, uj, P.kd, P.row_info != nullptr);
-            sh.sample = !sh.accept;
-          }
-        }
-      }
-      const int sample = __shfl_sync(0xFFFFFFFFu, sh.sample, 0);
-      if (sample && Rtot > 0.0f) {
-        const double t = static_cast<double>(sh.ug) * static_cast<double>(Rtot);
-        const bool cross = lane < C && tot > 0.0f && t >= static_cast<double>(before) &&
-                           t < static_cast<double>(pre);
-        const unsigned cm = __ballot_sync(0xFFFFFFFFu, cross);
-        const unsigned pm = __ballot_sync(0xFFFFFFFFu, lane < C && tot > 0.0f);
-        const int cr = cm ? __ffs(cm) - 1 : 31 - __clz(pm);
-        const float bcr = __shfl_sync(0xFFFFFFFFu, before, cr);
-        if (lane == 0) {
-          sh.publisher = cr;
-          if (cr == rank) {
-            // the segment of this CTA that holds t (or, past a rounding gap, none)
-            const double tl = cm ? t - static_cast<double>(bcr) : -1.0;
-            int sgi = -1;
-            if (cm)
-              for (int i = 0; i < nseg; ++i)
-                if (tl >= static_cast<double>(sh.seg[i]) && tl < static_cast<double>(sh.seg[i + 1]) &&
-                    sh.seg[i + 1] > sh.seg[i]) {
-                  sgi = i;
-                  break;
-                }
-            sh.cross_seg = sgi;
-            sh.t_seg = sgi >= 0 ? __double2float_rd(tl - static_cast<double>(sh.seg[sgi])) : 0.0f;
           }
         }
       }
     }
     cluster_arrive();  // no further reads of peer shared memory
     __syncthreads();
-
-    // ---- search (only in the publishing CTA)
-    if (sh.sample && sh.publisher == rank && sh.cross_seg != -2) {
-      int sgi = sh.cross_seg;
-      if (sgi < 0) {
-        // rounding left u R past the last boundary: take the last segment with weight
-        for (int i = nseg - 1; i >= 0; --i)
-          if (sh.seg[i + 1] > sh.seg[i]) { sgi = i; break; }
-      }
-      const int sw = sgi >= 0 ? sgi % kNW : -1;
-      if (warp == sw) {
-        const int r = (sgi / kNW) % kRounds, c = sgi / (kNW * kRounds);
-        const int n = R.chunk_len(c);
-        const int e = 8 * (r * kNT + tid);
-        float yq[8], yp[8], w[8];
-        const E *gq = R.gq + static_cast<size_t>(c) * kCH;
-        const E *gp = R.gp + static_cast<size_t>(c) * kCH;
-        if (pair) load8_gmem(gq, e, n, R.bulk, yq);
-        load8_gmem(gp, e, n, R.bulk, yp);
-        const float vs = pair ? vec_weights<true>(yq, yp, rs, w) : vec_weights<false>(yq, yp, rs, w);
-        const float incl = warp_incl_scan(vs, lane);
-        float excl = __shfl_up_sync(0xFFFFFFFFu, incl, 1);
-        if (lane == 0) excl = 0.0f;
-        const float t = sh.cross_seg >= 0 ? sh.t_seg : FLT_MAX;
-        int tok = -1;
-        const bool mine = t >= excl && t < incl && vs > 0.0f;
-        const unsigned mm = __ballot_sync(0xFFFFFFFFu, mine);
-        if (mm) {
-          if (lane == __ffs(mm) - 1) {
-            const float tt = __fsub_rn(t, excl);
-            float acc = 0.0f;
-            int last = -1;
-            for (int i = 0; i < 8; ++i) {
-              acc = __fadd_rn(acc, w[i]);
-              if (w[i] > 0.0f) last = i;
-              if (tok < 0 && acc > tt) tok = i;
-            }
-            if (tok < 0) tok = last;
-            tok = v0 + c * kCH + e + tok;
-          }
-          tok = __shfl_sync(0xFFFFFFFFu, tok, __ffs(mm) - 1);
-        } else {
-          // last positive weight of the segment
-          int last = -1;
-          for (int i = 0; i < 8; ++i)
-            if (w[i] > 0.0f) last = i;
-          const unsigned lm = __ballot_sync(0xFFFFFFFFu, last >= 0);
-          if (lm) {
-            const int ln = 31 - __clz(lm);
-            const int li = __shfl_sync(0xFFFFFFFFu, last, ln);
-            tok = v0 + c * kCH + 8 * (r * kNT + warp * 32 + ln) + li;
-          }
-        }
-        if (lane == 0) sh.cross_seg = tok;  // reused: the sampled token
-      }
-      __syncthreads();
-    }
   }
 
-  // ---- publish this unit; the last unit of the sequence finishes it
-  if (tid == 0 && rank == sh.publisher) {
-    if (!verify) {
+  if (!verify) {
+    if (tid == 0 && rank == 0) {
       const size_t r = static_cast<size_t>(b) * P.gamma + j;
       const bool bad = sh.err != 0;
       P.max_q[r] = bad ? NAN : sh.maxq;
       P.max_p[r] = bad ? NAN : sh.maxp;
       P.tv[r] = bad ? NAN : sh.tv;
-    } else {
-      const size_t r = static_cast<size_t>(b) * G1 + j;
-      const int cand = sh.sample && sh.need_p2 && sh.cross_seg >= 0 ? sh.cross_seg : -1;
-      if (P.row_info) {
-        float *ri = P.row_info + r * SC_ROW_FIELDS;
+    }
+  } else {
+    // ---- record the decision; the last CTA of each slice rank learns j*
+    if (tid == 0) {
+      const int flags = (sh.accept ? 1 : 0) | (sh.err ? 2 : 0);
+      float4 *rec = P.records + (static_cast<size_t>(b) * kMaxCluster + rank) * G1;
+      rec[j] = make_float4(sh.Rq, sh.Rp, sh.c, __int_as_float(flags));
+      if (rank == 0 && P.row_info) {
+        float *ri = P.row_info + (static_cast<size_t>(b) * G1 + j) * SC_ROW_FIELDS;
         ri[SC_ROW_MAXQ] = pair && !sh.err ? sh.maxq : NAN;
         ri[SC_ROW_MAXP] = !sh.err ? sh.maxp : NAN;
         ri[SC_ROW_TV] = sh.tv;
@@ -893,27 +912,157 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
         ri[SC_ROW_ACCEPT] = static_cast<float>(sh.accept);
         ri[SC_ROW_QX] = sh.qx;
         ri[SC_ROW_PIX] = sh.pix;
-        ri[SC_ROW_CAND] = static_cast<float>(cand);
+        ri[SC_ROW_CAND] = -1.0f;  // the sequence's finisher fills in row j*
       }
-      P.unit_flags[r] = (sh.accept ? 1 : 0) | (sh.err ? 2 : 0);
-      P.unit_cand[r] = cand;
-      uint32_t ticket;
-      asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;"
-                   : "=r"(ticket)
-                   : "l"(P.tickets + b)
-                   : "memory");
-      if (ticket == static_cast<uint32_t>(P.gamma)) {
-        int jstar = P.gamma, bad = 0;
-        const size_t base = static_cast<size_t>(b) * G1;
+      uint32_t *tk = P.rank_tickets + static_cast<size_t>(b) * kMaxCluster + rank;
+      const int last = atom_add_acq_rel(tk, 1u) == static_cast<uint32_t>(P.gamma);
+      sh.rank_last = last;
+      if (last) {
+        *tk = 0u;  // every unit of the sequence has arrived on this rank
+        int js = P.gamma, bad = 0;
         for (int jj = 0; jj <= P.gamma; ++jj) {
-          const int f = __ldcg(P.unit_flags + base + jj);
+          const int f = __float_as_int(__ldcg(&rec[jj].w));
           bad |= f & 2;
-          if (jj < P.gamma && !(f & 1) && jstar == P.gamma) jstar = jj;
+          if (jj < P.gamma && !(f & 1) && js == P.gamma) js = jj;  // j* = min{j : a_j = 0}
         }
-        const int tok = __ldcg(P.unit_cand + base + jstar);
-        P.num_accepted[b] = bad ? 0 : jstar;
-        P.next_token[b] = bad ? -1 : tok;
-        P.tickets[b] = 0u;
+        sh.jstar = js;
+        sh.bad = bad;
+        sh.rj = __ldcg(&rec[js]);
+      }
+    }
+    __syncthreads();
+
+    if (sh.rank_last) {
+      // ---- sample pass: weights of this rank's slice of row j* -- the residual
+      // max(0, p - q) of a rejected pair (Algorithm 4), or p of the bonus row
+      const int js = sh.jstar;
+      const RowScalars rs = {sh.rj.x, sh.rj.y, k, sh.rj.z};
+      float tot_r = 0.0f;
+      if (!sh.bad) {
+        const Ring<E> Rj = make_ring<E>(P, smem_raw, b, js, rank);
+        prime(Rj, sh);
+        tmo = slice_weights(Rj, sh, ph, rs, false, lane, warp);
+        tmo = __syncthreads_or(tmo);
+        if (tid == 0) {
+          tot_r = seg_prefix(sh, Rj.nch * kRounds * kNW);
+          if (tmo) {
+            tot_r = NAN;
+            flag_timeout(sh, P);
+          }
+          float *cp = P.chunk_pre + (static_cast<size_t>(b) * kMaxCluster + rank) * (kMaxChunks + 1);
+          for (int c = 0; c < Rj.nch; ++c) cp[c] = sh.seg[c * kRounds * kNW];
+          cp[Rj.nch] = tot_r;
+        }
+      }
+      if (tid == 0) {
+        P.slice_totals[static_cast<size_t>(b) * kMaxCluster + rank] = tot_r;
+        const int last = atom_add_acq_rel(P.seq_tickets + b, 1u) == static_cast<uint32_t>(C - 1);
+        sh.seq_last = last;
+        if (last) P.seq_tickets[b] = 0u;
+      }
+      __syncthreads();
+
+      if (sh.seq_last) {
+        // ---- the draw: inverse CDF over the slices in rank order, u = u[b][gamma]
+        if (warp == 0) {
+          float tot = 0.0f;
+          if (lane < C) tot = __ldcg(P.slice_totals + static_cast<size_t>(b) * kMaxCluster + lane);
+          const float pre = warp_incl_scan(tot, lane);  // through rank `lane`
+          const float Rtot = __shfl_sync(0xFFFFFFFFu, pre, C - 1);
+          float before = __shfl_up_sync(0xFFFFFFFFu, pre, 1);
+          if (lane == 0) before = 0.0f;
+          const float u = __shfl_sync(0xFFFFFFFFu, ug, 0);
+          const bool ok = !sh.bad && isfinite(Rtot);
+          int cr = -1;
+          double tl = -1.0;
+          if (ok && Rtot > 0.0f) {
+            const double t = static_cast<double>(u) * static_cast<double>(Rtot);
+            const bool cross = lane < C && tot > 0.0f && t >= static_cast<double>(before) &&
+                               t < static_cast<double>(pre);
+            const unsigned cm = __ballot_sync(0xFFFFFFFFu, cross);
+            const unsigned pm = __ballot_sync(0xFFFFFFFFu, lane < C && tot > 0.0f);
+            cr = cm ? __ffs(cm) - 1 : 31 - __clz(pm);
+            const float bcr = __shfl_sync(0xFFFFFFFFu, before, cr);
+            tl = cm ? t - static_cast<double>(bcr) : -1.0;
+          }
+          if (lane == 0) {
+            sh.sample_ok = ok;
+            sh.cross_rank = cr;
+            sh.t_slice = tl;
+            sh.token = -1;
+          }
+        }
+        __syncthreads();
+        const int cr = sh.cross_rank;
+        if (cr >= 0) {
+          // the chunk of the crossing slice that holds t, from the stored chunk
+          // prefixes (or, past a rounding gap, the last chunk with weight)
+          const Ring<E> Rc = make_ring<E>(P, smem_raw, b, js, cr);
+          if (tid == 0) {
+            const float *cp = P.chunk_pre + (static_cast<size_t>(b) * kMaxCluster + cr) * (kMaxChunks + 1);
+            const double tl = sh.t_slice;
+            int cc = -1, clast = -1;
+            for (int c = 0; c < Rc.nch; ++c) {
+              const float lo = __ldcg(cp + c), hi = __ldcg(cp + c + 1);
+              if (hi > lo) {
+                clast = c;
+                if (cc < 0 && tl >= static_cast<double>(lo) && tl < static_cast<double>(hi)) cc = c;
+              }
+            }
+            sh.cross_chunk = cc >= 0 ? cc : clast;
+            sh.have_t = cc >= 0;
+            sh.chunk_lo = sh.cross_chunk >= 0 ? __ldcg(cp + sh.cross_chunk) : 0.0f;
+          }
+          __syncthreads();
+          const int cc = sh.cross_chunk;
+          if (cc >= 0) {
+            chunk_segments(Rc, cc, rs, sh, lane, warp);
+            __syncthreads();
+            constexpr int kSegC = kRounds * kNW;  // segments per chunk
+            if (tid == 0) {
+              // exclusive prefixes continue from the chunk's stored start, as in the slice pass
+              float acc = sh.chunk_lo;
+              for (int i = 0; i < kSegC; ++i) {
+                const float t = sh.seg[i];
+                sh.seg[i] = acc;
+                acc = __fadd_rn(acc, t);
+              }
+              sh.seg[kSegC] = acc;
+              const double tl = sh.t_slice;
+              int sgi = -1;
+              if (sh.have_t)
+                for (int i = 0; i < kSegC; ++i)
+                  if (tl >= static_cast<double>(sh.seg[i]) && tl < static_cast<double>(sh.seg[i + 1]) &&
+                      sh.seg[i + 1] > sh.seg[i]) {
+                    sgi = i;
+                    break;
+                  }
+              sh.cross_seg = sgi;
+              sh.t_seg = sgi >= 0 ? __double2float_rd(tl - static_cast<double>(sh.seg[sgi])) : 0.0f;
+            }
+            __syncthreads();
+            int sgi = sh.cross_seg;
+            if (sgi < 0) {
+              // no t inside the chunk: its last segment with weight
+              for (int i = kSegC - 1; i >= 0; --i)
+                if (sh.seg[i + 1] > sh.seg[i]) { sgi = i; break; }
+            }
+            if (sgi >= 0 && warp == sgi % kNW) {
+              const int tok = search_segment(Rc, rs, cr * P.L, cc * kSegC + sgi, sh.cross_seg >= 0,
+                                             sh.t_seg, lane, warp);
+              if (lane == 0) sh.token = tok;
+            }
+            __syncthreads();
+          }
+        }
+        if (tid == 0) {
+          const bool ok = sh.sample_ok != 0;
+          P.num_accepted[b] = ok ? js : 0;
+          P.next_token[b] = ok ? sh.token : -1;
+          if (ok && P.row_info)
+            P.row_info[(static_cast<size_t>(b) * G1 + js) * SC_ROW_FIELDS + SC_ROW_CAND] =
+                static_cast<float>(sh.token);
+        }
       }
     }
   }
@@ -937,17 +1086,44 @@ std::mutex g_mu;
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+// Workspace of sc_verify for B sequences of gamma drafts: slice-rank tickets,
+// sequence tickets (both zero between calls), then unit records, slice totals
+// and chunk prefixes (written before they are read).
+struct WsLayout {
+  size_t rank_tickets, seq_tickets, zeroed, records, slice_totals, chunk_pre, total;
+};
+
+constexpr size_t align256(size_t x) { return (x + 255) / 256 * 256; }
+
+constexpr WsLayout ws_layout(size_t B, size_t units) {
+  WsLayout w = {};
+  w.rank_tickets = 0;
+  w.seq_tickets = align256(4 * kMaxCluster * B);
+  w.zeroed = w.seq_tickets + align256(4 * B);
+  w.records = w.zeroed;
+  w.slice_totals = w.records + align256(16 * kMaxCluster * units);
+  w.chunk_pre = w.slice_totals + align256(4 * kMaxCluster * B);
+  w.total = w.chunk_pre + align256(4 * kMaxCluster * (kMaxChunks + 1) * B);
+  return w;
+}
+
+
 template <typename E>
 size_t smem_bytes() {
   return static_cast<size_t>(kStages) * 2 * kCH * sizeof(E) + sizeof(Shared);
 }
 
 // Cluster size C and slice length L (multiple of 8) for a row of V logits.
-// Long slices amortise each unit's two cluster exchanges over more streamed
-// bytes; short ones give small batches enough CTAs to cover the GPU.
+// Long slices amortise each unit's cluster exchange, decision and ticket over
+// more streamed bytes and wait on fewer peers; short ones give small batches
+// enough CTAs to cover the GPU.  65536 logits per CTA once that still fills
+// the GPU four times over, else 32768, else (small batches) 8192.
 int pick_layout(int V, int units, int sms, int *C_out, int *L_out) {
+  const long resident = static_cast<long>(kMinBlocksPerSM) * sms;
+  auto ctas = [&](long t) { return static_cast<long>(units) * ((V + t - 1) / t); };
   long target = 32768;  // logits per row per CTA
-  if (static_cast<long>(units) * ((V + target - 1) / target) < 4L * sms) target = 8192;
+  if (ctas(65536) >= 4 * resident) target = 65536;
+  else if (ctas(32768) < 4L * sms) target = 8192;
   if (const char *s = getenv("SC_SLICE")) {
     const long t = atol(s);
     if (t >= 64) target = t;
@@ -994,7 +1170,9 @@ int launch(Params P, cudaStream_t stream, int units) {
       if (cudaFuncSetAttribute(sc_unit_kernel<E>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                static_cast<int>(smem_bytes<E>())) != cudaSuccess ||
           cudaFuncSetAttribute(sc_unit_kernel<E>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
-              cudaSuccess)
+              cudaSuccess ||
+          cudaFuncSetAttribute(sc_unit_kernel<E>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                               cudaSharedmemCarveoutMaxShared) != cudaSuccess)
         return SC_ERR_CUDA;
       di.configured[ti] = true;
     }
@@ -1037,12 +1215,12 @@ int common_checks(const void *draft, const void *target, int dtype, int B, int g
 
 // ------------------------------------------------------------------ fixed scratch
 
-// Workspace of sc_verify_static: tickets [SC_STATIC_MAX_B] then unit flags and
-// candidates [SC_STATIC_MAX_UNITS] each, in sc_workspace_bytes' layout for the
-// largest accepted batch.  One copy per device, zeroed when the module loads.
-constexpr size_t kStaticScratchBytes =
-    ((4 * static_cast<size_t>(SC_STATIC_MAX_B) + 255) / 256) * 256 +
-    2 * (((4 * static_cast<size_t>(SC_STATIC_MAX_UNITS) + 255) / 256) * 256);
+// Workspace of sc_verify_static: sc_verify's layout for the largest accepted
+// batch -- SC_STATIC_MAX_UNITS units, and at most half as many sequences since
+// gamma >= 1.  One copy per device, zeroed when the module loads.
+constexpr size_t kStaticMaxSeqs =
+    SC_STATIC_MAX_B < SC_STATIC_MAX_UNITS / 2 ? SC_STATIC_MAX_B : SC_STATIC_MAX_UNITS / 2;
+constexpr size_t kStaticScratchBytes = ws_layout(kStaticMaxSeqs, SC_STATIC_MAX_UNITS).total;
 static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
 
 void *g_static_ptr[64];
@@ -1075,8 +1253,7 @@ extern "C" {
 size_t sc_workspace_bytes(int B, int gamma, int V) {
   (void)V;
   if (B < 1 || gamma < 1) return 0;
-  const size_t n = static_cast<size_t>(B) * (gamma + 1);
-  return align_up(4 * static_cast<size_t>(B), 256) + 2 * align_up(4 * n, 256);
+  return ws_layout(static_cast<size_t>(B), static_cast<size_t>(B) * (gamma + 1)).total;
 }
 
 int sc_workspace_init(void *workspace, size_t workspace_bytes, cudaStream_t stream) {
@@ -1125,11 +1302,12 @@ int sc_verify_rows(const void *draft_logits, const void *target_logits, sc_dtype
   P.row_info = row_info;
   P.status = device_status;
   unsigned char *ws = static_cast<unsigned char *>(workspace);
-  const size_t n = static_cast<size_t>(B) * (gamma + 1);
-  const size_t off1 = align_up(4 * static_cast<size_t>(B), 256);
-  P.tickets = reinterpret_cast<uint32_t *>(ws);
-  P.unit_flags = reinterpret_cast<int32_t *>(ws + off1);
-  P.unit_cand = reinterpret_cast<int32_t *>(ws + off1 + align_up(4 * n, 256));
+  const WsLayout wl = ws_layout(static_cast<size_t>(B), static_cast<size_t>(B) * (gamma + 1));
+  P.rank_tickets = reinterpret_cast<uint32_t *>(ws + wl.rank_tickets);
+  P.seq_tickets = reinterpret_cast<uint32_t *>(ws + wl.seq_tickets);
+  P.records = reinterpret_cast<float4 *>(ws + wl.records);
+  P.slice_totals = reinterpret_cast<float *>(ws + wl.slice_totals);
+  P.chunk_pre = reinterpret_cast<float *>(ws + wl.chunk_pre);
   const int units = B * (gamma + 1);
   return dtype == SC_BF16 ? launch<uint16_t>(P, stream, units) : launch<float>(P, stream, units);
 }
@@ -1196,7 +1374,8 @@ int sc_verify_static(const void *draft_logits, const void *target_logits, sc_dty
   int rc = static_scratch(&ws);
   if (rc != SC_OK) return rc;
   // the previous call left the tickets at zero unless it was cut short: clear them
-  if (cudaMemsetAsync(ws, 0, 4 * static_cast<size_t>(B), stream) != cudaSuccess) return SC_ERR_CUDA;
+  const size_t zeroed = ws_layout(static_cast<size_t>(B), static_cast<size_t>(B) * (gamma + 1)).zeroed;
+  if (cudaMemsetAsync(ws, 0, zeroed, stream) != cudaSuccess) return SC_ERR_CUDA;
   return sc_verify_rows(draft_logits, target_logits, dtype, draft_tokens, uniforms, B, gamma, V,
                         rule, alpha, temperature, num_accepted, next_token, ws, need,
                         device_status, nullptr, stream);

@@ -4,9 +4,9 @@ Some callers of this library may not call cudaMalloc at all -- an inference
 server whose device memory is handed out by its own allocator before the first
 request, or code that must not trigger an allocation (and its implicit
 synchronisation) in the middle of a decode step.  sc_verify_static serves them:
-they pass only inputs and outputs, and the scratch the kernel needs (sequence
-tickets, per-position flags and candidates) lives in a fixed array inside the
-library.
+they pass only inputs and outputs, and the scratch the kernel needs (tickets,
+per-position decision records and per-slice totals) lives in a fixed array
+inside the library.
 
 This file checks, through the C ABI, that sc_verify_static gives the same
 outputs as the workspace-taking sc_verify on two calls in a row, and that a
