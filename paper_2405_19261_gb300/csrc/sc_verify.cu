@@ -69,7 +69,7 @@ constexpr int kVPC = kCH / 8;              // 8-element vectors per chunk
 constexpr int kRounds = kVPC / kNT;        // vectors per thread per chunk
 constexpr int kStages = SC_RING_STAGES;    // ring depth
 #ifndef SC_MAX_SLICE
-#define SC_MAX_SLICE 131072
+#define SC_MAX_SLICE 65536
 #endif
 constexpr int kMaxChunks = SC_MAX_SLICE / kCH;  // slice <= SC_MAX_SLICE logits per row
 constexpr int kMaxCluster = 16;
@@ -89,8 +89,8 @@ struct Params {
   int rule;
   float alpha;
   float temperature;
-  float k;        // log2(e) / T
-  double kd;      // log2(e) / T in f64, for the decision scalars
+  float k;        // log2(e) / T, the f32 factor of every exponent of pass 1
+  float kl;       // log2(e) / T - k: with k, log2(e) / T to twice f32 precision
   int L;          // slice length per CTA (multiple of 8 logits)
   int cluster;    // CTAs per unit
   int bulk;       // 1: TMA bulk copies, 0: per-thread loads (rows not 16-byte aligned)
@@ -102,11 +102,11 @@ struct Params {
   float *max_p;
   float *tv;
   // workspace (verification only)
-  uint32_t *rank_tickets;  // [B][kMaxCluster] arrivals of the CTAs of slice rank r; zero at rest
-  uint32_t *seq_tickets;   // [B] finished slice passes of the sampled row; zero at rest
+  unsigned long long *rank_tickets;  // [B][kMaxCluster] arrivals of the rank-r CTAs; zero at rest
+  uint32_t *seq_tickets;   // [B] finished sample passes (+1 for rank 0's last arrival); zero at rest
   float4 *records;         // [B][kMaxCluster][gamma+1] (R_q, R_p, c, flags) as seen by rank r
-  float *slice_totals;     // [B][kMaxCluster] total weight of slice r of the sampled row
-  float *chunk_pre;        // [B][kMaxCluster][kMaxChunks + 1] its exclusive prefix at each chunk start
+  float *chunk_pre;        // [B][kMaxCluster][kMaxChunks + 1] exclusive prefix of slice r of the
+                           // sampled row at each chunk start, then the slice total
   int32_t *status;
 };
 
@@ -252,8 +252,9 @@ struct __align__(16) Shared {
   float Mq, Sq, Mp, Sp, Rq, Rp, maxq, maxp, c, tv, qx, pix;
   int err, delta, accept, need_p2;
   // sequence finish
-  int rank_last;            // last CTA of this slice rank in the sequence: runs the sample pass
-  int seq_last;             // last sample pass of the sequence: draws the token
+  int owner;                // this CTA runs its rank's sample pass of row j*
+  int scan_records;         // j* must be read from the records (gamma + 1 > 32)
+  int seq_last;             // the sequence's last finisher: draws the token
   int jstar, bad, sample_ok;
   float4 rj;                // (R_q, R_p, c, flags) of row j*
   int cross_rank;           // slice holding u * R_tot
@@ -262,7 +263,7 @@ struct __align__(16) Shared {
   float chunk_lo;           // exclusive prefix of the slice at the start of that chunk
   int cross_seg;            // segment of that chunk holding it (-1: none)
   int token;                // the drawn token
-  double t_slice;           // u * R_tot minus the weight before the crossing slice
+  float2 t_slice;           // u * R_tot minus the weight before the crossing slice (hi + lo)
   float t_seg;              // ... minus the weight before the crossing segment
 };
 
@@ -403,8 +404,15 @@ __device__ __forceinline__ float warp_incl_scan(float v, int lane) {
   return v;
 }
 
-// Pass 2 on one chunk: per round, the warp's total weight (lane 31 of an
-// inclusive scan) lands in seg[(c, round, warp)].
+// Sum over a warp (butterfly, the same order in every lane and every call).
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = __fadd_rn(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
+  return v;
+}
+
+// Weights of one chunk in the ring: per round, the warp's total weight (the
+// segment total) lands in seg[(c, round, warp)].
 template <typename E, bool kPair, bool kFull>
 __device__ __forceinline__ void weights_chunk(const E *sq, const E *sp, int n, int c,
                                               const RowScalars &rs, Shared &sh, int lane,
@@ -420,37 +428,71 @@ __device__ __forceinline__ void weights_chunk(const E *sq, const E *sp, int n, i
       if constexpr (kPair) load8_smem(sq, e, n, yq);
       load8_smem(sp, e, n, yp);
     }
-    const float vs = vec_weights<kPair>(yq, yp, rs, w);
-    const float incl = warp_incl_scan(vs, lane);
-    if (lane == 31) sh.seg[(c * kRounds + r) * kNW + warp] = incl;
+    const float tot = warp_sum(vec_weights<kPair>(yq, yp, rs, w));
+    if (lane == 0) sh.seg[(c * kRounds + r) * kNW + warp] = tot;
   }
 }
 
-// exp2(a) for an f64 argument to f32 accuracy without f64 transcendentals:
-// a = hi + lo with hi = f32(a), 2^a ~= exp2f(hi) (1 + lo ln 2).
-__device__ __forceinline__ float exp2_split(double a) {
-  const float hi = static_cast<float>(a);
-  const float lo = static_cast<float>(a - static_cast<double>(hi));
-  return exp2f(hi) * fmaf(lo, 0.69314718f, 1.0f);
+// Double-float arithmetic in f32 (the GPU's f64 rate is a small fraction of
+// its f32 rate): a value is hi + lo with |lo| <= ulp(hi) / 2.  two_sum is
+// Knuth's error-free sum, a + b = s + e exactly; an FMA gives a product's
+// rounding error exactly.
+__device__ __forceinline__ float2 two_sum(float a, float b) {
+  const float s = __fadd_rn(a, b);
+  const float bb = __fsub_rn(s, a);
+  return make_float2(s, __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb)));
+}
+__device__ __forceinline__ float2 df_norm(float hi, float lo) {
+  const float s = __fadd_rn(hi, lo);
+  return make_float2(s, __fsub_rn(lo, __fsub_rn(s, hi)));
+}
+// y (k + kl) as hi + lo
+__device__ __forceinline__ float2 df_mul_k(float y, float k, float kl) {
+  const float p = __fmul_rn(y, k);
+  return make_float2(p, fmaf(y, kl, fmaf(y, k, -p)));
+}
+// a - b, and comparisons with a float
+__device__ __forceinline__ float2 df_sub(float2 a, float b) {
+  const float2 s = two_sum(a.x, -b);
+  return df_norm(s.x, __fadd_rn(s.y, a.y));
+}
+__device__ __forceinline__ bool df_ge(float2 a, float b) { return a.x > b || (a.x == b && a.y >= 0.0f); }
+__device__ __forceinline__ bool df_lt(float2 a, float b) { return a.x < b || (a.x == b && a.y < 0.0f); }
+// the largest float <= a
+__device__ __forceinline__ float df_floor(float2 a) { return a.y < 0.0f ? nextafterf(a.x, -INFINITY) : a.x; }
+// 2^a to f32 accuracy: 2^hi (1 + lo ln 2)
+__device__ __forceinline__ float df_exp2(float2 a) { return exp2f(a.x) * fmaf(a.y, 0.69314718f, 1.0f); }
+
+// log2 of a softmax probability, log2(2^{y k - R} / S) = y k - R - log2 S, as hi + lo
+__device__ __forceinline__ float2 log2_prob(float y, float R, float S, float k, float kl) {
+  const float2 yk = df_mul_k(y, k, kl);
+  const float2 t = two_sum(yk.x, -R);
+  return df_norm(t.x, __fadd_rn(__fadd_rn(t.y, yk.y), -log2f(S)));
 }
 
 // Acceptance of the draft token x (Algorithm 4): a = 1 when delta = 0 or
-// q(x) <= pi(x), else a = [u < pi(x)/q(x)].  log2 p(x) - log2 q(x) is formed in
-// f64 from the logits, so the ratio carries only the f32 error of S_q / S_p.
-// q(x) and pi(x) themselves are evaluated only for the diagnostics output.
-__device__ __forceinline__ void accept_test(Shared &sh, float yqx, float ypx, float u, double kd,
+// q(x) <= pi(x), else a = [u < pi(x)/q(x)].  L = log2 p(x) - log2 q(x)
+//   = (y_p(x) - y_q(x)) log2(e)/T - (R_p - R_q) + log2(S_q / S_p)
+// is formed in double-float from the logits, so the ratio 2^L carries
+// essentially only the f32 error of log2(S_q / S_p).  q(x) and pi(x)
+// themselves are evaluated only for the diagnostics output.
+__device__ __forceinline__ void accept_test(Shared &sh, float yqx, float ypx, float u, float k, float kl,
                                             bool want_probs) {
-  const double lq = static_cast<double>(yqx) * kd - static_cast<double>(sh.Rq);  // log2 q(x) + log2 S_q
-  const double lp = static_cast<double>(ypx) * kd - static_cast<double>(sh.Rp);
   int accept = 1;
   if (sh.delta) {
-    const double L = lp - lq + static_cast<double>(log2f(sh.Sq / sh.Sp));
-    if (L < 0.0) accept = u < exp2_split(L);
+    const float2 d = two_sum(ypx, -yqx);  // y_p(x) - y_q(x), exactly
+    const float2 dk = df_mul_k(d.x, k, kl);
+    const float2 r = two_sum(sh.Rp, -sh.Rq);
+    const float2 s = two_sum(dk.x, -r.x);
+    const float lo = __fadd_rn(__fadd_rn(__fadd_rn(s.y, dk.y), __fsub_rn(__fmul_rn(d.y, k), r.y)),
+                               log2f(sh.Sq / sh.Sp));
+    const float2 L = df_norm(s.x, lo);
+    if (df_lt(L, 0.0f)) accept = u < df_exp2(L);
   }
   sh.accept = accept;
   if (want_probs) {
-    const float qx = exp2_split(lq - static_cast<double>(log2f(sh.Sq)));
-    const float px = exp2_split(lp - static_cast<double>(log2f(sh.Sp)));
+    const float qx = df_exp2(log2_prob(yqx, sh.Rq, sh.Sq, k, kl));
+    const float px = df_exp2(log2_prob(ypx, sh.Rp, sh.Sp, k, kl));
     sh.qx = qx;
     sh.pix = sh.delta ? px : qx;
   }
@@ -568,10 +610,41 @@ __device__ __forceinline__ int stream_again(const Ring<E> &R, Shared &sh, uint32
   return tmo;
 }
 
+// A pass over the slice in reverse chunk order, newest first: a row streamed a
+// moment ago has its last chunks in L2 (and, with `resident`, its last
+// min(kStages, nch) chunks still in the ring in stages c % kStages, which
+// need no copy), while its first chunks may already have been evicted.
+template <typename E, typename Body>
+__device__ __forceinline__ int stream_rev(const Ring<E> &R, Shared &sh, uint32_t &ph, bool resident,
+                                          Body &&body) {
+  const int nch = R.nch;
+  const int nres = resident ? min(kStages, nch) : 0;
+  if (!resident && R.bulk && threadIdx.x == 0)
+    for (int c = nch - 1; c >= max(0, nch - kStages); --c) R.issue(sh, c, c % kStages);
+  int tmo = 0;
+  for (int i = 0; i < nch; ++i) {
+    const int c = nch - 1 - i, s = c % kStages;
+    if (i >= nres) {
+      if (R.bulk) {
+        tmo |= wait_stage(sh, s, ph);
+      } else {
+        R.load_sync(c, s);
+        __syncthreads();
+      }
+    }
+    body(c, s);
+    __syncthreads();  // every thread is done with stage s
+    if (R.bulk && threadIdx.x == 0 && c - kStages >= 0) R.issue(sh, c - kStages, s);
+  }
+  return tmo;
+}
+
 // Residual weights of one slice: per-(chunk, round, warp) totals in sh.seg.
+enum SliceOrder { kAgain, kNewestFirst, kNewestFirstResident };
+
 template <typename E>
 __device__ __forceinline__ int slice_weights(const Ring<E> &R, Shared &sh, uint32_t &ph,
-                                             const RowScalars &rs, bool again, int lane, int warp) {
+                                             const RowScalars &rs, SliceOrder order, int lane, int warp) {
   auto body = [&](int c, int s) {
     const int n = R.chunk_len(c);
     if (R.pair) {
@@ -582,7 +655,8 @@ __device__ __forceinline__ int slice_weights(const Ring<E> &R, Shared &sh, uint3
       else weights_chunk<E, false, false>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
     }
   };
-  return again ? stream_again(R, sh, ph, body) : stream(R, sh, ph, body);
+  if (order == kAgain) return stream_again(R, sh, ph, body);
+  return stream_rev(R, sh, ph, order == kNewestFirstResident, body);
 }
 
 // Thread 0: turn sh.seg[0, nseg) into exclusive prefixes in vocabulary order
@@ -598,27 +672,6 @@ __device__ __forceinline__ float seg_prefix(Shared &sh, int nseg) {
   return acc;
 }
 
-// Segment totals of one chunk straight from global memory (L2): the same
-// vec_weights and warp scans as weights_chunk, so the same values; the totals
-// land in sh.seg[round * kNW + warp].
-template <typename E>
-__device__ __forceinline__ void chunk_segments(const Ring<E> &R, int c, const RowScalars &rs,
-                                               Shared &sh, int lane, int warp) {
-  const int n = R.chunk_len(c);
-  const E *gq = R.gq + static_cast<size_t>(c) * kCH;
-  const E *gp = R.gp + static_cast<size_t>(c) * kCH;
-#pragma unroll
-  for (int r = 0; r < kRounds; ++r) {
-    const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
-    float yq[8], yp[8], w[8];
-    if (R.pair) load8_gmem(gq, e, n, R.bulk, yq);
-    load8_gmem(gp, e, n, R.bulk, yp);
-    const float vs = R.pair ? vec_weights<true>(yq, yp, rs, w) : vec_weights<false>(yq, yp, rs, w);
-    const float incl = warp_incl_scan(vs, lane);
-    if (lane == 31) sh.seg[r * kNW + warp] = incl;
-  }
-}
-
 __device__ __forceinline__ void flag_timeout(Shared &sh, const Params &P) {
   sh.timeout = 1;
   if (P.status) atomicOr(P.status, static_cast<int32_t>(SC_DEV_TIMEOUT));
@@ -631,24 +684,46 @@ __device__ __forceinline__ uint32_t atom_add_acq_rel(uint32_t *p, uint32_t v) {
   asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
   return old;
 }
+__device__ __forceinline__ unsigned long long atom_or_acq_rel(unsigned long long *p, unsigned long long v) {
+  unsigned long long old;
+  asm volatile("atom.acq_rel.gpu.global.or.b64 %0, [%1], %2;" : "=l"(old) : "l"(p), "l"(v) : "memory");
+  return old;
+}
+__device__ __forceinline__ unsigned long long atom_add_acq_rel(unsigned long long *p, unsigned long long v) {
+  unsigned long long old;
+  asm volatile("atom.acq_rel.gpu.global.add.u64 %0, [%1], %2;" : "=l"(old) : "l"(p), "l"(v) : "memory");
+  return old;
+}
 
-// The token inside segment sgi (chunk, round, warp) of a slice: the segment's
-// warp reloads its 8 x 32 logits from global memory (L2), recomputes their
-// weights with vec_weights -- the same values the slice pass summed -- and
-// takes the smallest k whose running sum passes t.  Without t (u R fell past
-// the last boundary by rounding), the segment's last positive weight.
+// With arrivals (bits 0..31) and rejections (bits 32..63) of one slice rank's
+// units, is j* = min{j : a_j = 0} settled -- the first rejection with every
+// earlier position in, or all gamma + 1 positions in without one?  Sets js.
+__device__ __forceinline__ bool jstar_settled(unsigned long long m, int G1, int &js) {
+  const uint32_t arr = static_cast<uint32_t>(m), rej = static_cast<uint32_t>(m >> 32);
+  if (rej) {
+    js = __ffs(rej) - 1;
+    const uint32_t need = js == 31 ? 0xFFFFFFFFu : (2u << js) - 1u;
+    return (arr & need) == need;
+  }
+  js = G1 - 1;
+  return arr == (G1 == 32 ? 0xFFFFFFFFu : (1u << G1) - 1u);
+}
+
+// The token inside segment (round r, this warp) of a chunk held in shared
+// memory (sq, sp; n valid logits): its weights are recomputed with vec_weights
+// -- the values weights_chunk summed -- and the smallest k whose running sum
+// passes t is taken (the smallest k with C_k > u R).  Without t (u R fell past
+// the last boundary by rounding), the segment's last positive weight.  v0 is
+// the vocabulary index of the chunk start.
 template <typename E>
-__device__ __forceinline__ int search_segment(const Ring<E> &R, const RowScalars &rs, int v0,
-                                              int sgi, bool have_t, float t, int lane, int warp) {
-  const int r = (sgi / kNW) % kRounds, c = sgi / (kNW * kRounds);
-  const int n = R.chunk_len(c);
+__device__ __forceinline__ int search_segment(const E *sq, const E *sp, int n, bool pair,
+                                              const RowScalars &rs, int v0, int r, bool have_t,
+                                              float t, int lane, int warp) {
   const int e = 8 * (r * kNT + warp * 32 + lane);
   float yq[8], yp[8], w[8];
-  const E *gq = R.gq + static_cast<size_t>(c) * kCH;
-  const E *gp = R.gp + static_cast<size_t>(c) * kCH;
-  if (R.pair) load8_gmem(gq, e, n, R.bulk, yq);
-  load8_gmem(gp, e, n, R.bulk, yp);
-  const float vs = R.pair ? vec_weights<true>(yq, yp, rs, w) : vec_weights<false>(yq, yp, rs, w);
+  if (pair) load8_smem(sq, e, n, yq);
+  load8_smem(sp, e, n, yp);
+  const float vs = pair ? vec_weights<true>(yq, yp, rs, w) : vec_weights<false>(yq, yp, rs, w);
   const float incl = warp_incl_scan(vs, lane);
   float excl = __shfl_up_sync(0xFFFFFFFFu, incl, 1);
   if (lane == 0) excl = 0.0f;
@@ -667,7 +742,7 @@ __device__ __forceinline__ int search_segment(const Ring<E> &R, const RowScalars
         if (tok < 0 && acc > tt) tok = i;
       }
       if (tok < 0) tok = last;
-      tok = v0 + c * kCH + e + tok;
+      tok = v0 + e + tok;
     }
     tok = __shfl_sync(0xFFFFFFFFu, tok, src);
   } else {
@@ -678,7 +753,7 @@ __device__ __forceinline__ int search_segment(const Ring<E> &R, const RowScalars
     if (lm) {
       const int ln = 31 - __clz(lm);
       const int li = __shfl_sync(0xFFFFFFFFu, last, ln);
-      tok = v0 + c * kCH + 8 * (r * kNT + warp * 32 + ln) + li;
+      tok = v0 + 8 * (r * kNT + warp * 32 + ln) + li;
     }
   }
   return tok;
@@ -844,7 +919,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
             default: sh.delta = 0; break;
           }
           if (pending) sh.need_p2 = 1;
-          else accept_test(sh, yqx, ypx, uj, P.kd, P.row_info != nullptr);
+          else accept_test(sh, yqx, ypx, uj, k, P.kl, P.row_info != nullptr);
         }
       }
       // keep the draft-token logits for a decision after the TV pass
@@ -858,7 +933,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   // ---- TV pass (sc_row_stats, or the OPT band): residual weights of this row
   if (sh.need_p2) {
     const RowScalars rs = {sh.Rq, sh.Rp, k, sh.c};
-    tmo = slice_weights(R, sh, ph, rs, true, lane, warp);
+    tmo = slice_weights(R, sh, ph, rs, kAgain, lane, warp);
     tmo = __syncthreads_or(tmo);
     if (tid == 0) {
       float acc = seg_prefix(sh, R.nch * kRounds * kNW);
@@ -880,7 +955,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
           sh.tv = fminf(1.0f, fmaxf(0.0f, Rtot / sh.Sq));  // Lemma 3: R = S_q D_TV(p, q)
           if (verify) {
             sh.delta = sh.maxq < sh.maxp - P.alpha * sh.tv;  // Eq. 10
-            accept_test(sh, sh.xq, sh.xp, uj, P.kd, P.row_info != nullptr);
+            accept_test(sh, sh.xq, sh.xp, uj, k, P.kl, P.row_info != nullptr);
           }
         }
       }
@@ -898,10 +973,11 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       P.tv[r] = bad ? NAN : sh.tv;
     }
   } else {
-    // ---- record the decision; the last CTA of each slice rank learns j*
+    // ---- record the decision and report it on this slice rank's ticket; the
+    // CTA whose report settles j* samples this rank's slice of row j*
+    float4 *rec = P.records + (static_cast<size_t>(b) * kMaxCluster + rank) * G1;
     if (tid == 0) {
       const int flags = (sh.accept ? 1 : 0) | (sh.err ? 2 : 0);
-      float4 *rec = P.records + (static_cast<size_t>(b) * kMaxCluster + rank) * G1;
       rec[j] = make_float4(sh.Rq, sh.Rp, sh.c, __int_as_float(flags));
       if (rank == 0 && P.row_info) {
         float *ri = P.row_info + (static_cast<size_t>(b) * G1 + j) * SC_ROW_FIELDS;
@@ -914,155 +990,226 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
         ri[SC_ROW_PIX] = sh.pix;
         ri[SC_ROW_CAND] = -1.0f;  // the sequence's finisher fills in row j*
       }
-      uint32_t *tk = P.rank_tickets + static_cast<size_t>(b) * kMaxCluster + rank;
-      const int last = atom_add_acq_rel(tk, 1u) == static_cast<uint32_t>(P.gamma);
-      sh.rank_last = last;
-      if (last) {
-        *tk = 0u;  // every unit of the sequence has arrived on this rank
-        int js = P.gamma, bad = 0;
-        for (int jj = 0; jj <= P.gamma; ++jj) {
-          const int f = __float_as_int(__ldcg(&rec[jj].w));
-          bad |= f & 2;
-          if (jj < P.gamma && !(f & 1) && js == P.gamma) js = jj;  // j* = min{j : a_j = 0}
-        }
-        sh.jstar = js;
-        sh.bad = bad;
-        sh.rj = __ldcg(&rec[js]);
+      unsigned long long *tk = P.rank_tickets + static_cast<size_t>(b) * kMaxCluster + rank;
+      int owner, all_in, js = P.gamma;
+      sh.scan_records = 0;
+      if (G1 <= 32) {
+        // arrival bit j, and rejection bit 32 + j (a_j = 0; the bonus row never rejects)
+        const unsigned long long mine = (1ull << j) | (pair && !sh.accept ? 1ull << (32 + j) : 0ull);
+        const unsigned long long old = atom_or_acq_rel(tk, mine);
+        int js_old;
+        owner = jstar_settled(old | mine, G1, js) && !jstar_settled(old, G1, js_old);
+        all_in = static_cast<uint32_t>(old | mine) == (G1 == 32 ? 0xFFFFFFFFu : (1u << G1) - 1u);
+      } else {
+        // long drafts: the last arrival settles j* and reads it from the records
+        owner = all_in = atom_add_acq_rel(tk, 1ull) == static_cast<unsigned long long>(P.gamma);
+        sh.scan_records = owner;
       }
+      if (all_in) *tk = 0ull;  // every unit of the sequence has reported on this rank
+      sh.owner = owner;
+      sh.jstar = js;
+      // the finisher needs every sample pass and all of rank 0's records
+      sh.seq_last = all_in && rank == 0 &&
+                    atom_add_acq_rel(P.seq_tickets + b, 1u) == static_cast<uint32_t>(C);
     }
     __syncthreads();
+    if (sh.scan_records && warp == 0) {
+      int js = P.gamma;
+      for (int base = 0; base < P.gamma; base += 32) {
+        const int jj = base + lane;
+        const int f = jj < P.gamma ? __float_as_int(__ldcg(&rec[jj].w)) : 1;
+        const unsigned m = __ballot_sync(0xFFFFFFFFu, !(f & 1));
+        if (m) {
+          js = base + __ffs(m) - 1;
+          break;
+        }
+      }
+      if (lane == 0) sh.jstar = js;
+    }
+    if (sh.owner && tid == 0) sh.rj = __ldcg(&rec[sh.jstar]);  // row j*'s record (it is in)
+    __syncthreads();
 
-    if (sh.rank_last) {
+    if (sh.owner) {
       // ---- sample pass: weights of this rank's slice of row j* -- the residual
       // max(0, p - q) of a rejected pair (Algorithm 4), or p of the bonus row
       const int js = sh.jstar;
       const RowScalars rs = {sh.rj.x, sh.rj.y, k, sh.rj.z};
-      float tot_r = 0.0f;
-      if (!sh.bad) {
-        const Ring<E> Rj = make_ring<E>(P, smem_raw, b, js, rank);
-        prime(Rj, sh);
-        tmo = slice_weights(Rj, sh, ph, rs, false, lane, warp);
-        tmo = __syncthreads_or(tmo);
-        if (tid == 0) {
-          tot_r = seg_prefix(sh, Rj.nch * kRounds * kNW);
-          if (tmo) {
-            tot_r = NAN;
-            flag_timeout(sh, P);
-          }
-          float *cp = P.chunk_pre + (static_cast<size_t>(b) * kMaxCluster + rank) * (kMaxChunks + 1);
-          for (int c = 0; c < Rj.nch; ++c) cp[c] = sh.seg[c * kRounds * kNW];
-          cp[Rj.nch] = tot_r;
-        }
-      }
+      const Ring<E> Rj = make_ring<E>(P, smem_raw, b, js, rank);
+      // this unit's own row, untouched since pass 1, still has its last chunks in the ring
+      const bool resident = js == j && !sh.need_p2;
+      tmo = slice_weights(Rj, sh, ph, rs, resident ? kNewestFirstResident : kNewestFirst, lane, warp);
+      tmo = __syncthreads_or(tmo);
       if (tid == 0) {
-        P.slice_totals[static_cast<size_t>(b) * kMaxCluster + rank] = tot_r;
-        const int last = atom_add_acq_rel(P.seq_tickets + b, 1u) == static_cast<uint32_t>(C - 1);
-        sh.seq_last = last;
-        if (last) P.seq_tickets[b] = 0u;
+        float tot_r = seg_prefix(sh, Rj.nch * kRounds * kNW);
+        if (tmo) {
+          tot_r = NAN;
+          flag_timeout(sh, P);
+        }
+        float *cp = P.chunk_pre + (static_cast<size_t>(b) * kMaxCluster + rank) * (kMaxChunks + 1);
+        for (int c = 0; c < Rj.nch; ++c) cp[c] = sh.seg[c * kRounds * kNW];
+        cp[Rj.nch] = tot_r;  // the slice total
+        sh.seq_last = atom_add_acq_rel(P.seq_tickets + b, 1u) == static_cast<uint32_t>(C);
       }
       __syncthreads();
+    }
 
-      if (sh.seq_last) {
-        // ---- the draw: inverse CDF over the slices in rank order, u = u[b][gamma]
-        if (warp == 0) {
-          float tot = 0.0f;
-          if (lane < C) tot = __ldcg(P.slice_totals + static_cast<size_t>(b) * kMaxCluster + lane);
-          const float pre = warp_incl_scan(tot, lane);  // through rank `lane`
-          const float Rtot = __shfl_sync(0xFFFFFFFFu, pre, C - 1);
-          float before = __shfl_up_sync(0xFFFFFFFFu, pre, 1);
-          if (lane == 0) before = 0.0f;
-          const float u = __shfl_sync(0xFFFFFFFFu, ug, 0);
-          const bool ok = !sh.bad && isfinite(Rtot);
-          int cr = -1;
-          double tl = -1.0;
-          if (ok && Rtot > 0.0f) {
-            const double t = static_cast<double>(u) * static_cast<double>(Rtot);
-            const bool cross = lane < C && tot > 0.0f && t >= static_cast<double>(before) &&
-                               t < static_cast<double>(pre);
-            const unsigned cm = __ballot_sync(0xFFFFFFFFu, cross);
-            const unsigned pm = __ballot_sync(0xFFFFFFFFu, lane < C && tot > 0.0f);
-            cr = cm ? __ffs(cm) - 1 : 31 - __clz(pm);
-            const float bcr = __shfl_sync(0xFFFFFFFFu, before, cr);
-            tl = cm ? t - static_cast<double>(bcr) : -1.0;
+    if (sh.seq_last) {
+      // ---- the draw (the ring is idle: stage 0 holds the chunk prefixes of
+      // every slice, the last stage the chunk searched)
+      constexpr int kCP = kMaxChunks + 1;
+      float *cpall = reinterpret_cast<float *>(smem_raw);  // [C][kCP]
+      if (tid == 0) P.seq_tickets[b] = 0u;  // every report of the sequence is in
+      // one round of loads: every slice's chunk prefixes (ending in its total) ...
+      const float *cpg = P.chunk_pre + static_cast<size_t>(b) * kMaxCluster * kCP;
+      for (int i = tid; i < C * kCP; i += kNT) {
+        const int r = i / kCP, c = i % kCP;
+        const int len = max(0, min(P.L, P.V - r * P.L));
+        if (c <= (len + kCH - 1) / kCH) cpall[i] = __ldcg(cpg + i);
+      }
+      // ... and, in warp 0, j* and the error flags from rank 0's records
+      if (warp == 0) {
+        const float4 *rec0 = P.records + static_cast<size_t>(b) * kMaxCluster * G1;
+        int js = P.gamma, bad = 0;
+        float4 rj = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+        for (int base = 0; base <= P.gamma; base += 32) {
+          const int jj = base + lane;
+          const float4 rv = jj <= P.gamma ? __ldcg(&rec0[jj]) : make_float4(0.0f, 0.0f, 0.0f, __int_as_float(1));
+          const int f = __float_as_int(rv.w);
+          bad |= __any_sync(0xFFFFFFFFu, f & 2);
+          const unsigned m = __ballot_sync(0xFFFFFFFFu, jj < P.gamma && !(f & 1));
+          const int hit = js == P.gamma ? (m ? base + __ffs(m) - 1 : (P.gamma - base < 32 ? P.gamma : -1)) : -1;
+          if (hit >= 0) {
+            js = hit;
+            const int src = hit - base;
+            rj = make_float4(__shfl_sync(0xFFFFFFFFu, rv.x, src), __shfl_sync(0xFFFFFFFFu, rv.y, src),
+                             __shfl_sync(0xFFFFFFFFu, rv.z, src), __shfl_sync(0xFFFFFFFFu, rv.w, src));
           }
-          if (lane == 0) {
-            sh.sample_ok = ok;
-            sh.cross_rank = cr;
-            sh.t_slice = tl;
-            sh.token = -1;
+        }
+        if (lane == 0) {
+          sh.jstar = js;
+          sh.bad = bad;
+          sh.rj = rj;
+        }
+      }
+      __syncthreads();
+      const int js = sh.jstar;
+      const RowScalars rs = {sh.rj.x, sh.rj.y, k, sh.rj.z};
+      // ---- inverse CDF over the slices in rank order, u = u[b][gamma], then
+      // over the chunks of the crossing slice
+      if (warp == 0) {
+        auto nch_of = [&](int r) {
+          const int len = max(0, min(P.L, P.V - r * P.L));
+          return (len + kCH - 1) / kCH;
+        };
+        const float tot = lane < C ? cpall[lane * kCP + nch_of(lane)] : 0.0f;
+        const float pre = warp_incl_scan(tot, lane);  // through rank `lane`
+        const float Rtot = __shfl_sync(0xFFFFFFFFu, pre, C - 1);
+        float before = __shfl_up_sync(0xFFFFFFFFu, pre, 1);
+        if (lane == 0) before = 0.0f;
+        const float u = __shfl_sync(0xFFFFFFFFu, ug, 0);
+        const bool ok = !sh.bad && isfinite(Rtot);
+        int cr = -1, cc = -1, clast = -1;
+        float2 tl = make_float2(-1.0f, 0.0f);  // (negative: u R fell past the last boundary)
+        if (ok && Rtot > 0.0f) {
+          const float th = __fmul_rn(u, Rtot);
+          const float2 t = make_float2(th, fmaf(u, Rtot, -th));  // u R_tot, exactly
+          const bool cross = lane < C && tot > 0.0f && df_ge(t, before) && df_lt(t, pre);
+          const unsigned cm = __ballot_sync(0xFFFFFFFFu, cross);
+          const unsigned pm = __ballot_sync(0xFFFFFFFFu, lane < C && tot > 0.0f);
+          cr = cm ? __ffs(cm) - 1 : 31 - __clz(pm);
+          const float bcr = __shfl_sync(0xFFFFFFFFu, before, cr);
+          if (cm) tl = df_sub(t, bcr);
+          // the chunk of slice cr holding tl (or, past a rounding gap, its last chunk with weight)
+          const float *cp = cpall + cr * kCP;
+          const int nch = nch_of(cr);
+          for (int base = 0; base < nch; base += 32) {
+            const int c = base + lane;
+            const float lo = c < nch ? cp[c] : 0.0f, hi = c < nch ? cp[c + 1] : 0.0f;
+            const bool pos = c < nch && hi > lo;
+            const unsigned mi = __ballot_sync(0xFFFFFFFFu, pos && df_ge(tl, lo) && df_lt(tl, hi));
+            const unsigned mp = __ballot_sync(0xFFFFFFFFu, pos);
+            if (cc < 0 && mi) cc = base + __ffs(mi) - 1;
+            if (mp) clast = base + 31 - __clz(mp);
           }
+        }
+        if (lane == 0) {
+          sh.sample_ok = ok;
+          sh.cross_rank = cr;
+          sh.t_slice = tl;
+          sh.token = -1;
+          sh.cross_chunk = cc >= 0 ? cc : clast;
+          sh.have_t = cc >= 0;
+          sh.chunk_lo = sh.cross_chunk >= 0 ? cpall[cr * kCP + sh.cross_chunk] : 0.0f;
+        }
+      }
+      __syncthreads();
+      const int cr = sh.cross_rank, cc = sh.cross_chunk;
+      if (cr >= 0 && cc >= 0) {
+        // the chunk's weights again, by the code the sample pass ran (the same values)
+        const Ring<E> Rc = make_ring<E>(P, smem_raw, b, js, cr);
+        const int sl = kStages - 1, n = Rc.chunk_len(cc);
+        if (Rc.bulk) {
+          if (tid == 0) Rc.issue(sh, cc, sl);
+          tmo = wait_stage(sh, sl, ph);
+        } else {
+          tmo = 0;
+          Rc.load_sync(cc, sl);
+        }
+        tmo = __syncthreads_or(tmo);
+        if (Rc.pair) {
+          if (n == kCH) weights_chunk<E, true, true>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
+          else weights_chunk<E, true, false>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
+        } else {
+          if (n == kCH) weights_chunk<E, false, true>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
+          else weights_chunk<E, false, false>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
+        }
+        if (tmo && tid == 0) {
+          flag_timeout(sh, P);
+          sh.sample_ok = 0;
         }
         __syncthreads();
-        const int cr = sh.cross_rank;
-        if (cr >= 0) {
-          // the chunk of the crossing slice that holds t, from the stored chunk
-          // prefixes (or, past a rounding gap, the last chunk with weight)
-          const Ring<E> Rc = make_ring<E>(P, smem_raw, b, js, cr);
-          if (tid == 0) {
-            const float *cp = P.chunk_pre + (static_cast<size_t>(b) * kMaxCluster + cr) * (kMaxChunks + 1);
-            const double tl = sh.t_slice;
-            int cc = -1, clast = -1;
-            for (int c = 0; c < Rc.nch; ++c) {
-              const float lo = __ldcg(cp + c), hi = __ldcg(cp + c + 1);
-              if (hi > lo) {
-                clast = c;
-                if (cc < 0 && tl >= static_cast<double>(lo) && tl < static_cast<double>(hi)) cc = c;
-              }
-            }
-            sh.cross_chunk = cc >= 0 ? cc : clast;
-            sh.have_t = cc >= 0;
-            sh.chunk_lo = sh.cross_chunk >= 0 ? __ldcg(cp + sh.cross_chunk) : 0.0f;
-          }
-          __syncthreads();
-          const int cc = sh.cross_chunk;
-          if (cc >= 0) {
-            chunk_segments(Rc, cc, rs, sh, lane, warp);
-            __syncthreads();
-            constexpr int kSegC = kRounds * kNW;  // segments per chunk
-            if (tid == 0) {
-              // exclusive prefixes continue from the chunk's stored start, as in the slice pass
-              float acc = sh.chunk_lo;
-              for (int i = 0; i < kSegC; ++i) {
-                const float t = sh.seg[i];
-                sh.seg[i] = acc;
-                acc = __fadd_rn(acc, t);
-              }
-              sh.seg[kSegC] = acc;
-              const double tl = sh.t_slice;
-              int sgi = -1;
-              if (sh.have_t)
-                for (int i = 0; i < kSegC; ++i)
-                  if (tl >= static_cast<double>(sh.seg[i]) && tl < static_cast<double>(sh.seg[i + 1]) &&
-                      sh.seg[i + 1] > sh.seg[i]) {
-                    sgi = i;
-                    break;
-                  }
-              sh.cross_seg = sgi;
-              sh.t_seg = sgi >= 0 ? __double2float_rd(tl - static_cast<double>(sh.seg[sgi])) : 0.0f;
-            }
-            __syncthreads();
-            int sgi = sh.cross_seg;
-            if (sgi < 0) {
-              // no t inside the chunk: its last segment with weight
-              for (int i = kSegC - 1; i >= 0; --i)
-                if (sh.seg[i + 1] > sh.seg[i]) { sgi = i; break; }
-            }
-            if (sgi >= 0 && warp == sgi % kNW) {
-              const int tok = search_segment(Rc, rs, cr * P.L, cc * kSegC + sgi, sh.cross_seg >= 0,
-                                             sh.t_seg, lane, warp);
-              if (lane == 0) sh.token = tok;
-            }
-            __syncthreads();
-          }
-        }
+        constexpr int kSegC = kRounds * kNW;  // segments per chunk
         if (tid == 0) {
-          const bool ok = sh.sample_ok != 0;
-          P.num_accepted[b] = ok ? js : 0;
-          P.next_token[b] = ok ? sh.token : -1;
-          if (ok && P.row_info)
-            P.row_info[(static_cast<size_t>(b) * G1 + js) * SC_ROW_FIELDS + SC_ROW_CAND] =
-                static_cast<float>(sh.token);
+          // exclusive prefixes continue from the chunk's stored start, as in the sample pass
+          float acc = sh.chunk_lo;
+          for (int i = 0; i < kSegC; ++i) {
+            const float t = sh.seg[i];
+            sh.seg[i] = acc;
+            acc = __fadd_rn(acc, t);
+          }
+          sh.seg[kSegC] = acc;
+          const float2 tl = sh.t_slice;
+          int sgi = -1;
+          if (sh.have_t)
+            for (int i = 0; i < kSegC; ++i)
+              if (df_ge(tl, sh.seg[i]) && df_lt(tl, sh.seg[i + 1]) && sh.seg[i + 1] > sh.seg[i]) {
+                sgi = i;
+                break;
+              }
+          sh.cross_seg = sgi;
+          sh.t_seg = sgi >= 0 ? df_floor(df_sub(tl, sh.seg[sgi])) : 0.0f;
         }
+        __syncthreads();
+        int sgi = sh.cross_seg;
+        if (sgi < 0) {
+          // no t inside the chunk: its last segment with weight
+          for (int i = kSegC - 1; i >= 0; --i)
+            if (sh.seg[i + 1] > sh.seg[i]) { sgi = i; break; }
+        }
+        if (sgi >= 0 && warp == sgi % kNW) {
+          const int tok = search_segment(Rc.q(sl), Rc.p(sl), n, Rc.pair, rs, cr * P.L + cc * kCH,
+                                         sgi / kNW, sh.cross_seg >= 0, sh.t_seg, lane, warp);
+          if (lane == 0) sh.token = tok;
+        }
+        __syncthreads();
+      }
+      if (tid == 0) {
+        const bool ok = sh.sample_ok != 0;
+        P.num_accepted[b] = ok ? js : 0;
+        P.next_token[b] = ok ? sh.token : -1;
+        if (ok && P.row_info)
+          P.row_info[(static_cast<size_t>(b) * G1 + js) * SC_ROW_FIELDS + SC_ROW_CAND] =
+              static_cast<float>(sh.token);
       }
     }
   }
@@ -1087,10 +1234,10 @@ std::mutex g_mu;
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // Workspace of sc_verify for B sequences of gamma drafts: slice-rank tickets,
-// sequence tickets (both zero between calls), then unit records, slice totals
-// and chunk prefixes (written before they are read).
+// sequence tickets (both zero between calls), then unit records and chunk
+// prefixes (written before they are read).
 struct WsLayout {
-  size_t rank_tickets, seq_tickets, zeroed, records, slice_totals, chunk_pre, total;
+  size_t rank_tickets, seq_tickets, zeroed, records, chunk_pre, total;
 };
 
 constexpr size_t align256(size_t x) { return (x + 255) / 256 * 256; }
@@ -1098,11 +1245,10 @@ constexpr size_t align256(size_t x) { return (x + 255) / 256 * 256; }
 constexpr WsLayout ws_layout(size_t B, size_t units) {
   WsLayout w = {};
   w.rank_tickets = 0;
-  w.seq_tickets = align256(4 * kMaxCluster * B);
+  w.seq_tickets = align256(8 * kMaxCluster * B);
   w.zeroed = w.seq_tickets + align256(4 * B);
   w.records = w.zeroed;
-  w.slice_totals = w.records + align256(16 * kMaxCluster * units);
-  w.chunk_pre = w.slice_totals + align256(4 * kMaxCluster * B);
+  w.chunk_pre = w.records + align256(16 * kMaxCluster * units);
   w.total = w.chunk_pre + align256(4 * kMaxCluster * (kMaxChunks + 1) * B);
   return w;
 }
@@ -1142,6 +1288,13 @@ int pick_layout(int V, int units, int sms, int *C_out, int *L_out) {
     return 0;
   }
   return -1;
+}
+
+// k = log2(e) / T as an f32 value plus its f32 remainder.
+void set_k(Params &P, float temperature) {
+  const double kd = 1.4426950408889634 / static_cast<double>(temperature);
+  P.k = static_cast<float>(kd);
+  P.kl = static_cast<float>(kd - static_cast<double>(P.k));
 }
 
 bool device_accessible(const void *p) {
@@ -1294,8 +1447,7 @@ int sc_verify_rows(const void *draft_logits, const void *target_logits, sc_dtype
   P.rule = static_cast<int>(rule);
   P.alpha = alpha;
   P.temperature = temperature;
-  P.k = static_cast<float>(1.4426950408889634 / static_cast<double>(temperature));
-  P.kd = 1.4426950408889634 / static_cast<double>(temperature);
+  set_k(P, temperature);
   P.mode = kVerify;
   P.num_accepted = num_accepted;
   P.next_token = next_token;
@@ -1303,10 +1455,9 @@ int sc_verify_rows(const void *draft_logits, const void *target_logits, sc_dtype
   P.status = device_status;
   unsigned char *ws = static_cast<unsigned char *>(workspace);
   const WsLayout wl = ws_layout(static_cast<size_t>(B), static_cast<size_t>(B) * (gamma + 1));
-  P.rank_tickets = reinterpret_cast<uint32_t *>(ws + wl.rank_tickets);
+  P.rank_tickets = reinterpret_cast<unsigned long long *>(ws + wl.rank_tickets);
   P.seq_tickets = reinterpret_cast<uint32_t *>(ws + wl.seq_tickets);
   P.records = reinterpret_cast<float4 *>(ws + wl.records);
-  P.slice_totals = reinterpret_cast<float *>(ws + wl.slice_totals);
   P.chunk_pre = reinterpret_cast<float *>(ws + wl.chunk_pre);
   const int units = B * (gamma + 1);
   return dtype == SC_BF16 ? launch<uint16_t>(P, stream, units) : launch<float>(P, stream, units);
@@ -1336,8 +1487,7 @@ int sc_row_stats(const void *draft_logits, const void *target_logits, sc_dtype d
   P.gamma = gamma;
   P.V = V;
   P.temperature = temperature;
-  P.k = static_cast<float>(1.4426950408889634 / static_cast<double>(temperature));
-  P.kd = 1.4426950408889634 / static_cast<double>(temperature);
+  set_k(P, temperature);
   P.mode = kStats;
   P.max_q = max_q;
   P.max_p = max_p;
