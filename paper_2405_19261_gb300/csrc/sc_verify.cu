@@ -163,11 +163,32 @@ __device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t by
       : "memory");
 }
 
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
 __device__ __forceinline__ void cluster_arrive() {
   asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
 }
 __device__ __forceinline__ void cluster_wait() {
   asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// Stores into the shared memory of the cluster's CTA `rank` (same offset as p here).
+__device__ __forceinline__ uint32_t peer_addr(const void *p, int rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(p)), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void st_peer(uint32_t a, float4 v) {
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(a), "f"(v.x), "f"(v.y), "f"(v.z),
+               "f"(v.w)
+               : "memory");
+}
+__device__ __forceinline__ void st_peer(uint32_t a, float2 v) {
+  asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(a), "f"(v.x), "f"(v.y) : "memory");
+}
+__device__ __forceinline__ void st_peer(uint32_t a, float v) {
+  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(a), "f"(v) : "memory");
 }
 
 // ------------------------------------------------------------------ logit types
@@ -239,13 +260,12 @@ __device__ __forceinline__ void load8_gmem(const E *g, int e, int n, bool vec, f
 
 struct __align__(16) Shared {
   uint64_t full[kStages];
-  // exchange 1: (m_q, s_q, m_p, s_p) of this CTA, raw logits at the draft token
-  float4 part_ms;
-  float2 part_x;
-  // exchange 2 (TV pass): this CTA's total residual weight
-  float part_r;
+  // cluster exchanges, written by every CTA of the cluster into slot [its rank]:
+  float4 all_ms[kMaxCluster];  // 1: (m_q, s_q, m_p, s_p) of the slice
+  float2 all_x[kMaxCluster];   // 1: raw logits at the draft token, if in the slice
+  float all_r[kMaxCluster];    // 2 (TV pass): the slice's total residual weight
   int timeout;
-  float red[kNW][4];
+  float4 red[kNW];          // (m_q, s_q, m_p, s_p) of each warp
   float seg[kEntries + 1];  // per-(chunk, round, warp) weights, then exclusive prefixes
   float xq, xp;             // raw logits at the draft token, when in this slice
   // row state, identical in every CTA of the cluster
@@ -279,12 +299,41 @@ __device__ __forceinline__ float max3(float a, float b, float c) {
 // logit's own term is 2^{fma(M, k, -R)}, not exactly 1, and is treated so).
 __device__ __forceinline__ float refk(float m, float k) { return fmaxf(__fmul_rn(m, k), -1e30f); }
 
-// Merge two (max, sum) partials; each sum is relative to refk of its max.
-__device__ __forceinline__ void ms_combine(float &m, float &s, float m2, float s2, float k) {
-  const float mn = fmaxf(m, m2);
-  const float rn = refk(mn, k);
-  s = s * ex2(refk(m, k) - rn) + s2 * ex2(refk(m2, k) - rn);
-  m = mn;
+// Merge the (max, sum) partials held by the 32 lanes of a warp (each sum is
+// relative to refk of its own max): the largest max M by a shuffle tree, then
+// every lane's sum rescaled to refk(M) by ONE exponential, then a butterfly
+// sum -- a short dependent chain, which matters when this warp shares its SM
+// with streaming warps.  Every lane ends with (M, S); identical inputs give
+// identical results in every CTA.  A lane with s = 0 contributes 0.
+__device__ __forceinline__ void warp_ms_merge(float &m, float &s, float k) {
+  float M = m;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xFFFFFFFFu, M, o));
+  float t = s * ex2(refk(m, k) - refk(M, k));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) t = __fadd_rn(t, __shfl_xor_sync(0xFFFFFFFFu, t, o));
+  m = M;
+  s = t;
+}
+
+// Merge n (m_q, s_q, m_p, s_p) partials in index order, in one thread: the
+// largest maxima first, then every sum rescaled to refk of its row's maximum
+// by one exponential (all independent).  Shared-memory reads and arithmetic
+// only: no shuffles, which queue behind the streaming warps' shared-memory
+// loads on the same SM.
+__device__ __forceinline__ float4 merge_partials(const float4 *v, int n, float k) {
+  float Mq = -FLT_MAX, Mp = -FLT_MAX;
+  for (int i = 0; i < n; ++i) {
+    Mq = fmaxf(Mq, v[i].x);
+    Mp = fmaxf(Mp, v[i].z);
+  }
+  const float Rq = refk(Mq, k), Rp = refk(Mp, k);
+  float Sq = 0.0f, Sp = 0.0f;
+  for (int i = 0; i < n; ++i) {
+    Sq = fmaf(v[i].y, ex2(refk(v[i].x, k) - Rq), Sq);
+    Sp = fmaf(v[i].w, ex2(refk(v[i].z, k) - Rp), Sp);
+  }
+  return make_float4(Mq, Sq, Mp, Sp);
 }
 
 // Pass 1 on one row of one chunk: this thread's kRounds vectors, online
@@ -583,33 +632,6 @@ __device__ __forceinline__ int stream(const Ring<E> &R, Shared &sh, uint32_t &ph
   return tmo;
 }
 
-// Second pass over the slice just streamed: its last min(kStages, nch) chunks
-// are still in the ring, so they are processed first with no copy; every stage
-// they free is refilled with the next chunk from the start of the slice
-// (L2-resident), so the first refill's latency overlaps work.
-template <typename E, typename Body>
-__device__ __forceinline__ int stream_again(const Ring<E> &R, Shared &sh, uint32_t &ph, Body &&body) {
-  const int nch = R.nch;
-  const int nres = min(kStages, nch);
-  int tmo = 0;
-  for (int it = 0; it < nch; ++it) {
-    const int s = (nch - nres + it % nres) % kStages;
-    const int c = it < nres ? nch - nres + it : it - nres;
-    if (it >= nres) {
-      if (R.bulk) {
-        tmo |= wait_stage(sh, s, ph);
-      } else {
-        R.load_sync(c, s);
-        __syncthreads();
-      }
-    }
-    body(c, s);
-    __syncthreads();  // every thread is done with stage s
-    if (R.bulk && threadIdx.x == 0 && it < nch - nres) R.issue(sh, it, s);
-  }
-  return tmo;
-}
-
 // A pass over the slice in reverse chunk order, newest first: a row streamed a
 // moment ago has its last chunks in L2 (and, with `resident`, its last
 // min(kStages, nch) chunks still in the ring in stages c % kStages, which
@@ -640,7 +662,7 @@ __device__ __forceinline__ int stream_rev(const Ring<E> &R, Shared &sh, uint32_t
 }
 
 // Residual weights of one slice: per-(chunk, round, warp) totals in sh.seg.
-enum SliceOrder { kAgain, kNewestFirst, kNewestFirstResident };
+enum SliceOrder { kNewestFirst, kNewestFirstResident };
 
 template <typename E>
 __device__ __forceinline__ int slice_weights(const Ring<E> &R, Shared &sh, uint32_t &ph,
@@ -655,7 +677,6 @@ __device__ __forceinline__ int slice_weights(const Ring<E> &R, Shared &sh, uint3
       else weights_chunk<E, false, false>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
     }
   };
-  if (order == kAgain) return stream_again(R, sh, ph, body);
   return stream_rev(R, sh, ph, order == kNewestFirstResident, body);
 }
 
@@ -804,6 +825,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     if (pair) x = P.tokens[static_cast<size_t>(b) * P.gamma + j];
   }
   __syncthreads();
+  cluster_arrive_relaxed();  // this CTA has started (peers may store into it after their wait)
 
   // ---- pass 1: online max and sum of exponentials
   const float k = P.k;
@@ -826,141 +848,121 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   });
   float s_q = s2q.x + s2q.y, s_p = s2p.x + s2p.y;
   tmo = __syncthreads_or(tmo);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float m2q = __shfl_down_sync(0xFFFFFFFFu, mq, o), s2q = __shfl_down_sync(0xFFFFFFFFu, s_q, o);
-    const float m2p = __shfl_down_sync(0xFFFFFFFFu, mp, o), s2p = __shfl_down_sync(0xFFFFFFFFu, s_p, o);
-    ms_combine(mq, s_q, m2q, s2q, k);
-    ms_combine(mp, s_p, m2p, s2p, k);
-  }
-  if (lane == 0) {
-    sh.red[warp][0] = mq; sh.red[warp][1] = s_q;
-    sh.red[warp][2] = mp; sh.red[warp][3] = s_p;
-  }
+  warp_ms_merge(mq, s_q, k);
+  warp_ms_merge(mp, s_p, k);
+  if (lane == 0) sh.red[warp] = make_float4(mq, s_q, mp, s_p);
   __syncthreads();
+  // ---- exchange 1: thread 0 merges the warp partials into the slice partial
+  // and pushes it into every CTA of the cluster; one barrier; then every read
+  // is local, and thread 0 decides
+  float4 part = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
   if (tid == 0) {
-    float a = sh.red[0][0], as = sh.red[0][1], c = sh.red[0][2], cs = sh.red[0][3];
-    for (int w = 1; w < kNW; ++w) {
-      ms_combine(a, as, sh.red[w][0], sh.red[w][1], k);
-      ms_combine(c, cs, sh.red[w][2], sh.red[w][3], k);
-    }
+    part = merge_partials(sh.red, kNW, k);
     if (tmo) {
-      as = NAN;
-      cs = NAN;
+      part.y = NAN;
+      part.w = NAN;
       flag_timeout(sh, P);
     }
-    sh.part_ms = make_float4(a, as, c, cs);
-    sh.part_x = make_float2(sh.xq, sh.xp);
   }
-  cluster.sync();  // exchange 1
+  cluster_wait();  // every CTA of the cluster has started
+  if (tid == 0) {
+    const float2 xv = make_float2(sh.xq, sh.xp);
+    for (int r = 0; r < C; ++r) {
+      st_peer(peer_addr(&sh.all_ms[rank], r), part);
+      st_peer(peer_addr(&sh.all_x[rank], r), xv);
+    }
+  }
+  cluster_arrive();
+  cluster_wait();
 
-  if (warp == 0) {
-    float4 v = make_float4(-FLT_MAX, 0.0f, -FLT_MAX, 0.0f);
-    float2 xv = make_float2(NAN, NAN);
-    if (lane < C) {
-      v = *cluster.map_shared_rank(&sh.part_ms, lane);
-      xv = *cluster.map_shared_rank(&sh.part_x, lane);
+  if (tid == 0) {  // thread 0 also holds the prefetched scalars
+    const float4 v = merge_partials(sh.all_ms, C, k);  // the row's M and S over the cluster
+    const float a = v.x, as = v.y, c = v.z, cs = v.w;
+    const float2 xv = sh.all_x[(x >= 0 && x < P.V) ? x / P.L : 0];
+    const float yqx = xv.x, ypx = xv.y;
+    // S = sum_v 2^{y_v k - R} with R = fl(M k); the max logit's own term is
+    // 2^{fma(M, k, -R)}, so max_v q(v) = 2^{fma(M, k, -R)} / S.
+    const float Rq = refk(a, k), Rp = refk(c, k);
+    sh.Mq = a; sh.Sq = as; sh.Mp = c; sh.Sp = cs;
+    sh.Rq = Rq;
+    sh.Rp = Rp;
+    sh.maxq = ex2(fmaf(a, k, -Rq)) / as;
+    sh.maxp = ex2(fmaf(c, k, -Rp)) / cs;
+    int err = 0;
+    const bool okq = !pair || (isfinite(a) && isfinite(as) && as > 0.0f);
+    const bool okp = isfinite(c) && isfinite(cs) && cs > 0.0f;
+    if (!(okq && okp)) err |= SC_DEV_BAD_LOGIT;
+    if (verify) {
+      if (!(uj >= 0.0f && uj < 1.0f)) err |= SC_DEV_BAD_UNIFORM;
+      if (pair && (x < 0 || x >= P.V)) err |= SC_DEV_BAD_TOKEN;
     }
-    float a = v.x, as = v.y, c = v.z, cs = v.w;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float a2 = __shfl_down_sync(0xFFFFFFFFu, a, o), as2 = __shfl_down_sync(0xFFFFFFFFu, as, o);
-      const float c2 = __shfl_down_sync(0xFFFFFFFFu, c, o), cs2 = __shfl_down_sync(0xFFFFFFFFu, cs, o);
-      ms_combine(a, as, a2, as2, k);
-      ms_combine(c, cs, c2, cs2, k);
-    }
-    const int xl = __shfl_sync(0xFFFFFFFFu, x, 0);
-    const int xr = (xl >= 0 && xl < P.V) ? xl / P.L : 0;
-    const float yqx = __shfl_sync(0xFFFFFFFFu, xv.x, xr);
-    const float ypx = __shfl_sync(0xFFFFFFFFu, xv.y, xr);
-    if (lane == 0) {  // thread 0: holds the prefetched scalars
-      // S = sum_v 2^{y_v k - R} with R = fl(M k); the max logit's own term is
-      // 2^{fma(M, k, -R)}, so max_v q(v) = 2^{fma(M, k, -R)} / S.
-      const float Rq = refk(a, k), Rp = refk(c, k);
-      sh.Mq = a; sh.Sq = as; sh.Mp = c; sh.Sp = cs;
-      sh.Rq = Rq;
-      sh.Rp = Rp;
-      sh.maxq = ex2(fmaf(a, k, -Rq)) / as;
-      sh.maxp = ex2(fmaf(c, k, -Rp)) / cs;
-      int err = 0;
-      const bool okq = !pair || (isfinite(a) && isfinite(as) && as > 0.0f);
-      const bool okp = isfinite(c) && isfinite(cs) && cs > 0.0f;
-      if (!(okq && okp)) err |= SC_DEV_BAD_LOGIT;
-      if (verify) {
-        if (!(uj >= 0.0f && uj < 1.0f)) err |= SC_DEV_BAD_UNIFORM;
-        if (pair && (x < 0 || x >= P.V)) err |= SC_DEV_BAD_TOKEN;
-      }
-      if (err && P.status && rank == 0) atomicOr(P.status, err);
-      sh.err = err;
-      sh.delta = 0;
-      sh.need_p2 = 0;
-      sh.accept = 0;
-      sh.tv = -1.0f;
-      sh.qx = 0.0f;
-      sh.pix = 0.0f;
-      sh.c = pair && !err ? log2f(as / cs) : 0.0f;
-      if (!err && pair) {
-        if (!verify) {
-          sh.need_p2 = 1;  // sc_row_stats: TV of every pair
-        } else {
-          // deferral rule (Table 1)
-          const float maxq = sh.maxq, maxp = sh.maxp, al = P.alpha;
-          bool pending = false;
-          switch (P.rule) {
-            case SC_RULE_CHOW: sh.delta = maxq < 1.0f - al; break;  // Eq. 2
-            case SC_RULE_DIFF: sh.delta = maxq < maxp - al; break;  // Eq. 5
-            case SC_RULE_OPT:                                       // Eq. 10
-              // alpha * TV lies in [0, alpha]: TV decides only inside that band
-              if (!(maxq < maxp)) sh.delta = 0;
-              else if (maxq < maxp - al) sh.delta = 1;
-              else pending = true;
-              break;
-            case SC_RULE_ALWAYS_DEFER: sh.delta = 1; break;
-            default: sh.delta = 0; break;
-          }
-          if (pending) sh.need_p2 = 1;
-          else accept_test(sh, yqx, ypx, uj, k, P.kl, P.row_info != nullptr);
+    if (err && P.status && rank == 0) atomicOr(P.status, err);
+    sh.err = err;
+    sh.delta = 0;
+    sh.need_p2 = 0;
+    sh.accept = 0;
+    sh.tv = -1.0f;
+    sh.qx = 0.0f;
+    sh.pix = 0.0f;
+    sh.c = pair && !err ? log2f(as / cs) : 0.0f;
+    if (!err && pair) {
+      if (!verify) {
+        sh.need_p2 = 1;  // sc_row_stats: TV of every pair
+      } else {
+        // deferral rule (Table 1)
+        const float maxq = sh.maxq, maxp = sh.maxp, al = P.alpha;
+        bool pending = false;
+        switch (P.rule) {
+          case SC_RULE_CHOW: sh.delta = maxq < 1.0f - al; break;  // Eq. 2
+          case SC_RULE_DIFF: sh.delta = maxq < maxp - al; break;  // Eq. 5
+          case SC_RULE_OPT:                                       // Eq. 10
+            // alpha * TV lies in [0, alpha]: TV decides only inside that band
+            if (!(maxq < maxp)) sh.delta = 0;
+            else if (maxq < maxp - al) sh.delta = 1;
+            else pending = true;
+            break;
+          case SC_RULE_ALWAYS_DEFER: sh.delta = 1; break;
+          default: sh.delta = 0; break;
         }
+        if (pending) sh.need_p2 = 1;
+        else accept_test(sh, yqx, ypx, uj, k, P.kl, P.row_info != nullptr);
       }
-      // keep the draft-token logits for a decision after the TV pass
-      sh.xq = yqx;
-      sh.xp = ypx;
     }
+    // keep the draft-token logits for a decision after the TV pass
+    sh.xq = yqx;
+    sh.xp = ypx;
   }
   __syncthreads();
-  if (!sh.need_p2) cluster_arrive();  // no further reads of peer shared memory
 
   // ---- TV pass (sc_row_stats, or the OPT band): residual weights of this row
   if (sh.need_p2) {
     const RowScalars rs = {sh.Rq, sh.Rp, k, sh.c};
-    tmo = slice_weights(R, sh, ph, rs, kAgain, lane, warp);
+    tmo = slice_weights(R, sh, ph, rs, kNewestFirstResident, lane, warp);
     tmo = __syncthreads_or(tmo);
+    // exchange 2: push the slice total, one barrier, local reads
     if (tid == 0) {
       float acc = seg_prefix(sh, R.nch * kRounds * kNW);
       if (tmo) {
         acc = NAN;
         flag_timeout(sh, P);
       }
-      sh.part_r = acc;
+      for (int r = 0; r < C; ++r) st_peer(peer_addr(&sh.all_r[rank], r), acc);
     }
-    cluster.sync();  // exchange 2
-    if (warp == 0) {
-      float tot = 0.0f;
-      if (lane < C) tot = *cluster.map_shared_rank(&sh.part_r, lane);
-      const float Rtot = __shfl_sync(0xFFFFFFFFu, warp_incl_scan(tot, lane), C - 1);
-      if (lane == 0) {
-        if (!isfinite(Rtot)) {
-          sh.err |= SC_DEV_TIMEOUT;
-        } else {
-          sh.tv = fminf(1.0f, fmaxf(0.0f, Rtot / sh.Sq));  // Lemma 3: R = S_q D_TV(p, q)
-          if (verify) {
-            sh.delta = sh.maxq < sh.maxp - P.alpha * sh.tv;  // Eq. 10
-            accept_test(sh, sh.xq, sh.xp, uj, k, P.kl, P.row_info != nullptr);
-          }
+    cluster_arrive();
+    cluster_wait();
+    if (tid == 0) {
+      float Rtot = 0.0f;  // in rank order
+      for (int r = 0; r < C; ++r) Rtot = __fadd_rn(Rtot, sh.all_r[r]);
+      if (!isfinite(Rtot)) {
+        sh.err |= SC_DEV_TIMEOUT;
+      } else {
+        sh.tv = fminf(1.0f, fmaxf(0.0f, Rtot / sh.Sq));  // Lemma 3: R = S_q D_TV(p, q)
+        if (verify) {
+          sh.delta = sh.maxq < sh.maxp - P.alpha * sh.tv;  // Eq. 10
+          accept_test(sh, sh.xq, sh.xp, uj, k, P.kl, P.row_info != nullptr);
         }
       }
     }
-    cluster_arrive();  // no further reads of peer shared memory
     __syncthreads();
   }
 
@@ -1217,7 +1219,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     // let copies still in flight land before this CTA's shared memory is released
     for (int s = 0; s < kStages; ++s) mbar_wait(&sh.full[s], 0), mbar_wait(&sh.full[s], 1);
   }
-  cluster_wait();  // peers are done reading this CTA's shared memory
+  // (no CTA touches a peer's shared memory after its last exchange barrier)
 }
 
 // ------------------------------------------------------------------ host side
