@@ -264,13 +264,14 @@ struct __align__(16) Shared {
   float4 all_ms[kMaxCluster];  // 1: (m_q, s_q, m_p, s_p) of the slice
   float2 all_x[kMaxCluster];   // 1: raw logits at the draft token, if in the slice
   float all_r[kMaxCluster];    // 2 (TV pass): the slice's total residual weight
+  float all_lb[kMaxCluster];   // OPT band: the slice's lower bound on D_TV
   int timeout;
   float4 red[kNW];          // (m_q, s_q, m_p, s_p) of each warp
   float seg[kEntries + 1];  // per-(chunk, round, warp) weights, then exclusive prefixes
   float xq, xp;             // raw logits at the draft token, when in this slice
   // row state, identical in every CTA of the cluster
   float Mq, Sq, Mp, Sp, Rq, Rp, maxq, maxp, c, tv, qx, pix;
-  int err, delta, accept, need_p2;
+  int err, delta, accept, need_p2, band;
   // sequence finish
   int owner;                // this CTA runs its rank's sample pass of row j*
   int scan_records;         // j* must be read from the records (gamma + 1 > 32)
@@ -847,6 +848,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     }
   });
   float s_q = s2q.x + s2q.y, s_p = s2p.x + s2p.y;
+  const float4 mine = make_float4(mq, s_q, mp, s_p);  // this thread's partial, kept for the D_TV bound
   tmo = __syncthreads_or(tmo);
   warp_ms_merge(mq, s_q, k);
   warp_ms_merge(mp, s_p, k);
@@ -900,6 +902,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     sh.err = err;
     sh.delta = 0;
     sh.need_p2 = 0;
+    sh.band = 0;
     sh.accept = 0;
     sh.tv = -1.0f;
     sh.qx = 0.0f;
@@ -924,7 +927,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
           case SC_RULE_ALWAYS_DEFER: sh.delta = 1; break;
           default: sh.delta = 0; break;
         }
-        if (pending) sh.need_p2 = 1;
+        if (pending) sh.need_p2 = sh.band = 1;
         else accept_test(sh, yqx, ypx, uj, k, P.kl, P.row_info != nullptr);
       }
     }
@@ -933,6 +936,37 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     sh.xp = ypx;
   }
   __syncthreads();
+
+  // ---- OPT band: a lower bound on D_TV from the pass-1 partials.  The threads'
+  // element sets partition the vocabulary, so sum_t max(0, P_t - Q_t) <= D_TV
+  // (P_t, Q_t: the probability mass of thread t's logits).  When alpha times
+  // that bound already reaches max p - max q, delta = 0 for the exact D_TV too
+  // (Eq. 10) and the TV pass is skipped.  The bound carries ~1e-6 of f32
+  // rounding over its 128 C terms; only a clear 1e-4 excess settles the row.
+  if (sh.band) {
+    const float pt = mine.w * ex2(refk(mine.z, k) - sh.Rp) / sh.Sp;
+    const float qt = mine.y * ex2(refk(mine.x, k) - sh.Rq) / sh.Sq;
+    const float lb = warp_sum(fmaxf(0.0f, pt - qt));
+    if (lane == 0) sh.red[warp].x = lb;
+    __syncthreads();
+    if (tid == 0) {
+      float acc = 0.0f;
+      for (int w = 0; w < kNW; ++w) acc = __fadd_rn(acc, sh.red[w].x);
+      for (int r = 0; r < C; ++r) st_peer(peer_addr(&sh.all_lb[rank], r), acc);
+    }
+    cluster_arrive();
+    cluster_wait();
+    if (tid == 0) {
+      float LB = 0.0f;  // in rank order
+      for (int r = 0; r < C; ++r) LB = __fadd_rn(LB, sh.all_lb[r]);
+      if (P.alpha * LB - (sh.maxp - sh.maxq) >= 1e-4f) {
+        sh.need_p2 = 0;
+        sh.delta = 0;
+        accept_test(sh, sh.xq, sh.xp, uj, k, P.kl, P.row_info != nullptr);
+      }
+    }
+    __syncthreads();
+  }
 
   // ---- TV pass (sc_row_stats, or the OPT band): residual weights of this row
   if (sh.need_p2) {

@@ -244,3 +244,25 @@ def test_repeatable_and_workspace_reuse(sc):
     ok = ~ref2.flagged
     np.testing.assert_array_equal(outs[1][0][ok], ref2.num_accepted[ok])
     np.testing.assert_array_equal(outs[1][1][ok], ref2.next_token[ok])
+
+
+@pytest.mark.parametrize("alpha", [0.2, 0.5, 1.0])
+def test_opt_band_settled_by_tv_lower_bound(sc, alpha):
+    # Inside the OPT band (max p - alpha <= max q < max p) the kernel first bounds
+    # D_TV from below by its threads' partial masses; rows the bound settles at
+    # delta = 0 report no TV (-1).  Their decisions must still be the oracle's.
+    w = synthetic(24, 8, 256000, dtype="bf16", kind="zipf", sigma=0.7, rule="opt", alpha=alpha,
+                  temperature=1.0, seed=31)
+    gpu = run_gpu(sc, w)
+    ref = oracle.verify_workload(w)
+    assert_parity(w, gpu, ref)
+    ri = gpu[2][:, :w.gamma]
+    maxq, maxp, tv = ref.row("maxq"), ref.row("maxp"), ri[..., 2]
+    band = (maxq < maxp) & (maxq >= maxp - alpha)
+    settled = band & (tv < 0)
+    assert settled.sum() > 0, "no band row was settled by the bound"
+    np.testing.assert_array_equal(ri[..., 3][settled], 0.0)
+    np.testing.assert_array_equal(ref.row("delta")[settled], 0.0)
+    # the rows left to the TV pass report an exact D_TV
+    exact = band & ~settled
+    np.testing.assert_allclose(tv[exact], ref.row("tv")[exact], atol=TOL)
