@@ -69,7 +69,7 @@ typedef enum {
 #define SC_ROW_MAXQ 0   /* max_v q_j(v) */
 #define SC_ROW_MAXP 1   /* max_v p_j(v) */
 #define SC_ROW_TV 2     /* D_TV(p_j, q_j) = sum_v max(0, p_j(v) - q_j(v)) (Lemma 3), or -1
-                           when the rule did not need it */
+                           when the decision did not need its exact value */
 #define SC_ROW_DELTA 3  /* delta_j in {0, 1} */
 #define SC_ROW_ACCEPT 4 /* a_j in {0, 1} (a_gamma = 0) */
 #define SC_ROW_QX 5     /* q_j(x_j) */
