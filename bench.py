@@ -183,11 +183,33 @@ def oracle_throughput(w, max_seqs=64, min_core_s=0.0):
                        f"V={w.V} each), {dt:.2f} s wall on {cores} threads ({dt * cores:.0f} core-s)"), dt, done
 
 
+# ------------------------------------------------------------------ multi-rank
+
+def max_over_ranks(value, world, device):
+    """The largest of every rank's value (all_reduce MAX); value itself on one rank."""
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank, world, ms_step):
+    """Units all ranks processed per second of the slowest rank's step."""
+    return units_per_rank * world / (ms_step / 1e3)
+
+
 # ------------------------------------------------------------------ main
 
-def workload_from(args):
+def workload_from(args, rank=0):
+    """The named workload; rank r > 0 of a multi-GPU run gets its own sequences
+    (seed offset 1000 r), so the ranks verify disjoint batches of one shape."""
     from paper_2405_19261_gb300.workloads import CONFIG_TEXT, config
     kw = {}
+    if rank > 0:
+        kw["seed"] = args.config + 1000 * rank
     if args.rule is not None:
         kw["rule"] = args.rule
     if args.alpha is not None:
@@ -238,7 +260,7 @@ def run_ours(args):
     dev = torch.device("cuda", local if world > 1 else 0)
     from paper_2405_19261_gb300 import binding
 
-    w, desc = workload_from(args)
+    w, desc = workload_from(args, rank)
     d, t, x, u = binding.to_device(w, dev)
     B, g = w.B, w.gamma
     ws = binding.new_workspace(B, g, dev)
@@ -304,13 +326,9 @@ def run_ours(args):
     sampler.stop()
     clocks = sampler.summary()
 
-    ms_step = ms_total / args.steps
-    if world > 1:
-        tt = torch.tensor([ms_step], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms_step = float(tt.item())
+    ms_step = max_over_ranks(ms_total / args.steps, world, dev)
     positions = B * g * world
-    value = positions / (ms_step / 1e3)
+    value = whole_job_rate(B * g, world, ms_step)
 
     # roofline of the verification kernel (the only kernel in a step)
     peak, peak_kind = measured_peaks()
@@ -353,13 +371,9 @@ def run_ours(args):
             e2e_step()
         a1.record(stream)
         torch.cuda.synchronize(dev)
-        e2e_ms = a0.elapsed_time(a1) / args.steps
-        if world > 1:
-            tt = torch.tensor([e2e_ms], device=dev)
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            e2e_ms = float(tt.item())
+        e2e_ms = max_over_ranks(a0.elapsed_time(a1) / args.steps, world, dev)
         h2d = sum(tn.numel() * tn.element_size() for tn in (hd, ht, hx, hu))
-        e2e = {"value": positions / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+        e2e = {"value": whole_job_rate(B * g, world, e2e_ms), "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": 8 * B, "ms_per_step": e2e_ms}
 
     cpu = None
