@@ -12,24 +12,28 @@
 //   pass 1  the slice streams from HBM through a two-stage shared-memory ring
 //           filled by TMA bulk copies (cp.async.bulk + mbarrier), 4096 logits
 //           per row per stage; each thread keeps an online (max, sum of exp);
-//           the CTA partials are merged over the cluster through distributed
-//           shared memory, giving M and S of both rows, max q = 1/S_q and
-//           max p = 1/S_p, the deferral decision of Table 1 and the acceptance
-//           test of the draft token;
-//   TV      only for the OPT rule inside the band where its TV term decides, and
-//           for sc_row_stats: the slice is streamed again (from L2) and the
-//           residual weights max(0, p - q) are summed over the cluster; their
-//           total is D_TV(p, q) S_q (Lemma 3);
-//   finish  every CTA writes its unit's decision record and takes a ticket of
-//           its slice rank r in the sequence.  The last CTA of rank r (all
-//           gamma + 1 decisions are in) knows j* = min{j : a_j = 0}, streams its
-//           slice of row j* -- the rejected pair, whose residual max(0, p - q)
-//           is sampled, or the bonus row p_gamma when all drafts were accepted --
-//           and stores the slice's total weight.  The last of those C slice
-//           passes does the inverse-CDF draw: it finds the slice and the
-//           (chunk, round, warp) segment holding u R, and one warp scans the
-//           segment's 256 logits.  Only the sampled row of each sequence gets a
-//           second pass, and no CTA ever waits on another cluster.
+//           thread 0 merges the warp partials and pushes the CTA partial into
+//           every CTA of the cluster (st.shared::cluster) before one cluster
+//           barrier, after which every read is local: M and S of both rows,
+//           max q = 1/S_q and max p = 1/S_p, the deferral decision of Table 1
+//           and the acceptance test of the draft token;
+//   TV      only inside the OPT band where the TV term of Eq. 10 decides: a
+//           lower bound on D_TV from the threads' partial masses settles many
+//           such rows at delta = 0; the rest, and sc_row_stats, sum the
+//           residual weights max(0, p - q) over the slice again (newest chunk
+//           first) and over the cluster: D_TV(p, q) S_q (Lemma 3);
+//   finish  every CTA writes its unit's decision record and reports its
+//           arrival (and rejection) on the ticket of its slice rank r in the
+//           sequence.  The CTA whose report settles j* = min{j : a_j = 0} --
+//           the first rejection with every earlier position in, or all
+//           gamma + 1 positions in without one -- streams its slice of row j*
+//           (the rejected pair, whose residual max(0, p - q) is sampled, or the
+//           bonus row p_gamma) and stores the slice's chunk prefixes.  The last
+//           of those C slice passes (and of rank 0's reports) does the
+//           inverse-CDF draw: it finds the slice and chunk holding u R, copies
+//           that chunk in and one warp scans the segment holding it.  Only the
+//           sampled row of each sequence gets a second pass, and no CTA ever
+//           waits on another cluster.
 //
 // Exponentials are ex2.approx of fma(y, log2(e)/T, -R), R = fl(M log2(e)/T):
 // one rounding per logit.  Every mbarrier wait is bounded and reports
