@@ -266,3 +266,44 @@ def test_opt_band_settled_by_tv_lower_bound(sc, alpha):
     # the rows left to the TV pass report an exact D_TV
     exact = band & ~settled
     np.testing.assert_allclose(tv[exact], ref.row("tv")[exact], atol=TOL)
+
+
+# ----------------------------------------------------------------- maximum sizes
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("rule", ["always", "opt"])
+def test_max_vocab(sc, dtype, rule):
+    import torch
+    V = sc.max_vocab(torch.bfloat16 if dtype == "bf16" else torch.float32)   # 16 CTAs x 16 chunks
+    w = synthetic(2, 2, V, dtype=dtype, kind="zipf", sigma=0.7, rule=rule, alpha=0.2,
+                  temperature=1.0, seed=11)
+    assert_parity(w, run_gpu(sc, w), oracle.verify_workload(w))
+
+
+@pytest.mark.parametrize("rule", ["always", "never"])
+def test_max_gamma(sc, rule):
+    # gamma + 1 = 256 positions: the arrival-count ticket instead of the 32-bit masks
+    w = synthetic(2, 255, 1000, dtype="bf16", kind="zipf", sigma=1.0, rule=rule, alpha=0.0, seed=255)
+    assert_parity(w, run_gpu(sc, w), oracle.verify_workload(w))
+
+
+def test_vocab_above_the_limit_is_refused(sc):
+    import torch
+    V = sc.max_vocab(torch.bfloat16) + 8
+    w = synthetic(1, 1, V, dtype="bf16", kind="gauss", seed=3)
+    d, t, x, u = sc.to_device(w)
+    with pytest.raises(sc.SCError):
+        sc.sc_verify(d, t, x, u, "opt", 0.2, 1.0)
+
+
+@pytest.fixture(scope="module")
+def cfg4_largest():
+    # the largest sweep point bench.py times: B=512, gamma=8 (4.46 GB of bf16 logits);
+    # generated once, the rules below run on the same logits
+    return config(4, B=512, gamma=8, rule="diff")
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("rule,alpha", [("chow", 0.5), ("diff", 0.1), ("opt", 0.2)])
+def test_cfg4_largest_point_sampled(sc, cfg4_largest, rule, alpha):
+    _sampled_parity(sc, cfg4_largest.with_rule(rule, alpha), nseq=6)
