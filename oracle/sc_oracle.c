@@ -21,6 +21,15 @@
  *     next token ~ norm(max(0, pi_{j*} - q_{j*}))  if j* < gamma
  *                ~ pi_gamma                         otherwise
  *
+ *   or with the token-specific target (Section 4.4, TokenSpecCascade):
+ *       r_j(v) in {0, 1} per token by a plug-in rule:
+ *          TokenV1: q(v) < max p - alpha
+ *          TokenV2: p(v) < max p - alpha
+ *          TokenV3: p(v) < max p * (1 - alpha)
+ *       eta_j = sum_v r_j(v) q_j(v)
+ *       pi_j(v) = q_j(v) (1 - r_j(v)) + eta_j p_j(v)
+ *     and the same acceptance, first rejection and residual draw.
+ *
  * Readings where the paper leaves a choice open:
  *   - the bonus position has no draft row, so pi_gamma := p_gamma (as in
  *     SpecDecode, Algorithm 1);
@@ -58,6 +67,9 @@
 #define OR_OPT 2
 #define OR_ALWAYS 3 /* delta = 1: standard speculative sampling (Algorithm 1) */
 #define OR_NEVER 4  /* delta = 0: pi = q */
+#define OR_TOKEN_V1 5 /* token-specific: r(v) = [q(v) < max p - alpha] */
+#define OR_TOKEN_V2 6 /* token-specific: r(v) = [p(v) < max p - alpha] */
+#define OR_TOKEN_V3 7 /* token-specific: r(v) = [p(v) < max p (1 - alpha)] */
 
 /* per-row record layout, [B][gamma][OR_ROW_FIELDS] */
 #define OR_ROW_MAXQ 0
@@ -203,6 +215,58 @@ static int deferral(int rule, double alpha, double maxq, double maxp, double tv,
 }
 
 /*
+ * Token-specific deferral of token v (Section 4.4): r(v) = 1 when the token is
+ * deferred to the target model.  lnp_rel = ln p(v) - ln max p, formed from the
+ * logits, is what TokenV3 compares (p(v) < max p (1 - alpha) <=> lnp_rel <
+ * ln(1 - alpha)); TokenV1 and TokenV2 compare probabilities with max p - alpha.
+ * *margin receives |lhs - rhs| in the units compared.
+ */
+static int token_r(int rule, double alpha, double qv, double pv, double maxp, double lnp_rel,
+                   double *margin)
+{
+    double lhs, rhs;
+    switch (rule) {
+    case OR_TOKEN_V1: lhs = qv; rhs = maxp - alpha; break;
+    case OR_TOKEN_V2: lhs = pv; rhs = maxp - alpha; break;
+    default:
+        if (alpha >= 1.0) { *margin = INFINITY; return 0; }   /* ln(0): nothing deferred */
+        lhs = lnp_rel; rhs = log1p(-alpha);
+        if (alpha == 0.0 && lnp_rel == 0.0) { *margin = INFINITY; return 0; }  /* the mode itself, exactly */
+        break;
+    }
+    *margin = fabs(lhs - rhs);
+    return lhs < rhs ? 1 : 0;
+}
+
+/*
+ * The token-specific target of one row: r(v) for every token, eta = sum_v r(v) q(v)
+ * and pi(v) = q(v) (1 - r(v)) + eta p(v).  r is written to rv[] (0/1); the
+ * returned margin is the smallest per-token margin among tokens with q(v) or
+ * p(v) of at least 1e-9 (flipping a lighter token moves eta and pi by less).
+ */
+static double token_target(int rule, double alpha, const void *zp, int dtype, size_t poff, double Mp,
+                           double T, const double *q, const double *p, int V, double maxp,
+                           double *rv, double *pi, double *margin)
+{
+    csum eta = {0.0, 0.0};
+    double mmin = INFINITY;
+    for (int v = 0; v < V; ++v) {
+        double m;
+        const double lnp_rel = logit_at(zp, dtype, poff + v) / T - Mp;  /* as the softmax forms y / T */
+        const int r = token_r(rule, alpha, q[v], p[v], maxp, lnp_rel, &m);
+        rv[v] = r;
+        if (r) csum_add(&eta, q[v]);
+        if ((q[v] >= 1e-9 || p[v] >= 1e-9) && m < mmin) mmin = m;
+    }
+    const double e = csum_value(&eta);
+    if (pi)
+        for (int v = 0; v < V; ++v)
+            pi[v] = q[v] * (1.0 - rv[v]) + e * p[v];
+    *margin = mmin;
+    return e;
+}
+
+/*
  * Inverse-CDF draw from the unnormalised weights w[0..V-1] >= 0 with the
  * uniform u: the smallest k with C_k = sum_{v<=k} w_v > u * R, R = sum_v w_v.
  * If rounding leaves u*R at or above the last cumulative value, the largest k
@@ -259,6 +323,7 @@ static void verify_sequence(const void *draft, const void *target, int dtype,
         if (!(u[j] >= 0.0f && u[j] < 1.0f))
             status |= OR_BAD_UNIFORM;
 
+    const int token = rule >= OR_TOKEN_V1;
     int jstar = gamma;          /* a_gamma = 0 */
     double min_margin = INFINITY;
     int delta_star = 0;         /* delta at j* */
@@ -272,10 +337,35 @@ static void verify_sequence(const void *draft, const void *target, int dtype,
         }
         double maxq = max_of(q, V), maxp = max_of(p, V), tv = tv_distance(p, q, V);
         double m_delta, m_acc = INFINITY;
-        int delta = deferral(rule, alpha, maxq, maxp, tv, &m_delta);
+        int delta;
         int accept = 1;
         double qx = 0.0, pix = 0.0;
-        if (!(status & OR_BAD_TOKEN)) {
+        if (token) {
+            /* token-specific target (TokenSpecCascade): w holds r(v) for this row */
+            const double eta = token_target(rule, alpha, target, dtype, tbase + (size_t)j * V, Mp, T,
+                                            q, p, V, maxp, w, NULL, &m_delta);
+            delta = 0;
+            if (!(status & OR_BAD_TOKEN)) {
+                const int rx = (int)w[x[j]];
+                delta = rx; /* reported: r(x_j), the draft token's own deferral */
+                qx = q[x[j]];
+                pix = qx * (1 - rx) + eta * p[x[j]];
+                if (rx) {
+                    /* pi(x)/q(x) = eta p(x)/q(x), from log-probabilities; a draft with
+                       q(x) <= pi(x) (or q(x) = 0) is always accepted */
+                    double lq = log_prob(draft, dtype, dbase + (size_t)j * V, x[j], T, Mq, lnSq);
+                    double lp = log_prob(target, dtype, tbase + (size_t)j * V, x[j], T, Mp, lnSp);
+                    double ratio = eta > 0.0 ? exp(lp - lq + log(eta)) : 0.0;
+                    if (lq > -INFINITY && ratio < 1.0) {
+                        accept = (double)u[j] < ratio;
+                        m_acc = fabs((double)u[j] - ratio);
+                    }
+                }
+            }
+        } else {
+            delta = deferral(rule, alpha, maxq, maxp, tv, &m_delta);
+        }
+        if (!token && !(status & OR_BAD_TOKEN)) {
             qx = q[x[j]];
             pix = delta ? p[x[j]] : qx; /* pi(x) = (1 - delta) q(x) + delta p(x) */
             if (delta) {
@@ -323,7 +413,20 @@ static void verify_sequence(const void *draft, const void *target, int dtype,
     int tok = -1;
     double m_sample = 0.0;
     if (status == 0) {
-        if (jstar < gamma) {
+        if (jstar < gamma && token) {
+            /* residual norm(max(0, pi - q)) of row j* with the token-specific
+               target: max(0, eta p(v) - r(v) q(v)) */
+            double Mp, lnSp, m_unused;
+            tempered_softmax(draft, dtype, dbase + (size_t)jstar * V, V, T, q);
+            tempered_softmax_ln(target, dtype, tbase + (size_t)jstar * V, V, T, p, &Mp, &lnSp);
+            const double eta = token_target(rule, alpha, target, dtype, tbase + (size_t)jstar * V, Mp,
+                                            T, q, p, V, max_of(p, V), w, NULL, &m_unused);
+            for (int v = 0; v < V; ++v) {
+                double d = eta * p[v] - w[v] * q[v];
+                w[v] = d > 0.0 ? d : 0.0;
+            }
+            tok = inverse_cdf(w, V, (double)u[gamma], &m_sample);
+        } else if (jstar < gamma) {
             /* residual norm(max(0, pi - q)) of row j*; pi = p there since a
                rejection implies delta = 1 */
             tempered_softmax(draft, dtype, dbase + (size_t)jstar * V, V, T, q);
@@ -387,7 +490,7 @@ int oracle_verify(const void *draft, const void *target, int dtype, const int32_
 {
     if (!draft || !target || !tokens || !uniforms || !num_accepted || !next_token)
         return -1;
-    if (B < 0 || gamma < 1 || V < 1 || !(T > 0.0) || rule < 0 || rule > 4)
+    if (B < 0 || gamma < 1 || V < 1 || !(T > 0.0) || rule < 0 || rule > OR_TOKEN_V3)
         return -1;
     int failed = 0;
 #ifdef _OPENMP

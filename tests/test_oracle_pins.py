@@ -339,3 +339,77 @@ def test_enumeration_agrees_with_fine_grid_bruteforce():
         tok0 = np.where(r.num_accepted >= 1, x, r.next_token)
         emit0 += q[x] * np.bincount(tok0, minlength=2) / len(U)
     np.testing.assert_allclose(emit0, [0.2, 0.8], atol=2.0 / n)
+
+
+# ----------------------------------------------------------------- token-specific targets
+
+def test_token_worked_examples():
+    """Hand-worked TokenSpecCascade runs (Section 4.4) on a 4-token vocabulary."""
+    g = load_golden("token_examples.json")
+    for ex in g["examples"]:
+        for c in ex["cases"]:
+            w = rows_workload(ex["q"], ex["p"], c["tokens"], c["u"], c["rule"], c["alpha"])
+            r = oracle.verify_workload(w)
+            assert not r.flagged[0], (ex["name"], c)
+            assert (r.num_accepted[0], r.next_token[0]) == (c["num_accepted"], c["next_token"]), (ex["name"], c)
+
+
+def _token_pi(rule, alpha, q, p):
+    """pi_Token(v) = q(v)(1 - r(v)) + eta p(v), eta = sum_v r(v) q(v), for one row
+    (Section 4.4; r by the TokenV1 / TokenV2 / TokenV3 plug-in rules)."""
+    maxp = p.max()
+    if rule == "token_v1":
+        r = q < maxp - alpha
+    elif rule == "token_v2":
+        r = p < maxp - alpha
+    else:
+        r = p < maxp * (1.0 - alpha)
+    eta = q[r].sum()
+    return np.where(r, 0.0, q) + eta * p, r
+
+
+TOKEN_ENUM_CASES = [
+    # (V, gamma, rule, alpha, T, seed)
+    (4, 2, "token_v3", 0.3, 1.0, 21),
+    (5, 2, "token_v3", 0.6, 0.8, 22),
+    (6, 1, "token_v3", 0.0, 1.0, 23),
+    (4, 3, "token_v2", 0.1, 1.0, 24),
+    (5, 2, "token_v1", 0.2, 1.0, 25),
+    (3, 3, "token_v1", 0.05, 1.5, 26),
+]
+
+
+@pytest.mark.parametrize("V,gamma,rule,alpha,T,seed", TOKEN_ENUM_CASES)
+def test_enumeration_token_specific_target(V, gamma, rule, alpha, T, seed):
+    """Speculative sampling with the token-specific target: conditional on
+    reaching position j, the emitted token is pi_Token-distributed, pi_Token sums
+    to one, and the rejection probability at j is sum_v max(0, q(v) - pi(v))
+    (Lemma 3 with pi in place of p); the bonus token is p_gamma-distributed."""
+    rng = np.random.default_rng(seed)
+    q_log = (rng.standard_normal((gamma, V)) * 1.5).astype(np.float32)
+    p_log = (q_log[np.r_[0:gamma, gamma - 1]] + rng.standard_normal((gamma + 1, V)) * 1.2).astype(np.float32)
+    w = rows_workload(np.exp(q_log), np.exp(p_log), np.zeros(gamma), np.zeros(gamma + 1), rule,
+                      alpha, temperature=T)
+    info = oracle.verify_workload(w)
+    q = np_softmax(logits_as_f64(w.draft[0], "f32"), T)
+    p = np_softmax(logits_as_f64(w.target[0], "f32"), T)
+    reach, laws, reject = exact_output_law(w)
+    tol = 4.0 * V / GRID + 1e-9
+    for j in range(gamma):
+        pi, r = _token_pi(rule, alpha, q[j], p[j])
+        assert abs(pi.sum() - 1.0) < 1e-12
+        assert info.row("delta")[0][j] == r[0]   # reported: r(x_j), x_j = 0 in the stored tokens
+        np.testing.assert_allclose(laws[j], pi, atol=tol, err_msg=f"position {j}")
+        assert abs(reject[j] - np.maximum(0.0, q[j] - pi).sum()) < tol, (j, reject[j])
+    np.testing.assert_allclose(laws[gamma], p[gamma], atol=tol, err_msg="bonus position")
+
+
+@pytest.mark.parametrize("rule", ["token_v1", "token_v2", "token_v3"])
+def test_token_rules_that_defer_nothing_accept_every_draft(rule):
+    # alpha = 1: TokenV3 compares p(v) < 0 and TokenV1/V2 compare with max p - 1 <= 0,
+    # so r = 0 everywhere, eta = 0 and pi = q: every draft is accepted
+    w = synthetic(8, 5, 1000, dtype="bf16", kind="zipf", sigma=1.0, rule=rule, alpha=1.0, seed=41)
+    r = oracle.verify_workload(w)
+    assert np.all(r.num_accepted == w.gamma)
+    assert np.all(r.row("delta") == 0) and np.all(r.row("accept") == 1)
+    np.testing.assert_allclose(r.row("pix"), r.row("qx"), rtol=1e-12)
