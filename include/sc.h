@@ -8,7 +8,9 @@
  *     pi_j = (1 - delta_j) q_j + delta_j p_j                          (Eq. 6)
  *
  * where q_j = softmax(draft_logits[b, j] / T), p_j = softmax(target_logits[b, j] / T)
- * and delta_j is a deferral rule of Table 1.  Per sequence b it accepts draft
+ * and delta_j is a deferral rule of Table 1 (with a token-specific rule of
+ * Section 4.4, pi_j(v) = q_j(v) (1 - r_j(v)) + eta_j p_j(v) instead, see
+ * SC_RULE_TOKEN_V1..3).  Per sequence b it accepts draft
  * token x_j when u[b, j] < min(1, pi_j(x_j) / q_j(x_j)), finds the first
  * rejection j*, and draws one new token from norm(max(0, pi_{j*} - q_{j*})),
  * or from pi_gamma when all gamma drafts are accepted.
@@ -44,7 +46,12 @@ typedef enum {
   SC_RULE_DIFF = 1,         /* max_v q(v) < max_v p(v) - alpha                  (Eq. 5)  */
   SC_RULE_OPT = 2,          /* max_v q(v) < max_v p(v) - alpha * D_TV(p, q)     (Eq. 10) */
   SC_RULE_ALWAYS_DEFER = 3, /* delta = 1: standard speculative sampling, pi = p (Algorithm 1) */
-  SC_RULE_NEVER_DEFER = 4   /* delta = 0: pi = q, every draft is accepted */
+  SC_RULE_NEVER_DEFER = 4,  /* delta = 0: pi = q, every draft is accepted */
+  /* Token-specific targets (Section 4.4, TokenSpecCascade): a per-token deferral
+   * r(v) in {0, 1}, eta = sum_v r(v) q(v) and pi(v) = q(v) (1 - r(v)) + eta p(v). */
+  SC_RULE_TOKEN_V1 = 5,     /* r(v) = [q(v) < max p - alpha] */
+  SC_RULE_TOKEN_V2 = 6,     /* r(v) = [p(v) < max p - alpha] */
+  SC_RULE_TOKEN_V3 = 7      /* r(v) = [p(v) < max p (1 - alpha)] */
 } sc_rule;
 
 typedef enum {
@@ -70,7 +77,7 @@ typedef enum {
 #define SC_ROW_MAXP 1   /* max_v p_j(v) */
 #define SC_ROW_TV 2     /* D_TV(p_j, q_j) = sum_v max(0, p_j(v) - q_j(v)) (Lemma 3), or -1
                            when the decision did not need its exact value */
-#define SC_ROW_DELTA 3  /* delta_j in {0, 1} */
+#define SC_ROW_DELTA 3  /* delta_j in {0, 1}; for a token rule r_j(x_j), the draft token's deferral */
 #define SC_ROW_ACCEPT 4 /* a_j in {0, 1} (a_gamma = 0) */
 #define SC_ROW_QX 5     /* q_j(x_j) */
 #define SC_ROW_PIX 6    /* pi_j(x_j) */
@@ -97,7 +104,7 @@ int sc_max_vocab(sc_dtype dtype);
  *   uniforms       [B][gamma+1] f32  u[b][j < gamma] is the Bernoulli draw of
  *                                    position j; u[b][gamma] is the single draw
  *                                    for the residual or bonus sample
- *   rule, alpha    deferral rule of Table 1 and its cost parameter
+ *   rule, alpha    deferral rule of Table 1 (or a token-specific rule) and its cost parameter
  *   temperature    T > 0; both q and p are softmax(logits / T)
  *   num_accepted   [B] int32 out: j* in [0, gamma]
  *   next_token     [B] int32 out: the token emitted at position j*.  The

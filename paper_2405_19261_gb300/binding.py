@@ -17,7 +17,8 @@ import torch
 HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "_lib", "libspeccascade.so")
 
-RULES = {"chow": 0, "diff": 1, "opt": 2, "always": 3, "never": 4}
+RULES = {"chow": 0, "diff": 1, "opt": 2, "always": 3, "never": 4,
+         "token_v1": 5, "token_v2": 6, "token_v3": 7}
 ROW_FIELDS = 8
 ROW = dict(maxq=0, maxp=1, tv=2, delta=3, accept=4, qx=5, pix=6, cand=7)
 DEV_BAD_TOKEN, DEV_BAD_LOGIT, DEV_BAD_UNIFORM, DEV_TIMEOUT = 1, 2, 4, 8

@@ -17,6 +17,10 @@
 //           barrier, after which every read is local: M and S of both rows,
 //           max q = 1/S_q and max p = 1/S_p, the deferral decision of Table 1
 //           and the acceptance test of the draft token;
+//   token   with a token-specific rule (Section 4.4) every pair makes a second
+//           pass for eta = sum_v r(v) q(v), r(v) the per-token deferral; the
+//           draft is accepted when r(x) = 0, else with ratio eta p(x)/q(x), and
+//           the residual weights are max(0, eta p - r q);
 //   TV      only inside the OPT band where the TV term of Eq. 10 decides: a
 //           lower bound on D_TV from the threads' partial masses settles many
 //           such rows at delta = 0; the rest, and sc_row_stats, sum the
@@ -109,6 +113,7 @@ struct Params {
   unsigned long long *rank_tickets;  // [B][kMaxCluster] arrivals of the rank-r CTAs; zero at rest
   uint32_t *seq_tickets;   // [B] finished sample passes (+1 for rank 0's last arrival); zero at rest
   float4 *records;         // [B][kMaxCluster][gamma+1] (R_q, R_p, c, flags) as seen by rank r
+  float4 *records2;        // [B][kMaxCluster][gamma+1] (eta, thr, token, on_q) of token rules
   float *chunk_pre;        // [B][kMaxCluster][kMaxChunks + 1] exclusive prefix of slice r of the
                            // sampled row at each chunk start, then the slice total
   int32_t *status;
@@ -276,12 +281,15 @@ struct __align__(16) Shared {
   // row state, identical in every CTA of the cluster
   float Mq, Sq, Mp, Sp, Rq, Rp, maxq, maxp, c, tv, qx, pix;
   int err, delta, accept, need_p2, band;
+  int tok, on_q;            // a token rule (Section 4.4) and its r(v) test's variable
+  float thr, eta;           // its r(v) threshold (exponent domain) and eta = sum_v r(v) q(v)
   // sequence finish
   int owner;                // this CTA runs its rank's sample pass of row j*
   int scan_records;         // j* must be read from the records (gamma + 1 > 32)
   int seq_last;             // the sequence's last finisher: draws the token
   int jstar, bad, sample_ok;
   float4 rj;                // (R_q, R_p, c, flags) of row j*
+  float4 rj2;               // (eta, thr, token, on_q) of row j*
   int cross_rank;           // slice holding u * R_tot
   int cross_chunk;          // chunk of that slice holding it (else its last chunk with weight)
   int have_t;               // u * R_tot lies inside that chunk (not past a rounding gap)
@@ -410,19 +418,37 @@ __device__ __forceinline__ void online_row<uint16_t, true>(const uint16_t *src, 
   s = acc;
 }
 
-// Row scalars of the weight formula.  With a_v = y^q_v k - R_q, b_v = y^p_v k - R_p
+// Row scalars of the weight formulas.  With a_v = y^q_v k - R_q, b_v = y^p_v k - R_p
 // (R = refk(M)) and c = log2(S_q / S_p):
 //   q_v = 2^{a_v} / S_q,   p_v = 2^{b_v} / S_p = 2^{b_v + c} / S_q,
-// so max(0, p_v - q_v) = max(0, 2^{b_v + c} - 2^{a_v}) / S_q.
+// and, up to the common factor 1/S_q, the weight of logit v is
+//   kResidual  max(0, p - q) = max(0, 2^{b + c} - 2^a)   a rejected draft (Eq. 6 with
+//              delta = 1), or the D_TV pass (Lemma 3)
+//   kEta       r(v) q(v)                                eta = sum_v r(v) q(v) of a token rule
+//   kTokenRes  max(0, eta p - r(v) q(v))                a rejected draft, token rule
+// where r(v) = [a_v < thr] (TokenV1) or [b_v < thr] (TokenV2, TokenV3).
+enum WeightKind : int { kResidual = 0, kEta = 1, kTokenRes = 2 };
+
 struct RowScalars {
   float Rq, Rp, k, c;
+  int kind;   // WeightKind
+  int on_q;   // r(v) compares a_v (TokenV1) rather than b_v
+  float thr;  // r(v) threshold, in the exponent domain of a or b
+  float eta;  // eta of the row (kTokenRes)
 };
 
-// Sampling weights of eight logits, up to the common factor 1/S_q: the
-// residual max(0, p - q) of a pair, or the unnormalised p of the bonus row,
-// computed two at a time in packed f32x2; returns their sum in index order.
-// Pass 2 and the search call exactly this, so the same logit always gets the
-// same weight and the same prefix sums.
+// The sampling weights' scalars of a row from its records (R_q, R_p, c, flags)
+// and (eta, thr, token, on_q): the residual max(0, pi - q) of a rejected draft
+// under either target, or p of the bonus row.
+__device__ __forceinline__ RowScalars sample_scalars(float4 r1, float4 r2, float k) {
+  return {r1.x, r1.y, k, r1.z, __float_as_int(r2.z) ? kTokenRes : kResidual, __float_as_int(r2.w),
+          r2.y, r2.x};
+}
+
+// Sampling weights of eight logits (see RowScalars), computed two at a time in
+// packed f32x2; the bonus row (kPair = false) weighs p.  Returns their sum in
+// index order.  Every pass and the search call exactly this, so the same logit
+// always gets the same weight and the same prefix sums.
 template <bool kPair>
 __device__ __forceinline__ float vec_weights(const float (&yq)[8], const float (&yp)[8],
                                              const RowScalars &r, float (&w)[8]) {
@@ -434,10 +460,22 @@ __device__ __forceinline__ float vec_weights(const float (&yq)[8], const float (
     if constexpr (kPair) {
       const float2 a = __ffma2_rn(make_float2(yq[e], yq[e + 1]), kk, make_float2(-r.Rq, -r.Rq));
       const float2 bc = __fadd2_rn(b, make_float2(r.c, r.c));
-      const float2 d = __ffma2_rn(make_float2(ex2(a.x), ex2(a.y)), make_float2(-1.0f, -1.0f),
-                                  make_float2(ex2(bc.x), ex2(bc.y)));
-      w[e] = fmaxf(0.0f, d.x);
-      w[e + 1] = fmaxf(0.0f, d.y);
+      if (r.kind == kResidual) {
+        const float2 d = __ffma2_rn(make_float2(ex2(a.x), ex2(a.y)), make_float2(-1.0f, -1.0f),
+                                    make_float2(ex2(bc.x), ex2(bc.y)));
+        w[e] = fmaxf(0.0f, d.x);
+        w[e + 1] = fmaxf(0.0f, d.y);
+      } else {
+        const bool r0 = (r.on_q ? a.x : b.x) < r.thr, r1 = (r.on_q ? a.y : b.y) < r.thr;
+        const float q0 = r0 ? ex2(a.x) : 0.0f, q1 = r1 ? ex2(a.y) : 0.0f;
+        if (r.kind == kEta) {
+          w[e] = q0;
+          w[e + 1] = q1;
+        } else {
+          w[e] = fmaxf(0.0f, fmaf(r.eta, ex2(bc.x), -q0));
+          w[e + 1] = fmaxf(0.0f, fmaf(r.eta, ex2(bc.y), -q1));
+        }
+      }
     } else {
       w[e] = ex2(b.x);
       w[e + 1] = ex2(b.y);
@@ -528,10 +566,17 @@ __device__ __forceinline__ float2 log2_prob(float y, float R, float S, float k, 
 // q(x) <= pi(x), else a = [u < pi(x)/q(x)].  L = log2 p(x) - log2 q(x)
 //   = (y_p(x) - y_q(x)) log2(e)/T - (R_p - R_q) + log2(S_q / S_p)
 // is formed in double-float from the logits, so the ratio 2^L carries
-// essentially only the f32 error of log2(S_q / S_p).  q(x) and pi(x)
-// themselves are evaluated only for the diagnostics output.
+// essentially only the f32 error of log2(S_q / S_p).  With a token rule
+// (Section 4.4) the draft token's own deferral r(x) takes delta's place and
+// pi(x)/q(x) = (1 - r(x)) + eta p(x)/q(x): accepted outright when r(x) = 0,
+// else [u < eta 2^L].  q(x) and pi(x) themselves are evaluated only for the
+// diagnostics output.
 __device__ __forceinline__ void accept_test(Shared &sh, float yqx, float ypx, float u, float k, float kl,
                                             bool want_probs) {
+  if (sh.tok) {
+    const float ax = fmaf(yqx, k, -sh.Rq), bx = fmaf(ypx, k, -sh.Rp);  // as vec_weights forms them
+    sh.delta = (sh.on_q ? ax : bx) < sh.thr;                           // reported: r(x)
+  }
   int accept = 1;
   if (sh.delta) {
     const float2 d = two_sum(ypx, -yqx);  // y_p(x) - y_q(x), exactly
@@ -541,14 +586,18 @@ __device__ __forceinline__ void accept_test(Shared &sh, float yqx, float ypx, fl
     const float lo = __fadd_rn(__fadd_rn(__fadd_rn(s.y, dk.y), __fsub_rn(__fmul_rn(d.y, k), r.y)),
                                log2f(sh.Sq / sh.Sp));
     const float2 L = df_norm(s.x, lo);
-    if (df_lt(L, 0.0f)) accept = u < df_exp2(L);
+    if (!sh.tok) {
+      if (df_lt(L, 0.0f)) accept = u < df_exp2(L);
+    } else if (L.x < INFINITY) {  // (q(x) = 0 accepts)
+      accept = u < sh.eta * df_exp2(L);
+    }
   }
   sh.accept = accept;
   if (want_probs) {
     const float qx = df_exp2(log2_prob(yqx, sh.Rq, sh.Sq, k, kl));
     const float px = df_exp2(log2_prob(ypx, sh.Rp, sh.Sp, k, kl));
     sh.qx = qx;
-    sh.pix = sh.delta ? px : qx;
+    sh.pix = sh.tok ? fmaf(sh.eta, px, sh.delta ? 0.0f : qx) : (sh.delta ? px : qx);
   }
 }
 
@@ -907,6 +956,10 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     sh.delta = 0;
     sh.need_p2 = 0;
     sh.band = 0;
+    sh.tok = 0;
+    sh.on_q = 0;
+    sh.thr = -INFINITY;
+    sh.eta = 0.0f;
     sh.accept = 0;
     sh.tv = -1.0f;
     sh.qx = 0.0f;
@@ -929,10 +982,28 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
             else pending = true;
             break;
           case SC_RULE_ALWAYS_DEFER: sh.delta = 1; break;
+          case SC_RULE_TOKEN_V1:
+          case SC_RULE_TOKEN_V2:
+          case SC_RULE_TOKEN_V3: {
+            // token-specific target (Section 4.4): r(v) compares a_v or b_v with a
+            // threshold; eta = sum_v r(v) q(v) needs a pass over the row
+            const float bM = fmaf(c, k, -Rp);  // b of the mode of p: max p = 2^bM / S_p
+            sh.tok = 1;
+            pending = true;
+            if (P.rule == SC_RULE_TOKEN_V3) {  // p(v) < max p (1 - alpha)  <=>  b_v < bM + log2(1 - alpha)
+              sh.thr = al < 1.0f ? bM + log2f(1.0f - al) : -INFINITY;
+            } else {                           // p(v) or q(v) < max p - alpha
+              const float m = maxp - al;
+              sh.on_q = P.rule == SC_RULE_TOKEN_V1;
+              sh.thr = m > 0.0f ? log2f(m * (sh.on_q ? as : cs)) : -INFINITY;
+            }
+            break;
+          }
           default: sh.delta = 0; break;
         }
-        if (pending) sh.need_p2 = sh.band = 1;
-        else accept_test(sh, yqx, ypx, uj, k, P.kl, P.row_info != nullptr);
+        if (pending) sh.need_p2 = 1;
+        if (pending && !sh.tok) sh.band = 1;
+        if (!pending) accept_test(sh, yqx, ypx, uj, k, P.kl, P.row_info != nullptr);
       }
     }
     // keep the draft-token logits for a decision after the TV pass
@@ -972,9 +1043,10 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     __syncthreads();
   }
 
-  // ---- TV pass (sc_row_stats, or the OPT band): residual weights of this row
+  // ---- TV pass (sc_row_stats, or the OPT band): residual weights of this row;
+  // for a token rule the same pass sums r(v) q(v) instead (eta)
   if (sh.need_p2) {
-    const RowScalars rs = {sh.Rq, sh.Rp, k, sh.c};
+    const RowScalars rs = {sh.Rq, sh.Rp, k, sh.c, sh.tok ? kEta : kResidual, sh.on_q, sh.thr, 0.0f};
     tmo = slice_weights(R, sh, ph, rs, kNewestFirstResident, lane, warp);
     tmo = __syncthreads_or(tmo);
     // exchange 2: push the slice total, one barrier, local reads
@@ -993,6 +1065,9 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       for (int r = 0; r < C; ++r) Rtot = __fadd_rn(Rtot, sh.all_r[r]);
       if (!isfinite(Rtot)) {
         sh.err |= SC_DEV_TIMEOUT;
+      } else if (sh.tok) {
+        sh.eta = Rtot / sh.Sq;  // eta = sum_v r(v) q(v)
+        accept_test(sh, sh.xq, sh.xp, uj, k, P.kl, P.row_info != nullptr);
       } else {
         sh.tv = fminf(1.0f, fmaxf(0.0f, Rtot / sh.Sq));  // Lemma 3: R = S_q D_TV(p, q)
         if (verify) {
@@ -1016,9 +1091,12 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     // ---- record the decision and report it on this slice rank's ticket; the
     // CTA whose report settles j* samples this rank's slice of row j*
     float4 *rec = P.records + (static_cast<size_t>(b) * kMaxCluster + rank) * G1;
+    float4 *rec2 = P.records2 + (static_cast<size_t>(b) * kMaxCluster + rank) * G1;
     if (tid == 0) {
       const int flags = (sh.accept ? 1 : 0) | (sh.err ? 2 : 0);
       rec[j] = make_float4(sh.Rq, sh.Rp, sh.c, __int_as_float(flags));
+      if (P.rule >= SC_RULE_TOKEN_V1)  // (only token rules read the second record)
+        rec2[j] = make_float4(sh.eta, sh.thr, __int_as_float(sh.tok), __int_as_float(sh.on_q));
       if (rank == 0 && P.row_info) {
         float *ri = P.row_info + (static_cast<size_t>(b) * G1 + j) * SC_ROW_FIELDS;
         ri[SC_ROW_MAXQ] = pair && !sh.err ? sh.maxq : NAN;
@@ -1066,14 +1144,17 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       }
       if (lane == 0) sh.jstar = js;
     }
-    if (sh.owner && tid == 0) sh.rj = __ldcg(&rec[sh.jstar]);  // row j*'s record (it is in)
+    if (sh.owner && tid == 0) {  // row j*'s records (they are in)
+      sh.rj = __ldcg(&rec[sh.jstar]);
+      sh.rj2 = P.rule >= SC_RULE_TOKEN_V1 ? __ldcg(&rec2[sh.jstar]) : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+    }
     __syncthreads();
 
     if (sh.owner) {
       // ---- sample pass: weights of this rank's slice of row j* -- the residual
       // max(0, p - q) of a rejected pair (Algorithm 4), or p of the bonus row
       const int js = sh.jstar;
-      const RowScalars rs = {sh.rj.x, sh.rj.y, k, sh.rj.z};
+      const RowScalars rs = sample_scalars(sh.rj, sh.rj2, k);
       const Ring<E> Rj = make_ring<E>(P, smem_raw, b, js, rank);
       // this unit's own row, untouched since pass 1, still has its last chunks in the ring
       const bool resident = js == j && !sh.need_p2;
@@ -1129,11 +1210,13 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
           sh.jstar = js;
           sh.bad = bad;
           sh.rj = rj;
+          sh.rj2 = P.rule >= SC_RULE_TOKEN_V1 ? __ldcg(P.records2 + static_cast<size_t>(b) * kMaxCluster * G1 + js)
+                                              : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
         }
       }
       __syncthreads();
       const int js = sh.jstar;
-      const RowScalars rs = {sh.rj.x, sh.rj.y, k, sh.rj.z};
+      const RowScalars rs = sample_scalars(sh.rj, sh.rj2, k);
       // ---- inverse CDF over the slices in rank order, u = u[b][gamma], then
       // over the chunks of the crossing slice
       if (warp == 0) {
@@ -1277,7 +1360,7 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 // sequence tickets (both zero between calls), then unit records and chunk
 // prefixes (written before they are read).
 struct WsLayout {
-  size_t rank_tickets, seq_tickets, zeroed, records, chunk_pre, total;
+  size_t rank_tickets, seq_tickets, zeroed, records, records2, chunk_pre, total;
 };
 
 constexpr size_t align256(size_t x) { return (x + 255) / 256 * 256; }
@@ -1288,7 +1371,8 @@ constexpr WsLayout ws_layout(size_t B, size_t units) {
   w.seq_tickets = align256(8 * kMaxCluster * B);
   w.zeroed = w.seq_tickets + align256(4 * B);
   w.records = w.zeroed;
-  w.chunk_pre = w.records + align256(16 * kMaxCluster * units);
+  w.records2 = w.records + align256(16 * kMaxCluster * units);
+  w.chunk_pre = w.records2 + align256(16 * kMaxCluster * units);
   w.total = w.chunk_pre + align256(4 * kMaxCluster * (kMaxChunks + 1) * B);
   return w;
 }
@@ -1466,7 +1550,7 @@ int sc_verify_rows(const void *draft_logits, const void *target_logits, sc_dtype
                    int32_t *device_status, float *row_info, cudaStream_t stream) {
   int rc = common_checks(draft_logits, target_logits, dtype, B, gamma, V, temperature);
   if (rc != SC_OK) return rc;
-  if (static_cast<int>(rule) < 0 || static_cast<int>(rule) > 4) return SC_ERR_INVALID_ARG;
+  if (static_cast<int>(rule) < 0 || static_cast<int>(rule) > SC_RULE_TOKEN_V3) return SC_ERR_INVALID_ARG;
   if (!(alpha >= 0.0f && alpha <= 1.0f)) return SC_ERR_INVALID_ARG;
   if (!device_accessible(draft_tokens) || !device_accessible(uniforms) ||
       !device_accessible(num_accepted) || !device_accessible(next_token))
@@ -1498,6 +1582,7 @@ int sc_verify_rows(const void *draft_logits, const void *target_logits, sc_dtype
   P.rank_tickets = reinterpret_cast<unsigned long long *>(ws + wl.rank_tickets);
   P.seq_tickets = reinterpret_cast<uint32_t *>(ws + wl.seq_tickets);
   P.records = reinterpret_cast<float4 *>(ws + wl.records);
+  P.records2 = reinterpret_cast<float4 *>(ws + wl.records2);
   P.chunk_pre = reinterpret_cast<float *>(ws + wl.chunk_pre);
   const int units = B * (gamma + 1);
   return dtype == SC_BF16 ? launch<uint16_t>(P, stream, units) : launch<float>(P, stream, units);

@@ -307,3 +307,38 @@ def cfg4_largest():
 @pytest.mark.parametrize("rule,alpha", [("chow", 0.5), ("diff", 0.1), ("opt", 0.2)])
 def test_cfg4_largest_point_sampled(sc, cfg4_largest, rule, alpha):
     _sampled_parity(sc, cfg4_largest.with_rule(rule, alpha), nseq=6)
+
+
+# ----------------------------------------------------------------- token-specific targets
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_token_worked_examples(sc, dtype):
+    g = load_golden("token_examples.json")
+    for ex in g["examples"]:
+        for c in ex["cases"]:
+            w = rows_workload(ex["q"], ex["p"], c["tokens"], c["u"], c["rule"], c["alpha"], dtype=dtype)
+            na, nt, _, status = run_gpu(sc, w)
+            assert status == 0
+            assert (na[0], nt[0]) == (c["num_accepted"], c["next_token"]), (ex["name"], c)
+
+
+@pytest.mark.parametrize("rule,alpha", [("token_v3", 0.0), ("token_v3", 0.3), ("token_v3", 0.6),
+                                        ("token_v3", 1.0), ("token_v2", 0.1), ("token_v1", 0.1)])
+@pytest.mark.parametrize("seed", range(3))
+def test_token_rules_t5_shape(sc, rule, alpha, seed):
+    w = synthetic(16, 5, 32128, dtype="bf16", kind="zipf", sigma=0.7, rule=rule, alpha=alpha,
+                  temperature=1.0, seed=2000 + seed)
+    assert_parity(w, run_gpu(sc, w), oracle.verify_workload(w))
+
+
+@pytest.mark.parametrize("V,dtype", [(7, "f32"), (4097, "bf16"), (10007, "f32")])
+def test_token_rules_ragged_vocab(sc, V, dtype):
+    w = synthetic(5, 3, V, dtype=dtype, kind="gauss", sigma=1.0, rule="token_v3", alpha=0.3,
+                  temperature=0.9, seed=V)
+    assert_parity(w, run_gpu(sc, w), oracle.verify_workload(w))
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("rule", ["token_v3", "token_v1"])
+def test_token_rules_gemma_shape_sampled(sc, rule):
+    _sampled_parity(sc, config(4, B=64, gamma=4, rule=rule), nseq=6)
