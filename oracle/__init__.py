@@ -22,7 +22,7 @@ SRC = os.path.join(HERE, "sc_oracle.c")
 LIB = os.path.join(HERE, "_build", "libscoracle.so")
 
 RULES = {"chow": 0, "diff": 1, "opt": 2, "always": 3, "never": 4,
-         "token_v1": 5, "token_v2": 6, "token_v3": 7}
+         "token_v1": 5, "token_v2": 6, "token_v3": 7, "lossy": 8, "bild": 9}
 DTYPES = {"f32": 0, "bf16": 1}
 ROW = dict(maxq=0, maxp=1, tv=2, delta=3, accept=4, qx=5, pix=6, margin_delta=7, margin_accept=8)
 SEQ = dict(min_margin=0, sample_margin=1, status=2, bonus_maxp=3)
@@ -49,7 +49,7 @@ def lib():
         build()
         L = ctypes.CDLL(LIB)
         P, I, D = ctypes.c_void_p, ctypes.c_int, ctypes.c_double
-        L.oracle_verify.argtypes = [P, P, I, P, P, I, I, I, I, D, D, P, P, P, P, I]
+        L.oracle_verify.argtypes = [P, P, I, P, P, I, I, I, I, D, D, D, P, P, P, P, I]
         L.oracle_verify.restype = I
         L.oracle_row_stats.argtypes = [P, P, I, I, I, I, D, P, P, P, I]
         L.oracle_row_stats.restype = I
@@ -108,8 +108,10 @@ class OracleResult:
 
 
 def verify(draft, target, dtype, tokens, uniforms, B, gamma, V, rule, alpha, temperature,
-           nthreads: int = 0) -> OracleResult:
-    """GenSpecSample (Algorithm 4) with the SpecCascade target (Algorithm 5), in fp64."""
+           nthreads: int = 0, beta: float = 1.0) -> OracleResult:
+    """GenSpecSample (Algorithm 4) with the SpecCascade target (Algorithm 5), a
+    token-specific target (Section 4.4) or a Table 3 target (lossy speculative
+    decoding with parameter beta, BiLD*), in fp64."""
     draft, target = _logits(draft, dtype), _logits(target, dtype)
     tokens = np.ascontiguousarray(tokens, dtype=np.int32)
     uniforms = np.ascontiguousarray(uniforms, dtype=np.float32)
@@ -121,18 +123,18 @@ def verify(draft, target, dtype, tokens, uniforms, B, gamma, V, rule, alpha, tem
     seqs = np.zeros((B, len(SEQ)), np.float64)
     rc = lib().oracle_verify(_ptr(draft), _ptr(target), DTYPES[dtype], _ptr(tokens), _ptr(uniforms),
                              B, gamma, V, RULES[rule] if isinstance(rule, str) else int(rule),
-                             float(alpha), float(temperature), _ptr(na), _ptr(nt), _ptr(rows),
+                             float(alpha), float(beta), float(temperature), _ptr(na), _ptr(nt), _ptr(rows),
                              _ptr(seqs), int(nthreads))
     if rc != 0:
         raise ValueError("oracle_verify rejected its arguments")
     return OracleResult(na, nt, rows, seqs)
 
 
-def verify_workload(w, nthreads: int = 0, rule=None, alpha=None) -> OracleResult:
+def verify_workload(w, nthreads: int = 0, rule=None, alpha=None, beta=None) -> OracleResult:
     """``verify`` on any object with the generator's workload attributes."""
     return verify(w.draft, w.target, w.dtype, w.tokens, w.uniforms, w.B, w.gamma, w.V,
                   w.rule if rule is None else rule, w.alpha if alpha is None else alpha,
-                  w.temperature, nthreads)
+                  w.temperature, nthreads, getattr(w, "beta", 1.0) if beta is None else beta)
 
 
 def row_stats(draft, target, dtype, B, gamma, V, temperature, nthreads: int = 0):

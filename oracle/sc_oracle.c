@@ -28,7 +28,15 @@
  *          TokenV3: p(v) < max p * (1 - alpha)
  *       eta_j = sum_v r_j(v) q_j(v)
  *       pi_j(v) = q_j(v) (1 - r_j(v)) + eta_j p_j(v)
- *     and the same acceptance, first rejection and residual draw.
+ *     and the same acceptance, first rejection and residual draw;
+ *
+ *   or the other targets of Table 3 run through Algorithm 4:
+ *       Lossy speculative decoding:  pi(v) = max{ min{ q(v), p(v)/(1 - alpha) }, p(v)/beta }
+ *          (Lemma 2: the acceptance is min(1, p(x)/((1 - alpha) q(x))) and the residual
+ *          norm(max(0, p/beta - q)); pi need not sum to one), beta >= 1 - alpha;
+ *       BiLD*:  delta = 1(D(q, p) > alpha), D(q, p) = -sum_v q(v) log p(v) (the
+ *          temperature-sampling discrepancy of the experiments' appendix),
+ *          pi = (1 - delta) q + delta p.
  *
  * Readings where the paper leaves a choice open:
  *   - the bonus position has no draft row, so pi_gamma := p_gamma (as in
@@ -70,6 +78,8 @@
 #define OR_TOKEN_V1 5 /* token-specific: r(v) = [q(v) < max p - alpha] */
 #define OR_TOKEN_V2 6 /* token-specific: r(v) = [p(v) < max p - alpha] */
 #define OR_TOKEN_V3 7 /* token-specific: r(v) = [p(v) < max p (1 - alpha)] */
+#define OR_LOSSY 8    /* lossy speculative decoding target (Table 3, Lemma 2), parameter beta */
+#define OR_BILD 9     /* BiLD*: delta = 1(-sum_v q(v) log p(v) > alpha) */
 
 /* per-row record layout, [B][gamma][OR_ROW_FIELDS] */
 #define OR_ROW_MAXQ 0
@@ -266,6 +276,34 @@ static double token_target(int rule, double alpha, const void *zp, int dtype, si
     return e;
 }
 
+/* The lossy speculative-decoding target of one token (Table 3). */
+static double lossy_pi(double qv, double pv, double alpha, double beta)
+{
+    double a = alpha < 1.0 ? pv / (1.0 - alpha) : INFINITY;
+    double m = qv < a ? qv : a;
+    double b = pv / beta;
+    return m > b ? m : b;
+}
+
+/*
+ * BiLD*'s discrepancy D(q, p) = -sum_v q(v) log p(v) of one row pair, with
+ * log p(v) from the logits (+infinity when some q(v) > 0 has p(v) = 0).
+ */
+static double cross_entropy(const double *q, const void *zp, int dtype, size_t poff, int V, double T,
+                            double Mp, double lnSp)
+{
+    csum D = {0.0, 0.0};
+    for (int v = 0; v < V; ++v) {
+        if (!(q[v] > 0.0))
+            continue;
+        const double lp = log_prob(zp, dtype, poff, v, T, Mp, lnSp);
+        if (lp == -INFINITY)
+            return INFINITY;
+        csum_add(&D, -q[v] * lp);
+    }
+    return csum_value(&D);
+}
+
 /*
  * Inverse-CDF draw from the unnormalised weights w[0..V-1] >= 0 with the
  * uniform u: the smallest k with C_k = sum_{v<=k} w_v > u * R, R = sum_v w_v.
@@ -307,7 +345,7 @@ static int inverse_cdf(const double *w, int V, double u, double *margin)
 
 static void verify_sequence(const void *draft, const void *target, int dtype,
                             const int32_t *tokens, const float *uniforms, int b, int gamma,
-                            int V, int rule, double alpha, double T, int32_t *num_accepted,
+                            int V, int rule, double alpha, double beta, double T, int32_t *num_accepted,
                             int32_t *next_token, double *row_info, double *seq_info,
                             double *q, double *p, double *w)
 {
@@ -323,7 +361,8 @@ static void verify_sequence(const void *draft, const void *target, int dtype,
         if (!(u[j] >= 0.0f && u[j] < 1.0f))
             status |= OR_BAD_UNIFORM;
 
-    const int token = rule >= OR_TOKEN_V1;
+    const int token = rule >= OR_TOKEN_V1 && rule <= OR_TOKEN_V3;
+    const int lossy = rule == OR_LOSSY;
     int jstar = gamma;          /* a_gamma = 0 */
     double min_margin = INFINITY;
     int delta_star = 0;         /* delta at j* */
@@ -362,10 +401,34 @@ static void verify_sequence(const void *draft, const void *target, int dtype,
                     }
                 }
             }
+        } else if (lossy) {
+            /* pi(x)/q(x) = max{ min{1, (p/q)/(1 - alpha)}, (p/q)/beta }, from log-probabilities */
+            delta = 1;
+            m_delta = INFINITY;
+            if (!(status & OR_BAD_TOKEN)) {
+                qx = q[x[j]];
+                pix = lossy_pi(qx, p[x[j]], alpha, beta);
+                double lq = log_prob(draft, dtype, dbase + (size_t)j * V, x[j], T, Mq, lnSq);
+                double lp = log_prob(target, dtype, tbase + (size_t)j * V, x[j], T, Mp, lnSp);
+                if (lq > -INFINITY) {
+                    double pq = exp(lp - lq);
+                    double a = alpha < 1.0 ? pq / (1.0 - alpha) : INFINITY;
+                    double ratio = a < 1.0 ? a : 1.0;
+                    if (pq / beta > ratio) ratio = pq / beta;
+                    if (ratio < 1.0) {
+                        accept = (double)u[j] < ratio;
+                        m_acc = fabs((double)u[j] - ratio);
+                    }
+                }
+            }
+        } else if (rule == OR_BILD) {
+            const double D = cross_entropy(q, target, dtype, tbase + (size_t)j * V, V, T, Mp, lnSp);
+            delta = D > alpha;  /* strict, as printed */
+            m_delta = isfinite(D) ? fabs(D - alpha) : INFINITY;
         } else {
             delta = deferral(rule, alpha, maxq, maxp, tv, &m_delta);
         }
-        if (!token && !(status & OR_BAD_TOKEN)) {
+        if (!token && !lossy && !(status & OR_BAD_TOKEN)) {
             qx = q[x[j]];
             pix = delta ? p[x[j]] : qx; /* pi(x) = (1 - delta) q(x) + delta p(x) */
             if (delta) {
@@ -423,6 +486,15 @@ static void verify_sequence(const void *draft, const void *target, int dtype,
                                             T, q, p, V, max_of(p, V), w, NULL, &m_unused);
             for (int v = 0; v < V; ++v) {
                 double d = eta * p[v] - w[v] * q[v];
+                w[v] = d > 0.0 ? d : 0.0;
+            }
+            tok = inverse_cdf(w, V, (double)u[gamma], &m_sample);
+        } else if (jstar < gamma && lossy) {
+            /* residual norm(max(0, pi - q)) of row j* with the lossy target */
+            tempered_softmax(draft, dtype, dbase + (size_t)jstar * V, V, T, q);
+            tempered_softmax(target, dtype, tbase + (size_t)jstar * V, V, T, p);
+            for (int v = 0; v < V; ++v) {
+                double d = lossy_pi(q[v], p[v], alpha, beta) - q[v];
                 w[v] = d > 0.0 ? d : 0.0;
             }
             tok = inverse_cdf(w, V, (double)u[gamma], &m_sample);
@@ -485,12 +557,14 @@ int oracle_num_threads(int nthreads)
  */
 int oracle_verify(const void *draft, const void *target, int dtype, const int32_t *tokens,
                   const float *uniforms, int B, int gamma, int V, int rule, double alpha,
-                  double T, int32_t *num_accepted, int32_t *next_token, double *row_info,
-                  double *seq_info, int nthreads)
+                  double beta, double T, int32_t *num_accepted, int32_t *next_token,
+                  double *row_info, double *seq_info, int nthreads)
 {
     if (!draft || !target || !tokens || !uniforms || !num_accepted || !next_token)
         return -1;
-    if (B < 0 || gamma < 1 || V < 1 || !(T > 0.0) || rule < 0 || rule > OR_TOKEN_V3)
+    if (B < 0 || gamma < 1 || V < 1 || !(T > 0.0) || rule < 0 || rule > OR_BILD)
+        return -1;
+    if (rule == OR_LOSSY && !(beta > 0.0 && beta >= 1.0 - alpha))
         return -1;
     int failed = 0;
 #ifdef _OPENMP
@@ -508,7 +582,7 @@ int oracle_verify(const void *draft, const void *target, int dtype, const int32_
 #endif
             for (int b = 0; b < B; ++b)
                 verify_sequence(draft, target, dtype, tokens, uniforms, b, gamma, V, rule, alpha,
-                                T, num_accepted, next_token, row_info, seq_info, q, p, w);
+                                beta, T, num_accepted, next_token, row_info, seq_info, q, p, w);
         }
         free(q);
         free(p);

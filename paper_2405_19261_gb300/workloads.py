@@ -44,13 +44,14 @@ from typing import Optional
 import numpy as np
 
 RULES = {"chow": 0, "diff": 1, "opt": 2, "always": 3, "never": 4,
-         "token_v1": 5, "token_v2": 6, "token_v3": 7}
+         "token_v1": 5, "token_v2": 6, "token_v3": 7, "lossy": 8, "bild": 9}
 DTYPES = {"f32": 0, "bf16": 1}
 T5_VOCAB = 32128
 GEMMA_VOCAB = 256000
 
 # Default alpha per rule for the throughput sweep (the sweep leaves alpha open).
-SWEEP_ALPHA = {"chow": 0.5, "diff": 0.1, "opt": 0.2, "token_v1": 0.1, "token_v2": 0.1, "token_v3": 0.3}
+SWEEP_ALPHA = {"chow": 0.5, "diff": 0.1, "opt": 0.2, "token_v1": 0.1, "token_v2": 0.1, "token_v3": 0.3,
+               "lossy": 0.3, "bild": 3.0}
 SWEEP_POINTS = [(B, g) for B in (64, 256, 512) for g in (4, 8)]
 
 

@@ -413,3 +413,82 @@ def test_token_rules_that_defer_nothing_accept_every_draft(rule):
     assert np.all(r.num_accepted == w.gamma)
     assert np.all(r.row("delta") == 0) and np.all(r.row("accept") == 1)
     np.testing.assert_allclose(r.row("pix"), r.row("qx"), rtol=1e-12)
+
+
+# ----------------------------------------------------------------- Table 3 targets
+
+def _lossy_sd_direct(q, p, x, u, alpha, beta):
+    """Lossy speculative decoding as its own procedure (Section 2): accept x_j with
+    probability min(1, p(x)/((1 - alpha) q(x))); at the first rejection draw from
+    norm(max(0, p/beta - q)); after full acceptance draw from p_gamma.  Inverse
+    CDF in ascending vocabulary order with the last uniform."""
+    g = len(x)
+    for j in range(g):
+        rho = min(1.0, p[j][x[j]] / ((1.0 - alpha) * q[j][x[j]])) if alpha < 1 else 1.0
+        if not u[j] < rho:
+            wts = np.maximum(0.0, p[j] / beta - q[j])
+            c = np.cumsum(wts)
+            return j, int(np.searchsorted(c, u[g] * c[-1], side="right")), abs(u[j] - rho)
+    c = np.cumsum(p[g])
+    return g, int(np.searchsorted(c, u[g] * c[-1], side="right")), np.inf
+
+
+@pytest.mark.parametrize("alpha,beta", [(0.0, 1.0), (0.2, 1.0), (0.5, 0.5), (0.5, 1.3), (0.9, 0.4)])
+@pytest.mark.parametrize("seed", range(3))
+def test_lossy_target_reproduces_lossy_speculative_decoding(alpha, beta, seed):
+    """Lemma 2: Algorithm 4 with pi = max{min{q, p/(1 - alpha)}, p/beta} accepts and
+    resamples exactly as lossy speculative decoding does."""
+    rng = np.random.default_rng(300 + seed)
+    V, g = 6, 2
+    q_log = (rng.standard_normal((g, V)) * 1.5).astype(np.float32)
+    p_log = (q_log[np.r_[0:g, g - 1]] + rng.standard_normal((g + 1, V))).astype(np.float32)
+    q = np_softmax(q_log.astype(np.float64), 1.0)
+    p = np_softmax(p_log.astype(np.float64), 1.0)
+    checked = 0
+    for trial in range(60):
+        x = rng.integers(0, V, size=g)
+        u = rng.random(g + 1).astype(np.float32)
+        w = rows_workload(np.exp(q_log), np.exp(p_log), x, u, "lossy", alpha)
+        w.beta = beta
+        r = oracle.verify_workload(w)
+        qq = np_softmax(logits_as_f64(w.draft[0], "f32"), 1.0)
+        pp = np_softmax(logits_as_f64(w.target[0], "f32"), 1.0)
+        ja, tok, margin = _lossy_sd_direct(qq, pp, x, u.astype(np.float64), alpha, beta)
+        if margin < 1e-9 or r.flagged[0]:
+            continue
+        assert (r.num_accepted[0], r.next_token[0]) == (ja, tok), (trial, x, u)
+        checked += 1
+    assert checked > 40
+
+
+def test_lossy_at_alpha_0_beta_1_is_standard_speculative_sampling():
+    # alpha = 0, beta = 1: pi = max{min{q, p}, p} = p, Algorithm 1
+    w = synthetic(16, 5, 2000, dtype="bf16", kind="zipf", sigma=0.7, rule="lossy", alpha=0.0, seed=51)
+    a = oracle.verify_workload(w)
+    b = oracle.verify_workload(w, rule="always")
+    np.testing.assert_array_equal(a.num_accepted, b.num_accepted)
+    np.testing.assert_array_equal(a.next_token, b.next_token)
+
+
+@pytest.mark.parametrize("alpha", [0.5, 2.0, 4.0])
+def test_bild_discrepancy_is_the_cross_entropy(alpha):
+    """BiLD*'s delta = 1(D(q, p) > alpha) with D = -sum_v q log p = H(q) + KL(q || p)
+    (scipy.stats.entropy), the temperature-sampling discrepancy of the experiments."""
+    from scipy.stats import entropy
+    w = synthetic(12, 4, 500, dtype="f32", kind="gauss", sigma=1.0, rule="bild", alpha=alpha,
+                  temperature=0.8, seed=61)
+    r = oracle.verify_workload(w)
+    decided = 0
+    for b in range(w.B):
+        for j in range(w.gamma):
+            q = np_softmax(logits_as_f64(w.draft[b, j], "f32"), 0.8)
+            p = np_softmax(logits_as_f64(w.target[b, j], "f32"), 0.8)
+            D = entropy(q) + entropy(q, p)
+            if abs(D - alpha) < 1e-9:
+                continue
+            assert r.row("delta")[b, j] == (1.0 if D > alpha else 0.0), (b, j, D)
+            decided += 1
+    assert decided == w.B * w.gamma
+    # a threshold above every discrepancy defers nothing: every draft is accepted
+    big = oracle.verify_workload(w, alpha=1e6)
+    assert np.all(big.num_accepted == w.gamma)
