@@ -22,7 +22,8 @@ SRC = os.path.join(HERE, "sc_oracle.c")
 LIB = os.path.join(HERE, "_build", "libscoracle.so")
 
 RULES = {"chow": 0, "diff": 1, "opt": 2, "always": 3, "never": 4,
-         "token_v1": 5, "token_v2": 6, "token_v3": 7, "lossy": 8, "bild": 9}
+         "token_v1": 5, "token_v2": 6, "token_v3": 7, "lossy": 8, "bild": 9,
+         "chow_log": 10, "diff_log": 11, "opt_log": 12}
 DTYPES = {"f32": 0, "bf16": 1}
 ROW = dict(maxq=0, maxp=1, tv=2, delta=3, accept=4, qx=5, pix=6, margin_delta=7, margin_accept=8)
 SEQ = dict(min_margin=0, sample_margin=1, status=2, bonus_maxp=3)

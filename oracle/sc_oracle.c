@@ -36,7 +36,19 @@
  *          norm(max(0, p/beta - q)); pi need not sum to one), beta >= 1 - alpha;
  *       BiLD*:  delta = 1(D(q, p) > alpha), D(q, p) = -sum_v q(v) log p(v) (the
  *          temperature-sampling discrepancy of the experiments' appendix),
- *          pi = (1 - delta) q + delta p.
+ *          pi = (1 - delta) q + delta p;
+ *
+ *   or the log-loss plug-in rules (appendix on log loss), delta by entropies:
+ *       ChowLog: H(q) > alpha;   DiffLog: sum q log q < sum p log p - alpha;
+ *       OPTLog:  sum q log q < sum p log p - alpha D_TV(p, q);
+ *
+ *   and, with T = 0, greedy decoding (appendix, the greedy special case): the
+ *   rule is evaluated on the untempered softmax (T = 1) except that its D_TV is
+ *   that of the one-hot q~, p~ at the argmaxes (lowest index on ties), i.e.
+ *   1(argmax q != argmax p), as in the greedy lemma; pi = (1 - delta) q~ + delta p~,
+ *   and Algorithm 4 runs on those:
+ *   a draft is rejected only when delta = 1 and it is not the verifier's argmax,
+ *   and the residual (and bonus) token is the verifier's argmax.
  *
  * Readings where the paper leaves a choice open:
  *   - the bonus position has no draft row, so pi_gamma := p_gamma (as in
@@ -80,6 +92,9 @@
 #define OR_TOKEN_V3 7 /* token-specific: r(v) = [p(v) < max p (1 - alpha)] */
 #define OR_LOSSY 8    /* lossy speculative decoding target (Table 3, Lemma 2), parameter beta */
 #define OR_BILD 9     /* BiLD*: delta = 1(-sum_v q(v) log p(v) > alpha) */
+#define OR_CHOW_LOG 10 /* H(q) > alpha */
+#define OR_DIFF_LOG 11 /* sum q log q < sum p log p - alpha */
+#define OR_OPT_LOG 12  /* sum q log q < sum p log p - alpha D_TV(p, q) */
 
 /* per-row record layout, [B][gamma][OR_ROW_FIELDS] */
 #define OR_ROW_MAXQ 0
@@ -276,6 +291,26 @@ static double token_target(int rule, double alpha, const void *zp, int dtype, si
     return e;
 }
 
+/* sum_v x(v) log x(v) of a distribution (0 log 0 = 0): minus its entropy. */
+static double neg_entropy(const double *x, int V)
+{
+    csum s = {0.0, 0.0};
+    for (int v = 0; v < V; ++v)
+        if (x[v] > 0.0)
+            csum_add(&s, x[v] * log(x[v]));
+    return csum_value(&s);
+}
+
+/* Lowest index of the largest entry. */
+static int argmax_of(const double *x, int V)
+{
+    int a = 0;
+    for (int v = 1; v < V; ++v)
+        if (x[v] > x[a])
+            a = v;
+    return a;
+}
+
 /* The lossy speculative-decoding target of one token (Table 3). */
 static double lossy_pi(double qv, double pv, double alpha, double beta)
 {
@@ -361,6 +396,8 @@ static void verify_sequence(const void *draft, const void *target, int dtype,
         if (!(u[j] >= 0.0f && u[j] < 1.0f))
             status |= OR_BAD_UNIFORM;
 
+    const int greedy = !(T > 0.0);       /* T = 0: greedy decoding */
+    const double Tr = greedy ? 1.0 : T;   /* temperature of the rule's distributions */
     const int token = rule >= OR_TOKEN_V1 && rule <= OR_TOKEN_V3;
     const int lossy = rule == OR_LOSSY;
     int jstar = gamma;          /* a_gamma = 0 */
@@ -368,20 +405,22 @@ static void verify_sequence(const void *draft, const void *target, int dtype,
     int delta_star = 0;         /* delta at j* */
     for (int j = 0; j < gamma; ++j) {
         double Mq, lnSq, Mp, lnSp;
-        int okq = tempered_softmax_ln(draft, dtype, dbase + (size_t)j * V, V, T, q, &Mq, &lnSq);
-        int okp = tempered_softmax_ln(target, dtype, tbase + (size_t)j * V, V, T, p, &Mp, &lnSp);
+        int okq = tempered_softmax_ln(draft, dtype, dbase + (size_t)j * V, V, Tr, q, &Mq, &lnSq);
+        int okp = tempered_softmax_ln(target, dtype, tbase + (size_t)j * V, V, Tr, p, &Mp, &lnSp);
         if (okq || okp) {
             status |= OR_BAD_LOGIT;
             continue;
         }
         double maxq = max_of(q, V), maxp = max_of(p, V), tv = tv_distance(p, q, V);
+        if (greedy)  /* the rules' D_TV is that of the one-hot q~, p~: 1(argmax q != argmax p) */
+            tv = argmax_of(q, V) != argmax_of(p, V);
         double m_delta, m_acc = INFINITY;
         int delta;
         int accept = 1;
         double qx = 0.0, pix = 0.0;
         if (token) {
             /* token-specific target (TokenSpecCascade): w holds r(v) for this row */
-            const double eta = token_target(rule, alpha, target, dtype, tbase + (size_t)j * V, Mp, T,
+            const double eta = token_target(rule, alpha, target, dtype, tbase + (size_t)j * V, Mp, Tr,
                                             q, p, V, maxp, w, NULL, &m_delta);
             delta = 0;
             if (!(status & OR_BAD_TOKEN)) {
@@ -392,8 +431,8 @@ static void verify_sequence(const void *draft, const void *target, int dtype,
                 if (rx) {
                     /* pi(x)/q(x) = eta p(x)/q(x), from log-probabilities; a draft with
                        q(x) <= pi(x) (or q(x) = 0) is always accepted */
-                    double lq = log_prob(draft, dtype, dbase + (size_t)j * V, x[j], T, Mq, lnSq);
-                    double lp = log_prob(target, dtype, tbase + (size_t)j * V, x[j], T, Mp, lnSp);
+                    double lq = log_prob(draft, dtype, dbase + (size_t)j * V, x[j], Tr, Mq, lnSq);
+                    double lp = log_prob(target, dtype, tbase + (size_t)j * V, x[j], Tr, Mp, lnSp);
                     double ratio = eta > 0.0 ? exp(lp - lq + log(eta)) : 0.0;
                     if (lq > -INFINITY && ratio < 1.0) {
                         accept = (double)u[j] < ratio;
@@ -408,8 +447,8 @@ static void verify_sequence(const void *draft, const void *target, int dtype,
             if (!(status & OR_BAD_TOKEN)) {
                 qx = q[x[j]];
                 pix = lossy_pi(qx, p[x[j]], alpha, beta);
-                double lq = log_prob(draft, dtype, dbase + (size_t)j * V, x[j], T, Mq, lnSq);
-                double lp = log_prob(target, dtype, tbase + (size_t)j * V, x[j], T, Mp, lnSp);
+                double lq = log_prob(draft, dtype, dbase + (size_t)j * V, x[j], Tr, Mq, lnSq);
+                double lp = log_prob(target, dtype, tbase + (size_t)j * V, x[j], Tr, Mp, lnSp);
                 if (lq > -INFINITY) {
                     double pq = exp(lp - lq);
                     double a = alpha < 1.0 ? pq / (1.0 - alpha) : INFINITY;
@@ -421,22 +460,38 @@ static void verify_sequence(const void *draft, const void *target, int dtype,
                     }
                 }
             }
+        } else if (rule >= OR_CHOW_LOG) {
+            const double nhq = neg_entropy(q, V), nhp = neg_entropy(p, V);
+            double lhs = nhq, rhs;
+            if (rule == OR_CHOW_LOG) { lhs = -nhq; rhs = alpha; delta = lhs > rhs; }  /* H(q) > alpha */
+            else {
+                rhs = rule == OR_DIFF_LOG ? nhp - alpha : nhp - alpha * tv;
+                delta = lhs < rhs;
+            }
+            m_delta = fabs(lhs - rhs);
         } else if (rule == OR_BILD) {
-            const double D = cross_entropy(q, target, dtype, tbase + (size_t)j * V, V, T, Mp, lnSp);
+            const double D = cross_entropy(q, target, dtype, tbase + (size_t)j * V, V, Tr, Mp, lnSp);
             delta = D > alpha;  /* strict, as printed */
             m_delta = isfinite(D) ? fabs(D - alpha) : INFINITY;
         } else {
             delta = deferral(rule, alpha, maxq, maxp, tv, &m_delta);
         }
-        if (!token && !lossy && !(status & OR_BAD_TOKEN)) {
+        if (greedy && !(status & OR_BAD_TOKEN)) {
+            /* one-hot q~, p~: pi(x)/q~(x) is 1 unless delta = 1 and x is not p's
+               argmax (then 0); a draft with q~(x) = 0 is accepted (reading 3) */
+            const int aq = argmax_of(q, V), ap = argmax_of(p, V);
+            qx = x[j] == aq;
+            pix = delta ? (double)(x[j] == ap) : qx;
+            accept = !(qx && delta && x[j] != ap);
+        } else if (!token && !lossy && !(status & OR_BAD_TOKEN)) {
             qx = q[x[j]];
             pix = delta ? p[x[j]] : qx; /* pi(x) = (1 - delta) q(x) + delta p(x) */
             if (delta) {
                 /* pi(x)/q(x) = p(x)/q(x), formed from log-probabilities so that it
                    stays exact when both underflow; q(x) <= pi(x) always accepts
                    (q(x) = 0 only for a -inf logit) */
-                double lq = log_prob(draft, dtype, dbase + (size_t)j * V, x[j], T, Mq, lnSq);
-                double lp = log_prob(target, dtype, tbase + (size_t)j * V, x[j], T, Mp, lnSp);
+                double lq = log_prob(draft, dtype, dbase + (size_t)j * V, x[j], Tr, Mq, lnSq);
+                double lp = log_prob(target, dtype, tbase + (size_t)j * V, x[j], Tr, Mp, lnSp);
                 if (lq > lp) {
                     double ratio = exp(lp - lq);
                     accept = (double)u[j] < ratio;
@@ -468,22 +523,30 @@ static void verify_sequence(const void *draft, const void *target, int dtype,
 
     /* The bonus row is always checked, so that its max p is reported. */
     double bonus_maxp = NAN;
-    if (tempered_softmax(target, dtype, tbase + (size_t)gamma * V, V, T, p) == 0)
+    if (tempered_softmax(target, dtype, tbase + (size_t)gamma * V, V, Tr, p) == 0)
         bonus_maxp = max_of(p, V);
     else
         status |= OR_BAD_LOGIT;
 
     int tok = -1;
     double m_sample = 0.0;
-    if (status == 0) {
+    if (status == 0 && greedy) {
+        /* the residual max(0, pi - q~) = delta max(0, p~ - q~) of row j*, and the
+           bonus pi_gamma = p~_gamma, are one-hot at the verifier's argmax */
+        tempered_softmax(target, dtype, tbase + (size_t)jstar * V, V, Tr, p);
+        tok = argmax_of(p, V);
+        m_sample = INFINITY;
+        num_accepted[b] = jstar;
+        next_token[b] = tok;
+    } else if (status == 0) {
         if (jstar < gamma && token) {
             /* residual norm(max(0, pi - q)) of row j* with the token-specific
                target: max(0, eta p(v) - r(v) q(v)) */
             double Mp, lnSp, m_unused;
-            tempered_softmax(draft, dtype, dbase + (size_t)jstar * V, V, T, q);
-            tempered_softmax_ln(target, dtype, tbase + (size_t)jstar * V, V, T, p, &Mp, &lnSp);
+            tempered_softmax(draft, dtype, dbase + (size_t)jstar * V, V, Tr, q);
+            tempered_softmax_ln(target, dtype, tbase + (size_t)jstar * V, V, Tr, p, &Mp, &lnSp);
             const double eta = token_target(rule, alpha, target, dtype, tbase + (size_t)jstar * V, Mp,
-                                            T, q, p, V, max_of(p, V), w, NULL, &m_unused);
+                                            Tr, q, p, V, max_of(p, V), w, NULL, &m_unused);
             for (int v = 0; v < V; ++v) {
                 double d = eta * p[v] - w[v] * q[v];
                 w[v] = d > 0.0 ? d : 0.0;
@@ -491,8 +554,8 @@ static void verify_sequence(const void *draft, const void *target, int dtype,
             tok = inverse_cdf(w, V, (double)u[gamma], &m_sample);
         } else if (jstar < gamma && lossy) {
             /* residual norm(max(0, pi - q)) of row j* with the lossy target */
-            tempered_softmax(draft, dtype, dbase + (size_t)jstar * V, V, T, q);
-            tempered_softmax(target, dtype, tbase + (size_t)jstar * V, V, T, p);
+            tempered_softmax(draft, dtype, dbase + (size_t)jstar * V, V, Tr, q);
+            tempered_softmax(target, dtype, tbase + (size_t)jstar * V, V, Tr, p);
             for (int v = 0; v < V; ++v) {
                 double d = lossy_pi(q[v], p[v], alpha, beta) - q[v];
                 w[v] = d > 0.0 ? d : 0.0;
@@ -501,8 +564,8 @@ static void verify_sequence(const void *draft, const void *target, int dtype,
         } else if (jstar < gamma) {
             /* residual norm(max(0, pi - q)) of row j*; pi = p there since a
                rejection implies delta = 1 */
-            tempered_softmax(draft, dtype, dbase + (size_t)jstar * V, V, T, q);
-            tempered_softmax(target, dtype, tbase + (size_t)jstar * V, V, T, p);
+            tempered_softmax(draft, dtype, dbase + (size_t)jstar * V, V, Tr, q);
+            tempered_softmax(target, dtype, tbase + (size_t)jstar * V, V, Tr, p);
             for (int v = 0; v < V; ++v) {
                 double pi = delta_star ? p[v] : q[v];
                 double d = pi - q[v];
@@ -562,8 +625,10 @@ int oracle_verify(const void *draft, const void *target, int dtype, const int32_
 {
     if (!draft || !target || !tokens || !uniforms || !num_accepted || !next_token)
         return -1;
-    if (B < 0 || gamma < 1 || V < 1 || !(T > 0.0) || rule < 0 || rule > OR_BILD)
+    if (B < 0 || gamma < 1 || V < 1 || !(T >= 0.0) || rule < 0 || rule > OR_OPT_LOG)
         return -1;
+    if (T == 0.0 && ((rule >= OR_TOKEN_V1 && rule <= OR_TOKEN_V3) || rule == OR_LOSSY))
+        return -1;  /* greedy decoding is defined for the scalar deferral rules */
     if (rule == OR_LOSSY && !(beta > 0.0 && beta >= 1.0 - alpha))
         return -1;
     int failed = 0;

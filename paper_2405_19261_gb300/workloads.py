@@ -44,7 +44,8 @@ from typing import Optional
 import numpy as np
 
 RULES = {"chow": 0, "diff": 1, "opt": 2, "always": 3, "never": 4,
-         "token_v1": 5, "token_v2": 6, "token_v3": 7, "lossy": 8, "bild": 9}
+         "token_v1": 5, "token_v2": 6, "token_v3": 7, "lossy": 8, "bild": 9,
+         "chow_log": 10, "diff_log": 11, "opt_log": 12}
 DTYPES = {"f32": 0, "bf16": 1}
 T5_VOCAB = 32128
 GEMMA_VOCAB = 256000
@@ -141,9 +142,12 @@ def draw_uniforms(rng: np.random.Generator, shape) -> np.ndarray:
 
 
 def gumbel_argmax(rng: np.random.Generator, y: np.ndarray, temperature: float) -> np.ndarray:
-    """One exact sample per row from softmax(y / T) by the Gumbel-max trick."""
+    """One exact sample per row from softmax(y / T) by the Gumbel-max trick; with
+    T = 0 (greedy decoding) the row's argmax, lowest index on ties."""
     y = np.asarray(y, dtype=np.float64)
     u = rng.random(size=y.shape)
+    if temperature == 0:
+        return np.argmax(y, axis=-1).astype(np.int32)
     # u in [0, 1): keep the logs finite.
     g = -np.log(-np.log(np.maximum(u, 1e-300)))
     return np.argmax(y / temperature + g, axis=-1).astype(np.int32)

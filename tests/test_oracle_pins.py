@@ -492,3 +492,64 @@ def test_bild_discrepancy_is_the_cross_entropy(alpha):
     # a threshold above every discrepancy defers nothing: every draft is accepted
     big = oracle.verify_workload(w, alpha=1e6)
     assert np.all(big.num_accepted == w.gamma)
+
+
+# ----------------------------------------------------------------- log-loss rules, greedy decoding
+
+@pytest.mark.parametrize("rule,alpha", [("chow_log", 2.0), ("chow_log", 3.5), ("diff_log", 0.2),
+                                        ("opt_log", 0.5), ("opt_log", 2.0)])
+def test_log_loss_rules_use_the_entropies(rule, alpha):
+    """ChowLog: H(q) > alpha; DiffLog: -H(q) < -H(p) - alpha; OPTLog: -H(q) < -H(p) -
+    alpha D_TV(p, q) (the log-loss plug-in rules), with H from scipy.stats.entropy."""
+    from scipy.stats import entropy
+    w = synthetic(10, 4, 300, dtype="f32", kind="gauss", sigma=1.0, rule=rule, alpha=alpha,
+                  temperature=1.2, seed=71)
+    r = oracle.verify_workload(w)
+    for b in range(w.B):
+        for j in range(w.gamma):
+            q = np_softmax(logits_as_f64(w.draft[b, j], "f32"), 1.2)
+            p = np_softmax(logits_as_f64(w.target[b, j], "f32"), 1.2)
+            hq, hp, tv = entropy(q), entropy(p), 0.5 * np.abs(p - q).sum()
+            lhs, rhs = {"chow_log": (hq, alpha), "diff_log": (-hq, -hp - alpha),
+                        "opt_log": (-hq, -hp - alpha * tv)}[rule]
+            want = lhs > rhs if rule == "chow_log" else lhs < rhs
+            if abs(lhs - rhs) > 1e-9:
+                assert r.row("delta")[b, j] == float(want), (b, j, lhs, rhs)
+
+
+def _greedy_spec_decoding(w):
+    """Greedy speculative decoding as its own procedure: a draft survives while it is
+    the verifier's argmax; the first one that is not is replaced by the verifier's
+    argmax, and after gamma survivors the bonus token is the argmax of p_gamma."""
+    na, nt = [], []
+    for b in range(w.B):
+        p = logits_as_f64(w.target[b], w.dtype)
+        for j in range(w.gamma + 1):
+            ap = int(np.argmax(p[j]))
+            if j == w.gamma or w.tokens[b, j] != ap:
+                na.append(j)
+                nt.append(ap)
+                break
+    return np.array(na), np.array(nt)
+
+
+def test_greedy_always_defer_is_greedy_speculative_decoding():
+    w = synthetic(16, 5, 400, dtype="bf16", kind="zipf", sigma=0.3, rule="always", alpha=0.0,
+                  temperature=0.0, seed=81)
+    r = oracle.verify_workload(w)
+    na, nt = _greedy_spec_decoding(w)
+    np.testing.assert_array_equal(r.num_accepted, na)
+    np.testing.assert_array_equal(r.next_token, nt)
+
+
+@pytest.mark.parametrize("alpha", [0.0, 0.05, 0.2, 0.6, 1.0])
+def test_greedy_opt_equals_greedy_diff(alpha):
+    """The greedy special case (appendix): with T -> 0 the OPT rule's TV term is
+    1(argmax q != argmax p), and running OPT is equivalent to running Diff."""
+    w = synthetic(32, 4, 300, dtype="f32", kind="gauss", sigma=1.0, rule="opt", alpha=alpha,
+                  temperature=0.0, seed=91)
+    a = oracle.verify_workload(w)
+    d = oracle.verify_workload(w, rule="diff")
+    np.testing.assert_array_equal(a.num_accepted, d.num_accepted)
+    np.testing.assert_array_equal(a.next_token, d.next_token)
+    assert np.all(a.status == 0)
