@@ -562,6 +562,11 @@ __device__ __forceinline__ float2 log2_prob(float y, float R, float S, float k, 
   return df_norm(t.x, __fadd_rn(__fadd_rn(t.y, yk.y), -log2f(S)));
 }
 
+// A softmax probability from its logit; 0 for a masked (-inf) logit.
+__device__ __forceinline__ float prob_of(float y, float R, float S, float k, float kl) {
+  return y > -INFINITY ? df_exp2(log2_prob(y, R, S, k, kl)) : 0.0f;
+}
+
 // Acceptance of the draft token x (Algorithm 4): a = 1 when delta = 0 or
 // q(x) <= pi(x), else a = [u < pi(x)/q(x)].  L = log2 p(x) - log2 q(x)
 //   = (y_p(x) - y_q(x)) log2(e)/T - (R_p - R_q) + log2(S_q / S_p)
@@ -569,8 +574,10 @@ __device__ __forceinline__ float2 log2_prob(float y, float R, float S, float k, 
 // essentially only the f32 error of log2(S_q / S_p).  With a token rule
 // (Section 4.4) the draft token's own deferral r(x) takes delta's place and
 // pi(x)/q(x) = (1 - r(x)) + eta p(x)/q(x): accepted outright when r(x) = 0,
-// else [u < eta 2^L].  q(x) and pi(x) themselves are evaluated only for the
-// diagnostics output.
+// else [u < eta 2^L].  A masked logit (-inf) is handled before L, whose
+// double-float terms it would turn into NaN: q(x) = 0 accepts, and p(x) = 0 <
+// q(x) makes the ratio 1 - delta.  q(x) and pi(x) themselves are evaluated
+// only for the diagnostics output.
 __device__ __forceinline__ void accept_test(Shared &sh, float yqx, float ypx, float u, float k, float kl,
                                             bool want_probs) {
   if (sh.tok) {
@@ -578,7 +585,11 @@ __device__ __forceinline__ void accept_test(Shared &sh, float yqx, float ypx, fl
     sh.delta = (sh.on_q ? ax : bx) < sh.thr;                           // reported: r(x)
   }
   int accept = 1;
-  if (sh.delta) {
+  if (!(yqx > -INFINITY)) {
+    // q(x) = 0: accepted
+  } else if (!(ypx > -INFINITY)) {
+    accept = !sh.delta;  // p(x) = 0 < q(x): pi(x)/q(x) = 1 - delta (also eta p/q = 0 for a token rule)
+  } else if (sh.delta) {
     const float2 d = two_sum(ypx, -yqx);  // y_p(x) - y_q(x), exactly
     const float2 dk = df_mul_k(d.x, k, kl);
     const float2 r = two_sum(sh.Rp, -sh.Rq);
@@ -594,8 +605,8 @@ __device__ __forceinline__ void accept_test(Shared &sh, float yqx, float ypx, fl
   }
   sh.accept = accept;
   if (want_probs) {
-    const float qx = df_exp2(log2_prob(yqx, sh.Rq, sh.Sq, k, kl));
-    const float px = df_exp2(log2_prob(ypx, sh.Rp, sh.Sp, k, kl));
+    const float qx = prob_of(yqx, sh.Rq, sh.Sq, k, kl);
+    const float px = prob_of(ypx, sh.Rp, sh.Sp, k, kl);
     sh.qx = qx;
     sh.pix = sh.tok ? fmaf(sh.eta, px, sh.delta ? 0.0f : qx) : (sh.delta ? px : qx);
   }

@@ -17,8 +17,9 @@ def load_golden(name):
 def rows_workload(q_probs, p_probs, tokens, uniforms, rule, alpha, temperature=1.0,
                   dtype="f32", B=1):
     """A one-sequence workload (tiled B times) whose logits are log-probabilities."""
-    q = np.log(np.asarray(q_probs, np.float64)).astype(np.float32)
-    p = np.log(np.asarray(p_probs, np.float64)).astype(np.float32)
+    with np.errstate(divide="ignore"):  # probability 0 is the logit -inf
+        q = np.log(np.asarray(q_probs, np.float64)).astype(np.float32)
+        p = np.log(np.asarray(p_probs, np.float64)).astype(np.float32)
     gamma, V = q.shape
     assert p.shape == (gamma + 1, V)
     q = np.broadcast_to(q * np.float32(temperature), (B, gamma, V)).copy()

@@ -171,6 +171,27 @@ def test_forced_rejection_is_rejected():
     assert np.all(r.row("accept")[b, j0] == 0)
 
 
+@pytest.mark.parametrize("u0", [0.0, 0.4, 0.999])
+@pytest.mark.parametrize("u_gamma,token", [(0.3, 0), (0.7, 1)])
+def test_masked_target_token_is_rejected_when_deferring(u0, u_gamma, token):
+    # q = (1/3, 1/3, 1/3), p = (1/2, 1/2, 0), x = 2: p(x) = 0 < q(x), so with delta = 1
+    # min(1, pi(x)/q(x)) = 0 and no uniform accepts (Algorithm 4's Bernoulli draw).
+    # The residual max(0, p - q) = (1/6, 1/6, 0) puts u_gamma = 0.3 on token 0, 0.7 on 1.
+    q = [[1 / 3, 1 / 3, 1 / 3]]
+    p = [[0.5, 0.5, 0.0], [0.2, 0.3, 0.5]]
+    for dtype in ("f32", "bf16"):
+        w = rows_workload(q, p, [2], [u0, u_gamma], "always", 0.0, dtype=dtype)
+        r = oracle.verify_workload(w)
+        assert (r.num_accepted[0], r.next_token[0]) == (0, token)
+        assert r.row("accept")[0, 0] == 0 and r.row("pix")[0, 0] == 0.0
+        # not deferring keeps the draft: pi = q
+        r = oracle.verify_workload(w, rule="never")
+        assert r.num_accepted[0] == 1 and r.row("accept")[0, 0] == 1
+        # a token rule defers x (r(x) = [p(x) < (1 - alpha) max p] = 1): pi(x)/q(x) = eta p(x)/q(x) = 0
+        r = oracle.verify_workload(w, rule="token_v3", alpha=0.3)
+        assert r.num_accepted[0] == 0 and r.row("delta")[0, 0] == 1
+
+
 def test_invalid_inputs_give_defined_outputs():
     w = _random_workload(20, 3, 1, "opt", 0.2, B=5)
     w.tokens[1, 2] = 20            # out of range
