@@ -218,9 +218,6 @@ struct Elt<uint16_t> {  // bf16 bit patterns
   __device__ __forceinline__ static void load8(const uint16_t *s, float (&y)[8]) {
     unpack(*reinterpret_cast<const uint4 *>(s), y);
   }
-  __device__ __forceinline__ static void load8_global(const uint16_t *g, float (&y)[8]) {
-    unpack(__ldcs(reinterpret_cast<const uint4 *>(g)), y);
-  }
   __device__ __forceinline__ static float at(const uint16_t *g, size_t i) {
     return __uint_as_float(static_cast<uint32_t>(g[i]) << 16);
   }
@@ -231,12 +228,6 @@ struct Elt<float> {
   __device__ __forceinline__ static void load8(const float *s, float (&y)[8]) {
     const float4 a = *reinterpret_cast<const float4 *>(s);
     const float4 b = *reinterpret_cast<const float4 *>(s + 4);
-    y[0] = a.x; y[1] = a.y; y[2] = a.z; y[3] = a.w;
-    y[4] = b.x; y[5] = b.y; y[6] = b.z; y[7] = b.w;
-  }
-  __device__ __forceinline__ static void load8_global(const float *g, float (&y)[8]) {
-    const float4 a = __ldcs(reinterpret_cast<const float4 *>(g));
-    const float4 b = __ldcs(reinterpret_cast<const float4 *>(g + 4));
     y[0] = a.x; y[1] = a.y; y[2] = a.z; y[3] = a.w;
     y[4] = b.x; y[5] = b.y; y[6] = b.z; y[7] = b.w;
   }
@@ -252,16 +243,6 @@ __device__ __forceinline__ void load8_smem(const E *s, int e, int n, float (&y)[
   } else {
 #pragma unroll
     for (int i = 0; i < 8; ++i) y[i] = e + i < n ? Elt<E>::at(s, e + i) : -INFINITY;
-  }
-}
-
-template <typename E>
-__device__ __forceinline__ void load8_gmem(const E *g, int e, int n, bool vec, float (&y)[8]) {
-  if (vec && e + 8 <= n) {
-    Elt<E>::load8_global(g + e, y);
-  } else {
-#pragma unroll
-    for (int i = 0; i < 8; ++i) y[i] = e + i < n ? Elt<E>::at(g, e + i) : -INFINITY;
   }
 }
 
@@ -449,7 +430,7 @@ __device__ __forceinline__ RowScalars sample_scalars(float4 r1, float4 r2, float
 // packed f32x2; the bonus row (kPair = false) weighs p.  Returns their sum in
 // index order.  Every pass and the search call exactly this, so the same logit
 // always gets the same weight and the same prefix sums.
-template <bool kPair>
+template <bool kPair, bool kTok>
 __device__ __forceinline__ float vec_weights(const float (&yq)[8], const float (&yp)[8],
                                              const RowScalars &r, float (&w)[8]) {
   const float2 kk = make_float2(r.k, r.k);
@@ -460,7 +441,7 @@ __device__ __forceinline__ float vec_weights(const float (&yq)[8], const float (
     if constexpr (kPair) {
       const float2 a = __ffma2_rn(make_float2(yq[e], yq[e + 1]), kk, make_float2(-r.Rq, -r.Rq));
       const float2 bc = __fadd2_rn(b, make_float2(r.c, r.c));
-      if (r.kind == kResidual) {
+      if (!kTok || r.kind == kResidual) {  // (kTok: the kernel serves a token rule)
         const float2 d = __ffma2_rn(make_float2(ex2(a.x), ex2(a.y)), make_float2(-1.0f, -1.0f),
                                     make_float2(ex2(bc.x), ex2(bc.y)));
         w[e] = fmaxf(0.0f, d.x);
@@ -505,7 +486,7 @@ __device__ __forceinline__ float warp_sum(float v) {
 
 // Weights of one chunk in the ring: per round, the warp's total weight (the
 // segment total) lands in seg[(c, round, warp)].
-template <typename E, bool kPair, bool kFull>
+template <typename E, bool kPair, bool kFull, bool kTok>
 __device__ __forceinline__ void weights_chunk(const E *sq, const E *sp, int n, int c,
                                               const RowScalars &rs, Shared &sh, int lane,
                                               int warp) {
@@ -520,7 +501,7 @@ __device__ __forceinline__ void weights_chunk(const E *sq, const E *sp, int n, i
       if constexpr (kPair) load8_smem(sq, e, n, yq);
       load8_smem(sp, e, n, yp);
     }
-    const float tot = warp_sum(vec_weights<kPair>(yq, yp, rs, w));
+    const float tot = warp_sum(vec_weights<kPair, kTok>(yq, yp, rs, w));
     if (lane == 0) sh.seg[(c * kRounds + r) * kNW + warp] = tot;
   }
 }
@@ -578,9 +559,10 @@ __device__ __forceinline__ float prob_of(float y, float R, float S, float k, flo
 // double-float terms it would turn into NaN: q(x) = 0 accepts, and p(x) = 0 <
 // q(x) makes the ratio 1 - delta.  q(x) and pi(x) themselves are evaluated
 // only for the diagnostics output.
+template <bool kTok>
 __device__ __forceinline__ void accept_test(Shared &sh, float yqx, float ypx, float u, float k, float kl,
                                             bool want_probs) {
-  if (sh.tok) {
+  if (kTok && sh.tok) {
     const float ax = fmaf(yqx, k, -sh.Rq), bx = fmaf(ypx, k, -sh.Rp);  // as vec_weights forms them
     sh.delta = (sh.on_q ? ax : bx) < sh.thr;                           // reported: r(x)
   }
@@ -597,7 +579,7 @@ __device__ __forceinline__ void accept_test(Shared &sh, float yqx, float ypx, fl
     const float lo = __fadd_rn(__fadd_rn(__fadd_rn(s.y, dk.y), __fsub_rn(__fmul_rn(d.y, k), r.y)),
                                log2f(sh.Sq / sh.Sp));
     const float2 L = df_norm(s.x, lo);
-    if (!sh.tok) {
+    if (!(kTok && sh.tok)) {
       if (df_lt(L, 0.0f)) accept = u < df_exp2(L);
     } else if (L.x < INFINITY) {  // (q(x) = 0 accepts)
       accept = u < sh.eta * df_exp2(L);
@@ -608,7 +590,7 @@ __device__ __forceinline__ void accept_test(Shared &sh, float yqx, float ypx, fl
     const float qx = prob_of(yqx, sh.Rq, sh.Sq, k, kl);
     const float px = prob_of(ypx, sh.Rp, sh.Sp, k, kl);
     sh.qx = qx;
-    sh.pix = sh.tok ? fmaf(sh.eta, px, sh.delta ? 0.0f : qx) : (sh.delta ? px : qx);
+    sh.pix = kTok && sh.tok ? fmaf(sh.eta, px, sh.delta ? 0.0f : qx) : (sh.delta ? px : qx);
   }
 }
 
@@ -729,17 +711,17 @@ __device__ __forceinline__ int stream_rev(const Ring<E> &R, Shared &sh, uint32_t
 // Residual weights of one slice: per-(chunk, round, warp) totals in sh.seg.
 enum SliceOrder { kNewestFirst, kNewestFirstResident };
 
-template <typename E>
+template <bool kTok, typename E>
 __device__ __forceinline__ int slice_weights(const Ring<E> &R, Shared &sh, uint32_t &ph,
                                              const RowScalars &rs, SliceOrder order, int lane, int warp) {
   auto body = [&](int c, int s) {
     const int n = R.chunk_len(c);
     if (R.pair) {
-      if (n == kCH) weights_chunk<E, true, true>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
-      else weights_chunk<E, true, false>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
+      if (n == kCH) weights_chunk<E, true, true, kTok>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
+      else weights_chunk<E, true, false, kTok>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
     } else {
-      if (n == kCH) weights_chunk<E, false, true>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
-      else weights_chunk<E, false, false>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
+      if (n == kCH) weights_chunk<E, false, true, kTok>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
+      else weights_chunk<E, false, false, kTok>(R.q(s), R.p(s), n, c, rs, sh, lane, warp);
     }
   };
   return stream_rev(R, sh, ph, order == kNewestFirstResident, body);
@@ -801,7 +783,7 @@ __device__ __forceinline__ bool jstar_settled(unsigned long long m, int G1, int 
 // passes t is taken (the smallest k with C_k > u R).  Without t (u R fell past
 // the last boundary by rounding), the segment's last positive weight.  v0 is
 // the vocabulary index of the chunk start.
-template <typename E>
+template <bool kTok, typename E>
 __device__ __forceinline__ int search_segment(const E *sq, const E *sp, int n, bool pair,
                                               const RowScalars &rs, int v0, int r, bool have_t,
                                               float t, int lane, int warp) {
@@ -809,7 +791,7 @@ __device__ __forceinline__ int search_segment(const E *sq, const E *sp, int n, b
   float yq[8], yp[8], w[8];
   if (pair) load8_smem(sq, e, n, yq);
   load8_smem(sp, e, n, yp);
-  const float vs = pair ? vec_weights<true>(yq, yp, rs, w) : vec_weights<false>(yq, yp, rs, w);
+  const float vs = pair ? vec_weights<true, kTok>(yq, yp, rs, w) : vec_weights<false, kTok>(yq, yp, rs, w);
   const float incl = warp_incl_scan(vs, lane);
   float excl = __shfl_up_sync(0xFFFFFFFFu, incl, 1);
   if (lane == 0) excl = 0.0f;
@@ -845,7 +827,7 @@ __device__ __forceinline__ int search_segment(const E *sq, const E *sp, int n, b
   return tok;
 }
 
-template <typename E>
+template <typename E, bool kTok>
 __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Params P) {
   extern __shared__ __align__(128) unsigned char smem_raw[];
   cg::cluster_group cluster = cg::this_cluster();
@@ -1014,7 +996,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
         }
         if (pending) sh.need_p2 = 1;
         if (pending && !sh.tok) sh.band = 1;
-        if (!pending) accept_test(sh, yqx, ypx, uj, k, P.kl, P.row_info != nullptr);
+        if (!pending) accept_test<kTok>(sh, yqx, ypx, uj, k, P.kl, P.row_info != nullptr);
       }
     }
     // keep the draft-token logits for a decision after the TV pass
@@ -1048,7 +1030,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       if (P.alpha * LB - (sh.maxp - sh.maxq) >= 1e-4f) {
         sh.need_p2 = 0;
         sh.delta = 0;
-        accept_test(sh, sh.xq, sh.xp, uj, k, P.kl, P.row_info != nullptr);
+        accept_test<kTok>(sh, sh.xq, sh.xp, uj, k, P.kl, P.row_info != nullptr);
       }
     }
     __syncthreads();
@@ -1058,7 +1040,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   // for a token rule the same pass sums r(v) q(v) instead (eta)
   if (sh.need_p2) {
     const RowScalars rs = {sh.Rq, sh.Rp, k, sh.c, sh.tok ? kEta : kResidual, sh.on_q, sh.thr, 0.0f};
-    tmo = slice_weights(R, sh, ph, rs, kNewestFirstResident, lane, warp);
+    tmo = slice_weights<kTok>(R, sh, ph, rs, kNewestFirstResident, lane, warp);
     tmo = __syncthreads_or(tmo);
     // exchange 2: push the slice total, one barrier, local reads
     if (tid == 0) {
@@ -1078,12 +1060,12 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
         sh.err |= SC_DEV_TIMEOUT;
       } else if (sh.tok) {
         sh.eta = Rtot / sh.Sq;  // eta = sum_v r(v) q(v)
-        accept_test(sh, sh.xq, sh.xp, uj, k, P.kl, P.row_info != nullptr);
+        accept_test<kTok>(sh, sh.xq, sh.xp, uj, k, P.kl, P.row_info != nullptr);
       } else {
         sh.tv = fminf(1.0f, fmaxf(0.0f, Rtot / sh.Sq));  // Lemma 3: R = S_q D_TV(p, q)
         if (verify) {
           sh.delta = sh.maxq < sh.maxp - P.alpha * sh.tv;  // Eq. 10
-          accept_test(sh, sh.xq, sh.xp, uj, k, P.kl, P.row_info != nullptr);
+          accept_test<kTok>(sh, sh.xq, sh.xp, uj, k, P.kl, P.row_info != nullptr);
         }
       }
     }
@@ -1169,7 +1151,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       const Ring<E> Rj = make_ring<E>(P, smem_raw, b, js, rank);
       // this unit's own row, untouched since pass 1, still has its last chunks in the ring
       const bool resident = js == j && !sh.need_p2;
-      tmo = slice_weights(Rj, sh, ph, rs, resident ? kNewestFirstResident : kNewestFirst, lane, warp);
+      tmo = slice_weights<kTok>(Rj, sh, ph, rs, resident ? kNewestFirstResident : kNewestFirst, lane, warp);
       tmo = __syncthreads_or(tmo);
       if (tid == 0) {
         float tot_r = seg_prefix(sh, Rj.nch * kRounds * kNW);
@@ -1291,11 +1273,11 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
         }
         tmo = __syncthreads_or(tmo);
         if (Rc.pair) {
-          if (n == kCH) weights_chunk<E, true, true>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
-          else weights_chunk<E, true, false>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
+          if (n == kCH) weights_chunk<E, true, true, kTok>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
+          else weights_chunk<E, true, false, kTok>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
         } else {
-          if (n == kCH) weights_chunk<E, false, true>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
-          else weights_chunk<E, false, false>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
+          if (n == kCH) weights_chunk<E, false, true, kTok>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
+          else weights_chunk<E, false, false, kTok>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
         }
         if (tmo && tid == 0) {
           flag_timeout(sh, P);
@@ -1331,7 +1313,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
             if (sh.seg[i + 1] > sh.seg[i]) { sgi = i; break; }
         }
         if (sgi >= 0 && warp == sgi % kNW) {
-          const int tok = search_segment(Rc.q(sl), Rc.p(sl), n, Rc.pair, rs, cr * P.L + cc * kCH,
+          const int tok = search_segment<kTok>(Rc.q(sl), Rc.p(sl), n, Rc.pair, rs, cr * P.L + cc * kCH,
                                          sgi / kNW, sh.cross_seg >= 0, sh.t_seg, lane, warp);
           if (lane == 0) sh.token = tok;
         }
@@ -1359,7 +1341,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
 struct DeviceInfo {
   int smem_optin = 0;
   int sms = 0;
-  bool configured[2] = {false, false};
+  bool configured[4] = {false, false, false, false};  // [dtype][token rule]
 };
 
 DeviceInfo g_dev[64];
@@ -1442,12 +1424,17 @@ bool device_accessible(const void *p) {
   return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
 }
 
+// The kernel is compiled once per rule family: the token-specific rules of
+// Section 4.4 need per-logit r(v) in the weight passes, the SpecCascade rules
+// do not, and a runtime branch there costs the common case a few percent.
 template <typename E>
 int launch(Params P, cudaStream_t stream, int units) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return SC_ERR_CUDA;
   DeviceInfo &di = g_dev[dev];
-  const int ti = sizeof(E) == 2 ? 1 : 0;
+  const bool tok = P.rule >= SC_RULE_TOKEN_V1;
+  const auto kernel = tok ? sc_unit_kernel<E, true> : sc_unit_kernel<E, false>;
+  const int ti = (sizeof(E) == 2 ? 2 : 0) + (tok ? 1 : 0);
   {
     std::lock_guard<std::mutex> lock(g_mu);
     if (!di.smem_optin &&
@@ -1455,11 +1442,11 @@ int launch(Params P, cudaStream_t stream, int units) {
          cudaDeviceGetAttribute(&di.sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess))
       return SC_ERR_CUDA;
     if (!di.configured[ti]) {
-      if (cudaFuncSetAttribute(sc_unit_kernel<E>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                static_cast<int>(smem_bytes<E>())) != cudaSuccess ||
-          cudaFuncSetAttribute(sc_unit_kernel<E>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+          cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
               cudaSuccess ||
-          cudaFuncSetAttribute(sc_unit_kernel<E>, cudaFuncAttributePreferredSharedMemoryCarveout,
+          cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
                                cudaSharedmemCarveoutMaxShared) != cudaSuccess)
         return SC_ERR_CUDA;
       di.configured[ti] = true;
@@ -1486,7 +1473,7 @@ int launch(Params P, cudaStream_t stream, int units) {
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  if (cudaLaunchKernelEx(&cfg, sc_unit_kernel<E>, P) != cudaSuccess) return SC_ERR_CUDA;
+  if (cudaLaunchKernelEx(&cfg, kernel, P) != cudaSuccess) return SC_ERR_CUDA;
   return SC_OK;
 }
 
