@@ -340,6 +340,7 @@ def run_ours(args):
     clocks = sampler.summary()
 
     ms_step = max_over_ranks(ms_total / args.steps, world, dev)
+    mean_accepted = float(na.float().mean().item())  # j* of the last step (the method's own statistic)
     positions = B * g * world
     value = whole_job_rate(B * g, world, ms_step)
 
@@ -400,6 +401,8 @@ def run_ours(args):
                 "config": {"workload": desc, "B": B, "gamma": g, "V": w.V, "logits": w.dtype,
                            "rule": w.rule, "alpha": w.alpha, "temperature": w.temperature,
                            "rows_per_s": w.rows * world / (ms_step / 1e3),
+                           "mean_accepted": mean_accepted,
+                           "acceptance_rate": mean_accepted / g,
                            "l2": ("L2 flushed before every timed step (2x L2 write, then 2x L2 read of another buffer); "
                                   "the steps are queued behind a spin kernel before the first, so no interval waits on the host"
                                   if flush else
