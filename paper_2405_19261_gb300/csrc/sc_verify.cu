@@ -88,6 +88,14 @@ constexpr int kMinBlocksPerSM = SC_MIN_BLOCKS;
 
 enum Mode : int { kVerify = 0, kStats = 1 };
 
+// The kernel is compiled once per rule family.  kFamCascade: the deferral
+// rules of Table 1 and lossy speculative decoding (Table 3); kFamToken: the
+// token-specific rules of Section 4.4, whose weight passes evaluate r(v) per
+// logit; kFamExt: the rules that read entropies or a cross entropy (BiLD*, the
+// log-loss rules) and greedy decoding (T = 0), whose pass 1 also accumulates
+// first moments of the exponents and the rows' argmaxes.
+enum Family : int { kFamCascade = 0, kFamToken = 1, kFamExt = 2 };
+
 struct Params {
   const void *draft;
   const void *target;
@@ -103,6 +111,10 @@ struct Params {
   int cluster;    // CTAs per unit
   int bulk;       // 1: TMA bulk copies, 0: per-thread loads (rows not 16-byte aligned)
   int mode;
+  int greedy;     // T = 0: greedy decoding; the rules' statistics use T = 1 (k = log2(e))
+  float lossy_l;  // lossy speculative decoding: -log2(1 - alpha) as lossy_l + lossy_ll,
+  float lossy_ll; // the shift of log2 of the acceptance ratio (+inf: alpha = 1)
+  float lossy_c;  // -log2(beta): the residual max(0, p / beta - q) is 2^{b + c + lossy_c} - 2^a
   int32_t *num_accepted;
   int32_t *next_token;
   float *row_info;
@@ -255,14 +267,21 @@ struct __align__(16) Shared {
   float2 all_x[kMaxCluster];   // 1: raw logits at the draft token, if in the slice
   float all_r[kMaxCluster];    // 2 (TV pass): the slice's total residual weight
   float all_lb[kMaxCluster];   // OPT band: the slice's lower bound on D_TV
+  float4 all_ext[kMaxCluster]; // 1 (kFamExt): (A_q, A_p, X, -) of the slice, see ExtState
+  int2 all_idx[kMaxCluster];   // 1 (kFamExt): the slice's argmax of q and of p
   int timeout;
   float4 red[kNW];          // (m_q, s_q, m_p, s_p) of each warp
+  float4 ext_red[kNW];      // (kFamExt) (A_q, A_p, X, -) of each warp
+  int2 idx_red[kNW];        // (kFamExt) argmax of q and of p of each warp
   float seg[kEntries + 1];  // per-(chunk, round, warp) weights, then exclusive prefixes
   float xq, xp;             // raw logits at the draft token, when in this slice
   // row state, identical in every CTA of the cluster
   float Mq, Sq, Mp, Sp, Rq, Rp, maxq, maxp, c, tv, qx, pix;
   int err, delta, accept, need_p2, band;
   int tok, on_q;            // a token rule (Section 4.4) and its r(v) test's variable
+  float dl, dr;             // OPT and OPTLog: delta = [dl < dr - alpha D_TV]
+  float nhq, nhp;           // (kFamExt) sum_v q log q and sum_v p log p, in nats
+  int iq, ip;               // (kFamExt) argmax q and argmax p, lowest index on ties
   float thr, eta;           // its r(v) threshold (exponent domain) and eta = sum_v r(v) q(v)
   // sequence finish
   int owner;                // this CTA runs its rank's sample pass of row j*
@@ -397,6 +416,148 @@ __device__ __forceinline__ void online_row<uint16_t, true>(const uint16_t *src, 
   }
   m = mn;
   s = acc;
+}
+
+// Pass-1 state of the kFamExt rules.  With a_v = y^q_v k - r_q and
+// b_v = y^p_v k - r_p relative to the references r = refk(m) of the running
+// maxima m:
+//   sq = sum 2^a,  aq = sum 2^a a,  sp = sum 2^b,  ap = sum 2^b b,  x = sum 2^a b,
+// so that, for the row's final references and sums (log2 q_v = a_v - log2 S_q),
+//   sum_v q log2 q = A_q / S_q - log2 S_q,   sum_v q log2 p = X / S_q - log2 S_p.
+// iq and ip are the lowest indices of the largest q and p logits seen (-1: none).
+// A term whose exponential is 0 contributes 0 to the moments.
+struct ExtState {
+  float mq, sq, aq, mp, sp, ap, x;
+  int iq, ip;
+};
+
+__device__ __forceinline__ ExtState ext_empty() {
+  return {-FLT_MAX, 0.0f, 0.0f, -FLT_MAX, 0.0f, 0.0f, 0.0f, -1, -1};
+}
+
+// Re-reference a partial by dq = r_q - r_q' <= 0 and dp = r_p - r_p' <= 0:
+// a' = a + dq and 2^{a'} = 2^{dq} 2^a, so A' = 2^{dq} (A + dq S) and
+// X' = 2^{dq} (X + dp S_q).  (A reference floored at -1e30 comes with S = 0.)
+__device__ __forceinline__ void ext_rebase(ExtState &e, float dq, float dp) {
+  const float fq = ex2(dq), fp = ex2(dp);
+  e.x = fq * fmaf(dp, e.sq, e.x);
+  e.aq = fq * fmaf(dq, e.sq, e.aq);
+  e.sq = fq * e.sq;
+  e.ap = fp * fmaf(dp, e.sp, e.ap);
+  e.sp = fp * e.sp;
+}
+
+// The index of the larger of two maxima, the lower index on a tie (-1: none).
+__device__ __forceinline__ int pick_index(float ma, int ia, float mb, int ib) {
+  if (ma > mb) return ia;
+  if (mb > ma) return ib;
+  if (ia < 0) return ib;
+  if (ib < 0) return ia;
+  return min(ia, ib);
+}
+
+// b += a: both re-referenced to the larger maxima, then summed.
+__device__ __forceinline__ void ext_merge(ExtState &b, ExtState a, float k) {
+  const float Mq = fmaxf(a.mq, b.mq), Mp = fmaxf(a.mp, b.mp);
+  const float Rq = refk(Mq, k), Rp = refk(Mp, k);
+  ext_rebase(a, refk(a.mq, k) - Rq, refk(a.mp, k) - Rp);
+  ext_rebase(b, refk(b.mq, k) - Rq, refk(b.mp, k) - Rp);
+  b.iq = pick_index(b.mq, b.iq, a.mq, a.iq);
+  b.ip = pick_index(b.mp, b.ip, a.mp, a.ip);
+  b.mq = Mq;
+  b.mp = Mp;
+  b.sq = __fadd_rn(b.sq, a.sq);
+  b.aq = __fadd_rn(b.aq, a.aq);
+  b.sp = __fadd_rn(b.sp, a.sp);
+  b.ap = __fadd_rn(b.ap, a.ap);
+  b.x = __fadd_rn(b.x, a.x);
+}
+
+// Merge the partials of the 32 lanes of a warp (butterfly); lane 0 ends with
+// the warp's partial.
+__device__ __forceinline__ void ext_warp_merge(ExtState &e, float k) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    ExtState t;
+    t.mq = __shfl_xor_sync(0xFFFFFFFFu, e.mq, o);
+    t.sq = __shfl_xor_sync(0xFFFFFFFFu, e.sq, o);
+    t.aq = __shfl_xor_sync(0xFFFFFFFFu, e.aq, o);
+    t.mp = __shfl_xor_sync(0xFFFFFFFFu, e.mp, o);
+    t.sp = __shfl_xor_sync(0xFFFFFFFFu, e.sp, o);
+    t.ap = __shfl_xor_sync(0xFFFFFFFFu, e.ap, o);
+    t.x = __shfl_xor_sync(0xFFFFFFFFu, e.x, o);
+    t.iq = __shfl_xor_sync(0xFFFFFFFFu, e.iq, o);
+    t.ip = __shfl_xor_sync(0xFFFFFFFFu, e.ip, o);
+    ext_merge(e, t, k);
+  }
+}
+
+// Pass 1 of kFamExt on one chunk of the slice (both rows at once, or the bonus
+// row's p alone): this thread's kRounds vectors, in increasing vocabulary
+// order, so that a strict comparison keeps the lowest index of a maximum.  v0
+// is the vocabulary index of the chunk start.  The chunk's terms are summed
+// apart and then added, which keeps the f32 sums short.
+template <typename E, bool kFull, bool kPair>
+__device__ __forceinline__ void ext_chunk(const E *srcq, const E *srcp, int n, int v0, float k,
+                                          ExtState &st) {
+  float yq[kRounds][8], yp[kRounds][8];
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r) {
+    const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
+    if constexpr (kFull) {
+      if constexpr (kPair) Elt<E>::load8(srcq + e, yq[r]);
+      Elt<E>::load8(srcp + e, yp[r]);
+    } else {
+      if constexpr (kPair) load8_smem(srcq, e, n, yq[r]);
+      load8_smem(srcp, e, n, yp[r]);
+    }
+  }
+  float mq = st.mq, mp = st.mp;
+  int iq = st.iq, ip = st.ip;
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r)
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int v = v0 + 8 * (r * kNT + static_cast<int>(threadIdx.x)) + i;
+      if constexpr (kPair) {
+        if (yq[r][i] > mq) {
+          mq = yq[r][i];
+          iq = v;
+        }
+      }
+      if (yp[r][i] > mp) {
+        mp = yp[r][i];
+        ip = v;
+      }
+    }
+  const float rq = refk(mq, k), rp = refk(mp, k);
+  ext_rebase(st, refk(st.mq, k) - rq, refk(st.mp, k) - rp);
+  float sq = 0.0f, aq = 0.0f, sp = 0.0f, ap = 0.0f, x = 0.0f;
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r)
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const float b = fmaf(yp[r][i], k, -rp);
+      const float eb = ex2(b);
+      sp += eb;
+      ap += eb > 0.0f ? eb * b : 0.0f;
+      if constexpr (kPair) {
+        const float a = fmaf(yq[r][i], k, -rq);
+        const float ea = ex2(a);
+        sq += ea;
+        aq += ea > 0.0f ? ea * a : 0.0f;
+        x += ea > 0.0f ? ea * b : 0.0f;
+      }
+    }
+  st.mq = mq;
+  st.mp = mp;
+  st.iq = iq;
+  st.ip = ip;
+  st.sq = __fadd_rn(st.sq, sq);
+  st.aq = __fadd_rn(st.aq, aq);
+  st.sp = __fadd_rn(st.sp, sp);
+  st.ap = __fadd_rn(st.ap, ap);
+  st.x = __fadd_rn(st.x, x);
 }
 
 // Row scalars of the weight formulas.  With a_v = y^q_v k - R_q, b_v = y^p_v k - R_p
