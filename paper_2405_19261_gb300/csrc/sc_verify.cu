@@ -115,6 +115,7 @@ struct Params {
   float lossy_l;  // lossy speculative decoding: -log2(1 - alpha) as lossy_l + lossy_ll,
   float lossy_ll; // the shift of log2 of the acceptance ratio (+inf: alpha = 1)
   float lossy_c;  // -log2(beta): the residual max(0, p / beta - q) is 2^{b + c + lossy_c} - 2^a
+  float beta;     // lossy speculative decoding's beta (Table 3), >= 1 - alpha
   int32_t *num_accepted;
   int32_t *next_token;
   float *row_info;
@@ -207,6 +208,9 @@ __device__ __forceinline__ void st_peer(uint32_t a, float4 v) {
 }
 __device__ __forceinline__ void st_peer(uint32_t a, float2 v) {
   asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(a), "f"(v.x), "f"(v.y) : "memory");
+}
+__device__ __forceinline__ void st_peer(uint32_t a, int2 v) {
+  asm volatile("st.shared::cluster.v2.s32 [%0], {%1, %2};" ::"r"(a), "r"(v.x), "r"(v.y) : "memory");
 }
 __device__ __forceinline__ void st_peer(uint32_t a, float v) {
   asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(a), "f"(v) : "memory");
@@ -492,63 +496,74 @@ __device__ __forceinline__ void ext_warp_merge(ExtState &e, float k) {
   }
 }
 
+__device__ __forceinline__ ExtState ext_load(float4 ms, float4 m1, int2 idx) {
+  return {ms.x, ms.y, m1.x, ms.z, ms.w, m1.y, m1.z, idx.x, idx.y};
+}
+
 // Pass 1 of kFamExt on one chunk of the slice (both rows at once, or the bonus
 // row's p alone): this thread's kRounds vectors, in increasing vocabulary
 // order, so that a strict comparison keeps the lowest index of a maximum.  v0
-// is the vocabulary index of the chunk start.  The chunk's terms are summed
+// is the vocabulary index of the chunk start.  Two reads of shared memory (the
+// maxima, then the terms) keep few logits live; the chunk's terms are summed
 // apart and then added, which keeps the f32 sums short.
+template <typename E, bool kFull>
+__device__ __forceinline__ void load8_chunk(const E *src, int e, int n, float (&y)[8]) {
+  if constexpr (kFull) {
+    Elt<E>::load8(src + e, y);
+  } else {
+    load8_smem(src, e, n, y);
+  }
+}
+
 template <typename E, bool kFull, bool kPair>
 __device__ __forceinline__ void ext_chunk(const E *srcq, const E *srcp, int n, int v0, float k,
                                           ExtState &st) {
-  float yq[kRounds][8], yp[kRounds][8];
-#pragma unroll
-  for (int r = 0; r < kRounds; ++r) {
-    const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
-    if constexpr (kFull) {
-      if constexpr (kPair) Elt<E>::load8(srcq + e, yq[r]);
-      Elt<E>::load8(srcp + e, yp[r]);
-    } else {
-      if constexpr (kPair) load8_smem(srcq, e, n, yq[r]);
-      load8_smem(srcp, e, n, yp[r]);
-    }
-  }
   float mq = st.mq, mp = st.mp;
   int iq = st.iq, ip = st.ip;
 #pragma unroll
-  for (int r = 0; r < kRounds; ++r)
+  for (int r = 0; r < kRounds; ++r) {
+    const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
+    float yq[8], yp[8];
+    if constexpr (kPair) load8_chunk<E, kFull>(srcq, e, n, yq);
+    load8_chunk<E, kFull>(srcp, e, n, yp);
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-      const int v = v0 + 8 * (r * kNT + static_cast<int>(threadIdx.x)) + i;
       if constexpr (kPair) {
-        if (yq[r][i] > mq) {
-          mq = yq[r][i];
-          iq = v;
+        if (yq[i] > mq) {
+          mq = yq[i];
+          iq = v0 + e + i;
         }
       }
-      if (yp[r][i] > mp) {
-        mp = yp[r][i];
-        ip = v;
+      if (yp[i] > mp) {
+        mp = yp[i];
+        ip = v0 + e + i;
       }
     }
+  }
   const float rq = refk(mq, k), rp = refk(mp, k);
   ext_rebase(st, refk(st.mq, k) - rq, refk(st.mp, k) - rp);
   float sq = 0.0f, aq = 0.0f, sp = 0.0f, ap = 0.0f, x = 0.0f;
 #pragma unroll
-  for (int r = 0; r < kRounds; ++r)
+  for (int r = 0; r < kRounds; ++r) {
+    const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
+    float yq[8], yp[8];
+    if constexpr (kPair) load8_chunk<E, kFull>(srcq, e, n, yq);
+    load8_chunk<E, kFull>(srcp, e, n, yp);
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-      const float b = fmaf(yp[r][i], k, -rp);
+      const float b = fmaf(yp[i], k, -rp);
       const float eb = ex2(b);
       sp += eb;
       ap += eb > 0.0f ? eb * b : 0.0f;
       if constexpr (kPair) {
-        const float a = fmaf(yq[r][i], k, -rq);
+        const float a = fmaf(yq[i], k, -rq);
         const float ea = ex2(a);
         sq += ea;
         aq += ea > 0.0f ? ea * a : 0.0f;
         x += ea > 0.0f ? ea * b : 0.0f;
       }
     }
+  }
   st.mq = mq;
   st.mp = mp;
   st.iq = iq;
@@ -716,13 +731,29 @@ __device__ __forceinline__ float prob_of(float y, float R, float S, float k, flo
 // essentially only the f32 error of log2(S_q / S_p).  With a token rule
 // (Section 4.4) the draft token's own deferral r(x) takes delta's place and
 // pi(x)/q(x) = (1 - r(x)) + eta p(x)/q(x): accepted outright when r(x) = 0,
-// else [u < eta 2^L].  A masked logit (-inf) is handled before L, whose
-// double-float terms it would turn into NaN: q(x) = 0 accepts, and p(x) = 0 <
-// q(x) makes the ratio 1 - delta.  q(x) and pi(x) themselves are evaluated
-// only for the diagnostics output.
-template <bool kTok>
-__device__ __forceinline__ void accept_test(Shared &sh, float yqx, float ypx, float u, float k, float kl,
-                                            bool want_probs) {
+// else [u < eta 2^L].  With lossy speculative decoding (Table 3, delta = 1)
+// the ratio is min(1, p(x) / ((1 - alpha) q(x))) (Lemma 2): L shifted by
+// -log2(1 - alpha).  Greedy decoding compares indices only.  A masked logit
+// (-inf) is handled before L, whose double-float terms it would turn into NaN:
+// q(x) = 0 accepts, and p(x) = 0 < q(x) makes the ratio 1 - delta.  q(x) and
+// pi(x) themselves are evaluated only for the diagnostics output.
+template <int kFam>
+__device__ __forceinline__ void accept_test(Shared &sh, const Params &P, int x, float yqx, float ypx,
+                                            float u, float k) {
+  constexpr bool kTok = kFam == kFamToken;
+  const float kl = P.kl;
+  if constexpr (kFam == kFamExt) {
+    if (P.greedy) {
+      // one-hot q~ and p~ at the argmaxes: pi(x)/q~(x) is 1 unless delta = 1 and
+      // x is not p's argmax (then 0); a draft with q~(x) = 0 is accepted
+      const bool on_q = x == sh.iq, on_p = x == sh.ip;
+      sh.accept = !(on_q && sh.delta && !on_p);
+      sh.qx = on_q ? 1.0f : 0.0f;
+      sh.pix = sh.delta ? (on_p ? 1.0f : 0.0f) : sh.qx;
+      return;
+    }
+  }
+  const bool lossy = kFam == kFamCascade && P.rule == SC_RULE_LOSSY;
   if (kTok && sh.tok) {
     const float ax = fmaf(yqx, k, -sh.Rq), bx = fmaf(ypx, k, -sh.Rp);  // as vec_weights forms them
     sh.delta = (sh.on_q ? ax : bx) < sh.thr;                           // reported: r(x)
@@ -739,19 +770,29 @@ __device__ __forceinline__ void accept_test(Shared &sh, float yqx, float ypx, fl
     const float2 s = two_sum(dk.x, -r.x);
     const float lo = __fadd_rn(__fadd_rn(__fadd_rn(s.y, dk.y), __fsub_rn(__fmul_rn(d.y, k), r.y)),
                                log2f(sh.Sq / sh.Sp));
-    const float2 L = df_norm(s.x, lo);
-    if (!(kTok && sh.tok)) {
+    float2 L = df_norm(s.x, lo);
+    if (kTok && sh.tok) {
+      if (L.x < INFINITY) accept = u < sh.eta * df_exp2(L);  // (q(x) = 0 accepts)
+    } else {
+      if (lossy) {
+        if (P.lossy_l < INFINITY) {
+          const float2 t = two_sum(L.x, P.lossy_l);
+          L = df_norm(t.x, __fadd_rn(__fadd_rn(t.y, L.y), P.lossy_ll));
+        } else {
+          L = make_float2(0.0f, 0.0f);  // alpha = 1: the ratio is 1
+        }
+      }
       if (df_lt(L, 0.0f)) accept = u < df_exp2(L);
-    } else if (L.x < INFINITY) {  // (q(x) = 0 accepts)
-      accept = u < sh.eta * df_exp2(L);
     }
   }
   sh.accept = accept;
-  if (want_probs) {
+  if (P.row_info != nullptr) {
     const float qx = prob_of(yqx, sh.Rq, sh.Sq, k, kl);
     const float px = prob_of(ypx, sh.Rp, sh.Sp, k, kl);
     sh.qx = qx;
-    sh.pix = kTok && sh.tok ? fmaf(sh.eta, px, sh.delta ? 0.0f : qx) : (sh.delta ? px : qx);
+    if (kTok && sh.tok) sh.pix = fmaf(sh.eta, px, sh.delta ? 0.0f : qx);
+    else if (lossy) sh.pix = fmaxf(fminf(qx, P.alpha < 1.0f ? px / (1.0f - P.alpha) : INFINITY), px / P.beta);
+    else sh.pix = sh.delta ? px : qx;
   }
 }
 
@@ -988,8 +1029,10 @@ __device__ __forceinline__ int search_segment(const E *sq, const E *sp, int n, b
   return tok;
 }
 
-template <typename E, bool kTok>
+template <typename E, int kFam>
 __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Params P) {
+  constexpr bool kTok = kFam == kFamToken;
+  constexpr bool kExt = kFam == kFamExt;
   extern __shared__ __align__(128) unsigned char smem_raw[];
   cg::cluster_group cluster = cg::this_cluster();
   const int C = P.cluster;
@@ -1039,10 +1082,20 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   const float k = P.k;
   float mq = -FLT_MAX, mp = -FLT_MAX;
   float2 s2q = make_float2(0.0f, 0.0f), s2p = make_float2(0.0f, 0.0f);
+  ExtState ex = ext_empty();  // (kFamExt) moments and argmaxes
   const int lx = x - v0;  // draft token's offset in this slice (thread 0 only)
   int tmo = stream(R, sh, ph, [&](int c, int s) {
     const int n = R.chunk_len(c);
-    if (n == kCH) {
+    if constexpr (kExt) {
+      const int vc = v0 + c * kCH;
+      if (pair) {
+        if (n == kCH) ext_chunk<E, true, true>(R.q(s), R.p(s), n, vc, k, ex);
+        else ext_chunk<E, false, true>(R.q(s), R.p(s), n, vc, k, ex);
+      } else {
+        if (n == kCH) ext_chunk<E, true, false>(R.q(s), R.p(s), n, vc, k, ex);
+        else ext_chunk<E, false, false>(R.q(s), R.p(s), n, vc, k, ex);
+      }
+    } else if (n == kCH) {
       if (pair) online_row<E, true>(R.q(s), n, k, mq, s2q);
       online_row<E, true>(R.p(s), n, k, mp, s2p);
     } else {
@@ -1054,19 +1107,44 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       sh.xp = Elt<E>::at(R.p(s), lx - c * kCH);
     }
   });
+  if constexpr (kExt) {
+    mq = ex.mq;
+    mp = ex.mp;
+    s2q = make_float2(ex.sq, 0.0f);
+    s2p = make_float2(ex.sp, 0.0f);
+  }
   float s_q = s2q.x + s2q.y, s_p = s2p.x + s2p.y;
   const float4 mine = make_float4(mq, s_q, mp, s_p);  // this thread's partial, kept for the D_TV bound
   tmo = __syncthreads_or(tmo);
-  warp_ms_merge(mq, s_q, k);
-  warp_ms_merge(mp, s_p, k);
-  if (lane == 0) sh.red[warp] = make_float4(mq, s_q, mp, s_p);
+  if constexpr (kExt) {
+    ext_warp_merge(ex, k);
+    if (lane == 0) {
+      sh.red[warp] = make_float4(ex.mq, ex.sq, ex.mp, ex.sp);
+      sh.ext_red[warp] = make_float4(ex.aq, ex.ap, ex.x, 0.0f);
+      sh.idx_red[warp] = make_int2(ex.iq, ex.ip);
+    }
+  } else {
+    warp_ms_merge(mq, s_q, k);
+    warp_ms_merge(mp, s_p, k);
+    if (lane == 0) sh.red[warp] = make_float4(mq, s_q, mp, s_p);
+  }
   __syncthreads();
   // ---- exchange 1: thread 0 merges the warp partials into the slice partial
   // and pushes it into every CTA of the cluster; one barrier; then every read
   // is local, and thread 0 decides
   float4 part = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+  float4 part_ext = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+  int2 part_idx = make_int2(-1, -1);
   if (tid == 0) {
-    part = merge_partials(sh.red, kNW, k);
+    if constexpr (kExt) {
+      ExtState e = ext_load(sh.red[0], sh.ext_red[0], sh.idx_red[0]);
+      for (int w = 1; w < kNW; ++w) ext_merge(e, ext_load(sh.red[w], sh.ext_red[w], sh.idx_red[w]), k);
+      part = make_float4(e.mq, e.sq, e.mp, e.sp);
+      part_ext = make_float4(e.aq, e.ap, e.x, 0.0f);
+      part_idx = make_int2(e.iq, e.ip);
+    } else {
+      part = merge_partials(sh.red, kNW, k);
+    }
     if (tmo) {
       part.y = NAN;
       part.w = NAN;
@@ -1079,13 +1157,26 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     for (int r = 0; r < C; ++r) {
       st_peer(peer_addr(&sh.all_ms[rank], r), part);
       st_peer(peer_addr(&sh.all_x[rank], r), xv);
+      if constexpr (kExt) {
+        st_peer(peer_addr(&sh.all_ext[rank], r), part_ext);
+        st_peer(peer_addr(&sh.all_idx[rank], r), part_idx);
+      }
     }
   }
   cluster_arrive();
   cluster_wait();
 
   if (tid == 0) {  // thread 0 also holds the prefetched scalars
-    const float4 v = merge_partials(sh.all_ms, C, k);  // the row's M and S over the cluster
+    // the row's M and S over the cluster (and, for kFamExt, its moments and argmaxes)
+    ExtState g = ext_empty();
+    float4 v;
+    if constexpr (kExt) {
+      g = ext_load(sh.all_ms[0], sh.all_ext[0], sh.all_idx[0]);
+      for (int r = 1; r < C; ++r) ext_merge(g, ext_load(sh.all_ms[r], sh.all_ext[r], sh.all_idx[r]), k);
+      v = make_float4(g.mq, g.sq, g.mp, g.sp);
+    } else {
+      v = merge_partials(sh.all_ms, C, k);
+    }
     const float a = v.x, as = v.y, c = v.z, cs = v.w;
     const float2 xv = sh.all_x[(x >= 0 && x < P.V) ? x / P.L : 0];
     const float yqx = xv.x, ypx = xv.y;
@@ -1119,6 +1210,19 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     sh.qx = 0.0f;
     sh.pix = 0.0f;
     sh.c = pair && !err ? log2f(as / cs) : 0.0f;
+    sh.dl = sh.maxq;
+    sh.dr = sh.maxp;
+    float xent = 0.0f;  // (kFamExt) BiLD*'s discrepancy D(q, p) = -sum_v q log p, in nats
+    if constexpr (kExt) {
+      // sum q ln q = ln 2 (A_q / S_q - log2 S_q), sum q ln p = ln 2 (X / S_q - log2 S_p)
+      constexpr float kLn2 = 0.69314718f;
+      sh.iq = g.iq;
+      sh.ip = g.ip;
+      sh.nhq = kLn2 * (g.aq / as - log2f(as));
+      sh.nhp = kLn2 * (g.ap / cs - log2f(cs));
+      xent = kLn2 * (log2f(cs) - g.x / as);
+      if (P.greedy && pair) sh.tv = g.iq != g.ip ? 1.0f : 0.0f;  // D_TV of the one-hot q~, p~
+    }
     if (!err && pair) {
       if (!verify) {
         sh.need_p2 = 1;  // sc_row_stats: TV of every pair
@@ -1130,12 +1234,29 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
           case SC_RULE_CHOW: sh.delta = maxq < 1.0f - al; break;  // Eq. 2
           case SC_RULE_DIFF: sh.delta = maxq < maxp - al; break;  // Eq. 5
           case SC_RULE_OPT:                                       // Eq. 10
+            if (kExt) {  // greedy decoding: the one-hot D_TV is known
+              sh.delta = maxq < maxp - al * sh.tv;
+              break;
+            }
             // alpha * TV lies in [0, alpha]: TV decides only inside that band
             if (!(maxq < maxp)) sh.delta = 0;
             else if (maxq < maxp - al) sh.delta = 1;
             else pending = true;
             break;
           case SC_RULE_ALWAYS_DEFER: sh.delta = 1; break;
+          case SC_RULE_LOSSY: sh.delta = 1; break;  // Table 3: the target min/max of q, p
+          // Table 3 and the log-loss rules
+          case SC_RULE_BILD: sh.delta = xent > al; break;              // D(q, p) > alpha
+          case SC_RULE_CHOW_LOG: sh.delta = -sh.nhq > al; break;       // H(q) > alpha
+          case SC_RULE_DIFF_LOG: sh.delta = sh.nhq < sh.nhp - al; break;
+          case SC_RULE_OPT_LOG:  // sum q log q < sum p log p - alpha D_TV
+            sh.dl = sh.nhq;
+            sh.dr = sh.nhp;
+            if (P.greedy) sh.delta = sh.nhq < sh.nhp - al * sh.tv;
+            else if (!(sh.nhq < sh.nhp)) sh.delta = 0;
+            else if (sh.nhq < sh.nhp - al) sh.delta = 1;
+            else pending = true;
+            break;
           case SC_RULE_TOKEN_V1:
           case SC_RULE_TOKEN_V2:
           case SC_RULE_TOKEN_V3: {
@@ -1157,7 +1278,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
         }
         if (pending) sh.need_p2 = 1;
         if (pending && !sh.tok) sh.band = 1;
-        if (!pending) accept_test<kTok>(sh, yqx, ypx, uj, k, P.kl, P.row_info != nullptr);
+        if (!pending) accept_test<kFam>(sh, P, x, yqx, ypx, uj, k);
       }
     }
     // keep the draft-token logits for a decision after the TV pass
@@ -1169,8 +1290,9 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   // ---- OPT band: a lower bound on D_TV from the pass-1 partials.  The threads'
   // element sets partition the vocabulary, so sum_t max(0, P_t - Q_t) <= D_TV
   // (P_t, Q_t: the probability mass of thread t's logits).  When alpha times
-  // that bound already reaches max p - max q, delta = 0 for the exact D_TV too
-  // (Eq. 10) and the TV pass is skipped.  The bound carries ~1e-6 of f32
+  // that bound already reaches dr - dl (max p - max q for OPT, Eq. 10; the
+  // negative-entropy gap for OPTLog), delta = 0 for the exact D_TV too and the
+  // TV pass is skipped.  The bound carries ~1e-6 of f32
   // rounding over its 128 C terms; only a clear 1e-4 excess settles the row.
   if (sh.band) {
     const float pt = mine.w * ex2(refk(mine.z, k) - sh.Rp) / sh.Sp;
@@ -1188,10 +1310,10 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     if (tid == 0) {
       float LB = 0.0f;  // in rank order
       for (int r = 0; r < C; ++r) LB = __fadd_rn(LB, sh.all_lb[r]);
-      if (P.alpha * LB - (sh.maxp - sh.maxq) >= 1e-4f) {
+      if (P.alpha * LB - (sh.dr - sh.dl) >= 1e-4f) {
         sh.need_p2 = 0;
         sh.delta = 0;
-        accept_test<kTok>(sh, sh.xq, sh.xp, uj, k, P.kl, P.row_info != nullptr);
+        accept_test<kFam>(sh, P, x, sh.xq, sh.xp, uj, k);
       }
     }
     __syncthreads();
@@ -1221,12 +1343,12 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
         sh.err |= SC_DEV_TIMEOUT;
       } else if (sh.tok) {
         sh.eta = Rtot / sh.Sq;  // eta = sum_v r(v) q(v)
-        accept_test<kTok>(sh, sh.xq, sh.xp, uj, k, P.kl, P.row_info != nullptr);
+        accept_test<kFam>(sh, P, x, sh.xq, sh.xp, uj, k);
       } else {
         sh.tv = fminf(1.0f, fmaxf(0.0f, Rtot / sh.Sq));  // Lemma 3: R = S_q D_TV(p, q)
         if (verify) {
-          sh.delta = sh.maxq < sh.maxp - P.alpha * sh.tv;  // Eq. 10
-          accept_test<kTok>(sh, sh.xq, sh.xp, uj, k, P.kl, P.row_info != nullptr);
+          sh.delta = sh.dl < sh.dr - P.alpha * sh.tv;  // Eq. 10 (or OPTLog)
+          accept_test<kFam>(sh, P, x, sh.xq, sh.xp, uj, k);
         }
       }
     }
@@ -1248,8 +1370,12 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     float4 *rec2 = P.records2 + (static_cast<size_t>(b) * kMaxCluster + rank) * G1;
     if (tid == 0) {
       const int flags = (sh.accept ? 1 : 0) | (sh.err ? 2 : 0);
-      rec[j] = make_float4(sh.Rq, sh.Rp, sh.c, __int_as_float(flags));
-      if (P.rule >= SC_RULE_TOKEN_V1)  // (only token rules read the second record)
+      float4 r1 = make_float4(sh.Rq, sh.Rp, sh.c, __int_as_float(flags));
+      if (kFam == kFamCascade && P.rule == SC_RULE_LOSSY)
+        r1.z = sh.c + P.lossy_c;  // the residual max(0, p / beta - q) (Lemma 2)
+      if (kExt && P.greedy) r1.x = __int_as_float(sh.ip);  // greedy: the token emitted at row j*
+      rec[j] = r1;
+      if (kTok)  // (only token rules read the second record)
         rec2[j] = make_float4(sh.eta, sh.thr, __int_as_float(sh.tok), __int_as_float(sh.on_q));
       if (rank == 0 && P.row_info) {
         float *ri = P.row_info + (static_cast<size_t>(b) * G1 + j) * SC_ROW_FIELDS;
@@ -1300,11 +1426,15 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     }
     if (sh.owner && tid == 0) {  // row j*'s records (they are in)
       sh.rj = __ldcg(&rec[sh.jstar]);
-      sh.rj2 = P.rule >= SC_RULE_TOKEN_V1 ? __ldcg(&rec2[sh.jstar]) : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+      sh.rj2 = kTok ? __ldcg(&rec2[sh.jstar]) : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
     }
     __syncthreads();
 
-    if (sh.owner) {
+    if (sh.owner && kExt && P.greedy) {
+      // greedy decoding emits row j*'s argmax p (in the records): nothing to sample
+      if (tid == 0) sh.seq_last = atom_add_acq_rel(P.seq_tickets + b, 1u) == static_cast<uint32_t>(C);
+      __syncthreads();
+    } else if (sh.owner) {
       // ---- sample pass: weights of this rank's slice of row j* -- the residual
       // max(0, p - q) of a rejected pair (Algorithm 4), or p of the bonus row
       const int js = sh.jstar;
@@ -1336,7 +1466,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       if (tid == 0) P.seq_tickets[b] = 0u;  // every report of the sequence is in
       // one round of loads: every slice's chunk prefixes (ending in its total) ...
       const float *cpg = P.chunk_pre + static_cast<size_t>(b) * kMaxCluster * kCP;
-      for (int i = tid; i < C * kCP; i += kNT) {
+      for (int i = tid; i < C * kCP && !(kExt && P.greedy); i += kNT) {
         const int r = i / kCP, c = i % kCP;
         const int len = max(0, min(P.L, P.V - r * P.L));
         if (c <= (len + kCH - 1) / kCH) cpall[i] = __ldcg(cpg + i);
@@ -1364,129 +1494,141 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
           sh.jstar = js;
           sh.bad = bad;
           sh.rj = rj;
-          sh.rj2 = P.rule >= SC_RULE_TOKEN_V1 ? __ldcg(P.records2 + static_cast<size_t>(b) * kMaxCluster * G1 + js)
+          sh.rj2 = kTok ? __ldcg(P.records2 + static_cast<size_t>(b) * kMaxCluster * G1 + js)
                                               : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
         }
       }
       __syncthreads();
       const int js = sh.jstar;
-      const RowScalars rs = sample_scalars(sh.rj, sh.rj2, k);
-      // ---- inverse CDF over the slices in rank order, u = u[b][gamma], then
-      // over the chunks of the crossing slice
-      if (warp == 0) {
-        auto nch_of = [&](int r) {
-          const int len = max(0, min(P.L, P.V - r * P.L));
-          return (len + kCH - 1) / kCH;
-        };
-        const float tot = lane < C ? cpall[lane * kCP + nch_of(lane)] : 0.0f;
-        const float pre = warp_incl_scan(tot, lane);  // through rank `lane`
-        const float Rtot = __shfl_sync(0xFFFFFFFFu, pre, C - 1);
-        float before = __shfl_up_sync(0xFFFFFFFFu, pre, 1);
-        if (lane == 0) before = 0.0f;
-        const float u = __shfl_sync(0xFFFFFFFFu, ug, 0);
-        const bool ok = !sh.bad && isfinite(Rtot);
-        int cr = -1, cc = -1, clast = -1;
-        float2 tl = make_float2(-1.0f, 0.0f);  // (negative: u R fell past the last boundary)
-        if (ok && Rtot > 0.0f) {
-          const float th = __fmul_rn(u, Rtot);
-          const float2 t = make_float2(th, fmaf(u, Rtot, -th));  // u R_tot, exactly
-          const bool cross = lane < C && tot > 0.0f && df_ge(t, before) && df_lt(t, pre);
-          const unsigned cm = __ballot_sync(0xFFFFFFFFu, cross);
-          const unsigned pm = __ballot_sync(0xFFFFFFFFu, lane < C && tot > 0.0f);
-          cr = cm ? __ffs(cm) - 1 : 31 - __clz(pm);
-          const float bcr = __shfl_sync(0xFFFFFFFFu, before, cr);
-          if (cm) tl = df_sub(t, bcr);
-          // the chunk of slice cr holding tl (or, past a rounding gap, its last chunk with weight)
-          const float *cp = cpall + cr * kCP;
-          const int nch = nch_of(cr);
-          for (int base = 0; base < nch; base += 32) {
-            const int c = base + lane;
-            const float lo = c < nch ? cp[c] : 0.0f, hi = c < nch ? cp[c + 1] : 0.0f;
-            const bool pos = c < nch && hi > lo;
-            const unsigned mi = __ballot_sync(0xFFFFFFFFu, pos && df_ge(tl, lo) && df_lt(tl, hi));
-            const unsigned mp = __ballot_sync(0xFFFFFFFFu, pos);
-            if (cc < 0 && mi) cc = base + __ffs(mi) - 1;
-            if (mp) clast = base + 31 - __clz(mp);
-          }
-        }
-        if (lane == 0) {
-          sh.sample_ok = ok;
-          sh.cross_rank = cr;
-          sh.t_slice = tl;
-          sh.token = -1;
-          sh.cross_chunk = cc >= 0 ? cc : clast;
-          sh.have_t = cc >= 0;
-          sh.chunk_lo = sh.cross_chunk >= 0 ? cpall[cr * kCP + sh.cross_chunk] : 0.0f;
-        }
-      }
-      __syncthreads();
-      const int cr = sh.cross_rank, cc = sh.cross_chunk;
-      if (cr >= 0 && cc >= 0) {
-        // the chunk's weights again, by the code the sample pass ran (the same values)
-        const Ring<E> Rc = make_ring<E>(P, smem_raw, b, js, cr);
-        const int sl = kStages - 1, n = Rc.chunk_len(cc);
-        if (Rc.bulk) {
-          if (tid == 0) Rc.issue(sh, cc, sl);
-          tmo = wait_stage(sh, sl, ph);
-        } else {
-          tmo = 0;
-          Rc.load_sync(cc, sl);
-        }
-        tmo = __syncthreads_or(tmo);
-        if (Rc.pair) {
-          if (n == kCH) weights_chunk<E, true, true, kTok>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
-          else weights_chunk<E, true, false, kTok>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
-        } else {
-          if (n == kCH) weights_chunk<E, false, true, kTok>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
-          else weights_chunk<E, false, false, kTok>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
-        }
-        if (tmo && tid == 0) {
-          flag_timeout(sh, P);
-          sh.sample_ok = 0;
-        }
-        __syncthreads();
-        constexpr int kSegC = kRounds * kNW;  // segments per chunk
+      if (kExt && P.greedy) {
+        // greedy decoding: the argmax p of row j*, from rank 0's record
         if (tid == 0) {
-          // exclusive prefixes continue from the chunk's stored start, as in the sample pass
-          float acc = sh.chunk_lo;
-          for (int i = 0; i < kSegC; ++i) {
-            const float t = sh.seg[i];
-            sh.seg[i] = acc;
-            acc = __fadd_rn(acc, t);
+          const bool ok = !sh.bad;
+          const int tok = __float_as_int(sh.rj.x);
+          P.num_accepted[b] = ok ? js : 0;
+          P.next_token[b] = ok ? tok : -1;
+          if (ok && P.row_info)
+            P.row_info[(static_cast<size_t>(b) * G1 + js) * SC_ROW_FIELDS + SC_ROW_CAND] = static_cast<float>(tok);
+        }
+      } else {
+        const RowScalars rs = sample_scalars(sh.rj, sh.rj2, k);
+        // ---- inverse CDF over the slices in rank order, u = u[b][gamma], then
+        // over the chunks of the crossing slice
+        if (warp == 0) {
+          auto nch_of = [&](int r) {
+            const int len = max(0, min(P.L, P.V - r * P.L));
+            return (len + kCH - 1) / kCH;
+          };
+          const float tot = lane < C ? cpall[lane * kCP + nch_of(lane)] : 0.0f;
+          const float pre = warp_incl_scan(tot, lane);  // through rank `lane`
+          const float Rtot = __shfl_sync(0xFFFFFFFFu, pre, C - 1);
+          float before = __shfl_up_sync(0xFFFFFFFFu, pre, 1);
+          if (lane == 0) before = 0.0f;
+          const float u = __shfl_sync(0xFFFFFFFFu, ug, 0);
+          const bool ok = !sh.bad && isfinite(Rtot);
+          int cr = -1, cc = -1, clast = -1;
+          float2 tl = make_float2(-1.0f, 0.0f);  // (negative: u R fell past the last boundary)
+          if (ok && Rtot > 0.0f) {
+            const float th = __fmul_rn(u, Rtot);
+            const float2 t = make_float2(th, fmaf(u, Rtot, -th));  // u R_tot, exactly
+            const bool cross = lane < C && tot > 0.0f && df_ge(t, before) && df_lt(t, pre);
+            const unsigned cm = __ballot_sync(0xFFFFFFFFu, cross);
+            const unsigned pm = __ballot_sync(0xFFFFFFFFu, lane < C && tot > 0.0f);
+            cr = cm ? __ffs(cm) - 1 : 31 - __clz(pm);
+            const float bcr = __shfl_sync(0xFFFFFFFFu, before, cr);
+            if (cm) tl = df_sub(t, bcr);
+            // the chunk of slice cr holding tl (or, past a rounding gap, its last chunk with weight)
+            const float *cp = cpall + cr * kCP;
+            const int nch = nch_of(cr);
+            for (int base = 0; base < nch; base += 32) {
+              const int c = base + lane;
+              const float lo = c < nch ? cp[c] : 0.0f, hi = c < nch ? cp[c + 1] : 0.0f;
+              const bool pos = c < nch && hi > lo;
+              const unsigned mi = __ballot_sync(0xFFFFFFFFu, pos && df_ge(tl, lo) && df_lt(tl, hi));
+              const unsigned mp = __ballot_sync(0xFFFFFFFFu, pos);
+              if (cc < 0 && mi) cc = base + __ffs(mi) - 1;
+              if (mp) clast = base + 31 - __clz(mp);
+            }
           }
-          sh.seg[kSegC] = acc;
-          const float2 tl = sh.t_slice;
-          int sgi = -1;
-          if (sh.have_t)
-            for (int i = 0; i < kSegC; ++i)
-              if (df_ge(tl, sh.seg[i]) && df_lt(tl, sh.seg[i + 1]) && sh.seg[i + 1] > sh.seg[i]) {
-                sgi = i;
-                break;
-              }
-          sh.cross_seg = sgi;
-          sh.t_seg = sgi >= 0 ? df_floor(df_sub(tl, sh.seg[sgi])) : 0.0f;
+          if (lane == 0) {
+            sh.sample_ok = ok;
+            sh.cross_rank = cr;
+            sh.t_slice = tl;
+            sh.token = -1;
+            sh.cross_chunk = cc >= 0 ? cc : clast;
+            sh.have_t = cc >= 0;
+            sh.chunk_lo = sh.cross_chunk >= 0 ? cpall[cr * kCP + sh.cross_chunk] : 0.0f;
+          }
         }
         __syncthreads();
-        int sgi = sh.cross_seg;
-        if (sgi < 0) {
-          // no t inside the chunk: its last segment with weight
-          for (int i = kSegC - 1; i >= 0; --i)
-            if (sh.seg[i + 1] > sh.seg[i]) { sgi = i; break; }
+        const int cr = sh.cross_rank, cc = sh.cross_chunk;
+        if (cr >= 0 && cc >= 0) {
+          // the chunk's weights again, by the code the sample pass ran (the same values)
+          const Ring<E> Rc = make_ring<E>(P, smem_raw, b, js, cr);
+          const int sl = kStages - 1, n = Rc.chunk_len(cc);
+          if (Rc.bulk) {
+            if (tid == 0) Rc.issue(sh, cc, sl);
+            tmo = wait_stage(sh, sl, ph);
+          } else {
+            tmo = 0;
+            Rc.load_sync(cc, sl);
+          }
+          tmo = __syncthreads_or(tmo);
+          if (Rc.pair) {
+            if (n == kCH) weights_chunk<E, true, true, kTok>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
+            else weights_chunk<E, true, false, kTok>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
+          } else {
+            if (n == kCH) weights_chunk<E, false, true, kTok>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
+            else weights_chunk<E, false, false, kTok>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
+          }
+          if (tmo && tid == 0) {
+            flag_timeout(sh, P);
+            sh.sample_ok = 0;
+          }
+          __syncthreads();
+          constexpr int kSegC = kRounds * kNW;  // segments per chunk
+          if (tid == 0) {
+            // exclusive prefixes continue from the chunk's stored start, as in the sample pass
+            float acc = sh.chunk_lo;
+            for (int i = 0; i < kSegC; ++i) {
+              const float t = sh.seg[i];
+              sh.seg[i] = acc;
+              acc = __fadd_rn(acc, t);
+            }
+            sh.seg[kSegC] = acc;
+            const float2 tl = sh.t_slice;
+            int sgi = -1;
+            if (sh.have_t)
+              for (int i = 0; i < kSegC; ++i)
+                if (df_ge(tl, sh.seg[i]) && df_lt(tl, sh.seg[i + 1]) && sh.seg[i + 1] > sh.seg[i]) {
+                  sgi = i;
+                  break;
+                }
+            sh.cross_seg = sgi;
+            sh.t_seg = sgi >= 0 ? df_floor(df_sub(tl, sh.seg[sgi])) : 0.0f;
+          }
+          __syncthreads();
+          int sgi = sh.cross_seg;
+          if (sgi < 0) {
+            // no t inside the chunk: its last segment with weight
+            for (int i = kSegC - 1; i >= 0; --i)
+              if (sh.seg[i + 1] > sh.seg[i]) { sgi = i; break; }
+          }
+          if (sgi >= 0 && warp == sgi % kNW) {
+            const int tok = search_segment<kTok>(Rc.q(sl), Rc.p(sl), n, Rc.pair, rs, cr * P.L + cc * kCH,
+                                           sgi / kNW, sh.cross_seg >= 0, sh.t_seg, lane, warp);
+            if (lane == 0) sh.token = tok;
+          }
+          __syncthreads();
         }
-        if (sgi >= 0 && warp == sgi % kNW) {
-          const int tok = search_segment<kTok>(Rc.q(sl), Rc.p(sl), n, Rc.pair, rs, cr * P.L + cc * kCH,
-                                         sgi / kNW, sh.cross_seg >= 0, sh.t_seg, lane, warp);
-          if (lane == 0) sh.token = tok;
+        if (tid == 0) {
+          const bool ok = sh.sample_ok != 0;
+          P.num_accepted[b] = ok ? js : 0;
+          P.next_token[b] = ok ? sh.token : -1;
+          if (ok && P.row_info)
+            P.row_info[(static_cast<size_t>(b) * G1 + js) * SC_ROW_FIELDS + SC_ROW_CAND] =
+                static_cast<float>(sh.token);
         }
-        __syncthreads();
-      }
-      if (tid == 0) {
-        const bool ok = sh.sample_ok != 0;
-        P.num_accepted[b] = ok ? js : 0;
-        P.next_token[b] = ok ? sh.token : -1;
-        if (ok && P.row_info)
-          P.row_info[(static_cast<size_t>(b) * G1 + js) * SC_ROW_FIELDS + SC_ROW_CAND] =
-              static_cast<float>(sh.token);
       }
     }
   }
@@ -1502,7 +1644,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
 struct DeviceInfo {
   int smem_optin = 0;
   int sms = 0;
-  bool configured[4] = {false, false, false, false};  // [dtype][token rule]
+  bool configured[6] = {};  // [dtype][rule family]
 };
 
 DeviceInfo g_dev[64];
@@ -1585,17 +1727,24 @@ bool device_accessible(const void *p) {
   return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
 }
 
-// The kernel is compiled once per rule family: the token-specific rules of
-// Section 4.4 need per-logit r(v) in the weight passes, the SpecCascade rules
-// do not, and a runtime branch there costs the common case a few percent.
+// The rule family of a call (see Family): each family is its own kernel, so
+// the SpecCascade rules run without the per-logit branches of the others.
+int family_of(const Params &P) {
+  if (P.greedy || P.rule >= SC_RULE_BILD) return kFamExt;
+  if (P.rule >= SC_RULE_TOKEN_V1 && P.rule <= SC_RULE_TOKEN_V3) return kFamToken;
+  return kFamCascade;
+}
+
 template <typename E>
 int launch(Params P, cudaStream_t stream, int units) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return SC_ERR_CUDA;
   DeviceInfo &di = g_dev[dev];
-  const bool tok = P.rule >= SC_RULE_TOKEN_V1;
-  const auto kernel = tok ? sc_unit_kernel<E, true> : sc_unit_kernel<E, false>;
-  const int ti = (sizeof(E) == 2 ? 2 : 0) + (tok ? 1 : 0);
+  const int fam = family_of(P);
+  const auto kernel = fam == kFamExt     ? sc_unit_kernel<E, kFamExt>
+                      : fam == kFamToken ? sc_unit_kernel<E, kFamToken>
+                                         : sc_unit_kernel<E, kFamCascade>;
+  const int ti = (sizeof(E) == 2 ? 3 : 0) + fam;
   {
     std::lock_guard<std::mutex> lock(g_mu);
     if (!di.smem_optin &&
@@ -1638,12 +1787,14 @@ int launch(Params P, cudaStream_t stream, int units) {
   return SC_OK;
 }
 
+// greedy_ok: T = 0 (greedy decoding) is accepted.
 int common_checks(const void *draft, const void *target, int dtype, int B, int gamma, int V,
-                  float temperature) {
+                  float temperature, bool greedy_ok) {
   if (dtype != SC_F32 && dtype != SC_BF16) return SC_ERR_INVALID_ARG;
   if (B < 1 || gamma < 1 || gamma > SC_MAX_GAMMA || V < 1) return SC_ERR_INVALID_ARG;
   if (V > sc_max_vocab(static_cast<sc_dtype>(dtype))) return SC_ERR_UNSUPPORTED;
-  if (!(temperature > 0.0f) || !std::isfinite(temperature)) return SC_ERR_INVALID_ARG;
+  if (!(temperature > 0.0f || (greedy_ok && temperature == 0.0f)) || !std::isfinite(temperature))
+    return SC_ERR_INVALID_ARG;
   if (static_cast<double>(B) * (gamma + 1) * kMaxCluster > 2147483647.0) return SC_ERR_INVALID_ARG;
   if (!device_accessible(draft) || !device_accessible(target)) return SC_ERR_INVALID_ARG;
   return SC_OK;
@@ -1702,15 +1853,25 @@ int sc_max_vocab(sc_dtype dtype) {
   return kMaxCluster * kMaxChunks * kCH;
 }
 
-int sc_verify_rows(const void *draft_logits, const void *target_logits, sc_dtype dtype,
-                   const int32_t *draft_tokens, const float *uniforms, int B, int gamma, int V,
-                   sc_rule rule, float alpha, float temperature, int32_t *num_accepted,
-                   int32_t *next_token, void *workspace, size_t workspace_bytes,
-                   int32_t *device_status, float *row_info, cudaStream_t stream) {
-  int rc = common_checks(draft_logits, target_logits, dtype, B, gamma, V, temperature);
+int sc_verify_ex(const void *draft_logits, const void *target_logits, sc_dtype dtype,
+                 const int32_t *draft_tokens, const float *uniforms, int B, int gamma, int V,
+                 sc_rule rule, float alpha, float beta, float temperature, int32_t *num_accepted,
+                 int32_t *next_token, void *workspace, size_t workspace_bytes,
+                 int32_t *device_status, float *row_info, cudaStream_t stream) {
+  int rc = common_checks(draft_logits, target_logits, dtype, B, gamma, V, temperature, true);
   if (rc != SC_OK) return rc;
-  if (static_cast<int>(rule) < 0 || static_cast<int>(rule) > SC_RULE_TOKEN_V3) return SC_ERR_INVALID_ARG;
-  if (!(alpha >= 0.0f && alpha <= 1.0f)) return SC_ERR_INVALID_ARG;
+  const int ri = static_cast<int>(rule);
+  if (ri < 0 || ri > SC_RULE_OPT_LOG) return SC_ERR_INVALID_ARG;
+  // alpha: a probability-scale cost for Table 1, lossy and token rules, a
+  // threshold on a (cross) entropy for BiLD* and the log-loss rules
+  if (ri <= SC_RULE_LOSSY ? !(alpha >= 0.0f && alpha <= 1.0f) : !(alpha >= 0.0f && std::isfinite(alpha)))
+    return SC_ERR_INVALID_ARG;
+  const bool greedy = temperature == 0.0f;
+  // greedy decoding is defined for the scalar deferral rules only
+  if (greedy && ((ri >= SC_RULE_TOKEN_V1 && ri <= SC_RULE_TOKEN_V3) || ri == SC_RULE_LOSSY))
+    return SC_ERR_INVALID_ARG;
+  if (ri == SC_RULE_LOSSY && !(beta > 0.0f && std::isfinite(beta) && beta >= 1.0f - alpha))
+    return SC_ERR_INVALID_ARG;
   if (!device_accessible(draft_tokens) || !device_accessible(uniforms) ||
       !device_accessible(num_accepted) || !device_accessible(next_token))
     return SC_ERR_INVALID_ARG;
@@ -1727,10 +1888,19 @@ int sc_verify_rows(const void *draft_logits, const void *target_logits, sc_dtype
   P.B = B;
   P.gamma = gamma;
   P.V = V;
-  P.rule = static_cast<int>(rule);
+  P.rule = ri;
   P.alpha = alpha;
   P.temperature = temperature;
-  set_k(P, temperature);
+  P.greedy = greedy ? 1 : 0;
+  set_k(P, greedy ? 1.0f : temperature);  // greedy: the rules' statistics at T = 1
+  if (ri == SC_RULE_LOSSY) {
+    // -log2(1 - alpha) as hi + lo, and -log2(beta)
+    const double l = alpha < 1.0f ? -std::log2(1.0 - static_cast<double>(alpha)) : HUGE_VAL;
+    P.lossy_l = static_cast<float>(l);
+    P.lossy_ll = std::isfinite(l) ? static_cast<float>(l - static_cast<double>(P.lossy_l)) : 0.0f;
+    P.lossy_c = static_cast<float>(-std::log2(static_cast<double>(beta)));
+    P.beta = beta;
+  }
   P.mode = kVerify;
   P.num_accepted = num_accepted;
   P.next_token = next_token;
@@ -1747,6 +1917,16 @@ int sc_verify_rows(const void *draft_logits, const void *target_logits, sc_dtype
   return dtype == SC_BF16 ? launch<uint16_t>(P, stream, units) : launch<float>(P, stream, units);
 }
 
+int sc_verify_rows(const void *draft_logits, const void *target_logits, sc_dtype dtype,
+                   const int32_t *draft_tokens, const float *uniforms, int B, int gamma, int V,
+                   sc_rule rule, float alpha, float temperature, int32_t *num_accepted,
+                   int32_t *next_token, void *workspace, size_t workspace_bytes,
+                   int32_t *device_status, float *row_info, cudaStream_t stream) {
+  return sc_verify_ex(draft_logits, target_logits, dtype, draft_tokens, uniforms, B, gamma, V, rule,
+                      alpha, 1.0f, temperature, num_accepted, next_token, workspace, workspace_bytes,
+                      device_status, row_info, stream);
+}
+
 int sc_verify(const void *draft_logits, const void *target_logits, sc_dtype dtype,
               const int32_t *draft_tokens, const float *uniforms, int B, int gamma, int V,
               sc_rule rule, float alpha, float temperature, int32_t *num_accepted,
@@ -1760,7 +1940,7 @@ int sc_verify(const void *draft_logits, const void *target_logits, sc_dtype dtyp
 int sc_row_stats(const void *draft_logits, const void *target_logits, sc_dtype dtype, int B,
                  int gamma, int V, float temperature, float *max_q, float *max_p, float *tv,
                  cudaStream_t stream) {
-  int rc = common_checks(draft_logits, target_logits, dtype, B, gamma, V, temperature);
+  int rc = common_checks(draft_logits, target_logits, dtype, B, gamma, V, temperature, false);
   if (rc != SC_OK) return rc;
   if (!device_accessible(max_q) || !device_accessible(max_p) || !device_accessible(tv))
     return SC_ERR_INVALID_ARG;
