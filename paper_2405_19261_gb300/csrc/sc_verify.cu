@@ -127,6 +127,8 @@ struct Params {
   uint32_t *seq_tickets;   // [B] finished sample passes (+1 for rank 0's last arrival); zero at rest
   float4 *records;         // [B][kMaxCluster][gamma+1] (R_q, R_p, c, flags) as seen by rank r
   float4 *records2;        // [B][kMaxCluster][gamma+1] (eta, thr, token, on_q) of token rules
+  float *bonus_pre;        // [B][kMaxCluster][kMaxChunks + 1] the same for the bonus row p_gamma,
+                           // written by the bonus unit from its pass-1 chunk totals
   float *chunk_pre;        // [B][kMaxCluster][kMaxChunks + 1] exclusive prefix of slice r of the
                            // sampled row at each chunk start, then the slice total
   int32_t *status;
@@ -660,6 +662,57 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
+// Pass 1 on a chunk of the bonus row p_gamma: online_row's running (max, sum)
+// and, per warp, the chunk's total weight sum_v 2^{y_v k - refk(W)}, W the
+// warp's largest logit of the chunk, in seg[c kNW + warp] (W in
+// seg[kBonusRef + c kNW + warp]).  After exchange 1 these give the chunk
+// prefixes of p_gamma's inverse CDF, so a sequence that accepts every draft
+// needs no second pass over its bonus row.
+constexpr int kBonusRef = kMaxChunks * kNW;
+static_assert(2 * kMaxChunks * kNW <= kEntries, "bonus chunk totals live in seg");
+
+template <typename E, bool kFull>
+__device__ __forceinline__ void bonus_row(const E *src, int n, float k, float &m, float2 &s, int c,
+                                          float *seg, int lane, int warp) {
+  float y[kRounds][8];
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r) {
+    const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
+    if constexpr (kFull) {
+      Elt<E>::load8(src + e, y[r]);
+    } else {
+      load8_smem(src, e, n, y[r]);
+    }
+  }
+  float W = -FLT_MAX;
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r)
+#pragma unroll
+    for (int i = 0; i < 8; i += 2) W = max3(W, y[r][i], y[r][i + 1]);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) W = fmaxf(W, __shfl_xor_sync(0xFFFFFFFFu, W, o));
+  const float rw = refk(W, k);
+  float c0 = 0.0f, c1 = 0.0f;
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r)
+#pragma unroll
+    for (int i = 0; i < 8; i += 2) {
+      c0 += ex2(fmaf(y[r][i], k, -rw));
+      c1 += ex2(fmaf(y[r][i + 1], k, -rw));
+    }
+  const float cs = c0 + c1;
+  // fold the chunk into the running sum, referenced to refk(max(m, W))
+  const float mn = fmaxf(m, W), rn = refk(mn, k);
+  const float so = ex2(refk(m, k) - rn);
+  s = make_float2(fmaf(cs, ex2(rw - rn), s.x * so), s.y * so);
+  m = mn;
+  const float tot = warp_sum(cs);
+  if (lane == 0) {
+    seg[c * kNW + warp] = tot;
+    seg[kBonusRef + c * kNW + warp] = W;
+  }
+}
+
 // Weights of one chunk in the ring: per round, the warp's total weight (the
 // segment total) lands in seg[(c, round, warp)].
 template <typename E, bool kPair, bool kFull, bool kTok>
@@ -1083,10 +1136,15 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   float mq = -FLT_MAX, mp = -FLT_MAX;
   float2 s2q = make_float2(0.0f, 0.0f), s2p = make_float2(0.0f, 0.0f);
   ExtState ex = ext_empty();  // (kFamExt) moments and argmaxes
+  // the bonus row also leaves its per-(chunk, warp) totals for the sampler
+  const bool bonus_tot = verify && !pair && !P.greedy;
   const int lx = x - v0;  // draft token's offset in this slice (thread 0 only)
   int tmo = stream(R, sh, ph, [&](int c, int s) {
     const int n = R.chunk_len(c);
-    if constexpr (kExt) {
+    if (bonus_tot) {
+      if (n == kCH) bonus_row<E, true>(R.p(s), n, k, mp, s2p, c, sh.seg, lane, warp);
+      else bonus_row<E, false>(R.p(s), n, k, mp, s2p, c, sh.seg, lane, warp);
+    } else if constexpr (kExt) {
       const int vc = v0 + c * kCH;
       if (pair) {
         if (n == kCH) ext_chunk<E, true, true>(R.q(s), R.p(s), n, vc, k, ex);
@@ -1108,6 +1166,10 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     }
   });
   if constexpr (kExt) {
+    if (bonus_tot) {
+      ex.mp = mp;
+      ex.sp = s2p.x + s2p.y;
+    }
     mq = ex.mq;
     mp = ex.mp;
     s2q = make_float2(ex.sq, 0.0f);
@@ -1210,6 +1272,20 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     sh.qx = 0.0f;
     sh.pix = 0.0f;
     sh.c = pair && !err ? log2f(as / cs) : 0.0f;
+    if (bonus_tot) {
+      // p_gamma's chunk prefixes over this slice from pass 1's per-(chunk, warp)
+      // totals, re-referenced to R_p: what a sampling pass over the row would store
+      float *cp = P.bonus_pre + (static_cast<size_t>(b) * kMaxCluster + rank) * (kMaxChunks + 1);
+      float acc = 0.0f;
+      for (int c2 = 0; c2 < R.nch; ++c2) {
+        cp[c2] = acc;
+        float t = 0.0f;
+        for (int w = 0; w < kNW; ++w)
+          t = fmaf(sh.seg[c2 * kNW + w], ex2(refk(sh.seg[kBonusRef + c2 * kNW + w], k) - Rp), t);
+        acc = __fadd_rn(acc, t);
+      }
+      cp[R.nch] = err || tmo ? NAN : acc;
+    }
     sh.dl = sh.maxq;
     sh.dr = sh.maxp;
     float xent = 0.0f;  // (kFamExt) BiLD*'s discrepancy D(q, p) = -sum_v q log p, in nats
@@ -1430,8 +1506,9 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     }
     __syncthreads();
 
-    if (sh.owner && kExt && P.greedy) {
-      // greedy decoding emits row j*'s argmax p (in the records): nothing to sample
+    if (sh.owner && ((kExt && P.greedy) || sh.jstar == P.gamma)) {
+      // nothing to sample: greedy decoding emits row j*'s argmax p (in the
+      // records), and the bonus row's chunk prefixes came from its pass 1
       if (tid == 0) sh.seq_last = atom_add_acq_rel(P.seq_tickets + b, 1u) == static_cast<uint32_t>(C);
       __syncthreads();
     } else if (sh.owner) {
@@ -1464,14 +1541,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       constexpr int kCP = kMaxChunks + 1;
       float *cpall = reinterpret_cast<float *>(smem_raw);  // [C][kCP]
       if (tid == 0) P.seq_tickets[b] = 0u;  // every report of the sequence is in
-      // one round of loads: every slice's chunk prefixes (ending in its total) ...
-      const float *cpg = P.chunk_pre + static_cast<size_t>(b) * kMaxCluster * kCP;
-      for (int i = tid; i < C * kCP && !(kExt && P.greedy); i += kNT) {
-        const int r = i / kCP, c = i % kCP;
-        const int len = max(0, min(P.L, P.V - r * P.L));
-        if (c <= (len + kCH - 1) / kCH) cpall[i] = __ldcg(cpg + i);
-      }
-      // ... and, in warp 0, j* and the error flags from rank 0's records
+      // warp 0: j* and the error flags from rank 0's records
       if (warp == 0) {
         const float4 *rec0 = P.records + static_cast<size_t>(b) * kMaxCluster * G1;
         int js = P.gamma, bad = 0;
@@ -1500,6 +1570,14 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       }
       __syncthreads();
       const int js = sh.jstar;
+      // one round of loads: every slice's chunk prefixes of row j* (ending in its total)
+      const float *cpg = (js == P.gamma ? P.bonus_pre : P.chunk_pre) + static_cast<size_t>(b) * kMaxCluster * kCP;
+      for (int i = tid; i < C * kCP && !(kExt && P.greedy); i += kNT) {
+        const int r = i / kCP, c = i % kCP;
+        const int len = max(0, min(P.L, P.V - r * P.L));
+        if (c <= (len + kCH - 1) / kCH) cpall[i] = __ldcg(cpg + i);
+      }
+      __syncthreads();
       if (kExt && P.greedy) {
         // greedy decoding: the argmax p of row j*, from rank 0's record
         if (tid == 0) {
@@ -1656,7 +1734,7 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 // sequence tickets (both zero between calls), then unit records and chunk
 // prefixes (written before they are read).
 struct WsLayout {
-  size_t rank_tickets, seq_tickets, zeroed, records, records2, chunk_pre, total;
+  size_t rank_tickets, seq_tickets, zeroed, records, records2, chunk_pre, bonus_pre, total;
 };
 
 constexpr size_t align256(size_t x) { return (x + 255) / 256 * 256; }
@@ -1669,7 +1747,8 @@ constexpr WsLayout ws_layout(size_t B, size_t units) {
   w.records = w.zeroed;
   w.records2 = w.records + align256(16 * kMaxCluster * units);
   w.chunk_pre = w.records2 + align256(16 * kMaxCluster * units);
-  w.total = w.chunk_pre + align256(4 * kMaxCluster * (kMaxChunks + 1) * B);
+  w.bonus_pre = w.chunk_pre + align256(4 * kMaxCluster * (kMaxChunks + 1) * B);
+  w.total = w.bonus_pre + align256(4 * kMaxCluster * (kMaxChunks + 1) * B);
   return w;
 }
 
@@ -1913,6 +1992,7 @@ int sc_verify_ex(const void *draft_logits, const void *target_logits, sc_dtype d
   P.records = reinterpret_cast<float4 *>(ws + wl.records);
   P.records2 = reinterpret_cast<float4 *>(ws + wl.records2);
   P.chunk_pre = reinterpret_cast<float *>(ws + wl.chunk_pre);
+  P.bonus_pre = reinterpret_cast<float *>(ws + wl.bonus_pre);
   const int units = B * (gamma + 1);
   return dtype == SC_BF16 ? launch<uint16_t>(P, stream, units) : launch<float>(P, stream, units);
 }
