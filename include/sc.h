@@ -186,7 +186,7 @@ const char *sc_status_string(int code);
  * exit.
  *
  * Limits: B <= SC_STATIC_MAX_B and B * (gamma + 1) <= SC_STATIC_MAX_UNITS
- * (about 6.5 MiB of scratch); larger batches return SC_ERR_SCRATCH_LIMIT and queue no
+ * (about 10.8 MiB of scratch); larger batches return SC_ERR_SCRATCH_LIMIT and queue no
  * work.  Other arguments are those of sc_verify and are checked the same way.
  *
  * The first call on a device looks up the array's device address (the library's

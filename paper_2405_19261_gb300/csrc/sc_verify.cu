@@ -127,6 +127,8 @@ struct Params {
   uint32_t *seq_tickets;   // [B] finished sample passes (+1 for rank 0's last arrival); zero at rest
   float4 *records;         // [B][kMaxCluster][gamma+1] (R_q, R_p, c, flags) as seen by rank r
   float4 *records2;        // [B][kMaxCluster][gamma+1] (eta, thr, token, on_q) of token rules
+  int spec_res;            // a rejected pair stores its residual's chunk prefixes itself (row_pre)
+  float *row_pre;          // [B][gamma+1][kMaxCluster][kMaxChunks + 1] those prefixes, per row
   float *bonus_pre;        // [B][kMaxCluster][kMaxChunks + 1] the same for the bonus row p_gamma,
                            // written by the bonus unit from its pass-1 chunk totals
   float *chunk_pre;        // [B][kMaxCluster][kMaxChunks + 1] exclusive prefix of slice r of the
@@ -1431,6 +1433,30 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     __syncthreads();
   }
 
+  // ---- small batches: a rejected pair stores its own residual's chunk prefixes
+  // now, while its slice is in the ring and in L2, so that no pass is left for
+  // the end of the sequence's chain (the row is j* unless an earlier one also
+  // rejects).  The OPT band's TV pass has summed exactly these weights already.
+  if (P.spec_res && verify && pair && !sh.accept && !sh.err && !(kExt && P.greedy)) {
+    if (!(sh.need_p2 && !sh.tok)) {
+      const bool lossy = kFam == kFamCascade && P.rule == SC_RULE_LOSSY;
+      const RowScalars rs = {sh.Rq, sh.Rp, k, lossy ? sh.c + P.lossy_c : sh.c,
+                             sh.tok ? kTokenRes : kResidual, sh.on_q, sh.thr, sh.eta};
+      tmo = slice_weights<kTok>(R, sh, ph, rs, sh.need_p2 ? kNewestFirst : kNewestFirstResident, lane, warp);
+      tmo = __syncthreads_or(tmo);
+      if (tid == 0) {
+        seg_prefix(sh, R.nch * kRounds * kNW);
+        if (tmo) flag_timeout(sh, P);
+      }
+    }
+    if (tid == 0) {
+      float *cp = P.row_pre + ((static_cast<size_t>(b) * G1 + j) * kMaxCluster + rank) * (kMaxChunks + 1);
+      for (int c = 0; c < R.nch; ++c) cp[c] = sh.seg[c * kRounds * kNW];
+      cp[R.nch] = sh.timeout ? NAN : sh.seg[R.nch * kRounds * kNW];
+    }
+    __syncthreads();
+  }
+
   if (!verify) {
     if (tid == 0 && rank == 0) {
       const size_t r = static_cast<size_t>(b) * P.gamma + j;
@@ -1506,9 +1532,10 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     }
     __syncthreads();
 
-    if (sh.owner && ((kExt && P.greedy) || sh.jstar == P.gamma)) {
+    if (sh.owner && ((kExt && P.greedy) || sh.jstar == P.gamma || P.spec_res)) {
       // nothing to sample: greedy decoding emits row j*'s argmax p (in the
-      // records), and the bonus row's chunk prefixes came from its pass 1
+      // records), the bonus row's chunk prefixes came from its pass 1, and
+      // with spec_res row j* stored its own
       if (tid == 0) sh.seq_last = atom_add_acq_rel(P.seq_tickets + b, 1u) == static_cast<uint32_t>(C);
       __syncthreads();
     } else if (sh.owner) {
@@ -1571,7 +1598,9 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       __syncthreads();
       const int js = sh.jstar;
       // one round of loads: every slice's chunk prefixes of row j* (ending in its total)
-      const float *cpg = (js == P.gamma ? P.bonus_pre : P.chunk_pre) + static_cast<size_t>(b) * kMaxCluster * kCP;
+      const float *cpg = js == P.gamma ? P.bonus_pre + static_cast<size_t>(b) * kMaxCluster * kCP
+                         : P.spec_res  ? P.row_pre + (static_cast<size_t>(b) * G1 + js) * kMaxCluster * kCP
+                                       : P.chunk_pre + static_cast<size_t>(b) * kMaxCluster * kCP;
       for (int i = tid; i < C * kCP && !(kExt && P.greedy); i += kNT) {
         const int r = i / kCP, c = i % kCP;
         const int len = max(0, min(P.L, P.V - r * P.L));
@@ -1734,7 +1763,7 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 // sequence tickets (both zero between calls), then unit records and chunk
 // prefixes (written before they are read).
 struct WsLayout {
-  size_t rank_tickets, seq_tickets, zeroed, records, records2, chunk_pre, bonus_pre, total;
+  size_t rank_tickets, seq_tickets, zeroed, records, records2, chunk_pre, bonus_pre, row_pre, total;
 };
 
 constexpr size_t align256(size_t x) { return (x + 255) / 256 * 256; }
@@ -1748,7 +1777,8 @@ constexpr WsLayout ws_layout(size_t B, size_t units) {
   w.records2 = w.records + align256(16 * kMaxCluster * units);
   w.chunk_pre = w.records2 + align256(16 * kMaxCluster * units);
   w.bonus_pre = w.chunk_pre + align256(4 * kMaxCluster * (kMaxChunks + 1) * B);
-  w.total = w.bonus_pre + align256(4 * kMaxCluster * (kMaxChunks + 1) * B);
+  w.row_pre = w.bonus_pre + align256(4 * kMaxCluster * (kMaxChunks + 1) * B);
+  w.total = w.row_pre + align256(4 * kMaxCluster * (kMaxChunks + 1) * units);
   return w;
 }
 
@@ -1845,6 +1875,12 @@ int launch(Params P, cudaStream_t stream, int units) {
   if (pick_layout(P.V, units, di.sms, &C, &L) != 0) return SC_ERR_UNSUPPORTED;
   P.L = L;
   P.cluster = C;
+  // Up to about two waves of CTAs the end of each sequence's chain is exposed:
+  // rejected pairs then store their residual's prefixes themselves.  Beyond,
+  // other units' streaming hides the owners' passes, and the extra passes of
+  // rejected rows after j* would only add bytes.
+  P.spec_res = static_cast<long>(units) * C <= 2L * kMinBlocksPerSM * di.sms;
+  if (const char *e = getenv("SC_SPEC_RES")) P.spec_res = atoi(e) != 0;
   const size_t row_bytes = static_cast<size_t>(P.V) * sizeof(E);
   P.bulk = (row_bytes % 16 == 0) && (reinterpret_cast<uintptr_t>(P.draft) % 16 == 0) &&
            (reinterpret_cast<uintptr_t>(P.target) % 16 == 0);
@@ -1993,6 +2029,7 @@ int sc_verify_ex(const void *draft_logits, const void *target_logits, sc_dtype d
   P.records2 = reinterpret_cast<float4 *>(ws + wl.records2);
   P.chunk_pre = reinterpret_cast<float *>(ws + wl.chunk_pre);
   P.bonus_pre = reinterpret_cast<float *>(ws + wl.bonus_pre);
+  P.row_pre = reinterpret_cast<float *>(ws + wl.row_pre);
   const int units = B * (gamma + 1);
   return dtype == SC_BF16 ? launch<uint16_t>(P, stream, units) : launch<float>(P, stream, units);
 }
