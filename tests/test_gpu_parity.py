@@ -212,6 +212,25 @@ def test_masked_target_logit_at_the_draft_token(sc, dtype, rule, alpha):
     assert_parity(w, run_gpu(sc, w), ref)
 
 
+@pytest.mark.parametrize("rule,alpha,T", [("opt", 0.3, 1.0), ("diff", 0.05, 0.7), ("token_v3", 0.3, 1.0),
+                                          ("chow", 0.5, 1.0)])
+def test_self_sampled_residuals_match_the_owners_pass(sc, monkeypatch, rule, alpha, T):
+    # a rejected pair storing its own residual prefixes (small batches) and the
+    # owner's sampling pass (large batches) sum the same weights with the same
+    # code: the draws are identical, and both match the oracle
+    w = synthetic(24, 6, 32128, dtype="bf16", kind="zipf", sigma=0.7, rule=rule, alpha=alpha,
+                  temperature=T, seed=61, force_reject_frac=0.5)
+    ref = oracle.verify_workload(w)
+    out = {}
+    for mode in ("0", "1"):
+        monkeypatch.setenv("SC_SPEC_RES", mode)
+        out[mode] = run_gpu(sc, w)
+        assert_parity(w, out[mode], ref)
+    np.testing.assert_array_equal(out["0"][0], out["1"][0])
+    np.testing.assert_array_equal(out["0"][1], out["1"][1])
+    assert np.any(ref.num_accepted < w.gamma) and np.any(ref.num_accepted == w.gamma)
+
+
 def test_invalid_inputs_flagged_on_device(sc):
     w = synthetic(5, 3, 300, dtype="f32", kind="gauss", sigma=1.0, rule="opt", alpha=0.2, seed=8)
     w.tokens[1, 2] = 300
