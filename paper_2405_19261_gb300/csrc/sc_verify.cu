@@ -275,6 +275,8 @@ struct __align__(16) Shared {
   float2 all_x[kMaxCluster];   // 1: raw logits at the draft token, if in the slice
   float all_r[kMaxCluster];    // 2 (TV pass): the slice's total residual weight
   float all_lb[kMaxCluster];   // OPT band: the slice's lower bound on D_TV
+  float2 all_scr[kMaxCluster]; // token rules: the slice's sum of q over its undeferred tokens, and
+                               // whether its screen is exact (1) or not (0)
   float4 all_ext[kMaxCluster]; // 1 (kFamExt): (A_q, A_p, X, -) of the slice, see ExtState
   int2 all_idx[kMaxCluster];   // 1 (kFamExt): the slice's argmax of q and of p
   int timeout;
@@ -577,6 +579,38 @@ __device__ __forceinline__ void ext_chunk(const E *srcq, const E *srcp, int n, i
   st.sp = __fadd_rn(st.sp, sp);
   st.ap = __fadd_rn(st.ap, ap);
   st.x = __fadd_rn(st.x, x);
+}
+
+// Pass-1 screen of a token rule: per thread, the two largest logits of the row
+// that r(v) tests (q for TokenV1, p otherwise) and the draft logit at the
+// largest.  When every thread's second largest turns out deferred (r = 1), the
+// tokens that are not deferred are exactly the threads' largest ones that pass
+// the test, so eta = 1 - (their q) needs no pass over the row.
+struct Top2 {
+  float y1, y2, z1;
+};
+
+template <typename E, bool kFull>
+__device__ __forceinline__ void screen_chunk(const E *ssrc, const E *qsrc, int n, Top2 &t) {
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r) {
+    const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
+    float y[8], z[8];
+    load8_chunk<E, kFull>(ssrc, e, n, y);
+    load8_chunk<E, kFull>(qsrc, e, n, z);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      if (y[i] > t.y2) {
+        if (y[i] > t.y1) {
+          t.y2 = t.y1;
+          t.y1 = y[i];
+          t.z1 = z[i];
+        } else {
+          t.y2 = y[i];
+        }
+      }
+    }
+  }
 }
 
 // Row scalars of the weight formulas.  With a_v = y^q_v k - R_q, b_v = y^p_v k - R_p
@@ -1138,6 +1172,8 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   float mq = -FLT_MAX, mp = -FLT_MAX;
   float2 s2q = make_float2(0.0f, 0.0f), s2p = make_float2(0.0f, 0.0f);
   ExtState ex = ext_empty();  // (kFamExt) moments and argmaxes
+  Top2 top = {-FLT_MAX, -FLT_MAX, -FLT_MAX};  // (kFamToken) the eta screen
+  const bool scr_q = P.rule == SC_RULE_TOKEN_V1;
   // the bonus row also leaves its per-(chunk, warp) totals for the sampler
   const bool bonus_tot = verify && !pair && !P.greedy;
   const int lx = x - v0;  // draft token's offset in this slice (thread 0 only)
@@ -1158,9 +1194,11 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     } else if (n == kCH) {
       if (pair) online_row<E, true>(R.q(s), n, k, mq, s2q);
       online_row<E, true>(R.p(s), n, k, mp, s2p);
+      if (kTok && pair) screen_chunk<E, true>(scr_q ? R.q(s) : R.p(s), R.q(s), n, top);
     } else {
       if (pair) online_row<E, false>(R.q(s), n, k, mq, s2q);
       online_row<E, false>(R.p(s), n, k, mp, s2p);
+      if (kTok && pair) screen_chunk<E, false>(scr_q ? R.q(s) : R.p(s), R.q(s), n, top);
     }
     if (tid == 0 && static_cast<unsigned>(lx - c * kCH) < static_cast<unsigned>(n)) {
       sh.xq = Elt<E>::at(R.q(s), lx - c * kCH);
@@ -1350,6 +1388,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
               sh.on_q = P.rule == SC_RULE_TOKEN_V1;
               sh.thr = m > 0.0f ? log2f(m * (sh.on_q ? as : cs)) : -INFINITY;
             }
+            if (sh.thr == -INFINITY) pending = false;  // r = 0 everywhere: eta = 0, pi = q
             break;
           }
           default: sh.delta = 0; break;
@@ -1364,6 +1403,43 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     sh.xp = ypx;
   }
   __syncthreads();
+
+  // ---- token rules: eta without a pass when the pass-1 screen settles it.  A
+  // thread whose second-largest screened logit is deferred holds at most one
+  // undeferred token, its largest; if that holds in every thread of the
+  // cluster, eta = (S_q - sum of 2^a over those tokens) / S_q.
+  if (kTok && sh.tok && sh.need_p2) {
+    const float Rs = sh.on_q ? sh.Rq : sh.Rp;  // r(v) tests a_v or b_v, formed as vec_weights forms them
+    const bool ok = !(fmaf(top.y2, k, -Rs) >= sh.thr);
+    const float h = fmaf(top.y1, k, -Rs) >= sh.thr ? ex2(fmaf(top.z1, k, -sh.Rq)) : 0.0f;
+    const bool wok = __all_sync(0xFFFFFFFFu, ok);
+    const float hs = warp_sum(h);
+    if (lane == 0) sh.red[warp] = make_float4(hs, wok ? 1.0f : 0.0f, 0.0f, 0.0f);
+    __syncthreads();
+    if (tid == 0) {
+      float acc = 0.0f, okc = 1.0f;
+      for (int w = 0; w < kNW; ++w) {
+        acc = __fadd_rn(acc, sh.red[w].x);
+        okc = fminf(okc, sh.red[w].y);
+      }
+      for (int r = 0; r < C; ++r) st_peer(peer_addr(&sh.all_scr[rank], r), make_float2(acc, okc));
+    }
+    cluster_arrive();
+    cluster_wait();
+    if (tid == 0) {
+      float H = 0.0f, okc = 1.0f;  // in rank order
+      for (int r = 0; r < C; ++r) {
+        H = __fadd_rn(H, sh.all_scr[r].x);
+        okc = fminf(okc, sh.all_scr[r].y);
+      }
+      if (okc > 0.0f) {
+        sh.need_p2 = 0;
+        sh.eta = fmaxf(0.0f, sh.Sq - H) / sh.Sq;  // eta = sum_v r(v) q(v) = 1 - sum over undeferred
+        accept_test<kFam>(sh, P, x, sh.xq, sh.xp, uj, k);
+      }
+    }
+    __syncthreads();
+  }
 
   // ---- OPT band: a lower bound on D_TV from the pass-1 partials.  The threads'
   // element sets partition the vocabulary, so sum_t max(0, P_t - Q_t) <= D_TV

@@ -231,6 +231,28 @@ def test_self_sampled_residuals_match_the_owners_pass(sc, monkeypatch, rule, alp
     assert np.any(ref.num_accepted < w.gamma) and np.any(ref.num_accepted == w.gamma)
 
 
+@pytest.mark.parametrize("rule,alpha", [("token_v3", 0.0), ("token_v3", 0.3), ("token_v2", 0.05), ("token_v1", 0.05)])
+def test_token_eta_screen_and_its_fallback(sc, rule, alpha):
+    # eta comes from the pass-1 screen when each thread holds at most one
+    # undeferred token, else from a pass over the row.  Sequences 0-1: many tied
+    # largest logits spread over the row (TokenV3 falls back; for TokenV1/V2
+    # max p < alpha, so nothing is deferred); 2-3: two tied largest logits in one
+    # thread's vector, q = p = 1/2 there (every rule falls back); the rest are
+    # ordinary rows (the screen)
+    B, g, V = 12, 4, 32128
+    w = synthetic(B, g, V, dtype="bf16", kind="zipf", sigma=0.7, rule=rule, alpha=alpha, seed=71)
+    top = np.uint16(0x4180)  # 16.0, above every sampled logit
+    for b in range(2):
+        w.draft[b, :, ::97] = top
+        w.target[b, :, ::89] = top
+    for b in (2, 3):
+        w.draft[b, :, 1000:1002] = top
+        w.target[b, :, 1000:1002] = top
+        w.tokens[b] = 1000 + b % 2
+    ref = oracle.verify_workload(w)
+    assert_parity(w, run_gpu(sc, w), ref)
+
+
 def test_invalid_inputs_flagged_on_device(sc):
     w = synthetic(5, 3, 300, dtype="f32", kind="gauss", sigma=1.0, rule="opt", alpha=0.2, seed=8)
     w.tokens[1, 2] = 300
