@@ -217,7 +217,7 @@ def _batched(w, X, K):
     target = np.broadcast_to(w.target[:1], (N,) + w.target.shape[1:]).copy()
     u = (K.astype(np.float64) / GRID).astype(np.float32)
     r = oracle.verify(draft, target, w.dtype, X.astype(np.int32), u, N, w.gamma, w.V, w.rule,
-                      w.alpha, w.temperature, nthreads=1)
+                      w.alpha, w.temperature, nthreads=1, beta=getattr(w, "beta", 1.0))
     return r
 
 
@@ -341,6 +341,74 @@ def test_enumeration_emitted_token_is_pi_distributed(V, gamma, rule, alpha, T, s
     # P(reach j + 1) = P(reach j) (1 - delta_j TV_j)
     for j in range(gamma):
         assert abs(reach[j + 1] - reach[j] * (1 - delta[j] * tv[j])) < tol
+
+
+def _entropy_delta(rule, alpha, q, p, tv):
+    """delta of BiLD* and the log-loss rules from scipy's entropies."""
+    from scipy.stats import entropy
+    Hq, Hp = entropy(q), entropy(p)
+    if rule == "bild":
+        return float(Hq + entropy(q, p) > alpha)   # D(q, p) = H(q) + KL(q || p)
+    if rule == "chow_log":
+        return float(Hq > alpha)
+    if rule == "diff_log":
+        return float(-Hq < -Hp - alpha)
+    return float(-Hq < -Hp - alpha * tv)             # opt_log
+
+
+TABLE3_ENUM_CASES = [
+    # (V, gamma, rule, alpha, beta, T, seed); alpha None: the median of the rule's statistic
+    (4, 2, "lossy", 0.3, 1.0, 1.0, 21),
+    (5, 2, "lossy", 0.5, 0.6, 1.0, 22),
+    (3, 3, "lossy", 0.2, 0.9, 0.7, 23),
+    (4, 3, "bild", None, 1.0, 1.0, 24),
+    (5, 2, "chow_log", None, 1.0, 1.0, 25),
+    (4, 3, "diff_log", None, 1.0, 0.8, 26),
+    (6, 2, "opt_log", 0.5, 1.0, 1.0, 27),    # position 0: the alpha D_TV term decides (DiffLog would not defer)
+]
+
+
+@pytest.mark.parametrize("V,gamma,rule,alpha,beta,T,seed", TABLE3_ENUM_CASES)
+def test_enumeration_table3_and_log_loss_targets(V, gamma, rule, alpha, beta, T, seed):
+    """Algorithm 4 with any target pi: a draft x is kept with probability
+    min(1, pi(x)/q(x)) and otherwise replaced from norm(max(0, pi - q)), so the
+    token emitted at a reached position has law
+        min(q, pi) + (sum max(0, q - pi) / sum max(0, pi - q)) max(0, pi - q),
+    which is pi itself when pi sums to one, and the rejection probability is
+    sum max(0, q - pi).  pi is built here from its definition: the lossy target
+    of Table 3, or (1 - delta) q + delta p with delta from scipy's entropies."""
+    rng = np.random.default_rng(seed)
+    q_log = (rng.standard_normal((gamma, V)) * 1.5).astype(np.float32)
+    p_log = (q_log[np.r_[0:gamma, gamma - 1]] + rng.standard_normal((gamma + 1, V)) * 1.2).astype(np.float32)
+    qs = np_softmax(q_log.astype(np.float64), 1.0)
+    ps = np_softmax(p_log.astype(np.float64), 1.0)
+    tv = 0.5 * np.abs(ps[:gamma] - qs).sum(1)
+    if alpha is None:   # a threshold between the rows' statistics, so that delta takes both values
+        from scipy.stats import entropy
+        Hq = np.array([entropy(qs[j]) for j in range(gamma)])
+        Hp = np.array([entropy(ps[j]) for j in range(gamma)])
+        stat = {"bild": Hq + np.array([entropy(qs[j], ps[j]) for j in range(gamma)]),
+                "chow_log": Hq, "diff_log": Hq - Hp, "opt_log": (Hq - Hp) / np.maximum(tv, 1e-3)}[rule]
+        alpha = float(max(0.0, np.median(stat)))
+    w = rows_workload(np.exp(q_log), np.exp(p_log), np.zeros(gamma), np.zeros(gamma + 1), rule,
+                      alpha, temperature=T)
+    w.beta = beta
+    q = np_softmax(logits_as_f64(w.draft[0], "f32"), T)
+    p = np_softmax(logits_as_f64(w.target[0], "f32"), T)
+    reach, laws, reject = exact_output_law(w)
+    tol = 4.0 * V / GRID + 1e-9
+    for j in range(gamma):
+        if rule == "lossy":
+            pi = np.maximum(np.minimum(q[j], p[j] / (1.0 - alpha)), p[j] / beta)
+        else:
+            d = _entropy_delta(rule, alpha, q[j], p[j], 0.5 * np.abs(p[j] - q[j]).sum())
+            pi = (1 - d) * q[j] + d * p[j]
+        out, res = np.maximum(0.0, q[j] - pi), np.maximum(0.0, pi - q[j])
+        law = np.minimum(q[j], pi) + (out.sum() / res.sum() if res.sum() > 0 else 0.0) * res
+        np.testing.assert_allclose(laws[j], law, atol=tol, err_msg=f"{rule} position {j}")
+        assert abs(reject[j] - out.sum()) < tol, (j, reject[j], out.sum())
+        assert abs(reach[j + 1] - reach[j] * (1 - out.sum())) < tol
+    np.testing.assert_allclose(laws[gamma], p[gamma], atol=tol, err_msg="bonus position")
 
 
 def test_enumeration_agrees_with_fine_grid_bruteforce():
