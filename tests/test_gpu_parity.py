@@ -273,9 +273,11 @@ def test_host_argument_errors(sc):
     with pytest.raises(sc.SCError):
         sc.sc_verify(d, t, x, u, "opt", 1.5, 1.0)       # alpha outside [0, 1]
     with pytest.raises(sc.SCError):
-        sc.sc_verify(d, t, x, u, "opt", 0.2, 0.0)       # T = 0
+        sc.sc_verify(d, t, x, u, "opt", 0.2, -1.0)      # T < 0 (T = 0 is greedy decoding)
     with pytest.raises(sc.SCError):
-        sc.sc_verify(d, t, x, u, 9, 0.2, 1.0)           # unknown rule
+        sc.sc_verify(d, t, x, u, "token_v3", 0.2, 0.0)  # greedy decoding with a token rule
+    with pytest.raises(sc.SCError):
+        sc.sc_verify(d, t, x, u, 13, 0.2, 1.0)          # unknown rule
     with pytest.raises(sc.SCError):
         sc.sc_verify(d, t, x, u, "opt", 0.2, 1.0, workspace=torch.zeros(4, dtype=torch.uint8, device="cuda"))
     with pytest.raises(TypeError):
