@@ -443,6 +443,20 @@ def test_token_worked_examples():
             assert (r.num_accepted[0], r.next_token[0]) == (c["num_accepted"], c["next_token"]), (ex["name"], c)
 
 
+def test_table3_and_log_loss_worked_examples():
+    """Hand-worked runs of Algorithm 4 with the lossy target (Table 3, Lemma 2),
+    BiLD*, the log-loss rules and greedy decoding on a 3-token vocabulary."""
+    g = load_golden("table3_logloss_examples.json")
+    for ex in g["examples"]:
+        for c in ex["cases"]:
+            # logits are the log-probabilities at T = 1; T = 0 reads the same logits greedily
+            w = rows_workload(ex["q"], ex["p"], c["tokens"], c["u"], c["rule"], c["alpha"])
+            w.temperature = c["T"]
+            r = oracle.verify_workload(w, beta=c.get("beta", 1.0))
+            assert not r.flagged[0], (ex["name"], c)
+            assert (r.num_accepted[0], r.next_token[0]) == (c["num_accepted"], c["next_token"]), (ex["name"], c)
+
+
 def _token_pi(rule, alpha, q, p):
     """pi_Token(v) = q(v)(1 - r(v)) + eta p(v), eta = sum_v r(v) q(v), for one row
     (Section 4.4; r by the TokenV1 / TokenV2 / TokenV3 plug-in rules)."""
