@@ -15,6 +15,7 @@ import numpy as np
 import pytest
 
 import oracle
+from helpers import load_golden, rows_workload
 from paper_2405_19261_gb300.workloads import config, logits_as_f64, synthetic
 
 pytestmark = pytest.mark.gpu
@@ -83,6 +84,26 @@ def _sampled(sc, w, nseq, beta=1.0, seed=0):
     ref = oracle.verify_workload(sub, beta=beta)
     na, nt, ri, status = gpu
     assert_parity(sub, (na[pick], nt[pick], ri[pick], status), ref)
+
+
+# ----------------------------------------------------------------- hand-worked goldens
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_worked_examples(sc, dtype):
+    g = load_golden("table3_logloss_examples.json")
+    for ex in g["examples"]:
+        for c in ex["cases"]:
+            w = rows_workload(ex["q"], ex["p"], c["tokens"], c["u"], c["rule"], c["alpha"], dtype=dtype, B=3)
+            w.temperature = c["T"]
+            beta = c.get("beta", 1.0)
+            ref = oracle.verify_workload(w, beta=beta)
+            na, nt, ri, status = run_gpu(sc, w, beta=beta)
+            assert status == 0
+            if dtype == "f32":   # bf16 rounding of the log-probabilities moves no decision here either
+                assert (na[0], nt[0]) == (c["num_accepted"], c["next_token"]), (ex["name"], c)
+            ok = ~ref.flagged
+            np.testing.assert_array_equal(na[ok], ref.num_accepted[ok])
+            np.testing.assert_array_equal(nt[ok], ref.next_token[ok])
 
 
 # ----------------------------------------------------------------- lossy speculative decoding
