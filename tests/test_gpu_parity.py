@@ -282,6 +282,15 @@ def test_host_argument_errors(sc):
         sc.sc_verify(d, t, x, u, "opt", 0.2, 1.0, workspace=torch.zeros(4, dtype=torch.uint8, device="cuda"))
     with pytest.raises(TypeError):
         sc.sc_verify(d.cpu(), t, x, u, "opt", 0.2, 1.0)
+    # empty batches, drafts and vocabularies are refused before anything is queued
+    for shape in ((0, 2, 64), (2, 0, 64), (2, 2, 0)):
+        B0, g0, V0 = shape
+        d0 = torch.zeros((B0, g0, V0), dtype=torch.float32, device="cuda")
+        t0 = torch.zeros((B0, g0 + 1, V0), dtype=torch.float32, device="cuda")
+        x0 = torch.zeros((B0, g0), dtype=torch.int32, device="cuda")
+        u0 = torch.zeros((B0, g0 + 1), dtype=torch.float32, device="cuda")
+        with pytest.raises(sc.SCError):
+            sc.sc_verify(d0, t0, x0, u0, "opt", 0.2, 1.0, workspace=torch.zeros(1 << 16, dtype=torch.uint8, device="cuda"))
     with pytest.raises(ValueError):
         sc.sc_verify(d, t[:, :2], x, u, "opt", 0.2, 1.0)
 
