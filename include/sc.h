@@ -85,6 +85,11 @@ typedef enum {
 
 #define SC_MAX_GAMMA 255
 
+/* Layout overrides, read from the environment at every call and meant for
+ * measurements (the default layout is chosen from V, the batch and the SM count):
+ *   SC_SLICE=n    logits per CTA slice of a row (n >= 64, rounded to a multiple of 8)
+ *   SC_CLUSTER=c  CTAs per row pair (1 <= c <= 16; raised if the slices would not fit) */
+
 /* Per-position diagnostics written by sc_verify_rows, [B][gamma+1][SC_ROW_FIELDS]
  * float32.  Position gamma (the bonus position) fills only MAXP and CAND. */
 #define SC_ROW_MAXQ 0   /* max_v q_j(v) */
