@@ -69,6 +69,9 @@ namespace {
 #ifndef SC_MIN_BLOCKS
 #define SC_MIN_BLOCKS 6
 #endif
+#ifndef SC_L2_PREFETCH
+#define SC_L2_PREFETCH 1  // second passes prefetch their slice into L2 before streaming it
+#endif
 
 constexpr int kNT = 128;                   // threads per CTA
 constexpr int kNW = kNT / 32;              // warps per CTA
@@ -187,6 +190,11 @@ __device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t by
           "r"(smem_u32(dst)),
       "l"(src), "r"(bytes), "r"(smem_u32(bar))
       : "memory");
+}
+
+// Hint: bring [src, src + bytes) into L2 (16-byte aligned, a multiple of 16 bytes).
+__device__ __forceinline__ void prefetch_l2(const void *src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
 }
 
 __device__ __forceinline__ void cluster_arrive_relaxed() {
@@ -906,6 +914,12 @@ struct Ring {
     if (pair) bulk_g2s(q(s), gq + static_cast<size_t>(c) * kCH, bytes, &sh.full[s]);
     bulk_g2s(p(s), gp + static_cast<size_t>(c) * kCH, bytes, &sh.full[s]);
   }
+  // thread 0, bulk mode: hint chunk c into L2
+  __device__ void prefetch(int c) const {
+    const uint32_t bytes = static_cast<uint32_t>(chunk_len(c)) * sizeof(E);
+    if (pair) prefetch_l2(gq + static_cast<size_t>(c) * kCH, bytes);
+    prefetch_l2(gp + static_cast<size_t>(c) * kCH, bytes);
+  }
   // all threads, per-thread mode: copy chunk c into stage s
   __device__ void load_sync(int c, int s) const {
     const int n = chunk_len(c);
@@ -981,6 +995,10 @@ __device__ __forceinline__ int stream_rev(const Ring<E> &R, Shared &sh, uint32_t
   const int nres = resident ? min(kStages, nch) : 0;
   if (!resident && R.bulk && threadIdx.x == 0)
     for (int c = nch - 1; c >= max(0, nch - kStages); --c) R.issue(sh, c, c % kStages);
+  // a second pass finds its older chunks mostly gone from L2 and streams them with
+  // only the ring in flight: ask for all of them at once, in the order they are used
+  if (SC_L2_PREFETCH && R.bulk && threadIdx.x == 0)
+    for (int c = nch - 1 - kStages; c >= 0; --c) R.prefetch(c);
   int tmo = 0;
   for (int i = 0; i < nch; ++i) {
     const int c = nch - 1 - i, s = c % kStages;
