@@ -181,6 +181,23 @@ def test_gemma_shape_sampled(sc, rule, alpha, beta):
     _sampled(sc, config(4, B=64, gamma=4, rule=rule, alpha=alpha), nseq=6, beta=beta)
 
 
+@pytest.mark.parametrize("rule,alpha,beta", [("lossy", 0.3, 0.8), ("bild", 6.5, 1.0), ("opt_log", 0.5, 1.0),
+                                             ("diff_log", 0.1, 1.0)])
+def test_self_sampled_residuals_match_the_owners_pass(sc, monkeypatch, rule, alpha, beta):
+    # the lossy residual's shifted constant and the moment kernel's rows (OPTLog
+    # band rows reuse their TV pass) through both sampling paths: same draws
+    w = synthetic(24, 6, 32128, dtype="bf16", kind="zipf", sigma=0.7, rule=rule, alpha=alpha, seed=62,
+                  force_reject_frac=0.5)
+    ref = oracle.verify_workload(w, beta=beta)
+    out = {}
+    for mode in ("0", "1"):
+        monkeypatch.setenv("SC_SPEC_RES", mode)
+        out[mode] = run_gpu(sc, w, beta=beta)
+        assert_parity(w, out[mode], ref)
+    np.testing.assert_array_equal(out["0"][0], out["1"][0])
+    np.testing.assert_array_equal(out["0"][1], out["1"][1])
+
+
 # ----------------------------------------------------------------- greedy decoding (T = 0)
 
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
