@@ -89,8 +89,8 @@ typedef enum {
  * measurements (the default layout is chosen from V, the batch and the SM count):
  *   SC_SLICE=n    logits per CTA slice of a row (n >= 64, rounded to a multiple of 8)
  *   SC_CLUSTER=c  CTAs per row pair (1 <= c <= 16; raised if the slices would not fit)
- *   SC_SPEC_RES=0|1  whether rejected pairs store their own residual prefixes (default:
- *                 up to about two waves of CTAs) or leave them to the owners' sampling passes */
+ *   SC_SPEC_RES=0|1  whether rejected pairs store their own residual prefixes (default 1)
+ *                 or leave them to the owners' sampling passes */
 
 /* Per-position diagnostics written by sc_verify_rows, [B][gamma+1][SC_ROW_FIELDS]
  * float32.  Position gamma (the bonus position) fills only MAXP and CAND. */

@@ -302,6 +302,7 @@ struct __align__(16) Shared {
   int iq, ip;               // (kFamExt) argmax q and argmax p, lowest index on ties
   float thr, eta;           // its r(v) threshold (exponent domain) and eta = sum_v r(v) q(v)
   // sequence finish
+  int spec_skip;            // a rejection of an earlier position is already reported: not row j*
   int owner;                // this CTA runs its rank's sample pass of row j*
   int scan_records;         // j* must be read from the records (gamma + 1 > 32)
   int seq_last;             // the sequence's last finisher: draws the token
@@ -1326,6 +1327,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     sh.thr = -INFINITY;
     sh.eta = 0.0f;
     sh.accept = 0;
+    sh.spec_skip = 0;
     sh.tv = -1.0f;
     sh.qx = 0.0f;
     sh.pix = 0.0f;
@@ -1531,7 +1533,17 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   // now, while its slice is in the ring and in L2, so that no pass is left for
   // the end of the sequence's chain (the row is j* unless an earlier one also
   // rejects).  The OPT band's TV pass has summed exactly these weights already.
-  if (P.spec_res && verify && pair && !sh.accept && !sh.err && !(kExt && P.greedy)) {
+  // A rejected pair whose rank already shows a rejection at an earlier position
+  // is not row j* and skips the pass (a stale read of the ticket only costs the
+  // pass; row j* itself never sees an earlier rejection).
+  if (P.spec_res && verify && pair && !sh.accept && !sh.err && !(kExt && P.greedy) && j > 0 && G1 <= 32) {
+    if (tid == 0) {
+      const unsigned long long t = __ldcg(P.rank_tickets + static_cast<size_t>(b) * kMaxCluster + rank);
+      sh.spec_skip = ((t >> 32) & ((1ull << j) - 1ull)) != 0ull;
+    }
+    __syncthreads();
+  }
+  if (P.spec_res && verify && pair && !sh.accept && !sh.err && !(kExt && P.greedy) && !sh.spec_skip) {
     if (!(sh.need_p2 && !sh.tok)) {
       const bool lossy = kFam == kFamCascade && P.rule == SC_RULE_LOSSY;
       const RowScalars rs = {sh.Rq, sh.Rp, k, lossy ? sh.c + P.lossy_c : sh.c,
@@ -1969,11 +1981,10 @@ int launch(Params P, cudaStream_t stream, int units) {
   if (pick_layout(P.V, units, di.sms, &C, &L) != 0) return SC_ERR_UNSUPPORTED;
   P.L = L;
   P.cluster = C;
-  // Up to about two waves of CTAs the end of each sequence's chain is exposed:
-  // rejected pairs then store their residual's prefixes themselves.  Beyond,
-  // other units' streaming hides the owners' passes, and the extra passes of
-  // rejected rows after j* would only add bytes.
-  P.spec_res = static_cast<long>(units) * C <= 2L * kMinBlocksPerSM * di.sms;
+  // Rejected pairs store their residual's prefixes themselves, right after their
+  // decision and from their ring and L2, unless their rank already shows an
+  // earlier rejection; the owners then never stream a second pass.
+  P.spec_res = 1;
   if (const char *e = getenv("SC_SPEC_RES")) P.spec_res = atoi(e) != 0;
   const size_t row_bytes = static_cast<size_t>(P.V) * sizeof(E);
   P.bulk = (row_bytes % 16 == 0) && (reinterpret_cast<uintptr_t>(P.draft) % 16 == 0) &&
