@@ -406,6 +406,7 @@ def run_ours(args):
                 "config": {"workload": desc, "B": B, "gamma": g, "V": w.V, "logits": w.dtype,
                            "rule": w.rule, "alpha": w.alpha, "temperature": w.temperature,
                            "rows_per_s": w.rows * world / (ms_step / 1e3),
+                           "sequences_per_s": B * world / (ms_step / 1e3),
                            "mean_accepted": mean_accepted,
                            "acceptance_rate": mean_accepted / g,
                            "l2": ("L2 flushed before every timed step (2x L2 write, then 2x L2 read of another buffer); "

@@ -111,6 +111,52 @@ def test_inverse_cdf_brackets_u_times_total():
 
 # ----------------------------------------------------------------- worked examples
 
+def test_residual_draw_frequencies_chi_square():
+    """At a certain rejection (Algorithm 4, delta = 1), the replacement token of a
+    V = 4096 row pair is norm(max(0, p - q))-distributed: 40,000 seeded draws
+    of u_gamma against 32 contiguous bins of equal residual mass (chi-square),
+    with max(0, p - q) from numpy's fp64 softmax of the stored logits."""
+    from scipy.stats import chi2
+    V, N, chunk, nbins = 4096, 40000, 4000, 32
+    rng = np.random.default_rng(7)
+    q_log = (rng.standard_normal(V) * 2.0).astype(np.float32)
+    p_log = (q_log + rng.standard_normal(V) * 1.0).astype(np.float32)
+    draft = f32_to_bf16_bits(q_log[None, None, :])
+    target = f32_to_bf16_bits(np.stack([p_log, p_log])[None])
+    q = np_softmax(logits_as_f64(draft[0, 0], "bf16"), 1.0)
+    p = np_softmax(logits_as_f64(target[0, 0], "bf16"), 1.0)
+    x = int(np.argmin(p / q))                    # p(x)/q(x) far below 0.99: rejected for sure
+    assert p[x] / q[x] < 0.5
+    r = np.maximum(0.0, p - q)
+    r /= r.sum()
+    # contiguous bins in vocabulary order, each closed once it holds 1/nbins of the mass
+    bounds, acc = [], 0.0
+    for t in range(V):
+        acc += r[t]
+        if acc >= 1.0 / nbins:
+            bounds.append(t)
+            acc = 0.0
+    bounds[-1] = V - 1
+    bounds = np.array(bounds)
+    nbins = len(bounds)
+    cs = np.cumsum(r)
+    expected = np.diff(np.concatenate([[0.0], cs[bounds]])) * N
+    assert expected.min() > 50
+    ks = rng.integers(0, 1 << 24, size=N)
+    counts = np.zeros(len(bounds))
+    for lo in range(0, N, chunk):
+        n = min(chunk, N - lo)
+        u = np.stack([np.full(n, 0.99, np.float32), (ks[lo:lo + n] / float(1 << 24)).astype(np.float32)], 1)
+        res = oracle.verify(np.repeat(draft, n, 0), np.repeat(target, n, 0), "bf16", np.full((n, 1), x, np.int32),
+                            u, n, 1, V, "always", 0.0, 1.0)
+        assert np.all(res.num_accepted == 0)
+        tok = res.next_token
+        assert np.all(r[tok] > 0.0)
+        counts += np.bincount(np.searchsorted(bounds, tok, side="left"), minlength=nbins)
+    stat = float(np.sum((counts - expected) ** 2 / expected))
+    assert chi2.sf(stat, nbins - 1) > 1e-3, (stat, counts, expected)
+
+
 def test_worked_examples_golden():
     g = load_golden("worked_examples.json")
     for ex in g["examples"]:
