@@ -39,7 +39,7 @@ def test_softmax_extreme_logits():
     # +-large logits must neither overflow nor lose the head; -inf means probability 0.
     z = np.array([1e4, -1e4, 9990.0, -np.inf, 0.0], np.float32)
     got = oracle.softmax(z, "f32", 1.0)
-    want = np_softmax(np.where(np.isinf(z), -1e300, z), 1.0)
+    want = np_softmax(np.where(np.isinf(z), -1e300, z.astype(np.float64)), 1.0)
     np.testing.assert_allclose(got, want, rtol=1e-12, atol=1e-300)
     assert got[3] == 0.0
     for bad in (np.nan, np.inf):
