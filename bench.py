@@ -61,6 +61,8 @@ def parse():
     ap.add_argument("--temperature", type=float, default=None, help="config 4 only; 0 = greedy decoding")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--record-traffic", metavar="NCU_CSV", default=None,
+                    help="store the DRAM bytes of an ncu capture of this workload for the current kernel source")
     ap.add_argument("--min-warmup-s", type=float, default=0.5,
                     help="keep warming up (untimed) until this long has passed, for clock samples")
     return ap.parse_args()
@@ -92,6 +94,41 @@ def measured_peaks():
             d = json.load(f)
         return float(d["hbm_gbs"]), "measured"
     return 6800.0, "fallback"
+
+
+_NCU_UNITS = {"byte": 1, "Kbyte": 1e3, "Mbyte": 1e6, "Gbyte": 1e9, "Tbyte": 1e12}
+
+
+def record_traffic(csv_path, workload_name, command=""):
+    """Store, for the current kernel source, the DRAM bytes ncu measured for one
+    sc_unit_kernel launch (the first one in an `ncu --metrics
+    dram__bytes_read.sum,dram__bytes_write.sum --csv --log-file` capture)."""
+    import csv
+    with open(csv_path, encoding="utf-8") as f:
+        rows = list(csv.DictReader(ln for ln in f if ln.startswith('"')))
+    launches = {}
+    for r in rows:
+        if "sc_unit_kernel" in r.get("Kernel Name", ""):
+            unit = _NCU_UNITS[r["Metric Unit"]] if r["Metric Unit"] in _NCU_UNITS else None
+            if unit is not None:
+                launches.setdefault(r["ID"], {})[r["Metric Name"]] = float(r["Metric Value"].replace(",", "")) * unit
+    done = [m for m in launches.values() if "dram__bytes_read.sum" in m and "dram__bytes_write.sum" in m]
+    if not done:
+        raise SystemExit(f"{csv_path}: no sc_unit_kernel launch with both DRAM byte counts")
+    m = done[0]
+    d = {}
+    if os.path.exists(TRAFFIC_FILE):
+        with open(TRAFFIC_FILE) as f:
+            d = json.load(f)
+    d[workload_name] = {"kernel_sha": kernel_sha(),
+                        "dram_bytes_per_launch": int(m["dram__bytes_read.sum"] + m["dram__bytes_write.sum"]),
+                        "dram_bytes_read": int(m["dram__bytes_read.sum"]),
+                        "dram_bytes_write": int(m["dram__bytes_write.sum"]),
+                        "source": command}
+    with open(TRAFFIC_FILE, "w") as f:
+        json.dump(d, f, indent=2)
+        f.write("\n")
+    return d[workload_name]
 
 
 def stored_traffic(workload_name):
@@ -423,6 +460,10 @@ def run_ours(args):
 
 def main():
     args = parse()
+    if args.record_traffic:
+        _, desc = workload_from(args)
+        print(json.dumps(record_traffic(args.record_traffic, desc, " ".join(sys.argv))))
+        return
     if args.impl == "reference":
         run_reference(args)
     else:

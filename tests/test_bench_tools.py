@@ -1,0 +1,42 @@
+"""Host-side tools of bench.py (no GPU): recording ncu's DRAM traffic for the
+current kernel source and finding it again."""
+import json
+import os
+import sys
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+HEADER = ('"ID","Process ID","Process Name","Host Name","Kernel Name","Context","Stream","Block Size",'
+          '"Grid Size","Device","CC","Section Name","Metric Name","Metric Unit","Metric Value"')
+
+
+def _row(i, kernel, metric, unit, value):
+    return (f'"{i}","1","python3","h","{kernel}","1","7","(128, 1, 1)","(4096, 1, 1)","0","10.3",'
+            f'"Command line profiler metrics","{metric}","{unit}","{value}"')
+
+
+def test_record_traffic_from_an_ncu_csv(tmp_path, monkeypatch):
+    import bench
+    k = "void <unnamed>::sc_unit_kernel<unsigned short, false>(<unnamed>::Params)"
+    lines = ["==PROF== Connected to process 1", HEADER,
+             _row(0, "void at::native::FillFunctor<unsigned char>", "dram__bytes_read.sum", "byte", "7"),
+             _row(1, k, "dram__bytes_read.sum", "Mbyte", "1,079.37"),
+             _row(1, k, "dram__bytes_write.sum", "Kbyte", "3,649.28"),
+             _row(1, k, "gpu__time_duration.sum", "usecond", "195.5"),
+             _row(2, k, "dram__bytes_read.sum", "byte", "5")]
+    csv_path = tmp_path / "traffic.csv"
+    csv_path.write_text("\n".join(lines) + "\n")
+    monkeypatch.setattr(bench, "TRAFFIC_FILE", str(tmp_path / "traffic.json"))
+    e = bench.record_traffic(str(csv_path), "cfgX: a workload", "ncu ... python bench.py")
+    assert e["dram_bytes_read"] == 1_079_370_000 and e["dram_bytes_write"] == 3_649_280
+    assert e["dram_bytes_per_launch"] == 1_079_370_000 + 3_649_280
+    assert e["kernel_sha"] == bench.kernel_sha()
+    assert bench.stored_traffic("cfgX: a workload") == e["dram_bytes_per_launch"]
+    assert bench.stored_traffic("another workload") is None
+    # an entry recorded for other kernel code is not used
+    d = json.loads((tmp_path / "traffic.json").read_text())
+    d["cfgX: a workload"]["kernel_sha"] = "0" * 16
+    (tmp_path / "traffic.json").write_text(json.dumps(d))
+    assert bench.stored_traffic("cfgX: a workload") is None
