@@ -56,3 +56,32 @@ def test_null_pointers_are_rejected_without_a_gpu(so):
     assert rc == -1
     rc = so.sc_verify(None, None, 1, None, None, 0, 1, 8, 0, 0.5, 1.0, None, None, None, 0, None, None)
     assert rc == -1
+
+
+def test_header_is_plain_c(tmp_path):
+    """include/sc.h is a C header: a C11 translation unit that calls every entry
+    point compiles with warnings as errors."""
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    cuda_inc = next((d for d in ("/usr/local/cuda/include",) if os.path.isdir(d)), None)
+    if not gcc or not cuda_inc:
+        pytest.skip("gcc or the CUDA headers are missing")
+    src = tmp_path / "use_sc.c"
+    src.write_text("""
+#include "sc.h"
+int use_sc(const void *q, const void *p, const int32_t *x, const float *u, int32_t *na, int32_t *nt,
+           float *mq, float *mp, float *tv, float *rows, int32_t *st, cudaStream_t s) {
+  size_t n = sc_workspace_bytes(2, 3, 100);
+  void *ws = 0;
+  int rc = sc_workspace_init(ws, n, s);
+  rc |= sc_verify(q, p, SC_BF16, x, u, 2, 3, 100, SC_RULE_OPT, 0.2f, 1.0f, na, nt, ws, n, st, s);
+  rc |= sc_verify_rows(q, p, SC_F32, x, u, 2, 3, 100, SC_RULE_TOKEN_V3, 0.3f, 0.7f, na, nt, ws, n, st, rows, s);
+  rc |= sc_row_stats(q, p, SC_BF16, 2, 3, 100, 1.0f, mq, mp, tv, s);
+  rc |= sc_verify_static(q, p, SC_BF16, x, u, 2, 3, 100, SC_RULE_DIFF, 0.1f, 1.0f, na, nt, st, s);
+  return rc + sc_max_vocab(SC_BF16) + (sc_status_string(rc) != 0);
+}
+""")
+    r = subprocess.run([gcc, "-std=c11", "-Wall", "-Wextra", "-Werror", "-fsyntax-only", "-I",
+                        os.path.join(ROOT, "include"), "-I", cuda_inc, str(src)], capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
