@@ -69,6 +69,9 @@ namespace {
 #ifndef SC_MIN_BLOCKS
 #define SC_MIN_BLOCKS 6
 #endif
+#ifndef SC_BONUS_LAST
+#define SC_BONUS_LAST 0  // 1: launch all pair units before the bonus rows
+#endif
 #ifndef SC_L2_PREFETCH
 #define SC_L2_PREFETCH 1  // second passes prefetch their slice into L2 before streaming it
 #endif
@@ -1151,7 +1154,13 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   const bool verify = P.mode == kVerify;
 
   int b, j;
-  if (verify) {
+  if (verify && SC_BONUS_LAST) {
+    // every pair unit first, then the bonus rows: the last, partial wave of CTAs
+    // holds the shorter (target-only) units
+    const int pairs = P.B * P.gamma;
+    b = unit < pairs ? unit / P.gamma : unit - pairs;
+    j = unit < pairs ? unit % P.gamma : P.gamma;
+  } else if (verify) {
     b = unit / G1;
     j = unit % G1;
   } else {
