@@ -35,7 +35,8 @@
  *          (Lemma 2: the acceptance is min(1, p(x)/((1 - alpha) q(x))) and the residual
  *          norm(max(0, p/beta - q)); pi need not sum to one), beta >= 1 - alpha;
  *       BiLD*:  delta = 1(D(q, p) > alpha), D(q, p) = -sum_v q(v) log p(v) (the
- *          temperature-sampling discrepancy of the experiments' appendix),
+ *          temperature-sampling discrepancy of the experiments' appendix; with
+ *          greedy decoding the appendix's -log p(argmax q)),
  *          pi = (1 - delta) q + delta p;
  *
  *   or the log-loss plug-in rules (appendix on log loss), delta by entropies:
@@ -45,7 +46,9 @@
  *   and, with T = 0, greedy decoding (appendix, the greedy special case): the
  *   rule is evaluated on the untempered softmax (T = 1) except that its D_TV is
  *   that of the one-hot q~, p~ at the argmaxes (lowest index on ties), i.e.
- *   1(argmax q != argmax p), as in the greedy lemma; pi = (1 - delta) q~ + delta p~,
+ *   1(argmax q != argmax p), as in the greedy lemma, and BiLD*'s discrepancy is
+ *   -log p(argmax q) as the experiments' appendix sets it for greedy decoding;
+ *   pi = (1 - delta) q~ + delta p~,
  *   and Algorithm 4 runs on those:
  *   a draft is rejected only when delta = 1 and it is not the verifier's argmax,
  *   and the residual (and bonus) token is the verifier's argmax.
@@ -91,7 +94,7 @@
 #define OR_TOKEN_V2 6 /* token-specific: r(v) = [p(v) < max p - alpha] */
 #define OR_TOKEN_V3 7 /* token-specific: r(v) = [p(v) < max p (1 - alpha)] */
 #define OR_LOSSY 8    /* lossy speculative decoding target (Table 3, Lemma 2), parameter beta */
-#define OR_BILD 9     /* BiLD*: delta = 1(-sum_v q(v) log p(v) > alpha) */
+#define OR_BILD 9     /* BiLD*: delta = 1(D(q, p) > alpha), D = -sum_v q(v) log p(v) (T > 0) or -log p(argmax q) (T = 0) */
 #define OR_CHOW_LOG 10 /* H(q) > alpha */
 #define OR_DIFF_LOG 11 /* sum q log q < sum p log p - alpha */
 #define OR_OPT_LOG 12  /* sum q log q < sum p log p - alpha D_TV(p, q) */
@@ -470,7 +473,10 @@ static void verify_sequence(const void *draft, const void *target, int dtype,
             }
             m_delta = fabs(lhs - rhs);
         } else if (rule == OR_BILD) {
-            const double D = cross_entropy(q, target, dtype, tbase + (size_t)j * V, V, Tr, Mp, lnSp);
+            /* greedy decoding: the BiLD baseline's D(q, p) = -log p(argmax q); with a
+               temperature, its analogue -sum_v q(v) log p(v) */
+            const double D = greedy ? -log_prob(target, dtype, tbase + (size_t)j * V, argmax_of(q, V), Tr, Mp, lnSp)
+                                    : cross_entropy(q, target, dtype, tbase + (size_t)j * V, V, Tr, Mp, lnSp);
             delta = D > alpha;  /* strict, as printed */
             m_delta = isfinite(D) ? fabs(D - alpha) : INFINITY;
         } else {

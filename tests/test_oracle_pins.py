@@ -691,6 +691,25 @@ def test_greedy_always_defer_is_greedy_speculative_decoding():
     np.testing.assert_array_equal(r.next_token, nt)
 
 
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_greedy_bild_uses_the_log_probability_of_q_argmax(seed):
+    """At T = 0 the BiLD baseline's discrepancy is D = -log p(argmax q) (lowest index
+    on ties), not the sampling analogue -sum q log p: delta = [D > alpha] per row."""
+    rng = np.random.default_rng(seed)
+    g, V = 6, 50
+    q_log = (rng.standard_normal((g, V)) * 2.0).astype(np.float32)
+    p_log = (q_log[np.r_[0:g, g - 1]] + rng.standard_normal((g + 1, V)) * 1.5).astype(np.float32)
+    q = np_softmax(q_log.astype(np.float64), 1.0)
+    p = np_softmax(p_log.astype(np.float64), 1.0)
+    D = -np.log(p[np.arange(g), q.argmax(1)])
+    alpha = float(np.median(D))
+    w = rows_workload(np.exp(q_log), np.exp(p_log), q_log.argmax(1), np.full(g + 1, 0.5), "bild", alpha)
+    w.temperature = 0.0
+    r = oracle.verify_workload(w)
+    np.testing.assert_array_equal(r.row("delta")[0], (D > alpha).astype(float))
+    assert 0 < (D > alpha).sum() < g
+
+
 @pytest.mark.parametrize("alpha", [0.0, 0.05, 0.2, 0.6, 1.0])
 def test_greedy_opt_equals_greedy_diff(alpha):
     """The greedy special case (appendix): with T -> 0 the OPT rule's TV term is
