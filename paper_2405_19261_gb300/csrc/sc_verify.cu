@@ -1366,6 +1366,14 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       sh.nhq = kLn2 * (g.aq / as - log2f(as));
       sh.nhp = kLn2 * (g.ap / cs - log2f(cs));
       xent = kLn2 * (log2f(cs) - g.x / as);
+      if (P.greedy && pair && P.rule == SC_RULE_BILD && g.iq >= 0 && g.iq < P.V) {
+        // greedy decoding: the BiLD baseline's D = -log p(argmax q), from the target
+        // logit at q's argmax (one load; every CTA of the cluster reads the same value)
+        const E *prow = static_cast<const E *>(P.target) + (static_cast<size_t>(b) * G1 + j) * P.V;
+        const float y = Elt<E>::at(prow, static_cast<size_t>(g.iq));
+        const float2 lp = log2_prob(y, Rp, cs, k, P.kl);
+        xent = y > -INFINITY ? -kLn2 * (lp.x + lp.y) : INFINITY;
+      }
       if (P.greedy && pair) sh.tv = g.iq != g.ip ? 1.0f : 0.0f;  // D_TV of the one-hot q~, p~
     }
     if (!err && pair) {
