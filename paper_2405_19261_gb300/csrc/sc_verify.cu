@@ -285,7 +285,7 @@ struct __align__(16) Shared {
   float4 all_ms[kMaxCluster];  // 1: (m_q, s_q, m_p, s_p) of the slice
   float2 all_x[kMaxCluster];   // 1: raw logits at the draft token, if in the slice
   float all_r[kMaxCluster];    // 2 (TV pass): the slice's total residual weight
-  float all_lb[kMaxCluster];   // OPT band: the slice's lower bound on D_TV
+  float2 all_lb[kMaxCluster];  // OPT band: the slice's lower bound on D_TV, and its sum of sqrt(q p)
   float2 all_scr[kMaxCluster]; // token rules: the slice's sum of q over its undeferred tokens, and
                                // whether its screen is exact (1) or not (0)
   float4 all_ext[kMaxCluster]; // 1 (kFamExt): (A_q, A_p, X, -) of the slice, see ExtState
@@ -761,6 +761,27 @@ __device__ __forceinline__ void bonus_row(const E *src, int n, float k, float &m
   }
 }
 
+// OPT: this thread's sum over a chunk of 2^{(a_v + b_v)/2} = 2^{((y^q_v + y^p_v) k - r_q - r_p)/2},
+// sqrt(q_v p_v) up to the rows' normalisers: the Bhattacharyya coefficient
+// BC = sum_v sqrt(q_v p_v) bounds D_TV from above, D_TV <= sqrt(1 - BC^2).
+template <typename E, bool kFull>
+__device__ __forceinline__ float bc_chunk(const E *srcq, const E *srcp, int n, float hk, float hr) {
+  float acc0 = 0.0f, acc1 = 0.0f;
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r) {
+    const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
+    float yq[8], yp[8];
+    load8_chunk<E, kFull>(srcq, e, n, yq);
+    load8_chunk<E, kFull>(srcp, e, n, yp);
+#pragma unroll
+    for (int i = 0; i < 8; i += 2) {
+      acc0 += ex2(fmaf(yq[i] + yp[i], hk, -hr));
+      acc1 += ex2(fmaf(yq[i + 1] + yp[i + 1], hk, -hr));
+    }
+  }
+  return acc0 + acc1;
+}
+
 // Weights of one chunk in the ring: per round, the warp's total weight (the
 // segment total) lands in seg[(c, round, warp)].
 template <typename E, bool kPair, bool kFull, bool kTok>
@@ -1202,6 +1223,9 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   ExtState ex = ext_empty();  // (kFamExt) moments and argmaxes
   Top2 top = {-FLT_MAX, -FLT_MAX, -FLT_MAX};  // (kFamToken) the eta screen
   const bool scr_q = P.rule == SC_RULE_TOKEN_V1;
+  // OPT: the pair's running sum of sqrt(q p) terms, relative to (r_q + r_p) / 2
+  const bool opt_bc = !kTok && !kExt && verify && pair && P.rule == SC_RULE_OPT;
+  float bc = 0.0f;
   // the bonus row also leaves its per-(chunk, warp) totals for the sampler
   const bool bonus_tot = verify && !pair && !P.greedy;
   const int lx = x - v0;  // draft token's offset in this slice (thread 0 only)
@@ -1219,14 +1243,24 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
         if (n == kCH) ext_chunk<E, true, false>(R.q(s), R.p(s), n, vc, k, ex);
         else ext_chunk<E, false, false>(R.q(s), R.p(s), n, vc, k, ex);
       }
-    } else if (n == kCH) {
-      if (pair) online_row<E, true>(R.q(s), n, k, mq, s2q);
-      online_row<E, true>(R.p(s), n, k, mp, s2p);
-      if (kTok && pair) screen_chunk<E, true>(scr_q ? R.q(s) : R.p(s), R.q(s), n, top);
     } else {
-      if (pair) online_row<E, false>(R.q(s), n, k, mq, s2q);
-      online_row<E, false>(R.p(s), n, k, mp, s2p);
-      if (kTok && pair) screen_chunk<E, false>(scr_q ? R.q(s) : R.p(s), R.q(s), n, top);
+      const float mq0 = mq, mp0 = mp;
+      if (n == kCH) {
+        if (pair) online_row<E, true>(R.q(s), n, k, mq, s2q);
+        online_row<E, true>(R.p(s), n, k, mp, s2p);
+        if (kTok && pair) screen_chunk<E, true>(scr_q ? R.q(s) : R.p(s), R.q(s), n, top);
+      } else {
+        if (pair) online_row<E, false>(R.q(s), n, k, mq, s2q);
+        online_row<E, false>(R.p(s), n, k, mp, s2p);
+        if (kTok && pair) screen_chunk<E, false>(scr_q ? R.q(s) : R.p(s), R.q(s), n, top);
+      }
+      if (opt_bc) {
+        const float rq = refk(mq, k), rp = refk(mp, k);
+        const float sc = ex2(0.5f * ((refk(mq0, k) - rq) + (refk(mp0, k) - rp)));
+        const float add = n == kCH ? bc_chunk<E, true>(R.q(s), R.p(s), n, 0.5f * k, 0.5f * (rq + rp))
+                                   : bc_chunk<E, false>(R.q(s), R.p(s), n, 0.5f * k, 0.5f * (rq + rp));
+        bc = fmaf(bc, sc, add);
+      }
     }
     if (tid == 0 && static_cast<unsigned>(lx - c * kCH) < static_cast<unsigned>(n)) {
       sh.xq = Elt<E>::at(R.q(s), lx - c * kCH);
@@ -1489,22 +1523,41 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     const float pt = mine.w * ex2(refk(mine.z, k) - sh.Rp) / sh.Sp;
     const float qt = mine.y * ex2(refk(mine.x, k) - sh.Rq) / sh.Sq;
     const float lb = warp_sum(fmaxf(0.0f, pt - qt));
-    if (lane == 0) sh.red[warp].x = lb;
+    // OPT: this thread's sum of sqrt(q p) terms at the row's references
+    const float bcw = warp_sum(bc * ex2(0.5f * ((refk(mine.x, k) - sh.Rq) + (refk(mine.z, k) - sh.Rp))));
+    if (lane == 0) sh.red[warp] = make_float4(lb, bcw, 0.0f, 0.0f);
     __syncthreads();
     if (tid == 0) {
-      float acc = 0.0f;
-      for (int w = 0; w < kNW; ++w) acc = __fadd_rn(acc, sh.red[w].x);
-      for (int r = 0; r < C; ++r) st_peer(peer_addr(&sh.all_lb[rank], r), acc);
+      float acc = 0.0f, accb = 0.0f;
+      for (int w = 0; w < kNW; ++w) {
+        acc = __fadd_rn(acc, sh.red[w].x);
+        accb = __fadd_rn(accb, sh.red[w].y);
+      }
+      for (int r = 0; r < C; ++r) st_peer(peer_addr(&sh.all_lb[rank], r), make_float2(acc, accb));
     }
     cluster_arrive();
     cluster_wait();
     if (tid == 0) {
-      float LB = 0.0f;  // in rank order
-      for (int r = 0; r < C; ++r) LB = __fadd_rn(LB, sh.all_lb[r]);
-      if (P.alpha * LB - (sh.dr - sh.dl) >= 1e-4f) {
+      float LB = 0.0f, BCs = 0.0f;  // in rank order
+      for (int r = 0; r < C; ++r) {
+        LB = __fadd_rn(LB, sh.all_lb[r].x);
+        BCs = __fadd_rn(BCs, sh.all_lb[r].y);
+      }
+      const float gap = sh.dr - sh.dl;
+      if (P.alpha * LB - gap >= 1e-4f) {
         sh.need_p2 = 0;
         sh.delta = 0;
         accept_test<kFam>(sh, P, x, sh.xq, sh.xp, uj, k);
+      } else if (opt_bc) {
+        // D_TV <= sqrt(1 - BC^2) (Hellinger): with BC deflated well past its f32
+        // error, alpha times that bound below max p - max q settles delta = 1 (Eq. 10)
+        const float bcl = fminf(1.0f, BCs / sqrtf(sh.Sq) / sqrtf(sh.Sp)) * (1.0f - 2e-4f);
+        const float ub = sqrtf(fmaxf(0.0f, 1.0f - bcl * bcl));
+        if (gap - P.alpha * ub >= 1e-4f) {
+          sh.need_p2 = 0;
+          sh.delta = 1;
+          accept_test<kFam>(sh, P, x, sh.xq, sh.xp, uj, k);
+        }
       }
     }
     __syncthreads();

@@ -319,10 +319,13 @@ def test_repeatable_and_workspace_reuse(sc):
 
 
 @pytest.mark.parametrize("alpha", [0.2, 0.5, 1.0])
-def test_opt_band_settled_by_tv_lower_bound(sc, alpha):
+def test_opt_band_settled_by_tv_bounds(sc, alpha):
     # Inside the OPT band (max p - alpha <= max q < max p) the kernel first bounds
-    # D_TV from below by its threads' partial masses; rows the bound settles at
-    # delta = 0 report no TV (-1).  Their decisions must still be the oracle's.
+    # D_TV from below by its threads' partial masses (settling delta = 0) and from
+    # above by sqrt(1 - BC^2), BC = sum_v sqrt(q p) (settling delta = 1); settled
+    # rows report no TV (-1).  Their decisions must still be the oracle's.
+    from paper_2405_19261_gb300.workloads import logits_as_f64
+    from scipy.special import softmax
     w = synthetic(24, 8, 256000, dtype="bf16", kind="zipf", sigma=0.7, rule="opt", alpha=alpha,
                   temperature=1.0, seed=31)
     gpu = run_gpu(sc, w)
@@ -332,12 +335,18 @@ def test_opt_band_settled_by_tv_lower_bound(sc, alpha):
     maxq, maxp, tv = ref.row("maxq"), ref.row("maxp"), ri[..., 2]
     band = (maxq < maxp) & (maxq >= maxp - alpha)
     settled = band & (tv < 0)
-    assert settled.sum() > 0, "no band row was settled by the bound"
-    np.testing.assert_array_equal(ri[..., 3][settled], 0.0)
-    np.testing.assert_array_equal(ref.row("delta")[settled], 0.0)
+    assert settled.sum() > 0, "no band row was settled by a bound"
+    np.testing.assert_array_equal(ri[..., 3][settled], ref.row("delta")[settled])
     # the rows left to the TV pass report an exact D_TV
     exact = band & ~settled
     np.testing.assert_allclose(tv[exact], ref.row("tv")[exact], atol=TOL)
+    # every band row whose Hellinger bound clearly decides delta = 1 was settled by it
+    q = softmax(logits_as_f64(w.draft, "bf16"), axis=-1)
+    p = softmax(logits_as_f64(w.target[:, :w.gamma], "bf16"), axis=-1)
+    ub = np.sqrt(np.maximum(0.0, 1.0 - np.sum(np.sqrt(q * p), axis=-1) ** 2))
+    clear = band & (maxp - maxq - alpha * ub >= 1e-3)
+    np.testing.assert_array_equal(tv[clear], -1.0)
+    np.testing.assert_array_equal(ri[..., 3][clear], 1.0)
 
 
 # ----------------------------------------------------------------- maximum sizes
