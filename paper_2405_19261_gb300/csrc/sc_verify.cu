@@ -69,6 +69,9 @@ namespace {
 #ifndef SC_MIN_BLOCKS
 #define SC_MIN_BLOCKS 6
 #endif
+#ifndef SC_OPT_UB
+#define SC_OPT_UB 1  // OPT band rows: settle delta = 1 by the Bhattacharyya bound on D_TV
+#endif
 #ifndef SC_BONUS_LAST
 #define SC_BONUS_LAST 0  // 1: launch all pair units before the bonus rows
 #endif
@@ -1224,7 +1227,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   Top2 top = {-FLT_MAX, -FLT_MAX, -FLT_MAX};  // (kFamToken) the eta screen
   const bool scr_q = P.rule == SC_RULE_TOKEN_V1;
   // OPT: the pair's running sum of sqrt(q p) terms, relative to (r_q + r_p) / 2
-  const bool opt_bc = !kTok && !kExt && verify && pair && P.rule == SC_RULE_OPT;
+  const bool opt_bc = SC_OPT_UB && !kTok && !kExt && verify && pair && P.rule == SC_RULE_OPT;
   float bc = 0.0f;
   // the bonus row also leaves its per-(chunk, warp) totals for the sampler
   const bool bonus_tot = verify && !pair && !P.greedy;
