@@ -538,7 +538,7 @@ __device__ __forceinline__ void load8_chunk(const E *src, int e, int n, float (&
 
 template <typename E, bool kFull, bool kPair>
 __device__ __forceinline__ void ext_chunk(const E *srcq, const E *srcp, int n, int v0, float k,
-                                          ExtState &st) {
+                                          ExtState &st, bool with_bc, float &bc) {
   float mq = st.mq, mp = st.mp;
   int iq = st.iq, ip = st.ip;
 #pragma unroll
@@ -562,8 +562,9 @@ __device__ __forceinline__ void ext_chunk(const E *srcq, const E *srcp, int n, i
     }
   }
   const float rq = refk(mq, k), rp = refk(mp, k);
+  if (with_bc) bc *= ex2(0.5f * ((refk(st.mq, k) - rq) + (refk(st.mp, k) - rp)));  // (OPTLog's bound)
   ext_rebase(st, refk(st.mq, k) - rq, refk(st.mp, k) - rp);
-  float sq = 0.0f, aq = 0.0f, sp = 0.0f, ap = 0.0f, x = 0.0f;
+  float sq = 0.0f, aq = 0.0f, sp = 0.0f, ap = 0.0f, x = 0.0f, h = 0.0f;
 #pragma unroll
   for (int r = 0; r < kRounds; ++r) {
     const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
@@ -582,9 +583,11 @@ __device__ __forceinline__ void ext_chunk(const E *srcq, const E *srcp, int n, i
         sq += ea;
         aq += ea > 0.0f ? ea * a : 0.0f;
         x += ea > 0.0f ? ea * b : 0.0f;
+        if (with_bc) h += ex2(0.5f * (a + b));  // sqrt(q p) up to the normalisers
       }
     }
   }
+  if (with_bc) bc += h;
   st.mq = mq;
   st.mp = mp;
   st.iq = iq;
@@ -1228,6 +1231,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   const bool scr_q = P.rule == SC_RULE_TOKEN_V1;
   // OPT: the pair's running sum of sqrt(q p) terms, relative to (r_q + r_p) / 2
   const bool opt_bc = SC_OPT_UB && !kTok && !kExt && verify && pair && P.rule == SC_RULE_OPT;
+  const bool optlog_bc = SC_OPT_UB && kExt && verify && pair && !P.greedy && P.rule == SC_RULE_OPT_LOG;
   float bc = 0.0f;
   // the bonus row also leaves its per-(chunk, warp) totals for the sampler
   const bool bonus_tot = verify && !pair && !P.greedy;
@@ -1240,11 +1244,11 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     } else if constexpr (kExt) {
       const int vc = v0 + c * kCH;
       if (pair) {
-        if (n == kCH) ext_chunk<E, true, true>(R.q(s), R.p(s), n, vc, k, ex);
-        else ext_chunk<E, false, true>(R.q(s), R.p(s), n, vc, k, ex);
+        if (n == kCH) ext_chunk<E, true, true>(R.q(s), R.p(s), n, vc, k, ex, optlog_bc, bc);
+        else ext_chunk<E, false, true>(R.q(s), R.p(s), n, vc, k, ex, optlog_bc, bc);
       } else {
-        if (n == kCH) ext_chunk<E, true, false>(R.q(s), R.p(s), n, vc, k, ex);
-        else ext_chunk<E, false, false>(R.q(s), R.p(s), n, vc, k, ex);
+        if (n == kCH) ext_chunk<E, true, false>(R.q(s), R.p(s), n, vc, k, ex, false, bc);
+        else ext_chunk<E, false, false>(R.q(s), R.p(s), n, vc, k, ex, false, bc);
       }
     } else {
       const float mq0 = mq, mp0 = mp;
@@ -1551,9 +1555,9 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
         sh.need_p2 = 0;
         sh.delta = 0;
         accept_test<kFam>(sh, P, x, sh.xq, sh.xp, uj, k);
-      } else if (opt_bc) {
+      } else if (opt_bc || optlog_bc) {
         // D_TV <= sqrt(1 - BC^2) (Hellinger): with BC deflated well past its f32
-        // error, alpha times that bound below max p - max q settles delta = 1 (Eq. 10)
+        // error, alpha times that bound below the gap settles delta = 1 (Eq. 10, OPTLog)
         const float bcl = fminf(1.0f, BCs / sqrtf(sh.Sq) / sqrtf(sh.Sp)) * (1.0f - 2e-4f);
         const float ub = sqrtf(fmaxf(0.0f, 1.0f - bcl * bcl));
         if (gap - P.alpha * ub >= 1e-4f) {
