@@ -180,6 +180,13 @@ int sc_row_stats(const void *draft_logits, const void *target_logits, sc_dtype d
 /* Static description of an sc_status code. */
 const char *sc_status_string(int code);
 
+/* Builds with -DSC_DEBUG=1 check the kernel's computed indices, copy sizes and
+ * alignments, skip an access that fails (its outputs are then undefined; a skipped
+ * copy ends in SC_DEV_TIMEOUT) and record the kernel source line of the first
+ * failure.  Returns that line (0: none), clearing it when `reset` is nonzero,
+ * SC_ERR_CUDA if it cannot be read, and -1 in builds without the checks. */
+int sc_debug_line(int reset);
+
 /*
  * sc_verify_static -- sc_verify for callers that cannot allocate device memory.
  *

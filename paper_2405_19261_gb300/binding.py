@@ -53,6 +53,8 @@ def lib():
         L.sc_verify_ex.restype = I
         L.sc_row_stats.argtypes = [P, P, I, I, I, I, F, P, P, P, P]
         L.sc_row_stats.restype = I
+        L.sc_debug_line.argtypes = [I]
+        L.sc_debug_line.restype = I
         L.sc_status_string.argtypes = [I]
         L.sc_status_string.restype = ctypes.c_char_p
         _lib = L
@@ -97,6 +99,12 @@ def workspace_bytes(B: int, gamma: int, V: int = 0) -> int:
 def new_workspace(B: int, gamma: int, device=None) -> torch.Tensor:
     """A zeroed workspace tensor for ``sc_verify`` (reusable across calls)."""
     return torch.zeros(workspace_bytes(B, gamma), dtype=torch.uint8, device=device or "cuda")
+
+
+def debug_line(reset: bool = False) -> int:
+    """Kernel source line of the first failed device-side check (a library built
+    with SC_DEBUG; 0: none), or -1 for a library built without the checks."""
+    return int(lib().sc_debug_line(1 if reset else 0))
 
 
 def max_vocab(dtype: torch.dtype) -> int:

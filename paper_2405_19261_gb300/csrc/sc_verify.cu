@@ -69,6 +69,9 @@ namespace {
 #ifndef SC_MIN_BLOCKS
 #define SC_MIN_BLOCKS 6
 #endif
+#ifndef SC_DEBUG
+#define SC_DEBUG 0  // 1: check computed indices and copy sizes, skip and record a failing access
+#endif
 #ifndef SC_OPT_UB
 #define SC_OPT_UB 1  // OPT band rows: settle delta = 1 by the Bhattacharyya bound on D_TV
 #endif
@@ -144,6 +147,20 @@ struct Params {
                            // sampled row at each chunk start, then the slice total
   int32_t *status;
 };
+
+// ------------------------------------------------------------------ debug checks
+
+// First source line whose check failed (SC_DEBUG builds; 0: none).
+__device__ int g_sc_debug_line;
+
+// In SC_DEBUG builds, false for a failed check (its line recorded, the access
+// skipped by the caller); always true otherwise, and compiled away.
+__device__ __forceinline__ bool sc_check(bool cond, int line) {
+  if (!SC_DEBUG || cond) return true;
+  atomicCAS(&g_sc_debug_line, 0, line);
+  return false;
+}
+#define SC_CHECK(cond) sc_check((cond), __LINE__)
 
 // ------------------------------------------------------------------ PTX helpers
 
@@ -941,6 +958,10 @@ struct Ring {
   // thread 0, bulk mode: start the copies of chunk c into stage s
   __device__ void issue(Shared &sh, int c, int s) const {
     const uint32_t bytes = static_cast<uint32_t>(chunk_len(c)) * sizeof(E);
+    if (!SC_CHECK(c >= 0 && c < nch && s >= 0 && s < kStages && bytes > 0 && bytes % 16 == 0 &&
+                  reinterpret_cast<uintptr_t>(gp + static_cast<size_t>(c) * kCH) % 16 == 0 &&
+                  (!pair || reinterpret_cast<uintptr_t>(gq + static_cast<size_t>(c) * kCH) % 16 == 0)))
+      return;
     mbar_expect_tx(&sh.full[s], pair ? 2 * bytes : bytes);
     if (pair) bulk_g2s(q(s), gq + static_cast<size_t>(c) * kCH, bytes, &sh.full[s]);
     bulk_g2s(p(s), gp + static_cast<size_t>(c) * kCH, bytes, &sh.full[s]);
@@ -953,6 +974,7 @@ struct Ring {
   }
   // all threads, per-thread mode: copy chunk c into stage s
   __device__ void load_sync(int c, int s) const {
+    if (!SC_CHECK(c >= 0 && c < nch && s >= 0 && s < kStages)) return;
     const int n = chunk_len(c);
     const size_t o = static_cast<size_t>(c) * kCH;
     for (int i = threadIdx.x; i < n; i += kNT) {
@@ -1388,13 +1410,13 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       float *cp = P.bonus_pre + (static_cast<size_t>(b) * kMaxCluster + rank) * (kMaxChunks + 1);
       float acc = 0.0f;
       for (int c2 = 0; c2 < R.nch; ++c2) {
-        cp[c2] = acc;
+        if (SC_CHECK(b < P.B && rank < kMaxCluster && c2 < kMaxChunks)) cp[c2] = acc;
         float t = 0.0f;
         for (int w = 0; w < kNW; ++w)
           t = fmaf(sh.seg[c2 * kNW + w], ex2(refk(sh.seg[kBonusRef + c2 * kNW + w], k) - Rp), t);
         acc = __fadd_rn(acc, t);
       }
-      cp[R.nch] = err || tmo ? NAN : acc;
+      if (SC_CHECK(b < P.B && rank < kMaxCluster && R.nch <= kMaxChunks)) cp[R.nch] = err || tmo ? NAN : acc;
     }
     sh.dl = sh.maxq;
     sh.dr = sh.maxp;
@@ -1634,8 +1656,10 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     }
     if (tid == 0) {
       float *cp = P.row_pre + ((static_cast<size_t>(b) * G1 + j) * kMaxCluster + rank) * (kMaxChunks + 1);
-      for (int c = 0; c < R.nch; ++c) cp[c] = sh.seg[c * kRounds * kNW];
-      cp[R.nch] = sh.timeout ? NAN : sh.seg[R.nch * kRounds * kNW];
+      if (SC_CHECK(b < P.B && j < G1 && rank < kMaxCluster && R.nch <= kMaxChunks)) {
+        for (int c = 0; c < R.nch; ++c) cp[c] = sh.seg[c * kRounds * kNW];
+        cp[R.nch] = sh.timeout ? NAN : sh.seg[R.nch * kRounds * kNW];
+      }
     }
     __syncthreads();
   }
@@ -1659,9 +1683,10 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       if (kFam == kFamCascade && P.rule == SC_RULE_LOSSY)
         r1.z = sh.c + P.lossy_c;  // the residual max(0, p / beta - q) (Lemma 2)
       if (kExt && P.greedy) r1.x = __int_as_float(sh.ip);  // greedy: the token emitted at row j*
-      rec[j] = r1;
+      if (SC_CHECK(b < P.B && rank < kMaxCluster && j < G1)) rec[j] = r1;
       if (kTok)  // (only token rules read the second record)
-        rec2[j] = make_float4(sh.eta, sh.thr, __int_as_float(sh.tok), __int_as_float(sh.on_q));
+        if (SC_CHECK(b < P.B && rank < kMaxCluster && j < G1))
+          rec2[j] = make_float4(sh.eta, sh.thr, __int_as_float(sh.tok), __int_as_float(sh.on_q));
       if (rank == 0 && P.row_info) {
         float *ri = P.row_info + (static_cast<size_t>(b) * G1 + j) * SC_ROW_FIELDS;
         ri[SC_ROW_MAXQ] = pair && !sh.err ? sh.maxq : NAN;
@@ -1738,8 +1763,10 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
           flag_timeout(sh, P);
         }
         float *cp = P.chunk_pre + (static_cast<size_t>(b) * kMaxCluster + rank) * (kMaxChunks + 1);
-        for (int c = 0; c < Rj.nch; ++c) cp[c] = sh.seg[c * kRounds * kNW];
-        cp[Rj.nch] = tot_r;  // the slice total
+        if (SC_CHECK(b < P.B && rank < kMaxCluster && Rj.nch <= kMaxChunks)) {
+          for (int c = 0; c < Rj.nch; ++c) cp[c] = sh.seg[c * kRounds * kNW];
+          cp[Rj.nch] = tot_r;  // the slice total
+        }
         sh.seq_last = atom_add_acq_rel(P.seq_tickets + b, 1u) == static_cast<uint32_t>(C);
       }
       __syncthreads();
@@ -1787,12 +1814,13 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       for (int i = tid; i < C * kCP && !(kExt && P.greedy); i += kNT) {
         const int r = i / kCP, c = i % kCP;
         const int len = max(0, min(P.L, P.V - r * P.L));
-        if (c <= (len + kCH - 1) / kCH) cpall[i] = __ldcg(cpg + i);
+        if (c <= (len + kCH - 1) / kCH && SC_CHECK(b < P.B && js <= P.gamma && C <= kMaxCluster))
+          cpall[i] = __ldcg(cpg + i);
       }
       __syncthreads();
       if (kExt && P.greedy) {
         // greedy decoding: the argmax p of row j*, from rank 0's record
-        if (tid == 0) {
+        if (tid == 0 && SC_CHECK(b < P.B && js >= 0 && js <= P.gamma)) {
           const bool ok = !sh.bad;
           const int tok = __float_as_int(sh.rj.x);
           P.num_accepted[b] = ok ? js : 0;
@@ -1911,7 +1939,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
           }
           __syncthreads();
         }
-        if (tid == 0) {
+        if (tid == 0 && SC_CHECK(b < P.B && js >= 0 && js <= P.gamma)) {
           const bool ok = sh.sample_ok != 0;
           P.num_accepted[b] = ok ? js : 0;
           P.next_token[b] = ok ? sh.token : -1;
@@ -2143,6 +2171,17 @@ size_t sc_workspace_bytes(int B, int gamma, int V) {
 int sc_workspace_init(void *workspace, size_t workspace_bytes, cudaStream_t stream) {
   if (!workspace) return SC_ERR_INVALID_ARG;
   return cudaMemsetAsync(workspace, 0, workspace_bytes, stream) == cudaSuccess ? SC_OK : SC_ERR_CUDA;
+}
+
+int sc_debug_line(int reset) {
+  if (!SC_DEBUG) return -1;
+  int line = 0;
+  if (cudaMemcpyFromSymbol(&line, g_sc_debug_line, sizeof(int)) != cudaSuccess) return SC_ERR_CUDA;
+  if (reset) {
+    const int zero = 0;
+    if (cudaMemcpyToSymbol(g_sc_debug_line, &zero, sizeof(int)) != cudaSuccess) return SC_ERR_CUDA;
+  }
+  return line;
 }
 
 int sc_max_vocab(sc_dtype dtype) {
