@@ -778,7 +778,7 @@ __device__ __forceinline__ void bonus_row(const E *src, int n, float k, float &m
   s = make_float2(fmaf(cs, ex2(rw - rn), s.x * so), s.y * so);
   m = mn;
   const float tot = warp_sum(cs);
-  if (lane == 0) {
+  if (lane == 0 && SC_CHECK(c >= 0 && c < kMaxChunks)) {
     seg[c * kNW + warp] = tot;
     seg[kBonusRef + c * kNW + warp] = W;
   }
@@ -823,7 +823,7 @@ __device__ __forceinline__ void weights_chunk(const E *sq, const E *sp, int n, i
       load8_smem(sp, e, n, yp);
     }
     const float tot = warp_sum(vec_weights<kPair, kTok>(yq, yp, rs, w));
-    if (lane == 0) sh.seg[(c * kRounds + r) * kNW + warp] = tot;
+    if (lane == 0 && SC_CHECK(c >= 0 && c < kMaxChunks)) sh.seg[(c * kRounds + r) * kNW + warp] = tot;
   }
 }
 
