@@ -231,6 +231,22 @@ def oracle_throughput(w, max_seqs=64, min_core_s=0.0):
 
 # ------------------------------------------------------------------ multi-rank
 
+def step_spread(ms_steps):
+    """Median, 10th and 90th percentile of the per-step device times (this rank's),
+    by linear interpolation between order statistics."""
+    xs = sorted(ms_steps)
+
+    def pct(q):
+        if not xs:
+            return None
+        h = (len(xs) - 1) * q
+        lo = int(h)
+        hi = min(lo + 1, len(xs) - 1)
+        return xs[lo] + (xs[hi] - xs[lo]) * (h - lo)
+
+    return {"p10": pct(0.1), "median": pct(0.5), "p90": pct(0.9), "n": len(xs)}
+
+
 def max_over_ranks(value, world, device):
     """The largest of every rank's value (all_reduce MAX); value itself on one rank."""
     if world <= 1:
@@ -367,21 +383,25 @@ def run_ours(args):
             step()
             e1.record(stream)
         torch.cuda.synchronize(dev)
-        ms_total = sum(e0.elapsed_time(e1) for e0, e1 in evs)
+        ms_steps = [e0.elapsed_time(e1) for e0, e1 in evs]
+        ms_total = sum(ms_steps)
     else:
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        for _ in range(args.steps):
+        # an event between consecutive steps: the K intervals tile the timed region
+        evs = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+        evs[0].record(stream)
+        for i in range(args.steps):
             step()
-        e1.record(stream)
+            evs[i + 1].record(stream)
         torch.cuda.synchronize(dev)
-        ms_total = e0.elapsed_time(e1)
+        ms_total = evs[0].elapsed_time(evs[-1])
+        ms_steps = [a.elapsed_time(b) for a, b in zip(evs[:-1], evs[1:])]
     if world > 1:
         dist.barrier()
     sampler.stop()
     clocks = sampler.summary()
 
     ms_step = max_over_ranks(ms_total / args.steps, world, dev)
+    spread = step_spread(ms_steps)
     mean_accepted = float(na.float().mean().item())  # j* of the last step (the method's own statistic)
     positions = B * g * world
     value = whole_job_rate(B * g, world, ms_step)
@@ -451,7 +471,7 @@ def run_ours(args):
                                   if flush else
                                   f"inputs {w.logit_bytes / 1e6:.0f} MB > L2 {l2 / 1e6:.0f} MB, back to back"),
                            "parallelism": f"{world} independent replica(s), no collective"},
-                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+                "step_ms": spread, "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
                 "gpu_launches": args.steps, "clocks": clocks}
         print(json.dumps(line), flush=True)
     if world > 1:

@@ -40,3 +40,17 @@ def test_record_traffic_from_an_ncu_csv(tmp_path, monkeypatch):
     d["cfgX: a workload"]["kernel_sha"] = "0" * 16
     (tmp_path / "traffic.json").write_text(json.dumps(d))
     assert bench.stored_traffic("cfgX: a workload") is None
+
+
+def test_step_spread_matches_linear_percentiles():
+    import numpy as np
+
+    import bench
+    rng = np.random.default_rng(5)
+    for n in (1, 2, 7, 50):
+        xs = list(rng.uniform(0.1, 0.3, n))
+        s = bench.step_spread(xs)
+        assert s["n"] == n
+        for key, q in (("p10", 10), ("median", 50), ("p90", 90)):
+            assert abs(s[key] - float(np.percentile(xs, q))) < 1e-12
+    assert bench.step_spread([])["median"] is None
