@@ -340,10 +340,12 @@ def test_opt_band_settled_by_tv_bounds(sc, alpha):
     # the rows left to the TV pass report an exact D_TV
     exact = band & ~settled
     np.testing.assert_allclose(tv[exact], ref.row("tv")[exact], atol=TOL)
-    # every band row whose Hellinger bound clearly decides delta = 1 was settled by it
+    # every band row whose Hellinger bound clearly decides delta = 1 was settled by
+    # it (the kernel shrinks BC by 2e-4 before the bound, far past its f32 error)
     q = softmax(logits_as_f64(w.draft, "bf16"), axis=-1)
     p = softmax(logits_as_f64(w.target[:, :w.gamma], "bf16"), axis=-1)
-    ub = np.sqrt(np.maximum(0.0, 1.0 - np.sum(np.sqrt(q * p), axis=-1) ** 2))
+    bc = np.minimum(1.0, np.sum(np.sqrt(q * p), axis=-1)) * (1.0 - 2e-4)
+    ub = np.sqrt(np.maximum(0.0, 1.0 - bc ** 2))
     clear = band & (maxp - maxq - alpha * ub >= 1e-3)
     np.testing.assert_array_equal(tv[clear], -1.0)
     np.testing.assert_array_equal(ri[..., 3][clear], 1.0)

@@ -169,7 +169,8 @@ def test_opt_log_band_settled_by_tv_bounds(sc, alpha):
     p = softmax(logits_as_f64(w.target[:, :w.gamma], "bf16"), axis=-1)
     gap = entropy(q, axis=-1) - entropy(p, axis=-1)          # sum p ln p - sum q ln q
     band = (gap > 0) & (gap <= alpha)
-    ub = np.sqrt(np.maximum(0.0, 1.0 - np.sum(np.sqrt(q * p), axis=-1) ** 2))
+    bc = np.minimum(1.0, np.sum(np.sqrt(q * p), axis=-1)) * (1.0 - 2e-4)  # as the kernel shrinks it
+    ub = np.sqrt(np.maximum(0.0, 1.0 - bc ** 2))
     clear = band & (gap - alpha * ub >= 1e-3)
     assert clear.sum() > 0
     np.testing.assert_array_equal(ri[..., 2][clear], -1.0)
