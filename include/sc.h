@@ -13,7 +13,8 @@
  * SC_RULE_TOKEN_V1..3).  Per sequence b it accepts draft
  * token x_j when u[b, j] < min(1, pi_j(x_j) / q_j(x_j)), finds the first
  * rejection j*, and draws one new token from norm(max(0, pi_{j*} - q_{j*})),
- * or from pi_gamma when all gamma drafts are accepted.
+ * or from pi_gamma := p_gamma (the drafter has no row at the bonus position)
+ * when all gamma drafts are accepted.
  *
  * Conventions of every entry point:
  *  - All array pointers are CUDA device pointers owned by the caller.  The
