@@ -206,12 +206,34 @@ class ClockSampler:
 
 # ------------------------------------------------------------------ oracle timing
 
-def oracle_throughput(w, max_seqs=64, min_core_s=0.0):
-    """Time the fp64 oracle (all host cores) on a bounded sample of sequences:
-    blocks of up to max_seqs sequences, cycling through the workload, until at
-    least min_core_s core-seconds (wall time x threads) have been spent."""
+def cpu_model():
+    """The host CPU's model name (x86 'model name', else lscpu's 'Model name', else the ISA)."""
+    import platform
+    import subprocess
+    try:
+        with open("/proc/cpuinfo") as f:
+            for ln in f:
+                if ln.lower().startswith("model name"):
+                    return ln.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for ln in out.splitlines():
+            if ln.startswith("Model name:"):
+                return ln.split(":", 1)[1].strip() + f" ({platform.machine()})"
+    except (OSError, subprocess.SubprocessError):
+        pass
+    return platform.machine()
+
+
+def oracle_throughput(w, max_seqs=64, min_core_s=0.0, threads=0):
+    """Time the fp64 oracle (all host cores, or `threads` of them) on a bounded
+    sample of sequences: blocks of up to max_seqs sequences, cycling through the
+    workload, until at least min_core_s core-seconds (wall time x threads) have
+    been spent."""
     import oracle
-    cores = oracle.num_threads(0)
+    cores = oracle.num_threads(threads)
     n = min(w.B, max(1, min(max_seqs, cores * 4)))
     done, passes, start = 0, 0, 0
     t0 = time.perf_counter()
@@ -455,6 +477,9 @@ def run_ours(args):
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu, _, _ = oracle_throughput(w, min_core_s=20.0)
+        one, _, _ = oracle_throughput(w, min_core_s=3.0, threads=1)
+        cpu["single_thread"] = {"value": one["value"], "sample": one["sample"]}
+        cpu["cpu_model"] = cpu_model()
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
