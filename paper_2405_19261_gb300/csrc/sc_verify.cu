@@ -78,6 +78,9 @@ namespace {
 #ifndef SC_BONUS_LAST
 #define SC_BONUS_LAST 0  // 1: launch all pair units before the bonus rows
 #endif
+#ifndef SC_PERSISTENT
+#define SC_PERSISTENT 0  // 1: a grid of co-resident clusters loops over the units (see the kernel)
+#endif
 #ifndef SC_L2_PREFETCH
 #define SC_L2_PREFETCH 1  // second passes prefetch their slice into L2 before streaming it
 #endif
@@ -119,6 +122,7 @@ struct Params {
   float temperature;
   float k;        // log2(e) / T, the f32 factor of every exponent of pass 1
   float kl;       // log2(e) / T - k: with k, log2(e) / T to twice f32 precision
+  int units;      // units of the call: B (gamma + 1) row pairs and bonus rows, or B gamma pairs
   int L;          // slice length per CTA (multiple of 8 logits)
   int cluster;    // CTAs per unit
   int bulk;       // 1: TMA bulk copies, 0: per-thread loads (rows not 16-byte aligned)
@@ -302,14 +306,17 @@ __device__ __forceinline__ void load8_smem(const E *s, int e, int n, float (&y)[
 struct __align__(16) Shared {
   uint64_t full[kStages];
   // cluster exchanges, written by every CTA of the cluster into slot [its rank]:
-  float4 all_ms[kMaxCluster];  // 1: (m_q, s_q, m_p, s_p) of the slice
-  float2 all_x[kMaxCluster];   // 1: raw logits at the draft token, if in the slice
+  // exchange 1 has two sets of slots, by the parity of the unit's iteration: a peer
+  // that loops on to its next unit pushes into the other set, never into the one
+  // this CTA may still be reading
+  float4 all_ms[2][kMaxCluster];  // 1: (m_q, s_q, m_p, s_p) of the slice
+  float2 all_x[2][kMaxCluster];   // 1: raw logits at the draft token, if in the slice
   float all_r[kMaxCluster];    // 2 (TV pass): the slice's total residual weight
   float2 all_lb[kMaxCluster];  // OPT band: the slice's lower bound on D_TV, and its sum of sqrt(q p)
   float2 all_scr[kMaxCluster]; // token rules: the slice's sum of q over its undeferred tokens, and
                                // whether its screen is exact (1) or not (0)
-  float4 all_ext[kMaxCluster]; // 1 (kFamExt): (A_q, A_p, X, -) of the slice, see ExtState
-  int2 all_idx[kMaxCluster];   // 1 (kFamExt): the slice's argmax of q and of p
+  float4 all_ext[2][kMaxCluster]; // 1 (kFamExt): (A_q, A_p, X, -) of the slice, see ExtState
+  int2 all_idx[2][kMaxCluster];   // 1 (kFamExt): the slice's argmax of q and of p
   int timeout;
   float4 red[kNW];          // (m_q, s_q, m_p, s_p) of each warp
   float4 ext_red[kNW];      // (kFamExt) (A_q, A_p, X, -) of each warp
@@ -1189,6 +1196,24 @@ __device__ __forceinline__ int search_segment(const E *sq, const E *sp, int n, b
   return tok;
 }
 
+// Row pair (b, j < gamma) or bonus row (b, gamma) of a unit (pairs only for sc_row_stats).
+__device__ __forceinline__ void unit_coords(const Params &P, int unit, int &b, int &j) {
+  const int G1 = P.gamma + 1;
+  if (P.mode == kVerify && SC_BONUS_LAST) {
+    // every pair unit first, then the bonus rows: the last, partial wave of CTAs
+    // holds the shorter (target-only) units
+    const int pairs = P.B * P.gamma;
+    b = unit < pairs ? unit / P.gamma : unit - pairs;
+    j = unit < pairs ? unit % P.gamma : P.gamma;
+  } else if (P.mode == kVerify) {
+    b = unit / G1;
+    j = unit % G1;
+  } else {
+    b = unit / P.gamma;
+    j = unit % P.gamma;
+  }
+}
+
 template <typename E, int kFam>
 __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Params P) {
   constexpr bool kTok = kFam == kFamToken;
@@ -1197,42 +1222,46 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   cg::cluster_group cluster = cg::this_cluster();
   const int C = P.cluster;
   const int rank = static_cast<int>(cluster.block_rank());
-  const int unit = static_cast<int>(blockIdx.x) / C;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int G1 = P.gamma + 1;
   const bool verify = P.mode == kVerify;
-
-  int b, j;
-  if (verify && SC_BONUS_LAST) {
-    // every pair unit first, then the bonus rows: the last, partial wave of CTAs
-    // holds the shorter (target-only) units
-    const int pairs = P.B * P.gamma;
-    b = unit < pairs ? unit / P.gamma : unit - pairs;
-    j = unit < pairs ? unit % P.gamma : P.gamma;
-  } else if (verify) {
-    b = unit / G1;
-    j = unit % G1;
-  } else {
-    b = unit / P.gamma;
-    j = unit % P.gamma;
-  }
-  const int v0 = rank * P.L;
-  const Ring<E> R = make_ring<E>(P, smem_raw, b, j, rank);
-  const bool pair = R.pair;
+  const int stride = static_cast<int>(gridDim.x) / C;  // clusters in the grid
   Shared &sh = *reinterpret_cast<Shared *>(smem_raw + static_cast<size_t>(kStages) * 2 * kCH * sizeof(E));
-
-  // ---- start the stream; prefetch the row's scalars
   if (tid == 0) {
     sh.timeout = 0;
-    sh.xq = NAN;
-    sh.xp = NAN;
-    if (R.bulk) {
+    if (P.bulk) {
       for (int s = 0; s < kStages; ++s) mbar_init(&sh.full[s], 1);
       asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
   }
-  uint32_t ph = 0;
+  uint32_t ph = 0;  // the ring's phase bits carry over from unit to unit
+
+  // Every CTA of a cluster walks the same units: blockIdx / C, then + stride.
+  // The default launch has one cluster per unit (one iteration); with
+  // SC_PERSISTENT the grid holds only the clusters that fit on the GPU at once,
+  // and each hints its next unit's first chunks into L2 when its pass 1 ends.
+#if SC_PERSISTENT
+  for (int unit = static_cast<int>(blockIdx.x) / C, it = 0; unit < P.units; unit += stride, ++it) {
+#else
+  {
+    const int unit = static_cast<int>(blockIdx.x) / C, it = 0;
+#endif
+  const int slot = it & 1;  // exchange-1 slot set of this unit
+  int b, j;
+  unit_coords(P, unit, b, j);
+  const int v0 = rank * P.L;
+  const Ring<E> R = make_ring<E>(P, smem_raw, b, j, rank);
+  const bool pair = R.pair;
+
+  // ---- start the stream; prefetch the row's scalars
+  if (tid == 0) {
+    sh.xq = NAN;
+    sh.xp = NAN;
+    // a previous unit's draw wrote ring memory with ordinary stores (its chunk
+    // prefixes); order them before this unit's copies into the same stages
+    if (it > 0 && P.bulk) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
   prime(R, sh);
   float uj = 0.0f, ug = 0.0f;
   int x = -1;
@@ -1242,7 +1271,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     if (pair) x = P.tokens[static_cast<size_t>(b) * P.gamma + j];
   }
   __syncthreads();
-  cluster_arrive_relaxed();  // this CTA has started (peers may store into it after their wait)
+  if (it == 0) cluster_arrive_relaxed();  // this CTA has started (peers may store into it after their wait)
 
   // ---- pass 1: online max and sum of exponentials
   const float k = P.k;
@@ -1296,6 +1325,14 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       sh.xp = Elt<E>::at(R.p(s), lx - c * kCH);
     }
   });
+  if (SC_PERSISTENT && tid == 0 && P.bulk && unit + stride < P.units) {
+    // the next unit's first chunks stream into L2 while this one is exchanged,
+    // decided and reported; its pass 1 then finds them there
+    int bn, jn;
+    unit_coords(P, unit + stride, bn, jn);
+    const Ring<E> Rn = make_ring<E>(P, smem_raw, bn, jn, rank);
+    for (int c = 0; c < min(kStages, Rn.nch); ++c) Rn.prefetch(c);
+  }
   if constexpr (kExt) {
     if (bonus_tot) {
       ex.mp = mp;
@@ -1338,21 +1375,21 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     } else {
       part = merge_partials(sh.red, kNW, k);
     }
-    if (tmo) {
+    if (tmo || sh.timeout) {  // (a copy of an earlier unit that never landed may land now)
       part.y = NAN;
       part.w = NAN;
       flag_timeout(sh, P);
     }
   }
-  cluster_wait();  // every CTA of the cluster has started
+  if (it == 0) cluster_wait();  // every CTA of the cluster has started
   if (tid == 0) {
     const float2 xv = make_float2(sh.xq, sh.xp);
     for (int r = 0; r < C; ++r) {
-      st_peer(peer_addr(&sh.all_ms[rank], r), part);
-      st_peer(peer_addr(&sh.all_x[rank], r), xv);
+      st_peer(peer_addr(&sh.all_ms[slot][rank], r), part);
+      st_peer(peer_addr(&sh.all_x[slot][rank], r), xv);
       if constexpr (kExt) {
-        st_peer(peer_addr(&sh.all_ext[rank], r), part_ext);
-        st_peer(peer_addr(&sh.all_idx[rank], r), part_idx);
+        st_peer(peer_addr(&sh.all_ext[slot][rank], r), part_ext);
+        st_peer(peer_addr(&sh.all_idx[slot][rank], r), part_idx);
       }
     }
   }
@@ -1364,14 +1401,15 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     ExtState g = ext_empty();
     float4 v;
     if constexpr (kExt) {
-      g = ext_load(sh.all_ms[0], sh.all_ext[0], sh.all_idx[0]);
-      for (int r = 1; r < C; ++r) ext_merge(g, ext_load(sh.all_ms[r], sh.all_ext[r], sh.all_idx[r]), k);
+      g = ext_load(sh.all_ms[slot][0], sh.all_ext[slot][0], sh.all_idx[slot][0]);
+      for (int r = 1; r < C; ++r)
+        ext_merge(g, ext_load(sh.all_ms[slot][r], sh.all_ext[slot][r], sh.all_idx[slot][r]), k);
       v = make_float4(g.mq, g.sq, g.mp, g.sp);
     } else {
-      v = merge_partials(sh.all_ms, C, k);
+      v = merge_partials(sh.all_ms[slot], C, k);
     }
     const float a = v.x, as = v.y, c = v.z, cs = v.w;
-    const float2 xv = sh.all_x[(x >= 0 && x < P.V) ? x / P.L : 0];
+    const float2 xv = sh.all_x[slot][(x >= 0 && x < P.V) ? x / P.L : 0];
     const float yqx = xv.x, ypx = xv.y;
     // S = sum_v 2^{y_v k - R} with R = fl(M k); the max logit's own term is
     // 2^{fma(M, k, -R)}, so max_v q(v) = 2^{fma(M, k, -R)} / S.
@@ -1950,7 +1988,8 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       }
     }
   }
-  if (sh.timeout && tid == 0 && R.bulk) {
+  }  // units
+  if (sh.timeout && tid == 0 && P.bulk) {
     // let copies still in flight land before this CTA's shared memory is released
     for (int s = 0; s < kStages; ++s) mbar_wait(&sh.full[s], 0), mbar_wait(&sh.full[s], 1);
   }
@@ -1963,6 +2002,7 @@ struct DeviceInfo {
   int smem_optin = 0;
   int sms = 0;
   bool configured[6] = {};  // [dtype][rule family]
+  int max_clusters[6][kMaxCluster + 1] = {};  // co-resident clusters per [kernel][C] (-1: unknown)
 };
 
 DeviceInfo g_dev[64];
@@ -2094,10 +2134,11 @@ int launch(Params P, cudaStream_t stream, int units) {
   const size_t row_bytes = static_cast<size_t>(P.V) * sizeof(E);
   P.bulk = (row_bytes % 16 == 0) && (reinterpret_cast<uintptr_t>(P.draft) % 16 == 0) &&
            (reinterpret_cast<uintptr_t>(P.target) % 16 == 0);
+  P.units = units;
   if (units == 0) return SC_OK;
 
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(static_cast<unsigned>(units) * static_cast<unsigned>(C), 1, 1);
+  cfg.gridDim = dim3(static_cast<unsigned>(C), 1, 1);
   cfg.blockDim = dim3(kNT, 1, 1);
   cfg.dynamicSmemBytes = smem_bytes<E>();
   cfg.stream = stream;
@@ -2108,6 +2149,21 @@ int launch(Params P, cudaStream_t stream, int units) {
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
+  // one cluster per unit, or (SC_PERSISTENT) as many as fit on the GPU at once,
+  // each looping over its share of the units; the kernel is correct for any grid
+  // since no cluster waits on another
+  int clusters = units;
+  if (SC_PERSISTENT) {
+    std::lock_guard<std::mutex> lock(g_mu);
+    int &mc = di.max_clusters[ti][C];
+    if (mc == 0) {
+      int n = 0;
+      mc = cudaOccupancyMaxActiveClusters(&n, kernel, &cfg) == cudaSuccess && n > 0 ? n : -1;
+      cudaGetLastError();
+    }
+    if (mc > 0 && mc < units) clusters = mc;
+  }
+  cfg.gridDim = dim3(static_cast<unsigned>(clusters) * static_cast<unsigned>(C), 1, 1);
   if (cudaLaunchKernelEx(&cfg, kernel, P) != cudaSuccess) return SC_ERR_CUDA;
   return SC_OK;
 }
