@@ -38,6 +38,8 @@ evaluating a softmax.
 
 from __future__ import annotations
 
+import os
+from concurrent.futures import ThreadPoolExecutor
 from dataclasses import dataclass, field
 from typing import Optional
 
@@ -117,13 +119,37 @@ class Workload:
 
 # ---------------------------------------------------------------- bit helpers
 
+def _row_blocks(n_rows: int, row_len: int, fn) -> None:
+    """fn(i0, i1) over blocks of rows, on a thread pool when the work is large
+    (numpy releases the GIL inside its element-wise loops, and each element's
+    result does not depend on how the rows are split)."""
+    per = max(1, (1 << 18) // max(1, row_len))  # ~256K elements per task
+    blocks = [(i, min(n_rows, i + per)) for i in range(0, n_rows, per)]
+    if len(blocks) < 2 or n_rows * row_len < (1 << 20):
+        for i0, i1 in blocks:
+            fn(i0, i1)
+        return
+    with ThreadPoolExecutor(max_workers=min(len(blocks), os.cpu_count() or 1)) as ex:
+        list(ex.map(lambda bl: fn(*bl), blocks))
+
+
 def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
     """Round float32 to bf16 (nearest, ties to even); returns uint16 bits.
 
     Inputs must be finite (the generators only make finite values)."""
-    b = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32)
-    b = b + (np.uint32(0x7FFF) + ((b >> np.uint32(16)) & np.uint32(1)))
-    return (b >> np.uint32(16)).astype(np.uint16)
+    src = np.ascontiguousarray(x, dtype=np.float32)
+    out = np.empty(src.shape, dtype=np.uint16)
+    n = src.shape[-1] if src.ndim else 1
+    b2 = src.reshape(-1, n).view(np.uint32)
+    o2 = out.reshape(-1, n)
+
+    def work(i0, i1):
+        b = b2[i0:i1]
+        b = b + (np.uint32(0x7FFF) + ((b >> np.uint32(16)) & np.uint32(1)))
+        o2[i0:i1] = b >> np.uint32(16)
+
+    _row_blocks(b2.shape[0], n, work)
+    return out
 
 
 def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
@@ -151,9 +177,23 @@ def gumbel_argmax(rng: np.random.Generator, y: np.ndarray, temperature: float) -
     u = rng.random(size=y.shape)
     if temperature == 0:
         return np.argmax(y, axis=-1).astype(np.int32)
-    # u in [0, 1): keep the logs finite.
-    g = -np.log(-np.log(np.maximum(u, 1e-300)))
-    return np.argmax(y / temperature + g, axis=-1).astype(np.int32)
+    n = y.shape[-1]
+    y2, u2 = y.reshape(-1, n), u.reshape(-1, n)
+    out = np.empty(y2.shape[0], dtype=np.int32)
+
+    def work(i0, i1):
+        # g = -log(-log(u)), u in [0, 1) kept off 0 so that the logs stay finite
+        g = np.maximum(u2[i0:i1], 1e-300)
+        np.log(g, out=g)
+        np.negative(g, out=g)
+        np.log(g, out=g)
+        np.negative(g, out=g)
+        s = y2[i0:i1] / temperature
+        s += g
+        out[i0:i1] = np.argmax(s, axis=-1)
+
+    _row_blocks(y2.shape[0], n, work)
+    return out.reshape(y.shape[:-1])
 
 
 # ---------------------------------------------------------------- row draws
