@@ -21,6 +21,11 @@
  *    library allocates no device memory per call and never synchronises: work
  *    is queued on `stream` and results are valid once the stream reaches them.
  *  - Logits are row-major, contiguous, float32 or bf16 (raw 16-bit patterns).
+ *  - CUDA graphs: a call may be captured into a graph (stream capture) once one
+ *    call outside capture has run on the device with the same logit type and rule
+ *    family (it configures the kernel); during capture the pointer arguments are
+ *    only checked for NULL.  A replay reuses the captured workspace, which every
+ *    call leaves ready for the next.
  *  - Synchronous argument errors return a negative sc_status and queue no work.
  *    Data errors found on the device never trap: they set bits in the optional
  *    `device_status` word (see SC_DEV_*) and the affected sequence receives the

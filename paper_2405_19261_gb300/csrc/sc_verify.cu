@@ -2077,8 +2077,23 @@ void set_k(Params &P, float temperature) {
   P.kl = static_cast<float>(kd - static_cast<double>(P.k));
 }
 
+// Set by each entry point: its stream is being captured into a CUDA graph.  The
+// pointer checks then only reject null pointers, so that nothing but the launch
+// itself happens inside the capture sequence.
+thread_local bool t_capturing = false;
+
+bool capturing(cudaStream_t stream) {
+  cudaStreamCaptureStatus st = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(stream, &st) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return st != cudaStreamCaptureStatusNone;
+}
+
 bool device_accessible(const void *p) {
   if (!p) return false;
+  if (t_capturing) return true;
   cudaPointerAttributes a;
   if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
     cudaGetLastError();
@@ -2250,6 +2265,7 @@ int sc_verify_ex(const void *draft_logits, const void *target_logits, sc_dtype d
                  sc_rule rule, float alpha, float beta, float temperature, int32_t *num_accepted,
                  int32_t *next_token, void *workspace, size_t workspace_bytes,
                  int32_t *device_status, float *row_info, cudaStream_t stream) {
+  t_capturing = capturing(stream);
   int rc = common_checks(draft_logits, target_logits, dtype, B, gamma, V, temperature, true);
   if (rc != SC_OK) return rc;
   const int ri = static_cast<int>(rule);
@@ -2334,6 +2350,7 @@ int sc_verify(const void *draft_logits, const void *target_logits, sc_dtype dtyp
 int sc_row_stats(const void *draft_logits, const void *target_logits, sc_dtype dtype, int B,
                  int gamma, int V, float temperature, float *max_q, float *max_p, float *tv,
                  cudaStream_t stream) {
+  t_capturing = capturing(stream);
   int rc = common_checks(draft_logits, target_logits, dtype, B, gamma, V, temperature, false);
   if (rc != SC_OK) return rc;
   if (!device_accessible(max_q) || !device_accessible(max_p) || !device_accessible(tv))
