@@ -976,6 +976,10 @@ struct Ring {
   // thread 0, bulk mode: hint chunk c into L2
   __device__ void prefetch(int c) const {
     const uint32_t bytes = static_cast<uint32_t>(chunk_len(c)) * sizeof(E);
+    if (!SC_CHECK(c >= 0 && c < nch && bytes > 0 && bytes % 16 == 0 &&
+                  reinterpret_cast<uintptr_t>(gp + static_cast<size_t>(c) * kCH) % 16 == 0 &&
+                  (!pair || reinterpret_cast<uintptr_t>(gq + static_cast<size_t>(c) * kCH) % 16 == 0)))
+      return;
     if (pair) prefetch_l2(gq + static_cast<size_t>(c) * kCH, bytes);
     prefetch_l2(gp + static_cast<size_t>(c) * kCH, bytes);
   }
