@@ -88,3 +88,21 @@ int use_sc(const void *q, const void *p, const int32_t *x, const float *u, int32
     r = subprocess.run([gcc, "-std=c11", "-Wall", "-Wextra", "-Werror", "-fsyntax-only", "-I",
                         os.path.join(ROOT, "include"), "-I", cuda_inc, str(src)], capture_output=True, text=True)
     assert r.returncode == 0, r.stderr
+
+
+def test_binding_constants_mirror_the_header():
+    # the Python binding passes rule codes, reads row_info fields and decodes
+    # device_status bits by number: each must be the header's value
+    from paper_2405_19261_gb300 import binding
+    text = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    enum = dict((k, int(v)) for k, v in re.findall(r"\b(SC_RULE_[A-Z0-9_]+)\s*=\s*(\d+)", text))
+    assert enum, "no sc_rule values found"
+    by_name = {"SC_RULE_" + ("ALWAYS_DEFER" if n == "always" else "NEVER_DEFER" if n == "never" else n.upper()): c
+               for n, c in binding.RULES.items()}
+    assert by_name == enum
+    defines = dict((k, int(v)) for k, v in re.findall(r"#define\s+(SC_(?:ROW|DEV)_[A-Z_]+)\s+(\d+)u?", text))
+    assert binding.ROW_FIELDS == defines["SC_ROW_FIELDS"]
+    for name, idx in binding.ROW.items():
+        assert idx == defines["SC_ROW_" + name.upper()], name
+    assert (binding.DEV_BAD_TOKEN, binding.DEV_BAD_LOGIT, binding.DEV_BAD_UNIFORM, binding.DEV_TIMEOUT) == (
+        defines["SC_DEV_BAD_TOKEN"], defines["SC_DEV_BAD_LOGIT"], defines["SC_DEV_BAD_UNIFORM"], defines["SC_DEV_TIMEOUT"])
