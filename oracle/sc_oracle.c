@@ -34,6 +34,8 @@
  *       Lossy speculative decoding:  pi(v) = max{ min{ q(v), p(v)/(1 - alpha) }, p(v)/beta }
  *          (Lemma 2: the acceptance is min(1, p(x)/((1 - alpha) q(x))) and the residual
  *          norm(max(0, p/beta - q)); pi need not sum to one), beta >= 1 - alpha;
+ *          alpha = 1 is the limit alpha -> 1-: p(v)/(1 - alpha) is +infinity where
+ *          p(v) > 0 and 0 where p(v) = 0, so a draft with p(x) = 0 is still rejected;
  *       BiLD*:  delta = 1(D(q, p) > alpha), D(q, p) = -sum_v q(v) log p(v) (the
  *          temperature-sampling discrepancy of the experiments' appendix; with
  *          greedy decoding the appendix's -log p(argmax q)),
@@ -317,7 +319,7 @@ static int argmax_of(const double *x, int V)
 /* The lossy speculative-decoding target of one token (Table 3). */
 static double lossy_pi(double qv, double pv, double alpha, double beta)
 {
-    double a = alpha < 1.0 ? pv / (1.0 - alpha) : INFINITY;
+    double a = alpha < 1.0 ? pv / (1.0 - alpha) : (pv > 0.0 ? INFINITY : 0.0);  /* alpha -> 1- */
     double m = qv < a ? qv : a;
     double b = pv / beta;
     return m > b ? m : b;
@@ -454,7 +456,7 @@ static void verify_sequence(const void *draft, const void *target, int dtype,
                 double lp = log_prob(target, dtype, tbase + (size_t)j * V, x[j], Tr, Mp, lnSp);
                 if (lq > -INFINITY) {
                     double pq = exp(lp - lq);
-                    double a = alpha < 1.0 ? pq / (1.0 - alpha) : INFINITY;
+                    double a = alpha < 1.0 ? pq / (1.0 - alpha) : (pq > 0.0 ? INFINITY : 0.0);
                     double ratio = a < 1.0 ? a : 1.0;
                     if (pq / beta > ratio) ratio = pq / beta;
                     if (ratio < 1.0) {

@@ -721,3 +721,22 @@ def test_greedy_opt_equals_greedy_diff(alpha):
     np.testing.assert_array_equal(a.num_accepted, d.num_accepted)
     np.testing.assert_array_equal(a.next_token, d.next_token)
     assert np.all(a.status == 0)
+
+
+def test_lossy_at_alpha_1_is_the_limit_of_alpha_below_1():
+    """Table 3 / Lemma 2 at alpha = 1, read as the limit alpha -> 1-: the acceptance
+    min(1, p(x)/((1 - alpha) q(x))) tends to 1 where p(x) > 0 and stays 0 where
+    p(x) = 0 (a masked target logit), so the oracle at alpha = 1 decides as it does
+    at alpha = 1 - 1e-12 and rejects exactly the drafts whose target logit is masked."""
+    w = synthetic(12, 4, 300, dtype="f32", kind="gauss", sigma=1.0, rule="lossy", alpha=1.0, seed=81)
+    for b in range(0, 12, 2):          # mask the target logit of one draft token per even sequence
+        j = b % 4
+        w.target[b, j, w.tokens[b, j]] = -np.inf
+    one = oracle.verify_workload(w, alpha=1.0)
+    near = oracle.verify_workload(w, alpha=1.0 - 1e-12)
+    np.testing.assert_array_equal(one.num_accepted, near.num_accepted)
+    np.testing.assert_array_equal(one.next_token, near.next_token)
+    np.testing.assert_array_equal(one.row("accept"), near.row("accept"))
+    for b in range(12):
+        first_masked = b % 4 if b % 2 == 0 else w.gamma
+        assert one.num_accepted[b] == first_masked, b
