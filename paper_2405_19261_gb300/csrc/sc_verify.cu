@@ -931,7 +931,7 @@ __device__ __forceinline__ void accept_test(Shared &sh, const Params &P, int x, 
           const float2 t = two_sum(L.x, P.lossy_l);
           L = df_norm(t.x, __fadd_rn(__fadd_rn(t.y, L.y), P.lossy_ll));
         } else {
-          L = make_float2(0.0f, 0.0f);  // alpha = 1: the ratio is 1
+          L = make_float2(0.0f, 0.0f);  // alpha = 1 and p(x) > 0 here: the ratio is 1
         }
       }
       if (df_lt(L, 0.0f)) accept = u < df_exp2(L);
@@ -943,7 +943,8 @@ __device__ __forceinline__ void accept_test(Shared &sh, const Params &P, int x, 
     const float px = prob_of(ypx, sh.Rp, sh.Sp, k, kl);
     sh.qx = qx;
     if (kTok && sh.tok) sh.pix = fmaf(sh.eta, px, sh.delta ? 0.0f : qx);
-    else if (lossy) sh.pix = fmaxf(fminf(qx, P.alpha < 1.0f ? px / (1.0f - P.alpha) : INFINITY), px / P.beta);
+    else if (lossy)  // (alpha = 1: the limit alpha -> 1-, p / (1 - alpha) = +inf where p > 0, 0 where p = 0)
+      sh.pix = fmaxf(fminf(qx, P.alpha < 1.0f ? px / (1.0f - P.alpha) : (px > 0.0f ? INFINITY : 0.0f)), px / P.beta);
     else sh.pix = sh.delta ? px : qx;
   }
 }

@@ -193,10 +193,13 @@ def test_degenerate_rows(sc):
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
-@pytest.mark.parametrize("rule,alpha", [("always", 0.0), ("opt", 0.2), ("token_v3", 0.3), ("token_v1", 0.1)])
+@pytest.mark.parametrize("rule,alpha", [("always", 0.0), ("opt", 0.2), ("token_v3", 0.3), ("token_v1", 0.1),
+                                        ("lossy", 0.3), ("lossy", 1.0)])
 def test_masked_target_logit_at_the_draft_token(sc, dtype, rule, alpha):
     # p(x) = 0 < q(x): pi(x)/q(x) = 1 - delta, so a deferred draft is rejected whatever
-    # its uniform; with both logits masked q(x) = 0 and the draft is accepted
+    # its uniform (lossy speculative decoding too, alpha = 1 being the limit
+    # alpha -> 1- of min(1, p/((1 - alpha) q)) = 0); with both logits masked q(x) = 0
+    # and the draft is accepted
     B, g, V = 8, 3, 600
     w = synthetic(B, g, V, dtype=dtype, kind="gauss", sigma=1.0, rule=rule, alpha=alpha, seed=41)
     ninf = np.uint16(0xFF80) if dtype == "bf16" else np.float32(-np.inf)
@@ -207,7 +210,7 @@ def test_masked_target_logit_at_the_draft_token(sc, dtype, rule, alpha):
     w.draft[1, 0, w.tokens[1, 0]] = ninf
     w.target[1, 0, w.tokens[1, 0]] = ninf
     ref = oracle.verify_workload(w)
-    if rule == "always":
+    if rule in ("always", "lossy"):
         assert np.all(ref.num_accepted[0::2] == 0)
     assert_parity(w, run_gpu(sc, w), ref)
 
