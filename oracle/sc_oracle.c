@@ -327,19 +327,22 @@ static double lossy_pi(double qv, double pv, double alpha, double beta)
 
 /*
  * BiLD*'s discrepancy D(q, p) = -sum_v q(v) log p(v) of one row pair, with
- * log p(v) from the logits (+infinity when some q(v) > 0 has p(v) = 0).
+ * log p(v) from the logits.  It is +infinity when some q(v) > 0 has p(v) = 0:
+ * q(v) > 0 exactly when the draft logit is finite (whether or not exp of it
+ * underflows in fp64), p(v) = 0 exactly when the target logit is -infinity.
  */
-static double cross_entropy(const double *q, const void *zp, int dtype, size_t poff, int V, double T,
-                            double Mp, double lnSp)
+static double cross_entropy(const double *q, const void *zq, size_t qoff, const void *zp, int dtype,
+                            size_t poff, int V, double T, double Mp, double lnSp)
 {
     csum D = {0.0, 0.0};
     for (int v = 0; v < V; ++v) {
-        if (!(q[v] > 0.0))
-            continue;
+        if (!(logit_at(zq, dtype, qoff + (size_t)v) > -INFINITY))
+            continue;  /* q(v) = 0 */
         const double lp = log_prob(zp, dtype, poff, v, T, Mp, lnSp);
         if (lp == -INFINITY)
             return INFINITY;
-        csum_add(&D, -q[v] * lp);
+        if (q[v] > 0.0)
+            csum_add(&D, -q[v] * lp);
     }
     return csum_value(&D);
 }
@@ -478,7 +481,8 @@ static void verify_sequence(const void *draft, const void *target, int dtype,
             /* greedy decoding: the BiLD baseline's D(q, p) = -log p(argmax q); with a
                temperature, its analogue -sum_v q(v) log p(v) */
             const double D = greedy ? -log_prob(target, dtype, tbase + (size_t)j * V, argmax_of(q, V), Tr, Mp, lnSp)
-                                    : cross_entropy(q, target, dtype, tbase + (size_t)j * V, V, Tr, Mp, lnSp);
+                                    : cross_entropy(q, draft, dbase + (size_t)j * V, target, dtype,
+                                                    tbase + (size_t)j * V, V, Tr, Mp, lnSp);
             delta = D > alpha;  /* strict, as printed */
             m_delta = isfinite(D) ? fabs(D - alpha) : INFINITY;
         } else {

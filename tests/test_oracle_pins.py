@@ -740,3 +740,25 @@ def test_lossy_at_alpha_1_is_the_limit_of_alpha_below_1():
     for b in range(12):
         first_masked = b % 4 if b % 2 == 0 else w.gamma
         assert one.num_accepted[b] == first_masked, b
+
+
+@pytest.mark.parametrize("gap", [50.0, 2000.0])
+def test_bild_discrepancy_is_infinite_where_p_is_zero_and_q_is_not(gap):
+    """D(q, p) = -sum_v q(v) log p(v) is +infinity as soon as one token has q(v) > 0
+    and p(v) = 0: any finite draft logit gives q(v) > 0, a -inf target logit p(v) = 0.
+    Here that token's draft logit lies `gap` below the row's largest, so q(v) is
+    tiny (50) or below fp64's range (2000, exp(-2000) = 0): BiLD* defers
+    (delta = 1) for any alpha either way, and does not where the masked target
+    token's draft logit is masked too."""
+    V, g = 5, 1
+    q = np.array([[0.0, 1.0, -0.5, -gap, 0.3]], dtype=np.float32)
+    p = np.array([[0.2, 0.9, -0.1, -np.inf, 0.0], [0.1, 0.2, 0.3, 0.4, 0.5]], dtype=np.float32)
+    for alpha in (0.5, 50.0, 1e6):
+        w = rows_workload(np.exp(q.astype(np.float64)), np.exp(p.astype(np.float64)), [1], [0.5, 0.5], "bild", alpha)
+        w.draft[0] = q
+        w.target[0] = p
+        r = oracle.verify_workload(w)
+        assert r.row("delta")[0, 0] == 1, (gap, alpha)
+        w.draft[0, 0, 3] = -np.inf   # now q(3) = 0 too: D is finite, about 1.4 nats
+        r = oracle.verify_workload(w)
+        assert r.row("delta")[0, 0] == (1 if alpha < 1.0 else 0), (gap, alpha)
