@@ -489,7 +489,7 @@ __device__ __forceinline__ ExtState ext_empty() {
 // X' = 2^{dq} (X + dp S_q).  (A reference floored at -1e30 comes with S = 0.)
 __device__ __forceinline__ void ext_rebase(ExtState &e, float dq, float dp) {
   const float fq = ex2(dq), fp = ex2(dp);
-  e.x = fq * fmaf(dp, e.sq, e.x);
+  e.x = e.x == -INFINITY ? e.x : fq * fmaf(dp, e.sq, e.x);  // (-inf: D(q, p) = +inf, kept)
   e.aq = fq * fmaf(dq, e.sq, e.aq);
   e.sq = fq * e.sq;
   e.ap = fp * fmaf(dp, e.sp, e.ap);
@@ -606,7 +606,9 @@ __device__ __forceinline__ void ext_chunk(const E *srcq, const E *srcp, int n, i
         const float ea = ex2(a);
         sq += ea;
         aq += ea > 0.0f ? ea * a : 0.0f;
-        x += ea > 0.0f ? ea * b : 0.0f;
+        // a finite draft logit with a masked target logit (q(v) > 0 = p(v)) makes
+        // D(q, p) = +inf even where 2^a underflows: X = -inf, kept by every merge
+        x += yq[i] > -INFINITY && !(yp[i] > -INFINITY) ? -INFINITY : (ea > 0.0f ? ea * b : 0.0f);
         if (with_bc) h += ex2(0.5f * (a + b));  // sqrt(q p) up to the normalisers
       }
     }

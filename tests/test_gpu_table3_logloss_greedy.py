@@ -303,3 +303,27 @@ def test_greedy_and_lossy_argument_checks(sc):
                                  (13, 0.1, 1.0, 1.0)]:
         with pytest.raises(sc.SCError):
             sc.sc_verify(d, t, x, u, rule, alpha, T, beta=beta)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_bild_infinite_discrepancy_on_a_masked_target_token(sc, dtype):
+    # D(q, p) = -sum_v q log p is +inf when some token has a finite draft logit
+    # (q(v) > 0) and a masked target logit (p(v) = 0), however far below the
+    # draft's largest logit it lies: 200 nats (2^a underflows in f32) or 2000 (exp
+    # underflows in fp64).  Such a pair defers (delta = 1) whatever alpha is.
+    from paper_2405_19261_gb300.workloads import f32_to_bf16_bits
+    B, g, V = 6, 3, 4099
+    w = synthetic(B, g, V, dtype=dtype, kind="gauss", sigma=1.0, rule="bild", alpha=1e6, seed=77)
+    dq = logits_as_f64(w.draft, dtype)
+
+    def put(arr, idx, val):
+        arr[idx] = f32_to_bf16_bits(np.float32(val))[0] if dtype == "bf16" else np.float32(val)
+
+    for b in range(B):
+        j, v = b % g, (4097 if b % 2 else 11)   # in the ragged last chunk, or the first
+        put(w.draft, (b, j, v), dq[b, j].max() - (200.0 if b < 3 else 2000.0))
+        put(w.target, (b, j, v), -np.inf)
+    ref = oracle.verify_workload(w)
+    for b in range(B):
+        assert ref.row("delta")[b, b % g] == 1, b
+    assert_parity(w, run_gpu(sc, w), ref)
