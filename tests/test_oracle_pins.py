@@ -762,3 +762,17 @@ def test_bild_discrepancy_is_infinite_where_p_is_zero_and_q_is_not(gap):
         w.draft[0, 0, 3] = -np.inf   # now q(3) = 0 too: D is finite, about 1.4 nats
         r = oracle.verify_workload(w)
         assert r.row("delta")[0, 0] == (1 if alpha < 1.0 else 0), (gap, alpha)
+
+
+def test_lossy_rejection_with_an_empty_residual():
+    """Lemma 2 with beta > 1: q = (1/2, 1/2), p = (0, 1), alpha = 0, beta = 2 give
+    pi = max{min{q, p}, p/2} = (0, 1/2), so the draft x = 0 is rejected (pi/q = 0),
+    while max(0, p/beta - q) = (0, 0) leaves no token to draw: next_token is -1,
+    num_accepted 0, and the sequence is flagged (no draw to compare)."""
+    w = rows_workload([[0.5, 0.5]], [[0.0, 1.0], [0.5, 0.5]], [0], [0.3, 0.7], "lossy", 0.0)
+    r = oracle.verify_workload(w, beta=2.0)
+    assert (r.num_accepted[0], r.next_token[0]) == (0, -1)
+    assert r.flagged[0]
+    # beta = 1: the residual is norm(max(0, p - q)) = (0, 1), token 1
+    r1 = oracle.verify_workload(w, beta=1.0)
+    assert (r1.num_accepted[0], r1.next_token[0]) == (0, 1) and not r1.flagged[0]
