@@ -65,7 +65,10 @@ typedef enum {
   SC_RULE_LOSSY = 8,        /* lossy speculative decoding: pi = max{min{q, p/(1 - alpha)}, p/beta}
                              * (pi need not sum to one; Lemma 2: the acceptance ratio is
                              * min(1, p(x)/((1 - alpha) q(x))), the residual norm(max(0, p/beta - q)));
-                             * beta >= 1 - alpha, 1 for sc_verify and sc_verify_rows */
+                             * beta >= 1 - alpha, 1 for sc_verify and sc_verify_rows; with
+                             * beta > 1 a rejection can leave the residual empty (p/beta <= q
+                             * everywhere): no token is defined, next_token = -1 and
+                             * num_accepted = j*, with no status bit */
   SC_RULE_BILD = 9,         /* BiLD*: delta = [D(q, p) > alpha], D(q, p) = -sum_v q(v) ln p(v) */
   /* Plug-in rules for the log loss (the paper's appendix on log loss), with
    * sum_v q ln q the negative entropy: */
