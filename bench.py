@@ -57,6 +57,8 @@ def parse():
     ap.add_argument("--gamma", type=int, default=None)
     ap.add_argument("--rule", default=None)
     ap.add_argument("--alpha", type=float, default=None)
+    ap.add_argument("--beta", type=float, default=1.0, help="lossy speculative decoding's beta")
+    ap.add_argument("--temperature", type=float, default=None, help="config 4 only; 0 = greedy decoding")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--record-traffic", metavar="NCU_CSV", default=None,
@@ -299,10 +301,13 @@ def workload_from(args, rank=0):
     if args.config == 4:
         kw["B"] = args.B or 64
         kw["gamma"] = args.gamma or 4
+        kw["temperature"] = args.temperature
     w = config(args.config, **kw)
+    w.beta = args.beta
     desc = CONFIG_TEXT[args.config]
     if args.config == 4:
-        desc = f"B={w.B} gamma={w.gamma} V=256000 bf16, zipf sigma=0.7, T=1, {w.rule} a={w.alpha}"
+        desc = (f"B={w.B} gamma={w.gamma} V=256000 bf16, zipf sigma=0.7, T={w.temperature:g}, "
+                f"{w.rule} a={w.alpha}" + (f" beta={w.beta:g}" if w.rule == "lossy" else ""))
     return w, f"cfg{args.config}: {desc}"
 
 
@@ -351,7 +356,7 @@ def run_ours(args):
     stream = torch.cuda.current_stream(dev)
 
     def step():
-        binding.sc_verify(d, t, x, u, w.rule, w.alpha, w.temperature, num_accepted=na,
+        binding.sc_verify(d, t, x, u, w.rule, w.alpha, w.temperature, beta=w.beta, num_accepted=na,
                           next_token=nt, workspace=ws, stream=stream)
 
     l2 = torch.cuda.get_device_properties(dev).L2_cache_size

@@ -21,12 +21,20 @@
  *    library allocates no device memory per call and never synchronises: work
  *    is queued on `stream` and results are valid once the stream reaches them.
  *  - Logits are row-major, contiguous, float32 or bf16 (raw 16-bit patterns).
+ *  - CUDA graphs: a call may be captured into a graph (stream capture) once one
+ *    call outside capture has run on the device with the same logit type and rule
+ *    family (it configures the kernel); during capture the pointer arguments are
+ *    only checked for NULL.  A replay reuses the captured workspace, which every
+ *    call leaves ready for the next.
  *  - Synchronous argument errors return a negative sc_status and queue no work.
  *    Data errors found on the device never trap: they set bits in the optional
  *    `device_status` word (see SC_DEV_*) and the affected sequence receives the
  *    defined outputs num_accepted = 0, next_token = -1.
  *  - Limits: B, gamma, V >= 1; gamma <= SC_MAX_GAMMA; V <= sc_max_vocab(dtype);
- *    0 < T < inf; 0 <= alpha <= 1 (the paper sweeps alpha over [0, 1]).
+ *    0 < T < inf, or T = 0 (greedy decoding) with a rule other than the token
+ *    rules and lossy speculative decoding; 0 <= alpha <= 1 (the paper sweeps
+ *    alpha over [0, 1]) for rules 0-8, 0 <= alpha < inf for rules 9-12 (a
+ *    threshold on an entropy or a cross entropy, in nats).
  */
 #ifndef SC_H_
 #define SC_H_
@@ -52,7 +60,21 @@ typedef enum {
    * r(v) in {0, 1}, eta = sum_v r(v) q(v) and pi(v) = q(v) (1 - r(v)) + eta p(v). */
   SC_RULE_TOKEN_V1 = 5,     /* r(v) = [q(v) < max p - alpha] */
   SC_RULE_TOKEN_V2 = 6,     /* r(v) = [p(v) < max p - alpha] */
-  SC_RULE_TOKEN_V3 = 7      /* r(v) = [p(v) < max p (1 - alpha)] */
+  SC_RULE_TOKEN_V3 = 7,     /* r(v) = [p(v) < max p (1 - alpha)] */
+  /* The other targets of Table 3, run through Algorithm 4 the same way. */
+  SC_RULE_LOSSY = 8,        /* lossy speculative decoding: pi = max{min{q, p/(1 - alpha)}, p/beta}
+                             * (pi need not sum to one; Lemma 2: the acceptance ratio is
+                             * min(1, p(x)/((1 - alpha) q(x))), the residual norm(max(0, p/beta - q)));
+                             * beta >= 1 - alpha, 1 for sc_verify and sc_verify_rows; with
+                             * beta > 1 a rejection can leave the residual empty (p/beta <= q
+                             * everywhere): no token is defined, next_token = -1 and
+                             * num_accepted = j*, with no status bit */
+  SC_RULE_BILD = 9,         /* BiLD*: delta = [D(q, p) > alpha], D(q, p) = -sum_v q(v) ln p(v) */
+  /* Plug-in rules for the log loss (the paper's appendix on log loss), with
+   * sum_v q ln q the negative entropy: */
+  SC_RULE_CHOW_LOG = 10,    /* H(q) > alpha */
+  SC_RULE_DIFF_LOG = 11,    /* sum q ln q < sum p ln p - alpha */
+  SC_RULE_OPT_LOG = 12      /* sum q ln q < sum p ln p - alpha D_TV(p, q) */
 } sc_rule;
 
 typedef enum {
@@ -75,7 +97,9 @@ typedef enum {
 /* Layout overrides, read from the environment at every call and meant for
  * measurements (the default layout is chosen from V, the batch and the SM count):
  *   SC_SLICE=n    logits per CTA slice of a row (n >= 64, rounded to a multiple of 8)
- *   SC_CLUSTER=c  CTAs per row pair (1 <= c <= 16; raised if the slices would not fit) */
+ *   SC_CLUSTER=c  CTAs per row pair (1 <= c <= 16; raised if the slices would not fit)
+ *   SC_SPEC_RES=0|1  whether rejected pairs store their own residual prefixes (default 1)
+ *                 or leave them to the owners' sampling passes */
 
 /* Per-position diagnostics written by sc_verify_rows, [B][gamma+1][SC_ROW_FIELDS]
  * float32.  Position gamma (the bonus position) fills only MAXP and CAND. */
@@ -110,8 +134,15 @@ int sc_max_vocab(sc_dtype dtype);
  *   uniforms       [B][gamma+1] f32  u[b][j < gamma] is the Bernoulli draw of
  *                                    position j; u[b][gamma] is the single draw
  *                                    for the residual or bonus sample
- *   rule, alpha    deferral rule of Table 1 (or a token-specific rule) and its cost parameter
- *   temperature    T > 0; both q and p are softmax(logits / T)
+ *   rule, alpha    deferral rule of Table 1 (or another rule of sc_rule) and its parameter
+ *   temperature    T > 0: both q and p are softmax(logits / T).  T = 0 is greedy
+ *                  decoding: the rule reads max q, max p and the entropies of
+ *                  softmax(logits), and its D_TV is that of the one-hot q~, p~ at
+ *                  the rows' argmaxes (lowest index on ties), 1(argmax q != argmax p);
+ *                  pi = (1 - delta) q~ + delta p~, so a draft is rejected only when
+ *                  delta = 1 and it is not the target's argmax, and the emitted
+ *                  token at j* is the target's argmax (the uniforms are not read
+ *                  for sampling)
  *   num_accepted   [B] int32 out: j* in [0, gamma]
  *   next_token     [B] int32 out: the token emitted at position j*.  The
  *                  emitted tokens of sequence b are draft_tokens[b][0 .. j*-1]
@@ -135,6 +166,14 @@ int sc_verify_rows(const void *draft_logits, const void *target_logits, sc_dtype
                    int32_t *next_token, void *workspace, size_t workspace_bytes,
                    int32_t *device_status, float *row_info, cudaStream_t stream);
 
+/* sc_verify_rows with lossy speculative decoding's beta (Table 3): beta > 0 and
+ * beta >= 1 - alpha when rule is SC_RULE_LOSSY, ignored otherwise. */
+int sc_verify_ex(const void *draft_logits, const void *target_logits, sc_dtype dtype,
+                 const int32_t *draft_tokens, const float *uniforms, int B, int gamma, int V,
+                 sc_rule rule, float alpha, float beta, float temperature, int32_t *num_accepted,
+                 int32_t *next_token, void *workspace, size_t workspace_bytes,
+                 int32_t *device_status, float *row_info, cudaStream_t stream);
+
 /*
  * sc_row_stats -- the per-position quantities the deferral rules of Table 1
  * read: max_v q_j(v), max_v p_j(v) and D_TV(p_j, q_j) (Lemma 3), for every pair
@@ -150,6 +189,13 @@ int sc_row_stats(const void *draft_logits, const void *target_logits, sc_dtype d
 /* Static description of an sc_status code. */
 const char *sc_status_string(int code);
 
+/* Builds with -DSC_DEBUG=1 check the kernel's computed indices, copy sizes and
+ * alignments, skip an access that fails (its outputs are then undefined; a skipped
+ * copy ends in SC_DEV_TIMEOUT) and record the kernel source line of the first
+ * failure.  Returns that line (0: none), clearing it when `reset` is nonzero,
+ * SC_ERR_CUDA if it cannot be read, and -1 in builds without the checks. */
+int sc_debug_line(int reset);
+
 /*
  * sc_verify_static -- sc_verify for callers that cannot allocate device memory.
  *
@@ -163,7 +209,7 @@ const char *sc_status_string(int code);
  * exit.
  *
  * Limits: B <= SC_STATIC_MAX_B and B * (gamma + 1) <= SC_STATIC_MAX_UNITS
- * (about 4.4 MiB of scratch); larger batches return SC_ERR_SCRATCH_LIMIT and queue no
+ * (about 10.8 MiB of scratch); larger batches return SC_ERR_SCRATCH_LIMIT and queue no
  * work.  Other arguments are those of sc_verify and are checked the same way.
  *
  * The first call on a device looks up the array's device address (the library's

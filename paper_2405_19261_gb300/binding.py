@@ -18,7 +18,8 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "_lib", "libspeccascade.so")
 
 RULES = {"chow": 0, "diff": 1, "opt": 2, "always": 3, "never": 4,
-         "token_v1": 5, "token_v2": 6, "token_v3": 7}
+         "token_v1": 5, "token_v2": 6, "token_v3": 7, "lossy": 8, "bild": 9,
+         "chow_log": 10, "diff_log": 11, "opt_log": 12}
 ROW_FIELDS = 8
 ROW = dict(maxq=0, maxp=1, tv=2, delta=3, accept=4, qx=5, pix=6, cand=7)
 DEV_BAD_TOKEN, DEV_BAD_LOGIT, DEV_BAD_UNIFORM, DEV_TIMEOUT = 1, 2, 4, 8
@@ -48,8 +49,12 @@ def lib():
         L.sc_verify.restype = I
         L.sc_verify_rows.argtypes = [P, P, I, P, P, I, I, I, I, F, F, P, P, P, S, P, P, P]
         L.sc_verify_rows.restype = I
+        L.sc_verify_ex.argtypes = [P, P, I, P, P, I, I, I, I, F, F, F, P, P, P, S, P, P, P]
+        L.sc_verify_ex.restype = I
         L.sc_row_stats.argtypes = [P, P, I, I, I, I, F, P, P, P, P]
         L.sc_row_stats.restype = I
+        L.sc_debug_line.argtypes = [I]
+        L.sc_debug_line.restype = I
         L.sc_status_string.argtypes = [I]
         L.sc_status_string.restype = ctypes.c_char_p
         _lib = L
@@ -96,12 +101,19 @@ def new_workspace(B: int, gamma: int, device=None) -> torch.Tensor:
     return torch.zeros(workspace_bytes(B, gamma), dtype=torch.uint8, device=device or "cuda")
 
 
+def debug_line(reset: bool = False) -> int:
+    """Kernel source line of the first failed device-side check (a library built
+    with SC_DEBUG; 0: none), or -1 for a library built without the checks."""
+    return int(lib().sc_debug_line(1 if reset else 0))
+
+
 def max_vocab(dtype: torch.dtype) -> int:
     return int(lib().sc_max_vocab(0 if dtype == torch.float32 else 1))
 
 
 def sc_verify(draft_logits: torch.Tensor, target_logits: torch.Tensor, draft_tokens: torch.Tensor,
               uniforms: torch.Tensor, rule, alpha: float, temperature: float, *,
+              beta: float = 1.0,
               num_accepted: Optional[torch.Tensor] = None, next_token: Optional[torch.Tensor] = None,
               workspace: Optional[torch.Tensor] = None, status: Optional[torch.Tensor] = None,
               row_info: Optional[torch.Tensor] = None, stream=None):
@@ -109,8 +121,10 @@ def sc_verify(draft_logits: torch.Tensor, target_logits: torch.Tensor, draft_tok
 
     draft_logits [B, gamma, V], target_logits [B, gamma+1, V] (float32 or
     bfloat16, same dtype), draft_tokens [B, gamma] int32, uniforms
-    [B, gamma+1] float32.  Outputs, workspace, status ([1] int32) and row_info
-    ([B, gamma+1, 8] float32) may be passed in to avoid allocations.
+    [B, gamma+1] float32.  ``beta`` is lossy speculative decoding's parameter
+    (rule "lossy"); temperature 0 is greedy decoding.  Outputs, workspace,
+    status ([1] int32) and row_info ([B, gamma+1, 8] float32) may be passed in
+    to avoid allocations.
     """
     _cuda(draft_logits, "draft_logits")
     _cuda(target_logits, "target_logits", draft_logits.dtype)
@@ -140,12 +154,12 @@ def sc_verify(draft_logits: torch.Tensor, target_logits: torch.Tensor, draft_tok
         if row_info.numel() < B * (gamma + 1) * ROW_FIELDS:
             raise ValueError("row_info too small")
     rule_code = RULES[rule] if isinstance(rule, str) else int(rule)
-    rc = lib().sc_verify_rows(_ptr(draft_logits), _ptr(target_logits), _dtype_code(draft_logits),
-                              _ptr(draft_tokens), _ptr(uniforms), B, gamma, V, rule_code,
-                              float(alpha), float(temperature), _ptr(num_accepted),
-                              _ptr(next_token), _ptr(workspace),
-                              workspace.numel() * workspace.element_size(), _ptr(status),
-                              _ptr(row_info), _stream(stream))
+    rc = lib().sc_verify_ex(_ptr(draft_logits), _ptr(target_logits), _dtype_code(draft_logits),
+                            _ptr(draft_tokens), _ptr(uniforms), B, gamma, V, rule_code,
+                            float(alpha), float(beta), float(temperature), _ptr(num_accepted),
+                            _ptr(next_token), _ptr(workspace),
+                            workspace.numel() * workspace.element_size(), _ptr(status),
+                            _ptr(row_info), _stream(stream))
     _check(rc, "sc_verify")
     return num_accepted, next_token
 

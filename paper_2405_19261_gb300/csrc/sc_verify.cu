@@ -69,6 +69,21 @@ namespace {
 #ifndef SC_MIN_BLOCKS
 #define SC_MIN_BLOCKS 6
 #endif
+#ifndef SC_DEBUG
+#define SC_DEBUG 0  // 1: check computed indices and copy sizes, skip and record a failing access
+#endif
+#ifndef SC_OPT_UB
+#define SC_OPT_UB 1  // OPT band rows: settle delta = 1 by the Bhattacharyya bound on D_TV
+#endif
+#ifndef SC_BONUS_LAST
+#define SC_BONUS_LAST 0  // 1: launch all pair units before the bonus rows
+#endif
+#ifndef SC_PERSISTENT
+#define SC_PERSISTENT 0  // 1: a grid of co-resident clusters loops over the units (see the kernel)
+#endif
+#ifndef SC_L2_PREFETCH
+#define SC_L2_PREFETCH 1  // second passes prefetch their slice into L2 before streaming it
+#endif
 
 constexpr int kNT = 128;                   // threads per CTA
 constexpr int kNW = kNT / 32;              // warps per CTA
@@ -88,6 +103,14 @@ constexpr int kMinBlocksPerSM = SC_MIN_BLOCKS;
 
 enum Mode : int { kVerify = 0, kStats = 1 };
 
+// The kernel is compiled once per rule family.  kFamCascade: the deferral
+// rules of Table 1 and lossy speculative decoding (Table 3); kFamToken: the
+// token-specific rules of Section 4.4, whose weight passes evaluate r(v) per
+// logit; kFamExt: the rules that read entropies or a cross entropy (BiLD*, the
+// log-loss rules) and greedy decoding (T = 0), whose pass 1 also accumulates
+// first moments of the exponents and the rows' argmaxes.
+enum Family : int { kFamCascade = 0, kFamToken = 1, kFamExt = 2 };
+
 struct Params {
   const void *draft;
   const void *target;
@@ -99,10 +122,16 @@ struct Params {
   float temperature;
   float k;        // log2(e) / T, the f32 factor of every exponent of pass 1
   float kl;       // log2(e) / T - k: with k, log2(e) / T to twice f32 precision
+  int units;      // units of the call: B (gamma + 1) row pairs and bonus rows, or B gamma pairs
   int L;          // slice length per CTA (multiple of 8 logits)
   int cluster;    // CTAs per unit
   int bulk;       // 1: TMA bulk copies, 0: per-thread loads (rows not 16-byte aligned)
   int mode;
+  int greedy;     // T = 0: greedy decoding; the rules' statistics use T = 1 (k = log2(e))
+  float lossy_l;  // lossy speculative decoding: -log2(1 - alpha) as lossy_l + lossy_ll,
+  float lossy_ll; // the shift of log2 of the acceptance ratio (+inf: alpha = 1)
+  float lossy_c;  // -log2(beta): the residual max(0, p / beta - q) is 2^{b + c + lossy_c} - 2^a
+  float beta;     // lossy speculative decoding's beta (Table 3), >= 1 - alpha
   int32_t *num_accepted;
   int32_t *next_token;
   float *row_info;
@@ -114,10 +143,28 @@ struct Params {
   uint32_t *seq_tickets;   // [B] finished sample passes (+1 for rank 0's last arrival); zero at rest
   float4 *records;         // [B][kMaxCluster][gamma+1] (R_q, R_p, c, flags) as seen by rank r
   float4 *records2;        // [B][kMaxCluster][gamma+1] (eta, thr, token, on_q) of token rules
+  int spec_res;            // a rejected pair stores its residual's chunk prefixes itself (row_pre)
+  float *row_pre;          // [B][gamma+1][kMaxCluster][kMaxChunks + 1] those prefixes, per row
+  float *bonus_pre;        // [B][kMaxCluster][kMaxChunks + 1] the same for the bonus row p_gamma,
+                           // written by the bonus unit from its pass-1 chunk totals
   float *chunk_pre;        // [B][kMaxCluster][kMaxChunks + 1] exclusive prefix of slice r of the
                            // sampled row at each chunk start, then the slice total
   int32_t *status;
 };
+
+// ------------------------------------------------------------------ debug checks
+
+// First source line whose check failed (SC_DEBUG builds; 0: none).
+__device__ int g_sc_debug_line;
+
+// In SC_DEBUG builds, false for a failed check (its line recorded, the access
+// skipped by the caller); always true otherwise, and compiled away.
+__device__ __forceinline__ bool sc_check(bool cond, int line) {
+  if (!SC_DEBUG || cond) return true;
+  atomicCAS(&g_sc_debug_line, 0, line);
+  return false;
+}
+#define SC_CHECK(cond) sc_check((cond), __LINE__)
 
 // ------------------------------------------------------------------ PTX helpers
 
@@ -172,6 +219,11 @@ __device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t by
       : "memory");
 }
 
+// Hint: bring [src, src + bytes) into L2 (16-byte aligned, a multiple of 16 bytes).
+__device__ __forceinline__ void prefetch_l2(const void *src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
+
 __device__ __forceinline__ void cluster_arrive_relaxed() {
   asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
 }
@@ -195,6 +247,9 @@ __device__ __forceinline__ void st_peer(uint32_t a, float4 v) {
 }
 __device__ __forceinline__ void st_peer(uint32_t a, float2 v) {
   asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(a), "f"(v.x), "f"(v.y) : "memory");
+}
+__device__ __forceinline__ void st_peer(uint32_t a, int2 v) {
+  asm volatile("st.shared::cluster.v2.s32 [%0], {%1, %2};" ::"r"(a), "r"(v.x), "r"(v.y) : "memory");
 }
 __device__ __forceinline__ void st_peer(uint32_t a, float v) {
   asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(a), "f"(v) : "memory");
@@ -251,20 +306,33 @@ __device__ __forceinline__ void load8_smem(const E *s, int e, int n, float (&y)[
 struct __align__(16) Shared {
   uint64_t full[kStages];
   // cluster exchanges, written by every CTA of the cluster into slot [its rank]:
-  float4 all_ms[kMaxCluster];  // 1: (m_q, s_q, m_p, s_p) of the slice
-  float2 all_x[kMaxCluster];   // 1: raw logits at the draft token, if in the slice
+  // exchange 1 has two sets of slots, by the parity of the unit's iteration: a peer
+  // that loops on to its next unit pushes into the other set, never into the one
+  // this CTA may still be reading
+  float4 all_ms[2][kMaxCluster];  // 1: (m_q, s_q, m_p, s_p) of the slice
+  float2 all_x[2][kMaxCluster];   // 1: raw logits at the draft token, if in the slice
   float all_r[kMaxCluster];    // 2 (TV pass): the slice's total residual weight
-  float all_lb[kMaxCluster];   // OPT band: the slice's lower bound on D_TV
+  float2 all_lb[kMaxCluster];  // OPT band: the slice's lower bound on D_TV, and its sum of sqrt(q p)
+  float2 all_scr[kMaxCluster]; // token rules: the slice's sum of q over its undeferred tokens, and
+                               // whether its screen is exact (1) or not (0)
+  float4 all_ext[2][kMaxCluster]; // 1 (kFamExt): (A_q, A_p, X, -) of the slice, see ExtState
+  int2 all_idx[2][kMaxCluster];   // 1 (kFamExt): the slice's argmax of q and of p
   int timeout;
   float4 red[kNW];          // (m_q, s_q, m_p, s_p) of each warp
+  float4 ext_red[kNW];      // (kFamExt) (A_q, A_p, X, -) of each warp
+  int2 idx_red[kNW];        // (kFamExt) argmax of q and of p of each warp
   float seg[kEntries + 1];  // per-(chunk, round, warp) weights, then exclusive prefixes
   float xq, xp;             // raw logits at the draft token, when in this slice
   // row state, identical in every CTA of the cluster
   float Mq, Sq, Mp, Sp, Rq, Rp, maxq, maxp, c, tv, qx, pix;
   int err, delta, accept, need_p2, band;
   int tok, on_q;            // a token rule (Section 4.4) and its r(v) test's variable
+  float dl, dr;             // OPT and OPTLog: delta = [dl < dr - alpha D_TV]
+  float nhq, nhp;           // (kFamExt) sum_v q log q and sum_v p log p, in nats
+  int iq, ip;               // (kFamExt) argmax q and argmax p, lowest index on ties
   float thr, eta;           // its r(v) threshold (exponent domain) and eta = sum_v r(v) q(v)
   // sequence finish
+  int spec_skip;            // a rejection of an earlier position is already reported: not row j*
   int owner;                // this CTA runs its rank's sample pass of row j*
   int scan_records;         // j* must be read from the records (gamma + 1 > 32)
   int seq_last;             // the sequence's last finisher: draws the token
@@ -399,6 +467,196 @@ __device__ __forceinline__ void online_row<uint16_t, true>(const uint16_t *src, 
   s = acc;
 }
 
+// Pass-1 state of the kFamExt rules.  With a_v = y^q_v k - r_q and
+// b_v = y^p_v k - r_p relative to the references r = refk(m) of the running
+// maxima m:
+//   sq = sum 2^a,  aq = sum 2^a a,  sp = sum 2^b,  ap = sum 2^b b,  x = sum 2^a b,
+// so that, for the row's final references and sums (log2 q_v = a_v - log2 S_q),
+//   sum_v q log2 q = A_q / S_q - log2 S_q,   sum_v q log2 p = X / S_q - log2 S_p.
+// iq and ip are the lowest indices of the largest q and p logits seen (-1: none).
+// A term whose exponential is 0 contributes 0 to the moments.
+struct ExtState {
+  float mq, sq, aq, mp, sp, ap, x;
+  int iq, ip;
+};
+
+__device__ __forceinline__ ExtState ext_empty() {
+  return {-FLT_MAX, 0.0f, 0.0f, -FLT_MAX, 0.0f, 0.0f, 0.0f, -1, -1};
+}
+
+// Re-reference a partial by dq = r_q - r_q' <= 0 and dp = r_p - r_p' <= 0:
+// a' = a + dq and 2^{a'} = 2^{dq} 2^a, so A' = 2^{dq} (A + dq S) and
+// X' = 2^{dq} (X + dp S_q).  (A reference floored at -1e30 comes with S = 0.)
+__device__ __forceinline__ void ext_rebase(ExtState &e, float dq, float dp) {
+  const float fq = ex2(dq), fp = ex2(dp);
+  e.x = e.x == -INFINITY ? e.x : fq * fmaf(dp, e.sq, e.x);  // (-inf: D(q, p) = +inf, kept)
+  e.aq = fq * fmaf(dq, e.sq, e.aq);
+  e.sq = fq * e.sq;
+  e.ap = fp * fmaf(dp, e.sp, e.ap);
+  e.sp = fp * e.sp;
+}
+
+// The index of the larger of two maxima, the lower index on a tie (-1: none).
+__device__ __forceinline__ int pick_index(float ma, int ia, float mb, int ib) {
+  if (ma > mb) return ia;
+  if (mb > ma) return ib;
+  if (ia < 0) return ib;
+  if (ib < 0) return ia;
+  return min(ia, ib);
+}
+
+// b += a: both re-referenced to the larger maxima, then summed.
+__device__ __forceinline__ void ext_merge(ExtState &b, ExtState a, float k) {
+  const float Mq = fmaxf(a.mq, b.mq), Mp = fmaxf(a.mp, b.mp);
+  const float Rq = refk(Mq, k), Rp = refk(Mp, k);
+  ext_rebase(a, refk(a.mq, k) - Rq, refk(a.mp, k) - Rp);
+  ext_rebase(b, refk(b.mq, k) - Rq, refk(b.mp, k) - Rp);
+  b.iq = pick_index(b.mq, b.iq, a.mq, a.iq);
+  b.ip = pick_index(b.mp, b.ip, a.mp, a.ip);
+  b.mq = Mq;
+  b.mp = Mp;
+  b.sq = __fadd_rn(b.sq, a.sq);
+  b.aq = __fadd_rn(b.aq, a.aq);
+  b.sp = __fadd_rn(b.sp, a.sp);
+  b.ap = __fadd_rn(b.ap, a.ap);
+  b.x = __fadd_rn(b.x, a.x);
+}
+
+// Merge the partials of the 32 lanes of a warp (butterfly); lane 0 ends with
+// the warp's partial.
+__device__ __forceinline__ void ext_warp_merge(ExtState &e, float k) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    ExtState t;
+    t.mq = __shfl_xor_sync(0xFFFFFFFFu, e.mq, o);
+    t.sq = __shfl_xor_sync(0xFFFFFFFFu, e.sq, o);
+    t.aq = __shfl_xor_sync(0xFFFFFFFFu, e.aq, o);
+    t.mp = __shfl_xor_sync(0xFFFFFFFFu, e.mp, o);
+    t.sp = __shfl_xor_sync(0xFFFFFFFFu, e.sp, o);
+    t.ap = __shfl_xor_sync(0xFFFFFFFFu, e.ap, o);
+    t.x = __shfl_xor_sync(0xFFFFFFFFu, e.x, o);
+    t.iq = __shfl_xor_sync(0xFFFFFFFFu, e.iq, o);
+    t.ip = __shfl_xor_sync(0xFFFFFFFFu, e.ip, o);
+    ext_merge(e, t, k);
+  }
+}
+
+__device__ __forceinline__ ExtState ext_load(float4 ms, float4 m1, int2 idx) {
+  return {ms.x, ms.y, m1.x, ms.z, ms.w, m1.y, m1.z, idx.x, idx.y};
+}
+
+// Pass 1 of kFamExt on one chunk of the slice (both rows at once, or the bonus
+// row's p alone): this thread's kRounds vectors, in increasing vocabulary
+// order, so that a strict comparison keeps the lowest index of a maximum.  v0
+// is the vocabulary index of the chunk start.  Two reads of shared memory (the
+// maxima, then the terms) keep few logits live; the chunk's terms are summed
+// apart and then added, which keeps the f32 sums short.
+template <typename E, bool kFull>
+__device__ __forceinline__ void load8_chunk(const E *src, int e, int n, float (&y)[8]) {
+  if constexpr (kFull) {
+    Elt<E>::load8(src + e, y);
+  } else {
+    load8_smem(src, e, n, y);
+  }
+}
+
+template <typename E, bool kFull, bool kPair>
+__device__ __forceinline__ void ext_chunk(const E *srcq, const E *srcp, int n, int v0, float k,
+                                          ExtState &st, bool with_bc, float &bc) {
+  float mq = st.mq, mp = st.mp;
+  int iq = st.iq, ip = st.ip;
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r) {
+    const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
+    float yq[8], yp[8];
+    if constexpr (kPair) load8_chunk<E, kFull>(srcq, e, n, yq);
+    load8_chunk<E, kFull>(srcp, e, n, yp);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      if constexpr (kPair) {
+        if (yq[i] > mq) {
+          mq = yq[i];
+          iq = v0 + e + i;
+        }
+      }
+      if (yp[i] > mp) {
+        mp = yp[i];
+        ip = v0 + e + i;
+      }
+    }
+  }
+  const float rq = refk(mq, k), rp = refk(mp, k);
+  if (with_bc) bc *= ex2(0.5f * ((refk(st.mq, k) - rq) + (refk(st.mp, k) - rp)));  // (OPTLog's bound)
+  ext_rebase(st, refk(st.mq, k) - rq, refk(st.mp, k) - rp);
+  float sq = 0.0f, aq = 0.0f, sp = 0.0f, ap = 0.0f, x = 0.0f, h = 0.0f;
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r) {
+    const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
+    float yq[8], yp[8];
+    if constexpr (kPair) load8_chunk<E, kFull>(srcq, e, n, yq);
+    load8_chunk<E, kFull>(srcp, e, n, yp);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const float b = fmaf(yp[i], k, -rp);
+      const float eb = ex2(b);
+      sp += eb;
+      ap += eb > 0.0f ? eb * b : 0.0f;
+      if constexpr (kPair) {
+        const float a = fmaf(yq[i], k, -rq);
+        const float ea = ex2(a);
+        sq += ea;
+        aq += ea > 0.0f ? ea * a : 0.0f;
+        // a finite draft logit with a masked target logit (q(v) > 0 = p(v)) makes
+        // D(q, p) = +inf even where 2^a underflows: X = -inf, kept by every merge
+        x += yq[i] > -INFINITY && !(yp[i] > -INFINITY) ? -INFINITY : (ea > 0.0f ? ea * b : 0.0f);
+        if (with_bc) h += ex2(0.5f * (a + b));  // sqrt(q p) up to the normalisers
+      }
+    }
+  }
+  if (with_bc) bc += h;
+  st.mq = mq;
+  st.mp = mp;
+  st.iq = iq;
+  st.ip = ip;
+  st.sq = __fadd_rn(st.sq, sq);
+  st.aq = __fadd_rn(st.aq, aq);
+  st.sp = __fadd_rn(st.sp, sp);
+  st.ap = __fadd_rn(st.ap, ap);
+  st.x = __fadd_rn(st.x, x);
+}
+
+// Pass-1 screen of a token rule: per thread, the two largest logits of the row
+// that r(v) tests (q for TokenV1, p otherwise) and the draft logit at the
+// largest.  When every thread's second largest turns out deferred (r = 1), the
+// tokens that are not deferred are exactly the threads' largest ones that pass
+// the test, so eta = 1 - (their q) needs no pass over the row.
+struct Top2 {
+  float y1, y2, z1;
+};
+
+template <typename E, bool kFull>
+__device__ __forceinline__ void screen_chunk(const E *ssrc, const E *qsrc, int n, Top2 &t) {
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r) {
+    const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
+    float y[8], z[8];
+    load8_chunk<E, kFull>(ssrc, e, n, y);
+    load8_chunk<E, kFull>(qsrc, e, n, z);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      if (y[i] > t.y2) {
+        if (y[i] > t.y1) {
+          t.y2 = t.y1;
+          t.y1 = y[i];
+          t.z1 = z[i];
+        } else {
+          t.y2 = y[i];
+        }
+      }
+    }
+  }
+}
+
 // Row scalars of the weight formulas.  With a_v = y^q_v k - R_q, b_v = y^p_v k - R_p
 // (R = refk(M)) and c = log2(S_q / S_p):
 //   q_v = 2^{a_v} / S_q,   p_v = 2^{b_v} / S_p = 2^{b_v + c} / S_q,
@@ -484,6 +742,78 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
+// Pass 1 on a chunk of the bonus row p_gamma: online_row's running (max, sum)
+// and, per warp, the chunk's total weight sum_v 2^{y_v k - refk(W)}, W the
+// warp's largest logit of the chunk, in seg[c kNW + warp] (W in
+// seg[kBonusRef + c kNW + warp]).  After exchange 1 these give the chunk
+// prefixes of p_gamma's inverse CDF, so a sequence that accepts every draft
+// needs no second pass over its bonus row.
+constexpr int kBonusRef = kMaxChunks * kNW;
+static_assert(2 * kMaxChunks * kNW <= kEntries, "bonus chunk totals live in seg");
+
+template <typename E, bool kFull>
+__device__ __forceinline__ void bonus_row(const E *src, int n, float k, float &m, float2 &s, int c,
+                                          float *seg, int lane, int warp) {
+  float y[kRounds][8];
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r) {
+    const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
+    if constexpr (kFull) {
+      Elt<E>::load8(src + e, y[r]);
+    } else {
+      load8_smem(src, e, n, y[r]);
+    }
+  }
+  float W = -FLT_MAX;
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r)
+#pragma unroll
+    for (int i = 0; i < 8; i += 2) W = max3(W, y[r][i], y[r][i + 1]);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) W = fmaxf(W, __shfl_xor_sync(0xFFFFFFFFu, W, o));
+  const float rw = refk(W, k);
+  float c0 = 0.0f, c1 = 0.0f;
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r)
+#pragma unroll
+    for (int i = 0; i < 8; i += 2) {
+      c0 += ex2(fmaf(y[r][i], k, -rw));
+      c1 += ex2(fmaf(y[r][i + 1], k, -rw));
+    }
+  const float cs = c0 + c1;
+  // fold the chunk into the running sum, referenced to refk(max(m, W))
+  const float mn = fmaxf(m, W), rn = refk(mn, k);
+  const float so = ex2(refk(m, k) - rn);
+  s = make_float2(fmaf(cs, ex2(rw - rn), s.x * so), s.y * so);
+  m = mn;
+  const float tot = warp_sum(cs);
+  if (lane == 0 && SC_CHECK(c >= 0 && c < kMaxChunks)) {
+    seg[c * kNW + warp] = tot;
+    seg[kBonusRef + c * kNW + warp] = W;
+  }
+}
+
+// OPT: this thread's sum over a chunk of 2^{(a_v + b_v)/2} = 2^{((y^q_v + y^p_v) k - r_q - r_p)/2},
+// sqrt(q_v p_v) up to the rows' normalisers: the Bhattacharyya coefficient
+// BC = sum_v sqrt(q_v p_v) bounds D_TV from above, D_TV <= sqrt(1 - BC^2).
+template <typename E, bool kFull>
+__device__ __forceinline__ float bc_chunk(const E *srcq, const E *srcp, int n, float hk, float hr) {
+  float acc0 = 0.0f, acc1 = 0.0f;
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r) {
+    const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
+    float yq[8], yp[8];
+    load8_chunk<E, kFull>(srcq, e, n, yq);
+    load8_chunk<E, kFull>(srcp, e, n, yp);
+#pragma unroll
+    for (int i = 0; i < 8; i += 2) {
+      acc0 += ex2(fmaf(yq[i] + yp[i], hk, -hr));
+      acc1 += ex2(fmaf(yq[i + 1] + yp[i + 1], hk, -hr));
+    }
+  }
+  return acc0 + acc1;
+}
+
 // Weights of one chunk in the ring: per round, the warp's total weight (the
 // segment total) lands in seg[(c, round, warp)].
 template <typename E, bool kPair, bool kFull, bool kTok>
@@ -502,7 +832,7 @@ __device__ __forceinline__ void weights_chunk(const E *sq, const E *sp, int n, i
       load8_smem(sp, e, n, yp);
     }
     const float tot = warp_sum(vec_weights<kPair, kTok>(yq, yp, rs, w));
-    if (lane == 0) sh.seg[(c * kRounds + r) * kNW + warp] = tot;
+    if (lane == 0 && SC_CHECK(c >= 0 && c < kMaxChunks)) sh.seg[(c * kRounds + r) * kNW + warp] = tot;
   }
 }
 
@@ -555,13 +885,29 @@ __device__ __forceinline__ float prob_of(float y, float R, float S, float k, flo
 // essentially only the f32 error of log2(S_q / S_p).  With a token rule
 // (Section 4.4) the draft token's own deferral r(x) takes delta's place and
 // pi(x)/q(x) = (1 - r(x)) + eta p(x)/q(x): accepted outright when r(x) = 0,
-// else [u < eta 2^L].  A masked logit (-inf) is handled before L, whose
-// double-float terms it would turn into NaN: q(x) = 0 accepts, and p(x) = 0 <
-// q(x) makes the ratio 1 - delta.  q(x) and pi(x) themselves are evaluated
-// only for the diagnostics output.
-template <bool kTok>
-__device__ __forceinline__ void accept_test(Shared &sh, float yqx, float ypx, float u, float k, float kl,
-                                            bool want_probs) {
+// else [u < eta 2^L].  With lossy speculative decoding (Table 3, delta = 1)
+// the ratio is min(1, p(x) / ((1 - alpha) q(x))) (Lemma 2): L shifted by
+// -log2(1 - alpha).  Greedy decoding compares indices only.  A masked logit
+// (-inf) is handled before L, whose double-float terms it would turn into NaN:
+// q(x) = 0 accepts, and p(x) = 0 < q(x) makes the ratio 1 - delta.  q(x) and
+// pi(x) themselves are evaluated only for the diagnostics output.
+template <int kFam>
+__device__ __forceinline__ void accept_test(Shared &sh, const Params &P, int x, float yqx, float ypx,
+                                            float u, float k) {
+  constexpr bool kTok = kFam == kFamToken;
+  const float kl = P.kl;
+  if constexpr (kFam == kFamExt) {
+    if (P.greedy) {
+      // one-hot q~ and p~ at the argmaxes: pi(x)/q~(x) is 1 unless delta = 1 and
+      // x is not p's argmax (then 0); a draft with q~(x) = 0 is accepted
+      const bool on_q = x == sh.iq, on_p = x == sh.ip;
+      sh.accept = !(on_q && sh.delta && !on_p);
+      sh.qx = on_q ? 1.0f : 0.0f;
+      sh.pix = sh.delta ? (on_p ? 1.0f : 0.0f) : sh.qx;
+      return;
+    }
+  }
+  const bool lossy = kFam == kFamCascade && P.rule == SC_RULE_LOSSY;
   if (kTok && sh.tok) {
     const float ax = fmaf(yqx, k, -sh.Rq), bx = fmaf(ypx, k, -sh.Rp);  // as vec_weights forms them
     sh.delta = (sh.on_q ? ax : bx) < sh.thr;                           // reported: r(x)
@@ -578,19 +924,30 @@ __device__ __forceinline__ void accept_test(Shared &sh, float yqx, float ypx, fl
     const float2 s = two_sum(dk.x, -r.x);
     const float lo = __fadd_rn(__fadd_rn(__fadd_rn(s.y, dk.y), __fsub_rn(__fmul_rn(d.y, k), r.y)),
                                log2f(sh.Sq / sh.Sp));
-    const float2 L = df_norm(s.x, lo);
-    if (!(kTok && sh.tok)) {
+    float2 L = df_norm(s.x, lo);
+    if (kTok && sh.tok) {
+      if (L.x < INFINITY) accept = u < sh.eta * df_exp2(L);  // (q(x) = 0 accepts)
+    } else {
+      if (lossy) {
+        if (P.lossy_l < INFINITY) {
+          const float2 t = two_sum(L.x, P.lossy_l);
+          L = df_norm(t.x, __fadd_rn(__fadd_rn(t.y, L.y), P.lossy_ll));
+        } else {
+          L = make_float2(0.0f, 0.0f);  // alpha = 1 and p(x) > 0 here: the ratio is 1
+        }
+      }
       if (df_lt(L, 0.0f)) accept = u < df_exp2(L);
-    } else if (L.x < INFINITY) {  // (q(x) = 0 accepts)
-      accept = u < sh.eta * df_exp2(L);
     }
   }
   sh.accept = accept;
-  if (want_probs) {
+  if (P.row_info != nullptr) {
     const float qx = prob_of(yqx, sh.Rq, sh.Sq, k, kl);
     const float px = prob_of(ypx, sh.Rp, sh.Sp, k, kl);
     sh.qx = qx;
-    sh.pix = kTok && sh.tok ? fmaf(sh.eta, px, sh.delta ? 0.0f : qx) : (sh.delta ? px : qx);
+    if (kTok && sh.tok) sh.pix = fmaf(sh.eta, px, sh.delta ? 0.0f : qx);
+    else if (lossy)  // (alpha = 1: the limit alpha -> 1-, p / (1 - alpha) = +inf where p > 0, 0 where p = 0)
+      sh.pix = fmaxf(fminf(qx, P.alpha < 1.0f ? px / (1.0f - P.alpha) : (px > 0.0f ? INFINITY : 0.0f)), px / P.beta);
+    else sh.pix = sh.delta ? px : qx;
   }
 }
 
@@ -611,12 +968,27 @@ struct Ring {
   // thread 0, bulk mode: start the copies of chunk c into stage s
   __device__ void issue(Shared &sh, int c, int s) const {
     const uint32_t bytes = static_cast<uint32_t>(chunk_len(c)) * sizeof(E);
+    if (!SC_CHECK(c >= 0 && c < nch && s >= 0 && s < kStages && bytes > 0 && bytes % 16 == 0 &&
+                  reinterpret_cast<uintptr_t>(gp + static_cast<size_t>(c) * kCH) % 16 == 0 &&
+                  (!pair || reinterpret_cast<uintptr_t>(gq + static_cast<size_t>(c) * kCH) % 16 == 0)))
+      return;
     mbar_expect_tx(&sh.full[s], pair ? 2 * bytes : bytes);
     if (pair) bulk_g2s(q(s), gq + static_cast<size_t>(c) * kCH, bytes, &sh.full[s]);
     bulk_g2s(p(s), gp + static_cast<size_t>(c) * kCH, bytes, &sh.full[s]);
   }
+  // thread 0, bulk mode: hint chunk c into L2
+  __device__ void prefetch(int c) const {
+    const uint32_t bytes = static_cast<uint32_t>(chunk_len(c)) * sizeof(E);
+    if (!SC_CHECK(c >= 0 && c < nch && bytes > 0 && bytes % 16 == 0 &&
+                  reinterpret_cast<uintptr_t>(gp + static_cast<size_t>(c) * kCH) % 16 == 0 &&
+                  (!pair || reinterpret_cast<uintptr_t>(gq + static_cast<size_t>(c) * kCH) % 16 == 0)))
+      return;
+    if (pair) prefetch_l2(gq + static_cast<size_t>(c) * kCH, bytes);
+    prefetch_l2(gp + static_cast<size_t>(c) * kCH, bytes);
+  }
   // all threads, per-thread mode: copy chunk c into stage s
   __device__ void load_sync(int c, int s) const {
+    if (!SC_CHECK(c >= 0 && c < nch && s >= 0 && s < kStages)) return;
     const int n = chunk_len(c);
     const size_t o = static_cast<size_t>(c) * kCH;
     for (int i = threadIdx.x; i < n; i += kNT) {
@@ -690,6 +1062,10 @@ __device__ __forceinline__ int stream_rev(const Ring<E> &R, Shared &sh, uint32_t
   const int nres = resident ? min(kStages, nch) : 0;
   if (!resident && R.bulk && threadIdx.x == 0)
     for (int c = nch - 1; c >= max(0, nch - kStages); --c) R.issue(sh, c, c % kStages);
+  // a second pass finds its older chunks mostly gone from L2 and streams them with
+  // only the ring in flight: ask for all of them at once, in the order they are used
+  if (SC_L2_PREFETCH && R.bulk && threadIdx.x == 0)
+    for (int c = nch - 1 - kStages; c >= 0; --c) R.prefetch(c);
   int tmo = 0;
   for (int i = 0; i < nch; ++i) {
     const int c = nch - 1 - i, s = c % kStages;
@@ -827,42 +1203,72 @@ __device__ __forceinline__ int search_segment(const E *sq, const E *sp, int n, b
   return tok;
 }
 
-template <typename E, bool kTok>
-__global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Params P) {
-  extern __shared__ __align__(128) unsigned char smem_raw[];
-  cg::cluster_group cluster = cg::this_cluster();
-  const int C = P.cluster;
-  const int rank = static_cast<int>(cluster.block_rank());
-  const int unit = static_cast<int>(blockIdx.x) / C;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+// Row pair (b, j < gamma) or bonus row (b, gamma) of a unit (pairs only for sc_row_stats).
+__device__ __forceinline__ void unit_coords(const Params &P, int unit, int &b, int &j) {
   const int G1 = P.gamma + 1;
-  const bool verify = P.mode == kVerify;
-
-  int b, j;
-  if (verify) {
+  if (P.mode == kVerify && SC_BONUS_LAST) {
+    // every pair unit first, then the bonus rows: the last, partial wave of CTAs
+    // holds the shorter (target-only) units
+    const int pairs = P.B * P.gamma;
+    b = unit < pairs ? unit / P.gamma : unit - pairs;
+    j = unit < pairs ? unit % P.gamma : P.gamma;
+  } else if (P.mode == kVerify) {
     b = unit / G1;
     j = unit % G1;
   } else {
     b = unit / P.gamma;
     j = unit % P.gamma;
   }
-  const int v0 = rank * P.L;
-  const Ring<E> R = make_ring<E>(P, smem_raw, b, j, rank);
-  const bool pair = R.pair;
-  Shared &sh = *reinterpret_cast<Shared *>(smem_raw + static_cast<size_t>(kStages) * 2 * kCH * sizeof(E));
+}
 
-  // ---- start the stream; prefetch the row's scalars
+template <typename E, int kFam>
+__global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Params P) {
+  constexpr bool kTok = kFam == kFamToken;
+  constexpr bool kExt = kFam == kFamExt;
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  cg::cluster_group cluster = cg::this_cluster();
+  const int C = P.cluster;
+  const int rank = static_cast<int>(cluster.block_rank());
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int G1 = P.gamma + 1;
+  const bool verify = P.mode == kVerify;
+  const int stride = static_cast<int>(gridDim.x) / C;  // clusters in the grid
+  Shared &sh = *reinterpret_cast<Shared *>(smem_raw + static_cast<size_t>(kStages) * 2 * kCH * sizeof(E));
   if (tid == 0) {
     sh.timeout = 0;
-    sh.xq = NAN;
-    sh.xp = NAN;
-    if (R.bulk) {
+    if (P.bulk) {
       for (int s = 0; s < kStages; ++s) mbar_init(&sh.full[s], 1);
       asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
   }
-  uint32_t ph = 0;
+  uint32_t ph = 0;  // the ring's phase bits carry over from unit to unit
+
+  // Every CTA of a cluster walks the same units: blockIdx / C, then + stride.
+  // The default launch has one cluster per unit (one iteration); with
+  // SC_PERSISTENT the grid holds only the clusters that fit on the GPU at once,
+  // and each hints its next unit's first chunks into L2 when its pass 1 ends.
+#if SC_PERSISTENT
+  for (int unit = static_cast<int>(blockIdx.x) / C, it = 0; unit < P.units; unit += stride, ++it) {
+#else
+  {
+    const int unit = static_cast<int>(blockIdx.x) / C, it = 0;
+#endif
+  const int slot = it & 1;  // exchange-1 slot set of this unit
+  int b, j;
+  unit_coords(P, unit, b, j);
+  const int v0 = rank * P.L;
+  const Ring<E> R = make_ring<E>(P, smem_raw, b, j, rank);
+  const bool pair = R.pair;
+
+  // ---- start the stream; prefetch the row's scalars
+  if (tid == 0) {
+    sh.xq = NAN;
+    sh.xp = NAN;
+    // a previous unit's draw wrote ring memory with ordinary stores (its chunk
+    // prefixes); order them before this unit's copies into the same stages
+    if (it > 0 && P.bulk) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
   prime(R, sh);
   float uj = 0.0f, ug = 0.0f;
   int x = -1;
@@ -872,61 +1278,145 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     if (pair) x = P.tokens[static_cast<size_t>(b) * P.gamma + j];
   }
   __syncthreads();
-  cluster_arrive_relaxed();  // this CTA has started (peers may store into it after their wait)
+  if (it == 0) cluster_arrive_relaxed();  // this CTA has started (peers may store into it after their wait)
 
   // ---- pass 1: online max and sum of exponentials
   const float k = P.k;
   float mq = -FLT_MAX, mp = -FLT_MAX;
   float2 s2q = make_float2(0.0f, 0.0f), s2p = make_float2(0.0f, 0.0f);
+  ExtState ex = ext_empty();  // (kFamExt) moments and argmaxes
+  Top2 top = {-FLT_MAX, -FLT_MAX, -FLT_MAX};  // (kFamToken) the eta screen
+  const bool scr_q = P.rule == SC_RULE_TOKEN_V1;
+  // OPT: the pair's running sum of sqrt(q p) terms, relative to (r_q + r_p) / 2
+  const bool opt_bc = SC_OPT_UB && !kTok && !kExt && verify && pair && P.rule == SC_RULE_OPT;
+  const bool optlog_bc = SC_OPT_UB && kExt && verify && pair && !P.greedy && P.rule == SC_RULE_OPT_LOG;
+  float bc = 0.0f;
+  // the bonus row also leaves its per-(chunk, warp) totals for the sampler
+  const bool bonus_tot = verify && !pair && !P.greedy;
   const int lx = x - v0;  // draft token's offset in this slice (thread 0 only)
   int tmo = stream(R, sh, ph, [&](int c, int s) {
     const int n = R.chunk_len(c);
-    if (n == kCH) {
-      if (pair) online_row<E, true>(R.q(s), n, k, mq, s2q);
-      online_row<E, true>(R.p(s), n, k, mp, s2p);
+    if (bonus_tot) {
+      if (n == kCH) bonus_row<E, true>(R.p(s), n, k, mp, s2p, c, sh.seg, lane, warp);
+      else bonus_row<E, false>(R.p(s), n, k, mp, s2p, c, sh.seg, lane, warp);
+    } else if constexpr (kExt) {
+      const int vc = v0 + c * kCH;
+      if (pair) {
+        if (n == kCH) ext_chunk<E, true, true>(R.q(s), R.p(s), n, vc, k, ex, optlog_bc, bc);
+        else ext_chunk<E, false, true>(R.q(s), R.p(s), n, vc, k, ex, optlog_bc, bc);
+      } else {
+        if (n == kCH) ext_chunk<E, true, false>(R.q(s), R.p(s), n, vc, k, ex, false, bc);
+        else ext_chunk<E, false, false>(R.q(s), R.p(s), n, vc, k, ex, false, bc);
+      }
     } else {
-      if (pair) online_row<E, false>(R.q(s), n, k, mq, s2q);
-      online_row<E, false>(R.p(s), n, k, mp, s2p);
+      const float mq0 = mq, mp0 = mp;
+      if (n == kCH) {
+        if (pair) online_row<E, true>(R.q(s), n, k, mq, s2q);
+        online_row<E, true>(R.p(s), n, k, mp, s2p);
+        if (kTok && pair) screen_chunk<E, true>(scr_q ? R.q(s) : R.p(s), R.q(s), n, top);
+      } else {
+        if (pair) online_row<E, false>(R.q(s), n, k, mq, s2q);
+        online_row<E, false>(R.p(s), n, k, mp, s2p);
+        if (kTok && pair) screen_chunk<E, false>(scr_q ? R.q(s) : R.p(s), R.q(s), n, top);
+      }
+      if (opt_bc) {
+        const float rq = refk(mq, k), rp = refk(mp, k);
+        const float sc = ex2(0.5f * ((refk(mq0, k) - rq) + (refk(mp0, k) - rp)));
+        const float add = n == kCH ? bc_chunk<E, true>(R.q(s), R.p(s), n, 0.5f * k, 0.5f * (rq + rp))
+                                   : bc_chunk<E, false>(R.q(s), R.p(s), n, 0.5f * k, 0.5f * (rq + rp));
+        bc = fmaf(bc, sc, add);
+      }
     }
     if (tid == 0 && static_cast<unsigned>(lx - c * kCH) < static_cast<unsigned>(n)) {
       sh.xq = Elt<E>::at(R.q(s), lx - c * kCH);
       sh.xp = Elt<E>::at(R.p(s), lx - c * kCH);
     }
   });
+  if (SC_PERSISTENT && tid == 0 && P.bulk && unit + stride < P.units) {
+    // the next unit's first chunks stream into L2 while this one is exchanged,
+    // decided and reported; its pass 1 then finds them there
+    int bn, jn;
+    unit_coords(P, unit + stride, bn, jn);
+    const Ring<E> Rn = make_ring<E>(P, smem_raw, bn, jn, rank);
+    for (int c = 0; c < min(kStages, Rn.nch); ++c) Rn.prefetch(c);
+  }
+  if constexpr (kExt) {
+    if (bonus_tot) {
+      ex.mp = mp;
+      ex.sp = s2p.x + s2p.y;
+    }
+    mq = ex.mq;
+    mp = ex.mp;
+    s2q = make_float2(ex.sq, 0.0f);
+    s2p = make_float2(ex.sp, 0.0f);
+  }
   float s_q = s2q.x + s2q.y, s_p = s2p.x + s2p.y;
   const float4 mine = make_float4(mq, s_q, mp, s_p);  // this thread's partial, kept for the D_TV bound
   tmo = __syncthreads_or(tmo);
-  warp_ms_merge(mq, s_q, k);
-  warp_ms_merge(mp, s_p, k);
-  if (lane == 0) sh.red[warp] = make_float4(mq, s_q, mp, s_p);
+  if constexpr (kExt) {
+    ext_warp_merge(ex, k);
+    if (lane == 0) {
+      sh.red[warp] = make_float4(ex.mq, ex.sq, ex.mp, ex.sp);
+      sh.ext_red[warp] = make_float4(ex.aq, ex.ap, ex.x, 0.0f);
+      sh.idx_red[warp] = make_int2(ex.iq, ex.ip);
+    }
+  } else {
+    warp_ms_merge(mq, s_q, k);
+    warp_ms_merge(mp, s_p, k);
+    if (lane == 0) sh.red[warp] = make_float4(mq, s_q, mp, s_p);
+  }
   __syncthreads();
   // ---- exchange 1: thread 0 merges the warp partials into the slice partial
   // and pushes it into every CTA of the cluster; one barrier; then every read
   // is local, and thread 0 decides
   float4 part = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+  float4 part_ext = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+  int2 part_idx = make_int2(-1, -1);
   if (tid == 0) {
-    part = merge_partials(sh.red, kNW, k);
-    if (tmo) {
+    if constexpr (kExt) {
+      ExtState e = ext_load(sh.red[0], sh.ext_red[0], sh.idx_red[0]);
+      for (int w = 1; w < kNW; ++w) ext_merge(e, ext_load(sh.red[w], sh.ext_red[w], sh.idx_red[w]), k);
+      part = make_float4(e.mq, e.sq, e.mp, e.sp);
+      part_ext = make_float4(e.aq, e.ap, e.x, 0.0f);
+      part_idx = make_int2(e.iq, e.ip);
+    } else {
+      part = merge_partials(sh.red, kNW, k);
+    }
+    if (tmo || sh.timeout) {  // (a copy of an earlier unit that never landed may land now)
       part.y = NAN;
       part.w = NAN;
       flag_timeout(sh, P);
     }
   }
-  cluster_wait();  // every CTA of the cluster has started
+  if (it == 0) cluster_wait();  // every CTA of the cluster has started
   if (tid == 0) {
     const float2 xv = make_float2(sh.xq, sh.xp);
     for (int r = 0; r < C; ++r) {
-      st_peer(peer_addr(&sh.all_ms[rank], r), part);
-      st_peer(peer_addr(&sh.all_x[rank], r), xv);
+      st_peer(peer_addr(&sh.all_ms[slot][rank], r), part);
+      st_peer(peer_addr(&sh.all_x[slot][rank], r), xv);
+      if constexpr (kExt) {
+        st_peer(peer_addr(&sh.all_ext[slot][rank], r), part_ext);
+        st_peer(peer_addr(&sh.all_idx[slot][rank], r), part_idx);
+      }
     }
   }
   cluster_arrive();
   cluster_wait();
 
   if (tid == 0) {  // thread 0 also holds the prefetched scalars
-    const float4 v = merge_partials(sh.all_ms, C, k);  // the row's M and S over the cluster
+    // the row's M and S over the cluster (and, for kFamExt, its moments and argmaxes)
+    ExtState g = ext_empty();
+    float4 v;
+    if constexpr (kExt) {
+      g = ext_load(sh.all_ms[slot][0], sh.all_ext[slot][0], sh.all_idx[slot][0]);
+      for (int r = 1; r < C; ++r)
+        ext_merge(g, ext_load(sh.all_ms[slot][r], sh.all_ext[slot][r], sh.all_idx[slot][r]), k);
+      v = make_float4(g.mq, g.sq, g.mp, g.sp);
+    } else {
+      v = merge_partials(sh.all_ms[slot], C, k);
+    }
     const float a = v.x, as = v.y, c = v.z, cs = v.w;
-    const float2 xv = sh.all_x[(x >= 0 && x < P.V) ? x / P.L : 0];
+    const float2 xv = sh.all_x[slot][(x >= 0 && x < P.V) ? x / P.L : 0];
     const float yqx = xv.x, ypx = xv.y;
     // S = sum_v 2^{y_v k - R} with R = fl(M k); the max logit's own term is
     // 2^{fma(M, k, -R)}, so max_v q(v) = 2^{fma(M, k, -R)} / S.
@@ -954,10 +1444,46 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     sh.thr = -INFINITY;
     sh.eta = 0.0f;
     sh.accept = 0;
+    sh.spec_skip = 0;
     sh.tv = -1.0f;
     sh.qx = 0.0f;
     sh.pix = 0.0f;
     sh.c = pair && !err ? log2f(as / cs) : 0.0f;
+    if (bonus_tot) {
+      // p_gamma's chunk prefixes over this slice from pass 1's per-(chunk, warp)
+      // totals, re-referenced to R_p: what a sampling pass over the row would store
+      float *cp = P.bonus_pre + (static_cast<size_t>(b) * kMaxCluster + rank) * (kMaxChunks + 1);
+      float acc = 0.0f;
+      for (int c2 = 0; c2 < R.nch; ++c2) {
+        if (SC_CHECK(b < P.B && rank < kMaxCluster && c2 < kMaxChunks)) cp[c2] = acc;
+        float t = 0.0f;
+        for (int w = 0; w < kNW; ++w)
+          t = fmaf(sh.seg[c2 * kNW + w], ex2(refk(sh.seg[kBonusRef + c2 * kNW + w], k) - Rp), t);
+        acc = __fadd_rn(acc, t);
+      }
+      if (SC_CHECK(b < P.B && rank < kMaxCluster && R.nch <= kMaxChunks)) cp[R.nch] = err || tmo ? NAN : acc;
+    }
+    sh.dl = sh.maxq;
+    sh.dr = sh.maxp;
+    float xent = 0.0f;  // (kFamExt) BiLD*'s discrepancy D(q, p) = -sum_v q log p, in nats
+    if constexpr (kExt) {
+      // sum q ln q = ln 2 (A_q / S_q - log2 S_q), sum q ln p = ln 2 (X / S_q - log2 S_p)
+      constexpr float kLn2 = 0.69314718f;
+      sh.iq = g.iq;
+      sh.ip = g.ip;
+      sh.nhq = kLn2 * (g.aq / as - log2f(as));
+      sh.nhp = kLn2 * (g.ap / cs - log2f(cs));
+      xent = kLn2 * (log2f(cs) - g.x / as);
+      if (P.greedy && pair && P.rule == SC_RULE_BILD && g.iq >= 0 && g.iq < P.V) {
+        // greedy decoding: the BiLD baseline's D = -log p(argmax q), from the target
+        // logit at q's argmax (one load; every CTA of the cluster reads the same value)
+        const E *prow = static_cast<const E *>(P.target) + (static_cast<size_t>(b) * G1 + j) * P.V;
+        const float y = Elt<E>::at(prow, static_cast<size_t>(g.iq));
+        const float2 lp = log2_prob(y, Rp, cs, k, P.kl);
+        xent = y > -INFINITY ? -kLn2 * (lp.x + lp.y) : INFINITY;
+      }
+      if (P.greedy && pair) sh.tv = g.iq != g.ip ? 1.0f : 0.0f;  // D_TV of the one-hot q~, p~
+    }
     if (!err && pair) {
       if (!verify) {
         sh.need_p2 = 1;  // sc_row_stats: TV of every pair
@@ -969,12 +1495,29 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
           case SC_RULE_CHOW: sh.delta = maxq < 1.0f - al; break;  // Eq. 2
           case SC_RULE_DIFF: sh.delta = maxq < maxp - al; break;  // Eq. 5
           case SC_RULE_OPT:                                       // Eq. 10
+            if (kExt) {  // greedy decoding: the one-hot D_TV is known
+              sh.delta = maxq < maxp - al * sh.tv;
+              break;
+            }
             // alpha * TV lies in [0, alpha]: TV decides only inside that band
             if (!(maxq < maxp)) sh.delta = 0;
             else if (maxq < maxp - al) sh.delta = 1;
             else pending = true;
             break;
           case SC_RULE_ALWAYS_DEFER: sh.delta = 1; break;
+          case SC_RULE_LOSSY: sh.delta = 1; break;  // Table 3: the target min/max of q, p
+          // Table 3 and the log-loss rules
+          case SC_RULE_BILD: sh.delta = xent > al; break;              // D(q, p) > alpha
+          case SC_RULE_CHOW_LOG: sh.delta = -sh.nhq > al; break;       // H(q) > alpha
+          case SC_RULE_DIFF_LOG: sh.delta = sh.nhq < sh.nhp - al; break;
+          case SC_RULE_OPT_LOG:  // sum q log q < sum p log p - alpha D_TV
+            sh.dl = sh.nhq;
+            sh.dr = sh.nhp;
+            if (P.greedy) sh.delta = sh.nhq < sh.nhp - al * sh.tv;
+            else if (!(sh.nhq < sh.nhp)) sh.delta = 0;
+            else if (sh.nhq < sh.nhp - al) sh.delta = 1;
+            else pending = true;
+            break;
           case SC_RULE_TOKEN_V1:
           case SC_RULE_TOKEN_V2:
           case SC_RULE_TOKEN_V3: {
@@ -990,13 +1533,14 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
               sh.on_q = P.rule == SC_RULE_TOKEN_V1;
               sh.thr = m > 0.0f ? log2f(m * (sh.on_q ? as : cs)) : -INFINITY;
             }
+            if (sh.thr == -INFINITY) pending = false;  // r = 0 everywhere: eta = 0, pi = q
             break;
           }
           default: sh.delta = 0; break;
         }
         if (pending) sh.need_p2 = 1;
         if (pending && !sh.tok) sh.band = 1;
-        if (!pending) accept_test<kTok>(sh, yqx, ypx, uj, k, P.kl, P.row_info != nullptr);
+        if (!pending) accept_test<kFam>(sh, P, x, yqx, ypx, uj, k);
       }
     }
     // keep the draft-token logits for a decision after the TV pass
@@ -1005,32 +1549,89 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   }
   __syncthreads();
 
+  // ---- token rules: eta without a pass when the pass-1 screen settles it.  A
+  // thread whose second-largest screened logit is deferred holds at most one
+  // undeferred token, its largest; if that holds in every thread of the
+  // cluster, eta = (S_q - sum of 2^a over those tokens) / S_q.
+  if (kTok && sh.tok && sh.need_p2) {
+    const float Rs = sh.on_q ? sh.Rq : sh.Rp;  // r(v) tests a_v or b_v, formed as vec_weights forms them
+    const bool ok = !(fmaf(top.y2, k, -Rs) >= sh.thr);
+    const float h = fmaf(top.y1, k, -Rs) >= sh.thr ? ex2(fmaf(top.z1, k, -sh.Rq)) : 0.0f;
+    const bool wok = __all_sync(0xFFFFFFFFu, ok);
+    const float hs = warp_sum(h);
+    if (lane == 0) sh.red[warp] = make_float4(hs, wok ? 1.0f : 0.0f, 0.0f, 0.0f);
+    __syncthreads();
+    if (tid == 0) {
+      float acc = 0.0f, okc = 1.0f;
+      for (int w = 0; w < kNW; ++w) {
+        acc = __fadd_rn(acc, sh.red[w].x);
+        okc = fminf(okc, sh.red[w].y);
+      }
+      for (int r = 0; r < C; ++r) st_peer(peer_addr(&sh.all_scr[rank], r), make_float2(acc, okc));
+    }
+    cluster_arrive();
+    cluster_wait();
+    if (tid == 0) {
+      float H = 0.0f, okc = 1.0f;  // in rank order
+      for (int r = 0; r < C; ++r) {
+        H = __fadd_rn(H, sh.all_scr[r].x);
+        okc = fminf(okc, sh.all_scr[r].y);
+      }
+      if (okc > 0.0f) {
+        sh.need_p2 = 0;
+        sh.eta = fmaxf(0.0f, sh.Sq - H) / sh.Sq;  // eta = sum_v r(v) q(v) = 1 - sum over undeferred
+        accept_test<kFam>(sh, P, x, sh.xq, sh.xp, uj, k);
+      }
+    }
+    __syncthreads();
+  }
+
   // ---- OPT band: a lower bound on D_TV from the pass-1 partials.  The threads'
   // element sets partition the vocabulary, so sum_t max(0, P_t - Q_t) <= D_TV
   // (P_t, Q_t: the probability mass of thread t's logits).  When alpha times
-  // that bound already reaches max p - max q, delta = 0 for the exact D_TV too
-  // (Eq. 10) and the TV pass is skipped.  The bound carries ~1e-6 of f32
+  // that bound already reaches dr - dl (max p - max q for OPT, Eq. 10; the
+  // negative-entropy gap for OPTLog), delta = 0 for the exact D_TV too and the
+  // TV pass is skipped.  The bound carries ~1e-6 of f32
   // rounding over its 128 C terms; only a clear 1e-4 excess settles the row.
   if (sh.band) {
     const float pt = mine.w * ex2(refk(mine.z, k) - sh.Rp) / sh.Sp;
     const float qt = mine.y * ex2(refk(mine.x, k) - sh.Rq) / sh.Sq;
     const float lb = warp_sum(fmaxf(0.0f, pt - qt));
-    if (lane == 0) sh.red[warp].x = lb;
+    // OPT: this thread's sum of sqrt(q p) terms at the row's references
+    const float bcw = warp_sum(bc * ex2(0.5f * ((refk(mine.x, k) - sh.Rq) + (refk(mine.z, k) - sh.Rp))));
+    if (lane == 0) sh.red[warp] = make_float4(lb, bcw, 0.0f, 0.0f);
     __syncthreads();
     if (tid == 0) {
-      float acc = 0.0f;
-      for (int w = 0; w < kNW; ++w) acc = __fadd_rn(acc, sh.red[w].x);
-      for (int r = 0; r < C; ++r) st_peer(peer_addr(&sh.all_lb[rank], r), acc);
+      float acc = 0.0f, accb = 0.0f;
+      for (int w = 0; w < kNW; ++w) {
+        acc = __fadd_rn(acc, sh.red[w].x);
+        accb = __fadd_rn(accb, sh.red[w].y);
+      }
+      for (int r = 0; r < C; ++r) st_peer(peer_addr(&sh.all_lb[rank], r), make_float2(acc, accb));
     }
     cluster_arrive();
     cluster_wait();
     if (tid == 0) {
-      float LB = 0.0f;  // in rank order
-      for (int r = 0; r < C; ++r) LB = __fadd_rn(LB, sh.all_lb[r]);
-      if (P.alpha * LB - (sh.maxp - sh.maxq) >= 1e-4f) {
+      float LB = 0.0f, BCs = 0.0f;  // in rank order
+      for (int r = 0; r < C; ++r) {
+        LB = __fadd_rn(LB, sh.all_lb[r].x);
+        BCs = __fadd_rn(BCs, sh.all_lb[r].y);
+      }
+      const float gap = sh.dr - sh.dl;
+      if (P.alpha * LB - gap >= 1e-4f) {
         sh.need_p2 = 0;
         sh.delta = 0;
-        accept_test<kTok>(sh, sh.xq, sh.xp, uj, k, P.kl, P.row_info != nullptr);
+        accept_test<kFam>(sh, P, x, sh.xq, sh.xp, uj, k);
+      } else if (opt_bc || optlog_bc) {
+        // D_TV <= sqrt(1 - BC^2) (Hellinger): with BC deflated well past its f32
+        // error, alpha times that bound below the gap settles delta = 1 (Eq. 10, OPTLog)
+        const float bcl = fminf(1.0f, BCs / sqrtf(sh.Sq) / sqrtf(sh.Sp)) * (1.0f - 2e-4f);
+        const float ub = sqrtf(fmaxf(0.0f, 1.0f - bcl * bcl));
+        if (gap - P.alpha * ub >= 1e-4f) {
+          sh.need_p2 = 0;
+          sh.delta = 1;
+          accept_test<kFam>(sh, P, x, sh.xq, sh.xp, uj, k);
+        }
       }
     }
     __syncthreads();
@@ -1060,13 +1661,49 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
         sh.err |= SC_DEV_TIMEOUT;
       } else if (sh.tok) {
         sh.eta = Rtot / sh.Sq;  // eta = sum_v r(v) q(v)
-        accept_test<kTok>(sh, sh.xq, sh.xp, uj, k, P.kl, P.row_info != nullptr);
+        accept_test<kFam>(sh, P, x, sh.xq, sh.xp, uj, k);
       } else {
         sh.tv = fminf(1.0f, fmaxf(0.0f, Rtot / sh.Sq));  // Lemma 3: R = S_q D_TV(p, q)
         if (verify) {
-          sh.delta = sh.maxq < sh.maxp - P.alpha * sh.tv;  // Eq. 10
-          accept_test<kTok>(sh, sh.xq, sh.xp, uj, k, P.kl, P.row_info != nullptr);
+          sh.delta = sh.dl < sh.dr - P.alpha * sh.tv;  // Eq. 10 (or OPTLog)
+          accept_test<kFam>(sh, P, x, sh.xq, sh.xp, uj, k);
         }
+      }
+    }
+    __syncthreads();
+  }
+
+  // ---- small batches: a rejected pair stores its own residual's chunk prefixes
+  // now, while its slice is in the ring and in L2, so that no pass is left for
+  // the end of the sequence's chain (the row is j* unless an earlier one also
+  // rejects).  The OPT band's TV pass has summed exactly these weights already.
+  // A rejected pair whose rank already shows a rejection at an earlier position
+  // is not row j* and skips the pass (a stale read of the ticket only costs the
+  // pass; row j* itself never sees an earlier rejection).
+  if (P.spec_res && verify && pair && !sh.accept && !sh.err && !(kExt && P.greedy) && j > 0 && G1 <= 32) {
+    if (tid == 0) {
+      const unsigned long long t = __ldcg(P.rank_tickets + static_cast<size_t>(b) * kMaxCluster + rank);
+      sh.spec_skip = ((t >> 32) & ((1ull << j) - 1ull)) != 0ull;
+    }
+    __syncthreads();
+  }
+  if (P.spec_res && verify && pair && !sh.accept && !sh.err && !(kExt && P.greedy) && !sh.spec_skip) {
+    if (!(sh.need_p2 && !sh.tok)) {
+      const bool lossy = kFam == kFamCascade && P.rule == SC_RULE_LOSSY;
+      const RowScalars rs = {sh.Rq, sh.Rp, k, lossy ? sh.c + P.lossy_c : sh.c,
+                             sh.tok ? kTokenRes : kResidual, sh.on_q, sh.thr, sh.eta};
+      tmo = slice_weights<kTok>(R, sh, ph, rs, sh.need_p2 ? kNewestFirst : kNewestFirstResident, lane, warp);
+      tmo = __syncthreads_or(tmo);
+      if (tid == 0) {
+        seg_prefix(sh, R.nch * kRounds * kNW);
+        if (tmo) flag_timeout(sh, P);
+      }
+    }
+    if (tid == 0) {
+      float *cp = P.row_pre + ((static_cast<size_t>(b) * G1 + j) * kMaxCluster + rank) * (kMaxChunks + 1);
+      if (SC_CHECK(b < P.B && j < G1 && rank < kMaxCluster && R.nch <= kMaxChunks)) {
+        for (int c = 0; c < R.nch; ++c) cp[c] = sh.seg[c * kRounds * kNW];
+        cp[R.nch] = sh.timeout ? NAN : sh.seg[R.nch * kRounds * kNW];
       }
     }
     __syncthreads();
@@ -1087,9 +1724,14 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     float4 *rec2 = P.records2 + (static_cast<size_t>(b) * kMaxCluster + rank) * G1;
     if (tid == 0) {
       const int flags = (sh.accept ? 1 : 0) | (sh.err ? 2 : 0);
-      rec[j] = make_float4(sh.Rq, sh.Rp, sh.c, __int_as_float(flags));
-      if (P.rule >= SC_RULE_TOKEN_V1)  // (only token rules read the second record)
-        rec2[j] = make_float4(sh.eta, sh.thr, __int_as_float(sh.tok), __int_as_float(sh.on_q));
+      float4 r1 = make_float4(sh.Rq, sh.Rp, sh.c, __int_as_float(flags));
+      if (kFam == kFamCascade && P.rule == SC_RULE_LOSSY)
+        r1.z = sh.c + P.lossy_c;  // the residual max(0, p / beta - q) (Lemma 2)
+      if (kExt && P.greedy) r1.x = __int_as_float(sh.ip);  // greedy: the token emitted at row j*
+      if (SC_CHECK(b < P.B && rank < kMaxCluster && j < G1)) rec[j] = r1;
+      if (kTok)  // (only token rules read the second record)
+        if (SC_CHECK(b < P.B && rank < kMaxCluster && j < G1))
+          rec2[j] = make_float4(sh.eta, sh.thr, __int_as_float(sh.tok), __int_as_float(sh.on_q));
       if (rank == 0 && P.row_info) {
         float *ri = P.row_info + (static_cast<size_t>(b) * G1 + j) * SC_ROW_FIELDS;
         ri[SC_ROW_MAXQ] = pair && !sh.err ? sh.maxq : NAN;
@@ -1139,11 +1781,17 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     }
     if (sh.owner && tid == 0) {  // row j*'s records (they are in)
       sh.rj = __ldcg(&rec[sh.jstar]);
-      sh.rj2 = P.rule >= SC_RULE_TOKEN_V1 ? __ldcg(&rec2[sh.jstar]) : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+      sh.rj2 = kTok ? __ldcg(&rec2[sh.jstar]) : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
     }
     __syncthreads();
 
-    if (sh.owner) {
+    if (sh.owner && ((kExt && P.greedy) || sh.jstar == P.gamma || P.spec_res)) {
+      // nothing to sample: greedy decoding emits row j*'s argmax p (in the
+      // records), the bonus row's chunk prefixes came from its pass 1, and
+      // with spec_res row j* stored its own
+      if (tid == 0) sh.seq_last = atom_add_acq_rel(P.seq_tickets + b, 1u) == static_cast<uint32_t>(C);
+      __syncthreads();
+    } else if (sh.owner) {
       // ---- sample pass: weights of this rank's slice of row j* -- the residual
       // max(0, p - q) of a rejected pair (Algorithm 4), or p of the bonus row
       const int js = sh.jstar;
@@ -1160,8 +1808,10 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
           flag_timeout(sh, P);
         }
         float *cp = P.chunk_pre + (static_cast<size_t>(b) * kMaxCluster + rank) * (kMaxChunks + 1);
-        for (int c = 0; c < Rj.nch; ++c) cp[c] = sh.seg[c * kRounds * kNW];
-        cp[Rj.nch] = tot_r;  // the slice total
+        if (SC_CHECK(b < P.B && rank < kMaxCluster && Rj.nch <= kMaxChunks)) {
+          for (int c = 0; c < Rj.nch; ++c) cp[c] = sh.seg[c * kRounds * kNW];
+          cp[Rj.nch] = tot_r;  // the slice total
+        }
         sh.seq_last = atom_add_acq_rel(P.seq_tickets + b, 1u) == static_cast<uint32_t>(C);
       }
       __syncthreads();
@@ -1173,14 +1823,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       constexpr int kCP = kMaxChunks + 1;
       float *cpall = reinterpret_cast<float *>(smem_raw);  // [C][kCP]
       if (tid == 0) P.seq_tickets[b] = 0u;  // every report of the sequence is in
-      // one round of loads: every slice's chunk prefixes (ending in its total) ...
-      const float *cpg = P.chunk_pre + static_cast<size_t>(b) * kMaxCluster * kCP;
-      for (int i = tid; i < C * kCP; i += kNT) {
-        const int r = i / kCP, c = i % kCP;
-        const int len = max(0, min(P.L, P.V - r * P.L));
-        if (c <= (len + kCH - 1) / kCH) cpall[i] = __ldcg(cpg + i);
-      }
-      // ... and, in warp 0, j* and the error flags from rank 0's records
+      // warp 0: j* and the error flags from rank 0's records
       if (warp == 0) {
         const float4 *rec0 = P.records + static_cast<size_t>(b) * kMaxCluster * G1;
         int js = P.gamma, bad = 0;
@@ -1203,133 +1846,157 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
           sh.jstar = js;
           sh.bad = bad;
           sh.rj = rj;
-          sh.rj2 = P.rule >= SC_RULE_TOKEN_V1 ? __ldcg(P.records2 + static_cast<size_t>(b) * kMaxCluster * G1 + js)
+          sh.rj2 = kTok ? __ldcg(P.records2 + static_cast<size_t>(b) * kMaxCluster * G1 + js)
                                               : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
         }
       }
       __syncthreads();
       const int js = sh.jstar;
-      const RowScalars rs = sample_scalars(sh.rj, sh.rj2, k);
-      // ---- inverse CDF over the slices in rank order, u = u[b][gamma], then
-      // over the chunks of the crossing slice
-      if (warp == 0) {
-        auto nch_of = [&](int r) {
-          const int len = max(0, min(P.L, P.V - r * P.L));
-          return (len + kCH - 1) / kCH;
-        };
-        const float tot = lane < C ? cpall[lane * kCP + nch_of(lane)] : 0.0f;
-        const float pre = warp_incl_scan(tot, lane);  // through rank `lane`
-        const float Rtot = __shfl_sync(0xFFFFFFFFu, pre, C - 1);
-        float before = __shfl_up_sync(0xFFFFFFFFu, pre, 1);
-        if (lane == 0) before = 0.0f;
-        const float u = __shfl_sync(0xFFFFFFFFu, ug, 0);
-        const bool ok = !sh.bad && isfinite(Rtot);
-        int cr = -1, cc = -1, clast = -1;
-        float2 tl = make_float2(-1.0f, 0.0f);  // (negative: u R fell past the last boundary)
-        if (ok && Rtot > 0.0f) {
-          const float th = __fmul_rn(u, Rtot);
-          const float2 t = make_float2(th, fmaf(u, Rtot, -th));  // u R_tot, exactly
-          const bool cross = lane < C && tot > 0.0f && df_ge(t, before) && df_lt(t, pre);
-          const unsigned cm = __ballot_sync(0xFFFFFFFFu, cross);
-          const unsigned pm = __ballot_sync(0xFFFFFFFFu, lane < C && tot > 0.0f);
-          cr = cm ? __ffs(cm) - 1 : 31 - __clz(pm);
-          const float bcr = __shfl_sync(0xFFFFFFFFu, before, cr);
-          if (cm) tl = df_sub(t, bcr);
-          // the chunk of slice cr holding tl (or, past a rounding gap, its last chunk with weight)
-          const float *cp = cpall + cr * kCP;
-          const int nch = nch_of(cr);
-          for (int base = 0; base < nch; base += 32) {
-            const int c = base + lane;
-            const float lo = c < nch ? cp[c] : 0.0f, hi = c < nch ? cp[c + 1] : 0.0f;
-            const bool pos = c < nch && hi > lo;
-            const unsigned mi = __ballot_sync(0xFFFFFFFFu, pos && df_ge(tl, lo) && df_lt(tl, hi));
-            const unsigned mp = __ballot_sync(0xFFFFFFFFu, pos);
-            if (cc < 0 && mi) cc = base + __ffs(mi) - 1;
-            if (mp) clast = base + 31 - __clz(mp);
-          }
-        }
-        if (lane == 0) {
-          sh.sample_ok = ok;
-          sh.cross_rank = cr;
-          sh.t_slice = tl;
-          sh.token = -1;
-          sh.cross_chunk = cc >= 0 ? cc : clast;
-          sh.have_t = cc >= 0;
-          sh.chunk_lo = sh.cross_chunk >= 0 ? cpall[cr * kCP + sh.cross_chunk] : 0.0f;
-        }
+      // one round of loads: every slice's chunk prefixes of row j* (ending in its total)
+      const float *cpg = js == P.gamma ? P.bonus_pre + static_cast<size_t>(b) * kMaxCluster * kCP
+                         : P.spec_res  ? P.row_pre + (static_cast<size_t>(b) * G1 + js) * kMaxCluster * kCP
+                                       : P.chunk_pre + static_cast<size_t>(b) * kMaxCluster * kCP;
+      for (int i = tid; i < C * kCP && !(kExt && P.greedy); i += kNT) {
+        const int r = i / kCP, c = i % kCP;
+        const int len = max(0, min(P.L, P.V - r * P.L));
+        if (c <= (len + kCH - 1) / kCH && SC_CHECK(b < P.B && js <= P.gamma && C <= kMaxCluster))
+          cpall[i] = __ldcg(cpg + i);
       }
       __syncthreads();
-      const int cr = sh.cross_rank, cc = sh.cross_chunk;
-      if (cr >= 0 && cc >= 0) {
-        // the chunk's weights again, by the code the sample pass ran (the same values)
-        const Ring<E> Rc = make_ring<E>(P, smem_raw, b, js, cr);
-        const int sl = kStages - 1, n = Rc.chunk_len(cc);
-        if (Rc.bulk) {
-          if (tid == 0) Rc.issue(sh, cc, sl);
-          tmo = wait_stage(sh, sl, ph);
-        } else {
-          tmo = 0;
-          Rc.load_sync(cc, sl);
+      if (kExt && P.greedy) {
+        // greedy decoding: the argmax p of row j*, from rank 0's record
+        if (tid == 0 && SC_CHECK(b < P.B && js >= 0 && js <= P.gamma)) {
+          const bool ok = !sh.bad;
+          const int tok = __float_as_int(sh.rj.x);
+          P.num_accepted[b] = ok ? js : 0;
+          P.next_token[b] = ok ? tok : -1;
+          if (ok && P.row_info)
+            P.row_info[(static_cast<size_t>(b) * G1 + js) * SC_ROW_FIELDS + SC_ROW_CAND] = static_cast<float>(tok);
         }
-        tmo = __syncthreads_or(tmo);
-        if (Rc.pair) {
-          if (n == kCH) weights_chunk<E, true, true, kTok>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
-          else weights_chunk<E, true, false, kTok>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
-        } else {
-          if (n == kCH) weights_chunk<E, false, true, kTok>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
-          else weights_chunk<E, false, false, kTok>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
-        }
-        if (tmo && tid == 0) {
-          flag_timeout(sh, P);
-          sh.sample_ok = 0;
-        }
-        __syncthreads();
-        constexpr int kSegC = kRounds * kNW;  // segments per chunk
-        if (tid == 0) {
-          // exclusive prefixes continue from the chunk's stored start, as in the sample pass
-          float acc = sh.chunk_lo;
-          for (int i = 0; i < kSegC; ++i) {
-            const float t = sh.seg[i];
-            sh.seg[i] = acc;
-            acc = __fadd_rn(acc, t);
+      } else {
+        const RowScalars rs = sample_scalars(sh.rj, sh.rj2, k);
+        // ---- inverse CDF over the slices in rank order, u = u[b][gamma], then
+        // over the chunks of the crossing slice
+        if (warp == 0) {
+          auto nch_of = [&](int r) {
+            const int len = max(0, min(P.L, P.V - r * P.L));
+            return (len + kCH - 1) / kCH;
+          };
+          const float tot = lane < C ? cpall[lane * kCP + nch_of(lane)] : 0.0f;
+          const float pre = warp_incl_scan(tot, lane);  // through rank `lane`
+          const float Rtot = __shfl_sync(0xFFFFFFFFu, pre, C - 1);
+          float before = __shfl_up_sync(0xFFFFFFFFu, pre, 1);
+          if (lane == 0) before = 0.0f;
+          const float u = __shfl_sync(0xFFFFFFFFu, ug, 0);
+          const bool ok = !sh.bad && isfinite(Rtot);
+          int cr = -1, cc = -1, clast = -1;
+          float2 tl = make_float2(-1.0f, 0.0f);  // (negative: u R fell past the last boundary)
+          if (ok && Rtot > 0.0f) {
+            const float th = __fmul_rn(u, Rtot);
+            const float2 t = make_float2(th, fmaf(u, Rtot, -th));  // u R_tot, exactly
+            const bool cross = lane < C && tot > 0.0f && df_ge(t, before) && df_lt(t, pre);
+            const unsigned cm = __ballot_sync(0xFFFFFFFFu, cross);
+            const unsigned pm = __ballot_sync(0xFFFFFFFFu, lane < C && tot > 0.0f);
+            cr = cm ? __ffs(cm) - 1 : 31 - __clz(pm);
+            const float bcr = __shfl_sync(0xFFFFFFFFu, before, cr);
+            if (cm) tl = df_sub(t, bcr);
+            // the chunk of slice cr holding tl (or, past a rounding gap, its last chunk with weight)
+            const float *cp = cpall + cr * kCP;
+            const int nch = nch_of(cr);
+            for (int base = 0; base < nch; base += 32) {
+              const int c = base + lane;
+              const float lo = c < nch ? cp[c] : 0.0f, hi = c < nch ? cp[c + 1] : 0.0f;
+              const bool pos = c < nch && hi > lo;
+              const unsigned mi = __ballot_sync(0xFFFFFFFFu, pos && df_ge(tl, lo) && df_lt(tl, hi));
+              const unsigned mp = __ballot_sync(0xFFFFFFFFu, pos);
+              if (cc < 0 && mi) cc = base + __ffs(mi) - 1;
+              if (mp) clast = base + 31 - __clz(mp);
+            }
           }
-          sh.seg[kSegC] = acc;
-          const float2 tl = sh.t_slice;
-          int sgi = -1;
-          if (sh.have_t)
-            for (int i = 0; i < kSegC; ++i)
-              if (df_ge(tl, sh.seg[i]) && df_lt(tl, sh.seg[i + 1]) && sh.seg[i + 1] > sh.seg[i]) {
-                sgi = i;
-                break;
-              }
-          sh.cross_seg = sgi;
-          sh.t_seg = sgi >= 0 ? df_floor(df_sub(tl, sh.seg[sgi])) : 0.0f;
+          if (lane == 0) {
+            sh.sample_ok = ok;
+            sh.cross_rank = cr;
+            sh.t_slice = tl;
+            sh.token = -1;
+            sh.cross_chunk = cc >= 0 ? cc : clast;
+            sh.have_t = cc >= 0;
+            sh.chunk_lo = sh.cross_chunk >= 0 ? cpall[cr * kCP + sh.cross_chunk] : 0.0f;
+          }
         }
         __syncthreads();
-        int sgi = sh.cross_seg;
-        if (sgi < 0) {
-          // no t inside the chunk: its last segment with weight
-          for (int i = kSegC - 1; i >= 0; --i)
-            if (sh.seg[i + 1] > sh.seg[i]) { sgi = i; break; }
+        const int cr = sh.cross_rank, cc = sh.cross_chunk;
+        if (cr >= 0 && cc >= 0) {
+          // the chunk's weights again, by the code the sample pass ran (the same values)
+          const Ring<E> Rc = make_ring<E>(P, smem_raw, b, js, cr);
+          const int sl = kStages - 1, n = Rc.chunk_len(cc);
+          if (Rc.bulk) {
+            if (tid == 0) Rc.issue(sh, cc, sl);
+            tmo = wait_stage(sh, sl, ph);
+          } else {
+            tmo = 0;
+            Rc.load_sync(cc, sl);
+          }
+          tmo = __syncthreads_or(tmo);
+          if (Rc.pair) {
+            if (n == kCH) weights_chunk<E, true, true, kTok>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
+            else weights_chunk<E, true, false, kTok>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
+          } else {
+            if (n == kCH) weights_chunk<E, false, true, kTok>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
+            else weights_chunk<E, false, false, kTok>(Rc.q(sl), Rc.p(sl), n, 0, rs, sh, lane, warp);
+          }
+          if (tmo && tid == 0) {
+            flag_timeout(sh, P);
+            sh.sample_ok = 0;
+          }
+          __syncthreads();
+          constexpr int kSegC = kRounds * kNW;  // segments per chunk
+          if (tid == 0) {
+            // exclusive prefixes continue from the chunk's stored start, as in the sample pass
+            float acc = sh.chunk_lo;
+            for (int i = 0; i < kSegC; ++i) {
+              const float t = sh.seg[i];
+              sh.seg[i] = acc;
+              acc = __fadd_rn(acc, t);
+            }
+            sh.seg[kSegC] = acc;
+            const float2 tl = sh.t_slice;
+            int sgi = -1;
+            if (sh.have_t)
+              for (int i = 0; i < kSegC; ++i)
+                if (df_ge(tl, sh.seg[i]) && df_lt(tl, sh.seg[i + 1]) && sh.seg[i + 1] > sh.seg[i]) {
+                  sgi = i;
+                  break;
+                }
+            sh.cross_seg = sgi;
+            sh.t_seg = sgi >= 0 ? df_floor(df_sub(tl, sh.seg[sgi])) : 0.0f;
+          }
+          __syncthreads();
+          int sgi = sh.cross_seg;
+          if (sgi < 0) {
+            // no t inside the chunk: its last segment with weight
+            for (int i = kSegC - 1; i >= 0; --i)
+              if (sh.seg[i + 1] > sh.seg[i]) { sgi = i; break; }
+          }
+          if (sgi >= 0 && warp == sgi % kNW) {
+            const int tok = search_segment<kTok>(Rc.q(sl), Rc.p(sl), n, Rc.pair, rs, cr * P.L + cc * kCH,
+                                           sgi / kNW, sh.cross_seg >= 0, sh.t_seg, lane, warp);
+            if (lane == 0) sh.token = tok;
+          }
+          __syncthreads();
         }
-        if (sgi >= 0 && warp == sgi % kNW) {
-          const int tok = search_segment<kTok>(Rc.q(sl), Rc.p(sl), n, Rc.pair, rs, cr * P.L + cc * kCH,
-                                         sgi / kNW, sh.cross_seg >= 0, sh.t_seg, lane, warp);
-          if (lane == 0) sh.token = tok;
+        if (tid == 0 && SC_CHECK(b < P.B && js >= 0 && js <= P.gamma)) {
+          const bool ok = sh.sample_ok != 0;
+          P.num_accepted[b] = ok ? js : 0;
+          P.next_token[b] = ok ? sh.token : -1;
+          if (ok && P.row_info)
+            P.row_info[(static_cast<size_t>(b) * G1 + js) * SC_ROW_FIELDS + SC_ROW_CAND] =
+                static_cast<float>(sh.token);
         }
-        __syncthreads();
-      }
-      if (tid == 0) {
-        const bool ok = sh.sample_ok != 0;
-        P.num_accepted[b] = ok ? js : 0;
-        P.next_token[b] = ok ? sh.token : -1;
-        if (ok && P.row_info)
-          P.row_info[(static_cast<size_t>(b) * G1 + js) * SC_ROW_FIELDS + SC_ROW_CAND] =
-              static_cast<float>(sh.token);
       }
     }
   }
-  if (sh.timeout && tid == 0 && R.bulk) {
+  }  // units
+  if (sh.timeout && tid == 0 && P.bulk) {
     // let copies still in flight land before this CTA's shared memory is released
     for (int s = 0; s < kStages; ++s) mbar_wait(&sh.full[s], 0), mbar_wait(&sh.full[s], 1);
   }
@@ -1341,7 +2008,8 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
 struct DeviceInfo {
   int smem_optin = 0;
   int sms = 0;
-  bool configured[4] = {false, false, false, false};  // [dtype][token rule]
+  bool configured[6] = {};  // [dtype][rule family]
+  int max_clusters[6][kMaxCluster + 1] = {};  // co-resident clusters per [kernel][C] (-1: unknown)
 };
 
 DeviceInfo g_dev[64];
@@ -1353,7 +2021,7 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 // sequence tickets (both zero between calls), then unit records and chunk
 // prefixes (written before they are read).
 struct WsLayout {
-  size_t rank_tickets, seq_tickets, zeroed, records, records2, chunk_pre, total;
+  size_t rank_tickets, seq_tickets, zeroed, records, records2, chunk_pre, bonus_pre, row_pre, total;
 };
 
 constexpr size_t align256(size_t x) { return (x + 255) / 256 * 256; }
@@ -1366,7 +2034,9 @@ constexpr WsLayout ws_layout(size_t B, size_t units) {
   w.records = w.zeroed;
   w.records2 = w.records + align256(16 * kMaxCluster * units);
   w.chunk_pre = w.records2 + align256(16 * kMaxCluster * units);
-  w.total = w.chunk_pre + align256(4 * kMaxCluster * (kMaxChunks + 1) * B);
+  w.bonus_pre = w.chunk_pre + align256(4 * kMaxCluster * (kMaxChunks + 1) * B);
+  w.row_pre = w.bonus_pre + align256(4 * kMaxCluster * (kMaxChunks + 1) * B);
+  w.total = w.row_pre + align256(4 * kMaxCluster * (kMaxChunks + 1) * units);
   return w;
 }
 
@@ -1414,8 +2084,23 @@ void set_k(Params &P, float temperature) {
   P.kl = static_cast<float>(kd - static_cast<double>(P.k));
 }
 
+// Set by each entry point: its stream is being captured into a CUDA graph.  The
+// pointer checks then only reject null pointers, so that nothing but the launch
+// itself happens inside the capture sequence.
+thread_local bool t_capturing = false;
+
+bool capturing(cudaStream_t stream) {
+  cudaStreamCaptureStatus st = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(stream, &st) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return st != cudaStreamCaptureStatusNone;
+}
+
 bool device_accessible(const void *p) {
   if (!p) return false;
+  if (t_capturing) return true;
   cudaPointerAttributes a;
   if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
     cudaGetLastError();
@@ -1424,17 +2109,24 @@ bool device_accessible(const void *p) {
   return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
 }
 
-// The kernel is compiled once per rule family: the token-specific rules of
-// Section 4.4 need per-logit r(v) in the weight passes, the SpecCascade rules
-// do not, and a runtime branch there costs the common case a few percent.
+// The rule family of a call (see Family): each family is its own kernel, so
+// the SpecCascade rules run without the per-logit branches of the others.
+int family_of(const Params &P) {
+  if (P.greedy || P.rule >= SC_RULE_BILD) return kFamExt;
+  if (P.rule >= SC_RULE_TOKEN_V1 && P.rule <= SC_RULE_TOKEN_V3) return kFamToken;
+  return kFamCascade;
+}
+
 template <typename E>
 int launch(Params P, cudaStream_t stream, int units) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return SC_ERR_CUDA;
   DeviceInfo &di = g_dev[dev];
-  const bool tok = P.rule >= SC_RULE_TOKEN_V1;
-  const auto kernel = tok ? sc_unit_kernel<E, true> : sc_unit_kernel<E, false>;
-  const int ti = (sizeof(E) == 2 ? 2 : 0) + (tok ? 1 : 0);
+  const int fam = family_of(P);
+  const auto kernel = fam == kFamExt     ? sc_unit_kernel<E, kFamExt>
+                      : fam == kFamToken ? sc_unit_kernel<E, kFamToken>
+                                         : sc_unit_kernel<E, kFamCascade>;
+  const int ti = (sizeof(E) == 2 ? 3 : 0) + fam;
   {
     std::lock_guard<std::mutex> lock(g_mu);
     if (!di.smem_optin &&
@@ -1456,13 +2148,19 @@ int launch(Params P, cudaStream_t stream, int units) {
   if (pick_layout(P.V, units, di.sms, &C, &L) != 0) return SC_ERR_UNSUPPORTED;
   P.L = L;
   P.cluster = C;
+  // Rejected pairs store their residual's prefixes themselves, right after their
+  // decision and from their ring and L2, unless their rank already shows an
+  // earlier rejection; the owners then never stream a second pass.
+  P.spec_res = 1;
+  if (const char *e = getenv("SC_SPEC_RES")) P.spec_res = atoi(e) != 0;
   const size_t row_bytes = static_cast<size_t>(P.V) * sizeof(E);
   P.bulk = (row_bytes % 16 == 0) && (reinterpret_cast<uintptr_t>(P.draft) % 16 == 0) &&
            (reinterpret_cast<uintptr_t>(P.target) % 16 == 0);
+  P.units = units;
   if (units == 0) return SC_OK;
 
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(static_cast<unsigned>(units) * static_cast<unsigned>(C), 1, 1);
+  cfg.gridDim = dim3(static_cast<unsigned>(C), 1, 1);
   cfg.blockDim = dim3(kNT, 1, 1);
   cfg.dynamicSmemBytes = smem_bytes<E>();
   cfg.stream = stream;
@@ -1473,16 +2171,33 @@ int launch(Params P, cudaStream_t stream, int units) {
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
+  // one cluster per unit, or (SC_PERSISTENT) as many as fit on the GPU at once,
+  // each looping over its share of the units; the kernel is correct for any grid
+  // since no cluster waits on another
+  int clusters = units;
+  if (SC_PERSISTENT) {
+    std::lock_guard<std::mutex> lock(g_mu);
+    int &mc = di.max_clusters[ti][C];
+    if (mc == 0) {
+      int n = 0;
+      mc = cudaOccupancyMaxActiveClusters(&n, kernel, &cfg) == cudaSuccess && n > 0 ? n : -1;
+      cudaGetLastError();
+    }
+    if (mc > 0 && mc < units) clusters = mc;
+  }
+  cfg.gridDim = dim3(static_cast<unsigned>(clusters) * static_cast<unsigned>(C), 1, 1);
   if (cudaLaunchKernelEx(&cfg, kernel, P) != cudaSuccess) return SC_ERR_CUDA;
   return SC_OK;
 }
 
+// greedy_ok: T = 0 (greedy decoding) is accepted.
 int common_checks(const void *draft, const void *target, int dtype, int B, int gamma, int V,
-                  float temperature) {
+                  float temperature, bool greedy_ok) {
   if (dtype != SC_F32 && dtype != SC_BF16) return SC_ERR_INVALID_ARG;
   if (B < 1 || gamma < 1 || gamma > SC_MAX_GAMMA || V < 1) return SC_ERR_INVALID_ARG;
   if (V > sc_max_vocab(static_cast<sc_dtype>(dtype))) return SC_ERR_UNSUPPORTED;
-  if (!(temperature > 0.0f) || !std::isfinite(temperature)) return SC_ERR_INVALID_ARG;
+  if (!(temperature > 0.0f || (greedy_ok && temperature == 0.0f)) || !std::isfinite(temperature))
+    return SC_ERR_INVALID_ARG;
   if (static_cast<double>(B) * (gamma + 1) * kMaxCluster > 2147483647.0) return SC_ERR_INVALID_ARG;
   if (!device_accessible(draft) || !device_accessible(target)) return SC_ERR_INVALID_ARG;
   return SC_OK;
@@ -1536,20 +2251,42 @@ int sc_workspace_init(void *workspace, size_t workspace_bytes, cudaStream_t stre
   return cudaMemsetAsync(workspace, 0, workspace_bytes, stream) == cudaSuccess ? SC_OK : SC_ERR_CUDA;
 }
 
+int sc_debug_line(int reset) {
+  if (!SC_DEBUG) return -1;
+  int line = 0;
+  if (cudaMemcpyFromSymbol(&line, g_sc_debug_line, sizeof(int)) != cudaSuccess) return SC_ERR_CUDA;
+  if (reset) {
+    const int zero = 0;
+    if (cudaMemcpyToSymbol(g_sc_debug_line, &zero, sizeof(int)) != cudaSuccess) return SC_ERR_CUDA;
+  }
+  return line;
+}
+
 int sc_max_vocab(sc_dtype dtype) {
   (void)dtype;  // the ring does not depend on V: one cluster covers kMaxCluster slices
   return kMaxCluster * kMaxChunks * kCH;
 }
 
-int sc_verify_rows(const void *draft_logits, const void *target_logits, sc_dtype dtype,
-                   const int32_t *draft_tokens, const float *uniforms, int B, int gamma, int V,
-                   sc_rule rule, float alpha, float temperature, int32_t *num_accepted,
-                   int32_t *next_token, void *workspace, size_t workspace_bytes,
-                   int32_t *device_status, float *row_info, cudaStream_t stream) {
-  int rc = common_checks(draft_logits, target_logits, dtype, B, gamma, V, temperature);
+int sc_verify_ex(const void *draft_logits, const void *target_logits, sc_dtype dtype,
+                 const int32_t *draft_tokens, const float *uniforms, int B, int gamma, int V,
+                 sc_rule rule, float alpha, float beta, float temperature, int32_t *num_accepted,
+                 int32_t *next_token, void *workspace, size_t workspace_bytes,
+                 int32_t *device_status, float *row_info, cudaStream_t stream) {
+  t_capturing = capturing(stream);
+  int rc = common_checks(draft_logits, target_logits, dtype, B, gamma, V, temperature, true);
   if (rc != SC_OK) return rc;
-  if (static_cast<int>(rule) < 0 || static_cast<int>(rule) > SC_RULE_TOKEN_V3) return SC_ERR_INVALID_ARG;
-  if (!(alpha >= 0.0f && alpha <= 1.0f)) return SC_ERR_INVALID_ARG;
+  const int ri = static_cast<int>(rule);
+  if (ri < 0 || ri > SC_RULE_OPT_LOG) return SC_ERR_INVALID_ARG;
+  // alpha: a probability-scale cost for Table 1, lossy and token rules, a
+  // threshold on a (cross) entropy for BiLD* and the log-loss rules
+  if (ri <= SC_RULE_LOSSY ? !(alpha >= 0.0f && alpha <= 1.0f) : !(alpha >= 0.0f && std::isfinite(alpha)))
+    return SC_ERR_INVALID_ARG;
+  const bool greedy = temperature == 0.0f;
+  // greedy decoding is defined for the scalar deferral rules only
+  if (greedy && ((ri >= SC_RULE_TOKEN_V1 && ri <= SC_RULE_TOKEN_V3) || ri == SC_RULE_LOSSY))
+    return SC_ERR_INVALID_ARG;
+  if (ri == SC_RULE_LOSSY && !(beta > 0.0f && std::isfinite(beta) && beta >= 1.0f - alpha))
+    return SC_ERR_INVALID_ARG;
   if (!device_accessible(draft_tokens) || !device_accessible(uniforms) ||
       !device_accessible(num_accepted) || !device_accessible(next_token))
     return SC_ERR_INVALID_ARG;
@@ -1566,10 +2303,19 @@ int sc_verify_rows(const void *draft_logits, const void *target_logits, sc_dtype
   P.B = B;
   P.gamma = gamma;
   P.V = V;
-  P.rule = static_cast<int>(rule);
+  P.rule = ri;
   P.alpha = alpha;
   P.temperature = temperature;
-  set_k(P, temperature);
+  P.greedy = greedy ? 1 : 0;
+  set_k(P, greedy ? 1.0f : temperature);  // greedy: the rules' statistics at T = 1
+  if (ri == SC_RULE_LOSSY) {
+    // -log2(1 - alpha) as hi + lo, and -log2(beta)
+    const double l = alpha < 1.0f ? -std::log2(1.0 - static_cast<double>(alpha)) : HUGE_VAL;
+    P.lossy_l = static_cast<float>(l);
+    P.lossy_ll = std::isfinite(l) ? static_cast<float>(l - static_cast<double>(P.lossy_l)) : 0.0f;
+    P.lossy_c = static_cast<float>(-std::log2(static_cast<double>(beta)));
+    P.beta = beta;
+  }
   P.mode = kVerify;
   P.num_accepted = num_accepted;
   P.next_token = next_token;
@@ -1582,8 +2328,20 @@ int sc_verify_rows(const void *draft_logits, const void *target_logits, sc_dtype
   P.records = reinterpret_cast<float4 *>(ws + wl.records);
   P.records2 = reinterpret_cast<float4 *>(ws + wl.records2);
   P.chunk_pre = reinterpret_cast<float *>(ws + wl.chunk_pre);
+  P.bonus_pre = reinterpret_cast<float *>(ws + wl.bonus_pre);
+  P.row_pre = reinterpret_cast<float *>(ws + wl.row_pre);
   const int units = B * (gamma + 1);
   return dtype == SC_BF16 ? launch<uint16_t>(P, stream, units) : launch<float>(P, stream, units);
+}
+
+int sc_verify_rows(const void *draft_logits, const void *target_logits, sc_dtype dtype,
+                   const int32_t *draft_tokens, const float *uniforms, int B, int gamma, int V,
+                   sc_rule rule, float alpha, float temperature, int32_t *num_accepted,
+                   int32_t *next_token, void *workspace, size_t workspace_bytes,
+                   int32_t *device_status, float *row_info, cudaStream_t stream) {
+  return sc_verify_ex(draft_logits, target_logits, dtype, draft_tokens, uniforms, B, gamma, V, rule,
+                      alpha, 1.0f, temperature, num_accepted, next_token, workspace, workspace_bytes,
+                      device_status, row_info, stream);
 }
 
 int sc_verify(const void *draft_logits, const void *target_logits, sc_dtype dtype,
@@ -1599,7 +2357,8 @@ int sc_verify(const void *draft_logits, const void *target_logits, sc_dtype dtyp
 int sc_row_stats(const void *draft_logits, const void *target_logits, sc_dtype dtype, int B,
                  int gamma, int V, float temperature, float *max_q, float *max_p, float *tv,
                  cudaStream_t stream) {
-  int rc = common_checks(draft_logits, target_logits, dtype, B, gamma, V, temperature);
+  t_capturing = capturing(stream);
+  int rc = common_checks(draft_logits, target_logits, dtype, B, gamma, V, temperature, false);
   if (rc != SC_OK) return rc;
   if (!device_accessible(max_q) || !device_accessible(max_p) || !device_accessible(tv))
     return SC_ERR_INVALID_ARG;

@@ -54,7 +54,10 @@ GEMMA_VOCAB = 256000
 
 # Default alpha per rule for the throughput sweep (the sweep leaves alpha open).
 SWEEP_ALPHA = {"chow": 0.5, "diff": 0.1, "opt": 0.2, "token_v1": 0.1, "token_v2": 0.1, "token_v3": 0.3,
-               "lossy": 0.3, "bild": 3.0}
+               "lossy": 0.3, "always": 0.0, "never": 0.0,
+               # thresholds in nats, near the medians of D(q, p), H(q) and H(q) - H(p) on
+               # the sweep's rows (about 7.4, 7.1 and 0.1)
+               "bild": 7.4, "chow_log": 7.1, "diff_log": 0.1, "opt_log": 0.5}
 SWEEP_POINTS = [(B, g) for B in (64, 256, 512) for g in (4, 8)]
 
 
@@ -300,8 +303,9 @@ CFG1_ALPHAS = (0.0, 0.1, 0.3, 0.5, 1.0)
 
 def config(cfg: int, *, seed: Optional[int] = None, rule: Optional[str] = None,
            alpha: Optional[float] = None, B: Optional[int] = None,
-           gamma: Optional[int] = None) -> Workload:
-    """The named workloads (seed defaults to the config id)."""
+           gamma: Optional[int] = None, temperature: Optional[float] = None) -> Workload:
+    """The named workloads (seed defaults to the config id).  ``temperature``
+    replaces the sweep's T = 1 (cfg 4 only; 0 is greedy decoding)."""
     s = cfg if seed is None else seed
     if cfg == 0:
         return synthetic(1, 4, T5_VOCAB, dtype="f32", kind="gauss", sigma=1.0,
@@ -327,5 +331,6 @@ def config(cfg: int, *, seed: Optional[int] = None, rule: Optional[str] = None,
             s = 100 + SWEEP_POINTS.index((B, gamma)) if (B, gamma) in SWEEP_POINTS else 100
         return synthetic(B, gamma, GEMMA_VOCAB, dtype="bf16", kind="zipf", sigma=0.7,
                          rule=rule, alpha=SWEEP_ALPHA[rule] if alpha is None else alpha,
-                         temperature=1.0, seed=s, name=f"cfg4(B={B},g={gamma},{rule})")
+                         temperature=1.0 if temperature is None else temperature, seed=s,
+                         name=f"cfg4(B={B},g={gamma},{rule})")
     raise ValueError(f"no config {cfg}")

@@ -79,6 +79,9 @@ int use_sc(const void *q, const void *p, const int32_t *x, const float *u, int32
   rc |= sc_verify_rows(q, p, SC_F32, x, u, 2, 3, 100, SC_RULE_TOKEN_V3, 0.3f, 0.7f, na, nt, ws, n, st, rows, s);
   rc |= sc_row_stats(q, p, SC_BF16, 2, 3, 100, 1.0f, mq, mp, tv, s);
   rc |= sc_verify_static(q, p, SC_BF16, x, u, 2, 3, 100, SC_RULE_DIFF, 0.1f, 1.0f, na, nt, st, s);
+  rc |= sc_verify_ex(q, p, SC_BF16, x, u, 2, 3, 100, SC_RULE_LOSSY, 0.3f, 0.9f, 1.0f, na, nt, ws, n, st, rows, s);
+  rc |= sc_verify(q, p, SC_BF16, x, u, 2, 3, 100, SC_RULE_OPT_LOG, 0.5f, 0.0f, na, nt, ws, n, st, s);
+  rc |= sc_debug_line(0);
   return rc + sc_max_vocab(SC_BF16) + (sc_status_string(rc) != 0);
 }
 """)

@@ -193,10 +193,13 @@ def test_degenerate_rows(sc):
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
-@pytest.mark.parametrize("rule,alpha", [("always", 0.0), ("opt", 0.2), ("token_v3", 0.3), ("token_v1", 0.1)])
+@pytest.mark.parametrize("rule,alpha", [("always", 0.0), ("opt", 0.2), ("token_v3", 0.3), ("token_v1", 0.1),
+                                        ("lossy", 0.3), ("lossy", 1.0)])
 def test_masked_target_logit_at_the_draft_token(sc, dtype, rule, alpha):
     # p(x) = 0 < q(x): pi(x)/q(x) = 1 - delta, so a deferred draft is rejected whatever
-    # its uniform; with both logits masked q(x) = 0 and the draft is accepted
+    # its uniform (lossy speculative decoding too, alpha = 1 being the limit
+    # alpha -> 1- of min(1, p/((1 - alpha) q)) = 0); with both logits masked q(x) = 0
+    # and the draft is accepted
     B, g, V = 8, 3, 600
     w = synthetic(B, g, V, dtype=dtype, kind="gauss", sigma=1.0, rule=rule, alpha=alpha, seed=41)
     ninf = np.uint16(0xFF80) if dtype == "bf16" else np.float32(-np.inf)
@@ -207,8 +210,49 @@ def test_masked_target_logit_at_the_draft_token(sc, dtype, rule, alpha):
     w.draft[1, 0, w.tokens[1, 0]] = ninf
     w.target[1, 0, w.tokens[1, 0]] = ninf
     ref = oracle.verify_workload(w)
-    if rule == "always":
+    if rule in ("always", "lossy"):
         assert np.all(ref.num_accepted[0::2] == 0)
+    assert_parity(w, run_gpu(sc, w), ref)
+
+
+@pytest.mark.parametrize("rule,alpha,T", [("opt", 0.3, 1.0), ("diff", 0.05, 0.7), ("token_v3", 0.3, 1.0),
+                                          ("chow", 0.5, 1.0)])
+def test_self_sampled_residuals_match_the_owners_pass(sc, monkeypatch, rule, alpha, T):
+    # a rejected pair storing its own residual prefixes (small batches) and the
+    # owner's sampling pass (large batches) sum the same weights with the same
+    # code: the draws are identical, and both match the oracle
+    w = synthetic(24, 6, 32128, dtype="bf16", kind="zipf", sigma=0.7, rule=rule, alpha=alpha,
+                  temperature=T, seed=61, force_reject_frac=0.5)
+    ref = oracle.verify_workload(w)
+    out = {}
+    for mode in ("0", "1"):
+        monkeypatch.setenv("SC_SPEC_RES", mode)
+        out[mode] = run_gpu(sc, w)
+        assert_parity(w, out[mode], ref)
+    np.testing.assert_array_equal(out["0"][0], out["1"][0])
+    np.testing.assert_array_equal(out["0"][1], out["1"][1])
+    assert np.any(ref.num_accepted < w.gamma) and np.any(ref.num_accepted == w.gamma)
+
+
+@pytest.mark.parametrize("rule,alpha", [("token_v3", 0.0), ("token_v3", 0.3), ("token_v2", 0.05), ("token_v1", 0.05)])
+def test_token_eta_screen_and_its_fallback(sc, rule, alpha):
+    # eta comes from the pass-1 screen when each thread holds at most one
+    # undeferred token, else from a pass over the row.  Sequences 0-1: many tied
+    # largest logits spread over the row (TokenV3 falls back; for TokenV1/V2
+    # max p < alpha, so nothing is deferred); 2-3: two tied largest logits in one
+    # thread's vector, q = p = 1/2 there (every rule falls back); the rest are
+    # ordinary rows (the screen)
+    B, g, V = 12, 4, 32128
+    w = synthetic(B, g, V, dtype="bf16", kind="zipf", sigma=0.7, rule=rule, alpha=alpha, seed=71)
+    top = np.uint16(0x4180)  # 16.0, above every sampled logit
+    for b in range(2):
+        w.draft[b, :, ::97] = top
+        w.target[b, :, ::89] = top
+    for b in (2, 3):
+        w.draft[b, :, 1000:1002] = top
+        w.target[b, :, 1000:1002] = top
+        w.tokens[b] = 1000 + b % 2
+    ref = oracle.verify_workload(w)
     assert_parity(w, run_gpu(sc, w), ref)
 
 
@@ -232,9 +276,11 @@ def test_host_argument_errors(sc):
     with pytest.raises(sc.SCError):
         sc.sc_verify(d, t, x, u, "opt", 1.5, 1.0)       # alpha outside [0, 1]
     with pytest.raises(sc.SCError):
-        sc.sc_verify(d, t, x, u, "opt", 0.2, 0.0)       # T = 0
+        sc.sc_verify(d, t, x, u, "opt", 0.2, -1.0)      # T < 0 (T = 0 is greedy decoding)
     with pytest.raises(sc.SCError):
-        sc.sc_verify(d, t, x, u, 9, 0.2, 1.0)           # unknown rule
+        sc.sc_verify(d, t, x, u, "token_v3", 0.2, 0.0)  # greedy decoding with a token rule
+    with pytest.raises(sc.SCError):
+        sc.sc_verify(d, t, x, u, 13, 0.2, 1.0)          # unknown rule
     with pytest.raises(sc.SCError):
         sc.sc_verify(d, t, x, u, "opt", 0.2, 1.0, workspace=torch.zeros(4, dtype=torch.uint8, device="cuda"))
     with pytest.raises(TypeError):
@@ -275,11 +321,51 @@ def test_repeatable_and_workspace_reuse(sc):
     np.testing.assert_array_equal(outs[1][1][ok], ref2.next_token[ok])
 
 
+@pytest.mark.parametrize("rule,alpha", [("opt", 0.0), ("token_v3", 0.3)])
+def test_cuda_graph_capture_and_replay(sc, rule, alpha):
+    # a decode loop can capture the verification in a CUDA graph: after one eager
+    # call (which configures the kernel), the captured launch replays on new inputs
+    # copied into the same buffers, reusing one workspace, and matches the oracle
+    import torch
+    wl = [synthetic(8, 5, 32128, dtype="bf16", kind="zipf", sigma=0.7, rule=rule, alpha=alpha,
+                    seed=s, force_reject_frac=0.5) for s in (81, 82, 83)]
+    w0 = wl[0]
+    d, t, x, u = sc.to_device(w0)
+    na = torch.empty(w0.B, dtype=torch.int32, device="cuda")
+    nt = torch.empty(w0.B, dtype=torch.int32, device="cuda")
+    ws = sc.new_workspace(w0.B, w0.gamma)
+
+    def call():
+        sc.sc_verify(d, t, x, u, rule, alpha, w0.temperature, num_accepted=na, next_token=nt, workspace=ws)
+
+    call()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        call()
+    torch.cuda.synchronize()
+    for w in wl + wl[:1]:
+        for dst, src in zip((d, t, x, u), sc.to_device(w)):
+            dst.copy_(src)
+        na.fill_(-9)
+        g.replay()
+        torch.cuda.synchronize()
+        ref = oracle.verify_workload(w)
+        ok = ~ref.flagged
+        assert ok.sum() >= w.B - 1
+        np.testing.assert_array_equal(na.cpu().numpy()[ok], ref.num_accepted[ok])
+        np.testing.assert_array_equal(nt.cpu().numpy()[ok], ref.next_token[ok])
+    assert torch.count_nonzero(ws[:(8 * 16 * w0.B + 255) // 256 * 256 + 256]).item() == 0  # tickets at rest
+
+
 @pytest.mark.parametrize("alpha", [0.2, 0.5, 1.0])
-def test_opt_band_settled_by_tv_lower_bound(sc, alpha):
+def test_opt_band_settled_by_tv_bounds(sc, alpha):
     # Inside the OPT band (max p - alpha <= max q < max p) the kernel first bounds
-    # D_TV from below by its threads' partial masses; rows the bound settles at
-    # delta = 0 report no TV (-1).  Their decisions must still be the oracle's.
+    # D_TV from below by its threads' partial masses (settling delta = 0) and from
+    # above by sqrt(1 - BC^2), BC = sum_v sqrt(q p) (settling delta = 1); settled
+    # rows report no TV (-1).  Their decisions must still be the oracle's.
+    from paper_2405_19261_gb300.workloads import logits_as_f64
+    from scipy.special import softmax
     w = synthetic(24, 8, 256000, dtype="bf16", kind="zipf", sigma=0.7, rule="opt", alpha=alpha,
                   temperature=1.0, seed=31)
     gpu = run_gpu(sc, w)
@@ -289,12 +375,20 @@ def test_opt_band_settled_by_tv_lower_bound(sc, alpha):
     maxq, maxp, tv = ref.row("maxq"), ref.row("maxp"), ri[..., 2]
     band = (maxq < maxp) & (maxq >= maxp - alpha)
     settled = band & (tv < 0)
-    assert settled.sum() > 0, "no band row was settled by the bound"
-    np.testing.assert_array_equal(ri[..., 3][settled], 0.0)
-    np.testing.assert_array_equal(ref.row("delta")[settled], 0.0)
+    assert settled.sum() > 0, "no band row was settled by a bound"
+    np.testing.assert_array_equal(ri[..., 3][settled], ref.row("delta")[settled])
     # the rows left to the TV pass report an exact D_TV
     exact = band & ~settled
     np.testing.assert_allclose(tv[exact], ref.row("tv")[exact], atol=TOL)
+    # every band row whose Hellinger bound clearly decides delta = 1 was settled by
+    # it (the kernel shrinks BC by 2e-4 before the bound, far past its f32 error)
+    q = softmax(logits_as_f64(w.draft, "bf16"), axis=-1)
+    p = softmax(logits_as_f64(w.target[:, :w.gamma], "bf16"), axis=-1)
+    bc = np.minimum(1.0, np.sum(np.sqrt(q * p), axis=-1)) * (1.0 - 2e-4)
+    ub = np.sqrt(np.maximum(0.0, 1.0 - bc ** 2))
+    clear = band & (maxp - maxq - alpha * ub >= 1e-3)
+    np.testing.assert_array_equal(tv[clear], -1.0)
+    np.testing.assert_array_equal(ri[..., 3][clear], 1.0)
 
 
 # ----------------------------------------------------------------- maximum sizes

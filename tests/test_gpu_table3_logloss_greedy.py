@@ -1,0 +1,329 @@
+"""Parity of the CUDA verification step with the fp64 oracle for the other
+targets of Table 3 (lossy speculative decoding, BiLD*), the plug-in rules for
+the log loss, and greedy decoding at T = 0 (GPU only).
+
+Bar: as for the SpecCascade rules (num_accepted and next_token bit-exact on
+every sequence the oracle does not flag; max q, max p, D_TV, q(x) and pi(x)
+within 1e-5; decisions equal where their margin is at least 1e-6), except that
+a decision made by an entropy or a cross entropy is compared only where the
+oracle's margin is at least ENT_MARGIN nats, and a sequence with a closer such
+decision at or before j* is not compared bit-exactly.  Those values are 6-9
+nats here, and the kernel sums their f32 terms over up to 2^20 logits: a
+relative error of a few 1e-6 at worst, well inside 1e-4 nats.
+"""
+import numpy as np
+import pytest
+
+import oracle
+from helpers import load_golden, rows_workload
+from paper_2405_19261_gb300.workloads import config, logits_as_f64, synthetic
+
+pytestmark = pytest.mark.gpu
+
+TOL = 1e-5
+ENT_MARGIN = 1e-4
+ENTROPY_RULES = ("bild", "chow_log", "diff_log", "opt_log")
+
+
+@pytest.fixture(scope="module")
+def sc():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2405_19261_gb300 import binding
+    binding.lib()
+    return binding
+
+
+def run_gpu(sc, w, beta=1.0, temperature=None):
+    import torch
+    d, t, x, u = sc.to_device(w)
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    ri = torch.full((w.B, w.gamma + 1, sc.ROW_FIELDS), -7.0, dtype=torch.float32, device="cuda")
+    na, nt = sc.sc_verify(d, t, x, u, w.rule, w.alpha, w.temperature if temperature is None else temperature,
+                          beta=beta, status=status, row_info=ri)
+    torch.cuda.synchronize()
+    return na.cpu().numpy(), nt.cpu().numpy(), ri.cpu().numpy(), int(status.item())
+
+
+def assert_parity(w, gpu, ref, min_compared=0.8):
+    na, nt, ri, status = gpu
+    assert status == 0
+    g = w.gamma
+    delta_margin = ENT_MARGIN if w.rule in ENTROPY_RULES else oracle.FLAG_MARGIN
+    md, ma = ref.row("margin_delta"), ref.row("margin_accept")
+    reach = np.arange(g)[None, :] <= ref.num_accepted[:, None]
+    ok = ~(ref.flagged | ((md < delta_margin) & reach).any(1))
+    assert ok.mean() >= min_compared, f"{w.name}: only {ok.sum()} of {w.B} sequences comparable"
+    bad = np.nonzero(ok & ((na != ref.num_accepted) | (nt != ref.next_token)))[0]
+    assert len(bad) == 0, (f"{w.name}: {len(bad)} unflagged mismatches, first b={bad[:5]}, "
+                           f"gpu={na[bad[:5]]},{nt[bad[:5]]} oracle={ref.num_accepted[bad[:5]]},{ref.next_token[bad[:5]]}")
+    R = ri[:, :g]
+    np.testing.assert_allclose(R[..., 0], ref.row("maxq"), atol=TOL)
+    np.testing.assert_allclose(R[..., 1], ref.row("maxp"), atol=TOL)
+    np.testing.assert_allclose(ri[:, g, 1], ref.seqs[:, oracle.SEQ["bonus_maxp"]], atol=TOL)
+    tv = R[..., 2]
+    have = tv >= 0
+    np.testing.assert_allclose(tv[have], ref.row("tv")[have], atol=TOL)
+    sure_d = md >= delta_margin
+    np.testing.assert_array_equal(R[..., 3][sure_d], ref.row("delta")[sure_d])
+    same_d = R[..., 3] == ref.row("delta")
+    sure_a = sure_d & (ma >= oracle.FLAG_MARGIN)
+    np.testing.assert_array_equal(R[..., 4][sure_a], ref.row("accept")[sure_a])
+    np.testing.assert_allclose(R[..., 5], ref.row("qx"), atol=TOL)
+    np.testing.assert_allclose(R[..., 6][same_d], ref.row("pix")[same_d], atol=TOL)
+    # the finisher marks row j* with the emitted token
+    cand = ri[np.arange(w.B), na, 7]
+    np.testing.assert_array_equal(cand[ok], nt[ok])
+
+
+def _sampled(sc, w, nseq, beta=1.0, seed=0):
+    gpu = run_gpu(sc, w, beta=beta)
+    pick = np.sort(np.random.default_rng(seed).choice(w.B, size=min(nseq, w.B), replace=False))
+    sub = w.subset(pick)
+    ref = oracle.verify_workload(sub, beta=beta)
+    na, nt, ri, status = gpu
+    assert_parity(sub, (na[pick], nt[pick], ri[pick], status), ref)
+
+
+# ----------------------------------------------------------------- hand-worked goldens
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_worked_examples(sc, dtype):
+    g = load_golden("table3_logloss_examples.json")
+    for ex in g["examples"]:
+        for c in ex["cases"]:
+            w = rows_workload(ex["q"], ex["p"], c["tokens"], c["u"], c["rule"], c["alpha"], dtype=dtype, B=3)
+            w.temperature = c["T"]
+            beta = c.get("beta", 1.0)
+            ref = oracle.verify_workload(w, beta=beta)
+            na, nt, ri, status = run_gpu(sc, w, beta=beta)
+            assert status == 0
+            if dtype == "f32":   # bf16 rounding of the log-probabilities moves no decision here either
+                assert (na[0], nt[0]) == (c["num_accepted"], c["next_token"]), (ex["name"], c)
+            ok = ~ref.flagged
+            np.testing.assert_array_equal(na[ok], ref.num_accepted[ok])
+            np.testing.assert_array_equal(nt[ok], ref.next_token[ok])
+
+
+# ----------------------------------------------------------------- lossy speculative decoding
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("alpha,beta", [(0.0, 1.0), (0.1, 1.0), (0.3, 0.8), (0.5, 0.5), (0.3, 1.5), (1.0, 1.0)])
+def test_lossy_t5_shape(sc, dtype, alpha, beta):
+    w = synthetic(16, 5, 32128, dtype=dtype, kind="zipf", sigma=0.7, rule="lossy", alpha=alpha,
+                  temperature=0.8, seed=int(100 * alpha + 10 * beta))
+    assert_parity(w, run_gpu(sc, w, beta=beta), oracle.verify_workload(w, beta=beta))
+
+
+def test_lossy_at_alpha_0_beta_1_is_speculative_sampling(sc):
+    # pi = max{min{q, p}, p} = p: the same accepted counts and tokens as delta = 1
+    w = synthetic(24, 5, 32128, dtype="bf16", kind="zipf", sigma=0.7, rule="lossy", alpha=0.0, seed=5)
+    na, nt, _, _ = run_gpu(sc, w, beta=1.0)
+    w.rule = "always"
+    na2, nt2, _, _ = run_gpu(sc, w)
+    np.testing.assert_array_equal(na, na2)
+    np.testing.assert_array_equal(nt, nt2)
+
+
+@pytest.mark.parametrize("V", [1, 7, 4097, 8193])
+def test_lossy_ragged_vocab(sc, V):
+    w = synthetic(5, 3, V, dtype="bf16", kind="gauss", sigma=1.0, rule="lossy", alpha=0.2, seed=V)
+    assert_parity(w, run_gpu(sc, w, beta=0.9), oracle.verify_workload(w, beta=0.9))
+
+
+# ----------------------------------------------------------------- BiLD* and the log-loss rules
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("rule,alpha", [("bild", 6.3), ("bild", 6.6), ("chow_log", 6.0), ("chow_log", 6.4),
+                                        ("diff_log", 0.0), ("diff_log", 0.1), ("opt_log", 0.2),
+                                        ("opt_log", 0.5), ("opt_log", 1.0)])
+def test_entropy_rules_t5_shape(sc, dtype, rule, alpha):
+    w = synthetic(16, 5, 32128, dtype=dtype, kind="zipf", sigma=0.7, rule=rule, alpha=alpha, seed=7)
+    assert_parity(w, run_gpu(sc, w), oracle.verify_workload(w))
+
+
+@pytest.mark.parametrize("rule,alpha", [("bild", 8.9), ("chow_log", 8.45), ("diff_log", 0.45), ("opt_log", 0.6)])
+def test_entropy_rules_flat_rows_and_temperature(sc, rule, alpha):
+    w = synthetic(12, 4, 32128, dtype="bf16", kind="gauss", sigma=1.0, rule=rule, alpha=alpha,
+                  temperature=1.0, seed=9)
+    assert_parity(w, run_gpu(sc, w), oracle.verify_workload(w))
+    w = synthetic(12, 4, 32128, dtype="bf16", kind="zipf", sigma=0.7, rule=rule, alpha=alpha / 2,
+                  temperature=0.6, seed=10)
+    assert_parity(w, run_gpu(sc, w), oracle.verify_workload(w), min_compared=0.5)
+
+
+@pytest.mark.parametrize("alpha", [0.3, 0.6])
+def test_opt_log_band_settled_by_tv_bounds(sc, alpha):
+    # OPTLog's band (sum p ln p - alpha <= sum q ln q < sum p ln p) is narrowed like
+    # OPT's: the partition bound settles delta = 0, sqrt(1 - BC^2) settles delta = 1;
+    # settled rows report no TV, and every row the upper bound clearly decides is settled
+    from scipy.special import softmax
+    from scipy.stats import entropy
+    w = synthetic(24, 6, 32128, dtype="bf16", kind="zipf", sigma=0.7, rule="opt_log", alpha=alpha, seed=73)
+    gpu = run_gpu(sc, w)
+    ref = oracle.verify_workload(w)
+    assert_parity(w, gpu, ref)
+    ri = gpu[2][:, :w.gamma]
+    q = softmax(logits_as_f64(w.draft, "bf16"), axis=-1)
+    p = softmax(logits_as_f64(w.target[:, :w.gamma], "bf16"), axis=-1)
+    gap = entropy(q, axis=-1) - entropy(p, axis=-1)          # sum p ln p - sum q ln q
+    band = (gap > 0) & (gap <= alpha)
+    bc = np.minimum(1.0, np.sum(np.sqrt(q * p), axis=-1)) * (1.0 - 2e-4)  # as the kernel shrinks it
+    ub = np.sqrt(np.maximum(0.0, 1.0 - bc ** 2))
+    clear = band & (gap - alpha * ub >= 1e-3)
+    assert clear.sum() > 0
+    np.testing.assert_array_equal(ri[..., 2][clear], -1.0)
+    np.testing.assert_array_equal(ri[..., 3][clear], 1.0)
+    np.testing.assert_array_equal(ref.row("delta")[clear], 1.0)
+
+
+@pytest.mark.parametrize("V,dtype", [(9, "bf16"), (4095, "f32"), (8193, "bf16")])
+@pytest.mark.parametrize("rule", ["bild", "opt_log"])
+def test_entropy_rules_ragged_vocab(sc, V, dtype, rule):
+    w = synthetic(5, 3, V, dtype=dtype, kind="gauss", sigma=1.0, rule=rule,
+                  alpha=0.9 * np.log(V) if rule == "bild" else 0.3, seed=V)
+    assert_parity(w, run_gpu(sc, w), oracle.verify_workload(w), min_compared=0.6)
+
+
+@pytest.mark.parametrize("rule", ["bild", "chow_log", "diff_log", "opt_log", "lossy"])
+@pytest.mark.parametrize("T", [1.0, 0.0])
+def test_single_token_vocabulary(sc, rule, T):
+    # V = 1: q = p = 1, every entropy and D(q, p) is 0 and every decision a tie,
+    # yet pi(x)/q(x) = 1 whatever delta is: all drafts kept, token 0 emitted
+    if rule == "lossy" and T == 0.0:
+        pytest.skip("greedy decoding is defined for the scalar deferral rules")
+    w = synthetic(4, 3, 1, dtype="f32", kind="gauss", sigma=1.0, rule=rule, alpha=0.0, temperature=T, seed=1)
+    na, nt, _, status = run_gpu(sc, w)
+    assert status == 0
+    np.testing.assert_array_equal(na, 3)
+    np.testing.assert_array_equal(nt, 0)
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("rule,alpha,beta", [("lossy", 0.3, 0.9), ("bild", 7.4, 1.0), ("opt_log", 0.5, 1.0)])
+def test_gemma_shape_sampled(sc, rule, alpha, beta):
+    _sampled(sc, config(4, B=64, gamma=4, rule=rule, alpha=alpha), nseq=6, beta=beta)
+
+
+@pytest.mark.parametrize("rule,alpha,beta", [("lossy", 0.3, 0.8), ("bild", 6.5, 1.0), ("opt_log", 0.5, 1.0),
+                                             ("diff_log", 0.1, 1.0)])
+def test_self_sampled_residuals_match_the_owners_pass(sc, monkeypatch, rule, alpha, beta):
+    # the lossy residual's shifted constant and the moment kernel's rows (OPTLog
+    # band rows reuse their TV pass) through both sampling paths: same draws
+    w = synthetic(24, 6, 32128, dtype="bf16", kind="zipf", sigma=0.7, rule=rule, alpha=alpha, seed=62,
+                  force_reject_frac=0.5)
+    ref = oracle.verify_workload(w, beta=beta)
+    out = {}
+    for mode in ("0", "1"):
+        monkeypatch.setenv("SC_SPEC_RES", mode)
+        out[mode] = run_gpu(sc, w, beta=beta)
+        assert_parity(w, out[mode], ref)
+    np.testing.assert_array_equal(out["0"][0], out["1"][0])
+    np.testing.assert_array_equal(out["0"][1], out["1"][1])
+
+
+# ----------------------------------------------------------------- greedy decoding (T = 0)
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("rule,alpha", [("chow", 0.5), ("diff", 0.1), ("opt", 0.1), ("always", 0.0),
+                                        ("never", 0.0), ("bild", 2.27), ("chow_log", 6.2),
+                                        ("diff_log", 0.1), ("opt_log", 0.3)])
+def test_greedy_t5_shape(sc, dtype, rule, alpha):
+    w = synthetic(16, 5, 32128, dtype=dtype, kind="zipf", sigma=0.7, rule=rule, alpha=alpha,
+                  temperature=0.0, seed=11)
+    ref = oracle.verify_workload(w)
+    assert_parity(w, run_gpu(sc, w), ref)
+
+
+def test_greedy_always_defer_is_greedy_speculative_decoding(sc):
+    # drafts are q's argmaxes; each is kept while it is also p's argmax, and the
+    # emitted token is p's argmax at the first disagreement (or at the bonus row)
+    w = synthetic(32, 6, 32128, dtype="bf16", kind="zipf", sigma=0.5, rule="always", alpha=0.0,
+                  temperature=0.0, seed=12)
+    na, nt, _, status = run_gpu(sc, w)
+    assert status == 0
+    q = logits_as_f64(w.draft, "bf16")
+    p = logits_as_f64(w.target, "bf16")
+    aq, ap = q.argmax(-1), p.argmax(-1)
+    assert np.array_equal(w.tokens, aq)
+    agree = aq == ap[:, :w.gamma]
+    js = np.where(agree.all(1), w.gamma, (~agree).argmax(1))
+    np.testing.assert_array_equal(na, js)
+    np.testing.assert_array_equal(nt, ap[np.arange(w.B), js])
+
+
+def test_greedy_opt_equals_greedy_diff(sc):
+    # with one-hot rows D_TV is 0 exactly when the argmaxes agree, and then the
+    # draft is kept whatever delta is; otherwise D_TV = 1 and OPT is Diff
+    w = synthetic(32, 5, 32128, dtype="bf16", kind="zipf", sigma=0.7, rule="opt", alpha=0.1,
+                  temperature=0.0, seed=13)
+    a = run_gpu(sc, w)
+    w.rule = "diff"
+    b = run_gpu(sc, w)
+    np.testing.assert_array_equal(a[0], b[0])
+    np.testing.assert_array_equal(a[1], b[1])
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_greedy_ties_take_the_lowest_index(sc, dtype):
+    # equal largest logits in several slices, warps and lanes of a row: the
+    # argmax is the lowest index, on the draft and the target side alike
+    B, g, V = 4, 3, 32128
+    w = synthetic(B, g, V, dtype=dtype, kind="gauss", sigma=1.0, rule="always", alpha=0.0,
+                  temperature=0.0, seed=14)
+    top = np.uint16(0x4200) if dtype == "bf16" else np.float32(32.0)   # 32.0, above every sampled logit
+    ties = [[7, 9000, 31000], [4096, 4097, 20000], [31999, 32127], [0, 8, 16]]
+    for b in range(B):
+        for j in range(g + 1):
+            for v in ties[b]:
+                w.target[b, j, v] = top
+                if j < g:
+                    w.draft[b, j, v] = top
+        w.tokens[b] = min(ties[b])
+    # sequence 3: the target's tie moves up one row at j = 1, so the draft there is rejected
+    w.target[3, 1, 0] = w.target[3, 1, 1]
+    ref = oracle.verify_workload(w)
+    gpu = run_gpu(sc, w)
+    assert_parity(w, gpu, ref)
+    na, nt, _, _ = gpu
+    np.testing.assert_array_equal(na, [g, g, g, 1])
+    np.testing.assert_array_equal(nt, [7, 4096, 31999, 8])
+
+
+def test_greedy_and_lossy_argument_checks(sc):
+    w = synthetic(2, 2, 64, dtype="f32", kind="gauss", seed=1)
+    d, t, x, u = sc.to_device(w)
+    for rule, alpha, beta, T in [("token_v3", 0.3, 1.0, 0.0),   # greedy needs a scalar rule
+                                 ("lossy", 0.3, 1.0, 0.0),
+                                 ("lossy", 0.3, 0.5, 1.0),      # beta < 1 - alpha
+                                 ("lossy", 0.3, 0.0, 1.0),
+                                 ("bild", -1.0, 1.0, 1.0),      # a threshold in nats is >= 0
+                                 ("opt", 1.5, 1.0, 0.0),
+                                 (13, 0.1, 1.0, 1.0)]:
+        with pytest.raises(sc.SCError):
+            sc.sc_verify(d, t, x, u, rule, alpha, T, beta=beta)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_bild_infinite_discrepancy_on_a_masked_target_token(sc, dtype):
+    # D(q, p) = -sum_v q log p is +inf when some token has a finite draft logit
+    # (q(v) > 0) and a masked target logit (p(v) = 0), however far below the
+    # draft's largest logit it lies: 200 nats (2^a underflows in f32) or 2000 (exp
+    # underflows in fp64).  Such a pair defers (delta = 1) whatever alpha is.
+    from paper_2405_19261_gb300.workloads import f32_to_bf16_bits
+    B, g, V = 6, 3, 4099
+    w = synthetic(B, g, V, dtype=dtype, kind="gauss", sigma=1.0, rule="bild", alpha=1e6, seed=77)
+    dq = logits_as_f64(w.draft, dtype)
+
+    def put(arr, idx, val):
+        arr[idx] = f32_to_bf16_bits(np.float32(val))[0] if dtype == "bf16" else np.float32(val)
+
+    for b in range(B):
+        j, v = b % g, (4097 if b % 2 else 11)   # in the ragged last chunk, or the first
+        put(w.draft, (b, j, v), dq[b, j].max() - (200.0 if b < 3 else 2000.0))
+        put(w.target, (b, j, v), -np.inf)
+    ref = oracle.verify_workload(w)
+    for b in range(B):
+        assert ref.row("delta")[b, b % g] == 1, b
+    assert_parity(w, run_gpu(sc, w), ref)

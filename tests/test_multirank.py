@@ -27,6 +27,8 @@ class _Args:
     alpha = None
     B = None
     gamma = None
+    beta = 1.0
+    temperature = None
 
 
 def _worker(rank, world, port, queue):
