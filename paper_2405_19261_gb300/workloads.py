@@ -119,13 +119,14 @@ class Workload:
 
 # ---------------------------------------------------------------- bit helpers
 
-def _row_blocks(n_rows: int, row_len: int, fn) -> None:
+def _row_blocks(n_rows: int, row_len: int, fn, threads: bool = True) -> None:
     """fn(i0, i1) over blocks of rows, on a thread pool when the work is large
     (numpy releases the GIL inside its element-wise loops, and each element's
-    result does not depend on how the rows are split)."""
+    result does not depend on how the rows are split).  ``threads=False`` runs
+    the blocks in this thread (a caller that is itself one of a pool's tasks)."""
     per = max(1, (1 << 18) // max(1, row_len))  # ~256K elements per task
     blocks = [(i, min(n_rows, i + per)) for i in range(0, n_rows, per)]
-    if len(blocks) < 2 or n_rows * row_len < (1 << 20):
+    if not threads or len(blocks) < 2 or n_rows * row_len < (1 << 20):
         for i0, i1 in blocks:
             fn(i0, i1)
         return
@@ -133,7 +134,7 @@ def _row_blocks(n_rows: int, row_len: int, fn) -> None:
         list(ex.map(lambda bl: fn(*bl), blocks))
 
 
-def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
+def f32_to_bf16_bits(x: np.ndarray, threads: bool = True) -> np.ndarray:
     """Round float32 to bf16 (nearest, ties to even); returns uint16 bits.
 
     Inputs must be finite (the generators only make finite values)."""
@@ -148,7 +149,7 @@ def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
         b = b + (np.uint32(0x7FFF) + ((b >> np.uint32(16)) & np.uint32(1)))
         o2[i0:i1] = b >> np.uint32(16)
 
-    _row_blocks(b2.shape[0], n, work)
+    _row_blocks(b2.shape[0], n, work, threads)
     return out
 
 
@@ -170,7 +171,8 @@ def draw_uniforms(rng: np.random.Generator, shape) -> np.ndarray:
     return (k.astype(np.float64) * 2.0 ** -24).astype(np.float32)
 
 
-def gumbel_argmax(rng: np.random.Generator, y: np.ndarray, temperature: float) -> np.ndarray:
+def gumbel_argmax(rng: np.random.Generator, y: np.ndarray, temperature: float,
+                  threads: bool = True) -> np.ndarray:
     """One exact sample per row from softmax(y / T) by the Gumbel-max trick; with
     T = 0 (greedy decoding) the row's argmax, lowest index on ties."""
     y = np.asarray(y, dtype=np.float64)
@@ -192,7 +194,7 @@ def gumbel_argmax(rng: np.random.Generator, y: np.ndarray, temperature: float) -
         s += g
         out[i0:i1] = np.argmax(s, axis=-1)
 
-    _row_blocks(y2.shape[0], n, work)
+    _row_blocks(y2.shape[0], n, work, threads)
     return out.reshape(y.shape[:-1])
 
 
@@ -217,8 +219,8 @@ def _zipf_rows(rng, n, V):
     return out
 
 
-def _store(x: np.ndarray, dtype: str) -> np.ndarray:
-    return f32_to_bf16_bits(x) if dtype == "bf16" else np.ascontiguousarray(x, dtype=np.float32)
+def _store(x: np.ndarray, dtype: str, threads: bool = True) -> np.ndarray:
+    return f32_to_bf16_bits(x, threads) if dtype == "bf16" else np.ascontiguousarray(x, dtype=np.float32)
 
 
 def synthetic(B: int, gamma: int, V: int, *, dtype: str = "bf16", kind: str = "zipf",
@@ -240,7 +242,8 @@ def synthetic(B: int, gamma: int, V: int, *, dtype: str = "bf16", kind: str = "z
     if rule not in RULES:
         raise ValueError(f"rule {rule!r}")
     ss = np.random.SeedSequence(seed)
-    g_logit, g_tok, g_u, g_force, g_sigma = (np.random.default_rng(s) for s in ss.spawn(5))
+    s_logit, s_tok, s_u, s_force, s_sigma = ss.spawn(5)
+    g_u, g_force, g_sigma = (np.random.default_rng(s) for s in (s_u, s_force, s_sigma))
     rows_fn = _zipf_rows if kind == "zipf" else _gauss_rows
     elt = np.uint16 if dtype == "bf16" else np.float32
     draft = np.empty((B, gamma, V), dtype=elt)
@@ -252,33 +255,50 @@ def synthetic(B: int, gamma: int, V: int, *, dtype: str = "bf16", kind: str = "z
     else:
         sig = np.full((B, gamma + 1), sigma, dtype=np.float32)
     forced = np.full(B, -1, dtype=np.int32)
+    y_forced = np.zeros(B, dtype=np.int64)
     if force_reject_frac > 0:
         hit = g_force.random(B) < force_reject_frac
         j0 = g_force.integers(0, min(2, gamma), size=B)
         forced[hit] = j0[hit]
+        y_forced = g_force.integers(0, max(1, V - 1), size=B)  # then shifted past x: uniform over V \ {x}
 
-    # Sequences are drawn in blocks to bound the float32 temporaries.
+    # Sequences are drawn in blocks (bounding the float32 temporaries), each
+    # block from its own child streams of the logit and token generators, so
+    # the blocks run on a thread pool and the bytes do not depend on the order
+    # in which they finish.
     seq_block = max(1, block_rows // (2 * gamma + 1))
-    for b0 in range(0, B, seq_block):
-        b1 = min(B, b0 + seq_block)
+    blocks = [(b0, min(B, b0 + seq_block)) for b0 in range(0, B, seq_block)]
+    ss_logit, ss_tok = s_logit.spawn(len(blocks)), s_tok.spawn(len(blocks))
+
+    def block(i):
+        b0, b1 = blocks[i]
         nb = b1 - b0
+        g_logit, g_tok = np.random.default_rng(ss_logit[i]), np.random.default_rng(ss_tok[i])
         d = rows_fn(g_logit, nb * (gamma + 1), V).reshape(nb, gamma + 1, V)
         noise = g_logit.standard_normal((nb, gamma + 1, V), dtype=np.float32)
         t = d + noise * sig[b0:b1, :, None]
         # Position gamma's draft-like row only seeds the bonus target row.
-        d = d[:, :gamma, :]
-        dq = _store(d, dtype)
+        dq = _store(d[:, :gamma, :], dtype, threads=False)
         draft[b0:b1] = dq
         dq64 = logits_as_f64(dq, dtype)
-        tokens[b0:b1] = gumbel_argmax(g_tok, dq64.reshape(nb * gamma, V), temperature).reshape(nb, gamma)
+        tokens[b0:b1] = gumbel_argmax(g_tok, dq64.reshape(nb * gamma, V), temperature,
+                                      threads=False).reshape(nb, gamma)
         for bb in range(nb):
             j0 = forced[b0 + bb]
             if j0 >= 0:
                 x = tokens[b0 + bb, j0]
-                y = int(g_force.integers(0, V - 1))
-                y = y + 1 if y >= x else y  # uniform over V \ {x}
+                y = int(y_forced[b0 + bb])
+                y = y + 1 if y >= x else y
                 t[bb, j0, y] = t[bb, j0].max() + np.float32(force_boost)
-        target[b0:b1] = _store(t, dtype)
+        target[b0:b1] = _store(t, dtype, threads=False)
+
+    workers = min(len(blocks), os.cpu_count() or 1)
+    if workers < 2 or B * (2 * gamma + 1) * V < (1 << 22):
+        for i in range(len(blocks)):
+            block(i)
+    else:
+        with ThreadPoolExecutor(max_workers=workers) as ex:
+            list(ex.map(block, range(len(blocks))))
 
     u = draw_uniforms(g_u, (B, gamma + 1))
     return Workload(name=name or f"synthetic(B={B},g={gamma},V={V},{dtype},{kind})",
