@@ -272,10 +272,12 @@ static int token_r(int rule, double alpha, double qv, double pv, double maxp, do
  * The token-specific target of one row: r(v) for every token, eta = sum_v r(v) q(v)
  * and pi(v) = q(v) (1 - r(v)) + eta p(v).  r is written to rv[] (0/1); the
  * returned margin is the smallest per-token margin among tokens with q(v) or
- * p(v) of at least 1e-9 (flipping a lighter token moves eta and pi by less).
+ * p(v) of at least 1e-9 (flipping a lighter token moves eta and pi by less),
+ * and always includes that of the draft token x (x < 0: none), whose own r(x)
+ * decides whether it is kept outright, whatever its mass.
  */
 static double token_target(int rule, double alpha, const void *zp, int dtype, size_t poff, double Mp,
-                           double T, const double *q, const double *p, int V, double maxp,
+                           double T, const double *q, const double *p, int V, double maxp, int x,
                            double *rv, double *pi, double *margin)
 {
     csum eta = {0.0, 0.0};
@@ -286,7 +288,7 @@ static double token_target(int rule, double alpha, const void *zp, int dtype, si
         const int r = token_r(rule, alpha, q[v], p[v], maxp, lnp_rel, &m);
         rv[v] = r;
         if (r) csum_add(&eta, q[v]);
-        if ((q[v] >= 1e-9 || p[v] >= 1e-9) && m < mmin) mmin = m;
+        if ((q[v] >= 1e-9 || p[v] >= 1e-9 || v == x) && m < mmin) mmin = m;
     }
     const double e = csum_value(&eta);
     if (pi)
@@ -429,7 +431,8 @@ static void verify_sequence(const void *draft, const void *target, int dtype,
         if (token) {
             /* token-specific target (TokenSpecCascade): w holds r(v) for this row */
             const double eta = token_target(rule, alpha, target, dtype, tbase + (size_t)j * V, Mp, Tr,
-                                            q, p, V, maxp, w, NULL, &m_delta);
+                                            q, p, V, maxp, (status & OR_BAD_TOKEN) ? -1 : x[j], w, NULL,
+                                            &m_delta);
             delta = 0;
             if (!(status & OR_BAD_TOKEN)) {
                 const int rx = (int)w[x[j]];
@@ -558,7 +561,7 @@ static void verify_sequence(const void *draft, const void *target, int dtype,
             tempered_softmax(draft, dtype, dbase + (size_t)jstar * V, V, Tr, q);
             tempered_softmax_ln(target, dtype, tbase + (size_t)jstar * V, V, Tr, p, &Mp, &lnSp);
             const double eta = token_target(rule, alpha, target, dtype, tbase + (size_t)jstar * V, Mp,
-                                            Tr, q, p, V, max_of(p, V), w, NULL, &m_unused);
+                                            Tr, q, p, V, max_of(p, V), -1, w, NULL, &m_unused);
             for (int v = 0; v < V; ++v) {
                 double d = eta * p[v] - w[v] * q[v];
                 w[v] = d > 0.0 ? d : 0.0;

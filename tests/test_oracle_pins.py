@@ -503,6 +503,38 @@ def test_table3_and_log_loss_worked_examples():
             assert (r.num_accepted[0], r.next_token[0]) == (c["num_accepted"], c["next_token"]), (ex["name"], c)
 
 
+@pytest.mark.parametrize("rule", ["token_v1", "token_v2"])
+def test_token_margin_counts_the_draft_token_however_light(rule):
+    """The draft token's own deferral r(x) decides whether it is kept outright
+    (Section 4.4: the acceptance ratio is (1 - r(x)) + eta p(x)/q(x)), so its
+    comparison counts towards the sequence's decision margin even when q(x) and
+    p(x) are far below the 1e-9 that lighter non-draft tokens need.  Hand-built
+    row: q = (0.6, 0.4 - 5e-10, 5e-10), p = (0.5, 0.5 - 1e-10, 1e-10), and alpha
+    put 6e-10 below max p, so the threshold max p - alpha = 6e-10 sits 1e-10 above
+    q(2) (TokenV1) and 5e-10 above p(2) (TokenV2): r(2) = 1 with a margin far below
+    1e-6.  With x = 2 the sequence is flagged; with x = 0 (r(0) = 0, margin 0.1 or
+    more) the same light token does not flag it."""
+    qrow = [[0.6, 0.4 - 5e-10, 5e-10]]
+    prow = [[0.5, 0.5 - 1e-10, 1e-10], [0.2, 0.3, 0.5]]
+    for x, flagged in ((2, True), (0, False)):
+        w = rows_workload(qrow, prow, [x], [0.5, 0.37], rule, 0.4)
+        maxp = oracle.verify_workload(w).row("maxp")[0, 0]
+        w.alpha = float(maxp - 6e-10)
+        r = oracle.verify_workload(w)
+        q = np_softmax(logits_as_f64(w.draft[0, 0], "f32"), 1.0)
+        p = np_softmax(logits_as_f64(w.target[0, 0], "f32"), 1.0)
+        light = q[2] if rule == "token_v1" else p[2]
+        assert light < 1e-9 and abs(light - 6e-10) < 6e-10
+        if flagged:
+            assert r.row("delta")[0, 0] == 1            # r(x) = 1: the light draft is deferred
+            assert abs(r.row("margin_delta")[0, 0] - abs(light - 6e-10)) < 1e-15
+            assert r.flagged[0]
+        else:
+            assert r.row("delta")[0, 0] == 0 and r.num_accepted[0] == 1
+            assert r.row("margin_delta")[0, 0] > 0.09
+            assert not r.flagged[0]
+
+
 def _token_pi(rule, alpha, q, p):
     """pi_Token(v) = q(v)(1 - r(v)) + eta p(v), eta = sum_v r(v) q(v), for one row
     (Section 4.4; r by the TokenV1 / TokenV2 / TokenV3 plug-in rules)."""
