@@ -209,18 +209,21 @@ int sc_debug_line(int reset);
  * exit.
  *
  * Limits: B <= SC_STATIC_MAX_B and B * (gamma + 1) <= SC_STATIC_MAX_UNITS
- * (about 10.8 MiB of scratch); larger batches return SC_ERR_SCRATCH_LIMIT and queue no
- * work.  Other arguments are those of sc_verify and are checked the same way.
+ * (gamma >= 1, so at most SC_STATIC_MAX_UNITS / 2 = SC_STATIC_MAX_B sequences;
+ * about 10.8 MiB of scratch); larger batches return SC_ERR_SCRATCH_LIMIT and
+ * queue no work.  Other arguments are those of sc_verify and are checked the
+ * same way, all before anything is queued.
  *
- * The first call on a device looks up the array's device address (the library's
- * module is loaded then); make that first call before any stream capture.  Every
- * call clears the tickets it uses on `stream` before launching.  All calls on a
+ * Every call looks up the array's device address in the current context; the
+ * first call on a device also loads the library's module there, so make it
+ * before any stream capture.  Every call clears the tickets it uses on `stream`
+ * before launching.  All calls on a
  * device share the one array and it keeps the last call's contents, so calls that
  * may overlap on the GPU (different streams without ordering between them) race
  * and must not be issued; order them on one stream or serialise them.  Nothing is
  * allocated or freed by this call.
  */
-#define SC_STATIC_MAX_B 4096
+#define SC_STATIC_MAX_B 2048
 #define SC_STATIC_MAX_UNITS 4096
 int sc_verify_static(const void *draft_logits, const void *target_logits, sc_dtype dtype,
                      const int32_t *draft_tokens, const float *uniforms, int B, int gamma, int V,

@@ -2203,34 +2203,58 @@ int common_checks(const void *draft, const void *target, int dtype, int B, int g
   return SC_OK;
 }
 
+// Every argument check of sc_verify_ex except the workspace's, in its order;
+// SC_OK or the status the entry point returns without queueing work.
+int verify_checks(const void *draft_logits, const void *target_logits, sc_dtype dtype,
+                  const int32_t *draft_tokens, const float *uniforms, int B, int gamma, int V,
+                  sc_rule rule, float alpha, float beta, float temperature,
+                  const int32_t *num_accepted, const int32_t *next_token,
+                  const int32_t *device_status, const float *row_info, cudaStream_t stream) {
+  t_capturing = capturing(stream);
+  int rc = common_checks(draft_logits, target_logits, dtype, B, gamma, V, temperature, true);
+  if (rc != SC_OK) return rc;
+  const int ri = static_cast<int>(rule);
+  if (ri < 0 || ri > SC_RULE_OPT_LOG) return SC_ERR_INVALID_ARG;
+  // alpha: a probability-scale cost for Table 1, lossy and token rules, a
+  // threshold on a (cross) entropy for BiLD* and the log-loss rules
+  if (ri <= SC_RULE_LOSSY ? !(alpha >= 0.0f && alpha <= 1.0f) : !(alpha >= 0.0f && std::isfinite(alpha)))
+    return SC_ERR_INVALID_ARG;
+  const bool greedy = temperature == 0.0f;
+  // greedy decoding is defined for the scalar deferral rules only
+  if (greedy && ((ri >= SC_RULE_TOKEN_V1 && ri <= SC_RULE_TOKEN_V3) || ri == SC_RULE_LOSSY))
+    return SC_ERR_INVALID_ARG;
+  if (ri == SC_RULE_LOSSY && !(beta > 0.0f && std::isfinite(beta) && beta >= 1.0f - alpha))
+    return SC_ERR_INVALID_ARG;
+  if (!device_accessible(draft_tokens) || !device_accessible(uniforms) ||
+      !device_accessible(num_accepted) || !device_accessible(next_token))
+    return SC_ERR_INVALID_ARG;
+  if (device_status && !device_accessible(device_status)) return SC_ERR_INVALID_ARG;
+  if (row_info && !device_accessible(row_info)) return SC_ERR_INVALID_ARG;
+  return SC_OK;
+}
+
 // ------------------------------------------------------------------ fixed scratch
 
 // Workspace of sc_verify_static: sc_verify's layout for the largest accepted
 // batch -- SC_STATIC_MAX_UNITS units, and at most half as many sequences since
-// gamma >= 1.  One copy per device, zeroed when the module loads.
-constexpr size_t kStaticMaxSeqs =
-    SC_STATIC_MAX_B < SC_STATIC_MAX_UNITS / 2 ? SC_STATIC_MAX_B : SC_STATIC_MAX_UNITS / 2;
+// gamma >= 1 (SC_STATIC_MAX_B is that half).  One copy per device, zeroed when
+// the module loads.
+static_assert(2 * SC_STATIC_MAX_B <= SC_STATIC_MAX_UNITS, "gamma >= 1 gives each sequence two units");
+constexpr size_t kStaticMaxSeqs = SC_STATIC_MAX_B;
 constexpr size_t kStaticScratchBytes = ws_layout(kStaticMaxSeqs, SC_STATIC_MAX_UNITS).total;
 static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
 
-void *g_static_ptr[64];
-std::mutex g_static_mu;
-
-// Device address of g_static_scratch on the current device, looked up once per
-// device.  The host-side name is only a stand-in and must never reach a kernel.
+// Device address of g_static_scratch in the current device's context.  The
+// host-side name is only a stand-in and must never reach a kernel.  It is looked
+// up on every call (a host-side table lookup once the module is loaded), so a
+// context torn down and recreated (cudaDeviceReset) never leaves a stale address.
 int static_scratch(void **out) {
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return SC_ERR_CUDA;
-  std::lock_guard<std::mutex> lock(g_static_mu);
-  if (!g_static_ptr[dev]) {
-    void *p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || !p) {
-      cudaGetLastError();
-      return SC_ERR_CUDA;
-    }
-    g_static_ptr[dev] = p;
+  void *p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || !p) {
+    cudaGetLastError();
+    return SC_ERR_CUDA;
   }
-  *out = g_static_ptr[dev];
+  *out = p;
   return SC_OK;
 }
 
@@ -2272,26 +2296,12 @@ int sc_verify_ex(const void *draft_logits, const void *target_logits, sc_dtype d
                  sc_rule rule, float alpha, float beta, float temperature, int32_t *num_accepted,
                  int32_t *next_token, void *workspace, size_t workspace_bytes,
                  int32_t *device_status, float *row_info, cudaStream_t stream) {
-  t_capturing = capturing(stream);
-  int rc = common_checks(draft_logits, target_logits, dtype, B, gamma, V, temperature, true);
+  int rc = verify_checks(draft_logits, target_logits, dtype, draft_tokens, uniforms, B, gamma, V, rule,
+                         alpha, beta, temperature, num_accepted, next_token, device_status, row_info,
+                         stream);
   if (rc != SC_OK) return rc;
   const int ri = static_cast<int>(rule);
-  if (ri < 0 || ri > SC_RULE_OPT_LOG) return SC_ERR_INVALID_ARG;
-  // alpha: a probability-scale cost for Table 1, lossy and token rules, a
-  // threshold on a (cross) entropy for BiLD* and the log-loss rules
-  if (ri <= SC_RULE_LOSSY ? !(alpha >= 0.0f && alpha <= 1.0f) : !(alpha >= 0.0f && std::isfinite(alpha)))
-    return SC_ERR_INVALID_ARG;
   const bool greedy = temperature == 0.0f;
-  // greedy decoding is defined for the scalar deferral rules only
-  if (greedy && ((ri >= SC_RULE_TOKEN_V1 && ri <= SC_RULE_TOKEN_V3) || ri == SC_RULE_LOSSY))
-    return SC_ERR_INVALID_ARG;
-  if (ri == SC_RULE_LOSSY && !(beta > 0.0f && std::isfinite(beta) && beta >= 1.0f - alpha))
-    return SC_ERR_INVALID_ARG;
-  if (!device_accessible(draft_tokens) || !device_accessible(uniforms) ||
-      !device_accessible(num_accepted) || !device_accessible(next_token))
-    return SC_ERR_INVALID_ARG;
-  if (device_status && !device_accessible(device_status)) return SC_ERR_INVALID_ARG;
-  if (row_info && !device_accessible(row_info)) return SC_ERR_INVALID_ARG;
   if (!workspace || workspace_bytes < sc_workspace_bytes(B, gamma, V)) return SC_ERR_WORKSPACE;
   if (!device_accessible(workspace)) return SC_ERR_WORKSPACE;
 
@@ -2391,19 +2401,26 @@ const char *sc_status_string(int code) {
 }
 
 // Same verification kernel, with its workspace in g_static_scratch instead of
-// caller memory.  No allocation: the tickets are cleared with a memset on the
-// caller's stream and sc_verify_rows runs on the fixed array.
+// caller memory.  No allocation: after the argument checks the tickets are
+// cleared with a memset on the caller's stream and sc_verify_rows runs on the
+// fixed array.
 int sc_verify_static(const void *draft_logits, const void *target_logits, sc_dtype dtype,
                      const int32_t *draft_tokens, const float *uniforms, int B, int gamma, int V,
                      sc_rule rule, float alpha, float temperature, int32_t *num_accepted,
                      int32_t *next_token, int32_t *device_status, cudaStream_t stream) {
   if (B < 1 || gamma < 1) return SC_ERR_INVALID_ARG;
-  if (B > SC_STATIC_MAX_B || static_cast<long>(B) * (gamma + 1) > SC_STATIC_MAX_UNITS)
+  if (B > SC_STATIC_MAX_B || static_cast<long>(B) * (static_cast<long>(gamma) + 1) > SC_STATIC_MAX_UNITS)
     return SC_ERR_SCRATCH_LIMIT;
   const size_t need = sc_workspace_bytes(B, gamma, V);
   if (need > kStaticScratchBytes) return SC_ERR_SCRATCH_LIMIT;
+  // every other argument is checked before the scratch is touched: a refused
+  // call queues nothing
+  int rc = verify_checks(draft_logits, target_logits, dtype, draft_tokens, uniforms, B, gamma, V, rule,
+                         alpha, 1.0f, temperature, num_accepted, next_token, device_status, nullptr,
+                         stream);
+  if (rc != SC_OK) return rc;
   void *ws = nullptr;
-  int rc = static_scratch(&ws);
+  rc = static_scratch(&ws);
   if (rc != SC_OK) return rc;
   // the previous call left the tickets at zero unless it was cut short: clear them
   const size_t zeroed = ws_layout(static_cast<size_t>(B), static_cast<size_t>(B) * (gamma + 1)).zeroed;

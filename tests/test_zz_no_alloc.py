@@ -24,7 +24,7 @@ from paper_2405_19261_gb300.workloads import config, synthetic
 pytestmark = pytest.mark.gpu
 
 SC_ERR_SCRATCH_LIMIT = -5
-STATIC_MAX_B = 4096
+STATIC_MAX_B = 2048
 STATIC_MAX_UNITS = 4096
 
 
@@ -78,15 +78,16 @@ def test_static_scratch_matches_workspace_entry_point(sc):
 def test_static_scratch_refuses_oversized_batches(sc):
     import torch
     binding, L = sc
-    w = config(1)
-    d, t, x, u = binding.to_device(w)
-    na = torch.zeros(w.B, dtype=torch.int32, device="cuda")
-    nt = torch.zeros(w.B, dtype=torch.int32, device="cuda")
-    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    # inputs of the claimed sizes (V = 8 keeps them small), so that a regressed
+    # limit check would give a wrong return code, never a read past a buffer
     for B, gamma in ((STATIC_MAX_B + 1, 1), (STATIC_MAX_UNITS // 4 + 1, 3)):
-        w2 = w.subset(list(range(w.B)))
-        w2.B, w2.gamma = B, gamma   # sizes only: the limit is checked before anything is read
-        rc = _static_call(binding, L, d, t, x, u, w2, na, nt, status)
+        w = synthetic(B, gamma, 8, dtype="f32", kind="gauss", sigma=1.0, rule="opt", alpha=0.2, seed=5)
+        d, t, x, u = binding.to_device(w)
+        na = torch.zeros(w.B, dtype=torch.int32, device="cuda")
+        nt = torch.zeros(w.B, dtype=torch.int32, device="cuda")
+        status = torch.zeros(1, dtype=torch.int32, device="cuda")
+        rc = _static_call(binding, L, d, t, x, u, w, na, nt, status)
+        torch.cuda.synchronize()
         assert rc == SC_ERR_SCRATCH_LIMIT
-    torch.cuda.synchronize()
-    assert int(status.item()) == 0
+        assert int(status.item()) == 0
+        assert int(torch.count_nonzero(na).item()) == 0 and int(torch.count_nonzero(nt).item()) == 0
