@@ -102,46 +102,32 @@ def test_many_seeds_t5_shape(sc, seed, rule):
     assert_parity(w, run_gpu(sc, w), oracle.verify_workload(w))
 
 
-def _sampled_parity(sc, w, nseq=12, seed=0):
-    gpu = run_gpu(sc, w)
-    pick = np.sort(np.random.default_rng(seed).choice(w.B, size=min(nseq, w.B), replace=False))
-    ref = oracle.verify_workload(w.subset(pick))
-    na, nt, ri, status = gpu
-    assert_parity(w.subset(pick), (na[pick], nt[pick], ri[pick], status), ref)
-    return gpu
-
-
-@pytest.mark.slow
-def test_cfg2_full_size_sampled(sc):
-    _sampled_parity(sc, config(2), nseq=12)
-
-
-@pytest.mark.slow
-def test_cfg3_full_size_sampled(sc):
-    w = config(3)
-    na, nt, ri, status = _sampled_parity(sc, w, nseq=12)
-    # planted rejections: every forced sequence stops at or before its forced position
-    f = w.forced >= 0
-    assert np.all(na[f] <= w.forced[f])
-
-
-@pytest.mark.slow
-@pytest.mark.parametrize("rule", ["chow", "diff", "opt"])
-def test_cfg4_smallest_point_sampled(sc, rule):
-    _sampled_parity(sc, config(4, B=64, gamma=4, rule=rule), nseq=6)
-
-
 # ----------------------------------------------------------------- row statistics
 
-@pytest.mark.parametrize("case", ["cfg1", "zipf-256k", "f32-odd"])
+ROW_STATS_CASES = {
+    "cfg1": lambda: config(1),
+    "zipf-256k": lambda: synthetic(3, 4, 256000, dtype="bf16", kind="zipf", sigma=0.7, seed=5, temperature=0.7),
+    "f32-odd": lambda: synthetic(4, 3, 10007, dtype="f32", kind="gauss", sigma=1.0, seed=6, temperature=1.3),
+    # ragged vocabularies: rows of a multiple of 16 bytes stream by TMA bulk copies,
+    # the others by per-thread loads
+    "bf16-4097": lambda: synthetic(5, 3, 4097, dtype="bf16", kind="gauss", sigma=1.0, seed=7),
+    "bf16-32127": lambda: synthetic(3, 2, 32127, dtype="bf16", kind="zipf", sigma=0.7, seed=8),
+    "f32-7": lambda: synthetic(6, 3, 7, dtype="f32", kind="gauss", sigma=1.0, seed=9),
+    "bf16-8200": lambda: synthetic(4, 3, 8200, dtype="bf16", kind="gauss", sigma=1.0, seed=10),
+    # long drafts
+    "gamma-12": lambda: synthetic(4, 12, 32128, dtype="bf16", kind="zipf", sigma=0.7, seed=11),
+    "gamma-40": lambda: synthetic(2, 40, 1000, dtype="bf16", kind="zipf", sigma=1.0, seed=12),
+    # the maximum vocabulary (16 CTAs x 16 chunks of 4096 logits per row)
+    "max-vocab": lambda: synthetic(1, 2, 1 << 20, dtype="bf16", kind="zipf", sigma=0.7, seed=13),
+    # a Gemma-vocabulary batch, every pair through the TV pass
+    "gemma-B64": lambda: config(4, B=64, gamma=4),
+}
+
+
+@pytest.mark.parametrize("case", list(ROW_STATS_CASES))
 def test_row_stats(sc, case):
     import torch
-    if case == "cfg1":
-        w = config(1)
-    elif case == "zipf-256k":
-        w = synthetic(3, 4, 256000, dtype="bf16", kind="zipf", sigma=0.7, seed=5, temperature=0.7)
-    else:
-        w = synthetic(4, 3, 10007, dtype="f32", kind="gauss", sigma=1.0, seed=6, temperature=1.3)
+    w = ROW_STATS_CASES[case]()
     d, t, _, _ = sc.to_device(w)
     mq, mp, tv = sc.sc_row_stats(d, t, w.temperature)
     torch.cuda.synchronize()
@@ -419,19 +405,6 @@ def test_vocab_above_the_limit_is_refused(sc):
         sc.sc_verify(d, t, x, u, "opt", 0.2, 1.0)
 
 
-@pytest.fixture(scope="module")
-def cfg4_largest():
-    # the largest sweep point bench.py times: B=512, gamma=8 (4.46 GB of bf16 logits);
-    # generated once, the rules below run on the same logits
-    return config(4, B=512, gamma=8, rule="diff")
-
-
-@pytest.mark.slow
-@pytest.mark.parametrize("rule,alpha", [("chow", 0.5), ("diff", 0.1), ("opt", 0.2)])
-def test_cfg4_largest_point_sampled(sc, cfg4_largest, rule, alpha):
-    _sampled_parity(sc, cfg4_largest.with_rule(rule, alpha), nseq=6)
-
-
 # ----------------------------------------------------------------- token-specific targets
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
@@ -459,9 +432,3 @@ def test_token_rules_ragged_vocab(sc, V, dtype):
     w = synthetic(5, 3, V, dtype=dtype, kind="gauss", sigma=1.0, rule="token_v3", alpha=0.3,
                   temperature=0.9, seed=V)
     assert_parity(w, run_gpu(sc, w), oracle.verify_workload(w))
-
-
-@pytest.mark.slow
-@pytest.mark.parametrize("rule", ["token_v3", "token_v1"])
-def test_token_rules_gemma_shape_sampled(sc, rule):
-    _sampled_parity(sc, config(4, B=64, gamma=4, rule=rule), nseq=6)

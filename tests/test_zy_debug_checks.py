@@ -1,4 +1,4 @@
-"""Runs last: with a library built with device-side checks (SC_BUILD_DEBUG=1 at
+"""Runs after the parity tests: with a library built with device-side checks (SC_BUILD_DEBUG=1 at
 build time), no computed index, copy size or alignment failed during any of the
 GPU tests before it."""
 import pytest
