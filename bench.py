@@ -1,11 +1,13 @@
 #!/usr/bin/env python3
 """Benchmark of the speculative-cascade verification step on GB300.
 
-Default: one GPU, workload cfg3 (B=128, gamma=7, V=256000 bf16 Zipf logits,
-T=0.7, Diff rule alpha=0.1, half the sequences with a planted early
-rejection): 983 MB of logits per step, more than the 129 MB L2, so steps run
-back to back without an L2 flush.  A step is one sc_verify call (one kernel
-launch) over the whole batch.
+Default: one GPU, the largest sweep point (B=512 sequences, gamma=8 drafted
+positions, V=256000 bf16 Zipf-shaped logits, T=1) under the plug-in optimal
+rule OPT alpha=0.2 (Eq. 10): 4.46 GB of logits per step, far more than the
+129 MB L2, so steps run back to back without an L2 flush.  A step is one
+sc_verify call (one kernel launch) over the whole batch.  Chow 0.5 and Diff 0.1
+are timed on the same logits in the same run and reported under
+config.other_rules; --sweep adds every sweep point under the three rules.
 
 Prints ONE JSON line (rank 0).  Keys beyond the base contract:
   roofline      achieved HBM GB/s of the verification kernel (algorithmic bytes
@@ -52,9 +54,9 @@ def parse():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--config", type=int, default=3)
-    ap.add_argument("--B", type=int, default=None)
-    ap.add_argument("--gamma", type=int, default=None)
+    ap.add_argument("--config", type=int, default=4)
+    ap.add_argument("--B", type=int, default=None, help="config 4: batch size (default 512)")
+    ap.add_argument("--gamma", type=int, default=None, help="config 4: drafted positions (default 8)")
     ap.add_argument("--rule", default=None)
     ap.add_argument("--alpha", type=float, default=None)
     ap.add_argument("--beta", type=float, default=1.0, help="lossy speculative decoding's beta")
@@ -63,8 +65,16 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--record-traffic", metavar="NCU_CSV", default=None,
                     help="store the DRAM bytes of an ncu capture of this workload for the current kernel source")
+    ap.add_argument("--traffic-from-B", type=int, default=None,
+                    help="with --record-traffic: the capture ran B0 sequences of this workload's shape; "
+                         "its bytes are scaled by B / B0")
     ap.add_argument("--min-warmup-s", type=float, default=0.5,
                     help="keep warming up (untimed) until this long has passed, for clock samples")
+    ap.add_argument("--other-rules", default=None,
+                    help="comma-separated rule[:alpha] list timed on the same logits after the headline "
+                         "(default for config 4: the other two Table 1 rules of the sweep; 'none' for none)")
+    ap.add_argument("--sweep", action="store_true",
+                    help="config 4: also time every sweep point (B x gamma) under Chow, Diff and OPT")
     return ap.parse_args()
 
 
@@ -99,10 +109,12 @@ def measured_peaks():
 _NCU_UNITS = {"byte": 1, "Kbyte": 1e3, "Mbyte": 1e6, "Gbyte": 1e9, "Tbyte": 1e12}
 
 
-def record_traffic(csv_path, workload_name, command=""):
+def record_traffic(csv_path, workload_name, command="", scale=1.0, note=""):
     """Store, for the current kernel source, the DRAM bytes ncu measured for one
     sc_unit_kernel launch (the first one in an `ncu --metrics
-    dram__bytes_read.sum,dram__bytes_write.sum --csv --log-file` capture)."""
+    dram__bytes_read.sum,dram__bytes_write.sum --csv --log-file` capture),
+    multiplied by `scale` when the capture ran a smaller batch of the same rows
+    (every unit reads its own rows, so the bytes grow with the units)."""
     import csv
     with open(csv_path, encoding="utf-8") as f:
         rows = list(csv.DictReader(ln for ln in f if ln.startswith('"')))
@@ -121,10 +133,12 @@ def record_traffic(csv_path, workload_name, command=""):
         with open(TRAFFIC_FILE) as f:
             d = json.load(f)
     d[workload_name] = {"kernel_sha": kernel_sha(),
-                        "dram_bytes_per_launch": int(m["dram__bytes_read.sum"] + m["dram__bytes_write.sum"]),
-                        "dram_bytes_read": int(m["dram__bytes_read.sum"]),
-                        "dram_bytes_write": int(m["dram__bytes_write.sum"]),
+                        "dram_bytes_per_launch": int(scale * (m["dram__bytes_read.sum"] + m["dram__bytes_write.sum"])),
+                        "dram_bytes_read": int(scale * m["dram__bytes_read.sum"]),
+                        "dram_bytes_write": int(scale * m["dram__bytes_write.sum"]),
                         "source": command}
+    if note:
+        d[workload_name]["scaled"] = note
     with open(TRAFFIC_FILE, "w") as f:
         json.dump(d, f, indent=2)
         f.write("\n")
@@ -287,6 +301,18 @@ def whole_job_rate(units_per_rank, world, ms_step):
 
 # ------------------------------------------------------------------ main
 
+def workload_desc(args):
+    """The workload's description (the key of its traffic record), without drawing it."""
+    from paper_2405_19261_gb300.workloads import CONFIG_TEXT, SWEEP_ALPHA
+    if args.config != 4:
+        return f"cfg{args.config}: {CONFIG_TEXT[args.config]}"
+    rule = args.rule or "opt"
+    alpha = SWEEP_ALPHA[rule] if args.alpha is None else args.alpha
+    T = 1.0 if args.temperature is None else args.temperature
+    return (f"cfg4: B={args.B or 512} gamma={args.gamma or 8} V=256000 bf16, zipf sigma=0.7, T={T:g}, "
+            f"{rule} a={float(alpha)}" + (f" beta={args.beta:g}" if rule == "lossy" else ""))
+
+
 def workload_from(args, rank=0):
     """The named workload; rank r > 0 of a multi-GPU run gets its own sequences
     (seed offset 1000 r), so the ranks verify disjoint batches of one shape."""
@@ -299,16 +325,16 @@ def workload_from(args, rank=0):
     if args.alpha is not None:
         kw["alpha"] = args.alpha
     if args.config == 4:
-        kw["B"] = args.B or 64
-        kw["gamma"] = args.gamma or 4
+        kw["B"] = args.B or 512
+        kw["gamma"] = args.gamma or 8
         kw["temperature"] = args.temperature
     w = config(args.config, **kw)
     w.beta = args.beta
-    desc = CONFIG_TEXT[args.config]
+    desc = workload_desc(args)
     if args.config == 4:
-        desc = (f"B={w.B} gamma={w.gamma} V=256000 bf16, zipf sigma=0.7, T={w.temperature:g}, "
-                f"{w.rule} a={w.alpha}" + (f" beta={w.beta:g}" if w.rule == "lossy" else ""))
-    return w, f"cfg{args.config}: {desc}"
+        assert desc == (f"cfg4: B={w.B} gamma={w.gamma} V=256000 bf16, zipf sigma=0.7, T={w.temperature:g}, "
+                        f"{w.rule} a={w.alpha}" + (f" beta={w.beta:g}" if w.rule == "lossy" else ""))
+    return w, desc
 
 
 def run_reference(args):
@@ -360,15 +386,46 @@ def run_ours(args):
                           next_token=nt, workspace=ws, stream=stream)
 
     l2 = torch.cuda.get_device_properties(dev).L2_cache_size
-    flush = w.logit_bytes < 3 * l2
-    flush_buf = torch.empty(int(2 * l2), dtype=torch.uint8, device=dev) if flush else None
-    clean_buf = torch.ones(int(2 * l2) // 4, dtype=torch.float32, device=dev) if flush else None
+    flush_buf = torch.empty(int(2 * l2), dtype=torch.uint8, device=dev)
+    clean_buf = torch.ones(int(2 * l2) // 4, dtype=torch.float32, device=dev)
 
     def flush_l2():
         # write a buffer larger than L2, then read another one so that the dirty
         # lines are written back now rather than during the timed step
         flush_buf.fill_(1)
         clean_buf.sum()
+
+    def timed(step_fn, steps, flush):
+        """K steps timed with CUDA events on the launching stream: (total ms,
+        per-step ms).  Inputs smaller than 3x L2 flush L2 before every step."""
+        if flush:
+            evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                   for _ in range(steps)]
+            # Hold the stream with a spin kernel while the host queues every step, so
+            # that no step's interval includes the host's launch latency (a small
+            # step is shorter than the Python call that launches it).
+            sleep = getattr(torch.cuda, "_sleep", None)
+            if sleep is not None:
+                sleep(int(2e9 * 200e-6 * steps))  # ~200 us of host time per step at ~2 GHz
+            for e0, e1 in evs:
+                flush_l2()
+                e0.record(stream)
+                step_fn()
+                e1.record(stream)
+            torch.cuda.synchronize(dev)
+            ms_steps = [e0.elapsed_time(e1) for e0, e1 in evs]
+            return sum(ms_steps), ms_steps
+        # an event between consecutive steps: the K intervals tile the timed region
+        evs = [torch.cuda.Event(enable_timing=True) for _ in range(steps + 1)]
+        evs[0].record(stream)
+        for i in range(steps):
+            step_fn()
+            evs[i + 1].record(stream)
+        torch.cuda.synchronize(dev)
+        return evs[0].elapsed_time(evs[-1]), [a.elapsed_time(b) for a, b in zip(evs[:-1], evs[1:])]
+
+    flush = w.logit_bytes < 3 * l2
+    peak, peak_kind = measured_peaks()
 
     props = torch.cuda.get_device_properties(dev)
     gpu_id = str(getattr(props, "uuid", "")) or str(local)
@@ -390,37 +447,9 @@ def run_ours(args):
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize(dev)
-    if flush:
-        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-               for _ in range(args.steps)]
-        # Hold the stream with a spin kernel while the host queues every step, so
-        # that no step's interval includes the host's launch latency (a small
-        # step is shorter than the Python call that launches it).
-        sleep = getattr(torch.cuda, "_sleep", None)
-        if sleep is not None:
-            sleep(int(2e9 * 200e-6 * args.steps))  # ~200 us of host time per step at ~2 GHz
-        for e0, e1 in evs:
-            flush_l2()
-            e0.record(stream)
-            step()
-            e1.record(stream)
-        torch.cuda.synchronize(dev)
-        ms_steps = [e0.elapsed_time(e1) for e0, e1 in evs]
-        ms_total = sum(ms_steps)
-    else:
-        # an event between consecutive steps: the K intervals tile the timed region
-        evs = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
-        evs[0].record(stream)
-        for i in range(args.steps):
-            step()
-            evs[i + 1].record(stream)
-        torch.cuda.synchronize(dev)
-        ms_total = evs[0].elapsed_time(evs[-1])
-        ms_steps = [a.elapsed_time(b) for a, b in zip(evs[:-1], evs[1:])]
+    ms_total, ms_steps = timed(step, args.steps, flush)
     if world > 1:
         dist.barrier()
-    sampler.stop()
-    clocks = sampler.summary()
 
     ms_step = max_over_ranks(ms_total / args.steps, world, dev)
     spread = step_spread(ms_steps)
@@ -429,7 +458,6 @@ def run_ours(args):
     value = whole_job_rate(B * g, world, ms_step)
 
     # roofline of the verification kernel (the only kernel in a step)
-    peak, peak_kind = measured_peaks()
     alg = w.algorithmic_bytes()
     achieved = alg / (ms_step / 1e3) / 1e9
     traffic = stored_traffic(desc)
@@ -438,6 +466,57 @@ def run_ours(args):
                 "peak_kind": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
                 "frac_of_nominal_8TBs": achieved / NOMINAL_HBM_GBS,
                 "algorithmic_bytes_per_launch": alg}
+
+    def rule_line(wr, ms, na_r):
+        a = wr.algorithmic_bytes() / (ms / 1e3) / 1e9
+        return {"rule": wr.rule, "alpha": wr.alpha, "B": wr.B, "gamma": wr.gamma, "us_per_step": ms * 1e3,
+                "positions_per_s": wr.B * wr.gamma / (ms / 1e3), "achieved_gbs": a, "frac": a / peak,
+                "frac_of_nominal_8TBs": a / NOMINAL_HBM_GBS, "mean_accepted": float(na_r.float().mean().item())}
+
+    def time_rule(wr, dd, tt, xx, uu):
+        """Warm-up and K timed steps of one workload (its own rule and alpha)."""
+        ws_r = binding.new_workspace(wr.B, wr.gamma, dev)
+        na_r = torch.empty(wr.B, dtype=torch.int32, device=dev)
+        nt_r = torch.empty(wr.B, dtype=torch.int32, device=dev)
+
+        def step_r():
+            binding.sc_verify(dd, tt, xx, uu, wr.rule, wr.alpha, wr.temperature, beta=getattr(wr, "beta", 1.0),
+                              num_accepted=na_r, next_token=nt_r, workspace=ws_r, stream=stream)
+
+        for _ in range(max(3, args.warmup)):
+            step_r()
+        torch.cuda.synchronize(dev)
+        tot, _ = timed(step_r, args.steps, wr.logit_bytes < 3 * l2)
+        return rule_line(wr, tot / args.steps, na_r)
+
+    other = []
+    others = args.other_rules
+    if others is None:
+        others = ",".join(r for r in ("chow", "diff", "opt") if r != w.rule) if args.config == 4 else "none"
+    if world == 1 and others != "none":
+        from paper_2405_19261_gb300.workloads import SWEEP_ALPHA
+        for item in others.split(","):
+            rname, _, a = item.partition(":")
+            wr = w.with_rule(rname, float(a) if a else SWEEP_ALPHA[rname])
+            wr.beta = w.beta
+            other.append(time_rule(wr, d, t, x, u))
+    sweep = []
+    if world == 1 and args.sweep and args.config == 4:
+        from paper_2405_19261_gb300.workloads import SWEEP_ALPHA, SWEEP_POINTS, config
+        for (Bs, gs) in SWEEP_POINTS:
+            if (Bs, gs) == (w.B, w.gamma):
+                pts = [rule_line(w, ms_step, na)] + [o for o in other]
+                sweep.extend(pts)
+                continue
+            wp = config(4, B=Bs, gamma=gs)
+            dp, tp, xp, up = binding.to_device(wp, dev)
+            for rname in ("chow", "diff", "opt"):
+                wr = wp.with_rule(rname, SWEEP_ALPHA[rname])
+                sweep.append(time_rule(wr, dp, tp, xp, up))
+            del dp, tp, xp, up
+            torch.cuda.empty_cache()
+    sampler.stop()  # the clock samples cover the warm-up and every timed step above
+    clocks = sampler.summary()
 
     # end to end through the public API with host buffers
     e2e = None
@@ -495,9 +574,12 @@ def run_ours(args):
                                   "the steps are queued behind a spin kernel before the first, so no interval waits on the host"
                                   if flush else
                                   f"inputs {w.logit_bytes / 1e6:.0f} MB > L2 {l2 / 1e6:.0f} MB, back to back"),
-                           "parallelism": f"{world} independent replica(s), no collective"},
+                           "parallelism": f"{world} independent replica(s), no collective",
+                           "other_rules": other},
                 "step_ms": spread, "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
                 "gpu_launches": args.steps, "clocks": clocks}
+        if sweep:
+            line["sweep"] = sweep
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
@@ -506,8 +588,14 @@ def run_ours(args):
 def main():
     args = parse()
     if args.record_traffic:
-        _, desc = workload_from(args)
-        print(json.dumps(record_traffic(args.record_traffic, desc, " ".join(sys.argv))))
+        w_b = args.B or 512
+        desc = workload_desc(args)
+        scale, note = 1.0, ""
+        if args.traffic_from_B:
+            scale = w_b / args.traffic_from_B
+            note = (f"captured at B={args.traffic_from_B} (same gamma, V, rule), scaled by {scale:g} "
+                    f"to B={w_b}: every unit reads its own rows")
+        print(json.dumps(record_traffic(args.record_traffic, desc, " ".join(sys.argv), scale, note)))
         return
     if args.impl == "reference":
         run_reference(args)
