@@ -866,23 +866,33 @@ __device__ __forceinline__ float df_floor(float2 a) { return a.y < 0.0f ? nextaf
 // 2^a to f32 accuracy: 2^hi (1 + lo ln 2)
 __device__ __forceinline__ float df_exp2(float2 a) { return exp2f(a.x) * fmaf(a.y, 0.69314718f, 1.0f); }
 
-// log2 of a softmax probability, log2(2^{y k - R} / S) = y k - R - log2 S, as hi + lo
-__device__ __forceinline__ float2 log2_prob(float y, float R, float S, float k, float kl) {
-  const float2 yk = df_mul_k(y, k, kl);
-  const float2 t = two_sum(yk.x, -R);
-  return df_norm(t.x, __fadd_rn(__fadd_rn(t.y, yk.y), -log2f(S)));
+// log2 of a softmax probability of the row with maximum M, reference R and
+// pass-1 sum S, as hi + lo.  S sums 2^{fma(y_v, k, -R)}: its exponents use the
+// f32 factor k, and differ from the exact y_v (k + kl) - R by -y_v kl =
+// -M kl - (y_v - M) kl.  For every term that S holds to f32 accuracy, (y_v - M) kl
+// is below ~1e-6 (y_v - M >= -24 / k there, |kl| <= ulp(k) / 2), so the exact
+// sum is 2^{M kl} S to that accuracy, and
+//   log2 p(y) = y (k + kl) - R - log2 S - M kl = y k - R + (y - M) kl - log2 S.
+// (M kl alone reaches 1e-3 for logits near 3e4 at T = 1, or 3e3 at T = 0.1.)
+__device__ __forceinline__ float2 log2_prob(float y, float M, float R, float S, float k, float kl) {
+  const float p = __fmul_rn(y, k);
+  const float e = fmaf(y, k, -p);  // y k = p + e exactly
+  const float2 t = two_sum(p, -R);
+  const float lo = __fadd_rn(__fadd_rn(t.y, e), __fmul_rn(__fsub_rn(y, M), kl));
+  return df_norm(t.x, __fadd_rn(lo, -log2f(S)));
 }
 
 // A softmax probability from its logit; 0 for a masked (-inf) logit.
-__device__ __forceinline__ float prob_of(float y, float R, float S, float k, float kl) {
-  return y > -INFINITY ? df_exp2(log2_prob(y, R, S, k, kl)) : 0.0f;
+__device__ __forceinline__ float prob_of(float y, float M, float R, float S, float k, float kl) {
+  return y > -INFINITY ? df_exp2(log2_prob(y, M, R, S, k, kl)) : 0.0f;
 }
 
 // Acceptance of the draft token x (Algorithm 4): a = 1 when delta = 0 or
 // q(x) <= pi(x), else a = [u < pi(x)/q(x)].  L = log2 p(x) - log2 q(x)
-//   = (y_p(x) - y_q(x)) log2(e)/T - (R_p - R_q) + log2(S_q / S_p)
-// is formed in double-float from the logits, so the ratio 2^L carries
-// essentially only the f32 error of log2(S_q / S_p).  With a token rule
+//   = (y_p(x) - y_q(x)) k - (R_p - R_q) + ((y_p(x) - M_p) - (y_q(x) - M_q)) kl
+//     + log2(S_q / S_p)
+// (see log2_prob) is formed in double-float from the logits, so the ratio 2^L
+// carries essentially only the f32 error of log2(S_q / S_p).  With a token rule
 // (Section 4.4) the draft token's own deferral r(x) takes delta's place and
 // pi(x)/q(x) = (1 - r(x)) + eta p(x)/q(x): accepted outright when r(x) = 0,
 // else [u < eta 2^L].  With lossy speculative decoding (Table 3, delta = 1)
@@ -919,10 +929,11 @@ __device__ __forceinline__ void accept_test(Shared &sh, const Params &P, int x, 
     accept = !sh.delta;  // p(x) = 0 < q(x): pi(x)/q(x) = 1 - delta (also eta p/q = 0 for a token rule)
   } else if (sh.delta) {
     const float2 d = two_sum(ypx, -yqx);  // y_p(x) - y_q(x), exactly
-    const float2 dk = df_mul_k(d.x, k, kl);
+    const float2 dk = df_mul_k(d.x, k, 0.0f);  // d.x k, exactly
     const float2 r = two_sum(sh.Rp, -sh.Rq);
     const float2 s = two_sum(dk.x, -r.x);
-    const float lo = __fadd_rn(__fadd_rn(__fadd_rn(s.y, dk.y), __fsub_rn(__fmul_rn(d.y, k), r.y)),
+    const float corr = __fmul_rn(__fsub_rn(__fsub_rn(ypx, sh.Mp), __fsub_rn(yqx, sh.Mq)), kl);
+    const float lo = __fadd_rn(__fadd_rn(__fadd_rn(__fadd_rn(s.y, dk.y), __fsub_rn(__fmul_rn(d.y, k), r.y)), corr),
                                log2f(sh.Sq / sh.Sp));
     float2 L = df_norm(s.x, lo);
     if (kTok && sh.tok) {
@@ -941,8 +952,8 @@ __device__ __forceinline__ void accept_test(Shared &sh, const Params &P, int x, 
   }
   sh.accept = accept;
   if (P.row_info != nullptr) {
-    const float qx = prob_of(yqx, sh.Rq, sh.Sq, k, kl);
-    const float px = prob_of(ypx, sh.Rp, sh.Sp, k, kl);
+    const float qx = prob_of(yqx, sh.Mq, sh.Rq, sh.Sq, k, kl);
+    const float px = prob_of(ypx, sh.Mp, sh.Rp, sh.Sp, k, kl);
     sh.qx = qx;
     if (kTok && sh.tok) sh.pix = fmaf(sh.eta, px, sh.delta ? 0.0f : qx);
     else if (lossy)  // (alpha = 1: the limit alpha -> 1-, p / (1 - alpha) = +inf where p > 0, 0 where p = 0)
@@ -1479,7 +1490,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
         // logit at q's argmax (one load; every CTA of the cluster reads the same value)
         const E *prow = static_cast<const E *>(P.target) + (static_cast<size_t>(b) * G1 + j) * P.V;
         const float y = Elt<E>::at(prow, static_cast<size_t>(g.iq));
-        const float2 lp = log2_prob(y, Rp, cs, k, P.kl);
+        const float2 lp = log2_prob(y, c, Rp, cs, k, P.kl);
         xent = y > -INFINITY ? -kLn2 * (lp.x + lp.y) : INFINITY;
       }
       if (P.greedy && pair) sh.tv = g.iq != g.ip ? 1.0f : 0.0f;  // D_TV of the one-hot q~, p~

@@ -179,6 +179,38 @@ def test_degenerate_rows(sc):
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("offset,T", [(0.0, 1.0), (3000.0, 0.1), (30000.0, 1.0), (-20000.0, 0.7)])
+def test_acceptance_ratio_with_offset_logits(sc, dtype, offset, T):
+    # A constant added to a row leaves its softmax unchanged but makes y k, the
+    # row's reference and its pass-1 sum large: the ratio p(x)/q(x) must still be
+    # formed to ~1e-7.  The target rows carry the offset, the draft rows none.
+    # Uniforms sit 2e-6 below or above the oracle's ratio (alternately), so every
+    # informative position's accept flag pins the kernel's ratio to 2e-6.
+    from paper_2405_19261_gb300.workloads import f32_to_bf16_bits
+    B, g, V = 16, 6, 2048
+    w = synthetic(B, g, V, dtype="f32", kind="gauss", sigma=0.6, rule="always", alpha=0.0,
+                  temperature=T, seed=5)
+    dq = (w.draft * np.float32(T / 2)).astype(np.float32)                     # tempered N(0, 1)
+    tp = (w.target * np.float32(T / 2) + np.float32(offset)).astype(np.float32)
+    if dtype == "bf16":
+        dq, tp = f32_to_bf16_bits(dq), f32_to_bf16_bits(tp)
+    w.draft, w.target, w.dtype = dq, tp, dtype
+    w.uniforms[:] = 0.5
+    ratio = np.minimum(1.0, oracle.verify_workload(w).row("pix") / oracle.verify_workload(w).row("qx"))
+    inform = (ratio > 1e-3) & (ratio < 1.0 - 1e-5)
+    below = (np.add.outer(np.arange(B), np.arange(g)) % 2 == 0)
+    u = np.where(below, ratio - 2e-6, ratio + 2e-6)
+    w.uniforms[:, :g] = np.where(inform, u, 0.5).astype(np.float32)
+    assert inform.sum() >= 20
+    ref = oracle.verify_workload(w)
+    gpu = run_gpu(sc, w)
+    assert_parity(w, gpu, ref)
+    acc = gpu[2][:, :g, 4]
+    np.testing.assert_array_equal(acc[inform & below], 1.0)
+    np.testing.assert_array_equal(acc[inform & ~below], 0.0)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
 @pytest.mark.parametrize("rule,alpha", [("always", 0.0), ("opt", 0.2), ("token_v3", 0.3), ("token_v1", 0.1),
                                         ("lossy", 0.3), ("lossy", 1.0)])
 def test_masked_target_logit_at_the_draft_token(sc, dtype, rule, alpha):
