@@ -576,6 +576,7 @@ def run_ours(args):
                                   f"inputs {w.logit_bytes / 1e6:.0f} MB > L2 {l2 / 1e6:.0f} MB, back to back"),
                            "parallelism": f"{world} independent replica(s), no collective",
                            "other_rules": other},
+                "kernel_sha": kernel_sha(),
                 "step_ms": spread, "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
                 "gpu_launches": args.steps, "clocks": clocks}
         if sweep:

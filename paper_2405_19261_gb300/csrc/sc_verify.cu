@@ -73,13 +73,7 @@ namespace {
 #define SC_DEBUG 0  // 1: check computed indices and copy sizes, skip and record a failing access
 #endif
 #ifndef SC_OPT_UB
-#define SC_OPT_UB 1  // OPT band rows: settle delta = 1 by the Bhattacharyya bound on D_TV
-#endif
-#ifndef SC_BONUS_LAST
-#define SC_BONUS_LAST 0  // 1: launch all pair units before the bonus rows
-#endif
-#ifndef SC_PERSISTENT
-#define SC_PERSISTENT 0  // 1: a grid of co-resident clusters loops over the units (see the kernel)
+#define SC_OPT_UB 1  // OPT and OPTLog band rows: settle delta = 1 by an upper bound on D_TV
 #endif
 #ifndef SC_L2_PREFETCH
 #define SC_L2_PREFETCH 1  // second passes prefetch their slice into L2 before streaming it
@@ -144,6 +138,8 @@ struct Params {
   float4 *records;         // [B][kMaxCluster][gamma+1] (R_q, R_p, c, flags) as seen by rank r
   float4 *records2;        // [B][kMaxCluster][gamma+1] (eta, thr, token, on_q) of token rules
   int spec_res;            // a rejected pair stores its residual's chunk prefixes itself (row_pre)
+  int pos_major;           // units in position-major order: (b, j) is unit j B + b
+  int opt_ub;              // OPT pairs accumulate sqrt(q p) in pass 1 for an upper bound on D_TV
   float *row_pre;          // [B][gamma+1][kMaxCluster][kMaxChunks + 1] those prefixes, per row
   float *bonus_pre;        // [B][kMaxCluster][kMaxChunks + 1] the same for the bonus row p_gamma,
                            // written by the bonus unit from its pass-1 chunk totals
@@ -306,17 +302,14 @@ __device__ __forceinline__ void load8_smem(const E *s, int e, int n, float (&y)[
 struct __align__(16) Shared {
   uint64_t full[kStages];
   // cluster exchanges, written by every CTA of the cluster into slot [its rank]:
-  // exchange 1 has two sets of slots, by the parity of the unit's iteration: a peer
-  // that loops on to its next unit pushes into the other set, never into the one
-  // this CTA may still be reading
-  float4 all_ms[2][kMaxCluster];  // 1: (m_q, s_q, m_p, s_p) of the slice
-  float2 all_x[2][kMaxCluster];   // 1: raw logits at the draft token, if in the slice
+  float4 all_ms[kMaxCluster];  // 1: (m_q, s_q, m_p, s_p) of the slice
+  float2 all_x[kMaxCluster];   // 1: raw logits at the draft token, if in the slice
   float all_r[kMaxCluster];    // 2 (TV pass): the slice's total residual weight
   float2 all_lb[kMaxCluster];  // OPT band: the slice's lower bound on D_TV, and its sum of sqrt(q p)
   float2 all_scr[kMaxCluster]; // token rules: the slice's sum of q over its undeferred tokens, and
                                // whether its screen is exact (1) or not (0)
-  float4 all_ext[2][kMaxCluster]; // 1 (kFamExt): (A_q, A_p, X, -) of the slice, see ExtState
-  int2 all_idx[2][kMaxCluster];   // 1 (kFamExt): the slice's argmax of q and of p
+  float4 all_ext[kMaxCluster];  // 1 (kFamExt): (A_q, A_p, X, -) of the slice, see ExtState
+  int2 all_idx[kMaxCluster];    // 1 (kFamExt): the slice's argmax of q and of p
   int timeout;
   float4 red[kNW];          // (m_q, s_q, m_p, s_p) of each warp
   float4 ext_red[kNW];      // (kFamExt) (A_q, A_p, X, -) of each warp
@@ -329,6 +322,7 @@ struct __align__(16) Shared {
   int tok, on_q;            // a token rule (Section 4.4) and its r(v) test's variable
   float dl, dr;             // OPT and OPTLog: delta = [dl < dr - alpha D_TV]
   float nhq, nhp;           // (kFamExt) sum_v q log q and sum_v p log p, in nats
+  float klqp;               // (kFamExt) KL(q || p) = sum_v q log q - sum_v q log p, in nats
   int iq, ip;               // (kFamExt) argmax q and argmax p, lowest index on ties
   float thr, eta;           // its r(v) threshold (exponent domain) and eta = sum_v r(v) q(v)
   // sequence finish
@@ -562,7 +556,7 @@ __device__ __forceinline__ void load8_chunk(const E *src, int e, int n, float (&
 
 template <typename E, bool kFull, bool kPair>
 __device__ __forceinline__ void ext_chunk(const E *srcq, const E *srcp, int n, int v0, float k,
-                                          ExtState &st, bool with_bc, float &bc) {
+                                          ExtState &st) {
   float mq = st.mq, mp = st.mp;
   int iq = st.iq, ip = st.ip;
 #pragma unroll
@@ -586,9 +580,8 @@ __device__ __forceinline__ void ext_chunk(const E *srcq, const E *srcp, int n, i
     }
   }
   const float rq = refk(mq, k), rp = refk(mp, k);
-  if (with_bc) bc *= ex2(0.5f * ((refk(st.mq, k) - rq) + (refk(st.mp, k) - rp)));  // (OPTLog's bound)
   ext_rebase(st, refk(st.mq, k) - rq, refk(st.mp, k) - rp);
-  float sq = 0.0f, aq = 0.0f, sp = 0.0f, ap = 0.0f, x = 0.0f, h = 0.0f;
+  float sq = 0.0f, aq = 0.0f, sp = 0.0f, ap = 0.0f, x = 0.0f;
 #pragma unroll
   for (int r = 0; r < kRounds; ++r) {
     const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
@@ -609,11 +602,9 @@ __device__ __forceinline__ void ext_chunk(const E *srcq, const E *srcp, int n, i
         // a finite draft logit with a masked target logit (q(v) > 0 = p(v)) makes
         // D(q, p) = +inf even where 2^a underflows: X = -inf, kept by every merge
         x += yq[i] > -INFINITY && !(yp[i] > -INFINITY) ? -INFINITY : (ea > 0.0f ? ea * b : 0.0f);
-        if (with_bc) h += ex2(0.5f * (a + b));  // sqrt(q p) up to the normalisers
       }
     }
   }
-  if (with_bc) bc += h;
   st.mq = mq;
   st.mp = mp;
   st.iq = iq;
@@ -750,6 +741,7 @@ __device__ __forceinline__ float warp_sum(float v) {
 // needs no second pass over its bonus row.
 constexpr int kBonusRef = kMaxChunks * kNW;
 static_assert(2 * kMaxChunks * kNW <= kEntries, "bonus chunk totals live in seg");
+static_assert(kMaxChunks <= 32, "one lane per chunk of a slice");
 
 template <typename E, bool kFull>
 __device__ __forceinline__ void bonus_row(const E *src, int n, float k, float &m, float2 &s, int c,
@@ -812,6 +804,57 @@ __device__ __forceinline__ float bc_chunk(const E *srcq, const E *srcp, int n, f
     }
   }
   return acc0 + acc1;
+}
+
+// OPT pair, full bf16 chunk: online_row of both rows and the chunk's
+// 2^{(a_v + b_v)/2} terms (bc_chunk) in one sweep over the registers, so the
+// logits are read from shared memory and unpacked once.  a_v and b_v are
+// relative to the rows' updated references, as in bc_chunk, and the running
+// sums are rescaled as online_row rescales its sums.
+__device__ __forceinline__ void online_pair_bc(const uint16_t *srcq, const uint16_t *srcp, float k,
+                                               float &mq, float2 &sq, float &mp, float2 &sp, float &bc) {
+  uint32_t wq[kRounds * 4], wp[kRounds * 4];
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r) {
+    const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
+    const uint4 vq = *reinterpret_cast<const uint4 *>(srcq + e);
+    const uint4 vp = *reinterpret_cast<const uint4 *>(srcp + e);
+    wq[4 * r] = vq.x; wq[4 * r + 1] = vq.y; wq[4 * r + 2] = vq.z; wq[4 * r + 3] = vq.w;
+    wp[4 * r] = vp.x; wp[4 * r + 1] = vp.y; wp[4 * r + 2] = vp.z; wp[4 * r + 3] = vp.w;
+  }
+  __nv_bfloat162 xq = as_bf162(wq[0]), xp = as_bf162(wp[0]);
+#pragma unroll
+  for (int i = 1; i < kRounds * 4; ++i) {
+    xq = __hmax2(xq, as_bf162(wq[i]));
+    xp = __hmax2(xp, as_bf162(wp[i]));
+  }
+  const float mqn = fmaxf(mq, fmaxf(__low2float(xq), __high2float(xq)));
+  const float mpn = fmaxf(mp, fmaxf(__low2float(xp), __high2float(xp)));
+  const float rq = refk(mqn, k), rp = refk(mpn, k);
+  const float dq = refk(mq, k) - rq, dp = refk(mp, k) - rp;
+  const float fq = ex2(dq), fp = ex2(dp);
+  float2 aq = __fmul2_rn(sq, make_float2(fq, fq));
+  float2 ap = __fmul2_rn(sp, make_float2(fp, fp));
+  float h0 = bc * ex2(0.5f * (dq + dp)), h1 = 0.0f;
+  const float2 kk = make_float2(k, k), nrq = make_float2(-rq, -rq), nrp = make_float2(-rp, -rp);
+  const float2 half = make_float2(0.5f, 0.5f);
+#pragma unroll
+  for (int i = 0; i < kRounds * 4; ++i) {
+    const float2 yq = make_float2(__uint_as_float(wq[i] << 16), __uint_as_float(wq[i] & 0xFFFF0000u));
+    const float2 yp = make_float2(__uint_as_float(wp[i] << 16), __uint_as_float(wp[i] & 0xFFFF0000u));
+    const float2 a = __ffma2_rn(yq, kk, nrq);
+    const float2 b = __ffma2_rn(yp, kk, nrp);
+    aq = __fadd2_rn(aq, make_float2(ex2(a.x), ex2(a.y)));
+    ap = __fadd2_rn(ap, make_float2(ex2(b.x), ex2(b.y)));
+    const float2 hh = __fmul2_rn(__fadd2_rn(a, b), half);
+    h0 += ex2(hh.x);
+    h1 += ex2(hh.y);
+  }
+  mq = mqn;
+  mp = mpn;
+  sq = aq;
+  sp = ap;
+  bc = h0 + h1;
 }
 
 // Weights of one chunk in the ring: per round, the warp's total weight (the
@@ -1114,17 +1157,26 @@ __device__ __forceinline__ int slice_weights(const Ring<E> &R, Shared &sh, uint3
   return stream_rev(R, sh, ph, order == kNewestFirstResident, body);
 }
 
-// Thread 0: turn sh.seg[0, nseg) into exclusive prefixes in vocabulary order
-// (chunk, round, warp); returns the slice total, also left in sh.seg[nseg].
-__device__ __forceinline__ float seg_prefix(Shared &sh, int nseg) {
-  float acc = 0.0f;
-  for (int i = 0; i < nseg; ++i) {
-    const float t = sh.seg[i];
+// One warp: turn sh.seg[0, nseg) into exclusive prefixes in vocabulary order
+// (chunk, round, warp); returns the slice total (in every lane), also left in
+// sh.seg[nseg].  Lane l sums its run of ceil(nseg / 32) entries in order, a warp
+// scan gives each run's start, and each lane writes its run's prefixes.
+__device__ __forceinline__ float seg_prefix(Shared &sh, int nseg, int lane) {
+  const int per = (nseg + 31) >> 5;
+  const int i0 = min(nseg, lane * per), i1 = min(nseg, i0 + per);
+  float t = 0.0f;
+  for (int i = i0; i < i1; ++i) t = __fadd_rn(t, sh.seg[i]);
+  const float incl = warp_incl_scan(t, lane);
+  float acc = __shfl_up_sync(0xFFFFFFFFu, incl, 1);
+  if (lane == 0) acc = 0.0f;
+  for (int i = i0; i < i1; ++i) {
+    const float v = sh.seg[i];
     sh.seg[i] = acc;
-    acc = __fadd_rn(acc, t);
+    acc = __fadd_rn(acc, v);
   }
-  sh.seg[nseg] = acc;
-  return acc;
+  const float tot = __shfl_sync(0xFFFFFFFFu, incl, 31);
+  if (lane == 0) sh.seg[nseg] = tot;
+  return tot;
 }
 
 __device__ __forceinline__ void flag_timeout(Shared &sh, const Params &P) {
@@ -1217,12 +1269,12 @@ __device__ __forceinline__ int search_segment(const E *sq, const E *sp, int n, b
 // Row pair (b, j < gamma) or bonus row (b, gamma) of a unit (pairs only for sc_row_stats).
 __device__ __forceinline__ void unit_coords(const Params &P, int unit, int &b, int &j) {
   const int G1 = P.gamma + 1;
-  if (P.mode == kVerify && SC_BONUS_LAST) {
-    // every pair unit first, then the bonus rows: the last, partial wave of CTAs
-    // holds the shorter (target-only) units
-    const int pairs = P.B * P.gamma;
-    b = unit < pairs ? unit / P.gamma : unit - pairs;
-    j = unit < pairs ? unit % P.gamma : P.gamma;
+  if (P.mode == kVerify && P.pos_major) {
+    // every sequence's position j before any sequence's position j + 1: a
+    // rejected pair then mostly finds an earlier rejection of its sequence
+    // already reported, and skips the residual pass of a row that is not j*
+    b = unit % P.B;
+    j = unit / P.B;
   } else if (P.mode == kVerify) {
     b = unit / G1;
     j = unit % G1;
@@ -1243,7 +1295,6 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int G1 = P.gamma + 1;
   const bool verify = P.mode == kVerify;
-  const int stride = static_cast<int>(gridDim.x) / C;  // clusters in the grid
   Shared &sh = *reinterpret_cast<Shared *>(smem_raw + static_cast<size_t>(kStages) * 2 * kCH * sizeof(E));
   if (tid == 0) {
     sh.timeout = 0;
@@ -1253,19 +1304,10 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
   }
-  uint32_t ph = 0;  // the ring's phase bits carry over from unit to unit
+  uint32_t ph = 0;  // phase bits of the ring's stages (see wait_stage)
 
-  // Every CTA of a cluster walks the same units: blockIdx / C, then + stride.
-  // The default launch has one cluster per unit (one iteration); with
-  // SC_PERSISTENT the grid holds only the clusters that fit on the GPU at once,
-  // and each hints its next unit's first chunks into L2 when its pass 1 ends.
-#if SC_PERSISTENT
-  for (int unit = static_cast<int>(blockIdx.x) / C, it = 0; unit < P.units; unit += stride, ++it) {
-#else
-  {
-    const int unit = static_cast<int>(blockIdx.x) / C, it = 0;
-#endif
-  const int slot = it & 1;  // exchange-1 slot set of this unit
+  // one cluster per unit: every CTA of the cluster works on unit blockIdx / C
+  const int unit = static_cast<int>(blockIdx.x) / C;
   int b, j;
   unit_coords(P, unit, b, j);
   const int v0 = rank * P.L;
@@ -1276,9 +1318,6 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   if (tid == 0) {
     sh.xq = NAN;
     sh.xp = NAN;
-    // a previous unit's draw wrote ring memory with ordinary stores (its chunk
-    // prefixes); order them before this unit's copies into the same stages
-    if (it > 0 && P.bulk) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
   prime(R, sh);
   float uj = 0.0f, ug = 0.0f;
@@ -1289,7 +1328,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     if (pair) x = P.tokens[static_cast<size_t>(b) * P.gamma + j];
   }
   __syncthreads();
-  if (it == 0) cluster_arrive_relaxed();  // this CTA has started (peers may store into it after their wait)
+  cluster_arrive_relaxed();  // this CTA has started (peers may store into it after their wait)
 
   // ---- pass 1: online max and sum of exponentials
   const float k = P.k;
@@ -1299,9 +1338,8 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   Top2 top = {-FLT_MAX, -FLT_MAX, -FLT_MAX};  // (kFamToken) the eta screen
   const bool scr_q = P.rule == SC_RULE_TOKEN_V1;
   // OPT: the pair's running sum of sqrt(q p) terms, relative to (r_q + r_p) / 2
-  const bool opt_bc = SC_OPT_UB && !kTok && !kExt && verify && pair && P.rule == SC_RULE_OPT;
-  const bool optlog_bc = SC_OPT_UB && kExt && verify && pair && !P.greedy && P.rule == SC_RULE_OPT_LOG;
-  float bc = 0.0f;
+  const bool opt_bc = SC_OPT_UB && P.opt_ub && !kTok && !kExt && verify && pair && P.rule == SC_RULE_OPT;
+  float bc = 0.0f;  // the pair's running sum of sqrt(q p) terms, relative to (r_q + r_p) / 2
   // the bonus row also leaves its per-(chunk, warp) totals for the sampler
   const bool bonus_tot = verify && !pair && !P.greedy;
   const int lx = x - v0;  // draft token's offset in this slice (thread 0 only)
@@ -1313,29 +1351,39 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     } else if constexpr (kExt) {
       const int vc = v0 + c * kCH;
       if (pair) {
-        if (n == kCH) ext_chunk<E, true, true>(R.q(s), R.p(s), n, vc, k, ex, optlog_bc, bc);
-        else ext_chunk<E, false, true>(R.q(s), R.p(s), n, vc, k, ex, optlog_bc, bc);
+        if (n == kCH) ext_chunk<E, true, true>(R.q(s), R.p(s), n, vc, k, ex);
+        else ext_chunk<E, false, true>(R.q(s), R.p(s), n, vc, k, ex);
       } else {
-        if (n == kCH) ext_chunk<E, true, false>(R.q(s), R.p(s), n, vc, k, ex, false, bc);
-        else ext_chunk<E, false, false>(R.q(s), R.p(s), n, vc, k, ex, false, bc);
+        if (n == kCH) ext_chunk<E, true, false>(R.q(s), R.p(s), n, vc, k, ex);
+        else ext_chunk<E, false, false>(R.q(s), R.p(s), n, vc, k, ex);
       }
     } else {
-      const float mq0 = mq, mp0 = mp;
-      if (n == kCH) {
-        if (pair) online_row<E, true>(R.q(s), n, k, mq, s2q);
-        online_row<E, true>(R.p(s), n, k, mp, s2p);
-        if (kTok && pair) screen_chunk<E, true>(scr_q ? R.q(s) : R.p(s), R.q(s), n, top);
-      } else {
-        if (pair) online_row<E, false>(R.q(s), n, k, mq, s2q);
-        online_row<E, false>(R.p(s), n, k, mp, s2p);
-        if (kTok && pair) screen_chunk<E, false>(scr_q ? R.q(s) : R.p(s), R.q(s), n, top);
+      bool fused = false;
+      if constexpr (sizeof(E) == 2) {
+        if (opt_bc && n == kCH) {
+          online_pair_bc(reinterpret_cast<const uint16_t *>(R.q(s)), reinterpret_cast<const uint16_t *>(R.p(s)),
+                         k, mq, s2q, mp, s2p, bc);
+          fused = true;
+        }
       }
-      if (opt_bc) {
-        const float rq = refk(mq, k), rp = refk(mp, k);
-        const float sc = ex2(0.5f * ((refk(mq0, k) - rq) + (refk(mp0, k) - rp)));
-        const float add = n == kCH ? bc_chunk<E, true>(R.q(s), R.p(s), n, 0.5f * k, 0.5f * (rq + rp))
-                                   : bc_chunk<E, false>(R.q(s), R.p(s), n, 0.5f * k, 0.5f * (rq + rp));
-        bc = fmaf(bc, sc, add);
+      if (!fused) {
+        const float mq0 = mq, mp0 = mp;
+        if (n == kCH) {
+          if (pair) online_row<E, true>(R.q(s), n, k, mq, s2q);
+          online_row<E, true>(R.p(s), n, k, mp, s2p);
+          if (kTok && pair) screen_chunk<E, true>(scr_q ? R.q(s) : R.p(s), R.q(s), n, top);
+        } else {
+          if (pair) online_row<E, false>(R.q(s), n, k, mq, s2q);
+          online_row<E, false>(R.p(s), n, k, mp, s2p);
+          if (kTok && pair) screen_chunk<E, false>(scr_q ? R.q(s) : R.p(s), R.q(s), n, top);
+        }
+        if (opt_bc) {
+          const float rq = refk(mq, k), rp = refk(mp, k);
+          const float sc = ex2(0.5f * ((refk(mq0, k) - rq) + (refk(mp0, k) - rp)));
+          const float add = n == kCH ? bc_chunk<E, true>(R.q(s), R.p(s), n, 0.5f * k, 0.5f * (rq + rp))
+                                     : bc_chunk<E, false>(R.q(s), R.p(s), n, 0.5f * k, 0.5f * (rq + rp));
+          bc = fmaf(bc, sc, add);
+        }
       }
     }
     if (tid == 0 && static_cast<unsigned>(lx - c * kCH) < static_cast<unsigned>(n)) {
@@ -1343,14 +1391,6 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       sh.xp = Elt<E>::at(R.p(s), lx - c * kCH);
     }
   });
-  if (SC_PERSISTENT && tid == 0 && P.bulk && unit + stride < P.units) {
-    // the next unit's first chunks stream into L2 while this one is exchanged,
-    // decided and reported; its pass 1 then finds them there
-    int bn, jn;
-    unit_coords(P, unit + stride, bn, jn);
-    const Ring<E> Rn = make_ring<E>(P, smem_raw, bn, jn, rank);
-    for (int c = 0; c < min(kStages, Rn.nch); ++c) Rn.prefetch(c);
-  }
   if constexpr (kExt) {
     if (bonus_tot) {
       ex.mp = mp;
@@ -1399,15 +1439,15 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       flag_timeout(sh, P);
     }
   }
-  if (it == 0) cluster_wait();  // every CTA of the cluster has started
+  cluster_wait();  // every CTA of the cluster has started
   if (tid == 0) {
     const float2 xv = make_float2(sh.xq, sh.xp);
     for (int r = 0; r < C; ++r) {
-      st_peer(peer_addr(&sh.all_ms[slot][rank], r), part);
-      st_peer(peer_addr(&sh.all_x[slot][rank], r), xv);
+      st_peer(peer_addr(&sh.all_ms[rank], r), part);
+      st_peer(peer_addr(&sh.all_x[rank], r), xv);
       if constexpr (kExt) {
-        st_peer(peer_addr(&sh.all_ext[slot][rank], r), part_ext);
-        st_peer(peer_addr(&sh.all_idx[slot][rank], r), part_idx);
+        st_peer(peer_addr(&sh.all_ext[rank], r), part_ext);
+        st_peer(peer_addr(&sh.all_idx[rank], r), part_idx);
       }
     }
   }
@@ -1419,15 +1459,15 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     ExtState g = ext_empty();
     float4 v;
     if constexpr (kExt) {
-      g = ext_load(sh.all_ms[slot][0], sh.all_ext[slot][0], sh.all_idx[slot][0]);
+      g = ext_load(sh.all_ms[0], sh.all_ext[0], sh.all_idx[0]);
       for (int r = 1; r < C; ++r)
-        ext_merge(g, ext_load(sh.all_ms[slot][r], sh.all_ext[slot][r], sh.all_idx[slot][r]), k);
+        ext_merge(g, ext_load(sh.all_ms[r], sh.all_ext[r], sh.all_idx[r]), k);
       v = make_float4(g.mq, g.sq, g.mp, g.sp);
     } else {
-      v = merge_partials(sh.all_ms[slot], C, k);
+      v = merge_partials(sh.all_ms, C, k);
     }
     const float a = v.x, as = v.y, c = v.z, cs = v.w;
-    const float2 xv = sh.all_x[slot][(x >= 0 && x < P.V) ? x / P.L : 0];
+    const float2 xv = sh.all_x[(x >= 0 && x < P.V) ? x / P.L : 0];
     const float yqx = xv.x, ypx = xv.y;
     // S = sum_v 2^{y_v k - R} with R = fl(M k); the max logit's own term is
     // 2^{fma(M, k, -R)}, so max_v q(v) = 2^{fma(M, k, -R)} / S.
@@ -1460,20 +1500,6 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     sh.qx = 0.0f;
     sh.pix = 0.0f;
     sh.c = pair && !err ? log2f(as / cs) : 0.0f;
-    if (bonus_tot) {
-      // p_gamma's chunk prefixes over this slice from pass 1's per-(chunk, warp)
-      // totals, re-referenced to R_p: what a sampling pass over the row would store
-      float *cp = P.bonus_pre + (static_cast<size_t>(b) * kMaxCluster + rank) * (kMaxChunks + 1);
-      float acc = 0.0f;
-      for (int c2 = 0; c2 < R.nch; ++c2) {
-        if (SC_CHECK(b < P.B && rank < kMaxCluster && c2 < kMaxChunks)) cp[c2] = acc;
-        float t = 0.0f;
-        for (int w = 0; w < kNW; ++w)
-          t = fmaf(sh.seg[c2 * kNW + w], ex2(refk(sh.seg[kBonusRef + c2 * kNW + w], k) - Rp), t);
-        acc = __fadd_rn(acc, t);
-      }
-      if (SC_CHECK(b < P.B && rank < kMaxCluster && R.nch <= kMaxChunks)) cp[R.nch] = err || tmo ? NAN : acc;
-    }
     sh.dl = sh.maxq;
     sh.dr = sh.maxp;
     float xent = 0.0f;  // (kFamExt) BiLD*'s discrepancy D(q, p) = -sum_v q log p, in nats
@@ -1485,6 +1511,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       sh.nhq = kLn2 * (g.aq / as - log2f(as));
       sh.nhp = kLn2 * (g.ap / cs - log2f(cs));
       xent = kLn2 * (log2f(cs) - g.x / as);
+      sh.klqp = sh.nhq + xent;
       if (P.greedy && pair && P.rule == SC_RULE_BILD && g.iq >= 0 && g.iq < P.V) {
         // greedy decoding: the BiLD baseline's D = -log p(argmax q), from the target
         // logit at q's argmax (one load; every CTA of the cluster reads the same value)
@@ -1559,6 +1586,22 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     sh.xp = ypx;
   }
   __syncthreads();
+  if (bonus_tot && warp == 0) {
+    // p_gamma's chunk prefixes over this slice from pass 1's per-(chunk, warp)
+    // totals, re-referenced to R_p: what a sampling pass over the row would store
+    // (lane c: chunk c; a warp scan in chunk order)
+    float t = 0.0f;
+    if (lane < R.nch)
+      for (int w = 0; w < kNW; ++w)
+        t = fmaf(sh.seg[lane * kNW + w], ex2(refk(sh.seg[kBonusRef + lane * kNW + w], k) - sh.Rp), t);
+    const float incl = warp_incl_scan(t, lane);
+    float excl = __shfl_up_sync(0xFFFFFFFFu, incl, 1);
+    if (lane == 0) excl = 0.0f;
+    float *cp = P.bonus_pre + (static_cast<size_t>(b) * kMaxCluster + rank) * (kMaxChunks + 1);
+    if (lane < R.nch && SC_CHECK(b < P.B && rank < kMaxCluster && lane < kMaxChunks)) cp[lane] = excl;
+    if (lane == max(R.nch - 1, 0) && SC_CHECK(b < P.B && rank < kMaxCluster && R.nch <= kMaxChunks))
+      cp[R.nch] = sh.err || tmo ? NAN : (R.nch > 0 ? incl : 0.0f);
+  }
 
   // ---- token rules: eta without a pass when the pass-1 screen settles it.  A
   // thread whose second-largest screened logit is deferred holds at most one
@@ -1597,13 +1640,18 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     __syncthreads();
   }
 
-  // ---- OPT band: a lower bound on D_TV from the pass-1 partials.  The threads'
-  // element sets partition the vocabulary, so sum_t max(0, P_t - Q_t) <= D_TV
-  // (P_t, Q_t: the probability mass of thread t's logits).  When alpha times
-  // that bound already reaches dr - dl (max p - max q for OPT, Eq. 10; the
-  // negative-entropy gap for OPTLog), delta = 0 for the exact D_TV too and the
-  // TV pass is skipped.  The bound carries ~1e-6 of f32
-  // rounding over its 128 C terms; only a clear 1e-4 excess settles the row.
+  // ---- OPT band: bounds on D_TV from the pass-1 partials.  The threads'
+  // logit sets partition the vocabulary, so sum_t max(0, P_t - Q_t) <= D_TV
+  // (P_t, Q_t: the probability mass of thread t's logits).  From above, OPT
+  // takes the Hellinger bound D_TV <= (1 - BC^2)^(1/2) with the Bhattacharyya
+  // coefficient BC = sum_v sqrt(q p) of pass 1, OPTLog Pinsker's
+  // D_TV <= (KL(q || p) / 2)^(1/2) from its entropy and cross entropy.  When alpha
+  // times the lower bound already reaches dr - dl (max p - max q for OPT, Eq. 10;
+  // the negative-entropy gap for OPTLog), delta = 0 for the exact D_TV too; when
+  // alpha times the upper bound stays below it, delta = 1; either way the TV pass
+  // is skipped.  The lower bound carries ~1e-6 of f32 rounding over its 128 C
+  // terms, BC is deflated and KL inflated well past their f32 errors: only a
+  // clear 1e-4 margin settles the row.
   if (sh.band) {
     const float pt = mine.w * ex2(refk(mine.z, k) - sh.Rp) / sh.Sp;
     const float qt = mine.y * ex2(refk(mine.x, k) - sh.Rq) / sh.Sq;
@@ -1629,20 +1677,23 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
         BCs = __fadd_rn(BCs, sh.all_lb[r].y);
       }
       const float gap = sh.dr - sh.dl;
+      float ub = INFINITY;
+      if (opt_bc) {
+        const float bcl = fminf(1.0f, BCs / sqrtf(sh.Sq) / sqrtf(sh.Sp)) * (1.0f - 2e-4f);
+        ub = sqrtf(fmaxf(0.0f, 1.0f - bcl * bcl));
+      } else if (kExt && SC_OPT_UB) {
+        const float kv = sh.klqp;  // NaN or +inf (masked logits) settle nothing
+        if (kv == kv)
+          ub = sqrtf(0.5f * fmaf(fmaxf(kv, 0.0f), 1.001f, 1e-5f * (1.0f + fabsf(sh.nhq) + fabsf(sh.nhq - kv))));
+      }
       if (P.alpha * LB - gap >= 1e-4f) {
         sh.need_p2 = 0;
         sh.delta = 0;
         accept_test<kFam>(sh, P, x, sh.xq, sh.xp, uj, k);
-      } else if (opt_bc || optlog_bc) {
-        // D_TV <= sqrt(1 - BC^2) (Hellinger): with BC deflated well past its f32
-        // error, alpha times that bound below the gap settles delta = 1 (Eq. 10, OPTLog)
-        const float bcl = fminf(1.0f, BCs / sqrtf(sh.Sq) / sqrtf(sh.Sp)) * (1.0f - 2e-4f);
-        const float ub = sqrtf(fmaxf(0.0f, 1.0f - bcl * bcl));
-        if (gap - P.alpha * ub >= 1e-4f) {
-          sh.need_p2 = 0;
-          sh.delta = 1;
-          accept_test<kFam>(sh, P, x, sh.xq, sh.xp, uj, k);
-        }
+      } else if (ub < INFINITY && gap - P.alpha * ub >= 1e-4f) {
+        sh.need_p2 = 0;
+        sh.delta = 1;
+        accept_test<kFam>(sh, P, x, sh.xq, sh.xp, uj, k);
       }
     }
     __syncthreads();
@@ -1655,13 +1706,15 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     tmo = slice_weights<kTok>(R, sh, ph, rs, kNewestFirstResident, lane, warp);
     tmo = __syncthreads_or(tmo);
     // exchange 2: push the slice total, one barrier, local reads
-    if (tid == 0) {
-      float acc = seg_prefix(sh, R.nch * kRounds * kNW);
-      if (tmo) {
-        acc = NAN;
-        flag_timeout(sh, P);
+    if (warp == 0) {
+      float acc = seg_prefix(sh, R.nch * kRounds * kNW, lane);
+      if (lane == 0) {
+        if (tmo) {
+          acc = NAN;
+          flag_timeout(sh, P);
+        }
+        for (int r = 0; r < C; ++r) st_peer(peer_addr(&sh.all_r[rank], r), acc);
       }
-      for (int r = 0; r < C; ++r) st_peer(peer_addr(&sh.all_r[rank], r), acc);
     }
     cluster_arrive();
     cluster_wait();
@@ -1705,10 +1758,11 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
                              sh.tok ? kTokenRes : kResidual, sh.on_q, sh.thr, sh.eta};
       tmo = slice_weights<kTok>(R, sh, ph, rs, sh.need_p2 ? kNewestFirst : kNewestFirstResident, lane, warp);
       tmo = __syncthreads_or(tmo);
-      if (tid == 0) {
-        seg_prefix(sh, R.nch * kRounds * kNW);
-        if (tmo) flag_timeout(sh, P);
+      if (warp == 0) {
+        seg_prefix(sh, R.nch * kRounds * kNW, lane);
+        if (lane == 0 && tmo) flag_timeout(sh, P);
       }
+      __syncthreads();
     }
     if (tid == 0) {
       float *cp = P.row_pre + ((static_cast<size_t>(b) * G1 + j) * kMaxCluster + rank) * (kMaxChunks + 1);
@@ -1812,8 +1866,10 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       const bool resident = js == j && !sh.need_p2;
       tmo = slice_weights<kTok>(Rj, sh, ph, rs, resident ? kNewestFirstResident : kNewestFirst, lane, warp);
       tmo = __syncthreads_or(tmo);
+      if (warp == 0) seg_prefix(sh, Rj.nch * kRounds * kNW, lane);
+      __syncthreads();
       if (tid == 0) {
-        float tot_r = seg_prefix(sh, Rj.nch * kRounds * kNW);
+        float tot_r = sh.seg[Rj.nch * kRounds * kNW];
         if (tmo) {
           tot_r = NAN;
           flag_timeout(sh, P);
@@ -2006,7 +2062,6 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       }
     }
   }
-  }  // units
   if (sh.timeout && tid == 0 && P.bulk) {
     // let copies still in flight land before this CTA's shared memory is released
     for (int s = 0; s < kStages; ++s) mbar_wait(&sh.full[s], 0), mbar_wait(&sh.full[s], 1);
@@ -2020,7 +2075,6 @@ struct DeviceInfo {
   int smem_optin = 0;
   int sms = 0;
   bool configured[6] = {};  // [dtype][rule family]
-  int max_clusters[6][kMaxCluster + 1] = {};  // co-resident clusters per [kernel][C] (-1: unknown)
 };
 
 DeviceInfo g_dev[64];
@@ -2164,6 +2218,19 @@ int launch(Params P, cudaStream_t stream, int units) {
   // earlier rejection; the owners then never stream a second pass.
   P.spec_res = 1;
   if (const char *e = getenv("SC_SPEC_RES")) P.spec_res = atoi(e) != 0;
+  // Position-major unit order (every sequence's position j before any position
+  // j + 1): a rejected pair then mostly sees its sequence's earlier rejection
+  // already reported and skips its residual pass (B=512, gamma=8: Chow 834 ->
+  // 738 us, OPT 874 -> 837 us; Diff unchanged).
+  P.pos_major = 1;
+  if (const char *e = getenv("SC_POS_MAJOR")) P.pos_major = atoi(e) != 0;
+  // The upper bound on D_TV costs OPT pairs one more exponential per logit pair
+  // in pass 1 and saves the TV pass of the band rows it settles.  With slices of
+  // up to 64000 logits (C <= 4, large batches) that pass mostly re-reads HBM and
+  // the bound pays (B=512, gamma=8: 873 -> 809 us); with the shorter slices of
+  // small batches the bound costs more than it saves (B=64, gamma=8: 143 -> 155 us).
+  P.opt_ub = C <= 4;
+  if (const char *e = getenv("SC_OPT_UB")) P.opt_ub = atoi(e) != 0;
   const size_t row_bytes = static_cast<size_t>(P.V) * sizeof(E);
   P.bulk = (row_bytes % 16 == 0) && (reinterpret_cast<uintptr_t>(P.draft) % 16 == 0) &&
            (reinterpret_cast<uintptr_t>(P.target) % 16 == 0);
@@ -2171,7 +2238,6 @@ int launch(Params P, cudaStream_t stream, int units) {
   if (units == 0) return SC_OK;
 
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(static_cast<unsigned>(C), 1, 1);
   cfg.blockDim = dim3(kNT, 1, 1);
   cfg.dynamicSmemBytes = smem_bytes<E>();
   cfg.stream = stream;
@@ -2182,21 +2248,8 @@ int launch(Params P, cudaStream_t stream, int units) {
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  // one cluster per unit, or (SC_PERSISTENT) as many as fit on the GPU at once,
-  // each looping over its share of the units; the kernel is correct for any grid
-  // since no cluster waits on another
-  int clusters = units;
-  if (SC_PERSISTENT) {
-    std::lock_guard<std::mutex> lock(g_mu);
-    int &mc = di.max_clusters[ti][C];
-    if (mc == 0) {
-      int n = 0;
-      mc = cudaOccupancyMaxActiveClusters(&n, kernel, &cfg) == cudaSuccess && n > 0 ? n : -1;
-      cudaGetLastError();
-    }
-    if (mc > 0 && mc < units) clusters = mc;
-  }
-  cfg.gridDim = dim3(static_cast<unsigned>(clusters) * static_cast<unsigned>(C), 1, 1);
+  // one cluster per unit; no cluster ever waits on another
+  cfg.gridDim = dim3(static_cast<unsigned>(units) * static_cast<unsigned>(C), 1, 1);
   if (cudaLaunchKernelEx(&cfg, kernel, P) != cudaSuccess) return SC_ERR_CUDA;
   return SC_OK;
 }

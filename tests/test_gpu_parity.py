@@ -377,13 +377,17 @@ def test_cuda_graph_capture_and_replay(sc, rule, alpha):
 
 
 @pytest.mark.parametrize("alpha", [0.2, 0.5, 1.0])
-def test_opt_band_settled_by_tv_bounds(sc, alpha):
+@pytest.mark.parametrize("ub", ["1", "0"])
+def test_opt_band_settled_by_tv_bounds(sc, monkeypatch, alpha, ub):
     # Inside the OPT band (max p - alpha <= max q < max p) the kernel first bounds
-    # D_TV from below by its threads' partial masses (settling delta = 0) and from
-    # above by sqrt(1 - BC^2), BC = sum_v sqrt(q p) (settling delta = 1); settled
-    # rows report no TV (-1).  Their decisions must still be the oracle's.
+    # D_TV from below by its threads' partial masses (settling delta = 0) and,
+    # where it accumulates BC = sum_v sqrt(q p) (SC_OPT_UB=1; by default only for
+    # the long slices of large batches), from above by sqrt(1 - BC^2) (settling
+    # delta = 1); settled rows report no TV (-1).  Their decisions must still be
+    # the oracle's, with the upper bound and without it.
     from paper_2405_19261_gb300.workloads import logits_as_f64
     from scipy.special import softmax
+    monkeypatch.setenv("SC_OPT_UB", ub)
     w = synthetic(24, 8, 256000, dtype="bf16", kind="zipf", sigma=0.7, rule="opt", alpha=alpha,
                   temperature=1.0, seed=31)
     gpu = run_gpu(sc, w)
@@ -403,9 +407,12 @@ def test_opt_band_settled_by_tv_bounds(sc, alpha):
     q = softmax(logits_as_f64(w.draft, "bf16"), axis=-1)
     p = softmax(logits_as_f64(w.target[:, :w.gamma], "bf16"), axis=-1)
     bc = np.minimum(1.0, np.sum(np.sqrt(q * p), axis=-1)) * (1.0 - 2e-4)
-    ub = np.sqrt(np.maximum(0.0, 1.0 - bc ** 2))
-    clear = band & (maxp - maxq - alpha * ub >= 1e-3)
-    np.testing.assert_array_equal(tv[clear], -1.0)
+    hub = np.sqrt(np.maximum(0.0, 1.0 - bc ** 2))
+    clear = band & (maxp - maxq - alpha * hub >= 1e-3)
+    if ub == "1":
+        np.testing.assert_array_equal(tv[clear], -1.0)
+    else:  # without the upper bound these rows take the TV pass
+        np.testing.assert_allclose(tv[clear], ref.row("tv")[clear], atol=TOL)
     np.testing.assert_array_equal(ri[..., 3][clear], 1.0)
 
 

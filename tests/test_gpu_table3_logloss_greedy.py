@@ -164,22 +164,24 @@ def test_entropy_rules_flat_rows_and_temperature(sc, rule, alpha):
 @pytest.mark.parametrize("alpha", [0.3, 0.6])
 def test_opt_log_band_settled_by_tv_bounds(sc, alpha):
     # OPTLog's band (sum p ln p - alpha <= sum q ln q < sum p ln p) is narrowed like
-    # OPT's: the partition bound settles delta = 0, sqrt(1 - BC^2) settles delta = 1;
-    # settled rows report no TV, and every row the upper bound clearly decides is settled
-    from scipy.special import softmax
+    # OPT's: the partition bound settles delta = 0, Pinsker's (KL(q || p) / 2)^(1/2),
+    # KL(q || p) = sum q ln q - sum q ln p from the moment kernel's entropies,
+    # settles delta = 1; settled rows report no TV, and every row the upper bound
+    # clearly decides is settled
+    from scipy.special import log_softmax
     from scipy.stats import entropy
     w = synthetic(24, 6, 32128, dtype="bf16", kind="zipf", sigma=0.7, rule="opt_log", alpha=alpha, seed=73)
     gpu = run_gpu(sc, w)
     ref = oracle.verify_workload(w)
     assert_parity(w, gpu, ref)
     ri = gpu[2][:, :w.gamma]
-    q = softmax(logits_as_f64(w.draft, "bf16"), axis=-1)
-    p = softmax(logits_as_f64(w.target[:, :w.gamma], "bf16"), axis=-1)
+    lq = log_softmax(logits_as_f64(w.draft, "bf16"), axis=-1)
+    lp = log_softmax(logits_as_f64(w.target[:, :w.gamma], "bf16"), axis=-1)
+    q, p = np.exp(lq), np.exp(lp)
     gap = entropy(q, axis=-1) - entropy(p, axis=-1)          # sum p ln p - sum q ln q
     band = (gap > 0) & (gap <= alpha)
-    bc = np.minimum(1.0, np.sum(np.sqrt(q * p), axis=-1)) * (1.0 - 2e-4)  # as the kernel shrinks it
-    ub = np.sqrt(np.maximum(0.0, 1.0 - bc ** 2))
-    clear = band & (gap - alpha * ub >= 1e-3)
+    pinsker = np.sqrt(0.5 * (q * (lq - lp)).sum(-1) * 1.001)
+    clear = band & (gap - alpha * pinsker >= 1e-3)
     assert clear.sum() > 0
     np.testing.assert_array_equal(ri[..., 2][clear], -1.0)
     np.testing.assert_array_equal(ri[..., 3][clear], 1.0)
