@@ -616,6 +616,92 @@ __device__ __forceinline__ void ext_chunk(const E *srcq, const E *srcp, int n, i
   st.x = __fadd_rn(st.x, x);
 }
 
+// kFamExt pass 1 of a pair, full bf16 chunk: ext_chunk's maxima, argmaxes,
+// sums and moments in one read of shared memory, two logits at a time.  The
+// maxima come from packed bf16x2 max trees; only a chunk that raises a running
+// maximum is scanned for the lowest index holding it (later chunks hold higher
+// indices, so an equal maximum keeps the earlier one).  The moments take the
+// logits clamped at -1e30, so that a masked (-inf) logit gives 2^a = 0 and a
+// finite product 0 * a = 0 where ext_chunk skips the term; a finite draft logit
+// with a masked target logit still makes X = -inf (D(q, p) = +inf), found by a
+// scan of the chunks whose target minimum is -inf.
+__device__ __forceinline__ int first_index_of(const uint32_t (&w)[kRounds * 4], float m, int v0) {
+#pragma unroll
+  for (int i = 0; i < kRounds * 4; ++i) {
+    const int e = 8 * ((i >> 2) * kNT + static_cast<int>(threadIdx.x)) + 2 * (i & 3);
+    if (__uint_as_float(w[i] << 16) == m) return v0 + e;
+    if (__uint_as_float(w[i] & 0xFFFF0000u) == m) return v0 + e + 1;
+  }
+  return -1;
+}
+
+__device__ __forceinline__ void ext_pair_bf16(const uint16_t *srcq, const uint16_t *srcp, int v0, float k,
+                                              ExtState &st) {
+  uint32_t wq[kRounds * 4], wp[kRounds * 4];
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r) {
+    const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
+    const uint4 vq = *reinterpret_cast<const uint4 *>(srcq + e);
+    const uint4 vp = *reinterpret_cast<const uint4 *>(srcp + e);
+    wq[4 * r] = vq.x; wq[4 * r + 1] = vq.y; wq[4 * r + 2] = vq.z; wq[4 * r + 3] = vq.w;
+    wp[4 * r] = vp.x; wp[4 * r + 1] = vp.y; wp[4 * r + 2] = vp.z; wp[4 * r + 3] = vp.w;
+  }
+  __nv_bfloat162 xq = as_bf162(wq[0]), xp = as_bf162(wp[0]), np = as_bf162(wp[0]);
+#pragma unroll
+  for (int i = 1; i < kRounds * 4; ++i) {
+    xq = __hmax2(xq, as_bf162(wq[i]));
+    xp = __hmax2(xp, as_bf162(wp[i]));
+    np = __hmin2(np, as_bf162(wp[i]));
+  }
+  const float cq = fmaxf(__low2float(xq), __high2float(xq));
+  const float cp = fmaxf(__low2float(xp), __high2float(xp));
+  float mq = st.mq, mp = st.mp;
+  int iq = st.iq, ip = st.ip;
+  if (cq > mq) {
+    mq = cq;
+    iq = first_index_of(wq, cq, v0);
+  }
+  if (cp > mp) {
+    mp = cp;
+    ip = first_index_of(wp, cp, v0);
+  }
+  const float rq = refk(mq, k), rp = refk(mp, k);
+  ext_rebase(st, refk(st.mq, k) - rq, refk(st.mp, k) - rp);
+  const __nv_bfloat162 lo = __float2bfloat162_rn(-1e30f);
+  const float2 kk = make_float2(k, k), nrq = make_float2(-rq, -rq), nrp = make_float2(-rp, -rp);
+  float2 sq = make_float2(0.0f, 0.0f), aq = sq, sp = sq, ap = sq, x = sq;
+#pragma unroll
+  for (int i = 0; i < kRounds * 4; ++i) {
+    const __nv_bfloat162 q2 = __hmax2(as_bf162(wq[i]), lo), p2 = __hmax2(as_bf162(wp[i]), lo);
+    const float2 a = __ffma2_rn(__bfloat1622float2(q2), kk, nrq);
+    const float2 b = __ffma2_rn(__bfloat1622float2(p2), kk, nrp);
+    const float2 ea = make_float2(ex2(a.x), ex2(a.y)), eb = make_float2(ex2(b.x), ex2(b.y));
+    sq = __fadd2_rn(sq, ea);
+    sp = __fadd2_rn(sp, eb);
+    aq = __ffma2_rn(ea, a, aq);
+    ap = __ffma2_rn(eb, b, ap);
+    x = __ffma2_rn(ea, b, x);
+  }
+  bool inf_x = false;
+  if (!(fminf(__low2float(np), __high2float(np)) > -INFINITY)) {
+#pragma unroll
+    for (int i = 0; i < kRounds * 4; ++i) {
+      const float q0 = __uint_as_float(wq[i] << 16), q1 = __uint_as_float(wq[i] & 0xFFFF0000u);
+      const float p0 = __uint_as_float(wp[i] << 16), p1 = __uint_as_float(wp[i] & 0xFFFF0000u);
+      inf_x |= (q0 > -INFINITY && !(p0 > -INFINITY)) || (q1 > -INFINITY && !(p1 > -INFINITY));
+    }
+  }
+  st.mq = mq;
+  st.mp = mp;
+  st.iq = iq;
+  st.ip = ip;
+  st.sq = __fadd_rn(st.sq, sq.x + sq.y);
+  st.aq = __fadd_rn(st.aq, aq.x + aq.y);
+  st.sp = __fadd_rn(st.sp, sp.x + sp.y);
+  st.ap = __fadd_rn(st.ap, ap.x + ap.y);
+  st.x = inf_x ? -INFINITY : __fadd_rn(st.x, x.x + x.y);
+}
+
 // Pass-1 screen of a token rule: per thread, the two largest logits of the row
 // that r(v) tests (q for TokenV1, p otherwise) and the draft logit at the
 // largest.  When every thread's second largest turns out deferred (r = 1), the
@@ -1351,8 +1437,18 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     } else if constexpr (kExt) {
       const int vc = v0 + c * kCH;
       if (pair) {
-        if (n == kCH) ext_chunk<E, true, true>(R.q(s), R.p(s), n, vc, k, ex);
-        else ext_chunk<E, false, true>(R.q(s), R.p(s), n, vc, k, ex);
+        bool done = false;
+        if constexpr (sizeof(E) == 2) {
+          if (n == kCH) {
+            ext_pair_bf16(reinterpret_cast<const uint16_t *>(R.q(s)), reinterpret_cast<const uint16_t *>(R.p(s)),
+                          vc, k, ex);
+            done = true;
+          }
+        }
+        if (!done) {
+          if (n == kCH) ext_chunk<E, true, true>(R.q(s), R.p(s), n, vc, k, ex);
+          else ext_chunk<E, false, true>(R.q(s), R.p(s), n, vc, k, ex);
+        }
       } else {
         if (n == kCH) ext_chunk<E, true, false>(R.q(s), R.p(s), n, vc, k, ex);
         else ext_chunk<E, false, false>(R.q(s), R.p(s), n, vc, k, ex);
