@@ -98,8 +98,9 @@ typedef enum {
  * measurements (the default layout is chosen from V, the batch and the SM count):
  *   SC_SLICE=n    logits per CTA slice of a row (n >= 64, rounded to a multiple of 8)
  *   SC_CLUSTER=c  CTAs per row pair (1 <= c <= 16; raised if the slices would not fit)
- *   SC_SPEC_RES=0|1  whether rejected pairs store their own residual prefixes (default 1)
- *                 or leave them to the owners' sampling passes
+ *   SC_SPEC_RES=0|1  whether a rejected pair that is certainly row j* (every earlier
+ *                 position of its slice reported without a rejection) stores its own
+ *                 residual prefixes (default 1), or the owners always sample
  *   SC_POS_MAJOR=0|1 units in position-major order (default 1) or sequence-major
  *   SC_OPT_UB=0|1 whether OPT pairs accumulate the Bhattacharyya coefficient in
  *                 pass 1 for an upper bound on D_TV that settles band rows without

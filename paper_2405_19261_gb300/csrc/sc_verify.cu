@@ -137,7 +137,8 @@ struct Params {
   uint32_t *seq_tickets;   // [B] finished sample passes (+1 for rank 0's last arrival); zero at rest
   float4 *records;         // [B][kMaxCluster][gamma+1] (R_q, R_p, c, flags) as seen by rank r
   float4 *records2;        // [B][kMaxCluster][gamma+1] (eta, thr, token, on_q) of token rules
-  int spec_res;            // a rejected pair stores its residual's chunk prefixes itself (row_pre)
+  int spec_res;            // a rejected pair that is certainly row j* stores its residual's chunk
+                           // prefixes itself (row_pre); 0: the owners always sample
   int pos_major;           // units in position-major order: (b, j) is unit j B + b
   int opt_ub;              // OPT pairs accumulate sqrt(q p) in pass 1 for an upper bound on D_TV
   float *row_pre;          // [B][gamma+1][kMaxCluster][kMaxChunks + 1] those prefixes, per row
@@ -326,7 +327,7 @@ struct __align__(16) Shared {
   int iq, ip;               // (kFamExt) argmax q and argmax p, lowest index on ties
   float thr, eta;           // its r(v) threshold (exponent domain) and eta = sum_v r(v) q(v)
   // sequence finish
-  int spec_skip;            // a rejection of an earlier position is already reported: not row j*
+  int self_res;             // this rejected pair stores its residual's chunk prefixes (row_pre)
   int owner;                // this CTA runs its rank's sample pass of row j*
   int scan_records;         // j* must be read from the records (gamma + 1 > 32)
   int seq_last;             // the sequence's last finisher: draws the token
@@ -1591,7 +1592,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     sh.thr = -INFINITY;
     sh.eta = 0.0f;
     sh.accept = 0;
-    sh.spec_skip = 0;
+    sh.self_res = 0;
     sh.tv = -1.0f;
     sh.qx = 0.0f;
     sh.pix = 0.0f;
@@ -1833,21 +1834,28 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     __syncthreads();
   }
 
-  // ---- small batches: a rejected pair stores its own residual's chunk prefixes
-  // now, while its slice is in the ring and in L2, so that no pass is left for
-  // the end of the sequence's chain (the row is j* unless an earlier one also
-  // rejects).  The OPT band's TV pass has summed exactly these weights already.
-  // A rejected pair whose rank already shows a rejection at an earlier position
-  // is not row j* and skips the pass (a stale read of the ticket only costs the
-  // pass; row j* itself never sees an earlier rejection).
-  if (P.spec_res && verify && pair && !sh.accept && !sh.err && !(kExt && P.greedy) && j > 0 && G1 <= 32) {
+  // ---- a rejected pair that is certainly row j* of its sequence stores its own
+  // residual's chunk prefixes now, while its slice is in the ring and in L2, so
+  // that no sampling pass is left for the end of the sequence's chain: certain
+  // when every earlier position of this slice rank has reported without a
+  // rejection.  A rejected pair whose rank shows an earlier rejection is not j*;
+  // one whose earlier positions have not all reported leaves the pass to the
+  // owner that settles j* (so no row but j* is ever sampled).  An OPT band row's
+  // TV pass has summed exactly these weights already: it always stores them.
+  // Drafts longer than 32 positions (an arrival count, no bits) leave it to the owner.
+  if (P.spec_res && verify && pair && !sh.accept && !sh.err && !(kExt && P.greedy)) {
     if (tid == 0) {
-      const unsigned long long t = __ldcg(P.rank_tickets + static_cast<size_t>(b) * kMaxCluster + rank);
-      sh.spec_skip = ((t >> 32) & ((1ull << j) - 1ull)) != 0ull;
+      int self = sh.need_p2 && !sh.tok;
+      if (!self && G1 <= 32) {
+        const unsigned long long t = __ldcg(P.rank_tickets + static_cast<size_t>(b) * kMaxCluster + rank);
+        const unsigned long long earlier = (1ull << j) - 1ull;
+        self = ((t >> 32) & earlier) == 0ull && (t & earlier) == earlier;
+      }
+      sh.self_res = self;
     }
     __syncthreads();
   }
-  if (P.spec_res && verify && pair && !sh.accept && !sh.err && !(kExt && P.greedy) && !sh.spec_skip) {
+  if (sh.self_res) {
     if (!(sh.need_p2 && !sh.tok)) {
       const bool lossy = kFam == kFamCascade && P.rule == SC_RULE_LOSSY;
       const RowScalars rs = {sh.Rq, sh.Rp, k, lossy ? sh.c + P.lossy_c : sh.c,
@@ -1884,7 +1892,8 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     float4 *rec = P.records + (static_cast<size_t>(b) * kMaxCluster + rank) * G1;
     float4 *rec2 = P.records2 + (static_cast<size_t>(b) * kMaxCluster + rank) * G1;
     if (tid == 0) {
-      const int flags = (sh.accept ? 1 : 0) | (sh.err ? 2 : 0);
+      // flags: 1 accepted, 2 invalid, 4 this rank's residual prefixes are in row_pre
+      const int flags = (sh.accept ? 1 : 0) | (sh.err ? 2 : 0) | (sh.self_res ? 4 : 0);
       float4 r1 = make_float4(sh.Rq, sh.Rp, sh.c, __int_as_float(flags));
       if (kFam == kFamCascade && P.rule == SC_RULE_LOSSY)
         r1.z = sh.c + P.lossy_c;  // the residual max(0, p / beta - q) (Lemma 2)
@@ -1946,10 +1955,10 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     }
     __syncthreads();
 
-    if (sh.owner && ((kExt && P.greedy) || sh.jstar == P.gamma || P.spec_res)) {
+    if (sh.owner && ((kExt && P.greedy) || sh.jstar == P.gamma || (__float_as_int(sh.rj.w) & 4))) {
       // nothing to sample: greedy decoding emits row j*'s argmax p (in the
-      // records), the bonus row's chunk prefixes came from its pass 1, and
-      // with spec_res row j* stored its own
+      // records), the bonus row's chunk prefixes came from its pass 1, or row
+      // j* stored this rank's prefixes itself (flag 4 of its record)
       if (tid == 0) sh.seq_last = atom_add_acq_rel(P.seq_tickets + b, 1u) == static_cast<uint32_t>(C);
       __syncthreads();
     } else if (sh.owner) {
@@ -2015,15 +2024,23 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       }
       __syncthreads();
       const int js = sh.jstar;
-      // one round of loads: every slice's chunk prefixes of row j* (ending in its total)
-      const float *cpg = js == P.gamma ? P.bonus_pre + static_cast<size_t>(b) * kMaxCluster * kCP
-                         : P.spec_res  ? P.row_pre + (static_cast<size_t>(b) * G1 + js) * kMaxCluster * kCP
-                                       : P.chunk_pre + static_cast<size_t>(b) * kMaxCluster * kCP;
+      // one round of loads: every slice's chunk prefixes of row j* (ending in its
+      // total), from the bonus row's pass 1, from row j* itself (flag 4 of that
+      // rank's record) or from that rank's owner
+      const float *bonus = P.bonus_pre + static_cast<size_t>(b) * kMaxCluster * kCP;
+      const float *self = P.row_pre + (static_cast<size_t>(b) * G1 + js) * kMaxCluster * kCP;
+      const float *owned = P.chunk_pre + static_cast<size_t>(b) * kMaxCluster * kCP;
       for (int i = tid; i < C * kCP && !(kExt && P.greedy); i += kNT) {
         const int r = i / kCP, c = i % kCP;
         const int len = max(0, min(P.L, P.V - r * P.L));
-        if (c <= (len + kCH - 1) / kCH && SC_CHECK(b < P.B && js <= P.gamma && C <= kMaxCluster))
-          cpall[i] = __ldcg(cpg + i);
+        if (c <= (len + kCH - 1) / kCH && SC_CHECK(b < P.B && js <= P.gamma && C <= kMaxCluster)) {
+          const float *src = bonus;
+          if (js < P.gamma) {
+            const int f = __float_as_int(__ldcg(&P.records[(static_cast<size_t>(b) * kMaxCluster + r) * G1 + js].w));
+            src = (f & 4) ? self : owned;
+          }
+          cpall[i] = __ldcg(src + i);
+        }
       }
       __syncthreads();
       if (kExt && P.greedy) {
