@@ -306,7 +306,7 @@ struct __align__(16) Shared {
   float4 all_ms[kMaxCluster];  // 1: (m_q, s_q, m_p, s_p) of the slice
   float2 all_x[kMaxCluster];   // 1: raw logits at the draft token, if in the slice
   float all_r[kMaxCluster];    // 2 (TV pass): the slice's total residual weight
-  float2 all_lb[kMaxCluster];  // OPT band: the slice's lower bound on D_TV, and its sum of sqrt(q p)
+  float2 all_lb[kMaxCluster];  // OPT band: the slice's parts of the lower and upper bounds on D_TV
   float2 all_scr[kMaxCluster]; // token rules: the slice's sum of q over its undeferred tokens, and
                                // whether its screen is exact (1) or not (0)
   float4 all_ext[kMaxCluster];  // 1 (kFamExt): (A_q, A_p, X, -) of the slice, see ExtState
@@ -876,7 +876,7 @@ __device__ __forceinline__ void bonus_row(const E *src, int n, float k, float &m
 // sqrt(q_v p_v) up to the rows' normalisers: the Bhattacharyya coefficient
 // BC = sum_v sqrt(q_v p_v) bounds D_TV from above, D_TV <= sqrt(1 - BC^2).
 template <typename E, bool kFull>
-__device__ __forceinline__ float bc_chunk(const E *srcq, const E *srcp, int n, float hk, float hr) {
+__device__ __forceinline__ float2 bc_chunk(const E *srcq, const E *srcp, int n, float hk, float hr) {
   float acc0 = 0.0f, acc1 = 0.0f;
 #pragma unroll
   for (int r = 0; r < kRounds; ++r) {
@@ -890,7 +890,7 @@ __device__ __forceinline__ float bc_chunk(const E *srcq, const E *srcp, int n, f
       acc1 += ex2(fmaf(yq[i + 1] + yp[i + 1], hk, -hr));
     }
   }
-  return acc0 + acc1;
+  return make_float2(acc0, acc1);  // (even, odd logits)
 }
 
 // OPT pair, full bf16 chunk: online_row of both rows and the chunk's
@@ -899,7 +899,7 @@ __device__ __forceinline__ float bc_chunk(const E *srcq, const E *srcp, int n, f
 // relative to the rows' updated references, as in bc_chunk, and the running
 // sums are rescaled as online_row rescales its sums.
 __device__ __forceinline__ void online_pair_bc(const uint16_t *srcq, const uint16_t *srcp, float k,
-                                               float &mq, float2 &sq, float &mp, float2 &sp, float &bc) {
+                                               float &mq, float2 &sq, float &mp, float2 &sp, float2 &bc) {
   uint32_t wq[kRounds * 4], wp[kRounds * 4];
 #pragma unroll
   for (int r = 0; r < kRounds; ++r) {
@@ -922,7 +922,8 @@ __device__ __forceinline__ void online_pair_bc(const uint16_t *srcq, const uint1
   const float fq = ex2(dq), fp = ex2(dp);
   float2 aq = __fmul2_rn(sq, make_float2(fq, fq));
   float2 ap = __fmul2_rn(sp, make_float2(fp, fp));
-  float h0 = bc * ex2(0.5f * (dq + dp)), h1 = 0.0f;
+  const float fb = ex2(0.5f * (dq + dp));
+  float h0 = bc.x * fb, h1 = bc.y * fb;
   const float2 kk = make_float2(k, k), nrq = make_float2(-rq, -rq), nrp = make_float2(-rp, -rp);
   const float2 half = make_float2(0.5f, 0.5f);
 #pragma unroll
@@ -941,7 +942,7 @@ __device__ __forceinline__ void online_pair_bc(const uint16_t *srcq, const uint1
   mp = mpn;
   sq = aq;
   sp = ap;
-  bc = h0 + h1;
+  bc = make_float2(h0, h1);
 }
 
 // Weights of one chunk in the ring: per round, the warp's total weight (the
@@ -1426,7 +1427,9 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   const bool scr_q = P.rule == SC_RULE_TOKEN_V1;
   // OPT: the pair's running sum of sqrt(q p) terms, relative to (r_q + r_p) / 2
   const bool opt_bc = SC_OPT_UB && P.opt_ub && !kTok && !kExt && verify && pair && P.rule == SC_RULE_OPT;
-  float bc = 0.0f;  // the pair's running sum of sqrt(q p) terms, relative to (r_q + r_p) / 2
+  // the pair's running sums of sqrt(q p) terms over this thread's even and odd logits,
+  // relative to (r_q + r_p) / 2
+  float2 bc = make_float2(0.0f, 0.0f);
   // the bonus row also leaves its per-(chunk, warp) totals for the sampler
   const bool bonus_tot = verify && !pair && !P.greedy;
   const int lx = x - v0;  // draft token's offset in this slice (thread 0 only)
@@ -1477,9 +1480,9 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
         if (opt_bc) {
           const float rq = refk(mq, k), rp = refk(mp, k);
           const float sc = ex2(0.5f * ((refk(mq0, k) - rq) + (refk(mp0, k) - rp)));
-          const float add = n == kCH ? bc_chunk<E, true>(R.q(s), R.p(s), n, 0.5f * k, 0.5f * (rq + rp))
-                                     : bc_chunk<E, false>(R.q(s), R.p(s), n, 0.5f * k, 0.5f * (rq + rp));
-          bc = fmaf(bc, sc, add);
+          const float2 add = n == kCH ? bc_chunk<E, true>(R.q(s), R.p(s), n, 0.5f * k, 0.5f * (rq + rp))
+                                      : bc_chunk<E, false>(R.q(s), R.p(s), n, 0.5f * k, 0.5f * (rq + rp));
+          bc = make_float2(fmaf(bc.x, sc, add.x), fmaf(bc.y, sc, add.y));
         }
       }
     }
@@ -1499,7 +1502,8 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     s2p = make_float2(ex.sp, 0.0f);
   }
   float s_q = s2q.x + s2q.y, s_p = s2p.x + s2p.y;
-  const float4 mine = make_float4(mq, s_q, mp, s_p);  // this thread's partial, kept for the D_TV bound
+  const float4 mine = make_float4(mq, s_q, mp, s_p);  // this thread's partial, kept for the D_TV bounds
+  const float4 mine2 = make_float4(s2q.x, s2q.y, s2p.x, s2p.y);  // ... split over its even and odd logits
   tmo = __syncthreads_or(tmo);
   if constexpr (kExt) {
     ext_warp_merge(ex, k);
@@ -1737,24 +1741,33 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     __syncthreads();
   }
 
-  // ---- OPT band: bounds on D_TV from the pass-1 partials.  The threads'
-  // logit sets partition the vocabulary, so sum_t max(0, P_t - Q_t) <= D_TV
-  // (P_t, Q_t: the probability mass of thread t's logits).  From above, OPT
-  // takes the Hellinger bound D_TV <= (1 - BC^2)^(1/2) with the Bhattacharyya
-  // coefficient BC = sum_v sqrt(q p) of pass 1, OPTLog Pinsker's
-  // D_TV <= (KL(q || p) / 2)^(1/2) from its entropy and cross entropy.  When alpha
-  // times the lower bound already reaches dr - dl (max p - max q for OPT, Eq. 10;
-  // the negative-entropy gap for OPTLog), delta = 0 for the exact D_TV too; when
-  // alpha times the upper bound stays below it, delta = 1; either way the TV pass
-  // is skipped.  The lower bound carries ~1e-6 of f32 rounding over its 128 C
-  // terms, BC is deflated and KL inflated well past their f32 errors: only a
-  // clear 1e-4 margin settles the row.
+  // ---- OPT band: bounds on D_TV from the pass-1 partials.  Each thread's even
+  // and odd logits form two sets t (the two lanes of its packed sums), with
+  // masses P_t, Q_t; the sets partition the vocabulary, so
+  // sum_t max(0, P_t - Q_t) <= D_TV.  From above, OPT takes Cauchy-Schwarz on
+  // sum |sqrt p - sqrt q| (sqrt p + sqrt q) within each set,
+  //   sum_{v in t} max(0, p - q) <= (((P_t + Q_t)^2 - 4 BC_t^2)^(1/2) + P_t - Q_t) / 2,
+  // BC_t = sum_{v in t} sqrt(q p) from pass 1, summed over t (never above the
+  // Hellinger bound (1 - BC^2)^(1/2)); OPTLog takes Pinsker's (KL(q || p) / 2)^(1/2)
+  // from its entropy and cross entropy.  When alpha times the lower bound already
+  // reaches dr - dl (max p - max q for OPT, Eq. 10; the negative-entropy gap for
+  // OPTLog), delta = 0 for the exact D_TV too; when alpha times the upper bound
+  // stays below it, delta = 1; either way the TV pass is skipped.  The bounds
+  // carry ~1e-6 of f32 rounding over their 256 C terms, BC_t is deflated and KL
+  // inflated well past their f32 errors: only a clear 1e-4 margin settles the row.
   if (sh.band) {
-    const float pt = mine.w * ex2(refk(mine.z, k) - sh.Rp) / sh.Sp;
-    const float qt = mine.y * ex2(refk(mine.x, k) - sh.Rq) / sh.Sq;
-    const float lb = warp_sum(fmaxf(0.0f, pt - qt));
-    // OPT: this thread's sum of sqrt(q p) terms at the row's references
-    const float bcw = warp_sum(bc * ex2(0.5f * ((refk(mine.x, k) - sh.Rq) + (refk(mine.z, k) - sh.Rp))));
+    const float dq = refk(mine.x, k) - sh.Rq, dp = refk(mine.z, k) - sh.Rp;
+    const float fq = ex2(dq) / sh.Sq, fp = ex2(dp) / sh.Sp;
+    const float qe = mine2.x * fq, qo = mine2.y * fq, pe = mine2.z * fp, po = mine2.w * fp;
+    const float lb = warp_sum(fmaxf(0.0f, pe - qe) + fmaxf(0.0f, po - qo));
+    float ubt = 0.0f;
+    if (opt_bc) {
+      const float fb = ex2(0.5f * (dq + dp)) / sqrtf(sh.Sq * sh.Sp) * (1.0f - 2e-4f);
+      const float be = bc.x * fb, bo = bc.y * fb, me = pe + qe, mo = po + qo;
+      ubt = 0.5f * (sqrtf(fmaxf(0.0f, fmaf(me, me, -4.0f * be * be))) + (pe - qe)) +
+            0.5f * (sqrtf(fmaxf(0.0f, fmaf(mo, mo, -4.0f * bo * bo))) + (po - qo));
+    }
+    const float bcw = warp_sum(ubt);
     if (lane == 0) sh.red[warp] = make_float4(lb, bcw, 0.0f, 0.0f);
     __syncthreads();
     if (tid == 0) {
@@ -1768,16 +1781,15 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     cluster_arrive();
     cluster_wait();
     if (tid == 0) {
-      float LB = 0.0f, BCs = 0.0f;  // in rank order
+      float LB = 0.0f, UBs = 0.0f;  // in rank order
       for (int r = 0; r < C; ++r) {
         LB = __fadd_rn(LB, sh.all_lb[r].x);
-        BCs = __fadd_rn(BCs, sh.all_lb[r].y);
+        UBs = __fadd_rn(UBs, sh.all_lb[r].y);
       }
       const float gap = sh.dr - sh.dl;
       float ub = INFINITY;
       if (opt_bc) {
-        const float bcl = fminf(1.0f, BCs / sqrtf(sh.Sq) / sqrtf(sh.Sp)) * (1.0f - 2e-4f);
-        ub = sqrtf(fmaxf(0.0f, 1.0f - bcl * bcl));
+        ub = UBs;
       } else if (kExt && SC_OPT_UB) {
         const float kv = sh.klqp;  // NaN or +inf (masked logits) settle nothing
         if (kv == kv)
