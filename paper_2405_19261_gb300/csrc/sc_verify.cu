@@ -394,10 +394,10 @@ __device__ __forceinline__ float4 merge_partials(const float4 *v, int n, float k
 }
 
 // Pass 1 on one row of one chunk: this thread's kRounds vectors, online
-// (max m, sum s of 2^{y k - refk(m)}), s kept as two partial sums.
+// (max m, sum s of 2^{y k - refk(m)}), s kept as four partial sums, over the logits 0, 1, 2, 3 (mod 4).
 // kFull: the chunk holds kCH logits.
 template <typename E, bool kFull>
-__device__ __forceinline__ void online_row(const E *src, int n, float k, float &m, float2 &s) {
+__device__ __forceinline__ void online_row(const E *src, int n, float k, float &m, float4 &s) {
   float y[kRounds][8];
 #pragma unroll
   for (int r = 0; r < kRounds; ++r) {
@@ -415,16 +415,18 @@ __device__ __forceinline__ void online_row(const E *src, int n, float k, float &
     for (int i = 0; i < 8; i += 2) mn = max3(mn, y[r][i], y[r][i + 1]);
   const float rn = refk(mn, k);
   const float sc = ex2(refk(m, k) - rn);
-  float s0 = s.x * sc, s1 = s.y * sc;
+  float s0 = s.x * sc, s1 = s.y * sc, s2 = s.z * sc, s3 = s.w * sc;
 #pragma unroll
   for (int r = 0; r < kRounds; ++r)
 #pragma unroll
-    for (int i = 0; i < 8; i += 2) {
+    for (int i = 0; i < 8; i += 4) {
       s0 += ex2(fmaf(y[r][i], k, -rn));
       s1 += ex2(fmaf(y[r][i + 1], k, -rn));
+      s2 += ex2(fmaf(y[r][i + 2], k, -rn));
+      s3 += ex2(fmaf(y[r][i + 3], k, -rn));
     }
   m = mn;
-  s = make_float2(s0, s1);
+  s = make_float4(s0, s1, s2, s3);
 }
 
 __device__ __forceinline__ __nv_bfloat162 as_bf162(uint32_t w) {
@@ -433,10 +435,10 @@ __device__ __forceinline__ __nv_bfloat162 as_bf162(uint32_t w) {
 
 // bf16 full chunk: the exact maximum from a packed bf16x2 max tree over the raw
 // words, then one packed f32x2 FMA per two logits for the exponent arguments
-// and packed f32x2 adds for the two partial sums.
+// and packed f32x2 adds for the four partial sums (two packed pairs).
 template <>
 __device__ __forceinline__ void online_row<uint16_t, true>(const uint16_t *src, int n, float k,
-                                                           float &m, float2 &s) {
+                                                           float &m, float4 &s) {
   (void)n;
   uint32_t w[kRounds * 4];
 #pragma unroll
@@ -450,16 +452,20 @@ __device__ __forceinline__ void online_row<uint16_t, true>(const uint16_t *src, 
   const float mn = fmaxf(m, fmaxf(__low2float(mx), __high2float(mx)));
   const float rn = refk(mn, k);
   const float sc = ex2(refk(m, k) - rn);
-  float2 acc = __fmul2_rn(s, make_float2(sc, sc));
+  float2 acc = __fmul2_rn(make_float2(s.x, s.y), make_float2(sc, sc));
+  float2 acb = __fmul2_rn(make_float2(s.z, s.w), make_float2(sc, sc));
   const float2 kk = make_float2(k, k), nr = make_float2(-rn, -rn);
 #pragma unroll
-  for (int i = 0; i < kRounds * 4; ++i) {
+  for (int i = 0; i < kRounds * 4; i += 2) {  // words 2j' hold logits 0, 1 (mod 4), words 2j' + 1 logits 2, 3
     const float2 y = make_float2(__uint_as_float(w[i] << 16), __uint_as_float(w[i] & 0xFFFF0000u));
     const float2 t = __ffma2_rn(y, kk, nr);
     acc = __fadd2_rn(acc, make_float2(ex2(t.x), ex2(t.y)));
+    const float2 y2 = make_float2(__uint_as_float(w[i + 1] << 16), __uint_as_float(w[i + 1] & 0xFFFF0000u));
+    const float2 t2 = __ffma2_rn(y2, kk, nr);
+    acb = __fadd2_rn(acb, make_float2(ex2(t2.x), ex2(t2.y)));
   }
   m = mn;
-  s = acc;
+  s = make_float4(acc.x, acc.y, acb.x, acb.y);
 }
 
 // Pass-1 state of the kFamExt rules.  With a_v = y^q_v k - r_q and
@@ -831,7 +837,7 @@ static_assert(2 * kMaxChunks * kNW <= kEntries, "bonus chunk totals live in seg"
 static_assert(kMaxChunks <= 32, "one lane per chunk of a slice");
 
 template <typename E, bool kFull>
-__device__ __forceinline__ void bonus_row(const E *src, int n, float k, float &m, float2 &s, int c,
+__device__ __forceinline__ void bonus_row(const E *src, int n, float k, float &m, float4 &s, int c,
                                           float *seg, int lane, int warp) {
   float y[kRounds][8];
 #pragma unroll
@@ -863,7 +869,7 @@ __device__ __forceinline__ void bonus_row(const E *src, int n, float k, float &m
   // fold the chunk into the running sum, referenced to refk(max(m, W))
   const float mn = fmaxf(m, W), rn = refk(mn, k);
   const float so = ex2(refk(m, k) - rn);
-  s = make_float2(fmaf(cs, ex2(rw - rn), s.x * so), s.y * so);
+  s = make_float4(fmaf(cs, ex2(rw - rn), s.x * so), s.y * so, s.z * so, s.w * so);
   m = mn;
   const float tot = warp_sum(cs);
   if (lane == 0 && SC_CHECK(c >= 0 && c < kMaxChunks)) {
@@ -876,8 +882,8 @@ __device__ __forceinline__ void bonus_row(const E *src, int n, float k, float &m
 // sqrt(q_v p_v) up to the rows' normalisers: the Bhattacharyya coefficient
 // BC = sum_v sqrt(q_v p_v) bounds D_TV from above, D_TV <= sqrt(1 - BC^2).
 template <typename E, bool kFull>
-__device__ __forceinline__ float2 bc_chunk(const E *srcq, const E *srcp, int n, float hk, float hr) {
-  float acc0 = 0.0f, acc1 = 0.0f;
+__device__ __forceinline__ float4 bc_chunk(const E *srcq, const E *srcp, int n, float hk, float hr) {
+  float acc0 = 0.0f, acc1 = 0.0f, acc2 = 0.0f, acc3 = 0.0f;
 #pragma unroll
   for (int r = 0; r < kRounds; ++r) {
     const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
@@ -885,12 +891,14 @@ __device__ __forceinline__ float2 bc_chunk(const E *srcq, const E *srcp, int n, 
     load8_chunk<E, kFull>(srcq, e, n, yq);
     load8_chunk<E, kFull>(srcp, e, n, yp);
 #pragma unroll
-    for (int i = 0; i < 8; i += 2) {
+    for (int i = 0; i < 8; i += 4) {
       acc0 += ex2(fmaf(yq[i] + yp[i], hk, -hr));
       acc1 += ex2(fmaf(yq[i + 1] + yp[i + 1], hk, -hr));
+      acc2 += ex2(fmaf(yq[i + 2] + yp[i + 2], hk, -hr));
+      acc3 += ex2(fmaf(yq[i + 3] + yp[i + 3], hk, -hr));
     }
   }
-  return make_float2(acc0, acc1);  // (even, odd logits)
+  return make_float4(acc0, acc1, acc2, acc3);  // (logits 0, 1, 2, 3 mod 4)
 }
 
 // OPT pair, full bf16 chunk: online_row of both rows and the chunk's
@@ -899,7 +907,7 @@ __device__ __forceinline__ float2 bc_chunk(const E *srcq, const E *srcp, int n, 
 // relative to the rows' updated references, as in bc_chunk, and the running
 // sums are rescaled as online_row rescales its sums.
 __device__ __forceinline__ void online_pair_bc(const uint16_t *srcq, const uint16_t *srcp, float k,
-                                               float &mq, float2 &sq, float &mp, float2 &sp, float2 &bc) {
+                                               float &mq, float4 &sq, float &mp, float4 &sp, float4 &bc) {
   uint32_t wq[kRounds * 4], wp[kRounds * 4];
 #pragma unroll
   for (int r = 0; r < kRounds; ++r) {
@@ -920,10 +928,13 @@ __device__ __forceinline__ void online_pair_bc(const uint16_t *srcq, const uint1
   const float rq = refk(mqn, k), rp = refk(mpn, k);
   const float dq = refk(mq, k) - rq, dp = refk(mp, k) - rp;
   const float fq = ex2(dq), fp = ex2(dp);
-  float2 aq = __fmul2_rn(sq, make_float2(fq, fq));
-  float2 ap = __fmul2_rn(sp, make_float2(fp, fp));
+  float2 aq = __fmul2_rn(make_float2(sq.x, sq.y), make_float2(fq, fq));
+  float2 ap = __fmul2_rn(make_float2(sp.x, sp.y), make_float2(fp, fp));
+  float2 aq2 = __fmul2_rn(make_float2(sq.z, sq.w), make_float2(fq, fq));
+  float2 ap2 = __fmul2_rn(make_float2(sp.z, sp.w), make_float2(fp, fp));
   const float fb = ex2(0.5f * (dq + dp));
-  float h0 = bc.x * fb, h1 = bc.y * fb;
+  float2 h = __fmul2_rn(make_float2(bc.x, bc.y), make_float2(fb, fb));
+  float2 h2 = __fmul2_rn(make_float2(bc.z, bc.w), make_float2(fb, fb));
   const float2 kk = make_float2(k, k), nrq = make_float2(-rq, -rq), nrp = make_float2(-rp, -rp);
   const float2 half = make_float2(0.5f, 0.5f);
 #pragma unroll
@@ -932,17 +943,24 @@ __device__ __forceinline__ void online_pair_bc(const uint16_t *srcq, const uint1
     const float2 yp = make_float2(__uint_as_float(wp[i] << 16), __uint_as_float(wp[i] & 0xFFFF0000u));
     const float2 a = __ffma2_rn(yq, kk, nrq);
     const float2 b = __ffma2_rn(yp, kk, nrp);
-    aq = __fadd2_rn(aq, make_float2(ex2(a.x), ex2(a.y)));
-    ap = __fadd2_rn(ap, make_float2(ex2(b.x), ex2(b.y)));
+    const float2 ea = make_float2(ex2(a.x), ex2(a.y)), eb = make_float2(ex2(b.x), ex2(b.y));
     const float2 hh = __fmul2_rn(__fadd2_rn(a, b), half);
-    h0 += ex2(hh.x);
-    h1 += ex2(hh.y);
+    const float2 eh = make_float2(ex2(hh.x), ex2(hh.y));
+    if (i & 1) {  // logits 2, 3 (mod 4)
+      aq2 = __fadd2_rn(aq2, ea);
+      ap2 = __fadd2_rn(ap2, eb);
+      h2 = __fadd2_rn(h2, eh);
+    } else {      // logits 0, 1 (mod 4)
+      aq = __fadd2_rn(aq, ea);
+      ap = __fadd2_rn(ap, eb);
+      h = __fadd2_rn(h, eh);
+    }
   }
   mq = mqn;
   mp = mpn;
-  sq = aq;
-  sp = ap;
-  bc = make_float2(h0, h1);
+  sq = make_float4(aq.x, aq.y, aq2.x, aq2.y);
+  sp = make_float4(ap.x, ap.y, ap2.x, ap2.y);
+  bc = make_float4(h.x, h.y, h2.x, h2.y);
 }
 
 // Weights of one chunk in the ring: per round, the warp's total weight (the
@@ -1421,15 +1439,15 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   // ---- pass 1: online max and sum of exponentials
   const float k = P.k;
   float mq = -FLT_MAX, mp = -FLT_MAX;
-  float2 s2q = make_float2(0.0f, 0.0f), s2p = make_float2(0.0f, 0.0f);
+  float4 s2q = make_float4(0.0f, 0.0f, 0.0f, 0.0f), s2p = s2q;
   ExtState ex = ext_empty();  // (kFamExt) moments and argmaxes
   Top2 top = {-FLT_MAX, -FLT_MAX, -FLT_MAX};  // (kFamToken) the eta screen
   const bool scr_q = P.rule == SC_RULE_TOKEN_V1;
   // OPT: the pair's running sum of sqrt(q p) terms, relative to (r_q + r_p) / 2
   const bool opt_bc = SC_OPT_UB && P.opt_ub && !kTok && !kExt && verify && pair && P.rule == SC_RULE_OPT;
-  // the pair's running sums of sqrt(q p) terms over this thread's even and odd logits,
-  // relative to (r_q + r_p) / 2
-  float2 bc = make_float2(0.0f, 0.0f);
+  // the pair's running sums of sqrt(q p) terms over this thread's logits 0, 1, 2, 3
+  // (mod 4), relative to (r_q + r_p) / 2
+  float4 bc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
   // the bonus row also leaves its per-(chunk, warp) totals for the sampler
   const bool bonus_tot = verify && !pair && !P.greedy;
   const int lx = x - v0;  // draft token's offset in this slice (thread 0 only)
@@ -1480,9 +1498,9 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
         if (opt_bc) {
           const float rq = refk(mq, k), rp = refk(mp, k);
           const float sc = ex2(0.5f * ((refk(mq0, k) - rq) + (refk(mp0, k) - rp)));
-          const float2 add = n == kCH ? bc_chunk<E, true>(R.q(s), R.p(s), n, 0.5f * k, 0.5f * (rq + rp))
+          const float4 add = n == kCH ? bc_chunk<E, true>(R.q(s), R.p(s), n, 0.5f * k, 0.5f * (rq + rp))
                                       : bc_chunk<E, false>(R.q(s), R.p(s), n, 0.5f * k, 0.5f * (rq + rp));
-          bc = make_float2(fmaf(bc.x, sc, add.x), fmaf(bc.y, sc, add.y));
+          bc = make_float4(fmaf(bc.x, sc, add.x), fmaf(bc.y, sc, add.y), fmaf(bc.z, sc, add.z), fmaf(bc.w, sc, add.w));
         }
       }
     }
@@ -1494,16 +1512,16 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   if constexpr (kExt) {
     if (bonus_tot) {
       ex.mp = mp;
-      ex.sp = s2p.x + s2p.y;
+      ex.sp = (s2p.x + s2p.y) + (s2p.z + s2p.w);
     }
     mq = ex.mq;
     mp = ex.mp;
-    s2q = make_float2(ex.sq, 0.0f);
-    s2p = make_float2(ex.sp, 0.0f);
+    s2q = make_float4(ex.sq, 0.0f, 0.0f, 0.0f);
+    s2p = make_float4(ex.sp, 0.0f, 0.0f, 0.0f);
   }
-  float s_q = s2q.x + s2q.y, s_p = s2p.x + s2p.y;
+  float s_q = (s2q.x + s2q.y) + (s2q.z + s2q.w), s_p = (s2p.x + s2p.y) + (s2p.z + s2p.w);
   const float4 mine = make_float4(mq, s_q, mp, s_p);  // this thread's partial, kept for the D_TV bounds
-  const float4 mine2 = make_float4(s2q.x, s2q.y, s2p.x, s2p.y);  // ... split over its even and odd logits
+  const float4 mq4 = s2q, mp4 = s2p;  // ... split over its logits 0, 1, 2, 3 (mod 4)
   tmo = __syncthreads_or(tmo);
   if constexpr (kExt) {
     ext_warp_merge(ex, k);
@@ -1741,9 +1759,9 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
     __syncthreads();
   }
 
-  // ---- OPT band: bounds on D_TV from the pass-1 partials.  Each thread's even
-  // and odd logits form two sets t (the two lanes of its packed sums), with
-  // masses P_t, Q_t; the sets partition the vocabulary, so
+  // ---- OPT band: bounds on D_TV from the pass-1 partials.  Each thread's logits
+  // 0, 1, 2 and 3 (mod 4) form four sets t (the lanes of its two packed sums),
+  // with masses P_t, Q_t; the sets partition the vocabulary, so
   // sum_t max(0, P_t - Q_t) <= D_TV.  From above, OPT takes Cauchy-Schwarz on
   // sum |sqrt p - sqrt q| (sqrt p + sqrt q) within each set,
   //   sum_{v in t} max(0, p - q) <= (((P_t + Q_t)^2 - 4 BC_t^2)^(1/2) + P_t - Q_t) / 2,
@@ -1753,20 +1771,23 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   // reaches dr - dl (max p - max q for OPT, Eq. 10; the negative-entropy gap for
   // OPTLog), delta = 0 for the exact D_TV too; when alpha times the upper bound
   // stays below it, delta = 1; either way the TV pass is skipped.  The bounds
-  // carry ~1e-6 of f32 rounding over their 256 C terms, BC_t is deflated and KL
+  // carry ~1e-6 of f32 rounding over their 512 C terms, BC_t is deflated and KL
   // inflated well past their f32 errors: only a clear 1e-4 margin settles the row.
   if (sh.band) {
     const float dq = refk(mine.x, k) - sh.Rq, dp = refk(mine.z, k) - sh.Rp;
     const float fq = ex2(dq) / sh.Sq, fp = ex2(dp) / sh.Sp;
-    const float qe = mine2.x * fq, qo = mine2.y * fq, pe = mine2.z * fp, po = mine2.w * fp;
-    const float lb = warp_sum(fmaxf(0.0f, pe - qe) + fmaxf(0.0f, po - qo));
-    float ubt = 0.0f;
-    if (opt_bc) {
-      const float fb = ex2(0.5f * (dq + dp)) / sqrtf(sh.Sq * sh.Sp) * (1.0f - 2e-4f);
-      const float be = bc.x * fb, bo = bc.y * fb, me = pe + qe, mo = po + qo;
-      ubt = 0.5f * (sqrtf(fmaxf(0.0f, fmaf(me, me, -4.0f * be * be))) + (pe - qe)) +
-            0.5f * (sqrtf(fmaxf(0.0f, fmaf(mo, mo, -4.0f * bo * bo))) + (po - qo));
+    const float qs[4] = {mq4.x * fq, mq4.y * fq, mq4.z * fq, mq4.w * fq};
+    const float ps[4] = {mp4.x * fp, mp4.y * fp, mp4.z * fp, mp4.w * fp};
+    const float bs[4] = {bc.x, bc.y, bc.z, bc.w};
+    const float fb = opt_bc ? ex2(0.5f * (dq + dp)) / sqrtf(sh.Sq * sh.Sp) * (1.0f - 2e-4f) : 0.0f;
+    float lbt = 0.0f, ubt = 0.0f;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      lbt += fmaxf(0.0f, ps[i] - qs[i]);
+      const float m = ps[i] + qs[i], bt = bs[i] * fb;
+      ubt += 0.5f * (sqrtf(fmaxf(0.0f, fmaf(m, m, -4.0f * bt * bt))) + (ps[i] - qs[i]));
     }
+    const float lb = warp_sum(lbt);
     const float bcw = warp_sum(ubt);
     if (lane == 0) sh.red[warp] = make_float4(lb, bcw, 0.0f, 0.0f);
     __syncthreads();
