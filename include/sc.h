@@ -102,6 +102,8 @@ typedef enum {
  *                 position of its slice reported without a rejection) stores its own
  *                 residual prefixes (default 1), or the owners always sample
  *   SC_POS_MAJOR=0|1 units in position-major order (default 1) or sequence-major
+ *   SC_L2_HINT=n  copy all but the newest n chunks of a pair's slice, and every bonus
+ *                 row, with the L2 evict-first policy (default 4; 0: no cache hints)
  *   SC_OPT_UB=0|1 whether OPT pairs accumulate the Bhattacharyya coefficient in
  *                 pass 1 for an upper bound on D_TV that settles band rows without
  *                 the TV pass (default: when C <= 4) */
