@@ -2,42 +2,44 @@
 //
 // One call of sc_verify runs GenSpecSample's verification phase (Algorithm 4)
 // with the SpecCascade target pi = (1 - delta) q + delta p (Algorithm 5, Eq. 6)
-// for B sequences of gamma drafted positions over a V-token vocabulary, in ONE
-// kernel launch:
+// -- or another target: the token-specific rules of Section 4.4, lossy
+// speculative decoding and BiLD* (Table 3), the log-loss rules, greedy
+// decoding -- for B sequences of gamma drafted positions over a V-token
+// vocabulary, in ONE kernel launch:
 //
 //   unit    one (b, j < gamma) row pair (draft row q_j, target row p_j), or the
-//           bonus target row (b, gamma);
+//           bonus target row (b, gamma); units in position-major order (every
+//           sequence's position j before any position j + 1);
 //   grid    one thread-block cluster of C CTAs per unit; CTA r of the cluster
 //           owns the vocabulary slice [r L, (r+1) L) of both rows;
 //   pass 1  the slice streams from HBM through a two-stage shared-memory ring
 //           filled by TMA bulk copies (cp.async.bulk + mbarrier), 4096 logits
-//           per row per stage; each thread keeps an online (max, sum of exp);
-//           thread 0 merges the warp partials and pushes the CTA partial into
-//           every CTA of the cluster (st.shared::cluster) before one cluster
-//           barrier, after which every read is local: M and S of both rows,
-//           max q = 1/S_q and max p = 1/S_p, the deferral decision of Table 1
-//           and the acceptance test of the draft token;
-//   token   with a token-specific rule (Section 4.4) every pair makes a second
-//           pass for eta = sum_v r(v) q(v), r(v) the per-token deferral; the
-//           draft is accepted when r(x) = 0, else with ratio eta p(x)/q(x), and
-//           the residual weights are max(0, eta p - r q);
-//   TV      only inside the OPT band where the TV term of Eq. 10 decides: a
-//           lower bound on D_TV from the threads' partial masses settles many
-//           such rows at delta = 0; the rest, and sc_row_stats, sum the
+//           per row per stage, the older chunks with the L2 evict-first
+//           policy; each thread keeps an online (max, sum of exp) in four
+//           lanes; thread 0 merges the warp partials and pushes the CTA partial
+//           into every CTA of the cluster (st.shared::cluster) before one
+//           cluster barrier, after which every read is local: M and S of both
+//           rows, max q and max p, the deferral decision and the acceptance
+//           test of the draft token;
+//   token   a token-specific rule evaluates r(v) per token; eta = sum r(v) q(v)
+//           comes from a pass-1 screen of each thread's two largest tested
+//           logits, or, where the screen cannot settle it, from a second pass;
+//   TV      only inside the OPT (or OPTLog) band, where the TV term of Eq. 10
+//           decides: lower and upper bounds on D_TV from the pass-1 partials
+//           settle most such rows; the rest, and sc_row_stats, sum the
 //           residual weights max(0, p - q) over the slice again (newest chunk
 //           first) and over the cluster: D_TV(p, q) S_q (Lemma 3);
 //   finish  every CTA writes its unit's decision record and reports its
 //           arrival (and rejection) on the ticket of its slice rank r in the
-//           sequence.  The CTA whose report settles j* = min{j : a_j = 0} --
-//           the first rejection with every earlier position in, or all
-//           gamma + 1 positions in without one -- streams its slice of row j*
-//           (the rejected pair, whose residual max(0, p - q) is sampled, or the
-//           bonus row p_gamma) and stores the slice's chunk prefixes.  The last
-//           of those C slice passes (and of rank 0's reports) does the
-//           inverse-CDF draw: it finds the slice and chunk holding u R, copies
-//           that chunk in and one warp scans the segment holding it.  Only the
-//           sampled row of each sequence gets a second pass, and no CTA ever
-//           waits on another cluster.
+//           sequence.  A rejected pair that is certainly row j* (every earlier
+//           position of its rank reported without a rejection) stores its own
+//           residual's chunk prefixes at once; otherwise the CTA whose report
+//           settles j* = min{j : a_j = 0} streams its slice of row j*.  The
+//           bonus row's prefixes come from its pass 1.  The last of a
+//           sequence's C owners does the inverse-CDF draw: it finds the slice
+//           and chunk holding u R, copies that chunk in and one warp scans the
+//           segment holding it.  Only row j* of each sequence is sampled, and
+//           no CTA ever waits on another cluster.
 //
 // Exponentials are ex2.approx of fma(y, log2(e)/T, -R), R = fl(M log2(e)/T):
 // one rounding per logit.  Every mbarrier wait is bounded and reports

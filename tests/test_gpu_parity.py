@@ -252,6 +252,24 @@ def test_self_sampled_residuals_match_the_owners_pass(sc, monkeypatch, rule, alp
     assert np.any(ref.num_accepted < w.gamma) and np.any(ref.num_accepted == w.gamma)
 
 
+@pytest.mark.parametrize("env", [{"SC_L2_HINT": "0"}, {"SC_L2_HINT": "1"}, {"SC_POS_MAJOR": "0"},
+                                 {"SC_OPT_UB": "0"}, {"SC_OPT_UB": "1"}, {"SC_SPEC_RES": "0"}])
+@pytest.mark.parametrize("rule,alpha", [("opt", 0.2), ("chow", 0.5), ("token_v3", 0.3)])
+def test_schedule_switches_leave_the_outputs_unchanged(sc, monkeypatch, env, rule, alpha):
+    # cache hints, the unit order, the upper bound on D_TV and who samples the
+    # residual change how the work is scheduled, never what is computed: the
+    # outputs equal the default run's bit for bit (and the oracle's)
+    w = synthetic(40, 6, 256000, dtype="bf16", kind="zipf", sigma=0.7, rule=rule, alpha=alpha, seed=91,
+                  force_reject_frac=0.3)
+    base = run_gpu(sc, w)
+    for k, v in env.items():
+        monkeypatch.setenv(k, v)
+    alt = run_gpu(sc, w)
+    np.testing.assert_array_equal(alt[0], base[0])
+    np.testing.assert_array_equal(alt[1], base[1])
+    assert_parity(w, alt, oracle.verify_workload(w))
+
+
 @pytest.mark.parametrize("rule,alpha", [("token_v3", 0.0), ("token_v3", 0.3), ("token_v2", 0.05), ("token_v1", 0.05)])
 def test_token_eta_screen_and_its_fallback(sc, rule, alpha):
     # eta comes from the pass-1 screen when each thread holds at most one
