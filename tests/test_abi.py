@@ -8,26 +8,29 @@ import pytest
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 HEADER = os.path.join(ROOT, "include", "sc.h")
+SHARD_HEADER = os.path.join(ROOT, "include", "sc_shard.h")
 
 
 @pytest.fixture(scope="module")
 def so():
     import __graft_entry__ as g
-    if not os.path.exists(g.LIB) or os.path.getmtime(g.LIB) < os.path.getmtime(g.CSRC):
+    if not os.path.exists(g.LIB) or os.path.getmtime(g.LIB) < max(os.path.getmtime(s) for s in g.SOURCES):
         g.build_library()
     return ctypes.CDLL(g.LIB)
 
 
-def declared_functions():
-    text = open(HEADER).read()
-    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    names = re.findall(r"\b(sc_[a-z_]+)\s*\(", text)
+def declared_functions(headers=(HEADER, SHARD_HEADER)):
+    names = []
+    for h in headers:
+        text = re.sub(r"/\*.*?\*/", "", open(h).read(), flags=re.S)
+        names += re.findall(r"\b(sc_[a-z_0-9]+)\s*\(", text)
     return sorted(set(names))
 
 
 def test_header_declares_the_boundary():
     names = declared_functions()
-    for n in ("sc_verify", "sc_row_stats", "sc_workspace_bytes", "sc_status_string"):
+    for n in ("sc_verify", "sc_row_stats", "sc_workspace_bytes", "sc_status_string", "sc_shard_pass1",
+              "sc_shard_decide", "sc_shard_accept", "sc_shard_draw", "sc_shard_finish"):
         assert n in names
 
 
@@ -106,3 +109,67 @@ def test_binding_constants_mirror_the_header():
         assert idx == defines["SC_ROW_" + name.upper()], name
     assert (binding.DEV_BAD_TOKEN, binding.DEV_BAD_LOGIT, binding.DEV_BAD_UNIFORM, binding.DEV_TIMEOUT) == (
         defines["SC_DEV_BAD_TOKEN"], defines["SC_DEV_BAD_LOGIT"], defines["SC_DEV_BAD_UNIFORM"], defines["SC_DEV_TIMEOUT"])
+
+
+def test_shard_host_only_entry_points(so):
+    S, I = ctypes.c_size_t, ctypes.c_int
+    so.sc_shard_message_bytes.restype = S
+    so.sc_shard_message_bytes.argtypes = [I, I, I]
+    so.sc_shard_workspace_bytes.restype = S
+    so.sc_shard_workspace_bytes.argtypes = [I, I, I, I]
+    B, g = 512, 8
+    # message 1: (m_q, s_q, m_p, s_p) per unit and the draft token's two logits
+    # per pair; 2: S_q D_TV per pair; 3: a total weight per sequence; 4: a token
+    assert so.sc_shard_message_bytes(B, g, 1) == B * (g + 1) * 16 + B * g * 8
+    assert so.sc_shard_message_bytes(B, g, 2) == B * g * 8
+    assert so.sc_shard_message_bytes(B, g, 3) == B * 8
+    assert so.sc_shard_message_bytes(B, g, 4) == B * 4
+    assert so.sc_shard_message_bytes(B, g, 5) == 0 and so.sc_shard_message_bytes(0, g, 1) == 0
+    # independent of V: the messages are tiny against the 4.46 GB of logits
+    assert sum(so.sc_shard_message_bytes(B, g, k) for k in (1, 2, 3, 4)) < 200_000
+    small, big = so.sc_shard_workspace_bytes(B, g, 8192, 1), so.sc_shard_workspace_bytes(B, g, 128000, 1)
+    assert 0 < small < big
+    assert so.sc_shard_workspace_bytes(B, g, 0, 1) == 0
+
+
+def test_shard_calls_reject_bad_arguments_without_a_gpu(so):
+    P, I, F, S, L64 = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_size_t, ctypes.c_int64
+    IA = ctypes.POINTER(ctypes.c_int)
+    so.sc_shard_pass1.argtypes = [P, P, I, L64, P, I, I, I, I, IA, F, P, S, P, P]
+    good = (ctypes.c_int * 3)(0, 100, 200)
+    unordered = (ctypes.c_int * 3)(0, 150, 120)
+    not_zero = (ctypes.c_int * 3)(5, 100, 200)
+    for bounds, W, rank, T in ((good, 2, 0, 1.0), (good, 2, 2, 1.0), (unordered, 2, 0, 1.0),
+                               (not_zero, 2, 0, 1.0), (good, 2, 0, 0.0), (good, 17, 0, 1.0), (None, 2, 0, 1.0)):
+        rc = so.sc_shard_pass1(None, None, 1, 100, None, 4, 3, W, rank, bounds, T, None, 0, None, None)
+        assert rc == -1, (W, rank, T)
+    so.sc_shard_finish.argtypes = [P, I, I, I, P, S, P, P, P]
+    assert so.sc_shard_finish(None, 4, 3, 2, None, 0, None, None, None) == -1
+
+
+def test_shard_header_is_plain_c(tmp_path):
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    cuda_inc = "/usr/local/cuda/include" if os.path.isdir("/usr/local/cuda/include") else None
+    if not gcc or not cuda_inc:
+        pytest.skip("gcc or the CUDA headers are missing")
+    src = tmp_path / "use_shard.c"
+    src.write_text("""
+#include "sc_shard.h"
+int use_shard(const void *q, const void *p, const int32_t *x, const float *u, void *ws, void *s1,
+              void *g1, void *s2, void *g2, void *s3, void *g3, void *s4, void *g4, int32_t *na,
+              int32_t *nt, int32_t *st, cudaStream_t s) {
+  const int bounds[3] = {0, 128000, 256000};
+  size_t n = sc_shard_workspace_bytes(4, 3, 128000, SC_BF16) + sc_shard_message_bytes(4, 3, 1);
+  int rc = sc_shard_pass1(q, p, SC_BF16, 128000, x, 4, 3, 2, 0, bounds, 1.0f, ws, n, s1, s);
+  rc |= sc_shard_decide(q, p, SC_BF16, 128000, g1, x, u, 4, 3, 2, 0, bounds, SC_RULE_OPT, 0.2f, 1.0f, ws, n, s2, st, s);
+  rc |= sc_shard_accept(q, p, SC_BF16, 128000, g2, u, 4, 3, 2, 0, bounds, SC_RULE_OPT, 0.2f, 1.0f, ws, n, s3, s);
+  rc |= sc_shard_draw(q, p, SC_BF16, 128000, g3, u, 4, 3, 2, 0, bounds, 1.0f, ws, n, s4, s);
+  rc |= sc_shard_finish(g4, 4, 3, 2, ws, n, na, nt, s);
+  return rc + SC_SHARD_MAX;
+}
+""")
+    r = subprocess.run([gcc, "-std=c11", "-Wall", "-Wextra", "-Werror", "-fsyntax-only", "-I",
+                        os.path.join(ROOT, "include"), "-I", cuda_inc, str(src)], capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
