@@ -14,16 +14,19 @@
  * message in rank order between the calls):
  *
  *   sc_shard_pass1   pass 1 over the local logits: per row the rank's
- *                    (max logit, sum of exponentials), and the logits of each
- *                    draft token the rank holds                -> message 1
+ *                    (max logit, sum of exponentials), the logits of each
+ *                    draft token the rank holds, and with SC_RULE_OPT the
+ *                    pair's Bhattacharyya sum (Hellinger's upper bound on
+ *                    D_TV)                                     -> message 1
  *   sc_shard_decide  merges the W messages 1 (the same arithmetic in the same
  *                    order on every rank, so every rank takes the same
  *                    decisions): M, S, max q and max p of every row, delta
  *                    (Table 1) and the acceptance test (Algorithm 4).  With
  *                    SC_RULE_OPT a pair inside the band
- *                    max p - alpha <= max q < max p needs D_TV (Eq. 10): the
- *                    rank sums its part of the residual weights of those
- *                    pairs (Lemma 3)                           -> message 2
+ *                    max p - alpha <= max q < max p needs D_TV (Eq. 10):
+ *                    where neither the upper bound nor this rank's part of a
+ *                    lower bound settles delta, the rank sums its part of the
+ *                    residual weights (Lemma 3)                -> message 2
  *   sc_shard_accept  merges the W messages 2, finishes delta and acceptance
  *                    of the band pairs, settles j* = min{j : a_j = 0}, and
  *                    sums the rank's part of the weights of the row it draws
@@ -86,7 +89,7 @@ size_t sc_shard_workspace_bytes(int B, int gamma, int width, sc_dtype dtype);
 
 int sc_shard_pass1(const void *draft_shard, const void *target_shard, sc_dtype dtype, int64_t ld,
                    const int32_t *draft_tokens, int B, int gamma, int W, int rank,
-                   const int *shard_begin, float temperature, void *workspace,
+                   const int *shard_begin, float temperature, sc_rule rule, void *workspace,
                    size_t workspace_bytes, void *send1, cudaStream_t stream);
 
 int sc_shard_decide(const void *draft_shard, const void *target_shard, sc_dtype dtype, int64_t ld,

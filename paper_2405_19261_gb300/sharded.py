@@ -43,7 +43,7 @@ def lib():
         L.sc_shard_message_bytes.restype = S
         L.sc_shard_workspace_bytes.argtypes = [I, I, I, I]
         L.sc_shard_workspace_bytes.restype = S
-        L.sc_shard_pass1.argtypes = [P, P, I, L64, P, I, I, I, I, IA, F, P, S, P, P]
+        L.sc_shard_pass1.argtypes = [P, P, I, L64, P, I, I, I, I, IA, F, I, P, S, P, P]
         L.sc_shard_decide.argtypes = [P, P, I, L64, P, P, P, I, I, I, I, IA, I, F, F, P, S, P, P, P]
         L.sc_shard_accept.argtypes = [P, P, I, L64, P, P, I, I, I, I, IA, I, F, F, P, S, P, P]
         L.sc_shard_draw.argtypes = [P, P, I, L64, P, P, I, I, I, I, IA, F, P, S, P, P]
@@ -118,13 +118,13 @@ class ShardRank:
         if g.numel() * g.element_size() < self.W * self.send[k].numel():
             raise ValueError(f"gathered message {k} must hold the {self.W} ranks' messages")
 
-    def pass1(self, draft, target, tokens, temperature, stream=None):
+    def pass1(self, draft, target, tokens, temperature, rule, stream=None):
         d, t, dt, ld = self._shard(draft, target)
         binding._cuda(tokens, "draft_tokens", torch.int32)
         if tuple(tokens.shape) != (self.B, self.gamma):
             raise ValueError(f"draft_tokens must be [{self.B}, {self.gamma}]")
         rc = lib().sc_shard_pass1(binding._ptr(d), binding._ptr(t), dt, ld, binding._ptr(tokens), self.B,
-                                  self.gamma, self.W, self.rank, self._cb, float(temperature),
+                                  self.gamma, self.W, self.rank, self._cb, float(temperature), _rule_code(rule),
                                   binding._ptr(self.workspace), self.workspace.numel(),
                                   binding._ptr(self.send[1]), binding._stream(stream))
         binding._check(rc, "sc_shard_pass1")
@@ -215,7 +215,7 @@ def sharded_step(ranks: List[ShardRank], shards: List[Tuple[torch.Tensor, torch.
     width_i]) of ranks[i]; tokens [B, gamma] int32 and uniforms [B, gamma+1]
     float32 are the same on every rank."""
     code = _rule_code(rule)
-    g1 = exchange([r.pass1(d, t, tokens, temperature, stream) for r, (d, t) in zip(ranks, shards)])
+    g1 = exchange([r.pass1(d, t, tokens, temperature, code, stream) for r, (d, t) in zip(ranks, shards)])
     s2 = [r.decide(d, t, g1, tokens, uniforms, code, alpha, temperature, stream) for r, (d, t) in zip(ranks, shards)]
     g2 = exchange(s2) if code == binding.RULES["opt"] else None
     g3 = exchange([r.accept(d, t, g2, uniforms, code, alpha, temperature, stream)
@@ -237,3 +237,28 @@ def emulated_step(draft: torch.Tensor, target: torch.Tensor, tokens: torch.Tenso
     shards = [(draft[:, :, bounds[r]:bounds[r + 1]], target[:, :, bounds[r]:bounds[r + 1]]) for r in range(W)]
     out = sharded_step(ranks, shards, tokens, uniforms, rule, alpha, temperature, LocalExchange(), stream)
     return out[0][0], out[0][1], ranks
+
+
+class EmulatedGraph:
+    """The W-rank step on one device (emulated_step) captured into a CUDA
+    graph: ``replay()`` runs every rank's kernels and the on-device exchanges
+    of one step with no host work between them.  The inputs are read from the
+    tensors given here; refill them in place between replays."""
+
+    def __init__(self, draft, target, tokens, uniforms, rule, alpha, temperature, bounds, warmup: int = 2):
+        self.ranks = None
+        side = torch.cuda.Stream(device=draft.device)
+        side.wait_stream(torch.cuda.current_stream(draft.device))
+        with torch.cuda.stream(side):
+            for _ in range(warmup):
+                _, _, self.ranks = emulated_step(draft, target, tokens, uniforms, rule, alpha, temperature, bounds,
+                                                 ranks=self.ranks)
+        torch.cuda.current_stream(draft.device).wait_stream(side)
+        self.graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(self.graph):
+            self.num_accepted, self.next_token, _ = emulated_step(draft, target, tokens, uniforms, rule, alpha,
+                                                                  temperature, bounds, ranks=self.ranks)
+
+    def replay(self):
+        self.graph.replay()
+        return self.num_accepted, self.next_token

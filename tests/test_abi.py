@@ -120,7 +120,7 @@ def test_shard_host_only_entry_points(so):
     B, g = 512, 8
     # message 1: (m_q, s_q, m_p, s_p) per unit and the draft token's two logits
     # per pair; 2: S_q D_TV per pair; 3: a total weight per sequence; 4: a token
-    assert so.sc_shard_message_bytes(B, g, 1) == B * (g + 1) * 16 + B * g * 8
+    assert so.sc_shard_message_bytes(B, g, 1) == B * (g + 1) * 16 + B * g * 8 + B * g * 4
     assert so.sc_shard_message_bytes(B, g, 2) == B * g * 8
     assert so.sc_shard_message_bytes(B, g, 3) == B * 8
     assert so.sc_shard_message_bytes(B, g, 4) == B * 4
@@ -135,13 +135,13 @@ def test_shard_host_only_entry_points(so):
 def test_shard_calls_reject_bad_arguments_without_a_gpu(so):
     P, I, F, S, L64 = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_size_t, ctypes.c_int64
     IA = ctypes.POINTER(ctypes.c_int)
-    so.sc_shard_pass1.argtypes = [P, P, I, L64, P, I, I, I, I, IA, F, P, S, P, P]
+    so.sc_shard_pass1.argtypes = [P, P, I, L64, P, I, I, I, I, IA, F, I, P, S, P, P]
     good = (ctypes.c_int * 3)(0, 100, 200)
     unordered = (ctypes.c_int * 3)(0, 150, 120)
     not_zero = (ctypes.c_int * 3)(5, 100, 200)
     for bounds, W, rank, T in ((good, 2, 0, 1.0), (good, 2, 2, 1.0), (unordered, 2, 0, 1.0),
                                (not_zero, 2, 0, 1.0), (good, 2, 0, 0.0), (good, 17, 0, 1.0), (None, 2, 0, 1.0)):
-        rc = so.sc_shard_pass1(None, None, 1, 100, None, 4, 3, W, rank, bounds, T, None, 0, None, None)
+        rc = so.sc_shard_pass1(None, None, 1, 100, None, 4, 3, W, rank, bounds, T, 2, None, 0, None, None)
         assert rc == -1, (W, rank, T)
     so.sc_shard_finish.argtypes = [P, I, I, I, P, S, P, P, P]
     assert so.sc_shard_finish(None, 4, 3, 2, None, 0, None, None, None) == -1
@@ -162,7 +162,7 @@ int use_shard(const void *q, const void *p, const int32_t *x, const float *u, vo
               int32_t *nt, int32_t *st, cudaStream_t s) {
   const int bounds[3] = {0, 128000, 256000};
   size_t n = sc_shard_workspace_bytes(4, 3, 128000, SC_BF16) + sc_shard_message_bytes(4, 3, 1);
-  int rc = sc_shard_pass1(q, p, SC_BF16, 128000, x, 4, 3, 2, 0, bounds, 1.0f, ws, n, s1, s);
+  int rc = sc_shard_pass1(q, p, SC_BF16, 128000, x, 4, 3, 2, 0, bounds, 1.0f, SC_RULE_OPT, ws, n, s1, s);
   rc |= sc_shard_decide(q, p, SC_BF16, 128000, g1, x, u, 4, 3, 2, 0, bounds, SC_RULE_OPT, 0.2f, 1.0f, ws, n, s2, st, s);
   rc |= sc_shard_accept(q, p, SC_BF16, 128000, g2, u, 4, 3, 2, 0, bounds, SC_RULE_OPT, 0.2f, 1.0f, ws, n, s3, s);
   rc |= sc_shard_draw(q, p, SC_BF16, 128000, g3, u, 4, 3, 2, 0, bounds, 1.0f, ws, n, s4, s);

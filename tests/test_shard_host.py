@@ -35,7 +35,7 @@ class PhaseProbe:
         want = torch.cat([torch.full((SIZES[k],), 10 * k + r, dtype=torch.uint8) for r in range(self.W)])
         assert torch.equal(g, want), (k, g)
 
-    def pass1(self, d, t, tokens, T, stream=None):
+    def pass1(self, d, t, tokens, T, rule, stream=None):
         self.log.append("pass1")
         return self._msg(1)
 
