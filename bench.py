@@ -23,6 +23,8 @@ Prints ONE JSON line (rank 0).  Keys beyond the base contract:
 method here) on the host cores, on bounded samples of the same workload.
 --gpus N under torchrun: every rank verifies its own full batch (weak scaling,
 no collective on the data path); value = all ranks' positions / max time.
+--vocab-shards W times the vocabulary-sharded step instead (one batch whose
+vocabulary is split over W shards; strong scaling when W = world size).
 """
 
 from __future__ import annotations
@@ -75,6 +77,10 @@ def parse():
                          "(default for config 4: the other two Table 1 rules of the sweep; 'none' for none)")
     ap.add_argument("--sweep", action="store_true",
                     help="config 4: also time every sweep point (B x gamma) under Chow, Diff and OPT")
+    ap.add_argument("--vocab-shards", type=int, default=0, metavar="W",
+                    help="time the vocabulary-sharded step (include/sc_shard.h) with W shards instead: W ranks "
+                         "emulated on one GPU (on-device exchanges, one CUDA graph per step), or under torchrun "
+                         "one shard per GPU (W = world size, NCCL all-gathers)")
     return ap.parse_args()
 
 
@@ -586,6 +592,102 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+def run_sharded(args):
+    """The vocabulary-sharded step on the default workload: W ranks emulated on
+    one GPU (world size 1: every rank's kernels and the on-device exchanges,
+    captured as one CUDA graph per step) or one shard per GPU under torchrun
+    (NCCL all-gathers between the phases)."""
+    import torch
+    import torch.distributed as dist
+
+    rank, world, local = dist_env()
+    W = args.vocab_shards
+    if world > 1:
+        if W != world:
+            raise SystemExit("--vocab-shards must equal the world size under torchrun")
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local if world > 1 else 0)
+    from paper_2405_19261_gb300 import binding, sharded
+
+    w, desc = workload_from(args, 0)  # one batch, split over the shards
+    bounds = sharded.shard_bounds(w.V, W)
+    d, t, x, u = binding.to_device(w, dev)
+    stream = torch.cuda.current_stream(dev)
+    if world == 1:
+        graph = sharded.EmulatedGraph(d, t, x, u, w.rule, w.alpha, w.temperature, bounds)
+        ranks = graph.ranks
+
+        def step():
+            graph.replay()
+        na = graph.num_accepted
+        mode = f"{W} ranks emulated on one GPU: every rank's kernels and on-device exchanges, one CUDA graph per step"
+    else:
+        lo, hi = bounds[rank], bounds[rank + 1]
+        ds, ts = d[:, :, lo:hi].contiguous(), t[:, :, lo:hi].contiguous()
+        del d, t
+        ranks = [sharded.ShardRank(w.B, w.gamma, bounds, rank, ds.dtype, dev)]
+        ex = sharded.DistExchange()
+
+        def step():
+            sharded.sharded_step(ranks, [(ds, ts)], x, u, w.rule, w.alpha, w.temperature, ex)
+        na = ranks[0].num_accepted
+        mode = f"one shard per GPU, {W} GPUs, NCCL all-gathers between the phases"
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        dist.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        dist.barrier()
+    ms_step = max_over_ranks(e0.elapsed_time(e1) / args.steps, world, dev)
+    mean_accepted = float(na.float().mean().item())
+    # roofline of the dominant kernel, the pass over the logits (rank 0's shard):
+    # its algorithmic bytes are the shard's logits read once
+    r0 = ranks[0]
+    dd = d[:, :, bounds[0]:bounds[1]] if world == 1 else ds
+    tt = t[:, :, bounds[0]:bounds[1]] if world == 1 else ts
+    for _ in range(3):
+        r0.pass1(dd, tt, x, w.temperature, w.rule)
+    p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    p0.record(stream)
+    for _ in range(args.steps):
+        r0.pass1(dd, tt, x, w.temperature, w.rule)
+    p1.record(stream)
+    torch.cuda.synchronize(dev)
+    ms_pass1 = p0.elapsed_time(p1) / args.steps
+    peak, peak_kind = measured_peaks()
+    alg1 = w.rows * (bounds[1] - bounds[0]) * w.elt_bytes
+    achieved = alg1 / (ms_pass1 / 1e3) / 1e9
+    alg = w.algorithmic_bytes()
+    launches = (10 if w.rule == "opt" else 8) * (W if world == 1 else 1)
+    if rank == 0:
+        line = {"metric": METRIC, "value": w.B * w.gamma / (ms_step / 1e3), "unit": UNIT, "n_gpus": world,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+                "scaling": "strong", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+                "config": {"workload": desc, "B": w.B, "gamma": w.gamma, "V": w.V, "logits": w.dtype,
+                           "rule": w.rule, "alpha": w.alpha, "temperature": w.temperature,
+                           "vocab_shards": W, "shard_bounds": bounds, "parallelism": mode,
+                           "mean_accepted": mean_accepted,
+                           "step_gbs_algorithmic": alg / (ms_step / 1e3) / 1e9,
+                           "step_frac_algorithmic": alg / (ms_step / 1e3) / 1e9 / peak,
+                           "l2": f"inputs {w.logit_bytes / 1e6:.0f} MB > L2, back to back"},
+                "roofline": {"bound": "hbm", "kernel": "shard_pass1_kernel (rank 0's shard)",
+                             "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                             "traffic": None, "peak_kind": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
+                             "algorithmic_bytes_per_launch": alg1, "us_per_launch": ms_pass1 * 1e3},
+                "cpu_baseline": None, "e2e": None, "gpu_launches": launches * args.steps}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
 def main():
     args = parse()
     if args.record_traffic:
@@ -600,6 +702,8 @@ def main():
         return
     if args.impl == "reference":
         run_reference(args)
+    elif args.vocab_shards:
+        run_sharded(args)
     else:
         run_ours(args)
 
