@@ -489,6 +489,46 @@ __device__ __forceinline__ void online_row<uint16_t, true>(const uint16_t *src, 
   s = make_float4(acc.x, acc.y, acb.x, acb.y);
 }
 
+// online_row<uint16_t, true> for the row a token rule screens: the chunk's two
+// largest logits of this thread (y1 >= y2, a tie giving y1 == y2) from packed
+// bf16x2 max/min over the raw words, in the sweep that takes the maximum.
+__device__ __forceinline__ void online_row_top2(const uint16_t *src, float k, float &m, float4 &s, float &y1,
+                                                float &y2) {
+  uint32_t w[kRounds * 4];
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r) {
+    const uint4 v = *reinterpret_cast<const uint4 *>(src + 8 * (r * kNT + static_cast<int>(threadIdx.x)));
+    w[4 * r] = v.x; w[4 * r + 1] = v.y; w[4 * r + 2] = v.z; w[4 * r + 3] = v.w;
+  }
+  __nv_bfloat162 m1 = as_bf162(w[0]), m2 = as_bf162(0xFF80FF80u);  // (-inf, -inf)
+#pragma unroll
+  for (int i = 1; i < kRounds * 4; ++i) {
+    const __nv_bfloat162 v = as_bf162(w[i]);
+    m2 = __hmax2(m2, __hmin2(m1, v));
+    m1 = __hmax2(m1, v);
+  }
+  const float a = __low2float(m1), b = __high2float(m1);
+  y1 = fmaxf(a, b);
+  y2 = fmaxf(fminf(a, b), fmaxf(__low2float(m2), __high2float(m2)));
+  const float mn = fmaxf(m, y1);
+  const float rn = refk(mn, k);
+  const float sc = ex2(refk(m, k) - rn);
+  float2 acc = __fmul2_rn(make_float2(s.x, s.y), make_float2(sc, sc));
+  float2 acb = __fmul2_rn(make_float2(s.z, s.w), make_float2(sc, sc));
+  const float2 kk = make_float2(k, k), nr = make_float2(-rn, -rn);
+#pragma unroll
+  for (int i = 0; i < kRounds * 4; i += 2) {
+    const float2 y = make_float2(__uint_as_float(w[i] << 16), __uint_as_float(w[i] & 0xFFFF0000u));
+    const float2 t = __ffma2_rn(y, kk, nr);
+    acc = __fadd2_rn(acc, make_float2(ex2(t.x), ex2(t.y)));
+    const float2 y3 = make_float2(__uint_as_float(w[i + 1] << 16), __uint_as_float(w[i + 1] & 0xFFFF0000u));
+    const float2 t2 = __ffma2_rn(y3, kk, nr);
+    acb = __fadd2_rn(acb, make_float2(ex2(t2.x), ex2(t2.y)));
+  }
+  m = mn;
+  s = make_float4(acc.x, acc.y, acb.x, acb.y);
+}
+
 // Pass-1 state of the kFamExt rules.  With a_v = y^q_v k - r_q and
 // b_v = y^p_v k - r_p relative to the references r = refk(m) of the running
 // maxima m:
@@ -737,6 +777,8 @@ __device__ __forceinline__ void ext_pair_bf16(const uint16_t *srcq, const uint16
 // the test, so eta = 1 - (their q) needs no pass over the row.
 struct Top2 {
   float y1, y2, z1;
+  int c1;      // chunk holding y1 (packed chunks: z1 not kept, looked up when needed)
+  bool known;  // z1 holds the draft logit at y1
 };
 
 template <typename E, bool kFull>
@@ -754,6 +796,7 @@ __device__ __forceinline__ void screen_chunk(const E *ssrc, const E *qsrc, int n
           t.y2 = t.y1;
           t.y1 = y[i];
           t.z1 = z[i];
+          t.known = true;
         } else {
           t.y2 = y[i];
         }
@@ -1473,7 +1516,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   float mq = -FLT_MAX, mp = -FLT_MAX;
   float4 s2q = make_float4(0.0f, 0.0f, 0.0f, 0.0f), s2p = s2q;
   ExtState ex = ext_empty();  // (kFamExt) moments and argmaxes
-  Top2 top = {-FLT_MAX, -FLT_MAX, -FLT_MAX};  // (kFamToken) the eta screen
+  Top2 top = {-FLT_MAX, -FLT_MAX, -FLT_MAX, -1, false};  // (kFamToken) the eta screen
   const bool scr_q = P.rule == SC_RULE_TOKEN_V1;
   // OPT: the pair's running sum of sqrt(q p) terms, relative to (r_q + r_p) / 2
   const bool opt_bc = SC_OPT_UB && P.opt_ub && !kTok && !kExt && verify && pair && P.rule == SC_RULE_OPT;
@@ -1518,7 +1561,34 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
       }
       if (!fused) {
         const float mq0 = mq, mp0 = mp;
-        if (n == kCH) {
+        bool screened = false;
+        if constexpr (kTok && sizeof(E) == 2) {
+          if (pair && n == kCH) {
+            // the screened row's top two come out of its max sweep; the draft
+            // logit at the largest is looked up only if the screen needs it
+            const uint16_t *sq16 = reinterpret_cast<const uint16_t *>(R.q(s));
+            const uint16_t *sp16 = reinterpret_cast<const uint16_t *>(R.p(s));
+            float c1, c2;
+            if (scr_q) {
+              online_row_top2(sq16, k, mq, s2q, c1, c2);
+              online_row<uint16_t, true>(sp16, n, k, mp, s2p);
+            } else {
+              online_row<uint16_t, true>(sq16, n, k, mq, s2q);
+              online_row_top2(sp16, k, mp, s2p, c1, c2);
+            }
+            if (c1 > top.y1) {
+              top.y2 = fmaxf(top.y1, c2);
+              top.y1 = c1;
+              top.c1 = c;
+              top.known = false;
+            } else {
+              top.y2 = fmaxf(top.y2, c1);
+            }
+            screened = true;
+          }
+        }
+        if (screened) {
+        } else if (n == kCH) {
           if (pair) online_row<E, true>(R.q(s), n, k, mq, s2q);
           online_row<E, true>(R.p(s), n, k, mp, s2p);
           if (kTok && pair) screen_chunk<E, true>(scr_q ? R.q(s) : R.p(s), R.q(s), n, top);
@@ -1760,8 +1830,30 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   // cluster, eta = (S_q - sum of 2^a over those tokens) / S_q.
   if (kTok && sh.tok && sh.need_p2) {
     const float Rs = sh.on_q ? sh.Rq : sh.Rp;  // r(v) tests a_v or b_v, formed as vec_weights forms them
-    const bool ok = !(fmaf(top.y2, k, -Rs) >= sh.thr);
-    const float h = fmaf(top.y1, k, -Rs) >= sh.thr ? ex2(fmaf(top.z1, k, -sh.Rq)) : 0.0f;
+    bool ok = !(fmaf(top.y2, k, -Rs) >= sh.thr);
+    float h = 0.0f;
+    if (fmaf(top.y1, k, -Rs) >= sh.thr) {
+      float z1 = top.z1;
+      bool have = top.known;
+      if (!have && SC_CHECK(top.c1 >= 0 && top.c1 < R.nch && R.chunk_len(top.c1) == kCH)) {
+        // y1 came from a full chunk swept in packed form: this thread's first
+        // logit equal to y1 in that chunk (the sweep's order) and the draft
+        // logit there, read element by element from the slice in global memory
+        const size_t c0 = static_cast<size_t>(top.c1) * kCH;
+        const E *ts = scr_q ? R.gq : R.gp;
+        for (int r = 0; r < kRounds && !have; ++r) {
+          const int e = 8 * (r * kNT + tid);
+          for (int i = 0; i < 8; ++i)
+            if (Elt<E>::at(ts, c0 + e + i) == top.y1) {
+              z1 = Elt<E>::at(R.gq, c0 + e + i);
+              have = true;
+              break;
+            }
+        }
+      }
+      ok = ok && have;  // (not found cannot happen; it would take the eta pass)
+      if (have) h = ex2(fmaf(z1, k, -sh.Rq));
+    }
     const bool wok = __all_sync(0xFFFFFFFFu, ok);
     const float hs = warp_sum(h);
     if (lane == 0) sh.red[warp] = make_float4(hs, wok ? 1.0f : 0.0f, 0.0f, 0.0f);
