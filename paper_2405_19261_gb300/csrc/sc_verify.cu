@@ -704,7 +704,7 @@ __device__ __forceinline__ int first_index_of(const uint32_t (&w)[kRounds * 4], 
 }
 
 __device__ __forceinline__ void ext_pair_bf16(const uint16_t *srcq, const uint16_t *srcp, int v0, float k,
-                                              ExtState &st) {
+                                              ExtState &st, bool argmax) {
   uint32_t wq[kRounds * 4], wp[kRounds * 4];
 #pragma unroll
   for (int r = 0; r < kRounds; ++r) {
@@ -725,13 +725,14 @@ __device__ __forceinline__ void ext_pair_bf16(const uint16_t *srcq, const uint16
   const float cp = fmaxf(__low2float(xp), __high2float(xp));
   float mq = st.mq, mp = st.mp;
   int iq = st.iq, ip = st.ip;
+  // (the argmaxes are read only by greedy decoding)
   if (cq > mq) {
     mq = cq;
-    iq = first_index_of(wq, cq, v0);
+    if (argmax) iq = first_index_of(wq, cq, v0);
   }
   if (cp > mp) {
     mp = cp;
-    ip = first_index_of(wp, cp, v0);
+    if (argmax) ip = first_index_of(wp, cp, v0);
   }
   const float rq = refk(mq, k), rp = refk(mp, k);
   ext_rebase(st, refk(st.mq, k) - rq, refk(st.mp, k) - rp);
@@ -1538,7 +1539,7 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
         if constexpr (sizeof(E) == 2) {
           if (n == kCH) {
             ext_pair_bf16(reinterpret_cast<const uint16_t *>(R.q(s)), reinterpret_cast<const uint16_t *>(R.p(s)),
-                          vc, k, ex);
+                          vc, k, ex, P.greedy != 0);
             done = true;
           }
         }
