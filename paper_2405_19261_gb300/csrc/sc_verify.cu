@@ -586,6 +586,19 @@ __device__ __forceinline__ void ext_merge(ExtState &b, ExtState a, float k) {
 
 // Merge the partials of the 32 lanes of a warp (butterfly); lane 0 ends with
 // the warp's partial.
+// The first of this thread's logits equal to m in the chunk starting at token
+// vc (the order of the sweep), as a token index; row = the slice's row in global
+// memory, v0 its first token.  -1 if none (cannot happen for a recorded maximum).
+template <typename E>
+__device__ __forceinline__ int ext_resolve_index(const E *row, int v0, int vc, float m) {
+  for (int r = 0; r < kRounds; ++r) {
+    const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
+    for (int i = 0; i < 8; ++i)
+      if (Elt<E>::at(row, static_cast<size_t>(vc - v0 + e + i)) == m) return vc + e + i;
+  }
+  return -1;
+}
+
 __device__ __forceinline__ void ext_warp_merge(ExtState &e, float k) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
@@ -693,15 +706,11 @@ __device__ __forceinline__ void ext_chunk(const E *srcq, const E *srcp, int n, i
 // finite product 0 * a = 0 where ext_chunk skips the term; a finite draft logit
 // with a masked target logit still makes X = -inf (D(q, p) = +inf), found by a
 // scan of the chunks whose target minimum is -inf.
-__device__ __forceinline__ int first_index_of(const uint32_t (&w)[kRounds * 4], float m, int v0) {
-#pragma unroll
-  for (int i = 0; i < kRounds * 4; ++i) {
-    const int e = 8 * ((i >> 2) * kNT + static_cast<int>(threadIdx.x)) + 2 * (i & 3);
-    if (__uint_as_float(w[i] << 16) == m) return v0 + e;
-    if (__uint_as_float(w[i] & 0xFFFF0000u) == m) return v0 + e + 1;
-  }
-  return -1;
-}
+// Greedy decoding's argmaxes in packed chunks are not located during the
+// sweep: a thread whose running maximum rises in the chunk starting at token
+// vc records the code -2 - vc, and ext_resolve_index finds the position later
+// for the threads that hold their warp's maximum.
+__device__ __forceinline__ int lazy_code(int vc) { return -2 - vc; }
 
 __device__ __forceinline__ void ext_pair_bf16(const uint16_t *srcq, const uint16_t *srcp, int v0, float k,
                                               ExtState &st, bool argmax) {
@@ -725,14 +734,14 @@ __device__ __forceinline__ void ext_pair_bf16(const uint16_t *srcq, const uint16
   const float cp = fmaxf(__low2float(xp), __high2float(xp));
   float mq = st.mq, mp = st.mp;
   int iq = st.iq, ip = st.ip;
-  // (the argmaxes are read only by greedy decoding)
+  // (the argmaxes are read only by greedy decoding, located after pass 1)
   if (cq > mq) {
     mq = cq;
-    if (argmax) iq = first_index_of(wq, cq, v0);
+    if (argmax) iq = lazy_code(v0);
   }
   if (cp > mp) {
     mp = cp;
-    if (argmax) ip = first_index_of(wp, cp, v0);
+    if (argmax) ip = lazy_code(v0);
   }
   const float rq = refk(mq, k), rp = refk(mp, k);
   ext_rebase(st, refk(st.mq, k) - rq, refk(st.mp, k) - rp);
@@ -1627,6 +1636,18 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
   const float4 mq4 = s2q, mp4 = s2p;  // ... split over its logits 0, 1, 2, 3 (mod 4)
   tmo = __syncthreads_or(tmo);
   if constexpr (kExt) {
+    if (P.greedy) {
+      // locate the argmaxes recorded as chunk codes, for the threads holding their
+      // warp's maximum (the others cannot win the merge)
+      float wq = ex.mq, wp = ex.mp;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        wq = fmaxf(wq, __shfl_xor_sync(0xFFFFFFFFu, wq, o));
+        wp = fmaxf(wp, __shfl_xor_sync(0xFFFFFFFFu, wp, o));
+      }
+      if (ex.iq <= -2 && ex.mq == wq) ex.iq = ext_resolve_index(R.gq, v0, -2 - ex.iq, ex.mq);
+      if (ex.ip <= -2 && ex.mp == wp) ex.ip = ext_resolve_index(R.gp, v0, -2 - ex.ip, ex.mp);
+    }
     ext_warp_merge(ex, k);
     if (lane == 0) {
       sh.red[warp] = make_float4(ex.mq, ex.sq, ex.mp, ex.sp);
