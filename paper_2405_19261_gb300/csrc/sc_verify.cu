@@ -589,6 +589,46 @@ __device__ __forceinline__ void ext_merge(ExtState &b, ExtState a, float k) {
 // The first of this thread's logits equal to m in the chunk starting at token
 // vc (the order of the sweep), as a token index; row = the slice's row in global
 // memory, v0 its first token.  -1 if none (cannot happen for a recorded maximum).
+// Greedy decoding's argmaxes in packed chunks are not located during the
+// sweep: a thread whose running maximum rises in the chunk starting at token
+// vc records the code -2 - vc, and ext_resolve_index finds the position later
+// for the threads that hold their warp's maximum.
+__device__ __forceinline__ int lazy_code(int vc) { return -2 - vc; }
+
+// Greedy decoding's bonus row (p only), full bf16 chunk: the maximum by a
+// packed max tree (its position recorded as a chunk code) and the sum of
+// exponentials by packed arithmetic; the bonus row needs no moments.
+__device__ __forceinline__ void ext_bonus_bf16(const uint16_t *srcp, int v0, float k, ExtState &st) {
+  uint32_t wp[kRounds * 4];
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r) {
+    const uint4 v = *reinterpret_cast<const uint4 *>(srcp + 8 * (r * kNT + static_cast<int>(threadIdx.x)));
+    wp[4 * r] = v.x; wp[4 * r + 1] = v.y; wp[4 * r + 2] = v.z; wp[4 * r + 3] = v.w;
+  }
+  __nv_bfloat162 xp = as_bf162(wp[0]);
+#pragma unroll
+  for (int i = 1; i < kRounds * 4; ++i) xp = __hmax2(xp, as_bf162(wp[i]));
+  const float cp = fmaxf(__low2float(xp), __high2float(xp));
+  float mp = st.mp;
+  int ip = st.ip;
+  if (cp > mp) {
+    mp = cp;
+    ip = lazy_code(v0);
+  }
+  const float rp = refk(mp, k);
+  const float sc = ex2(refk(st.mp, k) - rp);
+  const float2 kk = make_float2(k, k), nrp = make_float2(-rp, -rp);
+  float2 sp = make_float2(0.0f, 0.0f);
+#pragma unroll
+  for (int i = 0; i < kRounds * 4; ++i) {
+    const float2 b = __ffma2_rn(make_float2(__uint_as_float(wp[i] << 16), __uint_as_float(wp[i] & 0xFFFF0000u)), kk, nrp);
+    sp = __fadd2_rn(sp, make_float2(ex2(b.x), ex2(b.y)));
+  }
+  st.mp = mp;
+  st.ip = ip;
+  st.sp = fmaf(st.sp, sc, sp.x + sp.y);
+}
+
 template <typename E>
 __device__ __forceinline__ int ext_resolve_index(const E *row, int v0, int vc, float m) {
   for (int r = 0; r < kRounds; ++r) {
@@ -706,12 +746,6 @@ __device__ __forceinline__ void ext_chunk(const E *srcq, const E *srcp, int n, i
 // finite product 0 * a = 0 where ext_chunk skips the term; a finite draft logit
 // with a masked target logit still makes X = -inf (D(q, p) = +inf), found by a
 // scan of the chunks whose target minimum is -inf.
-// Greedy decoding's argmaxes in packed chunks are not located during the
-// sweep: a thread whose running maximum rises in the chunk starting at token
-// vc records the code -2 - vc, and ext_resolve_index finds the position later
-// for the threads that hold their warp's maximum.
-__device__ __forceinline__ int lazy_code(int vc) { return -2 - vc; }
-
 __device__ __forceinline__ void ext_pair_bf16(const uint16_t *srcq, const uint16_t *srcp, int v0, float k,
                                               ExtState &st, bool argmax) {
   uint32_t wq[kRounds * 4], wp[kRounds * 4];
@@ -1557,8 +1591,17 @@ __global__ void __launch_bounds__(kNT, kMinBlocksPerSM) sc_unit_kernel(const Par
           else ext_chunk<E, false, true>(R.q(s), R.p(s), n, vc, k, ex);
         }
       } else {
-        if (n == kCH) ext_chunk<E, true, false>(R.q(s), R.p(s), n, vc, k, ex);
-        else ext_chunk<E, false, false>(R.q(s), R.p(s), n, vc, k, ex);
+        bool done = false;
+        if constexpr (sizeof(E) == 2) {
+          if (n == kCH && P.greedy) {
+            ext_bonus_bf16(reinterpret_cast<const uint16_t *>(R.p(s)), vc, k, ex);
+            done = true;
+          }
+        }
+        if (!done) {
+          if (n == kCH) ext_chunk<E, true, false>(R.q(s), R.p(s), n, vc, k, ex);
+          else ext_chunk<E, false, false>(R.q(s), R.p(s), n, vc, k, ex);
+        }
       }
     } else {
       bool fused = false;
