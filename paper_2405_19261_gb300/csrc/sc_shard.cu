@@ -66,7 +66,7 @@ enum UnitKind : int { kAccepted = 0, kRejected = 1, kNeedTV = 2, kBonus = 3, kBa
 struct UnitState {
   double Sq, Sp;      // sums of 2^{fma(y, k, -R)} over the whole row
   double maxq, maxp;  // max_v q(v), max_v p(v)
-  double L;           // log2 p(x) - log2 q(x) (both finite)
+  float Lhi, Llo;     // log2 p(x) - log2 q(x) (both finite) as a double-float hi + lo
   float Rq, Rp;       // exponent references fl(M k)
   float c;            // log2(S_q / S_p) rounded to f32: the residual weights' shift
   int kind;           // UnitKind
@@ -95,6 +95,7 @@ struct Geom {
   int slots;  // slices of kL tokens of this rank
   long long ld;
   float k;    // log2(e) / T in f32
+  float kl;   // log2(e) / T - k: with k, log2(e) / T to twice f32 precision
   double kd;  // log2(e) / T in double
   int rule;
   double alpha;
@@ -535,12 +536,44 @@ __device__ __forceinline__ void merge_ranks(const float4 *const *recs, int W, si
   }
 }
 
+// Double-float f32 arithmetic (a value is hi + lo, |lo| <= ulp(hi) / 2): the
+// precision of the acceptance ratio at f32 speed (this GPU's f64 rate is low).
+// two_sum: a + b = s + e exactly (Knuth); an FMA gives a product's rounding error.
+__device__ __forceinline__ float2 two_sum(float a, float b) {
+  const float s = __fadd_rn(a, b);
+  const float bb = __fsub_rn(s, a);
+  return make_float2(s, __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb)));
+}
+__device__ __forceinline__ float2 quick_norm(float hi, float lo) {
+  const float s = __fadd_rn(hi, lo);
+  return make_float2(s, __fsub_rn(lo, __fsub_rn(s, hi)));
+}
+
+// log2 p(x) - log2 q(x) for logits yp, yq of rows with maxima Mp, Mq, references
+// Rp, Rq and sums Sp, Sq (of 2^{fma(y, k, -R)}):
+//   log2 p(y) = y (k + kl) - R - log2 S - M kl = y k - R + (y - M) kl - log2 S,
+// the f32 factor k of the sums' exponents corrected to log2(e) / T = k + kl for
+// each row's dominant terms (y near M).  The difference of the two is formed
+// from exact pieces: yp - yq by two_sum, its product with k by an FMA.
+__device__ __forceinline__ float2 log_ratio(float yp, float yq, float Mp, float Mq, float Rp, float Rq, float Sp,
+                                            float Sq, float k, float kl) {
+  const float2 d = two_sum(yp, -yq);                      // yp - yq = d.x + d.y
+  const float dk = __fmul_rn(d.x, k), dke = fmaf(d.x, k, -dk);  // d.x k = dk + dke
+  const float2 r = two_sum(Rp, -Rq);                      // Rp - Rq
+  const float2 t = two_sum(dk, -r.x);
+  const float corr = __fmul_rn(__fsub_rn(__fsub_rn(yp, Mp), __fsub_rn(yq, Mq)), kl);
+  const float lo = __fadd_rn(__fadd_rn(__fadd_rn(__fadd_rn(t.y, dke), __fsub_rn(__fmul_rn(d.y, k), r.y)), corr),
+                             log2f(Sq / Sp));
+  return quick_norm(t.x, lo);
+}
+
 // Acceptance of the draft token when delta = 1 (pi = p): [u < min(1, p(x)/q(x))];
-// q(x) = 0 accepts, p(x) = 0 < q(x) rejects.
+// q(x) = 0 accepts, p(x) = 0 < q(x) rejects.  2^L = 2^hi (1 + lo ln 2).
 __device__ __forceinline__ bool accept_deferred(const UnitState &s, float u) {
   if (s.xq0) return true;
   if (s.xp0) return false;
-  return s.L >= 0.0 || static_cast<double>(u) < exp2(s.L);
+  if (s.Lhi > 0.0f || (s.Lhi == 0.0f && s.Llo >= 0.0f)) return true;
+  return u < exp2f(s.Lhi) * fmaf(s.Llo, 0.69314718f, 1.0f);
 }
 
 // Margin by which a bound on D_TV must clear the OPT threshold to settle delta
@@ -609,21 +642,15 @@ __global__ void shard_decide_kernel(Geom G, const void *__restrict__ gathered1, 
     return;
   }
   s.maxq = ex2(fmaf(Mq, G.k, -Rq)) / Sq;
-  // double-precision work (log2(S_q / S_p), the acceptance ratio) on lane 0 only
-  const double lsr = lane == 0 ? log2(static_cast<double>(Sq) / static_cast<double>(Sp)) : 0.0;
-  s.c = static_cast<float>(lsr);
+  s.c = log2f(Sq / Sp);
   const float2 xl = msg1_at(const_cast<char *>(static_cast<const char *>(gathered1)) + owner_of(G, x) * msg1,
                             G.B, G.gamma).x[b * G.gamma + j];
   s.xq0 = !(xl.x > -INFINITY);
   s.xp0 = !(xl.y > -INFINITY);
-  if (lane == 0 && !s.xq0 && !s.xp0) {
-    // log2 p(x) - log2 q(x), each log2 p(y) = y kd - M (kd - k) - R - log2 S: the
-    // exponents' f32 factor k corrected to kd = log2(e) / T for the row's
-    // dominant terms (those with y near M)
-    const double kl = G.kd - static_cast<double>(G.k);
-    s.L = (static_cast<double>(xl.y) - static_cast<double>(xl.x)) * G.kd -
-          (static_cast<double>(Mp) - static_cast<double>(Mq)) * kl - (static_cast<double>(Rp) - static_cast<double>(Rq)) +
-          lsr;
+  if (!s.xq0 && !s.xp0) {
+    const float2 L = log_ratio(xl.y, xl.x, Mp, Mq, Rp, Rq, Sp, Sq, G.k, G.kl);
+    s.Lhi = L.x;
+    s.Llo = L.y;
   }
   int delta;
   switch (G.rule) {
@@ -752,7 +779,7 @@ __global__ void shard_accept_kernel(Geom G, const double *__restrict__ gathered2
           settled0 |= v < 0.0;  // delta = 0 by that rank's part of the lower bound
           R += v;
         }
-        const double tv = R / s.Sq;
+        const double tv = static_cast<float>(R) / static_cast<float>(s.Sq);  // (f32 division: f64 is slow here)
         acc = settled0 || !(s.maxq < s.maxp - G.alpha * tv) || accept_deferred(s, uniforms[b * (G.gamma + 1) + j]);
       }
       rej = !acc;
@@ -1105,6 +1132,7 @@ int make_geom(int B, int gamma, int W, int rank, const int *shard_begin, float t
   G->ld = ld;
   G->kd = 1.4426950408889634 / static_cast<double>(temperature);
   G->k = static_cast<float>(G->kd);
+  G->kl = static_cast<float>(G->kd - static_cast<double>(G->k));
   G->rule = rule;
   G->alpha = alpha;
   return SC_OK;
