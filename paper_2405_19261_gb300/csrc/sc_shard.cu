@@ -187,7 +187,8 @@ struct Raw8;
 template <>
 struct Raw8<uint16_t> {  // bf16 bit patterns
   uint4 v;
-  __device__ __forceinline__ void load(const uint16_t *s) { v = __ldg(reinterpret_cast<const uint4 *>(s)); }
+  // streaming loads (evict first): the slice is read once here
+  __device__ __forceinline__ void load(const uint16_t *s) { v = __ldcs(reinterpret_cast<const uint4 *>(s)); }
   __device__ __forceinline__ void to_float(float (&y)[8]) const {
     const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
