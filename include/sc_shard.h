@@ -7,8 +7,9 @@
  * target pi = (1 - delta) q + delta p, Eq. 6, for the deferral rules of Table 1
  * and SpecDecode's delta = 1), with the reductions over the vocabulary that
  * sc_verify does inside one thread-block cluster done in two levels: inside
- * each GPU, then across GPUs through four small messages that the caller
- * exchanges with an all-gather (e.g. NCCL).  No logit ever leaves its GPU.
+ * each GPU, then across GPUs through small messages that the caller exchanges
+ * with an all-gather (e.g. NCCL): four, five with SC_RULE_OPT.  No logit ever
+ * leaves its GPU.
  *
  * One step on every rank r, in this order (the caller all-gathers each
  * message in rank order between the calls):
@@ -24,19 +25,21 @@
  *                    (Table 1) and the acceptance test (Algorithm 4).  With
  *                    SC_RULE_OPT a pair inside the band
  *                    max p - alpha <= max q < max p needs D_TV (Eq. 10):
- *                    where neither the upper bound nor this rank's part of a
- *                    lower bound settles delta, the rank sums its part of the
- *                    residual weights (Lemma 3)                -> message 2
- *   sc_shard_accept  merges the W messages 2, finishes delta and acceptance
+ *                    where the upper bound does not settle delta, the rank
+ *                    sends its part of a lower bound on D_TV  -> message 2 (OPT)
+ *   sc_shard_tv      (SC_RULE_OPT only) sums the W parts of the lower bound;
+ *                    where it does not settle delta = 0 either, the rank sums
+ *                    its part of the residual weights (Lemma 3) -> message 3 (OPT)
+ *   sc_shard_accept  merges the W messages 3, finishes delta and acceptance
  *                    of the band pairs, settles j* = min{j : a_j = 0}, and
  *                    sums the rank's part of the weights of the row it draws
  *                    from: norm(max(0, p - q)) of row j*, or p of the bonus
- *                    row when j* = gamma                      -> message 3
+ *                    row when j* = gamma                      -> message 4
  *   sc_shard_draw    finds the rank, slice and segment holding u R (the
  *                    inverse CDF in ascending token order, u = uniforms[b][gamma]);
  *                    that rank draws the token, the others send -1
- *                                                              -> message 4
- *   sc_shard_finish  merges the W messages 4 into num_accepted and next_token
+ *                                                              -> message 5
+ *   sc_shard_finish  merges the W messages 5 into num_accepted and next_token
  *                    (identical on every rank).
  *
  * Conventions are those of sc.h: device pointers owned by the caller, work
@@ -80,7 +83,7 @@ extern "C" {
 
 #define SC_SHARD_MAX 16
 
-/* Bytes of one rank's message k (1..4) for B sequences of gamma drafts
+/* Bytes of one rank's message k (1..5) for B sequences of gamma drafts
  * (independent of V and W; 0 for another k). */
 size_t sc_shard_message_bytes(int B, int gamma, int message);
 
@@ -92,26 +95,33 @@ int sc_shard_pass1(const void *draft_shard, const void *target_shard, sc_dtype d
                    const int *shard_begin, float temperature, sc_rule rule, void *workspace,
                    size_t workspace_bytes, void *send1, cudaStream_t stream);
 
+/* send2 is written only with SC_RULE_OPT (NULL is allowed otherwise). */
 int sc_shard_decide(const void *draft_shard, const void *target_shard, sc_dtype dtype, int64_t ld,
                     const void *gathered1, const int32_t *draft_tokens, const float *uniforms,
                     int B, int gamma, int W, int rank, const int *shard_begin, sc_rule rule,
                     float alpha, float temperature, void *workspace, size_t workspace_bytes,
                     void *send2, int32_t *device_status, cudaStream_t stream);
 
-/* gathered2 is read only with SC_RULE_OPT (NULL is allowed otherwise). */
+/* SC_RULE_OPT only (another rule is SC_ERR_INVALID_ARG). */
+int sc_shard_tv(const void *draft_shard, const void *target_shard, sc_dtype dtype, int64_t ld,
+                const void *gathered2, int B, int gamma, int W, int rank, const int *shard_begin,
+                sc_rule rule, float alpha, float temperature, void *workspace,
+                size_t workspace_bytes, void *send3, cudaStream_t stream);
+
+/* gathered3 is read only with SC_RULE_OPT (NULL is allowed otherwise). */
 int sc_shard_accept(const void *draft_shard, const void *target_shard, sc_dtype dtype, int64_t ld,
-                    const void *gathered2, const float *uniforms, int B, int gamma, int W,
+                    const void *gathered3, const float *uniforms, int B, int gamma, int W,
                     int rank, const int *shard_begin, sc_rule rule, float alpha,
-                    float temperature, void *workspace, size_t workspace_bytes, void *send3,
+                    float temperature, void *workspace, size_t workspace_bytes, void *send4,
                     cudaStream_t stream);
 
 int sc_shard_draw(const void *draft_shard, const void *target_shard, sc_dtype dtype, int64_t ld,
-                  const void *gathered3, const float *uniforms, int B, int gamma, int W, int rank,
+                  const void *gathered4, const float *uniforms, int B, int gamma, int W, int rank,
                   const int *shard_begin, float temperature, void *workspace,
-                  size_t workspace_bytes, void *send4, cudaStream_t stream);
+                  size_t workspace_bytes, void *send5, cudaStream_t stream);
 
 /* num_accepted [B] int32: j*; next_token [B] int32: the token emitted at j*. */
-int sc_shard_finish(const void *gathered4, int B, int gamma, int W, const void *workspace,
+int sc_shard_finish(const void *gathered5, int B, int gamma, int W, const void *workspace,
                     size_t workspace_bytes, int32_t *num_accepted, int32_t *next_token,
                     cudaStream_t stream);
 

@@ -3,8 +3,8 @@
 //
 // Each rank holds the logits of a contiguous range of tokens of every row.
 // The step is Algorithm 4 with Algorithm 5's target, for the deferral rules of
-// Table 1 (and delta = 1, delta = 0), written as five phases with an
-// all-gather of a small message between consecutive phases:
+// Table 1 (and delta = 1, delta = 0), written as phases with an all-gather of
+// a small message between consecutive phases:
 //
 //   pass 1   grid (unit, slice): every CTA reads one slice of kL logits of a
 //            row pair (or of the bonus target row) with coalesced 16-byte
@@ -14,25 +14,24 @@
 //            per warp, kept for the lower bound on D_TV below, and per slice;
 //            OPT pairs also sum the Bhattacharyya terms 2^{(a + b)/2}; a
 //            second kernel merges the rank's slices per unit   -> message 1
-//   decide   one thread per unit merges the W ranks' partials in double
-//            precision, in rank order (identical on every rank): M, S, max q,
-//            max p, delta by the rule, and the acceptance test.  OPT pairs in
-//            the band max p - alpha <= max q < max p need D_TV (Eq. 10):
-//            every rank settles delta = 1 where the Hellinger bound
-//            D_TV <= (1 - BC^2)^{1/2} decides; a rank settles delta = 0 where
-//            its own part of the lower bound sum_t max(0, P_t - Q_t) over its
-//            warps' token sets decides (and says so in its message); the rest
-//            take a TV pass, a grid (pair, slice) summing the residual weights
-//            max(0, 2^{b + c} - 2^a) = S_q max(0, p - q) over the rank's part
-//            of the row                                          -> message 2
-//   accept   one thread per sequence finishes the band pairs (Eq. 10: delta = 0
-//            if any rank settled it, else from the exact D_TV),
-//            settles j*, and a grid (sequence, slice) sums the weights of the
-//            row to draw from -- the residual of row j*, or p of the bonus
-//            row -- per 256-token segment (warp scans in double) -> message 3
-//   draw     one warp per sequence finds the rank, slice, segment and token
-//            holding u R in ascending token order; only the rank holding it
-//            rescans that one segment                            -> message 4
+//   decide   one warp per unit merges the W ranks' partials in rank order
+//            (identical on every rank): M, S, max q, max p, delta by the rule,
+//            and the acceptance test.  OPT pairs in the band
+//            max p - alpha <= max q < max p need D_TV (Eq. 10): every rank
+//            settles delta = 1 where the Hellinger bound D_TV <= (1 - BC^2)^{1/2}
+//            decides; for the rest the rank sends its part of the lower bound
+//            sum_t max(0, P_t - Q_t) over its warps' token sets -> message 2
+//   tv       (OPT) the summed lower bound settles delta = 0 where it decides;
+//            the rest take a TV pass, a grid walking the work list of
+//            (pair, slice) items, summing max(0, 2^{b + c} - 2^a) =
+//            S_q max(0, p - q) over the rank's part of the row -> message 3
+//   accept   one warp per sequence finishes the band pairs (Eq. 10) and
+//            settles j*; a grid (sequence, slice) sums the residual weights of
+//            row j* of rejected sequences; a sequence that reaches the bonus
+//            row takes p's slice sums from pass 1             -> message 4
+//   draw     one CTA per sequence: the rank holding u R finds the slice, the
+//            segment and the token in ascending token order; the other ranks
+//            send -1                                          -> message 5
 //   finish   one thread per sequence takes the drawing rank's token.
 //
 // Every sum that a later phase splits again (rank totals into slices, slices
@@ -71,7 +70,7 @@ struct UnitState {
   float c;            // log2(S_q / S_p) rounded to f32: the residual weights' shift
   int kind;           // UnitKind
   int xq0, xp0;       // q(x) = 0, p(x) = 0 (masked logits at the draft token)
-  int settled0;       // kNeedTV: this rank's part of the lower bound on D_TV settles delta = 0
+  int settled0;       // kNeedTV: the lower bound on D_TV (every rank's part) settles delta = 0
 };
 
 // Pass-1 record of one (unit, slice), every sum relative to the references
@@ -119,9 +118,10 @@ size_t msg_bytes(int B, int gamma, int k) {
   const size_t units = static_cast<size_t>(B) * (gamma + 1), pairs = static_cast<size_t>(B) * gamma;
   switch (k) {
     case 1: return align16(units * sizeof(float4)) + align16(pairs * sizeof(float2)) + align16(pairs * sizeof(float));
-    case 2: return align16(pairs * sizeof(double));
-    case 3: return align16(static_cast<size_t>(B) * sizeof(double));
-    case 4: return align16(static_cast<size_t>(B) * sizeof(int32_t));
+    case 2: return align16(pairs * sizeof(float));
+    case 3: return align16(pairs * sizeof(double));
+    case 4: return align16(static_cast<size_t>(B) * sizeof(double));
+    case 5: return align16(static_cast<size_t>(B) * sizeof(int32_t));
     default: return 0;
   }
 }
@@ -599,7 +599,7 @@ __device__ __forceinline__ float rank_lower_bound(const Geom &G, const SlotRec *
 __global__ void shard_decide_kernel(Geom G, const void *__restrict__ gathered1, size_t msg1,
                                     const int32_t *__restrict__ tokens, const float *__restrict__ uniforms,
                                     const SlotRec *__restrict__ slot_rec, UnitState *__restrict__ unit,
-                                    int *__restrict__ tv_count, int *__restrict__ tv_list, int32_t *status) {
+                                    float *__restrict__ send2, int32_t *status) {
   // one warp per unit: every lane merges the ranks' records (the same values);
   // the lanes share the lower bound's slices; lane 0 writes
   const int lane = threadIdx.x & 31;
@@ -680,13 +680,13 @@ __global__ void shard_decide_kernel(Geom G, const void *__restrict__ gathered1, 
     if (s.maxq < s.maxp - G.alpha * ub - kBoundMargin) {
       delta = 1;
     } else {
+      // this rank's part of the lower bound, summed over the ranks by sc_shard_tv
       const float lb = rank_lower_bound(G, slot_rec + static_cast<size_t>(u) * G.slots, Rq, Rp, Sq, Sp, lane);
-      s.settled0 = s.maxq >= s.maxp - G.alpha * lb + kBoundMargin;
+      if (lane == 0) send2[b * G.gamma + j] = lb;
     }
   }
   if (delta < 0) {
     s.kind = kNeedTV;
-    if (!s.settled0 && lane == 0) tv_list[atomicAdd(tv_count, 1)] = b * G.gamma + j;  // the TV pass's work list
   } else if (lane == 0) {
     s.kind = !delta || accept_deferred(s, uj) ? kAccepted : kRejected;
   }
@@ -735,26 +735,42 @@ __global__ void __launch_bounds__(kT) shard_tv_kernel(const E *__restrict__ q, c
   }
 }
 
+// One thread per pair (OPT): the lower bound on D_TV summed over the ranks'
+// parts (rank order, the same on every rank) settles delta = 0 where it
+// decides; the other band pairs join the TV pass's work list.
+__global__ void shard_settle_kernel(Geom G, const float *__restrict__ gathered2, size_t msg2_floats,
+                                    UnitState *__restrict__ unit, int *__restrict__ tv_count,
+                                    int *__restrict__ tv_list) {
+  const int pr = blockIdx.x * blockDim.x + threadIdx.x;
+  if (pr >= G.B * G.gamma) return;
+  const int b = pr / G.gamma, j = pr % G.gamma;
+  UnitState &st = unit[b * (G.gamma + 1) + j];
+  if (st.kind != kNeedTV) return;
+  float lb = 0.0f;
+  for (int r = 0; r < G.W; ++r) lb += gathered2[r * msg2_floats + pr];
+  st.settled0 = st.maxq >= st.maxp - G.alpha * lb + kBoundMargin;
+  if (!st.settled0) tv_list[atomicAdd(tv_count, 1)] = pr;
+}
+
 // One thread per pair: the rank's part of S_q D_TV, in slice order (0 for a
-// pair that does not need it, -1 for one whose delta = 0 this rank settled).
-__global__ void shard_merge2_kernel(Geom G, const UnitState *__restrict__ unit, const float *__restrict__ tv_slot,
-                                    double *__restrict__ send2) {
+// pair that takes no TV pass).
+__global__ void shard_merge_tv_kernel(Geom G, const UnitState *__restrict__ unit, const float *__restrict__ tv_slot,
+                                      double *__restrict__ send3) {
   const int pr = blockIdx.x * blockDim.x + threadIdx.x;
   if (pr >= G.B * G.gamma) return;
   const int b = pr / G.gamma, j = pr % G.gamma;
   const UnitState &st = unit[b * (G.gamma + 1) + j];
   double t = 0.0;
-  if (st.kind == kNeedTV && st.settled0) t = -1.0;  // delta = 0 by this rank's lower bound
-  else if (st.kind == kNeedTV)
+  if (st.kind == kNeedTV && !st.settled0)
     for (int s = 0; s < G.slots; ++s) t += static_cast<double>(tv_slot[static_cast<size_t>(pr) * G.slots + s]);
-  send2[pr] = t;
+  send3[pr] = t;
 }
 
 // ------------------------------------------------------------------ accept
 
 // One warp per sequence (lane j takes position j): delta of the band pairs
 // from D_TV (Eq. 10), acceptance, and j* = min{j : a_j = 0}.
-__global__ void shard_accept_kernel(Geom G, const double *__restrict__ gathered2, size_t msg2_doubles,
+__global__ void shard_accept_kernel(Geom G, const double *__restrict__ gathered3, size_t msg3_doubles,
                                     const float *__restrict__ uniforms, const UnitState *__restrict__ unit,
                                     SeqState *__restrict__ seq) {
   const int lane = threadIdx.x & 31;
@@ -763,7 +779,7 @@ __global__ void shard_accept_kernel(Geom G, const double *__restrict__ gathered2
   const UnitState *us = unit + static_cast<size_t>(b) * (G.gamma + 1);
   int bad = 0;
   for (int j = lane; j <= G.gamma; j += 32)
-    bad |= us[j].kind == kBad || (us[j].kind == kNeedTV && gathered2 == nullptr);  // (decided as OPT, accepted as not)
+    bad |= us[j].kind == kBad || (us[j].kind == kNeedTV && gathered3 == nullptr);  // (decided as OPT, accepted as not)
   bad = __any_sync(0xFFFFFFFFu, bad);
   int jstar = G.gamma;
   for (int j0 = 0; !bad && j0 < G.gamma; j0 += 32) {
@@ -774,14 +790,10 @@ __global__ void shard_accept_kernel(Geom G, const double *__restrict__ gathered2
       bool acc = s.kind == kAccepted;
       if (s.kind == kNeedTV) {
         double R = 0.0;
-        bool settled0 = false;
-        for (int r = 0; r < G.W; ++r) {
-          const double v = gathered2[r * msg2_doubles + b * G.gamma + j];
-          settled0 |= v < 0.0;  // delta = 0 by that rank's part of the lower bound
-          R += v;
-        }
+        if (!s.settled0)
+          for (int r = 0; r < G.W; ++r) R += gathered3[r * msg3_doubles + b * G.gamma + j];
         const double tv = static_cast<float>(R) / static_cast<float>(s.Sq);  // (f32 division: f64 is slow here)
-        acc = settled0 || !(s.maxq < s.maxp - G.alpha * tv) || accept_deferred(s, uniforms[b * (G.gamma + 1) + j]);
+        acc = s.settled0 || !(s.maxq < s.maxp - G.alpha * tv) || accept_deferred(s, uniforms[b * (G.gamma + 1) + j]);
       }
       rej = !acc;
     }
@@ -1219,83 +1231,102 @@ int sc_shard_decide(const void *draft, const void *target, sc_dtype dtype, int64
   Geom G;
   int rc = make_geom(B, gamma, W, rank, shard_begin, temperature, rule, alpha, ld, &G);
   if (rc == SC_OK) rc = check_logits(draft, target, dtype);
-  if (rc == SC_OK && (!gathered1 || !draft_tokens || !uniforms || !send2 || !device_accessible(gathered1) ||
+  if (rc == SC_OK && (!gathered1 || !draft_tokens || !uniforms || !device_accessible(gathered1) ||
                       !device_accessible(draft_tokens) || !device_accessible(uniforms) ||
-                      !device_accessible(send2) || (device_status && !device_accessible(device_status))))
+                      (rule == SC_RULE_OPT && (!send2 || !device_accessible(send2))) ||
+                      (device_status && !device_accessible(device_status))))
     rc = SC_ERR_INVALID_ARG;
   if (rc == SC_OK) rc = check_work(G, workspace, workspace_bytes);
   if (rc != SC_OK) return rc;
   Work w;
   work_layout(B, gamma, G.slots, workspace, &w);
-  const int units = B * (gamma + 1), pairs = B * gamma;
-  if (rule == SC_RULE_OPT && cudaMemsetAsync(w.tv_count, 0, sizeof(int), stream) != cudaSuccess) return SC_ERR_CUDA;
+  const int units = B * (gamma + 1);
   shard_decide_kernel<<<(units * 32 + kT - 1) / kT, kT, 0, stream>>>(G, gathered1, msg_bytes(B, gamma, 1), draft_tokens,
-                                                               uniforms, w.slot_rec, w.unit, w.tv_count, w.tv_list,
-                                                               device_status);
-  if (rule == SC_RULE_OPT) {
-    const bool vec = vec_ok(draft, dtype, ld) && vec_ok(target, dtype, ld);
-    const int grid = std::min(pairs * G.slots, 8 * sm_count());  // CTAs walking the TV work list
-    SC_SHARD_DISPATCH(shard_tv_kernel, grid, G, w.unit, w.tv_count, w.tv_list, w.tv_slot);
-    shard_merge2_kernel<<<(pairs + kT - 1) / kT, kT, 0, stream>>>(G, w.unit, w.tv_slot,
-                                                                  static_cast<double *>(send2));
-  }
+                                                               uniforms, w.slot_rec, w.unit,
+                                                               static_cast<float *>(send2), device_status);
+  return launched();
+}
+
+int sc_shard_tv(const void *draft, const void *target, sc_dtype dtype, int64_t ld, const void *gathered2,
+                int B, int gamma, int W, int rank, const int *shard_begin, sc_rule rule, float alpha,
+                float temperature, void *workspace, size_t workspace_bytes, void *send3, cudaStream_t stream) {
+  t_capturing = capturing(stream);
+  Geom G;
+  int rc = make_geom(B, gamma, W, rank, shard_begin, temperature, rule, alpha, ld, &G);
+  if (rc == SC_OK && rule != SC_RULE_OPT) rc = SC_ERR_INVALID_ARG;
+  if (rc == SC_OK) rc = check_logits(draft, target, dtype);
+  if (rc == SC_OK && (!gathered2 || !send3 || !device_accessible(gathered2) || !device_accessible(send3)))
+    rc = SC_ERR_INVALID_ARG;
+  if (rc == SC_OK) rc = check_work(G, workspace, workspace_bytes);
+  if (rc != SC_OK) return rc;
+  Work w;
+  work_layout(B, gamma, G.slots, workspace, &w);
+  const int pairs = B * gamma;
+  if (cudaMemsetAsync(w.tv_count, 0, sizeof(int), stream) != cudaSuccess) return SC_ERR_CUDA;
+  shard_settle_kernel<<<(pairs + kT - 1) / kT, kT, 0, stream>>>(G, static_cast<const float *>(gathered2),
+                                                                msg_bytes(B, gamma, 2) / sizeof(float), w.unit,
+                                                                w.tv_count, w.tv_list);
+  const bool vec = vec_ok(draft, dtype, ld) && vec_ok(target, dtype, ld);
+  const int grid = std::min(pairs * G.slots, 8 * sm_count());  // CTAs walking the TV work list
+  SC_SHARD_DISPATCH(shard_tv_kernel, grid, G, w.unit, w.tv_count, w.tv_list, w.tv_slot);
+  shard_merge_tv_kernel<<<(pairs + kT - 1) / kT, kT, 0, stream>>>(G, w.unit, w.tv_slot, static_cast<double *>(send3));
   return launched();
 }
 
 int sc_shard_accept(const void *draft, const void *target, sc_dtype dtype, int64_t ld,
-                    const void *gathered2, const float *uniforms, int B, int gamma, int W,
+                    const void *gathered3, const float *uniforms, int B, int gamma, int W,
                     int rank, const int *shard_begin, sc_rule rule, float alpha,
-                    float temperature, void *workspace, size_t workspace_bytes, void *send3,
+                    float temperature, void *workspace, size_t workspace_bytes, void *send4,
                     cudaStream_t stream) {
   t_capturing = capturing(stream);
   Geom G;
   int rc = make_geom(B, gamma, W, rank, shard_begin, temperature, rule, alpha, ld, &G);
   if (rc == SC_OK) rc = check_logits(draft, target, dtype);
-  if (rc == SC_OK && (!uniforms || !send3 || !device_accessible(uniforms) || !device_accessible(send3)))
+  if (rc == SC_OK && (!uniforms || !send4 || !device_accessible(uniforms) || !device_accessible(send4)))
     rc = SC_ERR_INVALID_ARG;
-  if (rc == SC_OK && rule == SC_RULE_OPT && (!gathered2 || !device_accessible(gathered2))) rc = SC_ERR_INVALID_ARG;
+  if (rc == SC_OK && rule == SC_RULE_OPT && (!gathered3 || !device_accessible(gathered3))) rc = SC_ERR_INVALID_ARG;
   if (rc == SC_OK) rc = check_work(G, workspace, workspace_bytes);
   if (rc != SC_OK) return rc;
   Work w;
   work_layout(B, gamma, G.slots, workspace, &w);
   shard_accept_kernel<<<(B * 32 + kT - 1) / kT, kT, 0, stream>>>(
-      G, rule == SC_RULE_OPT ? static_cast<const double *>(gathered2) : nullptr,
-      msg_bytes(B, gamma, 2) / sizeof(double), uniforms, w.unit, w.seq);
+      G, rule == SC_RULE_OPT ? static_cast<const double *>(gathered3) : nullptr,
+      msg_bytes(B, gamma, 3) / sizeof(double), uniforms, w.unit, w.seq);
   const bool vec = vec_ok(draft, dtype, ld) && vec_ok(target, dtype, ld);
   SC_SHARD_DISPATCH(shard_mass_kernel, B * G.slots, G, w.unit, w.seq, w.slot_mass);
   shard_merge3_kernel<<<(B * 32 + kT - 1) / kT, kT, 0, stream>>>(G, w.unit, w.seq, w.slot_rec, w.slot_mass,
-                                                            static_cast<double *>(send3));
+                                                                 static_cast<double *>(send4));
   return launched();
 }
 
 int sc_shard_draw(const void *draft, const void *target, sc_dtype dtype, int64_t ld,
-                  const void *gathered3, const float *uniforms, int B, int gamma, int W, int rank,
+                  const void *gathered4, const float *uniforms, int B, int gamma, int W, int rank,
                   const int *shard_begin, float temperature, void *workspace,
-                  size_t workspace_bytes, void *send4, cudaStream_t stream) {
+                  size_t workspace_bytes, void *send5, cudaStream_t stream) {
   t_capturing = capturing(stream);
   Geom G;
   int rc = make_geom(B, gamma, W, rank, shard_begin, temperature, SC_RULE_CHOW, 0.0f, ld, &G);
   if (rc == SC_OK) rc = check_logits(draft, target, dtype);
-  if (rc == SC_OK && (!gathered3 || !uniforms || !send4 || !device_accessible(gathered3) ||
-                      !device_accessible(uniforms) || !device_accessible(send4)))
+  if (rc == SC_OK && (!gathered4 || !uniforms || !send5 || !device_accessible(gathered4) ||
+                      !device_accessible(uniforms) || !device_accessible(send5)))
     rc = SC_ERR_INVALID_ARG;
   if (rc == SC_OK) rc = check_work(G, workspace, workspace_bytes);
   if (rc != SC_OK) return rc;
   Work w;
   work_layout(B, gamma, G.slots, workspace, &w);
   const bool vec = vec_ok(draft, dtype, ld) && vec_ok(target, dtype, ld);
-  SC_SHARD_DISPATCH(shard_draw_kernel, B, G, static_cast<const double *>(gathered3),
-                    msg_bytes(B, gamma, 3) / sizeof(double), uniforms, w.unit, w.seq, w.slot_rec, w.slot_mass,
-                    static_cast<int32_t *>(send4));
+  SC_SHARD_DISPATCH(shard_draw_kernel, B, G, static_cast<const double *>(gathered4),
+                    msg_bytes(B, gamma, 4) / sizeof(double), uniforms, w.unit, w.seq, w.slot_rec, w.slot_mass,
+                    static_cast<int32_t *>(send5));
   return launched();
 }
 
-int sc_shard_finish(const void *gathered4, int B, int gamma, int W, const void *workspace,
+int sc_shard_finish(const void *gathered5, int B, int gamma, int W, const void *workspace,
                     size_t workspace_bytes, int32_t *num_accepted, int32_t *next_token,
                     cudaStream_t stream) {
   t_capturing = capturing(stream);
   if (B < 1 || gamma < 1 || gamma > SC_MAX_GAMMA || W < 1 || W > SC_SHARD_MAX) return SC_ERR_INVALID_ARG;
-  if (!gathered4 || !num_accepted || !next_token || !device_accessible(gathered4) ||
+  if (!gathered5 || !num_accepted || !next_token || !device_accessible(gathered5) ||
       !device_accessible(num_accepted) || !device_accessible(next_token))
     return SC_ERR_INVALID_ARG;
   // the sequence states sit at the same offset for every shard width
@@ -1303,8 +1334,8 @@ int sc_shard_finish(const void *gathered4, int B, int gamma, int W, const void *
   if (workspace_bytes < work_layout(B, gamma, 1, nullptr, nullptr)) return SC_ERR_WORKSPACE;
   Work w;
   work_layout(B, gamma, 1, const_cast<void *>(workspace), &w);
-  shard_finish_kernel<<<(B + kT - 1) / kT, kT, 0, stream>>>(B, W, static_cast<const int32_t *>(gathered4),
-                                                            msg_bytes(B, gamma, 4) / sizeof(int32_t), w.seq,
+  shard_finish_kernel<<<(B + kT - 1) / kT, kT, 0, stream>>>(B, W, static_cast<const int32_t *>(gathered5),
+                                                            msg_bytes(B, gamma, 5) / sizeof(int32_t), w.seq,
                                                             num_accepted, next_token);
   return launched();
 }

@@ -1,8 +1,8 @@
 """Vocabulary-sharded verification (include/sc_shard.h).
 
 Each rank holds the logits of a contiguous range of tokens of every row (a
-tensor-parallel LM head).  One step is five library calls per rank with an
-all-gather of a small message between consecutive calls; this module only
+tensor-parallel LM head).  One step is five library calls per rank (six with
+OPT) with an all-gather of a small message between consecutive calls; this module only
 marshals arguments and moves the messages: every step of the method runs in
 the library's kernels.
 
@@ -45,10 +45,12 @@ def lib():
         L.sc_shard_workspace_bytes.restype = S
         L.sc_shard_pass1.argtypes = [P, P, I, L64, P, I, I, I, I, IA, F, I, P, S, P, P]
         L.sc_shard_decide.argtypes = [P, P, I, L64, P, P, P, I, I, I, I, IA, I, F, F, P, S, P, P, P]
+        L.sc_shard_tv.argtypes = [P, P, I, L64, P, I, I, I, I, IA, I, F, F, P, S, P, P]
         L.sc_shard_accept.argtypes = [P, P, I, L64, P, P, I, I, I, I, IA, I, F, F, P, S, P, P]
         L.sc_shard_draw.argtypes = [P, P, I, L64, P, P, I, I, I, I, IA, F, P, S, P, P]
         L.sc_shard_finish.argtypes = [P, I, I, I, P, S, P, P, P]
-        for n in ("sc_shard_pass1", "sc_shard_decide", "sc_shard_accept", "sc_shard_draw", "sc_shard_finish"):
+        for n in ("sc_shard_pass1", "sc_shard_decide", "sc_shard_tv", "sc_shard_accept", "sc_shard_draw",
+                  "sc_shard_finish"):
             getattr(L, n).restype = I
         _declared = True
     return L
@@ -80,7 +82,7 @@ def _rule_code(rule) -> int:
 
 
 class ShardRank:
-    """The buffers of one rank: workspace, its four messages, its outputs."""
+    """The buffers of one rank: workspace, its five messages, its outputs."""
 
     def __init__(self, B: int, gamma: int, bounds: Sequence[int], rank: int, dtype: torch.dtype,
                  device=None):
@@ -95,7 +97,7 @@ class ShardRank:
         nws = int(L.sc_shard_workspace_bytes(B, gamma, self.width, binding._dtype_code(torch.empty(0, dtype=dtype))))
         self.workspace = torch.empty(nws, dtype=torch.uint8, device=dev)
         self.send = [None] + [torch.zeros(message_bytes(B, gamma, k), dtype=torch.uint8, device=dev)
-                              for k in (1, 2, 3, 4)]
+                              for k in (1, 2, 3, 4, 5)]
         self.num_accepted = torch.empty(B, dtype=torch.int32, device=dev)
         self.next_token = torch.empty(B, dtype=torch.int32, device=dev)
         self.status = torch.zeros(1, dtype=torch.int32, device=dev)
@@ -144,31 +146,41 @@ class ShardRank:
         binding._check(rc, "sc_shard_decide")
         return self.send[2]
 
-    def accept(self, draft, target, gathered2, uniforms, rule, alpha, temperature, stream=None):
+    def tv(self, draft, target, gathered2, rule, alpha, temperature, stream=None):
         d, t, dt, ld = self._shard(draft, target)
-        if gathered2 is not None:
-            self._gathered(gathered2, 2)
-        rc = lib().sc_shard_accept(binding._ptr(d), binding._ptr(t), dt, ld, binding._ptr(gathered2),
+        self._gathered(gathered2, 2)
+        rc = lib().sc_shard_tv(binding._ptr(d), binding._ptr(t), dt, ld, binding._ptr(gathered2), self.B,
+                               self.gamma, self.W, self.rank, self._cb, _rule_code(rule), float(alpha),
+                               float(temperature), binding._ptr(self.workspace), self.workspace.numel(),
+                               binding._ptr(self.send[3]), binding._stream(stream))
+        binding._check(rc, "sc_shard_tv")
+        return self.send[3]
+
+    def accept(self, draft, target, gathered3, uniforms, rule, alpha, temperature, stream=None):
+        d, t, dt, ld = self._shard(draft, target)
+        if gathered3 is not None:
+            self._gathered(gathered3, 3)
+        rc = lib().sc_shard_accept(binding._ptr(d), binding._ptr(t), dt, ld, binding._ptr(gathered3),
                                    binding._ptr(uniforms), self.B, self.gamma, self.W, self.rank, self._cb,
                                    _rule_code(rule), float(alpha), float(temperature),
                                    binding._ptr(self.workspace), self.workspace.numel(),
-                                   binding._ptr(self.send[3]), binding._stream(stream))
+                                   binding._ptr(self.send[4]), binding._stream(stream))
         binding._check(rc, "sc_shard_accept")
-        return self.send[3]
-
-    def draw(self, draft, target, gathered3, uniforms, temperature, stream=None):
-        d, t, dt, ld = self._shard(draft, target)
-        self._gathered(gathered3, 3)
-        rc = lib().sc_shard_draw(binding._ptr(d), binding._ptr(t), dt, ld, binding._ptr(gathered3),
-                                 binding._ptr(uniforms), self.B, self.gamma, self.W, self.rank, self._cb,
-                                 float(temperature), binding._ptr(self.workspace), self.workspace.numel(),
-                                 binding._ptr(self.send[4]), binding._stream(stream))
-        binding._check(rc, "sc_shard_draw")
         return self.send[4]
 
-    def finish(self, gathered4, stream=None) -> Tuple[torch.Tensor, torch.Tensor]:
+    def draw(self, draft, target, gathered4, uniforms, temperature, stream=None):
+        d, t, dt, ld = self._shard(draft, target)
         self._gathered(gathered4, 4)
-        rc = lib().sc_shard_finish(binding._ptr(gathered4), self.B, self.gamma, self.W,
+        rc = lib().sc_shard_draw(binding._ptr(d), binding._ptr(t), dt, ld, binding._ptr(gathered4),
+                                 binding._ptr(uniforms), self.B, self.gamma, self.W, self.rank, self._cb,
+                                 float(temperature), binding._ptr(self.workspace), self.workspace.numel(),
+                                 binding._ptr(self.send[5]), binding._stream(stream))
+        binding._check(rc, "sc_shard_draw")
+        return self.send[5]
+
+    def finish(self, gathered5, stream=None) -> Tuple[torch.Tensor, torch.Tensor]:
+        self._gathered(gathered5, 5)
+        rc = lib().sc_shard_finish(binding._ptr(gathered5), self.B, self.gamma, self.W,
                                    binding._ptr(self.workspace), self.workspace.numel(),
                                    binding._ptr(self.num_accepted), binding._ptr(self.next_token),
                                    binding._stream(stream))
@@ -215,13 +227,17 @@ def sharded_step(ranks: List[ShardRank], shards: List[Tuple[torch.Tensor, torch.
     width_i]) of ranks[i]; tokens [B, gamma] int32 and uniforms [B, gamma+1]
     float32 are the same on every rank."""
     code = _rule_code(rule)
+    opt = code == binding.RULES["opt"]
     g1 = exchange([r.pass1(d, t, tokens, temperature, code, stream) for r, (d, t) in zip(ranks, shards)])
     s2 = [r.decide(d, t, g1, tokens, uniforms, code, alpha, temperature, stream) for r, (d, t) in zip(ranks, shards)]
-    g2 = exchange(s2) if code == binding.RULES["opt"] else None
-    g3 = exchange([r.accept(d, t, g2, uniforms, code, alpha, temperature, stream)
+    g3 = None
+    if opt:  # the lower bound's parts, then the D_TV parts of the pairs it did not settle
+        g2 = exchange(s2)
+        g3 = exchange([r.tv(d, t, g2, code, alpha, temperature, stream) for r, (d, t) in zip(ranks, shards)])
+    g4 = exchange([r.accept(d, t, g3, uniforms, code, alpha, temperature, stream)
                    for r, (d, t) in zip(ranks, shards)])
-    g4 = exchange([r.draw(d, t, g3, uniforms, temperature, stream) for r, (d, t) in zip(ranks, shards)])
-    return [r.finish(g4, stream) for r in ranks]
+    g5 = exchange([r.draw(d, t, g4, uniforms, temperature, stream) for r, (d, t) in zip(ranks, shards)])
+    return [r.finish(g5, stream) for r in ranks]
 
 
 def emulated_step(draft: torch.Tensor, target: torch.Tensor, tokens: torch.Tensor, uniforms: torch.Tensor,

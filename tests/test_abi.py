@@ -30,7 +30,7 @@ def declared_functions(headers=(HEADER, SHARD_HEADER)):
 def test_header_declares_the_boundary():
     names = declared_functions()
     for n in ("sc_verify", "sc_row_stats", "sc_workspace_bytes", "sc_status_string", "sc_shard_pass1",
-              "sc_shard_decide", "sc_shard_accept", "sc_shard_draw", "sc_shard_finish"):
+              "sc_shard_decide", "sc_shard_tv", "sc_shard_accept", "sc_shard_draw", "sc_shard_finish"):
         assert n in names
 
 
@@ -118,15 +118,18 @@ def test_shard_host_only_entry_points(so):
     so.sc_shard_workspace_bytes.restype = S
     so.sc_shard_workspace_bytes.argtypes = [I, I, I, I]
     B, g = 512, 8
-    # message 1: (m_q, s_q, m_p, s_p) per unit and the draft token's two logits
-    # per pair; 2: S_q D_TV per pair; 3: a total weight per sequence; 4: a token
+    # message 1: (m_q, s_q, m_p, s_p) per unit, the draft token's two logits and
+    # the Bhattacharyya sum per pair; 2 (OPT): a part of the lower bound on D_TV
+    # per pair; 3 (OPT): a part of S_q D_TV per pair; 4: a total weight per
+    # sequence; 5: a token
     assert so.sc_shard_message_bytes(B, g, 1) == B * (g + 1) * 16 + B * g * 8 + B * g * 4
-    assert so.sc_shard_message_bytes(B, g, 2) == B * g * 8
-    assert so.sc_shard_message_bytes(B, g, 3) == B * 8
-    assert so.sc_shard_message_bytes(B, g, 4) == B * 4
-    assert so.sc_shard_message_bytes(B, g, 5) == 0 and so.sc_shard_message_bytes(0, g, 1) == 0
+    assert so.sc_shard_message_bytes(B, g, 2) == B * g * 4
+    assert so.sc_shard_message_bytes(B, g, 3) == B * g * 8
+    assert so.sc_shard_message_bytes(B, g, 4) == B * 8
+    assert so.sc_shard_message_bytes(B, g, 5) == B * 4
+    assert so.sc_shard_message_bytes(B, g, 6) == 0 and so.sc_shard_message_bytes(0, g, 1) == 0
     # independent of V: the messages are tiny against the 4.46 GB of logits
-    assert sum(so.sc_shard_message_bytes(B, g, k) for k in (1, 2, 3, 4)) < 200_000
+    assert sum(so.sc_shard_message_bytes(B, g, k) for k in (1, 2, 3, 4, 5)) < 200_000
     small, big = so.sc_shard_workspace_bytes(B, g, 8192, 1), so.sc_shard_workspace_bytes(B, g, 128000, 1)
     assert 0 < small < big
     assert so.sc_shard_workspace_bytes(B, g, 0, 1) == 0
@@ -158,15 +161,16 @@ def test_shard_header_is_plain_c(tmp_path):
     src.write_text("""
 #include "sc_shard.h"
 int use_shard(const void *q, const void *p, const int32_t *x, const float *u, void *ws, void *s1,
-              void *g1, void *s2, void *g2, void *s3, void *g3, void *s4, void *g4, int32_t *na,
-              int32_t *nt, int32_t *st, cudaStream_t s) {
+              void *g1, void *s2, void *g2, void *s3, void *g3, void *s4, void *g4, void *s5, void *g5,
+              int32_t *na, int32_t *nt, int32_t *st, cudaStream_t s) {
   const int bounds[3] = {0, 128000, 256000};
   size_t n = sc_shard_workspace_bytes(4, 3, 128000, SC_BF16) + sc_shard_message_bytes(4, 3, 1);
   int rc = sc_shard_pass1(q, p, SC_BF16, 128000, x, 4, 3, 2, 0, bounds, 1.0f, SC_RULE_OPT, ws, n, s1, s);
   rc |= sc_shard_decide(q, p, SC_BF16, 128000, g1, x, u, 4, 3, 2, 0, bounds, SC_RULE_OPT, 0.2f, 1.0f, ws, n, s2, st, s);
-  rc |= sc_shard_accept(q, p, SC_BF16, 128000, g2, u, 4, 3, 2, 0, bounds, SC_RULE_OPT, 0.2f, 1.0f, ws, n, s3, s);
-  rc |= sc_shard_draw(q, p, SC_BF16, 128000, g3, u, 4, 3, 2, 0, bounds, 1.0f, ws, n, s4, s);
-  rc |= sc_shard_finish(g4, 4, 3, 2, ws, n, na, nt, s);
+  rc |= sc_shard_tv(q, p, SC_BF16, 128000, g2, 4, 3, 2, 0, bounds, SC_RULE_OPT, 0.2f, 1.0f, ws, n, s3, s);
+  rc |= sc_shard_accept(q, p, SC_BF16, 128000, g3, u, 4, 3, 2, 0, bounds, SC_RULE_OPT, 0.2f, 1.0f, ws, n, s4, s);
+  rc |= sc_shard_draw(q, p, SC_BF16, 128000, g4, u, 4, 3, 2, 0, bounds, 1.0f, ws, n, s5, s);
+  rc |= sc_shard_finish(g5, 4, 3, 2, ws, n, na, nt, s);
   return rc + SC_SHARD_MAX;
 }
 """)

@@ -17,7 +17,7 @@ if ROOT not in sys.path:
 
 from paper_2405_19261_gb300 import sharded  # noqa: E402
 
-SIZES = {1: 48, 2: 16, 3: 8, 4: 8}
+SIZES = {1: 48, 2: 16, 3: 16, 4: 8, 5: 8}
 
 
 class PhaseProbe:
@@ -44,23 +44,29 @@ class PhaseProbe:
         self.log.append("decide")
         return self._msg(2)
 
-    def accept(self, d, t, g2, uniforms, rule, alpha, T, stream=None):
-        if rule == 2:  # OPT: the D_TV parts were exchanged
-            self._expect(g2, 2)
-        else:
-            assert g2 is None
-        self.log.append("accept")
+    def tv(self, d, t, g2, rule, alpha, T, stream=None):
+        assert rule == 2  # OPT only: the lower bound's parts were exchanged
+        self._expect(g2, 2)
+        self.log.append("tv")
         return self._msg(3)
 
-    def draw(self, d, t, g3, uniforms, T, stream=None):
-        self._expect(g3, 3)
-        self.log.append("draw")
+    def accept(self, d, t, g3, uniforms, rule, alpha, T, stream=None):
+        if rule == 2:  # OPT: the D_TV parts were exchanged
+            self._expect(g3, 3)
+        else:
+            assert g3 is None
+        self.log.append("accept")
         return self._msg(4)
 
-    def finish(self, g4, stream=None):
+    def draw(self, d, t, g4, uniforms, T, stream=None):
         self._expect(g4, 4)
+        self.log.append("draw")
+        return self._msg(5)
+
+    def finish(self, g5, stream=None):
+        self._expect(g5, 5)
         self.log.append("finish")
-        return torch.tensor([self.W]), g4.clone()
+        return torch.tensor([self.W]), g5.clone()
 
 
 def test_shard_bounds():
@@ -87,8 +93,9 @@ def test_phases_in_one_process(rule):
     W = 3
     ranks = [PhaseProbe(r, W) for r in range(W)]
     out = sharded.sharded_step(ranks, [(None, None)] * W, None, None, rule, 0.2, 1.0, sharded.LocalExchange())
+    phases = ["pass1", "decide"] + (["tv"] if rule == "opt" else []) + ["accept", "draw", "finish"]
     for r in ranks:
-        assert r.log == ["pass1", "decide", "accept", "draw", "finish"]
+        assert r.log == phases
     assert all(torch.equal(o[1], out[0][1]) for o in out)
 
 
@@ -130,6 +137,7 @@ def test_two_gloo_ranks_exchange_in_rank_order(rule):
         p.join(180)
         assert p.exitcode == 0
     res = sorted(queue.get(timeout=10) for _ in range(2))
+    phases = ["pass1", "decide"] + (["tv"] if rule == "opt" else []) + ["accept", "draw", "finish"]
     for rank, log, final in res:
-        assert log == ["pass1", "decide", "accept", "draw", "finish"]
+        assert log == phases
     assert res[0][2] == res[1][2]  # both ranks hold the same gathered result
