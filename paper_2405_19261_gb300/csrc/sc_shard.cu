@@ -52,12 +52,16 @@
 
 namespace {
 
-constexpr int kT = 256;                 // threads per CTA
+#ifndef SC_SHARD_THREADS
+#define SC_SHARD_THREADS 128
+#endif
+
+constexpr int kT = SC_SHARD_THREADS;    // threads per CTA
 constexpr int kWarps = kT / 32;         // warps per CTA
 constexpr int kSeg = 256;               // tokens per segment: one warp, 8 per lane
-constexpr int kSegs = 32;               // segments per slice
-constexpr int kL = kSeg * kSegs;        // 8192 tokens per slice
-constexpr int kRounds = kSegs / kWarps; // segments per warp per slice
+constexpr int kRounds = 4;              // segments per warp per slice
+constexpr int kSegs = kRounds * kWarps; // segments per slice
+constexpr int kL = kSeg * kSegs;        // tokens per slice (4096 at 128 threads)
 
 enum UnitKind : int { kAccepted = 0, kRejected = 1, kNeedTV = 2, kBonus = 3, kBad = 4 };
 
@@ -79,7 +83,7 @@ struct SlotRec {
   float4 ms;             // (m_q, s_q, m_p, s_p)
   float bc;              // OPT pairs: sum of 2^{(a + b)/2}, a and b the exponents of q and p
   float pad[3];
-  float2 set[8];         // (s_q, s_p) over the tokens of each warp (the lower bound's sets)
+  float2 set[kWarps];    // (s_q, s_p) over the tokens of each warp (the lower bound's sets)
 };
 
 struct SeqState {
@@ -99,7 +103,7 @@ struct Geom {
   int rule;
   double alpha;
 };
-static_assert(sizeof(float2[8]) == 64, "SlotRec layout");
+static_assert(sizeof(SlotRec) % 16 == 0, "SlotRec layout");
 
 __host__ __device__ inline size_t align16(size_t n) { return (n + 15) & ~static_cast<size_t>(15); }
 
