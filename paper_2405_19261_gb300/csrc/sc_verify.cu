@@ -748,21 +748,22 @@ __device__ __forceinline__ void ext_chunk(const E *srcq, const E *srcp, int n, i
 // scan of the chunks whose target minimum is -inf.
 __device__ __forceinline__ void ext_pair_bf16(const uint16_t *srcq, const uint16_t *srcp, int v0, float k,
                                               ExtState &st, bool argmax) {
-  uint32_t wq[kRounds * 4], wp[kRounds * 4];
-#pragma unroll
+  // two sweeps over the chunk in shared memory, one round (4 words per row) at
+  // a time and not unrolled across rounds: the maxima, then the sums and
+  // moments (the same order of additions as one sweep over all 16 words)
+  __nv_bfloat162 xq = as_bf162(0xFF80FF80u), xp = xq, np = as_bf162(0x7F807F80u);  // -inf, -inf, +inf
+#pragma unroll 1
   for (int r = 0; r < kRounds; ++r) {
     const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
     const uint4 vq = *reinterpret_cast<const uint4 *>(srcq + e);
     const uint4 vp = *reinterpret_cast<const uint4 *>(srcp + e);
-    wq[4 * r] = vq.x; wq[4 * r + 1] = vq.y; wq[4 * r + 2] = vq.z; wq[4 * r + 3] = vq.w;
-    wp[4 * r] = vp.x; wp[4 * r + 1] = vp.y; wp[4 * r + 2] = vp.z; wp[4 * r + 3] = vp.w;
-  }
-  __nv_bfloat162 xq = as_bf162(wq[0]), xp = as_bf162(wp[0]), np = as_bf162(wp[0]);
+    const uint32_t wq[4] = {vq.x, vq.y, vq.z, vq.w}, wp[4] = {vp.x, vp.y, vp.z, vp.w};
 #pragma unroll
-  for (int i = 1; i < kRounds * 4; ++i) {
-    xq = __hmax2(xq, as_bf162(wq[i]));
-    xp = __hmax2(xp, as_bf162(wp[i]));
-    np = __hmin2(np, as_bf162(wp[i]));
+    for (int i = 0; i < 4; ++i) {
+      xq = __hmax2(xq, as_bf162(wq[i]));
+      xp = __hmax2(xp, as_bf162(wp[i]));
+      np = __hmin2(np, as_bf162(wp[i]));
+    }
   }
   const float cq = fmaxf(__low2float(xq), __high2float(xq));
   const float cp = fmaxf(__low2float(xp), __high2float(xp));
@@ -781,26 +782,34 @@ __device__ __forceinline__ void ext_pair_bf16(const uint16_t *srcq, const uint16
   ext_rebase(st, refk(st.mq, k) - rq, refk(st.mp, k) - rp);
   const __nv_bfloat162 lo = __float2bfloat162_rn(-1e30f);
   const float2 kk = make_float2(k, k), nrq = make_float2(-rq, -rq), nrp = make_float2(-rp, -rp);
+  const bool check_inf = !(fminf(__low2float(np), __high2float(np)) > -INFINITY);
   float2 sq = make_float2(0.0f, 0.0f), aq = sq, sp = sq, ap = sq, x = sq;
-#pragma unroll
-  for (int i = 0; i < kRounds * 4; ++i) {
-    const __nv_bfloat162 q2 = __hmax2(as_bf162(wq[i]), lo), p2 = __hmax2(as_bf162(wp[i]), lo);
-    const float2 a = __ffma2_rn(__bfloat1622float2(q2), kk, nrq);
-    const float2 b = __ffma2_rn(__bfloat1622float2(p2), kk, nrp);
-    const float2 ea = make_float2(ex2(a.x), ex2(a.y)), eb = make_float2(ex2(b.x), ex2(b.y));
-    sq = __fadd2_rn(sq, ea);
-    sp = __fadd2_rn(sp, eb);
-    aq = __ffma2_rn(ea, a, aq);
-    ap = __ffma2_rn(eb, b, ap);
-    x = __ffma2_rn(ea, b, x);
-  }
   bool inf_x = false;
-  if (!(fminf(__low2float(np), __high2float(np)) > -INFINITY)) {
+#pragma unroll 1
+  for (int r = 0; r < kRounds; ++r) {
+    const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
+    const uint4 vq = *reinterpret_cast<const uint4 *>(srcq + e);
+    const uint4 vp = *reinterpret_cast<const uint4 *>(srcp + e);
+    const uint32_t wq[4] = {vq.x, vq.y, vq.z, vq.w}, wp[4] = {vp.x, vp.y, vp.z, vp.w};
 #pragma unroll
-    for (int i = 0; i < kRounds * 4; ++i) {
-      const float q0 = __uint_as_float(wq[i] << 16), q1 = __uint_as_float(wq[i] & 0xFFFF0000u);
-      const float p0 = __uint_as_float(wp[i] << 16), p1 = __uint_as_float(wp[i] & 0xFFFF0000u);
-      inf_x |= (q0 > -INFINITY && !(p0 > -INFINITY)) || (q1 > -INFINITY && !(p1 > -INFINITY));
+    for (int i = 0; i < 4; ++i) {
+      const __nv_bfloat162 q2 = __hmax2(as_bf162(wq[i]), lo), p2 = __hmax2(as_bf162(wp[i]), lo);
+      const float2 a = __ffma2_rn(__bfloat1622float2(q2), kk, nrq);
+      const float2 b = __ffma2_rn(__bfloat1622float2(p2), kk, nrp);
+      const float2 ea = make_float2(ex2(a.x), ex2(a.y)), eb = make_float2(ex2(b.x), ex2(b.y));
+      sq = __fadd2_rn(sq, ea);
+      sp = __fadd2_rn(sp, eb);
+      aq = __ffma2_rn(ea, a, aq);
+      ap = __ffma2_rn(eb, b, ap);
+      x = __ffma2_rn(ea, b, x);
+    }
+    if (check_inf) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float q0 = __uint_as_float(wq[i] << 16), q1 = __uint_as_float(wq[i] & 0xFFFF0000u);
+        const float p0 = __uint_as_float(wp[i] << 16), p1 = __uint_as_float(wp[i] & 0xFFFF0000u);
+        inf_x |= (q0 > -INFINITY && !(p0 > -INFINITY)) || (q1 > -INFINITY && !(p1 > -INFINITY));
+      }
     }
   }
   st.mq = mq;
