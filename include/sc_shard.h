@@ -66,7 +66,8 @@
  *   temperature    0 < T < inf (greedy decoding is sc_verify's)
  *   rule, alpha    SC_RULE_CHOW .. SC_RULE_NEVER_DEFER, 0 <= alpha <= 1
  * The calls of one step must see the same B, gamma, W, shard_begin, rule, alpha
- * and temperature on every rank.
+ * and temperature on every rank.  Size limit: B (gamma + 1) max(32, slices) <=
+ * 2^31 - 1, slices = ceil(shard width / 4096) (the kernels' grids).
  */
 #ifndef SC_SHARD_H_
 #define SC_SHARD_H_

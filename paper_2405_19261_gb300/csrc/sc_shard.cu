@@ -1146,6 +1146,8 @@ int make_geom(int B, int gamma, int W, int rank, const int *shard_begin, float t
   G->width = shard_begin[rank + 1] - shard_begin[rank];
   if (ld < G->width) return SC_ERR_INVALID_ARG;
   G->slots = slots_of(G->width);
+  // grids: B (gamma + 1) slices for pass 1, a warp per unit for the merges
+  if (static_cast<double>(B) * (gamma + 1) * std::max(G->slots, 32) > 2147483647.0) return SC_ERR_INVALID_ARG;
   G->ld = ld;
   G->kd = 1.4426950408889634 / static_cast<double>(temperature);
   G->k = static_cast<float>(G->kd);

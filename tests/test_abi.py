@@ -146,6 +146,9 @@ def test_shard_calls_reject_bad_arguments_without_a_gpu(so):
                                (not_zero, 2, 0, 1.0), (good, 2, 0, 0.0), (good, 17, 0, 1.0), (None, 2, 0, 1.0)):
         rc = so.sc_shard_pass1(None, None, 1, 100, None, 4, 3, W, rank, bounds, T, 2, None, 0, None, None)
         assert rc == -1, (W, rank, T)
+    # a batch whose grids would not fit is refused before anything else
+    rc = so.sc_shard_pass1(None, None, 1, 100, None, 1 << 24, 255, 2, 0, good, 1.0, 2, None, 0, None, None)
+    assert rc == -1
     so.sc_shard_finish.argtypes = [P, I, I, I, P, S, P, P, P]
     assert so.sc_shard_finish(None, 4, 3, 2, None, 0, None, None, None) == -1
 
