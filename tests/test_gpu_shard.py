@@ -214,3 +214,26 @@ def test_masked_logits(sh):
     got = run_sharded(sh, w, sh.shard_bounds(w.V, 4))
     assert_sharded_parity(w, got, ref)
     assert got[0][2] == 0
+
+
+def test_graph_replay_matches_the_eager_step(sh):
+    # the step captured as one CUDA graph (what bench.py --vocab-shards times):
+    # replays with new inputs copied into the captured tensors give the eager
+    # step's outputs and the oracle's
+    import torch
+    from paper_2405_19261_gb300 import binding
+    bounds = sh.shard_bounds(32128, 3)
+    w0 = synthetic(16, 5, 32128, dtype="bf16", kind="gauss", sigma=0.5, rule="opt", alpha=0.2, seed=41)
+    d, t, x, u = binding.to_device(w0)
+    G = sh.EmulatedGraph(d, t, x, u, "opt", 0.2, 1.0, bounds)
+    for seed in (42, 43):
+        w = synthetic(16, 5, 32128, dtype="bf16", kind="gauss", sigma=0.5, rule="opt", alpha=0.2, seed=seed)
+        d1, t1, x1, u1 = binding.to_device(w)
+        d.copy_(d1), t.copy_(t1), x.copy_(x1), u.copy_(u1)
+        na, nt = G.replay()
+        torch.cuda.synchronize()
+        got = (na.cpu().numpy().copy(), nt.cpu().numpy().copy())
+        na2, nt2, _ = sh.emulated_step(d1, t1, x1, u1, "opt", 0.2, 1.0, bounds)
+        torch.cuda.synchronize()
+        assert np.array_equal(got[0], na2.cpu().numpy()) and np.array_equal(got[1], nt2.cpu().numpy())
+        assert_sharded_parity(w, (got[0], got[1], 0), oracle.verify_workload(w))
