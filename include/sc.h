@@ -16,6 +16,9 @@
  * or from pi_gamma := p_gamma (the drafter has no row at the bonus position)
  * when all gamma drafts are accepted.
  *
+ * The same step with the vocabulary split across GPUs (a tensor-parallel LM
+ * head) is declared in sc_shard.h.
+ *
  * Conventions of every entry point:
  *  - All array pointers are CUDA device pointers owned by the caller.  The
  *    library allocates no device memory per call and never synchronises: work
