@@ -14,9 +14,9 @@ Prints ONE JSON line (rank 0).  Keys beyond the base contract:
                 / CUDA-event time) against the measured copy bandwidth
   cpu_baseline  the fp64 oracle timed on this machine's host cores on a bounded
                 sample of the same workload
-  e2e           the same metric through the public API with host buffers, the
-                host->device copy of the inputs and the device->host read of
-                the outputs inside the timed region
+  e2e           the same metric through the public API with host buffers
+                (binding.HostVerifier), the host->device copy of the inputs and
+                the device->host read of the outputs inside the timed region
   clocks        nvidia-smi SM clock samples taken while the kernel ran
 
 --impl reference times the oracle (the only other implementation of this
@@ -77,6 +77,9 @@ def parse():
                          "(default for config 4: the other two Table 1 rules of the sweep; 'none' for none)")
     ap.add_argument("--sweep", action="store_true",
                     help="config 4: also time every sweep point (B x gamma) under Chow, Diff and OPT")
+    ap.add_argument("--e2e-chunks", type=int, default=4,
+                    help="e2e: groups of sequences whose host-to-device copy overlaps the verification of the "
+                         "previous group (1: copy everything, then verify)")
     ap.add_argument("--vocab-shards", type=int, default=0, metavar="W",
                     help="time the vocabulary-sharded step (include/sc_shard.h) with W shards instead: W ranks "
                          "emulated on one GPU (on-device exchanges, one CUDA graph per step), or under torchrun "
@@ -531,17 +534,11 @@ def run_ours(args):
         ht = t.cpu().pin_memory()
         hx = x.cpu().pin_memory()
         hu = u.cpu().pin_memory()
-        hna = torch.empty(B, dtype=torch.int32).pin_memory()
-        hnt = torch.empty(B, dtype=torch.int32).pin_memory()
+        chunks = max(1, min(args.e2e_chunks, B))
+        hv = binding.HostVerifier(B, g, w.V, hd.dtype, chunks=chunks, device=dev)
 
         def e2e_step():
-            d.copy_(hd, non_blocking=True)
-            t.copy_(ht, non_blocking=True)
-            x.copy_(hx, non_blocking=True)
-            u.copy_(hu, non_blocking=True)
-            step()
-            hna.copy_(na, non_blocking=True)
-            hnt.copy_(nt, non_blocking=True)
+            hv(hd, ht, hx, hu, w.rule, w.alpha, w.temperature, beta=w.beta)
 
         for _ in range(max(3, args.warmup)):
             e2e_step()
@@ -557,7 +554,9 @@ def run_ours(args):
         e2e_ms = max_over_ranks(a0.elapsed_time(a1) / args.steps, world, dev)
         h2d = sum(tn.numel() * tn.element_size() for tn in (hd, ht, hx, hu))
         e2e = {"value": whole_job_rate(B * g, world, e2e_ms), "unit": UNIT, "h2d_bytes_per_step": h2d,
-               "d2h_bytes_per_step": 8 * B, "ms_per_step": e2e_ms}
+               "d2h_bytes_per_step": 8 * B, "ms_per_step": e2e_ms,
+               "api": f"binding.HostVerifier: pinned host inputs, {chunks} groups of sequences, each group's "
+                      "copy overlapping the previous group's verification"}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

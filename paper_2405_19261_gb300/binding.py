@@ -205,3 +205,64 @@ def to_device(w, device="cuda"):
         t = torch.from_numpy(np.ascontiguousarray(w.target))
     return (d.to(device), t.to(device), torch.from_numpy(np.ascontiguousarray(w.tokens)).to(device),
             torch.from_numpy(np.ascontiguousarray(w.uniforms)).to(device))
+
+
+class HostVerifier:
+    """sc_verify from pinned host tensors, the host-to-device copy overlapped
+    with the verification: the batch is cut into ``chunks`` groups of sequences;
+    group c+1 is copied on a copy stream while group c is verified on the
+    calling stream (sequences are independent, so a group is verified as soon as
+    its rows land).  Device buffers, the workspace and pinned output buffers are
+    allocated once and reused; a call's copies wait until the previous call has
+    finished reading the device buffers.
+
+    ``v(draft, target, tokens, uniforms, rule, alpha, temperature)`` returns the
+    pinned host tensors (num_accepted [B], next_token [B]), valid once the
+    calling stream reaches the end of the call (e.g. after its synchronize)."""
+
+    def __init__(self, B: int, gamma: int, V: int, dtype: torch.dtype, chunks: int = 4, device=None):
+        if not (1 <= chunks <= B):
+            raise ValueError("need 1 <= chunks <= B")
+        dev = torch.device(device or "cuda")
+        self.B, self.gamma, self.V, self.dtype = B, gamma, V, dtype
+        self.d = torch.empty(B, gamma, V, dtype=dtype, device=dev)
+        self.t = torch.empty(B, gamma + 1, V, dtype=dtype, device=dev)
+        self.x = torch.empty(B, gamma, dtype=torch.int32, device=dev)
+        self.u = torch.empty(B, gamma + 1, dtype=torch.float32, device=dev)
+        self.na = torch.empty(B, dtype=torch.int32, device=dev)
+        self.nt = torch.empty(B, dtype=torch.int32, device=dev)
+        step = -(-B // chunks)
+        self.bounds = [(b0, min(B, b0 + step)) for b0 in range(0, B, step)]
+        self.ws = new_workspace(step, gamma, dev)
+        self.hna = torch.empty(B, dtype=torch.int32).pin_memory()
+        self.hnt = torch.empty(B, dtype=torch.int32).pin_memory()
+        self.copy = torch.cuda.Stream(device=dev)
+        self.landed = [torch.cuda.Event() for _ in self.bounds]
+        self.done = torch.cuda.Event()
+        self.done.record(torch.cuda.current_stream(dev))
+
+    def __call__(self, draft: torch.Tensor, target: torch.Tensor, tokens: torch.Tensor, uniforms: torch.Tensor,
+                 rule, alpha: float, temperature: float, *, beta: float = 1.0):
+        shapes = ((draft, (self.B, self.gamma, self.V), self.dtype), (target, (self.B, self.gamma + 1, self.V), self.dtype),
+                  (tokens, (self.B, self.gamma), torch.int32), (uniforms, (self.B, self.gamma + 1), torch.float32))
+        for h, shape, dt in shapes:
+            if h.is_cuda or tuple(h.shape) != shape or h.dtype != dt or not h.is_contiguous():
+                raise ValueError(f"host inputs must be contiguous {shape} {dt} CPU tensors (pinned for overlap)")
+        comp = torch.cuda.current_stream(self.d.device)
+        self.copy.wait_event(self.done)  # the previous call has read the device buffers
+        for (b0, b1), ev in zip(self.bounds, self.landed):
+            with torch.cuda.stream(self.copy):
+                self.d[b0:b1].copy_(draft[b0:b1], non_blocking=True)
+                self.t[b0:b1].copy_(target[b0:b1], non_blocking=True)
+                self.x[b0:b1].copy_(tokens[b0:b1], non_blocking=True)
+                self.u[b0:b1].copy_(uniforms[b0:b1], non_blocking=True)
+                ev.record(self.copy)
+        for (b0, b1), ev in zip(self.bounds, self.landed):
+            comp.wait_event(ev)
+            sc_verify(self.d[b0:b1], self.t[b0:b1], self.x[b0:b1], self.u[b0:b1], rule, alpha, temperature,
+                      beta=beta, num_accepted=self.na[b0:b1], next_token=self.nt[b0:b1], workspace=self.ws,
+                      stream=comp)
+        self.done.record(comp)
+        self.hna.copy_(self.na, non_blocking=True)
+        self.hnt.copy_(self.nt, non_blocking=True)
+        return self.hna, self.hnt

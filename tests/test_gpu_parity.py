@@ -489,3 +489,27 @@ def test_token_rules_ragged_vocab(sc, V, dtype):
     w = synthetic(5, 3, V, dtype=dtype, kind="gauss", sigma=1.0, rule="token_v3", alpha=0.3,
                   temperature=0.9, seed=V)
     assert_parity(w, run_gpu(sc, w), oracle.verify_workload(w))
+
+
+@pytest.mark.parametrize("chunks", [1, 3, 8])
+def test_host_verifier_overlapped_copies(sc, chunks):
+    # sc_verify from pinned host tensors with the copy of each group of
+    # sequences overlapping the previous group's verification: the outputs are
+    # sc_verify's and the oracle's, over two calls on the same buffers
+    import torch
+    from paper_2405_19261_gb300.workloads import synthetic
+    B, g, V = 24, 5, 32128
+    hv = sc.HostVerifier(B, g, V, torch.bfloat16, chunks=chunks)
+    for seed in (61, 62):
+        w = synthetic(B, g, V, dtype="bf16", kind="gauss", sigma=0.5, rule="opt", alpha=0.2, seed=seed)
+        d, t, x, u = sc.to_device(w)
+        hd, ht, hx, hu = (a.cpu().pin_memory() for a in (d, t, x, u))
+        na, nt = hv(hd, ht, hx, hu, w.rule, w.alpha, w.temperature)
+        torch.cuda.synchronize()
+        na1, nt1 = sc.sc_verify(d, t, x, u, w.rule, w.alpha, w.temperature)
+        torch.cuda.synchronize()
+        assert np.array_equal(na.numpy(), na1.cpu().numpy()) and np.array_equal(nt.numpy(), nt1.cpu().numpy())
+        ref = oracle.verify_workload(w)
+        ok = ~ref.flagged
+        assert np.array_equal(na.numpy()[ok], ref.num_accepted[ok])
+        assert np.array_equal(nt.numpy()[ok], ref.next_token[ok])
