@@ -1081,11 +1081,16 @@ __device__ __forceinline__ void online_pair_bc(const uint16_t *srcq, const uint1
 }
 
 // Weights of one chunk in the ring: per round, the warp's total weight (the
-// segment total) lands in seg[(c, round, warp)].
+// segment total) lands in seg[(c, round, warp)].  Every round's weights come
+// before any reduction or store, so the rounds' shared-memory loads and
+// exponentials overlap (a store to seg between rounds would order the next
+// round's loads after it), and the rounds' warp sums run interleaved, each in
+// warp_sum's butterfly order (the same totals as one warp_sum per round).
 template <typename E, bool kPair, bool kFull, bool kTok>
 __device__ __forceinline__ void weights_chunk(const E *sq, const E *sp, int n, int c,
                                               const RowScalars &rs, Shared &sh, int lane,
                                               int warp) {
+  float tot[kRounds];
 #pragma unroll
   for (int r = 0; r < kRounds; ++r) {
     const int e = 8 * (r * kNT + static_cast<int>(threadIdx.x));
@@ -1097,8 +1102,16 @@ __device__ __forceinline__ void weights_chunk(const E *sq, const E *sp, int n, i
       if constexpr (kPair) load8_smem(sq, e, n, yq);
       load8_smem(sp, e, n, yp);
     }
-    const float tot = warp_sum(vec_weights<kPair, kTok>(yq, yp, rs, w));
-    if (lane == 0 && SC_CHECK(c >= 0 && c < kMaxChunks)) sh.seg[(c * kRounds + r) * kNW + warp] = tot;
+    tot[r] = vec_weights<kPair, kTok>(yq, yp, rs, w);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+#pragma unroll
+    for (int r = 0; r < kRounds; ++r) tot[r] = __fadd_rn(tot[r], __shfl_xor_sync(0xFFFFFFFFu, tot[r], o));
+  }
+  if (lane == 0 && SC_CHECK(c >= 0 && c < kMaxChunks)) {
+#pragma unroll
+    for (int r = 0; r < kRounds; ++r) sh.seg[(c * kRounds + r) * kNW + warp] = tot[r];
   }
 }
 
@@ -2459,12 +2472,15 @@ size_t smem_bytes() {
 // Long slices amortise each unit's cluster exchange, decision and ticket over
 // more streamed bytes and wait on fewer peers; short ones give small batches
 // enough CTAs to cover the GPU.  65536 logits per CTA once that still fills
-// the GPU four times over, else 32768, else (small batches) 8192.
+// the resident CTA slots one and a half times over, else 32768, else (small
+// batches) 8192.  V = 256000, gamma = 8 (OPT / Diff, us): B = 48 121 -> 116 /
+// 97 -> 89, B = 64 142 -> 131 / 119 -> 115 with 65536; below 1.5 waves it
+// loses (B = 64, gamma = 4: 89 -> 97 / 82 -> 88; B = 32, gamma = 5: 69 -> 70).
 int pick_layout(int V, int units, int sms, int *C_out, int *L_out) {
   const long resident = static_cast<long>(kMinBlocksPerSM) * sms;
   auto ctas = [&](long t) { return static_cast<long>(units) * ((V + t - 1) / t); };
   long target = 32768;  // logits per row per CTA
-  if (ctas(65536) >= 4 * resident) target = 65536;
+  if (2 * ctas(65536) >= 3 * resident) target = 65536;
   else if (ctas(32768) < 4L * sms) target = 8192;
   if (const char *s = getenv("SC_SLICE")) {
     const long t = atol(s);
@@ -2572,7 +2588,8 @@ int launch(Params P, cudaStream_t stream, int units) {
   // in pass 1 and saves the TV pass of the band rows it settles.  With slices of
   // up to 64000 logits (C <= 4, large batches) that pass mostly re-reads HBM and
   // the bound pays (B=512, gamma=8: 873 -> 809 us); with the shorter slices of
-  // small batches the bound costs more than it saves (B=64, gamma=8: 143 -> 155 us).
+  // C = 8 the bound costs more than it saves (B=64, gamma=8 held at C = 8:
+  // 143 -> 155 us; at its C = 4, with the bound, 131 us).
   P.opt_ub = C <= 4;
   if (const char *e = getenv("SC_OPT_UB")) P.opt_ub = atoi(e) != 0;
   // L2 eviction priorities (cp.async.bulk with an evict-first cache policy): a
