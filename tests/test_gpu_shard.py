@@ -237,3 +237,62 @@ def test_graph_replay_matches_the_eager_step(sh):
         torch.cuda.synchronize()
         assert np.array_equal(got[0], na2.cpu().numpy()) and np.array_equal(got[1], nt2.cpu().numpy())
         assert_sharded_parity(w, (got[0], got[1], 0), oracle.verify_workload(w))
+
+
+def _nccl_rank(port, queue):
+    # one rank of a one-GPU NCCL process group: the step through DistExchange
+    # (NCCL all-gathers of the device messages) and through LocalExchange
+    import os
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    sys.path.insert(0, root)
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK="0", WORLD_SIZE="1",
+                      NCCL_NVLS_ENABLE="0")
+    import torch
+    import torch.distributed as dist
+    from paper_2405_19261_gb300 import binding, sharded
+    try:
+        torch.cuda.set_device(0)
+        dist.init_process_group("nccl", rank=0, world_size=1)
+        w = synthetic(16, 5, 32128, dtype="bf16", kind="gauss", sigma=0.5, rule="opt", alpha=0.2, seed=51)
+        d, t, x, u = binding.to_device(w)
+        res = {}
+        for name, ex in (("nccl", sharded.DistExchange()), ("local", sharded.LocalExchange())):
+            r = sharded.ShardRank(w.B, w.gamma, [0, w.V], 0, d.dtype, d.device)
+            [(na, nt)] = sharded.sharded_step([r], [(d, t)], x, u, "opt", 0.2, 1.0, ex)
+            torch.cuda.synchronize()
+            res[name] = (na.cpu().tolist(), nt.cpu().tolist(), int(r.status.item()))
+        queue.put(("ok", dist.get_backend(), res))
+    except Exception as e:  # reported to the test, which fails on it
+        queue.put(("error", repr(e), None))
+    finally:
+        if dist.is_initialized():
+            dist.destroy_process_group()
+
+
+def test_nccl_exchange_on_one_gpu(sh):
+    # the multi-GPU exchange (torch.distributed all-gathers over NCCL) on the one
+    # GPU there is: a one-rank group, whose all-gathers copy each message into
+    # the gathered buffer on the device; the step must match the in-process
+    # exchange bit for bit, and the oracle
+    import socket
+    import torch.multiprocessing as mp
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        port = s.getsockname()[1]
+    ctx = mp.get_context("spawn")
+    queue = ctx.Queue()
+    p = ctx.Process(target=_nccl_rank, args=(port, queue))
+    p.start()
+    p.join(300)
+    if p.is_alive():  # a rendezvous that never completed
+        p.kill()
+        p.join()
+    assert p.exitcode == 0
+    kind, backend, res = queue.get(timeout=10)
+    assert kind == "ok", backend
+    assert backend == "nccl"
+    assert res["nccl"] == res["local"]
+    w = synthetic(16, 5, 32128, dtype="bf16", kind="gauss", sigma=0.5, rule="opt", alpha=0.2, seed=51)
+    na, nt, st = res["nccl"]
+    assert_sharded_parity(w, (np.array(na), np.array(nt), st), oracle.verify_workload(w))
