@@ -351,8 +351,8 @@ def run_reference(args):
     if rank != 0:
         return
     w, desc = workload_from(args)
-    for _ in range(max(0, args.warmup)):
-        pass  # the oracle has no warm state worth warming beyond its first call
+    for _ in range(max(0, args.warmup)):  # untimed: loads the oracle library, warms the caches
+        oracle_throughput(w, max_seqs=16)
     times, info = [], None
     for _ in range(args.steps):
         info, dt, n_seq = oracle_throughput(w, max_seqs=16)

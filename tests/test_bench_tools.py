@@ -54,3 +54,37 @@ def test_step_spread_matches_linear_percentiles():
         for key, q in (("p10", 10), ("median", 50), ("p90", 90)):
             assert abs(s[key] - float(np.percentile(xs, q))) < 1e-12
     assert bench.step_spread([])["median"] is None
+
+
+def _bench_lines(args, env=None):
+    import subprocess
+    e = dict(os.environ)
+    e.update(env or {})
+    out = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), *args], capture_output=True,
+                         text=True, timeout=600, cwd=ROOT, env=e)
+    assert out.returncode == 0, out.stderr[-2000:]
+    return [json.loads(ln) for ln in out.stdout.splitlines() if ln.startswith("{")]
+
+
+def test_reference_arm_prints_the_contract_line():
+    # the reference arm (the oracle on the host cores) on the smallest named
+    # workload: one JSON line with the bench's metric, the oracle as the CPU
+    # baseline and an end-to-end figure that moves no bytes to or from a GPU
+    lines = _bench_lines(["--impl", "reference", "--config", "1", "--steps", "2", "--warmup", "3"])
+    assert len(lines) == 1
+    d = lines[0]
+    assert d["impl"] == "reference" and d["metric"] == "verified positions/s"
+    assert d["unit"] == "positions/s" and d["higher_is_better"] is True
+    assert d["steps"] == 2 and d["warmup"] == 3 and d["n_gpus"] == 1
+    assert d["value"] > 0 and d["ms_per_step"] > 0 and d["vs_baseline"] is None
+    assert d["config"]["B"] == 8 and d["config"]["gamma"] == 5 and d["config"]["V"] == 32128
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and cb["sample"]
+    assert d["e2e"] == {"value": d["value"], "unit": "positions/s", "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}
+
+
+def test_reference_arm_prints_on_rank_zero_only():
+    # under torchrun only rank 0 runs the oracle and prints; the other ranks exit 0
+    assert _bench_lines(["--impl", "reference", "--config", "1", "--steps", "1", "--warmup", "3"],
+                        {"RANK": "1", "LOCAL_RANK": "1", "WORLD_SIZE": "2"}) == []
